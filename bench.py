@@ -1,0 +1,405 @@
+#!/usr/bin/env python
+"""Benchmark of the rollout / payoff-evaluation path on GB300.
+
+Default workload (one "step"): the empirical payoff table of Leduc hold'em for
+an 8 x 8 population of fp32 MLP policies 17-128-128-3, 65,536 Monte-Carlo
+hands per pair (64 pairs, ~14 M decisions): deal, observation, policy forward
+of the acting seat, masked softmax + Philox draw, transition, payoff reduction
+(malib_eval_payoff). Inputs (population, pair table) are resident in HBM; L2 is
+flushed (256 MiB write) before every timed step; each step uses a new seed.
+
+Prints ONE JSON line (rank 0). --impl reference times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "env-steps/sec incl. policy inference and payoff entries/sec on 1 GB300; % of roofline"
+UNIT = "env-steps/s"
+SM_COUNT_GB300 = 152
+FP32_LANES_PER_SM = 128
+# dram bytes (read + write) of one launch of the dominant kernel from the ncu
+# capture summarised under profiles/ (None until taken for the current kernel)
+NCU_TRAFFIC_PER_LAUNCH = {}
+
+
+def mlp_flop(dims):
+    i, h1, h2, o = dims
+    return 2 * (i * h1 + h1 * h2 + h2 * o)
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3"], default="leduc")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """Max of a per-rank number over all ranks (the timing aggregation)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, world: int, device=None) -> float:
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        return json.load(open(p))
+    except Exception:
+        return {}
+
+
+def workload(name: str, rank: int):
+    import workloads
+    if name == "leduc":
+        w = workloads.config(2)
+    elif name == "kuhn":
+        w = workloads.config(1)
+    else:
+        w = workloads.config(3, n_episodes=100)
+    return w
+
+
+def config_of(w, name):
+    if name == "leduc":
+        return {"workload": "leduc_holdem_8x8_mlp17-128-128-3_f32_65536hands",
+                "pairs": w.n_pairs, "hands_per_pair": w.n_episodes,
+                "policy": "MLP 17-128-128-3 fp32", "population_per_seat": w.rows,
+                "l2": "flushed (256 MiB write) before every timed step"}
+    if name == "kuhn":
+        return {"workload": "kuhn_4x4_tabular_10000hands", "pairs": w.n_pairs,
+                "hands_per_pair": w.n_episodes,
+                "l2": "flushed (256 MiB write) before every timed step"}
+    return {"workload": "spread_n3_4096env_mlp18-64-64-5_f32_100episodes", "envs": w.n_envs,
+            "combinations": w.n_pairs, "episodes_per_env": w.n_episodes, "episode_len": 25,
+            "l2": "trajectory output (2.5 GB per step) exceeds L2; flushed as well"}
+
+
+# ----------------------------------------------------------------- CPU oracle
+def oracle_leduc_sample(w, target_s: float, threads: int):
+    """Times the oracle on the first n hands of every pair, n sized so that the
+    run takes about target_s seconds. Returns (decisions/s, sample text)."""
+    import numpy as np
+    import oracle
+    params = [p.params for p in w.policies]
+    dims = w.policies[0].dims
+
+    def run(n):
+        dec = np.zeros(w.n_pairs, np.int64)
+        t0 = time.perf_counter()
+        oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, w.seed, n_sim=n,
+                          decisions=dec, n_threads=threads)
+        return time.perf_counter() - t0, int(dec.sum())
+
+    n = 8
+    dt, dec = run(n)
+    while dt < 0.5 and n < w.n_episodes:
+        n = min(w.n_episodes, n * 4)
+        dt, dec = run(n)
+    n2 = max(1, min(w.n_episodes, int(n * target_s / max(dt, 1e-6))))
+    if n2 != n:
+        dt, dec = run(n2)
+        n = n2
+    return dec / dt, f"first {n} hands of each of the {w.n_pairs} pairs ({dec} decisions, {dt:.1f} s)"
+
+
+def cpu_count():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    w = workload("leduc", 0)
+    threads = cpu_count()
+    per_step = max(0.2, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
+    import numpy as np
+    params = [p.params for p in w.policies]
+    dims = w.policies[0].dims
+    # size one step
+    rate, sample = oracle_leduc_sample(w, per_step, threads)
+    n = int(sample.split()[1])
+    for _ in range(args.warmup):
+        oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, w.seed, n_sim=n,
+                          n_threads=threads)
+    tot_dec, tot_t = 0, 0.0
+    for k in range(args.steps):
+        dec = np.zeros(w.n_pairs, np.int64)
+        t0 = time.perf_counter()
+        oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, w.seed + k, n_sim=n,
+                          decisions=dec, n_threads=threads)
+        tot_t += time.perf_counter() - t0
+        tot_dec += int(dec.sum())
+    value = tot_dec / tot_t
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * tot_t / max(1, args.steps), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_of(w, "leduc"),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"per step: first {n} hands of each of the 64 pairs"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------- GPU arm
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2106_07551_gb300 import Context, alloc_traj, make_spec, policy_desc
+
+    w = workload(args.workload, rank)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    ctx = Context(local, stream)
+    spec = make_spec(w.env_kind, w.n_agents, w.obs_dim, w.n_actions, w.n_landmarks,
+                     w.episode_len, w.n_envs)
+    d_params = [torch.from_numpy(p.params).to(dev) for p in w.policies]
+    ctx.pop_load(spec, [policy_desc(p.kind, p.dtype, p.seat, p.dims, d)
+                        for p, d in zip(w.policies, d_params)])
+    d_pairs = torch.from_numpy(w.pair_ids).to(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    seed0 = w.seed + 1_000_003 * rank
+    rollout = args.workload == "spread3"
+    if rollout:
+        traj = alloc_traj(spec, w.n_episodes)
+        steps_per_call = w.n_envs * w.episode_len * w.n_episodes
+        flop_per_unit = w.n_agents * mlp_flop(w.policies[0].dims)
+    else:
+        d_out = torch.empty((w.n_pairs, 4), dtype=torch.float64, device=dev)
+        flop_per_unit = mlp_flop(w.policies[0].dims) if w.env_kind == 2 else 0
+
+    def step(seed):
+        if rollout:
+            ctx.rollout(spec, d_pairs, w.n_episodes, seed, traj)
+            return steps_per_call
+        ctx.eval_payoff(d_pairs, w.n_episodes, seed, d_out)
+        return None
+
+    for k in range(args.warmup):
+        step(seed0 + 10_000 + k)
+    torch.cuda.synchronize(dev)
+    ctx.sync()
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    decisions = 0
+    ctx.main_kernel_ms(reset=True)
+    ctx.set_timing(True)
+    launches0 = ctx.launch_count()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clocks:
+        for k in range(args.steps):
+            flush.zero_()
+            ev[k][0].record(stream)
+            n = step(seed0 + k)
+            ev[k][1].record(stream)
+            decisions += n if n is not None else ctx.eval_decisions()
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    launches = ctx.launch_count() - launches0
+    ctx.set_timing(False)
+    ctx.sync()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+    kern_ms, kern_n = ctx.main_kernel_ms(reset=True)
+    clk = clocks.summary()
+
+    total_ms_max = max_over_ranks(total_ms, world, dev)
+    dec_all = sum_over_ranks(float(decisions), world, dev)
+    value = dec_all / (total_ms_max / 1e3)
+    entries = sum_over_ranks(float(w.n_pairs * args.steps), world, dev) / (total_ms_max / 1e3)
+
+    peaks = load_peaks()
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    peak_tflops = SM_COUNT_GB300 * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    achieved = (decisions * flop_per_unit / args.steps) / (kern_ms / kern_n / 1e3) / 1e12 \
+        if kern_n else 0.0
+    kname = {"leduc": "leduc_eval_f32_kernel<128>", "kuhn": "kuhn_eval_kernel",
+             "spread3": "spread_rollout_f32_kernel<3,18,64>"}[args.workload]
+    roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tflops, "unit": "TFLOP/s",
+                "frac": achieved / peak_tflops if peak_tflops else None,
+                "traffic": NCU_TRAFFIC_PER_LAUNCH.get(kname),
+                "kernel": kname, "kernel_ms_per_launch": kern_ms / max(1, kern_n),
+                "peak_basis": f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"
+                              f" x {sm_max:.0f} MHz (max SM clock of MEASURED_PEAKS.json)",
+                "algorithmic": f"{flop_per_unit} flop per env-step (MLP forward, padding excluded)"}
+    if clk.get("sm_mhz"):
+        roofline["frac_at_measured_clock"] = achieved / (peak_tflops * clk["sm_mhz"] / sm_max)
+
+    e2e = run_e2e(args, ctx, w, spec, dev, rollout) if rank == 0 else None
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "leduc":
+        rate, sample = oracle_leduc_sample(w, 12.0, cpu_count())
+        cpu = {"value": rate, "unit": UNIT, "cores": cpu_count(), "kind": "oracle",
+               "sample": sample}
+    ctx.close()
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                "data": "synthetic", "config": config_of(w, args.workload),
+                "payoff_entries_per_s": entries if not rollout else None,
+                "env_steps_per_step": decisions / args.steps,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+                "gpu_launches": launches}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, ctx, w, spec, dev, rollout):
+    """The same metric through the public API with host buffers: population
+    upload from pinned host memory, pair table in, payoff table back."""
+    import numpy as np
+    import torch
+    from paper_2106_07551_gb300 import policy_desc
+    if rollout:
+        return None
+    h_params = [torch.from_numpy(p.params).pin_memory() for p in w.policies]
+    h_pairs = torch.from_numpy(w.pair_ids).pin_memory()
+    h_out = torch.empty((w.n_pairs, 4), dtype=torch.float64).pin_memory()
+    descs = [policy_desc(p.kind, p.dtype, p.seat, p.dims, h) for p, h in zip(w.policies, h_params)]
+    h2d = sum(h.numel() * 4 for h in h_params) + h_pairs.numel() * 4
+    d2h = h_out.numel() * 8
+    n = max(1, args.e2e_steps)
+    tot, dec = 0.0, 0
+    for k in range(n + 1):
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        ctx.pop_reset()
+        ctx.pop_load(spec, descs)
+        ctx.eval_payoff(h_pairs, w.n_episodes, w.seed + 777 + k, h_out)   # returns after D2H
+        t1 = time.perf_counter()
+        d = ctx.eval_decisions()
+        if k > 0:            # first call warms the host path
+            tot += t1 - t0
+            dec += d
+    return {"value": dec / tot, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "steps": n}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,245 @@
+/*
+ * malib.h - C ABI of the GB300 rollout and payoff-evaluation path of MALib
+ * (Zhou et al., "MALib: A Parallel Framework for Population-based Multi-agent
+ * Reinforcement Learning", arXiv 2106.07551).
+ *
+ * Vocabulary (Sec. 3.1 "Defining the Task Graph"): a *population* holds policy
+ * pools; a *policy combination* Comb_t picks one policy per agent; a *rollout*
+ * draws trajectories X ~ P(s, a, s' | a ~ Comb_t). Sec. 3.2: the Evaluator
+ * keeps a *payoff table* with one entry per combination, which a PSRO-style
+ * meta-solver consumes; Sec. 4.2 estimates each entry by Monte-Carlo
+ * simulations of the combination.
+ *
+ * Conventions for every call:
+ *  - Return value: MALIB_OK (0) or a negative malib_status. No exception
+ *    crosses this boundary. malib_last_error() gives a message for the last
+ *    failing call on a context.
+ *  - Pointers: "device" means memory of the context's GPU (cudaMalloc /
+ *    torch tensors); "host or device" pointers are classified with
+ *    cudaPointerGetAttributes. The caller owns every buffer it passes; the
+ *    library keeps no pointer after the call's work has completed on the
+ *    context's stream.
+ *  - Ordering: calls are asynchronous and ordered on the context's CUDA stream,
+ *    except that a call given a HOST output buffer copies the result back and
+ *    waits for the stream before returning. Errors detected on the device
+ *    (an invalid policy id in a device-side pair table, an expired bounded
+ *    wait) are reported by the next malib_sync().
+ *  - Threads: one context must not be used from two threads at once.
+ */
+#ifndef MALIB_H
+#define MALIB_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum malib_status {
+    MALIB_OK = 0,
+    MALIB_EINVAL = -1,        /* bad argument (null pointer, size, id, layout) */
+    MALIB_ENOMEM = -2,        /* device or host allocation failed */
+    MALIB_ECUDA = -3,         /* a CUDA runtime call failed */
+    MALIB_ESTATE = -4,        /* no population loaded, or env/population mismatch */
+    MALIB_ETIMEOUT = -5,      /* a bounded device-side wait expired */
+    MALIB_EUNSUPPORTED = -6   /* valid request outside the built kernels' shapes */
+} malib_status;
+
+typedef enum malib_env_kind {
+    MALIB_ENV_KUHN = 1,       /* Kuhn poker: 3 cards, ante 1, one bet of 1, 2 seats */
+    MALIB_ENV_LEDUC = 2,      /* Leduc hold'em: 6 cards, 2 rounds, raises 2 then 4 */
+    MALIB_ENV_SPREAD = 3      /* cooperative particle spread (App. B.1) */
+} malib_env_kind;
+
+typedef enum malib_policy_kind {
+    MALIB_POL_TABULAR = 1,    /* Kuhn: P(bet) for each of 6 infosets */
+    MALIB_POL_MLP = 2         /* 3-layer ReLU MLP: in -> h1 -> h2 -> out logits */
+} malib_policy_kind;
+
+typedef enum malib_dtype {
+    MALIB_F32 = 0,            /* fp32 weights, fp32 FMA forward */
+    MALIB_BF16 = 1            /* bf16 weights and layer inputs, fp32 accumulation */
+} malib_dtype;
+
+/* Flags of malib_env_spec.flags and malib_eval_payoff_ex(). */
+#define MALIB_DUMP_LOGITS 1u          /* record logits (and obs, actions) in a malib_traj */
+#define MALIB_EXACT_EXPECTATION 2u    /* Kuhn: exact enumeration instead of Monte Carlo */
+
+typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
+
+/*
+ * Environment description (the paper's env_desc, App. C.1 single-instance
+ * example). Fixed shapes per kind:
+ *   KUHN:   n_agents 2, obs_dim 0 (infoset index), n_actions 2
+ *   LEDUC:  n_agents 2, obs_dim 17, n_actions 3 (fold, call/check, raise)
+ *   SPREAD: n_agents = n_landmarks in [2, 16], obs_dim >= 4 + 4 n_agents - 2,
+ *           n_actions 5 (noop, +x, -x, +y, -y), episode_len >= 1
+ * n_envs is the number of parallel environments of a rollout (SPREAD).
+ */
+typedef struct malib_env_spec {
+    int32_t env_kind;
+    int32_t n_agents;
+    int32_t n_landmarks;
+    int32_t obs_dim;
+    int32_t n_actions;
+    int32_t episode_len;
+    int64_t n_envs;
+    uint32_t flags;
+    uint32_t reserved;
+} malib_env_spec;
+
+/*
+ * One population member. params points to fp32 values (host or device) in the
+ * layout
+ *   TABULAR: p_bet[6], infoset index = card * 2 + h (card J=0, Q=1, K=2;
+ *            h = 1 when facing a bet, where "bet" means call)
+ *   MLP:     W1[h1][in], b1[h1], W2[h2][h1], b2[h2], W3[out][h2], b3[out]
+ * nbytes must equal the byte size of that layout. dtype MALIB_BF16 rounds the
+ * weights to bf16 (nearest-even) when loading; biases stay fp32.
+ * seat: owning seat of a poker population (0 or 1), or -1 for a shared pool.
+ */
+typedef struct malib_policy_desc {
+    int32_t kind;
+    int32_t dtype;
+    int32_t seat;
+    int32_t n_layers;         /* 3 for MLP, 1 for TABULAR */
+    int32_t dims[4];          /* MLP: in, h1, h2, out; TABULAR: 6, 0, 0, 1 */
+    const void* params;
+    int64_t nbytes;
+} malib_policy_desc;
+
+/*
+ * Trajectory buffers, all DEVICE pointers, caller-owned, 16-byte aligned.
+ * Rollout (SPREAD), T = episode_len, E = n_episodes per env, V = n_envs,
+ * N = n_agents, P4 = obs_dim rounded up to a multiple of 4:
+ *   obs     float [E][T][V][N][P4]  (padding columns are written as 0)
+ *   action  uint8 [E][T][V][N]
+ *   reward  float [E][T][V][N]
+ *   done    uint8 [E][T][V]         (1 at t = T-1)
+ *   logits  float [E][T][V][N][A]   (only with MALIB_DUMP_LOGITS; else may be NULL)
+ * Evaluation dump (malib_eval_payoff_ex), first n_dump episodes of every pair,
+ * S = max decisions per episode (Kuhn 3, Leduc 8), steps after the end padded:
+ *   obs     float [n_pairs][n_dump][S][P4]  (Leduc 17 -> 20; Kuhn: unused)
+ *   action  uint8 [n_pairs][n_dump][S]      (255 after the end)
+ *   reward  float [n_pairs][n_dump][S]      (seat-0 payoff at the final decision, else 0)
+ *   done    uint8 [n_pairs][n_dump][S]      (1 from the final decision on)
+ *   logits  float [n_pairs][n_dump][S][A]   (Kuhn: A = 2, [1 - P(bet), P(bet)])
+ * Any of the eval-dump pointers may be NULL to skip that field.
+ */
+typedef struct malib_traj {
+    float* obs;
+    uint8_t* action;
+    float* reward;
+    uint8_t* done;
+    float* logits;
+} malib_traj;
+
+/* Creates a context on CUDA device `device`, ordered on `cuda_stream`
+ * (a cudaStream_t; NULL = the legacy default stream). *out receives the
+ * context; on failure *out is NULL. */
+int malib_create(malib_ctx** out, int device, void* cuda_stream);
+
+/* Frees the context, its population arena and scratch. Waits for the stream. */
+void malib_destroy(malib_ctx* ctx);
+
+/* Message of the last failing call on ctx ("" if none). Valid until the next
+ * call on ctx. ctx may be NULL (message of the last failed malib_create). */
+const char* malib_last_error(const malib_ctx* ctx);
+
+/* Waits for the context's stream; returns deferred device-side errors
+ * (MALIB_EINVAL for an invalid device pair table, MALIB_ETIMEOUT) and clears them. */
+int malib_sync(malib_ctx* ctx);
+
+/* Replaces the stream further calls are ordered on. */
+int malib_set_stream(malib_ctx* ctx, void* cuda_stream);
+
+/*
+ * malib_pop_load - add policies to the population (Sec. 3.1: policy pools
+ * P = {P_i}, extended as PSRO adds best responses, App. C.2 main loop).
+ * Copies and converts the parameters into the context's device arena; the
+ * caller may free `pols[i].params` when the call returns. All policies of one
+ * context share env kind, kind, dtype and dims; the first call fixes them and
+ * `spec`. ids_out[n] receives the new policies' ids (consecutive, from 0).
+ * Errors: EINVAL (shape or size mismatch with spec), ESTATE (different spec
+ * than the loaded population), ENOMEM, ECUDA.
+ */
+int malib_pop_load(malib_ctx* ctx, const malib_env_spec* spec, const malib_policy_desc* pols,
+                   int32_t n, int32_t* ids_out);
+
+/* Drops the whole population (ids restart at 0). */
+int malib_pop_reset(malib_ctx* ctx);
+
+/*
+ * malib_rollout - batched multi-agent rollout (Sec. 3.1, X(theta) ~ P(s, a, s'
+ * | a ~ Comb_t); the Actor with k environments of the architecture figure).
+ * SPREAD only. pair_ids (host or device) int32 [n_pairs][n_agents] holds one
+ * policy id per agent for each combination; the n_envs environments are split
+ * evenly and contiguously over the combinations (n_envs % n_pairs == 0).
+ * Environment v of episode e uses global episode id g = e * n_envs + v; all
+ * randomness is Philox4x32-10 keyed by seed with counter (g, step, agent).
+ * traj_out (device buffers, layout above) receives n_episodes episodes per env.
+ * Errors: EINVAL, ESTATE, EUNSUPPORTED (a policy shape without a kernel).
+ */
+int malib_rollout(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pair_ids,
+                  int32_t n_pairs, int64_t n_episodes, uint64_t seed, malib_traj* traj_out);
+
+/*
+ * malib_eval_payoff - empirical payoff table (Sec. 3.2 Evaluator; Sec. 4.2,
+ * Monte-Carlo simulations per policy combination). KUHN and LEDUC.
+ * pair_ids (host or device) int32 [n_pairs][2] = (seat-0 policy id, seat-1
+ * policy id). Pair k plays n_episodes >= 1 hands with global episode ids
+ * g = k * n_episodes + e. payoff_out (host or device) double [n_pairs][4]
+ * receives, for the seat-0 payoff (seat 1 gets its negation):
+ *   mean, standard error of the mean (sample variance / n, 0 if n < 2),
+ *   sum, sum of squares (exact integers).
+ * n_pairs == 0 is a no-op. Errors: EINVAL, ESTATE, EUNSUPPORTED.
+ */
+int malib_eval_payoff(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pairs,
+                      int64_t n_episodes, uint64_t seed, double* payoff_out);
+
+/*
+ * malib_eval_payoff_ex - malib_eval_payoff with flags:
+ *   MALIB_DUMP_LOGITS: record the first n_dump (<= n_episodes) episodes of
+ *     every pair into `dump` (device buffers, eval-dump layout above);
+ *   MALIB_EXACT_EXPECTATION (KUHN): the entry's mean is the exact expected
+ *     payoff by enumeration of the 6 deals; SE, sum and sum of squares are 0
+ *     and n_episodes and seed are ignored.
+ */
+int malib_eval_payoff_ex(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pairs,
+                         int64_t n_episodes, uint64_t seed, uint32_t flags, double* payoff_out,
+                         const malib_traj* dump, int64_t n_dump);
+
+/* ---- measurement and self-test entry points (used by tests and the benchmark) ---- */
+
+/* Total decisions (env-steps: one decision by the acting seat) played by the
+ * most recent Monte-Carlo malib_eval_payoff[_ex] call on ctx. Waits for the
+ * stream. ESTATE if none has run. */
+int malib_eval_stats(malib_ctx* ctx, int64_t* n_decisions);
+
+/* Number of kernels this context has launched since creation. */
+int64_t malib_launch_count(const malib_ctx* ctx);
+
+/* Enables (1) or disables (0) CUDA-event timing of each call's main kernel on
+ * the context's stream; malib_main_kernel_ms() returns the summed milliseconds
+ * of the timed launches since the last reset (waits for the stream) and the
+ * number of launches timed in *n_launches (may be NULL); reset clears both. */
+int malib_set_timing(malib_ctx* ctx, int enable);
+double malib_main_kernel_ms(malib_ctx* ctx, int64_t* n_launches, int reset);
+
+/* Philox4x32-10 of n counters (device uint32 [n][4]) under key (seed lo, seed
+ * hi) into out (device uint32 [n][4]) - the generator every kernel draws from. */
+int malib_selftest_philox(malib_ctx* ctx, const uint32_t* ctr, uint64_t seed, uint32_t* out,
+                          int64_t n);
+
+/* The kernels' deterministic exp (Cody-Waite reduction, degree-7 Taylor) on n
+ * device floats, and the masked inverse-CDF draw on n rows of A <= 8 logits
+ * (device: logits [n][A], legal uint8 [n][A], u [n], out int32 [n]). */
+int malib_selftest_det_expf(malib_ctx* ctx, const float* x, float* y, int64_t n);
+int malib_selftest_sample(malib_ctx* ctx, const float* logits, const uint8_t* legal,
+                          const float* u, int32_t A, int32_t* out, int64_t n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MALIB_H */

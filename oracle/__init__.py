@@ -59,7 +59,7 @@ def _L():
                 "orc_leduc_play": (C.c_int, [C.c_int, C.c_int, C.c_int, P, C.c_int, P, P, P, P, P, P]),
                 "orc_leduc_exact": (C.c_double, [P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int]),
                 "orc_leduc_eval": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, i32, i64,
-                                          u64, P, i64, P, P, P, P, P, P, P, C.c_int]),
+                                          i64, u64, P, i64, P, P, P, P, P, P, P, P, C.c_int]),
                 "orc_spread_step": (None, [C.c_int, C.c_int, P, P, P]),
                 "orc_spread_obs": (None, [C.c_int, C.c_int, P, C.c_int, P]),
                 "orc_spread_reset": (None, [C.c_int, C.c_int, u64, u64, P]),
@@ -176,9 +176,13 @@ def _param_table(params_list):
 
 
 def leduc_eval(params_list, dims, pairs, n_episodes, seed, bf16=False, n_rec=0,
-               ext_logits=None, n_threads=0):
+               ext_logits=None, n_threads=0, n_sim=None, decisions=None):
     """Monte-Carlo payoff table for Leduc pairs; optional records of the first
-    n_rec episodes of every pair (and replay of external logits for them)."""
+    n_rec episodes of every pair (and replay of external logits for them).
+    Only hands [0, n_sim) of each pair are simulated (default: all n_episodes);
+    episode ids still follow g = pair * n_episodes + e. `decisions`, an int64
+    array [n_pairs], receives each pair's number of decisions."""
+    n_sim = n_episodes if n_sim is None else n_sim
     arrs, tbl = _param_table(params_list)
     pairs = _c(pairs, np.int32).reshape(-1, 2)
     n = pairs.shape[0]
@@ -195,7 +199,8 @@ def leduc_eval(params_list, dims, pairs, n_episodes, seed, bf16=False, n_rec=0,
         ptrs = [rec[k] for k in ("obs", "logits", "action", "seat", "payoff", "ndec")]
     ext = None if ext_logits is None else _c(ext_logits, np.float32).reshape(n, n_rec, 8, 3)
     _L().orc_leduc_eval(C.cast(tbl, C.c_void_p), *dims, int(bf16), _p(pairs), n, n_episodes,
-                        C.c_uint64(seed), _p(res), n_rec, _p(ext), *[_p(a) for a in ptrs], n_threads)
+                        n_sim, C.c_uint64(seed), _p(res), n_rec, _p(ext), *[_p(a) for a in ptrs],
+                        _p(decisions), n_threads)
     del arrs
     return res, rec
 

@@ -655,21 +655,22 @@ double orc_leduc_exact(const float* params0, const float* params1, int in, int h
 }
 
 // params: [n_pol] pointers to the plain layout; pairs [n_pairs][2].
-// out [n_pairs][4]. Optional per-episode records for episodes e < n_rec of every
+// Simulates hands e in [0, n_sim) of every pair, with global episode ids
+// g = pair * n_episodes + e; out [n_pairs][4] summarises those n_sim hands. Optional per-episode records for episodes e < n_rec of every
 // pair: obs [n_pairs][n_rec][8][17], logits [..][8][3], action/seat int8
 // [..][8] (-1 after the end), payoff int32 [n_pairs][n_rec], ndec int32.
 // ext_logits (optional, [n_pairs][n_rec][8][3]) drives the draws of those
 // episodes instead of the oracle's own logits.
 void orc_leduc_eval(const float* const* params, int in, int h1, int h2, int out, int bf16,
-                    const int32_t* pairs, int32_t n_pairs, int64_t n_episodes, uint64_t seed,
-                    double* res, int64_t n_rec, const float* ext_logits, float* rec_obs,
+                    const int32_t* pairs, int32_t n_pairs, int64_t n_episodes, int64_t n_sim,
+                    uint64_t seed, double* res, int64_t n_rec, const float* ext_logits, float* rec_obs,
                     float* rec_logits, int8_t* rec_action, int8_t* rec_seat, int32_t* rec_payoff,
-                    int32_t* rec_ndec, int n_threads) {
+                    int32_t* rec_ndec, int64_t* dec_per_pair, int n_threads) {
     parallel_for(n_pairs, n_threads, [&](int64_t p) {
         Mlp m0{params[pairs[2 * p]], in, h1, h2, out, bf16};
         Mlp m1{params[pairs[2 * p + 1]], in, h1, h2, out, bf16};
-        int64_t s1 = 0, s2 = 0;
-        for (int64_t e = 0; e < n_episodes; ++e) {
+        int64_t s1 = 0, s2 = 0, nd = 0;
+        for (int64_t e = 0; e < n_sim; ++e) {
             uint64_t g = (uint64_t)p * (uint64_t)n_episodes + (uint64_t)e;
             bool rec = e < n_rec;
             int64_t base = p * n_rec + e;
@@ -691,8 +692,10 @@ void orc_leduc_eval(const float* const* params, int in, int h1, int h2, int out,
                 r = leduc_episode(m0, m1, g, seed, nullptr, nullptr, nullptr, nullptr, nullptr, &n_dec);
             }
             s1 += r; s2 += (int64_t)r * r;
+            nd += n_dec;
         }
-        finish_entry(s1, s2, n_episodes, res + 4 * p);
+        finish_entry(s1, s2, n_sim, res + 4 * p);
+        if (dec_per_pair) dec_per_pair[p] = nd;
     });
 }
 

@@ -1,0 +1,98 @@
+// Internal interface between the host runtime (runtime.cu) and the kernels.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace malib {
+
+constexpr int kMaxAgents = 16;
+
+// Error bits raised by kernels into the context's device error word.
+enum : int {
+    ERRBIT_BAD_PAIR = 1,      // an id in a device pair table is out of range / wrong seat
+    ERRBIT_TIMEOUT = 2,       // a bounded mbarrier wait expired
+};
+
+// fp32 MLP policy, kernel layout of one population member (floats, every
+// sub-array 16-byte aligned):
+//   W1T[IN][H]   (k-major: W1T[k][j] = W1[j][k])
+//   b1[H]
+//   W2T[H][H]    (k-major)
+//   b2[H]
+//   W3[A][H]     (row-major as given)
+//   b3[A], padded to a multiple of 4
+template <int IN, int H, int A>
+struct F32Layout {
+    static constexpr int kW1T = 0;
+    static constexpr int kB1 = IN * H;
+    static constexpr int kW2T = kB1 + H;
+    static constexpr int kB2 = kW2T + H * H;
+    static constexpr int kW3 = kB2 + H;
+    static constexpr int kB3 = kW3 + A * H;
+    static constexpr int kSize = (kB3 + A + 3) / 4 * 4;
+    static_assert(IN * H % 4 == 0 && H % 8 == 0, "layout alignment");
+};
+
+// Output sums of the payoff reduction: per pair {sum r, sum r^2} as 64-bit
+// two's complement (integers, so any summation order gives the same bits).
+struct EvalArgs {
+    const float* arena;          // population arena (kernel layouts)
+    const int64_t* pol_offset;   // [n_pol] float offset of each policy in arena
+    const int32_t* pol_seat;     // [n_pol] owning seat (-1 shared)
+    int32_t n_pol;
+    const int32_t* pairs;        // device [n_pairs][2]
+    int32_t n_pairs;
+    int64_t n_episodes;
+    uint64_t seed;
+    unsigned long long* acc;     // [n_pairs][2]
+    unsigned long long* n_dec;   // total decisions (env-steps) of the call
+    int* err;
+    // optional dump of the first n_dump episodes of each pair
+    int64_t n_dump;
+    float* d_obs;
+    uint8_t* d_action;
+    float* d_reward;
+    uint8_t* d_done;
+    float* d_logits;
+};
+
+struct RolloutArgs {
+    const float* arena;
+    const int64_t* pol_offset;
+    int32_t n_pol;
+    const int32_t* pairs;        // device [n_pairs][N]
+    int32_t n_pairs;
+    int32_t n_agents;
+    int32_t obs_dim;
+    int32_t obs_pad;             // obs_dim rounded up to 4
+    int32_t episode_len;
+    int64_t n_envs;
+    int64_t n_episodes;
+    uint64_t seed;
+    int* err;
+    float* obs;
+    uint8_t* action;
+    float* reward;
+    uint8_t* done;
+    float* logits;               // may be null
+};
+
+// Launchers (return cudaGetLastError() of the launch). `grid_hint` = SM count.
+cudaError_t launch_kuhn_eval(const EvalArgs& a, int n_sm, cudaStream_t s);
+cudaError_t launch_kuhn_exact(const EvalArgs& a, double* out, cudaStream_t s);
+cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s);
+cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s);
+cudaError_t launch_zero_u64(unsigned long long* p, int64_t n, cudaStream_t s);
+cudaError_t launch_finalize(const unsigned long long* acc, int32_t n_pairs, int64_t n_episodes,
+                            double* out, cudaStream_t s);
+cudaError_t launch_selftest_philox(const uint32_t* ctr, uint64_t seed, uint32_t* out, int64_t n,
+                                   cudaStream_t s);
+cudaError_t launch_selftest_det_expf(const float* x, float* y, int64_t n, cudaStream_t s);
+cudaError_t launch_selftest_sample(const float* logits, const uint8_t* legal, const float* u,
+                                   int A, int32_t* out, int64_t n, cudaStream_t s);
+
+bool leduc_f32_supported(int hidden);
+bool spread_f32_supported(int n_agents, int obs_dim, int hidden);
+
+}  // namespace malib

@@ -1,0 +1,449 @@
+// Payoff-table evaluation for the poker games (Sec. 3.2 Evaluator, Sec. 4.2:
+// each entry of the empirical payoff table is the Monte-Carlo mean over
+// simulated hands of one policy combination).
+//
+// Kuhn: one thread per hand, tabular policies in registers.
+// Leduc (fp32 MLP policies): a persistent CTA owns a contiguous range of
+// (pair, hand) indices; both policies of the current pair are staged once into
+// shared memory by bulk copy; 248 hand slots advance one decision per step; the
+// observations of the slots are compacted by acting seat so every 4-row group
+// of the MLP engine uses one policy; finished hands are replaced from the
+// range at once so the slots stay full.
+#include "device_common.cuh"
+#include "internal.h"
+#include "mlp_f32.cuh"
+
+namespace malib {
+
+namespace {
+
+// Adds the block's payoff sums (sum r, sum r^2) into the pair's two 64-bit
+// accumulators and its decision count into the call's total.
+__device__ __forceinline__ void block_add_sums(long long s1, long long s2, long long nd,
+                                               unsigned long long* acc2,
+                                               unsigned long long* n_dec) {
+    __shared__ long long red[3][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    s1 = warp_sum_ll(s1);
+    s2 = warp_sum_ll(s2);
+    nd = warp_sum_ll(nd);
+    if (lane == 0) { red[0][warp] = s1; red[1][warp] = s2; red[2][warp] = nd; }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        long long t1 = 0, t2 = 0, t3 = 0;
+        for (int w = 0; w < (int)(blockDim.x + 31) / 32; ++w) {
+            t1 += red[0][w]; t2 += red[1][w]; t3 += red[2][w];
+        }
+        atomicAdd(acc2, (unsigned long long)t1);
+        atomicAdd(acc2 + 1, (unsigned long long)t2);
+        atomicAdd(n_dec, (unsigned long long)t3);
+    }
+    __syncthreads();
+}
+
+__device__ __forceinline__ bool pair_ok(const EvalArgs& a, int p0, int p1) {
+    if (p0 < 0 || p0 >= a.n_pol || p1 < 0 || p1 >= a.n_pol) return false;
+    const int s0 = a.pol_seat[p0], s1 = a.pol_seat[p1];
+    return (s0 == 0 || s0 == -1) && (s1 == 1 || s1 == -1);
+}
+
+// ---------------------------------------------------------------- Kuhn
+// Cards J=0 < Q=1 < K=2, ante 1, one bet of 1. Infoset index card*2 + h with
+// h = 1 when the seat faces a bet. Decision t uses counter (g, t, seat).
+struct KuhnHand { int n; int act[3]; float p[3]; int payoff; };
+
+__device__ __forceinline__ KuhnHand kuhn_play(const float* t0, const float* t1, uint64_t g,
+                                              uint64_t seed) {
+    const U4 d = draw(g, 0, kChance, seed);
+    const int c0 = (int)pick(d.x, 3);
+    const int j = (int)pick(d.y, 2);
+    const int c1 = j + (j >= c0 ? 1 : 0);
+    const int sd = c0 > c1 ? 1 : -1;
+    KuhnHand h;
+    h.n = 0;
+    auto decide = [&](int seat, float p) {
+        const float u = u24(draw(g, (uint32_t)h.n, (uint32_t)seat, seed).x);
+        const int a = u < p ? 1 : 0;
+        h.act[h.n] = a; h.p[h.n] = p; ++h.n;
+        return a;
+    };
+    if (decide(0, t0[c0 * 2])) {
+        h.payoff = decide(1, t1[c1 * 2 + 1]) ? 2 * sd : 1;
+    } else if (decide(1, t1[c1 * 2])) {
+        h.payoff = decide(0, t0[c0 * 2 + 1]) ? 2 * sd : -1;
+    } else {
+        h.payoff = sd;
+    }
+    return h;
+}
+
+__global__ void __launch_bounds__(256) kuhn_eval_kernel(EvalArgs a) {
+    const int pair = blockIdx.y;
+    const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
+    if (!pair_ok(a, p0, p1)) {
+        if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+        return;
+    }
+    float t0[6], t1[6];
+#pragma unroll
+    for (int i = 0; i < 6; ++i) {
+        t0[i] = a.arena[a.pol_offset[p0] + i];
+        t1[i] = a.arena[a.pol_offset[p1] + i];
+    }
+    long long s1 = 0, s2 = 0, nd = 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < a.n_episodes; e += stride) {
+        const uint64_t g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+        const KuhnHand h = kuhn_play(t0, t1, g, a.seed);
+        s1 += h.payoff;
+        s2 += (long long)h.payoff * h.payoff;
+        nd += h.n;
+        if (e < a.n_dump) {
+            const int64_t base = ((int64_t)pair * a.n_dump + e) * 3;
+            for (int t = 0; t < 3; ++t) {
+                const bool on = t < h.n;
+                if (a.d_action) a.d_action[base + t] = on ? (uint8_t)h.act[t] : (uint8_t)255;
+                if (a.d_reward) a.d_reward[base + t] = (t == h.n - 1) ? (float)h.payoff : 0.f;
+                if (a.d_done) a.d_done[base + t] = (t >= h.n - 1) ? 1 : 0;
+                if (a.d_logits) {
+                    a.d_logits[(base + t) * 2] = on ? 1.f - h.p[t] : 0.f;
+                    a.d_logits[(base + t) * 2 + 1] = on ? h.p[t] : 0.f;
+                }
+            }
+        }
+    }
+    block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+}
+
+// Exact expected seat-0 payoff: the 6 deals, each 1/6, times the betting tree.
+__global__ void kuhn_exact_kernel(EvalArgs a, double* out) {
+    const int pair = blockIdx.x * blockDim.x + threadIdx.x;
+    if (pair >= a.n_pairs) return;
+    const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
+    double v = 0.0;
+    if (!pair_ok(a, p0, p1)) {
+        atomicOr(a.err, ERRBIT_BAD_PAIR);
+        v = __longlong_as_double(0x7ff8000000000000ll);
+    } else {
+        const float* t0 = a.arena + a.pol_offset[p0];
+        const float* t1 = a.arena + a.pol_offset[p1];
+        for (int c0 = 0; c0 < 3; ++c0)
+            for (int c1 = 0; c1 < 3; ++c1) {
+                if (c0 == c1) continue;
+                const double sd = c0 > c1 ? 1.0 : -1.0;
+                const double pb = t0[c0 * 2], pc = t1[c1 * 2 + 1];
+                const double qb = t1[c1 * 2], qc = t0[c0 * 2 + 1];
+                const double bet = pc * 2.0 * sd + (1.0 - pc);
+                const double chk = (1.0 - qb) * sd + qb * (qc * 2.0 * sd - (1.0 - qc));
+                v += (pb * bet + (1.0 - pb) * chk) / 6.0;
+            }
+    }
+    out[4 * pair + 0] = v;
+    out[4 * pair + 1] = 0.0;
+    out[4 * pair + 2] = 0.0;
+    out[4 * pair + 3] = 0.0;
+}
+
+// ---------------------------------------------------------------- Leduc
+// Six cards (two each of J, Q, K; rank = card / 2), ante 1, two rounds with
+// raise sizes 2 and 4, at most two raises a round, seat 0 first in both rounds,
+// public card revealed in round 2. Actions: 0 fold, 1 call/check, 2 raise.
+struct LeducHand {
+    int c0, c1, pub;
+    int round, con0, con1, raises, nact, actor, done, payoff;
+    __device__ int con_of(int seat) const { return seat ? con1 : con0; }
+    __device__ int card_of(int seat) const { return seat ? c1 : c0; }
+};
+
+__device__ __forceinline__ void leduc_deal(LeducHand& h, uint64_t g, uint64_t seed) {
+    const U4 d = draw(g, 0, kChance, seed);
+    const int c0 = (int)pick(d.x, 6);
+    const int j = (int)pick(d.y, 5);
+    const int c1 = j + (j >= c0 ? 1 : 0);
+    const int lo = min(c0, c1), hi = max(c0, c1);
+    int p = (int)pick(d.z, 4);
+    if (p >= lo) ++p;
+    if (p >= hi) ++p;
+    h.c0 = c0; h.c1 = c1; h.pub = p;
+    h.round = 0; h.con0 = 1; h.con1 = 1; h.raises = 0; h.nact = 0;
+    h.actor = 0; h.done = 0; h.payoff = 0;
+}
+
+__device__ __forceinline__ unsigned leduc_legal(const LeducHand& h) {
+    const int me = h.actor;
+    return (h.con_of(1 - me) > h.con_of(me) ? 1u : 0u) | 2u | (h.raises < 2 ? 4u : 0u);
+}
+
+__device__ __forceinline__ void leduc_obs(const LeducHand& h, float (&o)[17]) {
+    const int me = h.actor, op = 1 - me;
+    const unsigned lg = leduc_legal(h);
+    const int rank = h.card_of(me) >> 1;
+    const int pubi = 3 + (h.round ? (h.pub >> 1) : 3);
+#pragma unroll
+    for (int i = 0; i < 3; ++i) o[i] = rank == i ? 1.f : 0.f;
+#pragma unroll
+    for (int i = 3; i < 7; ++i) o[i] = pubi == i ? 1.f : 0.f;
+    o[7] = h.round == 0 ? 1.f : 0.f;
+    o[8] = h.round == 1 ? 1.f : 0.f;
+    o[9] = __fdiv_rn((float)h.con_of(me), 13.0f);
+    o[10] = __fdiv_rn((float)h.con_of(op), 13.0f);
+#pragma unroll
+    for (int i = 0; i < 3; ++i) o[11 + i] = h.raises == i ? 1.f : 0.f;
+    o[14] = (lg & 1u) ? 1.f : 0.f;
+    o[15] = 1.f;
+    o[16] = (lg & 4u) ? 1.f : 0.f;
+}
+
+__device__ __forceinline__ int leduc_showdown(const LeducHand& h) {
+    const int r0 = h.c0 >> 1, r1 = h.c1 >> 1, rp = h.pub >> 1;
+    int w;
+    if (r0 == rp) w = 1;
+    else if (r1 == rp) w = -1;
+    else w = (r0 > r1) - (r0 < r1);
+    return w > 0 ? h.con1 : (w < 0 ? -h.con0 : 0);
+}
+
+__device__ __forceinline__ void leduc_apply(LeducHand& h, int a) {
+    const int me = h.actor, op = 1 - me;
+    if (a == 0) {
+        h.done = 1;
+        h.payoff = me == 0 ? -h.con0 : h.con1;
+        return;
+    }
+    ++h.nact;
+    const int c_op = h.con_of(op);
+    if (a == 2) {
+        const int c = c_op + (h.round == 0 ? 2 : 4);
+        if (me) h.con1 = c; else h.con0 = c;
+        ++h.raises;
+        h.actor = op;
+        return;
+    }
+    if (me) h.con1 = c_op; else h.con0 = c_op;
+    if (h.nact >= 2) {
+        if (h.round == 0) {
+            h.round = 1; h.raises = 0; h.nact = 0; h.actor = 0;
+        } else {
+            h.done = 1;
+            h.payoff = leduc_showdown(h);
+        }
+    } else {
+        h.actor = op;
+    }
+}
+
+constexpr int kLeducSlots = 248;      // hands in flight per CTA
+constexpr int kLeducRowsMax = 256;    // 4-aligned seat-0 rows + 4-aligned seat-1 rows
+constexpr int kLeducMaxDec = 8;
+
+template <int H>
+struct LeducF32Smem {
+    using M = MlpF32<17, H, 3>;
+    using L = typename M::L;
+    static constexpr int kW = 0;
+    static constexpr int kX = kW + 2 * L::kSize;
+    static constexpr int kH1 = kX + kLeducRowsMax * M::XS;
+    static constexpr int kLG = kH1 + M::kRowsPerPass * M::HS;
+    static constexpr int kFloats = kLG + kLeducRowsMax * M::LS;
+    static constexpr size_t kBytes = (size_t)kFloats * 4;
+    static_assert(kLeducRowsMax % M::kRowsPerPass == 0, "rows tile the passes");
+};
+
+template <int H>
+__global__ void __launch_bounds__(256, 1) leduc_eval_f32_kernel(EvalArgs a) {
+    using SM = LeducF32Smem<H>;
+    using M = typename SM::M;
+    using L = typename SM::L;
+    extern __shared__ __align__(128) float smem[];
+    float* Ws = smem + SM::kW;
+    float* X = smem + SM::kX;
+    float* H1 = smem + SM::kH1;
+    float* LG = smem + SM::kLG;
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int cnt[2][8];
+    __shared__ unsigned long long next_e;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < kLeducRowsMax * M::XS; i += blockDim.x) X[i] = 0.f;
+    if (tid == 0) mbar_init(&bar, 1);
+    __syncthreads();
+    uint32_t parity = 0;
+
+    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+    const int64_t per = (total + gridDim.x - 1) / gridDim.x;
+    const int64_t lo = (int64_t)blockIdx.x * per;
+    const int64_t hi = min(total, lo + per);
+
+    for (int64_t seg = lo; seg < hi;) {
+        const int pair = (int)(seg / a.n_episodes);
+        const int64_t e_lo = seg - (int64_t)pair * a.n_episodes;
+        const int64_t e_hi = min(a.n_episodes, e_lo + (hi - seg));
+        seg += e_hi - e_lo;
+        const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
+        if (!pair_ok(a, p0, p1)) {
+            if (tid == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+            continue;
+        }
+        // stage the two policies (seat 0 at Ws, seat 1 at Ws + kSize)
+        if (tid == 0) {
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(&bar, 2u * L::kSize * 4u);
+            for (int s = 0; s < 2; ++s) {
+                const float* src = a.arena + a.pol_offset[s == 0 ? p0 : p1];
+                for (uint32_t off = 0; off < (uint32_t)L::kSize * 4u; off += 32768u) {
+                    const uint32_t n = min(32768u, (uint32_t)L::kSize * 4u - off);
+                    bulk_g2s((char*)(Ws + s * L::kSize) + off, (const char*)src + off, n, &bar);
+                }
+            }
+        }
+        if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs)) {
+            if (tid == 0) atomicOr(a.err, ERRBIT_TIMEOUT);
+            mbar_wait_bounded(&bar, parity, kWaitLimitNs);
+            return;
+        }
+        parity ^= 1u;
+
+        // hand slots
+        LeducHand h;
+        bool live = false;
+        int64_t e = e_lo + tid;
+        uint64_t g = 0;
+        int t = 0;
+        long long s1 = 0, s2 = 0, nd = 0;
+        if (tid < kLeducSlots && e < e_hi) {
+            live = true;
+            g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+            leduc_deal(h, g, a.seed);
+        }
+        if (tid == 0) next_e = (unsigned long long)(e_lo + kLeducSlots);
+
+        while (true) {
+            const int seat = live ? h.actor : -1;
+            const unsigned b0 = __ballot_sync(0xffffffffu, seat == 0);
+            const unsigned b1 = __ballot_sync(0xffffffffu, seat == 1);
+            if (lane == 0) { cnt[0][warp] = __popc(b0); cnt[1][warp] = __popc(b1); }
+            __syncthreads();
+            int n0 = 0, n1 = 0, pre0 = 0, pre1 = 0;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) {
+                const int x0 = cnt[0][w], x1 = cnt[1][w];
+                if (w < warp) { pre0 += x0; pre1 += x1; }
+                n0 += x0; n1 += x1;
+            }
+            if (n0 + n1 == 0) break;
+            const int base1 = (n0 + 3) & ~3;
+            const int rows = base1 + ((n1 + 3) & ~3);
+            const unsigned lt = (1u << lane) - 1u;
+            const int row = seat == 0 ? pre0 + __popc(b0 & lt) : base1 + pre1 + __popc(b1 & lt);
+            float ob[17];
+            if (live) {
+                leduc_obs(h, ob);
+                float* xr = X + row * M::XS;
+#pragma unroll
+                for (int i = 0; i < 17; ++i) xr[i] = ob[i];
+            }
+            __syncthreads();
+            for (int r0 = 0; r0 < rows; r0 += M::kRowsPerPass) {
+                const int grp = r0 + (tid / M::TX) * 4;
+                const float* w = grp < base1 ? Ws : Ws + L::kSize;
+                M::pass(X, H1, LG, w, r0, r0 + M::warp_first_row() < rows);
+            }
+            if (live) {
+                float lg[3] = {LG[row * M::LS], LG[row * M::LS + 1], LG[row * M::LS + 2]};
+                const unsigned legal = leduc_legal(h);
+                const float u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);
+                const int act = sample_masked<3>(lg, legal, u);
+                const bool rec = e < a.n_dump;
+                const int64_t rb = ((int64_t)pair * a.n_dump + e) * kLeducMaxDec;
+                if (rec) {
+                    if (a.d_obs) {
+                        float* o = a.d_obs + (rb + t) * 20;
+#pragma unroll
+                        for (int i = 0; i < 17; ++i) o[i] = ob[i];
+                        o[17] = 0.f; o[18] = 0.f; o[19] = 0.f;
+                    }
+                    if (a.d_logits) {
+                        float* l = a.d_logits + (rb + t) * 3;
+                        l[0] = lg[0]; l[1] = lg[1]; l[2] = lg[2];
+                    }
+                    if (a.d_action) a.d_action[rb + t] = (uint8_t)act;
+                }
+                leduc_apply(h, act);
+                if (rec) {
+                    if (a.d_reward) a.d_reward[rb + t] = h.done ? (float)h.payoff : 0.f;
+                    if (a.d_done) a.d_done[rb + t] = h.done ? 1 : 0;
+                }
+                ++t;
+                ++nd;
+                if (h.done) {
+                    s1 += h.payoff;
+                    s2 += (long long)h.payoff * h.payoff;
+                    if (rec) {
+                        for (int k = t; k < kLeducMaxDec; ++k) {
+                            if (a.d_obs)
+                                for (int i = 0; i < 20; ++i) a.d_obs[(rb + k) * 20 + i] = 0.f;
+                            if (a.d_logits)
+                                for (int i = 0; i < 3; ++i) a.d_logits[(rb + k) * 3 + i] = 0.f;
+                            if (a.d_action) a.d_action[rb + k] = 255;
+                            if (a.d_reward) a.d_reward[rb + k] = 0.f;
+                            if (a.d_done) a.d_done[rb + k] = 1;
+                        }
+                    }
+                    e = (int64_t)atomicAdd(&next_e, 1ull);
+                    live = e < e_hi;
+                    if (live) {
+                        g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+                        leduc_deal(h, g, a.seed);
+                        t = 0;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+    }
+}
+
+}  // namespace
+
+bool leduc_f32_supported(int hidden) { return hidden == 128 || hidden == 64; }
+
+cudaError_t launch_kuhn_eval(const EvalArgs& a, int n_sm, cudaStream_t s) {
+    if (a.n_pairs == 0) return cudaSuccess;
+    int64_t blocks_per_pair = (a.n_episodes + 255) / 256;
+    const int64_t cap = max(1, (n_sm * 8) / max(1, a.n_pairs));
+    if (blocks_per_pair > cap) blocks_per_pair = cap;
+    if (blocks_per_pair > 65535) blocks_per_pair = 65535;
+    dim3 grid((unsigned)blocks_per_pair, (unsigned)a.n_pairs);
+    kuhn_eval_kernel<<<grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_kuhn_exact(const EvalArgs& a, double* out, cudaStream_t s) {
+    if (a.n_pairs == 0) return cudaSuccess;
+    kuhn_exact_kernel<<<(a.n_pairs + 127) / 128, 128, 0, s>>>(a, out);
+    return cudaGetLastError();
+}
+
+template <int H>
+static cudaError_t launch_leduc_h(const EvalArgs& a, int n_sm, cudaStream_t s) {
+    const size_t bytes = LeducF32Smem<H>::kBytes;
+    cudaError_t err = cudaFuncSetAttribute(leduc_eval_f32_kernel<H>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+    if (err != cudaSuccess) return err;
+    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+    int64_t grid = (total + kLeducSlots - 1) / kLeducSlots;
+    if (grid > n_sm) grid = n_sm;
+    if (grid < 1) grid = 1;
+    leduc_eval_f32_kernel<H><<<(unsigned)grid, 256, bytes, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s) {
+    if (a.n_pairs == 0) return cudaSuccess;
+    if (hidden == 128) return launch_leduc_h<128>(a, n_sm, s);
+    if (hidden == 64) return launch_leduc_h<64>(a, n_sm, s);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace malib

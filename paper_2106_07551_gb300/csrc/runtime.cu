@@ -1,0 +1,724 @@
+// Host runtime behind the C ABI of include/malib.h: context, population arena,
+// argument validation, pointer classification, launches, deferred device
+// errors and measurement hooks.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "internal.h"
+#include "malib.h"
+
+using namespace malib;
+
+namespace {
+
+struct PolicyRec {
+    int kind, dtype, seat;
+    int dims[4];
+    int64_t offset;   // floats into the arena
+};
+
+}  // namespace
+
+struct malib_ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    int n_sm = 1;
+    std::string err;
+
+    bool has_pop = false;
+    malib_env_spec spec{};
+    int pol_kind = 0, pol_dtype = 0;
+    int dims[4] = {0, 0, 0, 0};
+    std::vector<PolicyRec> pols;
+    std::vector<float> host_arena;     // mirror of the device arena
+    float* arena = nullptr;
+    int64_t arena_cap = 0;             // floats
+    int64_t* d_off = nullptr;
+    int32_t* d_seat = nullptr;
+    int64_t tbl_cap = 0;
+    int64_t seat_cap = 0;
+    bool tables_dirty = false;
+
+    unsigned long long* acc = nullptr;
+    int64_t acc_cap = 0;
+    int64_t last_pairs = -1;           // n_pairs of the last Monte-Carlo evaluation
+    int* d_err = nullptr;
+    int32_t* d_pairs = nullptr;
+    int64_t pairs_cap = 0;
+    double* d_out = nullptr;
+    int64_t out_cap = 0;
+
+    int64_t launches = 0;
+    bool timing = false;
+    std::vector<std::pair<cudaEvent_t, cudaEvent_t>> events;
+    double timed_ms = 0.0;
+    int64_t timed_n = 0;
+};
+
+namespace {
+
+thread_local std::string g_create_err;
+
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+int fail(malib_ctx* c, int code, const char* fmt, ...) __attribute__((format(printf, 3, 4)));
+int fail(malib_ctx* c, int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    if (c) c->err = buf;
+    else g_create_err = buf;
+    return code;
+}
+
+int cuda_fail(malib_ctx* c, cudaError_t e, const char* what) {
+    return fail(c, e == cudaErrorMemoryAllocation ? MALIB_ENOMEM : MALIB_ECUDA, "%s: %s", what,
+                cudaGetErrorString(e));
+}
+
+#define CK(call, what)                                 \
+    do {                                               \
+        cudaError_t e_ = (call);                       \
+        if (e_ != cudaSuccess) return cuda_fail(c, e_, what); \
+    } while (0)
+
+bool is_device_ptr(const void* p) {
+    cudaPointerAttributes at;
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+template <class T>
+int ensure(malib_ctx* c, T*& p, int64_t& cap, int64_t need, const char* what) {
+    if (need <= cap) return MALIB_OK;
+    int64_t n = cap > 0 ? cap : 64;
+    while (n < need) n *= 2;
+    if (p) cudaFreeAsync(p, c->stream);
+    p = nullptr;
+    cap = 0;
+    CK(cudaMallocAsync((void**)&p, (size_t)n * sizeof(T), c->stream), what);
+    cap = n;
+    return MALIB_OK;
+}
+
+int64_t mlp_param_floats(const int* d) {
+    return (int64_t)d[1] * d[0] + d[1] + (int64_t)d[2] * d[1] + d[2] + (int64_t)d[3] * d[2] + d[3];
+}
+
+int check_spec(malib_ctx* c, const malib_env_spec* s) {
+    if (!s) return fail(c, MALIB_EINVAL, "env spec is NULL");
+    switch (s->env_kind) {
+        case MALIB_ENV_KUHN:
+            if (s->n_agents != 2 || s->obs_dim != 0 || s->n_actions != 2)
+                return fail(c, MALIB_EINVAL, "Kuhn spec needs n_agents 2, obs_dim 0, n_actions 2");
+            break;
+        case MALIB_ENV_LEDUC:
+            if (s->n_agents != 2 || s->obs_dim != 17 || s->n_actions != 3)
+                return fail(c, MALIB_EINVAL, "Leduc spec needs n_agents 2, obs_dim 17, n_actions 3");
+            break;
+        case MALIB_ENV_SPREAD: {
+            const int n = s->n_agents;
+            if (n < 2 || n > kMaxAgents || s->n_landmarks != n || s->n_actions != 5)
+                return fail(c, MALIB_EINVAL,
+                            "spread spec needs 2 <= n_agents == n_landmarks <= 16 and n_actions 5");
+            if (s->obs_dim < 4 + 2 * n + 2 * (n - 1))
+                return fail(c, MALIB_EINVAL, "spread obs_dim %d below the %d features", s->obs_dim,
+                            4 + 2 * n + 2 * (n - 1));
+            if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
+            break;
+        }
+        default:
+            return fail(c, MALIB_EINVAL, "unknown env_kind %d", s->env_kind);
+    }
+    if (s->flags & ~(MALIB_DUMP_LOGITS | MALIB_EXACT_EXPECTATION))
+        return fail(c, MALIB_EINVAL, "unknown flags 0x%x", s->flags);
+    return MALIB_OK;
+}
+
+bool same_env(const malib_env_spec& a, const malib_env_spec& b) {
+    return a.env_kind == b.env_kind && a.n_agents == b.n_agents &&
+           a.n_landmarks == b.n_landmarks && a.obs_dim == b.obs_dim && a.n_actions == b.n_actions;
+}
+
+// fp32 kernel layout (internal.h F32Layout) from the plain layout.
+void to_f32_layout(const float* p, const int* d, float* out, int64_t size) {
+    const int in = d[0], h1 = d[1], h2 = d[2], a = d[3];
+    const float* W1 = p;
+    const float* b1 = W1 + (int64_t)h1 * in;
+    const float* W2 = b1 + h1;
+    const float* b2 = W2 + (int64_t)h2 * h1;
+    const float* W3 = b2 + h2;
+    const float* b3 = W3 + (int64_t)a * h2;
+    std::memset(out, 0, (size_t)size * 4);
+    float* o = out;
+    for (int k = 0; k < in; ++k)
+        for (int j = 0; j < h1; ++j) o[(int64_t)k * h1 + j] = W1[(int64_t)j * in + k];
+    o += (int64_t)in * h1;
+    for (int j = 0; j < h1; ++j) o[j] = b1[j];
+    o += h1;
+    for (int k = 0; k < h1; ++k)
+        for (int j = 0; j < h2; ++j) o[(int64_t)k * h2 + j] = W2[(int64_t)j * h1 + k];
+    o += (int64_t)h1 * h2;
+    for (int j = 0; j < h2; ++j) o[j] = b2[j];
+    o += h2;
+    for (int i = 0; i < a * h2; ++i) o[i] = W3[i];
+    o += (int64_t)a * h2;
+    for (int j = 0; j < a; ++j) o[j] = b3[j];
+}
+
+int upload_tables(malib_ctx* c) {
+    if (!c->tables_dirty) return MALIB_OK;
+    const int64_t n = (int64_t)c->pols.size();
+    int r;
+    if ((r = ensure(c, c->d_off, c->tbl_cap, std::max<int64_t>(n, 1), "policy table")) != MALIB_OK)
+        return r;
+    if ((r = ensure(c, c->d_seat, c->seat_cap, std::max<int64_t>(n, 1), "seat table")) != MALIB_OK)
+        return r;
+    std::vector<int64_t> off(n);
+    std::vector<int32_t> seat(n);
+    for (int64_t i = 0; i < n; ++i) { off[i] = c->pols[i].offset; seat[i] = c->pols[i].seat; }
+    CK(cudaMemcpyAsync(c->d_off, off.data(), n * 8, cudaMemcpyHostToDevice, c->stream), "upload");
+    CK(cudaMemcpyAsync(c->d_seat, seat.data(), n * 4, cudaMemcpyHostToDevice, c->stream), "upload");
+    CK(cudaStreamSynchronize(c->stream), "upload");
+    c->tables_dirty = false;
+    return MALIB_OK;
+}
+
+int stage_pairs(malib_ctx* c, const int32_t* pair_ids, int64_t n_ints, int width, bool poker,
+                const int32_t** dev_pairs) {
+    if (is_device_ptr(pair_ids)) {
+        *dev_pairs = pair_ids;      // validated by the kernels
+        return MALIB_OK;
+    }
+    const int64_t n_pol = (int64_t)c->pols.size();
+    for (int64_t i = 0; i < n_ints; ++i) {
+        const int32_t id = pair_ids[i];
+        if (id < 0 || id >= n_pol)
+            return fail(c, MALIB_EINVAL, "pair_ids[%lld] = %d is not a policy id (population %lld)",
+                        (long long)i, id, (long long)n_pol);
+        if (poker) {
+            const int want = (int)(i % width);
+            const int s = c->pols[id].seat;
+            if (s != -1 && s != want)
+                return fail(c, MALIB_EINVAL, "policy %d belongs to seat %d, used for seat %d", id, s,
+                            want);
+        }
+    }
+    int r;
+    if ((r = ensure(c, c->d_pairs, c->pairs_cap, std::max<int64_t>(n_ints, 1), "pair staging")) !=
+        MALIB_OK)
+        return r;
+    CK(cudaMemcpyAsync(c->d_pairs, pair_ids, n_ints * 4, cudaMemcpyHostToDevice, c->stream),
+       "pair upload");
+    *dev_pairs = c->d_pairs;
+    return MALIB_OK;
+}
+
+int read_device_errors(malib_ctx* c) {
+    int h = 0;
+    CK(cudaMemcpyAsync(&h, c->d_err, 4, cudaMemcpyDeviceToHost, c->stream), "error flag");
+    CK(cudaStreamSynchronize(c->stream), "sync");
+    if (h) {
+        CK(cudaMemsetAsync(c->d_err, 0, 4, c->stream), "error flag");
+        if (h & ERRBIT_TIMEOUT)
+            return fail(c, MALIB_ETIMEOUT, "a bounded device wait expired (staging copy)");
+        if (h & ERRBIT_BAD_PAIR)
+            return fail(c, MALIB_EINVAL, "a device pair table held an invalid policy id or seat");
+    }
+    return MALIB_OK;
+}
+
+void time_begin(malib_ctx* c, cudaEvent_t* a, cudaEvent_t* b) {
+    *a = *b = nullptr;
+    if (!c->timing) return;
+    if (cudaEventCreate(a) != cudaSuccess || cudaEventCreate(b) != cudaSuccess) {
+        cudaGetLastError();
+        *a = *b = nullptr;
+        return;
+    }
+    cudaEventRecord(*a, c->stream);
+}
+
+void time_end(malib_ctx* c, cudaEvent_t a, cudaEvent_t b) {
+    if (!a) return;
+    cudaEventRecord(b, c->stream);
+    c->events.emplace_back(a, b);
+}
+
+EvalArgs eval_args(malib_ctx* c) {
+    EvalArgs a{};
+    a.arena = c->arena;
+    a.pol_offset = c->d_off;
+    a.pol_seat = c->d_seat;
+    a.n_pol = (int32_t)c->pols.size();
+    a.err = c->d_err;
+    return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+int malib_create(malib_ctx** out, int device, void* cuda_stream) {
+    if (!out) return fail(nullptr, MALIB_EINVAL, "out is NULL");
+    *out = nullptr;
+    int n_dev = 0;
+    cudaError_t e = cudaGetDeviceCount(&n_dev);
+    if (e != cudaSuccess || n_dev == 0)
+        return fail(nullptr, MALIB_ECUDA, "no CUDA device: %s", cudaGetErrorString(e));
+    if (device < 0 || device >= n_dev)
+        return fail(nullptr, MALIB_EINVAL, "device %d out of range (%d devices)", device, n_dev);
+    DeviceGuard g(device);
+    malib_ctx* c = new malib_ctx();
+    c->device = device;
+    c->stream = (cudaStream_t)cuda_stream;
+    cudaDeviceProp prop;
+    if ((e = cudaGetDeviceProperties(&prop, device)) != cudaSuccess) {
+        delete c;
+        return fail(nullptr, MALIB_ECUDA, "device properties: %s", cudaGetErrorString(e));
+    }
+    c->n_sm = prop.multiProcessorCount;
+    if ((e = cudaMalloc((void**)&c->d_err, 4)) != cudaSuccess ||
+        (e = cudaMemset(c->d_err, 0, 4)) != cudaSuccess) {
+        delete c;
+        return fail(nullptr, MALIB_ENOMEM, "error flag: %s", cudaGetErrorString(e));
+    }
+    *out = c;
+    return MALIB_OK;
+}
+
+void malib_destroy(malib_ctx* c) {
+    if (!c) return;
+    DeviceGuard g(c->device);
+    cudaStreamSynchronize(c->stream);
+    for (auto& ev : c->events) { cudaEventDestroy(ev.first); cudaEventDestroy(ev.second); }
+    cudaFree(c->arena);
+    cudaFree(c->d_off);
+    cudaFree(c->d_seat);
+    cudaFree(c->acc);
+    cudaFree(c->d_err);
+    cudaFree(c->d_pairs);
+    cudaFree(c->d_out);
+    delete c;
+}
+
+const char* malib_last_error(const malib_ctx* c) {
+    return c ? c->err.c_str() : g_create_err.c_str();
+}
+
+int malib_sync(malib_ctx* c) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    CK(cudaStreamSynchronize(c->stream), "stream");
+    return read_device_errors(c);
+}
+
+int malib_set_stream(malib_ctx* c, void* s) {
+    if (!c) return MALIB_EINVAL;
+    c->stream = (cudaStream_t)s;
+    return MALIB_OK;
+}
+
+int malib_pop_reset(malib_ctx* c) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    CK(cudaStreamSynchronize(c->stream), "stream");
+    c->pols.clear();
+    c->host_arena.clear();
+    c->has_pop = false;
+    c->tables_dirty = true;
+    return MALIB_OK;
+}
+
+int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_desc* pols,
+                   int32_t n, int32_t* ids_out) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    int r;
+    if ((r = check_spec(c, spec)) != MALIB_OK) return r;
+    if (n < 0 || (n > 0 && (!pols || !ids_out))) return fail(c, MALIB_EINVAL, "bad policy list");
+    if (c->has_pop && !same_env(c->spec, *spec))
+        return fail(c, MALIB_ESTATE, "population was loaded for a different environment");
+    const bool poker = spec->env_kind != MALIB_ENV_SPREAD;
+    std::vector<std::vector<float>> converted(n);
+    std::vector<PolicyRec> recs(n);
+    for (int i = 0; i < n; ++i) {
+        const malib_policy_desc& d = pols[i];
+        PolicyRec rec{};
+        rec.kind = d.kind;
+        rec.dtype = d.dtype;
+        rec.seat = d.seat;
+        std::memcpy(rec.dims, d.dims, sizeof rec.dims);
+        if (d.dtype != MALIB_F32 && d.dtype != MALIB_BF16)
+            return fail(c, MALIB_EINVAL, "policy %d: unknown dtype %d", i, d.dtype);
+        if (poker ? (d.seat < -1 || d.seat > 1) : false)
+            return fail(c, MALIB_EINVAL, "policy %d: seat %d", i, d.seat);
+        int64_t count;
+        if (spec->env_kind == MALIB_ENV_KUHN) {
+            if (d.kind != MALIB_POL_TABULAR || d.dims[0] != 6 || d.dims[3] != 1)
+                return fail(c, MALIB_EINVAL, "policy %d: Kuhn needs a tabular policy of 6 infosets", i);
+            count = 6;
+        } else {
+            if (d.kind != MALIB_POL_MLP || d.n_layers != 3)
+                return fail(c, MALIB_EINVAL, "policy %d: needs a 3-layer MLP", i);
+            if (d.dims[0] != spec->obs_dim || d.dims[3] != spec->n_actions || d.dims[1] < 1 ||
+                d.dims[2] < 1)
+                return fail(c, MALIB_EINVAL, "policy %d: dims %d-%d-%d-%d do not fit obs %d / actions %d",
+                            i, d.dims[0], d.dims[1], d.dims[2], d.dims[3], spec->obs_dim,
+                            spec->n_actions);
+            count = mlp_param_floats(d.dims);
+        }
+        if (!d.params || d.nbytes != count * 4)
+            return fail(c, MALIB_EINVAL, "policy %d: params NULL or nbytes %lld != %lld", i,
+                        (long long)d.nbytes, (long long)(count * 4));
+        const bool first = !c->has_pop && i == 0;
+        const int* ref_dims = first ? d.dims : (c->has_pop ? c->dims : pols[0].dims);
+        const int ref_kind = first ? d.kind : (c->has_pop ? c->pol_kind : pols[0].kind);
+        const int ref_dtype = first ? d.dtype : (c->has_pop ? c->pol_dtype : pols[0].dtype);
+        if (d.kind != ref_kind || d.dtype != ref_dtype || std::memcmp(d.dims, ref_dims, 16) != 0)
+            return fail(c, MALIB_EINVAL, "policy %d: every policy of a population shares kind, dtype and dims", i);
+        std::vector<float> plain(count);
+        if (is_device_ptr(d.params)) {
+            CK(cudaMemcpy(plain.data(), d.params, count * 4, cudaMemcpyDeviceToHost), "params");
+        } else {
+            std::memcpy(plain.data(), d.params, count * 4);
+        }
+        if (d.kind == MALIB_POL_TABULAR) {
+            converted[i].assign(8, 0.f);
+            for (int k = 0; k < 6; ++k) converted[i][k] = plain[k];
+        } else {
+            const int64_t size = ((int64_t)d.dims[0] * d.dims[1] + d.dims[1] +
+                                  (int64_t)d.dims[1] * d.dims[2] + d.dims[2] +
+                                  (int64_t)d.dims[3] * d.dims[2] + d.dims[3] + 3) / 4 * 4;
+            if (d.dtype == MALIB_BF16) {
+                // weights rounded to bf16 (nearest even); biases stay fp32
+                auto rne = [](float x) {
+                    uint32_t b;
+                    std::memcpy(&b, &x, 4);
+                    if ((b & 0x7F800000u) != 0x7F800000u) {
+                        b += 0x7FFFu + ((b >> 16) & 1u);
+                        b &= 0xFFFF0000u;
+                    }
+                    float y;
+                    std::memcpy(&y, &b, 4);
+                    return y;
+                };
+                const int* D = d.dims;
+                int64_t k = 0;
+                for (int layer = 0; layer < 3; ++layer) {
+                    const int fi = D[layer], fo = D[layer + 1];
+                    for (int64_t q = 0; q < (int64_t)fi * fo; ++q, ++k) plain[k] = rne(plain[k]);
+                    k += fo;
+                }
+            }
+            converted[i].resize(size);
+            to_f32_layout(plain.data(), d.dims, converted[i].data(), size);
+        }
+        recs[i] = rec;
+    }
+    // append to the arena
+    int64_t add = 0;
+    for (int i = 0; i < n; ++i) add += (int64_t)converted[i].size();
+    const int64_t base = (int64_t)c->host_arena.size();
+    c->host_arena.resize(base + add);
+    int64_t off = base;
+    for (int i = 0; i < n; ++i) {
+        std::memcpy(c->host_arena.data() + off, converted[i].data(), converted[i].size() * 4);
+        recs[i].offset = off;
+        off += (int64_t)converted[i].size();
+    }
+    const int64_t need = (int64_t)c->host_arena.size();
+    if (need > c->arena_cap) {
+        int64_t cap = c->arena_cap > 0 ? c->arena_cap : 1 << 16;
+        while (cap < need) cap *= 2;
+        float* na = nullptr;
+        cudaError_t e = cudaMalloc((void**)&na, (size_t)cap * 4);
+        if (e != cudaSuccess) {
+            c->host_arena.resize(base);
+            return cuda_fail(c, e, "population arena");
+        }
+        cudaStreamSynchronize(c->stream);
+        cudaFree(c->arena);
+        c->arena = na;
+        c->arena_cap = cap;
+        CK(cudaMemcpyAsync(c->arena, c->host_arena.data(), need * 4, cudaMemcpyHostToDevice,
+                           c->stream), "arena upload");
+    } else if (add > 0) {
+        CK(cudaMemcpyAsync(c->arena + base, c->host_arena.data() + base, add * 4,
+                           cudaMemcpyHostToDevice, c->stream), "arena upload");
+    }
+    for (int i = 0; i < n; ++i) {
+        ids_out[i] = (int32_t)c->pols.size();
+        c->pols.push_back(recs[i]);
+    }
+    if (!c->has_pop && n > 0) {
+        c->has_pop = true;
+        c->spec = *spec;
+        c->pol_kind = pols[0].kind;
+        c->pol_dtype = pols[0].dtype;
+        std::memcpy(c->dims, pols[0].dims, sizeof c->dims);
+    }
+    c->tables_dirty = true;
+    if ((r = upload_tables(c)) != MALIB_OK) return r;
+    return MALIB_OK;
+}
+
+int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
+                         int64_t n_episodes, uint64_t seed, uint32_t flags, double* payoff_out,
+                         const malib_traj* dump, int64_t n_dump) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
+    const int kind = c->spec.env_kind;
+    if (kind != MALIB_ENV_KUHN && kind != MALIB_ENV_LEDUC)
+        return fail(c, MALIB_ESTATE, "payoff evaluation needs a Kuhn or Leduc population");
+    if (flags & ~(MALIB_DUMP_LOGITS | MALIB_EXACT_EXPECTATION))
+        return fail(c, MALIB_EINVAL, "unknown flags 0x%x", flags);
+    const bool exact = (flags & MALIB_EXACT_EXPECTATION) != 0;
+    if (exact && kind != MALIB_ENV_KUHN)
+        return fail(c, MALIB_EUNSUPPORTED, "exact expectation is built for Kuhn only");
+    if (n_pairs < 0) return fail(c, MALIB_EINVAL, "n_pairs < 0");
+    if (n_pairs == 0) return MALIB_OK;
+    if (!pair_ids || !payoff_out) return fail(c, MALIB_EINVAL, "pair_ids or payoff_out is NULL");
+    if (!exact && n_episodes < 1) return fail(c, MALIB_EINVAL, "n_episodes must be >= 1");
+    if (!exact && n_episodes > ((int64_t)1 << 40) / n_pairs)
+        return fail(c, MALIB_EINVAL, "n_pairs * n_episodes too large");
+    if (kind == MALIB_ENV_KUHN && n_pairs > 65535)
+        return fail(c, MALIB_EUNSUPPORTED, "Kuhn evaluation takes at most 65535 pairs per call");
+    const bool want_dump = (flags & MALIB_DUMP_LOGITS) != 0 && !exact;
+    if (want_dump) {
+        if (!dump) return fail(c, MALIB_EINVAL, "MALIB_DUMP_LOGITS without a dump buffer");
+        if (n_dump < 0 || n_dump > n_episodes) return fail(c, MALIB_EINVAL, "n_dump out of range");
+        const void* ptrs[5] = {dump->obs, dump->action, dump->reward, dump->done, dump->logits};
+        for (const void* p : ptrs)
+            if (p && !is_device_ptr(p)) return fail(c, MALIB_EINVAL, "dump buffers must be device memory");
+    }
+    if (kind == MALIB_ENV_LEDUC) {
+        if (c->pol_dtype != MALIB_F32 || !leduc_f32_supported(c->dims[1]) || c->dims[1] != c->dims[2])
+            return fail(c, MALIB_EUNSUPPORTED, "no Leduc kernel for %s hidden %d-%d",
+                        c->pol_dtype == MALIB_BF16 ? "bf16" : "fp32", c->dims[1], c->dims[2]);
+    }
+    int r;
+    if ((r = upload_tables(c)) != MALIB_OK) return r;
+    const int32_t* dpairs = nullptr;
+    if ((r = stage_pairs(c, pair_ids, (int64_t)n_pairs * 2, 2, true, &dpairs)) != MALIB_OK) return r;
+    const bool host_out = !is_device_ptr(payoff_out);
+    double* dout = payoff_out;
+    if (host_out) {
+        if ((r = ensure(c, c->d_out, c->out_cap, (int64_t)n_pairs * 4, "output staging")) != MALIB_OK)
+            return r;
+        dout = c->d_out;
+    }
+    EvalArgs a = eval_args(c);
+    a.pairs = dpairs;
+    a.n_pairs = n_pairs;
+    a.n_episodes = n_episodes;
+    a.seed = seed;
+    if (want_dump) {
+        a.n_dump = n_dump;
+        a.d_obs = dump->obs;
+        a.d_action = dump->action;
+        a.d_reward = dump->reward;
+        a.d_done = dump->done;
+        a.d_logits = dump->logits;
+    }
+    cudaEvent_t e0, e1;
+    if (exact) {
+        time_begin(c, &e0, &e1);
+        CK(launch_kuhn_exact(a, dout, c->stream), "Kuhn exact kernel");
+        time_end(c, e0, e1);
+        c->launches += 1;
+    } else {
+        if ((r = ensure(c, c->acc, c->acc_cap, (int64_t)n_pairs * 2 + 1, "payoff sums")) != MALIB_OK)
+            return r;
+        a.acc = c->acc;
+        a.n_dec = c->acc + (int64_t)n_pairs * 2;
+        c->last_pairs = n_pairs;
+        CK(launch_zero_u64(c->acc, (int64_t)n_pairs * 2 + 1, c->stream), "zero kernel");
+        time_begin(c, &e0, &e1);
+        if (kind == MALIB_ENV_KUHN) {
+            CK(launch_kuhn_eval(a, c->n_sm, c->stream), "Kuhn eval kernel");
+        } else {
+            CK(launch_leduc_eval_f32(a, c->dims[1], c->n_sm, c->stream), "Leduc eval kernel");
+        }
+        time_end(c, e0, e1);
+        CK(launch_finalize(c->acc, n_pairs, n_episodes, dout, c->stream), "finalize kernel");
+        c->launches += 3;
+    }
+    if (host_out) {
+        CK(cudaMemcpyAsync(payoff_out, dout, (size_t)n_pairs * 32, cudaMemcpyDeviceToHost,
+                           c->stream), "payoff download");
+        return read_device_errors(c);
+    }
+    return MALIB_OK;
+}
+
+int malib_eval_payoff(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs, int64_t n_episodes,
+                      uint64_t seed, double* payoff_out) {
+    return malib_eval_payoff_ex(c, pair_ids, n_pairs, n_episodes, seed, 0u, payoff_out, nullptr, 0);
+}
+
+int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids,
+                  int32_t n_pairs, int64_t n_episodes, uint64_t seed, malib_traj* traj) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    int r;
+    if ((r = check_spec(c, spec)) != MALIB_OK) return r;
+    if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
+    if (!same_env(c->spec, *spec))
+        return fail(c, MALIB_ESTATE, "rollout spec differs from the population's environment");
+    if (spec->env_kind != MALIB_ENV_SPREAD)
+        return fail(c, MALIB_EUNSUPPORTED, "rollout is built for the particle spread environment");
+    if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");
+    if (spec->n_envs < 1 || spec->n_envs % n_pairs != 0)
+        return fail(c, MALIB_EINVAL, "n_envs (%lld) must be a positive multiple of n_pairs (%d)",
+                    (long long)spec->n_envs, n_pairs);
+    if (n_episodes < 0) return fail(c, MALIB_EINVAL, "n_episodes < 0");
+    if (!pair_ids || !traj) return fail(c, MALIB_EINVAL, "pair_ids or traj_out is NULL");
+    const bool want_logits = (spec->flags & MALIB_DUMP_LOGITS) != 0;
+    if (!traj->obs || !traj->action || !traj->reward || !traj->done || (want_logits && !traj->logits))
+        return fail(c, MALIB_EINVAL, "trajectory buffer missing");
+    const void* ptrs[5] = {traj->obs, traj->action, traj->reward, traj->done,
+                           want_logits ? traj->logits : traj->obs};
+    for (const void* p : ptrs) {
+        if (!is_device_ptr(p)) return fail(c, MALIB_EINVAL, "trajectory buffers must be device memory");
+        if (((uintptr_t)p & 15u) != 0) return fail(c, MALIB_EINVAL, "trajectory buffers must be 16-byte aligned");
+    }
+    const int64_t epp = spec->n_envs / n_pairs;
+    if (c->pol_dtype != MALIB_F32 || c->dims[1] != c->dims[2] ||
+        !spread_f32_supported(spec->n_agents, spec->obs_dim, c->dims[1]) || epp > 128)
+        return fail(c, MALIB_EUNSUPPORTED,
+                    "no spread kernel for %s N=%d obs %d hidden %d with %lld envs per combination",
+                    c->pol_dtype == MALIB_BF16 ? "bf16" : "fp32", spec->n_agents, spec->obs_dim,
+                    c->dims[1], (long long)epp);
+    if (n_episodes == 0) return MALIB_OK;
+    if ((r = upload_tables(c)) != MALIB_OK) return r;
+    const int32_t* dpairs = nullptr;
+    if ((r = stage_pairs(c, pair_ids, (int64_t)n_pairs * spec->n_agents, spec->n_agents, false,
+                         &dpairs)) != MALIB_OK)
+        return r;
+    RolloutArgs a{};
+    a.arena = c->arena;
+    a.pol_offset = c->d_off;
+    a.n_pol = (int32_t)c->pols.size();
+    a.pairs = dpairs;
+    a.n_pairs = n_pairs;
+    a.n_agents = spec->n_agents;
+    a.obs_dim = spec->obs_dim;
+    a.obs_pad = (spec->obs_dim + 3) / 4 * 4;
+    a.episode_len = spec->episode_len;
+    a.n_envs = spec->n_envs;
+    a.n_episodes = n_episodes;
+    a.seed = seed;
+    a.err = c->d_err;
+    a.obs = traj->obs;
+    a.action = traj->action;
+    a.reward = traj->reward;
+    a.done = traj->done;
+    a.logits = want_logits ? traj->logits : nullptr;
+    cudaEvent_t e0, e1;
+    time_begin(c, &e0, &e1);
+    CK(launch_spread_rollout_f32(a, c->dims[1], c->n_sm, c->stream), "spread rollout kernel");
+    time_end(c, e0, e1);
+    c->launches += 1;
+    return MALIB_OK;
+}
+
+int malib_eval_stats(malib_ctx* c, int64_t* n_decisions) {
+    if (!c || !n_decisions) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    *n_decisions = 0;
+    if (c->last_pairs < 0) return fail(c, MALIB_ESTATE, "no Monte-Carlo evaluation has run");
+    unsigned long long v = 0;
+    CK(cudaMemcpyAsync(&v, c->acc + c->last_pairs * 2, 8, cudaMemcpyDeviceToHost, c->stream),
+       "decision count");
+    CK(cudaStreamSynchronize(c->stream), "sync");
+    *n_decisions = (int64_t)v;
+    return MALIB_OK;
+}
+
+int64_t malib_launch_count(const malib_ctx* c) { return c ? c->launches : 0; }
+
+int malib_set_timing(malib_ctx* c, int enable) {
+    if (!c) return MALIB_EINVAL;
+    c->timing = enable != 0;
+    return MALIB_OK;
+}
+
+double malib_main_kernel_ms(malib_ctx* c, int64_t* n_launches, int reset) {
+    if (!c) return -1.0;
+    DeviceGuard g(c->device);
+    for (auto& ev : c->events) {
+        float ms = 0.f;
+        if (cudaEventSynchronize(ev.second) == cudaSuccess &&
+            cudaEventElapsedTime(&ms, ev.first, ev.second) == cudaSuccess) {
+            c->timed_ms += ms;
+            c->timed_n += 1;
+        }
+        cudaGetLastError();
+        cudaEventDestroy(ev.first);
+        cudaEventDestroy(ev.second);
+    }
+    c->events.clear();
+    const double ms = c->timed_ms;
+    if (n_launches) *n_launches = c->timed_n;
+    if (reset) { c->timed_ms = 0.0; c->timed_n = 0; }
+    return ms;
+}
+
+int malib_selftest_philox(malib_ctx* c, const uint32_t* ctr, uint64_t seed, uint32_t* out,
+                          int64_t n) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (n < 0 || (n > 0 && (!ctr || !out || !is_device_ptr(ctr) || !is_device_ptr(out))))
+        return fail(c, MALIB_EINVAL, "philox self-test needs device buffers");
+    CK(launch_selftest_philox(ctr, seed, out, n, c->stream), "philox kernel");
+    c->launches += n > 0;
+    return MALIB_OK;
+}
+
+int malib_selftest_det_expf(malib_ctx* c, const float* x, float* y, int64_t n) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (n < 0 || (n > 0 && (!x || !y || !is_device_ptr(x) || !is_device_ptr(y))))
+        return fail(c, MALIB_EINVAL, "det_expf self-test needs device buffers");
+    CK(launch_selftest_det_expf(x, y, n, c->stream), "det_expf kernel");
+    c->launches += n > 0;
+    return MALIB_OK;
+}
+
+int malib_selftest_sample(malib_ctx* c, const float* logits, const uint8_t* legal, const float* u,
+                          int32_t A, int32_t* out, int64_t n) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (A < 2 || A > 8) return fail(c, MALIB_EINVAL, "A must be in [2, 8]");
+    if (n < 0 || (n > 0 && (!logits || !legal || !u || !out || !is_device_ptr(logits) ||
+                            !is_device_ptr(legal) || !is_device_ptr(u) || !is_device_ptr(out))))
+        return fail(c, MALIB_EINVAL, "sample self-test needs device buffers");
+    CK(launch_selftest_sample(logits, legal, u, A, out, n, c->stream), "sample kernel");
+    c->launches += n > 0;
+    return MALIB_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,266 @@
+// Batched rollout of the cooperative particle-spread scenario (App. B.1: N
+// agents cover N landmarks; shared reward minus the summed distance from each
+// landmark to its closest agent, minus one per collision) under policy
+// combinations (Sec. 3.1: X ~ P(s, a, s' | a ~ Comb_t)), fp32 MLP policies.
+//
+// Work item = (combination, episode): the combination's block of
+// envs_per_pair environments for T steps. A persistent CTA takes a contiguous
+// range of items (combination-major, so the N policies are staged into shared
+// memory by bulk copy only when the combination changes). One thread steps one
+// environment with its state in registers; per step the N agents' observations
+// form N blocks of rows, each block one policy, run through the fp32 MLP
+// engine; trajectories leave as coalesced 16-byte stores.
+#include "device_common.cuh"
+#include "internal.h"
+#include "mlp_f32.cuh"
+
+namespace malib {
+
+namespace {
+
+template <int N>
+struct SpreadEnv {
+    float px[N], py[N], vx[N], vy[N], lx[N], ly[N];
+};
+
+template <int N>
+__device__ __forceinline__ void spread_reset(SpreadEnv<N>& s, uint64_t g, uint64_t seed) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const U4 d = draw(g, (uint32_t)i, kChance, seed);
+        s.px[i] = __fsub_rn(__fmul_rn(u24(d.x), 2.0f), 1.0f);
+        s.py[i] = __fsub_rn(__fmul_rn(u24(d.y), 2.0f), 1.0f);
+        s.vx[i] = 0.f;
+        s.vy[i] = 0.f;
+    }
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        const U4 d = draw(g, 0x80000000u + (uint32_t)l, kChance, seed);
+        s.lx[l] = __fsub_rn(__fmul_rn(u24(d.x), 2.0f), 1.0f);
+        s.ly[l] = __fsub_rn(__fmul_rn(u24(d.y), 2.0f), 1.0f);
+    }
+}
+
+// Observation of agent i: velocity, position, landmarks relative to the agent,
+// the other agents relative to it (ascending), zeros up to the row stride.
+template <int N, int XS>
+__device__ __forceinline__ void spread_obs(const SpreadEnv<N>& s, int i, float* o) {
+    int k = 0;
+    o[k++] = s.vx[i];
+    o[k++] = s.vy[i];
+    o[k++] = s.px[i];
+    o[k++] = s.py[i];
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        o[k++] = __fsub_rn(s.lx[l], s.px[i]);
+        o[k++] = __fsub_rn(s.ly[l], s.py[i]);
+    }
+#pragma unroll
+    for (int j = 0; j < N; ++j) {
+        if (j == i) continue;
+        o[k++] = __fsub_rn(s.px[j], s.px[i]);
+        o[k++] = __fsub_rn(s.py[j], s.py[i]);
+    }
+    for (; k < XS; ++k) o[k] = 0.f;
+}
+
+__device__ __forceinline__ float dist2(float ax, float ay, float bx, float by) {
+    const float dx = __fsub_rn(ax, bx), dy = __fsub_rn(ay, by);
+    return __fsqrt_rn(__fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy)));
+}
+
+// Mass 1, dt 0.1, damping 0.25, unit force along the chosen axis; reward after
+// the move; collision when centres are closer than 2 x 0.15.
+template <int N>
+__device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N], float (&r)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const float fx = act[i] == 1 ? 1.f : (act[i] == 2 ? -1.f : 0.f);
+        const float fy = act[i] == 3 ? 1.f : (act[i] == 4 ? -1.f : 0.f);
+        s.vx[i] = __fadd_rn(__fmul_rn(s.vx[i], 0.75f), __fmul_rn(fx, 0.1f));
+        s.vy[i] = __fadd_rn(__fmul_rn(s.vy[i], 0.75f), __fmul_rn(fy, 0.1f));
+        s.px[i] = __fadd_rn(s.px[i], __fmul_rn(s.vx[i], 0.1f));
+        s.py[i] = __fadd_rn(s.py[i], __fmul_rn(s.vy[i], 0.1f));
+    }
+    float cover = 0.f;
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        float best = dist2(s.px[0], s.py[0], s.lx[l], s.ly[l]);
+#pragma unroll
+        for (int j = 1; j < N; ++j) {
+            const float d = dist2(s.px[j], s.py[j], s.lx[l], s.ly[l]);
+            best = d < best ? d : best;
+        }
+        cover = __fadd_rn(cover, best);
+    }
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        int coll = 0;
+#pragma unroll
+        for (int j = 0; j < N; ++j)
+            if (j != i && dist2(s.px[i], s.py[i], s.px[j], s.py[j]) < 0.3f) ++coll;
+        r[i] = -__fadd_rn(cover, (float)coll);
+    }
+}
+
+template <int N, int IN, int H>
+struct SpreadF32Smem {
+    using M = MlpF32<IN, H, 5>;
+    using L = typename M::L;
+    static constexpr int RPP = M::kRowsPerPass;
+    static constexpr int kW = 0;
+    static constexpr int kX = kW + N * L::kSize;
+    static constexpr int kH1 = kX + N * RPP * M::XS;
+    static constexpr int kLG = kH1 + RPP * M::HS;
+    static constexpr int kFloats = kLG + N * RPP * M::LS;
+    static constexpr size_t kBytes = (size_t)kFloats * 4;
+};
+
+template <int N, int IN, int H>
+__global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs a) {
+    using SM = SpreadF32Smem<N, IN, H>;
+    using M = typename SM::M;
+    using L = typename SM::L;
+    constexpr int RPP = SM::RPP;
+    constexpr int XS = M::XS;           // == obs_pad
+    extern __shared__ __align__(128) float smem[];
+    float* Ws = smem + SM::kW;
+    float* X = smem + SM::kX;
+    float* H1 = smem + SM::kH1;
+    float* LG = smem + SM::kLG;
+    __shared__ __align__(8) uint64_t bar;
+
+    const int tid = threadIdx.x;
+    for (int i = tid; i < N * RPP * XS; i += blockDim.x) X[i] = 0.f;
+    if (tid == 0) mbar_init(&bar, 1);
+    __syncthreads();
+    uint32_t parity = 0;
+
+    const int epp = (int)(a.n_envs / a.n_pairs);
+    const int T = a.episode_len;
+    const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
+    const int64_t per = (items + gridDim.x - 1) / gridDim.x;
+    const int64_t lo = (int64_t)blockIdx.x * per;
+    const int64_t hi = min(items, lo + per);
+    int staged = -1;
+
+    for (int64_t it = lo; it < hi; ++it) {
+        const int pair = (int)(it / a.n_episodes);
+        const int64_t ep = it - (int64_t)pair * a.n_episodes;
+        if (pair != staged) {
+            bool ok = true;
+            for (int i = 0; i < N; ++i) {
+                const int p = a.pairs[pair * N + i];
+                ok = ok && p >= 0 && p < a.n_pol;
+            }
+            if (!ok) {
+                if (tid == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+                continue;
+            }
+            __syncthreads();   // everyone is done with the previous weights
+            if (tid == 0) {
+                fence_proxy_async_smem();
+                mbar_arrive_expect_tx(&bar, (uint32_t)N * L::kSize * 4u);
+                for (int i = 0; i < N; ++i)
+                    bulk_g2s(Ws + i * L::kSize, a.arena + a.pol_offset[a.pairs[pair * N + i]],
+                             (uint32_t)L::kSize * 4u, &bar);
+            }
+            if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs)) {
+                if (tid == 0) atomicOr(a.err, ERRBIT_TIMEOUT);
+                mbar_wait_bounded(&bar, parity, kWaitLimitNs);
+                return;
+            }
+            parity ^= 1u;
+            staged = pair;
+        }
+
+        const bool mine = tid < epp;
+        const int64_t env = (int64_t)pair * epp + tid;
+        const uint64_t g = (uint64_t)ep * (uint64_t)a.n_envs + (uint64_t)env;
+        SpreadEnv<N> s;
+        if (mine) spread_reset<N>(s, g, a.seed);
+
+        for (int t = 0; t < T; ++t) {
+            if (mine) {
+#pragma unroll
+                for (int i = 0; i < N; ++i) {
+                    float o[XS];
+                    spread_obs<N, XS>(s, i, o);
+                    float4* xr = reinterpret_cast<float4*>(X + (i * RPP + tid) * XS);
+#pragma unroll
+                    for (int q = 0; q < XS / 4; ++q)
+                        xr[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                }
+            }
+            __syncthreads();
+            // coalesced trajectory store of the observations: [ep][t][env][agent][XS]
+            {
+                const int64_t row_base = ((ep * T + t) * a.n_envs + (int64_t)pair * epp) * N;
+                float4* dst = reinterpret_cast<float4*>(a.obs + row_base * XS);
+                const int n4 = epp * N * (XS / 4);
+                for (int q = tid; q < n4; q += blockDim.x) {
+                    const int v = q / (N * (XS / 4));
+                    const int rem = q - v * (N * (XS / 4));
+                    const int i = rem / (XS / 4), c = rem - i * (XS / 4);
+                    dst[q] = *reinterpret_cast<const float4*>(X + (i * RPP + v) * XS + 4 * c);
+                }
+            }
+            for (int i = 0; i < N; ++i)
+                M::pass(X + i * RPP * XS, H1, LG + i * RPP * M::LS, Ws + i * L::kSize, 0,
+                        M::warp_first_row() < epp);
+            if (mine) {
+                int act[N];
+                float r[N];
+                const int64_t ix = ((ep * T + t) * a.n_envs + env) * N;
+#pragma unroll
+                for (int i = 0; i < N; ++i) {
+                    float lg[5];
+#pragma unroll
+                    for (int k = 0; k < 5; ++k) lg[k] = LG[(i * RPP + tid) * M::LS + k];
+                    const float u = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
+                    act[i] = sample_masked<5>(lg, 0x1Fu, u);
+                    if (a.logits)
+#pragma unroll
+                        for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
+                }
+                spread_step<N>(s, act, r);
+#pragma unroll
+                for (int i = 0; i < N; ++i) {
+                    a.action[ix + i] = (uint8_t)act[i];
+                    a.reward[ix + i] = r[i];
+                }
+                a.done[(ep * T + t) * a.n_envs + env] = (t == T - 1) ? 1 : 0;
+            }
+            // X is rewritten next step only after the passes' trailing barrier;
+            // LG is rewritten only after next step's first barrier.
+        }
+    }
+}
+
+template <int N, int IN, int H>
+cudaError_t launch_spread_nih(const RolloutArgs& a, int n_sm, cudaStream_t s) {
+    using SM = SpreadF32Smem<N, IN, H>;
+    cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)SM::kBytes);
+    if (err != cudaSuccess) return err;
+    const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
+    int64_t grid = items < n_sm ? items : n_sm;
+    if (grid < 1) grid = 1;
+    spread_rollout_f32_kernel<N, IN, H><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool spread_f32_supported(int n_agents, int obs_dim, int hidden) {
+    return n_agents == 3 && obs_dim == 18 && hidden == 64;
+}
+
+cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s) {
+    if (a.n_pairs == 0 || a.n_episodes == 0) return cudaSuccess;
+    if (a.n_agents == 3 && a.obs_dim == 18 && hidden == 64) return launch_spread_nih<3, 18, 64>(a, n_sm, s);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace malib
