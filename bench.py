@@ -47,6 +47,8 @@ def parse():
     ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3"], default="leduc")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--hands", type=int, default=None,
+                    help="hands per pair (a smaller case for profiler captures)")
     return ap.parse_args()
 
 
@@ -142,20 +144,21 @@ def load_peaks():
         return {}
 
 
-def workload(name: str, rank: int):
+def workload(name: str, rank: int, hands=None):
     import workloads
+    over = {} if hands is None else {"n_episodes": hands}
     if name == "leduc":
-        w = workloads.config(2)
+        w = workloads.config(2, **over)
     elif name == "kuhn":
-        w = workloads.config(1)
+        w = workloads.config(1, **over)
     else:
-        w = workloads.config(3, n_episodes=100)
+        w = workloads.config(3, **({"n_episodes": 100} if hands is None else over))
     return w
 
 
 def config_of(w, name):
     if name == "leduc":
-        return {"workload": "leduc_holdem_8x8_mlp17-128-128-3_f32_65536hands",
+        return {"workload": f"leduc_holdem_8x8_mlp17-128-128-3_f32_{w.n_episodes}hands",
                 "pairs": w.n_pairs, "hands_per_pair": w.n_episodes,
                 "policy": "MLP 17-128-128-3 fp32", "population_per_seat": w.rows,
                 "l2": "flushed (256 MiB write) before every timed step"}
@@ -258,7 +261,7 @@ def run_ours(args):
     __graft_entry__.build()
     from paper_2106_07551_gb300 import Context, alloc_traj, make_spec, policy_desc
 
-    w = workload(args.workload, rank)
+    w = workload(args.workload, rank, args.hands)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     ctx = Context(local, stream)
