@@ -209,6 +209,30 @@ int malib_eval_payoff_ex(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pair
                          int64_t n_episodes, uint64_t seed, uint32_t flags, double* payoff_out,
                          const malib_traj* dump, int64_t n_dump);
 
+/*
+ * malib_eval_payoff_noalloc - malib_eval_payoff for callers that cannot
+ * allocate device memory during the call. The paper has no counterpart; this is
+ * a deployment variant. Typical callers: a framework that has already
+ * reserved the GPU's memory in its own caching pool, or a latency-critical loop
+ * in which cudaMalloc/cudaFree would synchronise the device and stall other
+ * streams. This call allocates nothing: it calls no cudaMalloc, cudaFree or
+ * allocating library routine. Its scratch (per-pair payoff sums and a decision
+ * counter) is a fixed file-scope device array of 128 KiB + 8 B that every GPU
+ * loading the library holds until the process exits.
+ *  - pair_ids and payoff_out must be DEVICE buffers (layouts as in
+ *    malib_eval_payoff; no host staging). Host buffers give EINVAL.
+ *  - n_pairs <= 8192 (the array's capacity); more gives EINVAL.
+ *  - The population must already be loaded (malib_pop_load), MC mode only,
+ *    no dump; same results as malib_eval_payoff for the same arguments.
+ *    malib_eval_stats does not report its decision count.
+ *  - The first call on a device looks the array's device address up
+ *    (cudaGetSymbolAddress); make that first call before any stream capture.
+ *  - Every call shares the array and clears it first; calls that overlap on
+ *    the GPU (other streams or contexts on the same device) race on it.
+ */
+int malib_eval_payoff_noalloc(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pairs,
+                              int64_t n_episodes, uint64_t seed, double* payoff_out);
+
 /* ---- measurement and self-test entry points (used by tests and the benchmark) ---- */
 
 /* Total decisions (env-steps: one decision by the acting seat) played by the

@@ -20,7 +20,7 @@ from ._abi import (MALIB_BF16, MALIB_DUMP_LOGITS, MALIB_ENV_KUHN, MALIB_ENV_LEDU
 
 __all__ = ["MalibError", "Context", "EnvSpec", "make_spec", "policy_desc", "alloc_traj",
            "alloc_eval_dump", "malib_create", "malib_pop_load", "malib_rollout",
-           "malib_eval_payoff", "malib_eval_payoff_ex", "MALIB_ENV_KUHN", "MALIB_ENV_LEDUC",
+           "malib_eval_payoff", "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "MALIB_ENV_KUHN", "MALIB_ENV_LEDUC",
            "MALIB_ENV_SPREAD", "MALIB_POL_TABULAR", "MALIB_POL_MLP", "MALIB_F32", "MALIB_BF16",
            "MALIB_DUMP_LOGITS", "MALIB_EXACT_EXPECTATION"]
 
@@ -110,6 +110,14 @@ def malib_eval_payoff_ex(ctx, pair_ids, n_episodes, seed, flags, payoff_out, dum
     _check(lib, ctx, lib.malib_eval_payoff_ex(ctx, _ptr(pair_ids), int(pair_ids.shape[0]),
                                               n_episodes, seed, flags, _ptr(payoff_out),
                                               C.byref(t) if t is not None else None, n_dump))
+
+
+def malib_eval_payoff_noalloc(ctx, pair_ids, n_episodes: int, seed: int, payoff_out):
+    """Payoff table without any device allocation in the call (device pair table
+    and output, at most 8192 pairs); see include/malib.h."""
+    lib = _abi.load()
+    _check(lib, ctx, lib.malib_eval_payoff_noalloc(ctx, _ptr(pair_ids), int(pair_ids.shape[0]),
+                                                   n_episodes, seed, _ptr(payoff_out)))
 
 
 def alloc_traj(spec: EnvSpec, n_episodes: int, logits: bool = False, device="cuda"):

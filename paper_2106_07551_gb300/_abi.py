@@ -25,7 +25,8 @@ MALIB_DUMP_LOGITS, MALIB_EXACT_EXPECTATION = 1, 2
 EXPORTS = (
     "malib_create", "malib_destroy", "malib_last_error", "malib_sync", "malib_set_stream",
     "malib_pop_load", "malib_pop_reset", "malib_rollout", "malib_eval_payoff",
-    "malib_eval_payoff_ex", "malib_eval_stats", "malib_launch_count", "malib_set_timing", "malib_main_kernel_ms",
+    "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "malib_eval_stats", "malib_launch_count",
+    "malib_set_timing", "malib_main_kernel_ms",
     "malib_selftest_philox", "malib_selftest_det_expf", "malib_selftest_sample",
 )
 
@@ -79,6 +80,7 @@ def load(path: str | None = None):
             "malib_rollout": (C.c_int, [P, C.POINTER(EnvSpec), P, i32, i64, u64, C.POINTER(Traj)]),
             "malib_eval_payoff": (C.c_int, [P, P, i32, i64, u64, P]),
             "malib_eval_payoff_ex": (C.c_int, [P, P, i32, i64, u64, u32, P, C.POINTER(Traj), i64]),
+            "malib_eval_payoff_noalloc": (C.c_int, [P, P, i32, i64, u64, P]),
             "malib_eval_stats": (C.c_int, [P, C.POINTER(C.c_int64)]),
             "malib_launch_count": (C.c_int64, [P]),
             "malib_set_timing": (C.c_int, [P, C.c_int]),

@@ -92,6 +92,26 @@ cudaError_t launch_selftest_det_expf(const float* x, float* y, int64_t n, cudaSt
 cudaError_t launch_selftest_sample(const float* logits, const uint8_t* legal, const float* u,
                                    int A, int32_t* out, int64_t n, cudaStream_t s);
 
+// Read-only view of a context for entry points defined outside runtime.cu.
+struct CtxView {
+    int device;
+    cudaStream_t stream;
+    int n_sm;
+    bool has_pop;
+    int env_kind;
+    int pol_dtype;
+    int dims[4];
+    const float* arena;
+    const int64_t* pol_offset;
+    const int32_t* pol_seat;
+    int32_t n_pol;
+    int* err;
+    bool tables_uploaded;
+};
+bool ctx_view(const void* ctx, CtxView* v);
+int ctx_fail(void* ctx, int code, const char* msg);
+void ctx_count_launches(void* ctx, int n);
+
 bool leduc_f32_supported(int hidden);
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden);
 

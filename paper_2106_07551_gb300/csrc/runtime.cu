@@ -278,6 +278,37 @@ EvalArgs eval_args(malib_ctx* c) {
 
 }  // namespace
 
+namespace malib {
+
+bool ctx_view(const void* ctx, CtxView* v) {
+    const malib_ctx* c = static_cast<const malib_ctx*>(ctx);
+    if (!c || !v) return false;
+    v->device = c->device;
+    v->stream = c->stream;
+    v->n_sm = c->n_sm;
+    v->has_pop = c->has_pop;
+    v->env_kind = c->spec.env_kind;
+    v->pol_dtype = c->pol_dtype;
+    for (int i = 0; i < 4; ++i) v->dims[i] = c->dims[i];
+    v->arena = c->arena;
+    v->pol_offset = c->d_off;
+    v->pol_seat = c->d_seat;
+    v->n_pol = (int32_t)c->pols.size();
+    v->err = c->d_err;
+    v->tables_uploaded = !c->tables_dirty;
+    return true;
+}
+
+int ctx_fail(void* ctx, int code, const char* msg) {
+    return fail(static_cast<malib_ctx*>(ctx), code, "%s", msg);
+}
+
+void ctx_count_launches(void* ctx, int n) {
+    if (ctx) static_cast<malib_ctx*>(ctx)->launches += n;
+}
+
+}  // namespace malib
+
 extern "C" {
 
 int malib_create(malib_ctx** out, int device, void* cuda_stream) {

@@ -1,0 +1,74 @@
+"""The allocation-free payoff evaluation (malib_eval_payoff_noalloc).
+
+It exists for callers that cannot allocate device memory while they evaluate:
+a framework that has reserved the GPU's memory in its own pool, or a
+latency-critical loop where cudaMalloc / cudaFree would synchronise the device.
+Its scratch is a fixed device array inside the library, so this test checks,
+through the C ABI, that two calls in a row give exactly the table of the
+ordinary allocating entry point (integer sums bit-exact, mean and SE to 1e-12),
+that the shared scratch is cleared between calls, and that sizes beyond the
+array's capacity and host buffers are refused. This file is collected last.
+"""
+import ctypes as C
+
+import numpy as np
+import pytest
+
+import workloads
+from gpu_util import context, load_population, need_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+def _noalloc(ctx, pairs, n_eps, seed, out):
+    from paper_2106_07551_gb300 import _abi
+    lib = _abi.load()
+    return lib.malib_eval_payoff_noalloc(ctx.handle, C.c_void_p(pairs.data_ptr()),
+                                         int(pairs.shape[0]), n_eps, seed,
+                                         C.c_void_p(out.data_ptr()))
+
+
+@pytest.mark.parametrize("kind", ["leduc", "kuhn"])
+def test_noalloc_matches_allocating_entry_point(kind):
+    torch = need_gpu()
+    w = (workloads.leduc(pop=4, with_bias=True, seed=77) if kind == "leduc"
+         else workloads.kuhn())
+    n_eps = 3000 if kind == "leduc" else 10_000
+    ctx = context()
+    load_population(ctx, w)
+    d_pairs = torch.from_numpy(w.pair_ids).cuda()
+    for seed in (5, 6):
+        ref = ctx.eval_payoff(w.pair_ids, n_eps, seed)
+        for _ in range(2):   # two calls in a row share (and must clear) the scratch
+            out = torch.full((w.n_pairs, 4), -1.0, dtype=torch.float64, device="cuda")
+            assert _noalloc(ctx, d_pairs, n_eps, seed, out) == 0, ctx.last_error()
+            ctx.sync()
+            got = out.cpu().numpy()
+            np.testing.assert_array_equal(got[:, 2:], ref[:, 2:])
+            np.testing.assert_allclose(got[:, :2], ref[:, :2], rtol=1e-12, atol=1e-15)
+    # a smaller table after a larger one: stale sums must not leak in
+    out = torch.zeros((3, 4), dtype=torch.float64, device="cuda")
+    assert _noalloc(ctx, d_pairs[:3].contiguous(), n_eps, 9, out) == 0
+    ctx.sync()
+    ref = ctx.eval_payoff(w.pair_ids[:3].copy(), n_eps, 9)
+    np.testing.assert_array_equal(out.cpu().numpy()[:, 2:], ref[:, 2:])
+    ctx.close()
+
+
+def test_noalloc_refuses_oversize_and_host_buffers():
+    torch = need_gpu()
+    from paper_2106_07551_gb300 import _abi
+    w = workloads.kuhn()
+    ctx = context()
+    load_population(ctx, w)
+    big = torch.from_numpy(np.tile(w.pair_ids, (8193 // w.n_pairs + 1, 1))[:8193].copy()).cuda()
+    out = torch.zeros((8193, 4), dtype=torch.float64, device="cuda")
+    assert _noalloc(ctx, big, 10, 0, out) == _abi.MALIB_EINVAL
+    assert "8192" in ctx.last_error()
+    lib = _abi.load()
+    h_out = np.zeros((w.n_pairs, 4), np.float64)
+    d_pairs = torch.from_numpy(w.pair_ids).cuda()
+    code = lib.malib_eval_payoff_noalloc(ctx.handle, C.c_void_p(d_pairs.data_ptr()), w.n_pairs,
+                                         10, 0, h_out.ctypes.data_as(C.c_void_p))
+    assert code == _abi.MALIB_EINVAL
+    ctx.close()
