@@ -6,7 +6,11 @@
 // pass of rows x H outputs as TY row-groups of 4 rows times TX column-groups of
 // 8 columns (columns {4tx..4tx+3} and {H/2+4tx..}); each k step then costs one
 // 16-byte load of the 4 rows' inputs (amortised over 4 k) and two 16-byte
-// weight loads for 32 FMAs. Every row-group may use its own policy (the caller
+// weight loads for 32 FMAs. A 16-byte shared load is served per half-warp, one
+// 128-byte wavefront per 128 distinct bytes, so lanes are laid out to give
+// every half-warp 8 column groups x 2 row groups: a weight load then costs 2
+// wavefronts per warp and an input load 2 (16 column groups in a half-warp
+// would cost 4 per weight load). Every row-group may use its own policy (the caller
 // passes that group's weight pointer), so rows compacted by acting policy in
 // multiples of 4 need no further sorting. Layer 3 is folded into layer 2's
 // epilogue: per-thread partial dot products reduced across the TX lanes of the
@@ -27,11 +31,25 @@ struct MlpF32 {
     static constexpr int XS = (IN + 3) / 4 * 4;   // input row stride (floats)
     static constexpr int HS = H + 4;              // hidden row stride (bank-skewed)
     static constexpr int LS = (A + 3) / 4 * 4;    // logits row stride
-    static_assert(TX >= 1 && TX <= 32 && (32 % TX) == 0, "column groups must tile a warp");
+    static constexpr int TYW = 32 / TX;           // row-groups per warp
+    static_assert(TX == 8 || TX == 16, "8 or 16 column groups (H = 64 or 128)");
     static_assert(A <= 8, "at most 8 actions");
 
+    // Lane -> (column group, row group). TX 16: lanes 0-7 and 8-15 hold column
+    // groups 0-7 of row groups 2w and 2w+1, lanes 16-31 column groups 8-15.
+    // TX 8: lanes 8r..8r+7 hold column groups 0-7 of row group 4w+r.
+    __device__ static int col_group() {
+        const int lane = threadIdx.x & 31;
+        return TX == 16 ? ((lane & 7) | ((lane >> 4) << 3)) : (lane & 7);
+    }
+    __device__ static int row_group() {
+        const int lane = threadIdx.x & 31;
+        const int tyl = TX == 16 ? ((lane >> 3) & 1) : (lane >> 3);
+        return (threadIdx.x >> 5) * TYW + tyl;
+    }
+
     // First local row of the warp's first row-group (for warp-uniform skips).
-    __device__ static int warp_first_row() { return ((threadIdx.x & ~31) / TX) * 4; }
+    __device__ static int warp_first_row() { return (threadIdx.x >> 5) * TYW * 4; }
 
     // One pass: rows [row0, row0 + kRowsPerPass) of X -> the same rows of LG.
     // w: weight blob of the calling thread's row-group. `active` must be
@@ -39,8 +57,8 @@ struct MlpF32 {
     __device__ static void pass(const float* __restrict__ X, float* __restrict__ H1,
                                 float* __restrict__ LG, const float* __restrict__ w, int row0,
                                 bool active) {
-        const int tx = threadIdx.x % TX;
-        const int ty = threadIdx.x / TX;
+        const int tx = col_group();
+        const int ty = row_group();
         const int lr = ty * 4;
         const int c0 = tx * 4, c1 = H / 2 + tx * 4;
         float acc[4][8];
@@ -144,8 +162,11 @@ struct MlpF32 {
                     pl[i][a] = s;
                 }
             }
+            // reduce over the lanes of the row-group: tx bits are lane bits
+            // 0-2 (and lane bit 4 when TX = 16)
 #pragma unroll
-            for (int o = TX / 2; o > 0; o >>= 1) {
+            for (int o = 1; o <= (TX == 16 ? 16 : 4); o <<= 1) {
+                if (o == 8) continue;
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
 #pragma unroll

@@ -344,7 +344,7 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_kernel(EvalArgs a) {
             }
             __syncthreads();
             for (int r0 = 0; r0 < rows; r0 += M::kRowsPerPass) {
-                const int grp = r0 + (tid / M::TX) * 4;
+                const int grp = r0 + M::row_group() * 4;
                 const float* w = grp < base1 ? Ws : Ws + L::kSize;
                 M::pass(X, H1, LG, w, r0, r0 + M::warp_first_row() < rows);
             }
