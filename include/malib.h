@@ -262,6 +262,15 @@ int malib_selftest_det_expf(malib_ctx* ctx, const float* x, float* y, int64_t n)
 int malib_selftest_sample(malib_ctx* ctx, const float* logits, const uint8_t* legal,
                           const float* u, int32_t A, int32_t* out, int64_t n);
 
+/* Tensor-core self-test: D[128][N] = A[128][K] . B[N][K]^T on one CTA with
+ * tcgen05 MMAs from shared memory and an fp32 accumulator in tensor memory -
+ * the operand layout and MMA path of the bf16 policy kernels. dtype MALIB_BF16:
+ * A, B hold bf16 bit patterns (K % 16 == 0); MALIB_F32: A, B fp32, multiplied
+ * as tf32 (K % 8 == 0). N % 16 == 0, 16 <= N <= 256; all device buffers,
+ * row-major. */
+int malib_selftest_mma(malib_ctx* ctx, int32_t dtype, const void* A, const void* B, float* D,
+                       int32_t N, int32_t K);
+
 #ifdef __cplusplus
 }
 #endif

@@ -234,6 +234,12 @@ class Context:
         _check(self.lib, self.handle,
                self.lib.malib_selftest_det_expf(self.handle, _ptr(x), _ptr(y), int(x.numel())))
 
+    def selftest_mma(self, dtype, A, B, D):
+        """D = A . B^T on the tensor cores (A [128][K], B [N][K]; bf16 bits or fp32)."""
+        N, K = int(B.shape[0]), int(B.shape[1])
+        _check(self.lib, self.handle,
+               self.lib.malib_selftest_mma(self.handle, dtype, _ptr(A), _ptr(B), _ptr(D), N, K))
+
     def selftest_sample(self, logits, legal, u, out):
         n, A = logits.shape
         _check(self.lib, self.handle,

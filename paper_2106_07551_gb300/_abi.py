@@ -28,6 +28,7 @@ EXPORTS = (
     "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "malib_eval_stats", "malib_launch_count",
     "malib_set_timing", "malib_main_kernel_ms",
     "malib_selftest_philox", "malib_selftest_det_expf", "malib_selftest_sample",
+    "malib_selftest_mma",
 )
 
 
@@ -88,6 +89,7 @@ def load(path: str | None = None):
             "malib_selftest_philox": (C.c_int, [P, P, u64, P, i64]),
             "malib_selftest_det_expf": (C.c_int, [P, P, P, i64]),
             "malib_selftest_sample": (C.c_int, [P, P, P, P, i32, P, i64]),
+            "malib_selftest_mma": (C.c_int, [P, i32, P, P, P, i32, i32]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)

@@ -1,0 +1,133 @@
+// 5th-generation tensor-core (tcgen05) building blocks for sm_103a: tensor
+// memory allocation, shared-memory matrix descriptors in the no-swizzle
+// K-major layout, instruction descriptors, MMA issue and completion, and tensor
+// memory loads. Single-CTA (cta_group::1) forms only.
+//
+// Operand layout ("core-matrix K-major, no swizzle"): a tile of R rows x K
+// elements is stored as core matrices of 8 rows x 16 bytes (rows 16 bytes
+// apart, 128 contiguous bytes). Core matrix (row group g = row / 8, K chunk
+// c = k / (16 / element size)) sits at byte ((c * R/8) + g) * 128, so
+// consecutive row groups are 128 B apart (SBO) and consecutive K chunks R*16 B
+// apart (LBO). One MMA consumes 2 K chunks (K = 16 bf16 or 8 tf32); the k-th
+// MMA's descriptor starts 2k chunks in.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "device_common.cuh"
+
+namespace malib {
+namespace tc {
+
+// Byte offset of element (row, k) in the core-matrix layout of a tile with
+// `rows` rows (multiple of 8) and elements of `es` bytes.
+__host__ __device__ __forceinline__ uint32_t cm_offset(int row, int k, int rows, int es) {
+    const int per_chunk = 16 / es;
+    const int c = k / per_chunk, w = k % per_chunk;
+    return (uint32_t)((c * (rows / 8) + (row >> 3)) * 128 + (row & 7) * 16 + w * es);
+}
+
+// Shared-memory matrix descriptor (tcgen05): start address, leading (K) and
+// stride (row-group) byte offsets, all >> 4; bits 46-47 = 1; no swizzle.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t smem_addr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((smem_addr >> 4) & 0x3FFFu);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    return d;
+}
+
+// Instruction descriptor, dense, D fp32, A and B K-major.
+// ab_format: 1 = bf16 (kind::f16), 2 = tf32 (kind::tf32).
+__host__ __device__ __forceinline__ uint32_t instr_desc(int M, int N, int ab_format) {
+    uint32_t d = 0;
+    d |= 1u << 4;                             // D format fp32
+    d |= (uint32_t)ab_format << 7;            // A format
+    d |= (uint32_t)ab_format << 10;           // B format
+    d |= (uint32_t)(N >> 3) << 17;            // N / 8
+    d |= (uint32_t)(M >> 4) << 24;            // M / 16
+    return d;
+}
+
+// ---- tensor memory (one warp executes alloc / relinquish / dealloc) --------
+__device__ __forceinline__ void tmem_alloc(uint32_t* smem_dst, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(smem_dst)),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+
+__device__ __forceinline__ void fence_before_sync() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_after_sync() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// ---- MMA (issued by one thread) ---------------------------------------------
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         bool accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"((uint32_t)accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         bool accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"((uint32_t)accumulate)
+        : "memory");
+}
+// Arrives on the mbarrier once every MMA issued so far by this thread is done.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            smem_u32(bar))
+        : "memory");
+}
+
+// ---- tensor memory -> registers: lanes of this warp's quarter, 32 columns ---
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+        "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, "
+        "%28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// TMEM address of (lane, column) given the allocation base.
+__device__ __forceinline__ uint32_t tmem_addr(uint32_t base, int lane, int col) {
+    return base + ((uint32_t)lane << 16) + (uint32_t)col;
+}
+
+// bf16 round-to-nearest-even of two floats packed low/high.
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+}  // namespace tc
+}  // namespace malib

@@ -68,3 +68,36 @@ def test_sample_bit_exact(ctx, orc, A):
     ctx.selftest_sample(d[0], d[1], d[2], out)
     ctx.sync()
     np.testing.assert_array_equal(out.cpu().numpy(), orc.sample(lg, legal, u))
+
+
+@pytest.mark.parametrize("dtype,N,K", [("bf16", 256, 256), ("bf16", 16, 16), ("bf16", 128, 48),
+                                       ("tf32", 256, 128), ("tf32", 64, 24)])
+def test_tensor_core_gemm(ctx, dtype, N, K):
+    """tcgen05 MMA with the kernels' operand layout against an fp64 matmul of
+    the same (bf16 / tf32-truncated) operands."""
+    torch = need_gpu()
+    from paper_2106_07551_gb300 import MALIB_BF16, MALIB_F32
+    g = torch.Generator().manual_seed(N * 1000 + K)
+    A = torch.randn(128, K, generator=g)
+    B = torch.randn(N, K, generator=g)
+    if dtype == "bf16":
+        Ab, Bb = A.to(torch.bfloat16), B.to(torch.bfloat16)
+        ref = Ab.double() @ Bb.double().T
+        dA, dB = Ab.view(torch.int16).cuda(), Bb.view(torch.int16).cuda()
+        code = MALIB_BF16
+    else:
+        mask = torch.tensor(-8192, dtype=torch.int32)      # keep 19 high bits (tf32)
+        At = (A.view(torch.int32) & mask).view(torch.float32)
+        Bt = (B.view(torch.int32) & mask).view(torch.float32)
+        ref = At.double() @ Bt.double().T
+        dA, dB = A.cuda(), B.cuda()
+        code = MALIB_F32
+    D = torch.full((128, N), float("nan"), device="cuda")
+    ctx.selftest_mma(code, dA, dB, D)
+    ctx.sync()
+    got = D.cpu().double()
+    scale = ref.abs().max().item()
+    err = (got - ref).abs().max().item()
+    # tf32 inputs may be rounded rather than truncated by the unit: allow 2^-10
+    tol = (1e-5 if dtype == "bf16" else 2e-3) * scale
+    assert err <= tol, (err, scale)
