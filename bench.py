@@ -44,7 +44,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3"], default="leduc")
+    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "leduc_bf16"],
+                    default="leduc")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--hands", type=int, default=None,
@@ -149,6 +150,8 @@ def workload(name: str, rank: int, hands=None):
     over = {} if hands is None else {"n_episodes": hands}
     if name == "leduc":
         w = workloads.config(2, **over)
+    elif name == "leduc_bf16":
+        w = workloads.config(5, **over)
     elif name == "kuhn":
         w = workloads.config(1, **over)
     else:
@@ -161,6 +164,11 @@ def config_of(w, name):
         return {"workload": f"leduc_holdem_8x8_mlp17-128-128-3_f32_{w.n_episodes}hands",
                 "pairs": w.n_pairs, "hands_per_pair": w.n_episodes,
                 "policy": "MLP 17-128-128-3 fp32", "population_per_seat": w.rows,
+                "l2": "flushed (256 MiB write) before every timed step"}
+    if name == "leduc_bf16":
+        return {"workload": f"leduc_holdem_64x64_mlp17-256-256-3_bf16_{w.n_episodes}hands",
+                "pairs": w.n_pairs, "hands_per_pair": w.n_episodes,
+                "policy": "MLP 17-256-256-3 bf16 (fp32 accumulate)", "population_per_seat": w.rows,
                 "l2": "flushed (256 MiB write) before every timed step"}
     if name == "kuhn":
         return {"workload": "kuhn_4x4_tabular_10000hands", "pairs": w.n_pairs,
@@ -184,7 +192,7 @@ def oracle_leduc_sample(w, target_s: float, threads: int):
         dec = np.zeros(w.n_pairs, np.int64)
         t0 = time.perf_counter()
         oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, w.seed, n_sim=n,
-                          decisions=dec, n_threads=threads)
+                          decisions=dec, n_threads=threads, bf16=w.policies[0].dtype == 1)
         return time.perf_counter() - t0, int(dec.sum())
 
     n = 8
@@ -281,6 +289,7 @@ def run_ours(args):
     else:
         d_out = torch.empty((w.n_pairs, 4), dtype=torch.float64, device=dev)
         flop_per_unit = mlp_flop(w.policies[0].dims) if w.env_kind == 2 else 0
+    tensor = args.workload == "leduc_bf16"
 
     def step(seed):
         if rollout:
@@ -332,21 +341,28 @@ def run_ours(args):
     achieved = (decisions * flop_per_unit / args.steps) / (kern_ms / kern_n / 1e3) / 1e12 \
         if kern_n else 0.0
     kname = {"leduc": "leduc_eval_f32_kernel<128>", "kuhn": "kuhn_eval_kernel",
-             "spread3": "spread_rollout_f32_kernel<3,18,64>"}[args.workload]
-    roofline = {"bound": "alu", "achieved": achieved, "peak": peak_tflops, "unit": "TFLOP/s",
+             "spread3": "spread_rollout_f32_kernel<3,18,64>",
+             "leduc_bf16": "leduc_eval_tc_kernel"}[args.workload]
+    basis = (f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"
+             f" x {sm_max:.0f} MHz (max SM clock of MEASURED_PEAKS.json)")
+    if tensor:
+        peak_tflops = float(peaks.get("bf16_tflops_sustained", 1700.0))
+        basis = "measured cuBLAS bf16 dense, sustained (MEASURED_PEAKS.json bf16_tflops_sustained)"
+    roofline = {"bound": "tensor" if tensor else "alu", "achieved": achieved,
+                "peak": peak_tflops, "unit": "TFLOP/s",
                 "frac": achieved / peak_tflops if peak_tflops else None,
                 "traffic": NCU_TRAFFIC_PER_LAUNCH.get(kname),
                 "kernel": kname, "kernel_ms_per_launch": kern_ms / max(1, kern_n),
-                "peak_basis": f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"
-                              f" x {sm_max:.0f} MHz (max SM clock of MEASURED_PEAKS.json)",
+                "peak_basis": basis,
                 "algorithmic": f"{flop_per_unit} flop per env-step (MLP forward, padding excluded)"}
-    if clk.get("sm_mhz"):
+    if clk.get("sm_mhz") and not tensor:
         roofline["frac_at_measured_clock"] = achieved / (peak_tflops * clk["sm_mhz"] / sm_max)
 
     e2e = run_e2e(args, ctx, w, spec, dev, rollout) if rank == 0 else None
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload == "leduc":
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload in ("leduc",
+                                                                                 "leduc_bf16"):
         rate, sample = oracle_leduc_sample(w, 12.0, cpu_count())
         cpu = {"value": rate, "unit": UNIT, "cores": cpu_count(), "kind": "oracle",
                "sample": sample}

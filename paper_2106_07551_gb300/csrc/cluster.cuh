@@ -1,0 +1,97 @@
+// Thread-block-cluster helpers: distributed shared memory (DSMEM) access to a
+// peer CTA's shared memory and a cluster-wide synchronisation whose waits are
+// bounded (epoch flags polled with a time limit, never an unbounded barrier).
+#pragma once
+
+#include <cstdint>
+
+#include "device_common.cuh"
+
+namespace malib {
+namespace cl {
+
+__device__ __forceinline__ uint32_t rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// shared::cluster address of `p` (this CTA's shared memory) in CTA `r`.
+__device__ __forceinline__ uint32_t map(const void* p, uint32_t r) {
+    uint32_t out;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(out) : "r"(smem_u32(p)), "r"(r));
+    return out;
+}
+
+__device__ __forceinline__ void st_u32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_f32(uint32_t addr, float v) {
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void st_v4(uint32_t addr, uint4 v) {
+    asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x),
+                 "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+__device__ __forceinline__ uint32_t ld_u32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ uint32_t atomic_add(uint32_t addr, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.relaxed.cluster.shared::cluster.add.u32 %0, [%1], %2;"
+                 : "=r"(old)
+                 : "r"(addr), "r"(v)
+                 : "memory");
+    return old;
+}
+
+__device__ __forceinline__ void fence_cluster() {
+    asm volatile("fence.acq_rel.cluster;" ::: "memory");
+}
+
+// Cluster-wide synchronisation. Every thread of every CTA of the cluster calls
+// it with the same epoch (increasing). flags: this CTA's array of `size`
+// epoch slots (one per source CTA), zero-initialised and never reset. Each
+// thread publishes its shared-memory writes (fence), the CTA synchronises, and
+// thread r stores the epoch into slot [my rank] of CTA r; thread 0 then polls
+// its own slots until every source has reached the epoch, for at most
+// kWaitLimitNs. Returns false (and raises ERRBIT_TIMEOUT) on expiry; callers
+// keep executing the same sequence of syncs so that no CTA of the cluster is
+// left waiting.
+__device__ __forceinline__ bool sync(uint32_t* flags, uint32_t epoch, uint32_t size, uint32_t me,
+                                     int* err, uint32_t* ok_slot) {
+    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+    fence_cluster();
+    __syncthreads();
+    if (threadIdx.x < size) {
+        const uint32_t a = map(&flags[me], threadIdx.x);
+        asm volatile("st.release.cluster.shared::cluster.u32 [%0], %1;" ::"r"(a), "r"(epoch)
+                     : "memory");
+    }
+    if (threadIdx.x == 0) {
+        bool ok = true;
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t r = 0; r < size && ok; ++r) {
+            while (true) {
+                uint32_t v;
+                asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];"
+                             : "=r"(v)
+                             : "r"(smem_u32(&flags[r]))
+                             : "memory");
+                if ((int32_t)(v - epoch) >= 0) break;
+                if (globaltimer_ns() - t0 > kWaitLimitNs) { ok = false; break; }
+            }
+        }
+        if (!ok) atomicOr(err, ERRBIT_TIMEOUT);
+        *ok_slot = ok ? 1u : 0u;
+    }
+    __syncthreads();
+    fence_cluster();
+    return *ok_slot != 0;
+}
+
+}  // namespace cl
+}  // namespace malib

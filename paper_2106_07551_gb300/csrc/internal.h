@@ -34,6 +34,18 @@ struct F32Layout {
     static_assert(IN * H % 4 == 0 && H % 8 == 0, "layout alignment");
 };
 
+// bf16 tensor-core policy image (bytes): W1 [256][K1], W2 [256][256], W3 [16][256]
+// as bf16 in the core-matrix K-major layout (K1 = input width rounded up to
+// 16, rows past the output width zero), then fp32 b1[256], b2[256], b3[16].
+// Built for populations with h1 = h2 = 256, input <= 48, output <= 16.
+inline bool tc_image_shape(const int* d) {
+    return d[1] == 256 && d[2] == 256 && d[0] >= 1 && d[0] <= 48 && d[3] >= 1 && d[3] <= 16;
+}
+inline int64_t tc_image_bytes(int in) {
+    const int64_t k1 = (in + 15) / 16 * 16;
+    return 256 * k1 * 2 + 256 * 256 * 2 + 16 * 256 * 2 + (256 + 256 + 16) * 4;
+}
+
 // Output sums of the payoff reduction: per pair {sum r, sum r^2} as 64-bit
 // two's complement (integers, so any summation order gives the same bits).
 struct EvalArgs {
@@ -82,6 +94,7 @@ struct RolloutArgs {
 cudaError_t launch_kuhn_eval(const EvalArgs& a, int n_sm, cudaStream_t s);
 cudaError_t launch_kuhn_exact(const EvalArgs& a, double* out, cudaStream_t s);
 cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s);
+cudaError_t launch_leduc_eval_tc(const EvalArgs& a, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s);
 cudaError_t launch_zero_u64(unsigned long long* p, int64_t n, cudaStream_t s);
 cudaError_t launch_finalize(const unsigned long long* acc, int32_t n_pairs, int64_t n_episodes,

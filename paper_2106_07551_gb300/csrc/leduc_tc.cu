@@ -1,0 +1,243 @@
+// Payoff-table evaluation of Leduc hold'em with bf16 MLP policies on the
+// tensor cores (Sec. 3.2 payoff table, Sec. 4.2 Monte-Carlo simulations per
+// policy combination).
+//
+// A cluster of two CTAs evaluates one pair at a time. CTA r keeps the policy of
+// seat r resident in shared memory (bf16 weight image, ~155 KB) and owns 128
+// hands in flight. Each step, every live hand claims a row in the tile of the
+// CTA whose seat is to act (remote atomic on that CTA's row counter) and writes
+// its bf16 observation there through distributed shared memory; each CTA then
+// runs its 128-row tile through the tensor-core MLP and writes the logits back
+// to the hands' owners. A hand that finds the tile full waits for the next
+// step (its randomness depends only on its own ids, so deferral changes no
+// result). Both CTAs take the same pair segments and leave a segment together,
+// when neither tile received a row.
+#include "cluster.cuh"
+#include "device_common.cuh"
+#include "eval_common.cuh"
+#include "internal.h"
+#include "leduc_env.cuh"
+#include "mlp_tc.cuh"
+
+namespace malib {
+
+namespace {
+
+using Eng = MlpTc<32, 256, 16>;
+constexpr int kSlots = 128;               // hands per CTA
+constexpr int kThreads = 256;
+constexpr uint32_t kLg = Eng::kSmemBytes;                 // logits by slot [128][4] fp32
+constexpr uint32_t kOwner = kLg + kSlots * 16;            // row -> (rank << 16 | slot)
+constexpr uint32_t kSmem = kOwner + 128 * 4;
+constexpr int kMaxDec = 8;
+
+__device__ __forceinline__ void cluster_barrier_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    leduc_eval_tc_kernel(EvalArgs a) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    __shared__ __align__(8) uint64_t stage_bar;
+    __shared__ __align__(8) uint64_t mma_bar;
+    __shared__ uint32_t tmem_base;
+    __shared__ uint32_t flags[2];
+    __shared__ uint32_t ctr[2];
+    __shared__ uint32_t ok_slot;
+    __shared__ unsigned long long next_k;
+
+    float* lgbuf = reinterpret_cast<float*>(smem + kLg);
+    uint32_t* owner = reinterpret_cast<uint32_t*>(smem + kOwner);
+    const uint32_t me = cl::rank(), peer = me ^ 1u;
+    const int tid = threadIdx.x;
+
+    if (tid == 0) {
+        mbar_init(&stage_bar, 1);
+        mbar_init(&mma_bar, 1);
+        flags[0] = flags[1] = 0;
+        ctr[0] = ctr[1] = 0;
+    }
+    if ((tid >> 5) == 0) {
+        tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
+        tc::tmem_relinquish();
+    }
+    // zero the activation tile so rows never read uninitialised bits
+    for (uint32_t i = tid * 16; i < Eng::kActBytes; i += kThreads * 16)
+        *reinterpret_cast<uint4*>(smem + Eng::kAct + i) = make_uint4(0, 0, 0, 0);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    cluster_barrier_all();          // peers' counters and flags exist before any remote access
+    const uint32_t tbase = tmem_base;
+
+    uint32_t stage_par = 0, mma_par = 0, epoch = 0, step = 0;
+    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+    const int64_t n_cl = gridDim.x / 2, cid = blockIdx.x / 2;
+    const int64_t per = (total + n_cl - 1) / n_cl;
+    const int64_t lo = cid * per, hi = min(total, lo + per);
+
+    for (int64_t seg = lo; seg < hi;) {
+        const int pair = (int)(seg / a.n_episodes);
+        const int64_t e_lo = seg - (int64_t)pair * a.n_episodes;
+        const int64_t e_hi = min(a.n_episodes, e_lo + (hi - seg));
+        seg += e_hi - e_lo;
+        const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
+        if (!pair_ok(a, p0, p1)) {          // same decision in both CTAs
+            if (tid == 0 && me == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+            continue;
+        }
+        const int pol = me == 0 ? p0 : p1;
+        const float* policy = a.arena + a.pol_offset[pol];
+        const float* bias = policy + Eng::kImageBytes / 4;
+        if (tid == 0) {
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(&stage_bar, Eng::kImageBytes);
+            for (uint32_t off = 0; off < Eng::kImageBytes; off += 32768u)
+                bulk_g2s(smem + off, reinterpret_cast<const uint8_t*>(policy) + off,
+                         min(32768u, Eng::kImageBytes - off), &stage_bar);
+        }
+        if (!mbar_wait_bounded(&stage_bar, stage_par, kWaitLimitNs) && tid == 0)
+            atomicOr(a.err, ERRBIT_TIMEOUT);
+        stage_par ^= 1u;
+
+        // this CTA's hands: e = e_lo + me + 2k
+        LeducHand h;
+        bool live = false;
+        int64_t e = -1;
+        uint64_t g = 0;
+        int t = 0;
+        long long s1 = 0, s2 = 0, nd = 0;
+        if (tid < kSlots) {
+            e = e_lo + me + 2 * (int64_t)tid;
+            live = e < e_hi;
+            if (live) {
+                g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+                leduc_deal(h, g, a.seed);
+            }
+        }
+        if (tid == 0) next_k = kSlots;
+        __syncthreads();
+
+        while (true) {
+            const uint32_t par = step & 1u;
+            bool placed = false;
+            float ob[17];
+            if (live) {
+                const uint32_t target = (uint32_t)h.actor;
+                const uint32_t row = cl::atomic_add(cl::map(&ctr[par], target), 1u);
+                if (row < 128) {
+                    placed = true;
+                    leduc_obs(h, ob);
+                    uint32_t w[16];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        w[i] = tc::pack_bf16(ob[2 * i], 2 * i + 1 < 17 ? ob[2 * i + 1] : 0.f);
+                    w[8] = tc::pack_bf16(ob[16], 0.f);
+#pragma unroll
+                    for (int i = 9; i < 16; ++i) w[i] = 0u;
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        cl::st_v4(cl::map(smem + Eng::kAct + Eng::act_offset((int)row, 8 * c), target),
+                                  make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]));
+                    cl::st_u32(cl::map(&owner[row], target), (me << 16) | (uint32_t)tid);
+                }
+            }
+            fence_proxy_async_smem();
+            asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
+            const uint32_t n_me = ctr[par];
+            const uint32_t n_peer = cl::ld_u32(cl::map(&ctr[par], peer));
+            if (n_me == 0 && n_peer == 0) break;
+            const int rows = (int)min(n_me, 128u);
+            Eng::forward(smem, bias, tbase, &mma_bar, mma_par, rows, a.err,
+                         [&](int row, const float* lg) {
+                             const uint32_t o = owner[row];
+                             const uint32_t dst = cl::map(lgbuf + (o & 0xFFFFu) * 4, o >> 16);
+                             cl::st_f32(dst, lg[0]);
+                             cl::st_f32(dst + 4, lg[1]);
+                             cl::st_f32(dst + 8, lg[2]);
+                         });
+            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
+            if (tid == 0) ctr[par] = 0;
+            if (placed) {
+                float lg[3] = {lgbuf[tid * 4], lgbuf[tid * 4 + 1], lgbuf[tid * 4 + 2]};
+                const unsigned legal = leduc_legal(h);
+                const int seat = h.actor;
+                const float u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);
+                const int act = sample_masked<3>(lg, legal, u);
+                const bool rec = e < a.n_dump;
+                const int64_t rb = ((int64_t)pair * a.n_dump + e) * kMaxDec;
+                if (rec) {
+                    if (a.d_obs) {
+                        float* o = a.d_obs + (rb + t) * 20;
+#pragma unroll
+                        for (int i = 0; i < 17; ++i) o[i] = ob[i];
+                        o[17] = 0.f; o[18] = 0.f; o[19] = 0.f;
+                    }
+                    if (a.d_logits) {
+                        float* l = a.d_logits + (rb + t) * 3;
+                        l[0] = lg[0]; l[1] = lg[1]; l[2] = lg[2];
+                    }
+                    if (a.d_action) a.d_action[rb + t] = (uint8_t)act;
+                }
+                leduc_apply(h, act);
+                if (rec) {
+                    if (a.d_reward) a.d_reward[rb + t] = h.done ? (float)h.payoff : 0.f;
+                    if (a.d_done) a.d_done[rb + t] = h.done ? 1 : 0;
+                }
+                ++t;
+                ++nd;
+                if (h.done) {
+                    s1 += h.payoff;
+                    s2 += (long long)h.payoff * h.payoff;
+                    if (rec) {
+                        for (int k = t; k < kMaxDec; ++k) {
+                            if (a.d_obs)
+                                for (int i = 0; i < 20; ++i) a.d_obs[(rb + k) * 20 + i] = 0.f;
+                            if (a.d_logits)
+                                for (int i = 0; i < 3; ++i) a.d_logits[(rb + k) * 3 + i] = 0.f;
+                            if (a.d_action) a.d_action[rb + k] = 255;
+                            if (a.d_reward) a.d_reward[rb + k] = 0.f;
+                            if (a.d_done) a.d_done[rb + k] = 1;
+                        }
+                    }
+                    const int64_t k = (int64_t)atomicAdd(&next_k, 1ull);
+                    e = e_lo + me + 2 * k;
+                    live = e < e_hi;
+                    if (live) {
+                        g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+                        leduc_deal(h, g, a.seed);
+                        t = 0;
+                    }
+                }
+            }
+            ++step;
+        }
+        block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+    }
+    tc::fence_before_sync();
+    __syncthreads();
+    cluster_barrier_all();          // no peer touches this CTA's shared memory after this
+    if ((tid >> 5) == 0) tc::tmem_dealloc(tbase, Eng::kTmemCols);
+}
+
+}  // namespace
+
+uint32_t leduc_tc_policy_floats() { return Eng::kPolicyBytes / 4; }
+
+cudaError_t launch_leduc_eval_tc(const EvalArgs& a, int n_sm, cudaStream_t s) {
+    if (a.n_pairs == 0) return cudaSuccess;
+    cudaError_t err = cudaFuncSetAttribute(leduc_eval_tc_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+    if (err != cudaSuccess) return err;
+    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+    int64_t clusters = (total + 2 * kSlots - 1) / (2 * kSlots);
+    const int64_t max_clusters = n_sm / 2;
+    if (clusters > max_clusters) clusters = max_clusters;
+    if (clusters < 1) clusters = 1;
+    leduc_eval_tc_kernel<<<(unsigned)(2 * clusters), kThreads, kSmem, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace malib

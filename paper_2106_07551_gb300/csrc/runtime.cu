@@ -12,6 +12,7 @@
 
 #include "internal.h"
 #include "malib.h"
+#include "tc_common.cuh"
 
 using namespace malib;
 
@@ -35,6 +36,7 @@ struct malib_ctx {
     malib_env_spec spec{};
     int pol_kind = 0, pol_dtype = 0;
     int dims[4] = {0, 0, 0, 0};
+    bool tc_layout = false;            // bf16 tensor-core images in the arena
     std::vector<PolicyRec> pols;
     std::vector<float> host_arena;     // mirror of the device arena
     float* arena = nullptr;
@@ -185,6 +187,43 @@ void to_f32_layout(const float* p, const int* d, float* out, int64_t size) {
     for (int i = 0; i < a * h2; ++i) o[i] = W3[i];
     o += (int64_t)a * h2;
     for (int j = 0; j < a; ++j) o[j] = b3[j];
+}
+
+// bf16 tensor-core image (internal.h) from the plain fp32 layout.
+void to_tc_image(const float* p, const int* d, float* out_floats) {
+    const int in = d[0], H = 256, A = d[3];
+    const int k1 = (in + 15) / 16 * 16;
+    const float* W1 = p;
+    const float* b1 = W1 + (int64_t)H * in;
+    const float* W2 = b1 + H;
+    const float* b2 = W2 + (int64_t)H * H;
+    const float* W3 = b2 + H;
+    const float* b3 = W3 + (int64_t)A * H;
+    uint8_t* img = reinterpret_cast<uint8_t*>(out_floats);
+    const int64_t bytes = tc_image_bytes(in);
+    std::memset(img, 0, (size_t)bytes);
+    auto bf = [](float x) -> uint16_t {
+        uint32_t b;
+        std::memcpy(&b, &x, 4);
+        if ((b & 0x7F800000u) != 0x7F800000u) b += 0x7FFFu + ((b >> 16) & 1u);
+        return (uint16_t)(b >> 16);
+    };
+    auto put = [&](uint8_t* base, int row, int k, int rows, float v) {
+        const uint16_t h = bf(v);
+        std::memcpy(base + tc::cm_offset(row, k, rows, 2), &h, 2);
+    };
+    uint8_t* w1 = img;
+    uint8_t* w2 = w1 + (int64_t)H * k1 * 2;
+    uint8_t* w3 = w2 + (int64_t)H * H * 2;
+    float* bias = reinterpret_cast<float*>(w3 + 16 * H * 2);
+    for (int n = 0; n < H; ++n)
+        for (int k = 0; k < in; ++k) put(w1, n, k, H, W1[(int64_t)n * in + k]);
+    for (int n = 0; n < H; ++n)
+        for (int k = 0; k < H; ++k) put(w2, n, k, H, W2[(int64_t)n * H + k]);
+    for (int n = 0; n < A; ++n)
+        for (int k = 0; k < H; ++k) put(w3, n, k, 16, W3[(int64_t)n * H + k]);
+    for (int j = 0; j < H; ++j) { bias[j] = b1[j]; bias[H + j] = b2[j]; }
+    for (int j = 0; j < A; ++j) bias[2 * H + j] = b3[j];
 }
 
 int upload_tables(malib_ctx* c) {
@@ -442,6 +481,12 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
             const int64_t size = ((int64_t)d.dims[0] * d.dims[1] + d.dims[1] +
                                   (int64_t)d.dims[1] * d.dims[2] + d.dims[2] +
                                   (int64_t)d.dims[3] * d.dims[2] + d.dims[3] + 3) / 4 * 4;
+            if (d.dtype == MALIB_BF16 && tc_image_shape(d.dims)) {
+                converted[i].assign((size_t)(tc_image_bytes(d.dims[0]) / 4), 0.f);
+                to_tc_image(plain.data(), d.dims, converted[i].data());
+                recs[i] = rec;
+                continue;
+            }
             if (d.dtype == MALIB_BF16) {
                 // weights rounded to bf16 (nearest even); biases stay fp32
                 auto rne = [](float x) {
@@ -509,6 +554,8 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
         c->pol_kind = pols[0].kind;
         c->pol_dtype = pols[0].dtype;
         std::memcpy(c->dims, pols[0].dims, sizeof c->dims);
+        c->tc_layout = pols[0].kind == MALIB_POL_MLP && pols[0].dtype == MALIB_BF16 &&
+                       tc_image_shape(pols[0].dims);
     }
     c->tables_dirty = true;
     if ((r = upload_tables(c)) != MALIB_OK) return r;
@@ -545,7 +592,9 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
         for (const void* p : ptrs)
             if (p && !is_device_ptr(p)) return fail(c, MALIB_EINVAL, "dump buffers must be device memory");
     }
-    if (kind == MALIB_ENV_LEDUC) {
+    const bool leduc_tc = kind == MALIB_ENV_LEDUC && c->tc_layout && c->dims[0] == 17 &&
+                          c->dims[3] == 3;
+    if (kind == MALIB_ENV_LEDUC && !leduc_tc) {
         if (c->pol_dtype != MALIB_F32 || !leduc_f32_supported(c->dims[1]) || c->dims[1] != c->dims[2])
             return fail(c, MALIB_EUNSUPPORTED, "no Leduc kernel for %s hidden %d-%d",
                         c->pol_dtype == MALIB_BF16 ? "bf16" : "fp32", c->dims[1], c->dims[2]);
@@ -590,6 +639,8 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
         time_begin(c, &e0, &e1);
         if (kind == MALIB_ENV_KUHN) {
             CK(launch_kuhn_eval(a, c->n_sm, c->stream), "Kuhn eval kernel");
+        } else if (leduc_tc) {
+            CK(launch_leduc_eval_tc(a, c->n_sm, c->stream), "Leduc tensor-core eval kernel");
         } else {
             CK(launch_leduc_eval_f32(a, c->dims[1], c->n_sm, c->stream), "Leduc eval kernel");
         }
