@@ -44,7 +44,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "leduc_bf16"],
+    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "leduc_bf16", "spread8"],
                     default="leduc")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -154,6 +154,8 @@ def workload(name: str, rank: int, hands=None):
         w = workloads.config(5, **over)
     elif name == "kuhn":
         w = workloads.config(1, **over)
+    elif name == "spread8":
+        w = workloads.config(4, **({"n_episodes": 2} if hands is None else over))
     else:
         w = workloads.config(3, **({"n_episodes": 100} if hands is None else over))
     return w
@@ -170,6 +172,10 @@ def config_of(w, name):
                 "pairs": w.n_pairs, "hands_per_pair": w.n_episodes,
                 "policy": "MLP 17-256-256-3 bf16 (fp32 accumulate)", "population_per_seat": w.rows,
                 "l2": "flushed (256 MiB write) before every timed step"}
+    if name == "spread8":
+        return {"workload": f"spread_n8_65536env_mlp34-256-256-5_bf16_{w.n_episodes}episodes",
+                "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
+                "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
     if name == "kuhn":
         return {"workload": "kuhn_4x4_tabular_10000hands", "pairs": w.n_pairs,
                 "hands_per_pair": w.n_episodes,
@@ -281,7 +287,7 @@ def run_ours(args):
     d_pairs = torch.from_numpy(w.pair_ids).to(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     seed0 = w.seed + 1_000_003 * rank
-    rollout = args.workload == "spread3"
+    rollout = args.workload in ("spread3", "spread8")
     if rollout:
         traj = alloc_traj(spec, w.n_episodes)
         steps_per_call = w.n_envs * w.episode_len * w.n_episodes
@@ -289,7 +295,7 @@ def run_ours(args):
     else:
         d_out = torch.empty((w.n_pairs, 4), dtype=torch.float64, device=dev)
         flop_per_unit = mlp_flop(w.policies[0].dims) if w.env_kind == 2 else 0
-    tensor = args.workload == "leduc_bf16"
+    tensor = args.workload in ("leduc_bf16", "spread8")
 
     def step(seed):
         if rollout:
@@ -342,7 +348,8 @@ def run_ours(args):
         if kern_n else 0.0
     kname = {"leduc": "leduc_eval_f32_kernel<128>", "kuhn": "kuhn_eval_kernel",
              "spread3": "spread_rollout_f32_kernel<3,18,64>",
-             "leduc_bf16": "leduc_eval_tc_kernel"}[args.workload]
+             "leduc_bf16": "leduc_eval_tc_kernel",
+             "spread8": "spread_rollout_tc_kernel"}[args.workload]
     basis = (f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"
              f" x {sm_max:.0f} MHz (max SM clock of MEASURED_PEAKS.json)")
     if tensor:

@@ -54,19 +54,19 @@ __device__ __forceinline__ void fence_cluster() {
 
 // Cluster-wide synchronisation. Every thread of every CTA of the cluster calls
 // it with the same epoch (increasing). flags: this CTA's array of `size`
-// epoch slots (one per source CTA), zero-initialised and never reset. Each
-// thread publishes its shared-memory writes (fence), the CTA synchronises, and
-// thread r stores the epoch into slot [my rank] of CTA r; thread 0 then polls
+// epoch slots (one per source CTA), zero-initialised and never reset. The CTA
+// synchronises (so the signalling threads have observed every write of the
+// CTA), then thread r releases the epoch into slot [my rank] of CTA r at
+// cluster scope; thread 0 then polls
 // its own slots until every source has reached the epoch, for at most
 // kWaitLimitNs. Returns false (and raises ERRBIT_TIMEOUT) on expiry; callers
 // keep executing the same sequence of syncs so that no CTA of the cluster is
 // left waiting.
 __device__ __forceinline__ bool sync(uint32_t* flags, uint32_t epoch, uint32_t size, uint32_t me,
                                      int* err, uint32_t* ok_slot) {
-    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
-    fence_cluster();
     __syncthreads();
     if (threadIdx.x < size) {
+        fence_cluster();
         const uint32_t a = map(&flags[me], threadIdx.x);
         asm volatile("st.release.cluster.shared::cluster.u32 [%0], %1;" ::"r"(a), "r"(epoch)
                      : "memory");
@@ -89,7 +89,6 @@ __device__ __forceinline__ bool sync(uint32_t* flags, uint32_t epoch, uint32_t s
         *ok_slot = ok ? 1u : 0u;
     }
     __syncthreads();
-    fence_cluster();
     return *ok_slot != 0;
 }
 

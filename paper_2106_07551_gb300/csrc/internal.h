@@ -96,6 +96,8 @@ cudaError_t launch_kuhn_exact(const EvalArgs& a, double* out, cudaStream_t s);
 cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s);
 cudaError_t launch_leduc_eval_tc(const EvalArgs& a, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s);
+cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s);
+bool spread_tc_supported(int n_agents, int obs_dim, int n_actions, int64_t envs_per_pair);
 cudaError_t launch_zero_u64(unsigned long long* p, int64_t n, cudaStream_t s);
 cudaError_t launch_finalize(const unsigned long long* acc, int32_t n_pairs, int64_t n_episodes,
                             double* out, cudaStream_t s);

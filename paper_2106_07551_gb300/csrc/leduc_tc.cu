@@ -3,15 +3,16 @@
 // policy combination).
 //
 // A cluster of two CTAs evaluates one pair at a time. CTA r keeps the policy of
-// seat r resident in shared memory (bf16 weight image, ~155 KB) and owns 128
-// hands in flight. Each step, every live hand claims a row in the tile of the
-// CTA whose seat is to act (remote atomic on that CTA's row counter) and writes
-// its bf16 observation there through distributed shared memory; each CTA then
-// runs its 128-row tile through the tensor-core MLP and writes the logits back
-// to the hands' owners. A hand that finds the tile full waits for the next
-// step (its randomness depends only on its own ids, so deferral changes no
-// result). Both CTAs take the same pair segments and leave a segment together,
-// when neither tile received a row.
+// seat r resident in shared memory (bf16 weight image and biases, ~157 KB) and
+// owns 128 hands in flight. Rows 64 s .. 64 s + 63 of each CTA's 128-row tile
+// belong to the hands of CTA s. Each step, the hands of a CTA are ranked by
+// acting seat with warp ballots; the first 64 acting as seat r write their bf16
+// observation into rows of CTA r's tile through distributed shared memory (the
+// rest wait a step: a hand's randomness depends only on its own ids, so
+// deferral changes no result). Each CTA runs its tile through the tensor-core
+// MLP and returns every valid row's logits to the hand's CTA. Both CTAs take
+// the same pair segments and leave a segment together, when neither holds a
+// live hand.
 #include "cluster.cuh"
 #include "device_common.cuh"
 #include "eval_common.cuh"
@@ -25,10 +26,10 @@ namespace {
 
 using Eng = MlpTc<32, 256, 16>;
 constexpr int kSlots = 128;               // hands per CTA
+constexpr int kPart = 64;                 // tile rows per source CTA
 constexpr int kThreads = 256;
-constexpr uint32_t kLg = Eng::kSmemBytes;                 // logits by slot [128][4] fp32
-constexpr uint32_t kOwner = kLg + kSlots * 16;            // row -> (rank << 16 | slot)
-constexpr uint32_t kSmem = kOwner + 128 * 4;
+constexpr uint32_t kLg = Eng::kSmemBytes;                 // logits [target][row][4] fp32
+constexpr uint32_t kSmem = kLg + 2 * 128 * 16;
 constexpr int kMaxDec = 8;
 
 __device__ __forceinline__ void cluster_barrier_all() {
@@ -38,37 +39,36 @@ __device__ __forceinline__ void cluster_barrier_all() {
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     leduc_eval_tc_kernel(EvalArgs a) {
-    extern __shared__ __align__(1024) uint8_t smem[];
+    extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t stage_bar;
     __shared__ __align__(8) uint64_t mma_bar;
     __shared__ uint32_t tmem_base;
     __shared__ uint32_t flags[2];
-    __shared__ uint32_t ctr[2];
+    __shared__ uint32_t nrows[2];         // valid rows from each source CTA (this step)
+    __shared__ uint32_t live_of[2];       // live hands of each CTA (this step)
+    __shared__ int wcnt[2][8];
     __shared__ uint32_t ok_slot;
     __shared__ unsigned long long next_k;
 
     float* lgbuf = reinterpret_cast<float*>(smem + kLg);
-    uint32_t* owner = reinterpret_cast<uint32_t*>(smem + kOwner);
-    const uint32_t me = cl::rank(), peer = me ^ 1u;
-    const int tid = threadIdx.x;
+    const uint32_t me = cl::rank();
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
     if (tid == 0) {
         mbar_init(&stage_bar, 1);
         mbar_init(&mma_bar, 1);
         flags[0] = flags[1] = 0;
-        ctr[0] = ctr[1] = 0;
     }
-    if ((tid >> 5) == 0) {
+    if (warp == 0) {
         tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
         tc::tmem_relinquish();
     }
-    // zero the activation tile so rows never read uninitialised bits
     for (uint32_t i = tid * 16; i < Eng::kActBytes; i += kThreads * 16)
         *reinterpret_cast<uint4*>(smem + Eng::kAct + i) = make_uint4(0, 0, 0, 0);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
-    cluster_barrier_all();          // peers' counters and flags exist before any remote access
+    cluster_barrier_all();          // peers' flags exist before any remote access
     const uint32_t tbase = tmem_base;
 
     uint32_t stage_par = 0, mma_par = 0, epoch = 0, step = 0;
@@ -87,15 +87,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (tid == 0 && me == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
             continue;
         }
-        const int pol = me == 0 ? p0 : p1;
-        const float* policy = a.arena + a.pol_offset[pol];
-        const float* bias = policy + Eng::kImageBytes / 4;
+        const float* policy = a.arena + a.pol_offset[me == 0 ? p0 : p1];
         if (tid == 0) {
             fence_proxy_async_smem();
-            mbar_arrive_expect_tx(&stage_bar, Eng::kImageBytes);
-            for (uint32_t off = 0; off < Eng::kImageBytes; off += 32768u)
+            mbar_arrive_expect_tx(&stage_bar, Eng::kStageBytes);
+            for (uint32_t off = 0; off < Eng::kStageBytes; off += 32768u)
                 bulk_g2s(smem + off, reinterpret_cast<const uint8_t*>(policy) + off,
-                         min(32768u, Eng::kImageBytes - off), &stage_bar);
+                         min(32768u, Eng::kStageBytes - off), &stage_bar);
         }
         if (!mbar_wait_bounded(&stage_bar, stage_par, kWaitLimitNs) && tid == 0)
             atomicOr(a.err, ERRBIT_TIMEOUT);
@@ -117,53 +115,62 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
         }
         if (tid == 0) next_k = kSlots;
-        __syncthreads();
 
         while (true) {
-            const uint32_t par = step & 1u;
-            bool placed = false;
-            float ob[17];
-            if (live) {
-                const uint32_t target = (uint32_t)h.actor;
-                const uint32_t row = cl::atomic_add(cl::map(&ctr[par], target), 1u);
-                if (row < 128) {
-                    placed = true;
-                    leduc_obs(h, ob);
-                    uint32_t w[16];
+            // rank this CTA's live hands by acting seat
+            const int seat = live ? h.actor : -1;
+            const unsigned b0 = __ballot_sync(0xffffffffu, seat == 0);
+            const unsigned b1 = __ballot_sync(0xffffffffu, seat == 1);
+            if (lane == 0) { wcnt[0][warp] = __popc(b0); wcnt[1][warp] = __popc(b1); }
+            __syncthreads();
+            int pre = 0, c0 = 0, c1 = 0;
 #pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        w[i] = tc::pack_bf16(ob[2 * i], 2 * i + 1 < 17 ? ob[2 * i + 1] : 0.f);
-                    w[8] = tc::pack_bf16(ob[16], 0.f);
-#pragma unroll
-                    for (int i = 9; i < 16; ++i) w[i] = 0u;
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        cl::st_v4(cl::map(smem + Eng::kAct + Eng::act_offset((int)row, 8 * c), target),
-                                  make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]));
-                    cl::st_u32(cl::map(&owner[row], target), (me << 16) | (uint32_t)tid);
-                }
+            for (int w = 0; w < 8; ++w) {
+                c0 += wcnt[0][w];
+                c1 += wcnt[1][w];
+                if (w < warp) pre += seat == 1 ? wcnt[1][w] : wcnt[0][w];
             }
-            fence_proxy_async_smem();
-            asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
-            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
-            const uint32_t n_me = ctr[par];
-            const uint32_t n_peer = cl::ld_u32(cl::map(&ctr[par], peer));
-            if (n_me == 0 && n_peer == 0) break;
-            const int rows = (int)min(n_me, 128u);
-            Eng::forward(smem, bias, tbase, &mma_bar, mma_par, rows, a.err,
-                         [&](int row, const float* lg) {
-                             const uint32_t o = owner[row];
-                             const uint32_t dst = cl::map(lgbuf + (o & 0xFFFFu) * 4, o >> 16);
-                             cl::st_f32(dst, lg[0]);
-                             cl::st_f32(dst + 4, lg[1]);
-                             cl::st_f32(dst + 8, lg[2]);
-                         });
-            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
-            if (tid == 0) ctr[par] = 0;
+            const unsigned mine = seat == 1 ? b1 : b0;
+            const int rank = pre + __popc(mine & ((1u << lane) - 1u));
+            const bool placed = live && rank < kPart;
+            const int row = (int)me * kPart + rank;
+            float ob[17];
             if (placed) {
-                float lg[3] = {lgbuf[tid * 4], lgbuf[tid * 4 + 1], lgbuf[tid * 4 + 2]};
+                const uint32_t target = (uint32_t)seat;
+                leduc_obs(h, ob);
+                uint32_t w[16];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) w[i] = tc::pack_bf16(ob[2 * i], ob[2 * i + 1]);
+                w[8] = tc::pack_bf16(ob[16], 0.f);
+#pragma unroll
+                for (int i = 9; i < 16; ++i) w[i] = 0u;
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    cl::st_v4(cl::map(smem + Eng::kAct + Eng::act_offset(row, 8 * c), target),
+                              make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]));
+                asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+            }
+            if (tid < 2) {                  // thread s tells CTA s how many rows it got from us
+                const uint32_t n = (uint32_t)min(tid == 0 ? c0 : c1, kPart);
+                cl::st_u32(cl::map(&nrows[me], (uint32_t)tid), n);
+                cl::st_u32(cl::map(&live_of[me], (uint32_t)tid), (uint32_t)(c0 + c1));
+            }
+            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
+            if (live_of[0] == 0 && live_of[1] == 0) break;
+            Eng::forward(smem, nullptr, tbase, &mma_bar, mma_par, a.err, [&](int r, const float* lg) {
+                const uint32_t src = (uint32_t)(r / kPart);
+                if ((uint32_t)(r % kPart) < nrows[src]) {
+                    const uint32_t dst = cl::map(lgbuf + (me * 128 + r) * 4, src);
+                    cl::st_f32(dst, lg[0]);
+                    cl::st_f32(dst + 4, lg[1]);
+                    cl::st_f32(dst + 8, lg[2]);
+                }
+            });
+            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
+            if (placed) {
+                const float* lp = lgbuf + (seat * 128 + row) * 4;
+                float lg[3] = {lp[0], lp[1], lp[2]};
                 const unsigned legal = leduc_legal(h);
-                const int seat = h.actor;
                 const float u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);
                 const int act = sample_masked<3>(lg, legal, u);
                 const bool rec = e < a.n_dump;
@@ -219,7 +226,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tc::fence_before_sync();
     __syncthreads();
     cluster_barrier_all();          // no peer touches this CTA's shared memory after this
-    if ((tid >> 5) == 0) tc::tmem_dealloc(tbase, Eng::kTmemCols);
+    if (warp == 0) tc::tmem_dealloc(tbase, Eng::kTmemCols);
 }
 
 }  // namespace

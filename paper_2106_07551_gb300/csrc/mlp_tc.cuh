@@ -6,10 +6,11 @@
 // Shared memory holds the policy's weight image (staged once by bulk copy):
 // W1 [H][K1], W2 [H][H], W3 [NOUT][H] in the core-matrix K-major layout of
 // tc_common.cuh (K1 = input width padded to 16, NOUT = actions padded to 16),
-// followed by one activation tile [128][H]. The observation tile X [128][K1]
-// lives at the start of that activation tile: every layer's A operand is the
-// previous layer's output, so X, h1 and h2 reuse the same 64 KB. Biases are
-// read from global memory (L1-resident). One 256-column TMEM accumulator is
+// then the fp32 biases b1 [H], b2 [H], b3 [NOUT] (staged with the image), then
+// one activation tile [128][H]. The observation tile X [128][K1] lives at the
+// start of that activation tile: every layer's A operand is the previous
+// layer's output, so X, h1 and h2 reuse the same 64 KB. One 256-column TMEM
+// accumulator is
 // reused by the three layers. Thread 0 issues the MMAs; the 8 warps split each
 // epilogue (warp w: TMEM lane quarter w % 4, column half w / 4).
 #pragma once
@@ -21,7 +22,9 @@
 
 namespace malib {
 
-template <int K1, int H, int NOUT>
+// kSmemBias: stage the biases with the weights (true) or read them from the
+// policy's global image through L1 (false, when shared memory is short).
+template <int K1, int H, int NOUT, bool kSmemBias = true>
 struct MlpTc {
     static_assert(K1 % 16 == 0 && H == 256 && NOUT == 16, "shapes built: K1 % 16, H 256, NOUT 16");
     static constexpr uint32_t kW1 = 0;
@@ -29,10 +32,13 @@ struct MlpTc {
     static constexpr uint32_t kW3 = kW2 + H * H * 2;
     static constexpr uint32_t kImageBytes = kW3 + NOUT * H * 2;     // staged into shared memory
     static constexpr uint32_t kBiasFloats = H + H + NOUT;           // b1, b2, b3 after the image
-    static constexpr uint32_t kPolicyBytes = kImageBytes + kBiasFloats * 4;
-    static constexpr uint32_t kAct = kImageBytes;                   // activation tile offset
+    static constexpr uint32_t kPolicyBytes = kImageBytes + kBiasFloats * 4;   // global image
+    static constexpr uint32_t kStageBytes = kSmemBias ? kPolicyBytes : kImageBytes;
+    static constexpr uint32_t kBias = kImageBytes;                  // biases (after the image)
+    static constexpr uint32_t kAct = kStageBytes;                   // activation tile offset
     static constexpr uint32_t kActBytes = 128 * H * 2;
-    static constexpr uint32_t kSmemBytes = kImageBytes + kActBytes;
+    static constexpr uint32_t kSmemBytes = kStageBytes + kActBytes;
+    static_assert(kStageBytes % 16 == 0, "activation tile 16-byte aligned");
     static constexpr uint32_t kTmemCols = 256;
     static constexpr uint32_t kLboAct = (128 / 8) * 128;            // K-chunk stride, 128 rows
     static constexpr uint32_t kLboW = (H / 8) * 128;                // K-chunk stride, H rows
@@ -58,26 +64,35 @@ struct MlpTc {
     }
 
     // D + bias -> relu -> bf16 into the activation tile (this thread: one row,
-    // one half of the H columns).
-    __device__ static void epilogue_hidden(uint8_t* act, const float* __restrict__ bias,
-                                           uint32_t tbase) {
+    // one half of the H columns; 64 columns per tensor-memory wait).
+    __device__ static void epilogue_hidden(uint8_t* act, const float* bias, uint32_t tbase) {
         const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
         const int q = warp & 3, half = warp >> 2;
         const int row = 32 * q + lane;
 #pragma unroll 1
-        for (int cc = 0; cc < H / 2 / 32; ++cc) {
-            const int c0 = half * (H / 2) + cc * 32;
-            float v[32];
-            tc::tmem_ld32(tc::tmem_addr(tbase, 32 * q, c0), v);
+        for (int cc = 0; cc < H / 2 / 64; ++cc) {
+            const int c0 = half * (H / 2) + cc * 64;
+            uint32_t r0[32], r1[32];
+            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0), r0);
+            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0 + 32), r1);
+            tc::tmem_wait_ld();
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float4 b0 = __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j));
-                const float4 b1 = __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4));
+            for (int j = 0; j < 8; ++j) {
+                const uint32_t* r = j < 4 ? r0 : r1;
+                const int jj = (j & 3) * 8;
+                const float4 b0 = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 8 * j)
+                                            : __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j));
+                const float4 b1 = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4)
+                                            : __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4));
                 uint4 pk;
-                pk.x = tc::pack_bf16(fmaxf(v[8 * j + 0] + b0.x, 0.f), fmaxf(v[8 * j + 1] + b0.y, 0.f));
-                pk.y = tc::pack_bf16(fmaxf(v[8 * j + 2] + b0.z, 0.f), fmaxf(v[8 * j + 3] + b0.w, 0.f));
-                pk.z = tc::pack_bf16(fmaxf(v[8 * j + 4] + b1.x, 0.f), fmaxf(v[8 * j + 5] + b1.y, 0.f));
-                pk.w = tc::pack_bf16(fmaxf(v[8 * j + 6] + b1.z, 0.f), fmaxf(v[8 * j + 7] + b1.w, 0.f));
+                pk.x = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 0]) + b0.x, 0.f),
+                                     fmaxf(__uint_as_float(r[jj + 1]) + b0.y, 0.f));
+                pk.y = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 2]) + b0.z, 0.f),
+                                     fmaxf(__uint_as_float(r[jj + 3]) + b0.w, 0.f));
+                pk.z = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 4]) + b1.x, 0.f),
+                                     fmaxf(__uint_as_float(r[jj + 5]) + b1.y, 0.f));
+                pk.w = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 6]) + b1.z, 0.f),
+                                     fmaxf(__uint_as_float(r[jj + 7]) + b1.w, 0.f));
                 *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
             }
         }
@@ -94,11 +109,14 @@ struct MlpTc {
 
     // Full forward of the 128-row tile whose X has been written (and published
     // by the caller's synchronisation). out(row, logits[16]) is called by the
-    // threads of warps 0-3 (thread = row) for rows < n_rows. All threads call.
+    // threads of warps 0-3 (thread = row) for every row; the caller knows which
+    // rows hold observations. gbias: the policy's biases in global memory (used
+    // when kSmemBias is false). All threads call.
     template <class Out>
-    __device__ static void forward(uint8_t* smem, const float* __restrict__ bias, uint32_t tbase,
-                                   uint64_t* bar, uint32_t& parity, int n_rows, int* err, Out out) {
+    __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bar,
+                                   uint32_t& parity, int* err, Out out) {
         uint8_t* act = smem + kAct;
+        const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
         const uint32_t s_act = smem_u32(act);
         const uint32_t s_w1 = smem_u32(smem + kW1), s_w2 = smem_u32(smem + kW2);
         const uint32_t s_w3 = smem_u32(smem + kW3);
@@ -127,11 +145,9 @@ struct MlpTc {
             const int row = threadIdx.x;
             float v[16];
             tc::tmem_ld16(tc::tmem_addr(tbase, 32 * warp, 0), v);
-            if (row < n_rows) {
 #pragma unroll
-                for (int i = 0; i < 16; ++i) v[i] += __ldg(bias + 2 * H + i);
-                out(row, v);
-            }
+            for (int i = 0; i < 16; ++i) v[i] += kSmemBias ? bias[2 * H + i] : __ldg(bias + 2 * H + i);
+            out(row, v);
         }
         tc::fence_before_sync();
         __syncthreads();

@@ -688,8 +688,10 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
         if (((uintptr_t)p & 15u) != 0) return fail(c, MALIB_EINVAL, "trajectory buffers must be 16-byte aligned");
     }
     const int64_t epp = spec->n_envs / n_pairs;
-    if (c->pol_dtype != MALIB_F32 || c->dims[1] != c->dims[2] ||
-        !spread_f32_supported(spec->n_agents, spec->obs_dim, c->dims[1]) || epp > 128)
+    const bool use_tc = c->tc_layout && spread_tc_supported(spec->n_agents, spec->obs_dim,
+                                                            spec->n_actions, epp);
+    if (!use_tc && (c->pol_dtype != MALIB_F32 || c->dims[1] != c->dims[2] ||
+                    !spread_f32_supported(spec->n_agents, spec->obs_dim, c->dims[1]) || epp > 128))
         return fail(c, MALIB_EUNSUPPORTED,
                     "no spread kernel for %s N=%d obs %d hidden %d with %lld envs per combination",
                     c->pol_dtype == MALIB_BF16 ? "bf16" : "fp32", spec->n_agents, spec->obs_dim,
@@ -721,7 +723,11 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     a.logits = want_logits ? traj->logits : nullptr;
     cudaEvent_t e0, e1;
     time_begin(c, &e0, &e1);
-    CK(launch_spread_rollout_f32(a, c->dims[1], c->n_sm, c->stream), "spread rollout kernel");
+    if (use_tc) {
+        CK(launch_spread_rollout_tc(a, c->n_sm, c->stream), "spread tensor-core rollout kernel");
+    } else {
+        CK(launch_spread_rollout_f32(a, c->dims[1], c->n_sm, c->stream), "spread rollout kernel");
+    }
     time_end(c, e0, e1);
     c->launches += 1;
     return MALIB_OK;

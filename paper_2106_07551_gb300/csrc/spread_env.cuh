@@ -1,0 +1,96 @@
+// Cooperative particle spread (App. B.1) on the device, one environment per
+// thread with its state in registers; shared by the fp32 and tensor-core
+// rollout kernels. Every arithmetic step is an explicit correctly-rounded fp32
+// operation so that any two implementations of these steps agree bit for bit.
+#pragma once
+
+#include "device_common.cuh"
+
+namespace malib {
+
+template <int N>
+struct SpreadEnv {
+    float px[N], py[N], vx[N], vy[N], lx[N], ly[N];
+};
+
+template <int N>
+__device__ __forceinline__ void spread_reset(SpreadEnv<N>& s, uint64_t g, uint64_t seed) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const U4 d = draw(g, (uint32_t)i, kChance, seed);
+        s.px[i] = __fsub_rn(__fmul_rn(u24(d.x), 2.0f), 1.0f);
+        s.py[i] = __fsub_rn(__fmul_rn(u24(d.y), 2.0f), 1.0f);
+        s.vx[i] = 0.f;
+        s.vy[i] = 0.f;
+    }
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        const U4 d = draw(g, 0x80000000u + (uint32_t)l, kChance, seed);
+        s.lx[l] = __fsub_rn(__fmul_rn(u24(d.x), 2.0f), 1.0f);
+        s.ly[l] = __fsub_rn(__fmul_rn(u24(d.y), 2.0f), 1.0f);
+    }
+}
+
+// Observation of agent i: velocity, position, landmarks relative to the agent,
+// the other agents relative to it (ascending), zeros up to the row stride.
+template <int N, int XS>
+__device__ __forceinline__ void spread_obs(const SpreadEnv<N>& s, int i, float* o) {
+    int k = 0;
+    o[k++] = s.vx[i];
+    o[k++] = s.vy[i];
+    o[k++] = s.px[i];
+    o[k++] = s.py[i];
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        o[k++] = __fsub_rn(s.lx[l], s.px[i]);
+        o[k++] = __fsub_rn(s.ly[l], s.py[i]);
+    }
+#pragma unroll
+    for (int j = 0; j < N; ++j) {
+        if (j == i) continue;
+        o[k++] = __fsub_rn(s.px[j], s.px[i]);
+        o[k++] = __fsub_rn(s.py[j], s.py[i]);
+    }
+    for (; k < XS; ++k) o[k] = 0.f;
+}
+
+__device__ __forceinline__ float dist2(float ax, float ay, float bx, float by) {
+    const float dx = __fsub_rn(ax, bx), dy = __fsub_rn(ay, by);
+    return __fsqrt_rn(__fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy)));
+}
+
+// Mass 1, dt 0.1, damping 0.25, unit force along the chosen axis; reward after
+// the move; collision when centres are closer than 2 x 0.15.
+template <int N>
+__device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N], float (&r)[N]) {
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const float fx = act[i] == 1 ? 1.f : (act[i] == 2 ? -1.f : 0.f);
+        const float fy = act[i] == 3 ? 1.f : (act[i] == 4 ? -1.f : 0.f);
+        s.vx[i] = __fadd_rn(__fmul_rn(s.vx[i], 0.75f), __fmul_rn(fx, 0.1f));
+        s.vy[i] = __fadd_rn(__fmul_rn(s.vy[i], 0.75f), __fmul_rn(fy, 0.1f));
+        s.px[i] = __fadd_rn(s.px[i], __fmul_rn(s.vx[i], 0.1f));
+        s.py[i] = __fadd_rn(s.py[i], __fmul_rn(s.vy[i], 0.1f));
+    }
+    float cover = 0.f;
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        float best = dist2(s.px[0], s.py[0], s.lx[l], s.ly[l]);
+#pragma unroll
+        for (int j = 1; j < N; ++j) {
+            const float d = dist2(s.px[j], s.py[j], s.lx[l], s.ly[l]);
+            best = d < best ? d : best;
+        }
+        cover = __fadd_rn(cover, best);
+    }
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        int coll = 0;
+#pragma unroll
+        for (int j = 0; j < N; ++j)
+            if (j != i && dist2(s.px[i], s.py[i], s.px[j], s.py[j]) < 0.3f) ++coll;
+        r[i] = -__fadd_rn(cover, (float)coll);
+    }
+}
+
+}  // namespace malib

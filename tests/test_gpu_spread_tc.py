@@ -1,0 +1,73 @@
+"""GPU parity for the particle-spread rollout with N = 8 agents and bf16 MLP
+policies 34-256-256-5 on the tensor cores (8-CTA clusters, one agent's policy
+per CTA, actions exchanged through distributed shared memory).
+
+The oracle replays the same environments with the GPU's logits (bf16
+emulation for its own logits): observations (with zero padding), actions,
+rewards and done flags must match bit for bit, and the GPU logits must match
+the oracle's within 2e-2 relative. The full 65,536-env workload is checked on
+sampled env slices."""
+import numpy as np
+import pytest
+
+import workloads
+from gpu_util import context, load_population, logits_close, need_gpu, spec_of
+
+pytestmark = pytest.mark.gpu
+
+from paper_2106_07551_gb300 import MALIB_DUMP_LOGITS, alloc_traj
+
+RTOL = 2e-2
+
+
+def rollout(ctx, w, n_eps, seed):
+    spec = spec_of(w, MALIB_DUMP_LOGITS)
+    traj = alloc_traj(spec, n_eps, logits=True)
+    ctx.rollout(spec, w.pair_ids, n_eps, seed, traj)
+    ctx.sync()
+    return {k: v.cpu().numpy() for k, v in traj.items()}
+
+
+def check(orc, w, g, n_eps, seed, lo, hi):
+    params = [p.params for p in w.policies]
+    dims = w.policies[0].dims
+    sl = slice(lo, hi)
+    ref = orc.spread_rollout(params, dims, w.n_agents, w.n_landmarks, w.episode_len, w.n_envs,
+                             w.pair_ids, n_eps, seed, bf16=True, env_lo=lo, env_hi=hi,
+                             ext_logits=g["logits"][:, :, sl])
+    np.testing.assert_array_equal(g["obs"][:, :, sl, :, :w.obs_dim], ref["obs"])
+    assert np.all(g["obs"][..., w.obs_dim:] == 0)
+    np.testing.assert_array_equal(g["action"][:, :, sl].astype(np.int8), ref["action"])
+    np.testing.assert_array_equal(g["reward"][:, :, sl], ref["reward"])
+    done = g["done"][:, :, sl]
+    assert np.all(done[:, -1] == 1) and np.all(done[:, :-1] == 0)
+    n_bad, worst = logits_close(g["logits"][:, :, sl], ref["logits"], RTOL)
+    assert n_bad == 0, (n_bad, worst)
+
+
+@pytest.mark.parametrize("n_envs,epp,n_eps", [(512, 128, 2), (192, 64, 1), (40, 40, 3)])
+def test_full_replay_parity(orc, n_envs, epp, n_eps):
+    need_gpu()
+    w = workloads.spread(n_agents=8, n_envs=n_envs, pop=5, hidden=256, dtype=workloads.BF16,
+                         envs_per_pair=epp, with_bias=True, seed=700 + epp)
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, n_eps, 4321)
+    check(orc, w, g, n_eps, 4321, 0, n_envs)
+    g2 = rollout(ctx, w, n_eps, 4321)
+    for k in g:
+        np.testing.assert_array_equal(g2[k], g[k])
+    ctx.close()
+
+
+def test_full_workload_sampled_envs(orc):
+    """65,536 envs, 512 combinations of 128 envs, population 32, one episode."""
+    need_gpu()
+    w = workloads.config(4)
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 1, w.seed)
+    for lo, hi in ((0, 24), (30000, 30010), (65530, 65536)):
+        check(orc, w, g, 1, w.seed, lo, hi)
+    assert np.all(g["reward"] <= 0)
+    ctx.close()
