@@ -183,4 +183,162 @@ struct MlpF32 {
     }
 };
 
+
+// Packed fp32 pair helpers: fma.rn.f32x2 performs two independent IEEE fp32
+// fused multiply-adds (round to nearest), so results equal scalar fmaf.
+__device__ __forceinline__ unsigned long long f2_dup(float v) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(v));
+    return r;
+}
+__device__ __forceinline__ void f2_fma(unsigned long long& d, unsigned long long a,
+                                       unsigned long long b) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(d) : "l"(a), "l"(b));
+}
+__device__ __forceinline__ float2 f2_split(unsigned long long v) {
+    float lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+    return make_float2(lo, hi);
+}
+
+// 128-row pass of one policy with 8x8 register tiles (256 threads, H = 128):
+// thread (tx, ty) computes rows ty + 16 i (i = 0..7) and columns
+// {4tx..4tx+3} and {64+4tx..64+4tx+3}, accumulating adjacent column pairs
+// with packed fp32 FMAs (2 FMAs per instruction). Per k it issues 4 16-byte
+// shared loads (2 for its 8 inputs, amortised over 4 k, and 2 for its 8
+// weights, which arrive as 4 column pairs), 8 duplications of an input into a
+// pair, and 32 packed FMAs for 64 FMAs. Rows interleaved by 16 put the two row
+// groups of a half-warp on adjacent rows, which the bank-skewed strides place
+// in different banks. The weights arrive as separate pointers so that W2 can
+// live in a buffer of its own (restaged per policy) while the small layers of
+// several policies stay resident. Layer 3 is folded into layer 2's epilogue
+// (shuffle reduction over the 16 column lanes of a row group, which share one
+// warp).
+template <int IN, int A>
+struct MlpF32T8 {
+    static constexpr int H = 128;
+    static constexpr int kThreads = 256;
+    static constexpr int kRows = 128;
+    static constexpr int XS = (IN + 3) / 4 * 4;
+    static constexpr int HS = H + 4;
+    static constexpr int LS = (A + 3) / 4 * 4;
+    using u64 = unsigned long long;
+
+    __device__ static int col_group() {
+        const int lane = threadIdx.x & 31;
+        return (lane & 7) | ((lane >> 4) << 3);
+    }
+    __device__ static int row_group() { return (threadIdx.x >> 5) * 2 + ((threadIdx.x >> 3) & 1); }
+
+    // acc[i][p]: row i, column pair p (p 0,1: c0..c0+3; p 2,3: c1..c1+3)
+    __device__ static void init(u64 (&acc)[8][4], const float* __restrict__ b, int c0, int c1) {
+        const ulonglong2 bA = *reinterpret_cast<const ulonglong2*>(b + c0);
+        const ulonglong2 bB = *reinterpret_cast<const ulonglong2*>(b + c1);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) { acc[i][0] = bA.x; acc[i][1] = bA.y; acc[i][2] = bB.x; acc[i][3] = bB.y; }
+    }
+
+    // acc += rows' inputs [4 k from xa] x W rows k0..k0+3 (kk < kmax)
+    __device__ static void block(u64 (&acc)[8][4], const float4 (&xa)[8], const float* __restrict__ W,
+                                 int k0, int kmax, int c0, int c1) {
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+            if (kk < kmax) {
+                const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(W + (k0 + kk) * H + c0);
+                const ulonglong2 wB = *reinterpret_cast<const ulonglong2*>(W + (k0 + kk) * H + c1);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float xv = kk == 0 ? xa[i].x : kk == 1 ? xa[i].y : kk == 2 ? xa[i].z : xa[i].w;
+                    const u64 x2 = f2_dup(xv);
+                    f2_fma(acc[i][0], x2, wA.x);
+                    f2_fma(acc[i][1], x2, wA.y);
+                    f2_fma(acc[i][2], x2, wB.x);
+                    f2_fma(acc[i][3], x2, wB.y);
+                }
+            }
+        }
+    }
+
+    // Layer 1 into H1 (rows of X [128][XS]). Ends with __syncthreads.
+    __device__ static void layer1(const float* __restrict__ X, float* __restrict__ H1,
+                                  const float* __restrict__ W1T, const float* __restrict__ b1) {
+        const int tx = col_group(), ty = row_group();
+        const int c0 = tx * 4, c1 = H / 2 + tx * 4;
+        u64 acc[8][4];
+        init(acc, b1, c0, c1);
+#pragma unroll
+        for (int k0 = 0; k0 < IN; k0 += 4) {
+            float4 xa[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                xa[i] = *reinterpret_cast<const float4*>(X + (ty + 16 * i) * XS + k0);
+            block(acc, xa, W1T, k0, IN - k0, c0, c1);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            float* hr = H1 + (ty + 16 * i) * HS;
+            const float2 p0 = f2_split(acc[i][0]), p1 = f2_split(acc[i][1]);
+            const float2 p2 = f2_split(acc[i][2]), p3 = f2_split(acc[i][3]);
+            *reinterpret_cast<float4*>(hr + c0) = make_float4(fmaxf(p0.x, 0.f), fmaxf(p0.y, 0.f),
+                                                              fmaxf(p1.x, 0.f), fmaxf(p1.y, 0.f));
+            *reinterpret_cast<float4*>(hr + c1) = make_float4(fmaxf(p2.x, 0.f), fmaxf(p2.y, 0.f),
+                                                              fmaxf(p3.x, 0.f), fmaxf(p3.y, 0.f));
+        }
+        __syncthreads();
+    }
+
+    // Layers 2 and 3: H1 -> logits rows of LG [128][LS]. Ends with __syncthreads.
+    __device__ static void layer23(const float* __restrict__ H1, float* __restrict__ LG,
+                                   const float* __restrict__ W2T, const float* __restrict__ b2,
+                                   const float* __restrict__ W3, const float* __restrict__ b3) {
+        const int tx = col_group(), ty = row_group();
+        const int c0 = tx * 4, c1 = H / 2 + tx * 4;
+        u64 acc[8][4];
+        init(acc, b2, c0, c1);
+#pragma unroll 2
+        for (int k0 = 0; k0 < H; k0 += 4) {
+            float4 ha[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                ha[i] = *reinterpret_cast<const float4*>(H1 + (ty + 16 * i) * HS + k0);
+            block(acc, ha, W2T, k0, 4, c0, c1);
+        }
+        float pl[8][A];
+#pragma unroll
+        for (int a = 0; a < A; ++a) {
+            const float4 vA = *reinterpret_cast<const float4*>(W3 + a * H + c0);
+            const float4 vB = *reinterpret_cast<const float4*>(W3 + a * H + c1);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float2 p0 = f2_split(acc[i][0]), p1 = f2_split(acc[i][1]);
+                const float2 p2 = f2_split(acc[i][2]), p3 = f2_split(acc[i][3]);
+                float t = fmaxf(p0.x, 0.f) * vA.x;
+                t = fmaf(fmaxf(p0.y, 0.f), vA.y, t);
+                t = fmaf(fmaxf(p1.x, 0.f), vA.z, t);
+                t = fmaf(fmaxf(p1.y, 0.f), vA.w, t);
+                t = fmaf(fmaxf(p2.x, 0.f), vB.x, t);
+                t = fmaf(fmaxf(p2.y, 0.f), vB.y, t);
+                t = fmaf(fmaxf(p3.x, 0.f), vB.z, t);
+                t = fmaf(fmaxf(p3.y, 0.f), vB.w, t);
+                pl[i][a] = t;
+            }
+        }
+#pragma unroll
+        for (int o = 1; o <= 16; o <<= 1) {
+            if (o == 8) continue;
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int a = 0; a < A; ++a) pl[i][a] += __shfl_xor_sync(0xffffffffu, pl[i][a], o);
+        }
+        if (tx == 0) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int a = 0; a < A; ++a) LG[(ty + 16 * i) * LS + a] = pl[i][a] + b3[a];
+        }
+        __syncthreads();
+    }
+};
+
 }  // namespace malib

@@ -288,6 +288,197 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_kernel(EvalArgs a) {
     }
 }
 
+
+// Seat-phased Leduc evaluation for H = 128 (8x8 register tiles). Each step runs
+// two 128-row passes, one per acting seat. Only one seat's W2 (64 KB) is
+// resident; the small layers (W1, biases, W3) of both seats stay resident. The
+// seat order alternates each step, so W2 is restaged once per step by bulk copy,
+// overlapped with the second seat's layer 1. A seat with more than 128 acting
+// hands defers the rest to the next step (their results do not depend on it).
+namespace t8 {
+using E = MlpF32T8<17, 3>;
+using L = F32Layout<17, 128, 3>;
+constexpr int kSlots = 248;
+constexpr int kSmall = L::kW2T + (L::kSize - L::kB2);        // W1T|b1 then b2|W3|b3
+constexpr int kOffSmall = 0;
+constexpr int kOffW2 = kOffSmall + 2 * kSmall;
+constexpr int kOffX = kOffW2 + 128 * 128;
+constexpr int kOffH1 = kOffX + 2 * E::kRows * E::XS;
+constexpr int kOffLG = kOffH1 + E::kRows * E::HS;
+constexpr int kFloats = kOffLG + 2 * E::kRows * E::LS;
+constexpr size_t kBytes = (size_t)kFloats * 4;
+static_assert(kSmall % 4 == 0 && kOffW2 % 4 == 0 && kOffX % 4 == 0 && kOffH1 % 4 == 0, "16-B");
+}  // namespace t8
+
+__global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
+    using namespace t8;
+    extern __shared__ __align__(128) float smem[];
+    float* X = smem + kOffX;
+    float* H1 = smem + kOffH1;
+    float* LG = smem + kOffLG;
+    float* W2s = smem + kOffW2;
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int cnt[2][8];
+    __shared__ unsigned long long next_e;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < 2 * E::kRows * E::XS; i += blockDim.x) X[i] = 0.f;
+    if (tid == 0) mbar_init(&bar, 1);
+    __syncthreads();
+    uint32_t parity = 0;
+
+    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+    const int64_t per = (total + gridDim.x - 1) / gridDim.x;
+    const int64_t lo = (int64_t)blockIdx.x * per;
+    const int64_t hi = min(total, lo + per);
+
+    for (int64_t seg = lo; seg < hi;) {
+        const int pair = (int)(seg / a.n_episodes);
+        const int64_t e_lo = seg - (int64_t)pair * a.n_episodes;
+        const int64_t e_hi = min(a.n_episodes, e_lo + (hi - seg));
+        seg += e_hi - e_lo;
+        const int pid[2] = {a.pairs[2 * pair], a.pairs[2 * pair + 1]};
+        if (!pair_ok(a, pid[0], pid[1])) {
+            if (tid == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+            continue;
+        }
+        const float* pol0 = a.arena + a.pol_offset[pid[0]];
+        const float* pol1 = a.arena + a.pol_offset[pid[1]];
+        int res = 0;                                    // seat whose W2 is resident
+        if (tid == 0) {
+            fence_proxy_async_smem();
+            mbar_arrive_expect_tx(&bar, 2u * kSmall * 4u + 128u * 128u * 4u);
+            for (int s = 0; s < 2; ++s) {
+                const float* src = s == 0 ? pol0 : pol1;
+                float* dst = smem + kOffSmall + s * kSmall;
+                bulk_g2s(dst, src, L::kW2T * 4u, &bar);
+                bulk_g2s(dst + L::kW2T, src + L::kB2, (L::kSize - L::kB2) * 4u, &bar);
+            }
+            bulk_g2s(W2s, pol0 + L::kW2T, 32768u, &bar);
+            bulk_g2s(W2s + 8192, pol0 + L::kW2T + 8192, 32768u, &bar);
+        }
+        if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs) && tid == 0) atomicOr(a.err, ERRBIT_TIMEOUT);
+        parity ^= 1u;
+
+        LeducHand h;
+        bool live = false;
+        int64_t e = e_lo + tid;
+        uint64_t g = 0;
+        int t = 0;
+        long long s1 = 0, s2 = 0, nd = 0;
+        if (tid < kSlots && e < e_hi) {
+            live = true;
+            g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+            leduc_deal(h, g, a.seed);
+        }
+        if (tid == 0) next_e = (unsigned long long)(e_lo + kSlots);
+
+        while (true) {
+            const int seat = live ? h.actor : -1;
+            const unsigned b0 = __ballot_sync(0xffffffffu, seat == 0);
+            const unsigned b1 = __ballot_sync(0xffffffffu, seat == 1);
+            if (lane == 0) { cnt[0][warp] = __popc(b0); cnt[1][warp] = __popc(b1); }
+            __syncthreads();
+            int c[2] = {0, 0}, pre = 0;
+#pragma unroll
+            for (int w = 0; w < 8; ++w) {
+                c[0] += cnt[0][w];
+                c[1] += cnt[1][w];
+                if (w < warp) pre += seat == 1 ? cnt[1][w] : cnt[0][w];
+            }
+            if (c[0] + c[1] == 0) break;
+            const unsigned mine = seat == 1 ? b1 : b0;
+            const int rank = pre + __popc(mine & ((1u << lane) - 1u));
+            const bool placed = live && rank < E::kRows;
+            float ob[17];
+            if (placed) {
+                leduc_obs(h, ob);
+                float* xr = X + (seat * E::kRows + rank) * E::XS;
+#pragma unroll
+                for (int i = 0; i < 17; ++i) xr[i] = ob[i];
+            }
+            __syncthreads();
+            const int first = res, second = 1 - res;
+            const float* sf = smem + kOffSmall + first * kSmall;
+            const float* ss = smem + kOffSmall + second * kSmall;
+            const int off_b2 = L::kW2T, off_w3 = L::kW2T + (L::kW3 - L::kB2),
+                      off_b3 = L::kW2T + (L::kB3 - L::kB2);
+            if (c[first] > 0) {
+                E::layer1(X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
+                E::layer23(H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3, sf + off_b3);
+            }
+            if (c[second] > 0) {
+                const float* src = (second == 0 ? pol0 : pol1) + L::kW2T;
+                if (tid == 0) {                       // every read of W2s has passed a barrier
+                    fence_proxy_async_smem();
+                    mbar_arrive_expect_tx(&bar, 128u * 128u * 4u);
+                    bulk_g2s(W2s, src, 32768u, &bar);
+                    bulk_g2s(W2s + 8192, src + 8192, 32768u, &bar);
+                }
+                E::layer1(X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
+                if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs) && tid == 0)
+                    atomicOr(a.err, ERRBIT_TIMEOUT);
+                parity ^= 1u;
+                E::layer23(H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3, ss + off_b3);
+                res = second;
+            }
+            if (placed) {
+                const float* lp = LG + (seat * E::kRows + rank) * E::LS;
+                float lg[3] = {lp[0], lp[1], lp[2]};
+                const unsigned legal = leduc_legal(h);
+                const float u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);
+                const int act = sample_masked<3>(lg, legal, u);
+                const bool rec = e < a.n_dump;
+                const int64_t rb = ((int64_t)pair * a.n_dump + e) * kLeducMaxDec;
+                if (rec) {
+                    if (a.d_obs) {
+                        float* o = a.d_obs + (rb + t) * 20;
+#pragma unroll
+                        for (int i = 0; i < 17; ++i) o[i] = ob[i];
+                        o[17] = 0.f; o[18] = 0.f; o[19] = 0.f;
+                    }
+                    if (a.d_logits) {
+                        float* l = a.d_logits + (rb + t) * 3;
+                        l[0] = lg[0]; l[1] = lg[1]; l[2] = lg[2];
+                    }
+                    if (a.d_action) a.d_action[rb + t] = (uint8_t)act;
+                }
+                leduc_apply(h, act);
+                if (rec) {
+                    if (a.d_reward) a.d_reward[rb + t] = h.done ? (float)h.payoff : 0.f;
+                    if (a.d_done) a.d_done[rb + t] = h.done ? 1 : 0;
+                }
+                ++t;
+                ++nd;
+                if (h.done) {
+                    s1 += h.payoff;
+                    s2 += (long long)h.payoff * h.payoff;
+                    if (rec) {
+                        for (int k = t; k < kLeducMaxDec; ++k) {
+                            if (a.d_obs)
+                                for (int i = 0; i < 20; ++i) a.d_obs[(rb + k) * 20 + i] = 0.f;
+                            if (a.d_logits)
+                                for (int i = 0; i < 3; ++i) a.d_logits[(rb + k) * 3 + i] = 0.f;
+                            if (a.d_action) a.d_action[rb + k] = 255;
+                            if (a.d_reward) a.d_reward[rb + k] = 0.f;
+                            if (a.d_done) a.d_done[rb + k] = 1;
+                        }
+                    }
+                    e = (int64_t)atomicAdd(&next_e, 1ull);
+                    live = e < e_hi;
+                    if (live) {
+                        g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
+                        leduc_deal(h, g, a.seed);
+                        t = 0;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+        block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+    }
+}
+
 }  // namespace
 
 bool leduc_f32_supported(int hidden) { return hidden == 128 || hidden == 64; }
@@ -325,7 +516,18 @@ static cudaError_t launch_leduc_h(const EvalArgs& a, int n_sm, cudaStream_t s) {
 
 cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0) return cudaSuccess;
-    if (hidden == 128) return launch_leduc_h<128>(a, n_sm, s);
+    if (hidden == 128) {
+        cudaError_t err = cudaFuncSetAttribute(leduc_eval_f32_t8_kernel,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)t8::kBytes);
+        if (err != cudaSuccess) return err;
+        const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+        int64_t grid = (total + t8::kSlots - 1) / t8::kSlots;
+        if (grid > n_sm) grid = n_sm;
+        if (grid < 1) grid = 1;
+        leduc_eval_f32_t8_kernel<<<(unsigned)grid, 256, t8::kBytes, s>>>(a);
+        return cudaGetLastError();
+    }
     if (hidden == 64) return launch_leduc_h<64>(a, n_sm, s);
     return cudaErrorInvalidValue;
 }
