@@ -66,7 +66,6 @@ __device__ __forceinline__ bool sync(uint32_t* flags, uint32_t epoch, uint32_t s
                                      int* err, uint32_t* ok_slot) {
     __syncthreads();
     if (threadIdx.x < size) {
-        fence_cluster();
         const uint32_t a = map(&flags[me], threadIdx.x);
         asm volatile("st.release.cluster.shared::cluster.u32 [%0], %1;" ::"r"(a), "r"(epoch)
                      : "memory");
@@ -75,14 +74,14 @@ __device__ __forceinline__ bool sync(uint32_t* flags, uint32_t epoch, uint32_t s
         bool ok = true;
         const uint64_t t0 = globaltimer_ns();
         for (uint32_t r = 0; r < size && ok; ++r) {
-            while (true) {
+            for (uint32_t spin = 0;; ++spin) {
                 uint32_t v;
                 asm volatile("ld.acquire.cluster.shared::cta.u32 %0, [%1];"
                              : "=r"(v)
                              : "r"(smem_u32(&flags[r]))
                              : "memory");
                 if ((int32_t)(v - epoch) >= 0) break;
-                if (globaltimer_ns() - t0 > kWaitLimitNs) { ok = false; break; }
+                if ((spin & 63u) == 63u && globaltimer_ns() - t0 > kWaitLimitNs) { ok = false; break; }
             }
         }
         if (!ok) atomicOr(err, ERRBIT_TIMEOUT);

@@ -135,7 +135,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const bool placed = live && rank < kPart;
             const int row = (int)me * kPart + rank;
             float ob[17];
+            float u = 0.f;
             if (placed) {
+                u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);   // ready before the logits
                 const uint32_t target = (uint32_t)seat;
                 leduc_obs(h, ob);
                 uint32_t w[16];
@@ -165,13 +167,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     cl::st_f32(dst + 4, lg[1]);
                     cl::st_f32(dst + 8, lg[2]);
                 }
-            });
+            }, /*x_published=*/true);
             cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
             if (placed) {
                 const float* lp = lgbuf + (seat * 128 + row) * 4;
                 float lg[3] = {lp[0], lp[1], lp[2]};
                 const unsigned legal = leduc_legal(h);
-                const float u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);
                 const int act = sample_masked<3>(lg, legal, u);
                 const bool rec = e < a.n_dump;
                 const int64_t rb = ((int64_t)pair * a.n_dump + e) * kMaxDec;

@@ -21,6 +21,23 @@
 
 namespace malib {
 
+// Packed fp32 pair helpers: fma.rn.f32x2 performs two independent IEEE fp32
+// fused multiply-adds (round to nearest), so results equal scalar fmaf.
+__device__ __forceinline__ unsigned long long f2_dup(float v) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(v));
+    return r;
+}
+__device__ __forceinline__ void f2_fma(unsigned long long& d, unsigned long long a,
+                                       unsigned long long b) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(d) : "l"(a), "l"(b));
+}
+__device__ __forceinline__ float2 f2_split(unsigned long long v) {
+    float lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+    return make_float2(lo, hi);
+}
+
 template <int IN, int H, int A>
 struct MlpF32 {
     using L = F32Layout<IN, H, A>;
@@ -118,8 +135,17 @@ struct MlpF32 {
                 acc[i][0] = bA.x; acc[i][1] = bA.y; acc[i][2] = bA.z; acc[i][3] = bA.w;
                 acc[i][4] = bB.x; acc[i][5] = bB.y; acc[i][6] = bB.z; acc[i][7] = bB.w;
             }
+            // packed pairs: p[i][0..3] = column pairs (c0,c0+1) (c0+2,c0+3) (c1,..) (c1+2,..)
+            unsigned long long p[4][4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                asm("mov.b64 %0, {%1, %2};" : "=l"(p[i][0]) : "f"(acc[i][0]), "f"(acc[i][1]));
+                asm("mov.b64 %0, {%1, %2};" : "=l"(p[i][1]) : "f"(acc[i][2]), "f"(acc[i][3]));
+                asm("mov.b64 %0, {%1, %2};" : "=l"(p[i][2]) : "f"(acc[i][4]), "f"(acc[i][5]));
+                asm("mov.b64 %0, {%1, %2};" : "=l"(p[i][3]) : "f"(acc[i][6]), "f"(acc[i][7]));
+            }
             const float* hr = H1 + lr * HS;
-#pragma unroll 2
+#pragma unroll 4
             for (int k0 = 0; k0 < H; k0 += 4) {
                 float4 ha[4];
 #pragma unroll
@@ -127,21 +153,25 @@ struct MlpF32 {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const float* wk = w + L::kW2T + (k0 + kk) * H;
-                    const float4 wA = *reinterpret_cast<const float4*>(wk + c0);
-                    const float4 wB = *reinterpret_cast<const float4*>(wk + c1);
+                    const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(wk + c0);
+                    const ulonglong2 wB = *reinterpret_cast<const ulonglong2*>(wk + c1);
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         const float hv = kk == 0 ? ha[i].x : kk == 1 ? ha[i].y : kk == 2 ? ha[i].z : ha[i].w;
-                        acc[i][0] = fmaf(hv, wA.x, acc[i][0]);
-                        acc[i][1] = fmaf(hv, wA.y, acc[i][1]);
-                        acc[i][2] = fmaf(hv, wA.z, acc[i][2]);
-                        acc[i][3] = fmaf(hv, wA.w, acc[i][3]);
-                        acc[i][4] = fmaf(hv, wB.x, acc[i][4]);
-                        acc[i][5] = fmaf(hv, wB.y, acc[i][5]);
-                        acc[i][6] = fmaf(hv, wB.z, acc[i][6]);
-                        acc[i][7] = fmaf(hv, wB.w, acc[i][7]);
+                        const unsigned long long h2 = f2_dup(hv);
+                        f2_fma(p[i][0], h2, wA.x);
+                        f2_fma(p[i][1], h2, wA.y);
+                        f2_fma(p[i][2], h2, wB.x);
+                        f2_fma(p[i][3], h2, wB.y);
                     }
                 }
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 q0 = f2_split(p[i][0]), q1 = f2_split(p[i][1]);
+                const float2 q2 = f2_split(p[i][2]), q3 = f2_split(p[i][3]);
+                acc[i][0] = q0.x; acc[i][1] = q0.y; acc[i][2] = q1.x; acc[i][3] = q1.y;
+                acc[i][4] = q2.x; acc[i][5] = q2.y; acc[i][6] = q3.x; acc[i][7] = q3.y;
             }
             // layer 3 partials over this thread's 8 columns
             float pl[4][A];
@@ -183,23 +213,6 @@ struct MlpF32 {
     }
 };
 
-
-// Packed fp32 pair helpers: fma.rn.f32x2 performs two independent IEEE fp32
-// fused multiply-adds (round to nearest), so results equal scalar fmaf.
-__device__ __forceinline__ unsigned long long f2_dup(float v) {
-    unsigned long long r;
-    asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(v));
-    return r;
-}
-__device__ __forceinline__ void f2_fma(unsigned long long& d, unsigned long long a,
-                                       unsigned long long b) {
-    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(d) : "l"(a), "l"(b));
-}
-__device__ __forceinline__ float2 f2_split(unsigned long long v) {
-    float lo, hi;
-    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-    return make_float2(lo, hi);
-}
 
 // 128-row pass of one policy with 8x8 register tiles (256 threads, H = 128):
 // thread (tx, ty) computes rows ty + 16 i (i = 0..7) and columns

@@ -64,37 +64,39 @@ struct MlpTc {
     }
 
     // D + bias -> relu -> bf16 into the activation tile (this thread: one row,
-    // one half of the H columns; 64 columns per tensor-memory wait).
+    // one half of the H columns, in 32-column chunks; the next chunk's tensor
+    // memory load is in flight while the current chunk is processed).
     __device__ static void epilogue_hidden(uint8_t* act, const float* bias, uint32_t tbase) {
         const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
         const int q = warp & 3, half = warp >> 2;
         const int row = 32 * q + lane;
-#pragma unroll 1
-        for (int cc = 0; cc < H / 2 / 64; ++cc) {
-            const int c0 = half * (H / 2) + cc * 64;
-            uint32_t r0[32], r1[32];
-            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0), r0);
-            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0 + 32), r1);
-            tc::tmem_wait_ld();
+        constexpr int kChunks = H / 2 / 32;
+        uint32_t r[2][32];
+        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, half * (H / 2)), r[0]);
+        tc::tmem_wait_ld();
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const uint32_t* r = j < 4 ? r0 : r1;
-                const int jj = (j & 3) * 8;
+        for (int cc = 0; cc < kChunks; ++cc) {
+            const int c0 = half * (H / 2) + cc * 32;
+            if (cc + 1 < kChunks) tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0 + 32), r[(cc + 1) & 1]);
+            const uint32_t* v = r[cc & 1];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
                 const float4 b0 = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 8 * j)
                                             : __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j));
                 const float4 b1 = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4)
                                             : __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4));
                 uint4 pk;
-                pk.x = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 0]) + b0.x, 0.f),
-                                     fmaxf(__uint_as_float(r[jj + 1]) + b0.y, 0.f));
-                pk.y = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 2]) + b0.z, 0.f),
-                                     fmaxf(__uint_as_float(r[jj + 3]) + b0.w, 0.f));
-                pk.z = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 4]) + b1.x, 0.f),
-                                     fmaxf(__uint_as_float(r[jj + 5]) + b1.y, 0.f));
-                pk.w = tc::pack_bf16(fmaxf(__uint_as_float(r[jj + 6]) + b1.z, 0.f),
-                                     fmaxf(__uint_as_float(r[jj + 7]) + b1.w, 0.f));
+                pk.x = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 0]) + b0.x, 0.f),
+                                     fmaxf(__uint_as_float(v[8 * j + 1]) + b0.y, 0.f));
+                pk.y = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 2]) + b0.z, 0.f),
+                                     fmaxf(__uint_as_float(v[8 * j + 3]) + b0.w, 0.f));
+                pk.z = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 4]) + b1.x, 0.f),
+                                     fmaxf(__uint_as_float(v[8 * j + 5]) + b1.y, 0.f));
+                pk.w = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 6]) + b1.z, 0.f),
+                                     fmaxf(__uint_as_float(v[8 * j + 7]) + b1.w, 0.f));
                 *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
             }
+            if (cc + 1 < kChunks) tc::tmem_wait_ld();
         }
     }
 
@@ -112,15 +114,22 @@ struct MlpTc {
     // threads of warps 0-3 (thread = row) for every row; the caller knows which
     // rows hold observations. gbias: the policy's biases in global memory (used
     // when kSmemBias is false). All threads call.
+    // x_published: the caller's X writers already fenced (proxy) and the CTA
+    // has synchronised since (e.g. a cluster sync), so MMA 1 issues at once.
     template <class Out>
     __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bar,
-                                   uint32_t& parity, int* err, Out out) {
+                                   uint32_t& parity, int* err, Out out, bool x_published = false) {
         uint8_t* act = smem + kAct;
         const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
         const uint32_t s_act = smem_u32(act);
         const uint32_t s_w1 = smem_u32(smem + kW1), s_w2 = smem_u32(smem + kW2);
         const uint32_t s_w3 = smem_u32(smem + kW3);
-        handoff();
+        if (x_published) {
+            if (threadIdx.x == 0) fence_proxy_async_smem();
+            tc::fence_after_sync();
+        } else {
+            handoff();
+        }
         if (threadIdx.x == 0) {
             issue(tbase, s_act, s_w1, kLboW, K1, tc::instr_desc(128, H, 1));
             tc::mma_commit(bar);
@@ -136,7 +145,14 @@ struct MlpTc {
         epilogue_hidden(act, bias + H, tbase);
         handoff();
         if (threadIdx.x == 0) {
-            issue(tbase, s_act, s_w3, kLboW3, H, tc::instr_desc(128, NOUT, 1));
+            // four independent accumulators (TMEM columns 16j..16j+15) over K
+            // quarters, so the 16 small MMAs form 4 short chains
+            const uint32_t idesc3 = tc::instr_desc(128, NOUT, 1);
+            for (int s = 0; s < H / 16; ++s)
+                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (H / 64))),
+                             tc::smem_desc(s_act + 2u * s * kLboAct, kLboAct, 128),
+                             tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
+                             (s % (H / 64)) != 0);
             tc::mma_commit(bar);
         }
         wait_mma(bar, parity, err);
@@ -144,7 +160,16 @@ struct MlpTc {
         if (warp < 4) {
             const int row = threadIdx.x;
             float v[16];
-            tc::tmem_ld16(tc::tmem_addr(tbase, 32 * warp, 0), v);
+            {
+                uint32_t r[32], r2[32];
+                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * warp, 0), r);
+                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * warp, 32), r2);
+                tc::tmem_wait_ld();
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    v[i] = (__uint_as_float(r[i]) + __uint_as_float(r[16 + i])) +
+                           (__uint_as_float(r2[i]) + __uint_as_float(r2[16 + i]));
+            }
 #pragma unroll
             for (int i = 0; i < 16; ++i) v[i] += kSmemBias ? bias[2 * H + i] : __ldg(bias + 2 * H + i);
             out(row, v);

@@ -54,6 +54,35 @@ __device__ __forceinline__ void spread_obs(const SpreadEnv<N>& s, int i, float* 
     for (; k < XS; ++k) o[k] = 0.f;
 }
 
+// spread_obs for a run-time agent index: the same values and operations, with
+// every register array indexed at compile time (selects instead of indexing).
+template <int N, int XS>
+__device__ __forceinline__ void spread_obs_dyn(const SpreadEnv<N>& s, int i, float* o) {
+    float px = 0.f, py = 0.f, vx = 0.f, vy = 0.f;
+#pragma unroll
+    for (int j = 0; j < N; ++j)
+        if (j == i) { px = s.px[j]; py = s.py[j]; vx = s.vx[j]; vy = s.vy[j]; }
+    int k = 0;
+    o[k++] = vx;
+    o[k++] = vy;
+    o[k++] = px;
+    o[k++] = py;
+#pragma unroll
+    for (int l = 0; l < N; ++l) {
+        o[k++] = __fsub_rn(s.lx[l], px);
+        o[k++] = __fsub_rn(s.ly[l], py);
+    }
+#pragma unroll
+    for (int m = 0; m < N - 1; ++m) {
+        const float qx = m < i ? s.px[m] : s.px[m + 1];
+        const float qy = m < i ? s.py[m] : s.py[m + 1];
+        o[k++] = __fsub_rn(qx, px);
+        o[k++] = __fsub_rn(qy, py);
+    }
+#pragma unroll
+    for (; k < XS; ++k) o[k] = 0.f;
+}
+
 __device__ __forceinline__ float dist2(float ax, float ay, float bx, float by) {
     const float dx = __fsub_rn(ax, bx), dy = __fsub_rn(ay, by);
     return __fsqrt_rn(__fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy)));

@@ -111,9 +111,11 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         for (int t = 0; t < T; ++t) {
             const uint32_t par = step & 1u;
             const int64_t ix = ((ep * T + t) * a.n_envs + env) * kN;
+            float u = 0.f;
             if (mine) {
+                u = u24(draw(g, (uint32_t)t, me, a.seed).x);      // ready before the logits
                 float o[kObsPad];
-                spread_obs<kN, kObsPad>(s, (int)me, o);
+                spread_obs_dyn<kN, kObsPad>(s, (int)me, o);
                 float4* dst = reinterpret_cast<float4*>(a.obs + (ix + me) * kObsPad);
 #pragma unroll
                 for (int q = 0; q < kObsPad / 4; ++q)
@@ -132,7 +134,6 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     float l5[kA];
 #pragma unroll
                     for (int k = 0; k < kA; ++k) l5[k] = lg[k];
-                    const float u = u24(draw(g, (uint32_t)t, me, a.seed).x);
                     const int act = sample_masked<kA>(l5, 0x1Fu, u);
                     if (a.logits)
 #pragma unroll
@@ -153,7 +154,11 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                 for (int i = 0; i < kN; ++i) act[i] = acts[(par * kN + i) * 128 + tid];
                 float r[kN];
                 spread_step<kN>(s, act, r);
-                a.reward[ix + me] = r[me];
+                float rm = 0.f;
+#pragma unroll
+                for (int i = 0; i < kN; ++i)
+                    if (i == (int)me) rm = r[i];
+                a.reward[ix + me] = rm;
                 if (me == 0) a.done[(ep * T + t) * a.n_envs + env] = (t == T - 1) ? 1 : 0;
             }
             ++step;
