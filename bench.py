@@ -29,8 +29,10 @@ UNIT = "env-steps/s"
 SM_COUNT_GB300 = 152
 FP32_LANES_PER_SM = 128
 # dram bytes (read + write) of one launch of the dominant kernel from the ncu
-# capture summarised under profiles/ (None until taken for the current kernel)
-NCU_TRAFFIC_PER_LAUNCH = {}
+# capture summarised under profiles/ (None until taken for the current kernel).
+# leduc_eval_f32_t8_kernel: profiles/leduc_eval_f32_t8_kernel_c2.md (the one-time
+# read of the population; independent of the hand count).
+NCU_TRAFFIC_PER_LAUNCH = {"leduc_eval_f32_kernel<128>": 1316096}
 
 
 def mlp_flop(dims):
