@@ -32,7 +32,7 @@ FP32_LANES_PER_SM = 128
 # capture summarised under profiles/ (None until taken for the current kernel).
 # leduc_eval_f32_t8_kernel: profiles/leduc_eval_f32_t8_kernel_c2.md (the one-time
 # read of the population; independent of the hand count).
-NCU_TRAFFIC_PER_LAUNCH = {"leduc_eval_f32_kernel<128>": 1316096}
+NCU_TRAFFIC_PER_LAUNCH = {"leduc_eval_f32_t8_kernel": 1316096}
 
 
 def mlp_flop(dims):
@@ -348,7 +348,7 @@ def run_ours(args):
     peak_tflops = SM_COUNT_GB300 * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
     achieved = (decisions * flop_per_unit / args.steps) / (kern_ms / kern_n / 1e3) / 1e12 \
         if kern_n else 0.0
-    kname = {"leduc": "leduc_eval_f32_kernel<128>", "kuhn": "kuhn_eval_kernel",
+    kname = {"leduc": "leduc_eval_f32_t8_kernel", "kuhn": "kuhn_eval_kernel",
              "spread3": "spread_rollout_f32_kernel<3,18,64>",
              "leduc_bf16": "leduc_eval_tc_kernel",
              "spread8": "spread_rollout_tc_kernel"}[args.workload]
