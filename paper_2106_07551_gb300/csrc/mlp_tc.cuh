@@ -65,26 +65,36 @@ struct MlpTc {
 
     // D + bias -> relu -> bf16 into the activation tile (this thread: one row,
     // one half of the H columns, in 32-column chunks; the next chunk's tensor
-    // memory load is in flight while the current chunk is processed).
+    // memory load and bias loads are in flight while the current chunk is
+    // processed).
     __device__ static void epilogue_hidden(uint8_t* act, const float* bias, uint32_t tbase) {
         const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
         const int q = warp & 3, half = warp >> 2;
         const int row = 32 * q + lane;
         constexpr int kChunks = H / 2 / 32;
         uint32_t r[2][32];
+        float4 bs[2][8];
+        auto load_bias = [&](int buf, int c0) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                bs[buf][j] = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
+                                       : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
+        };
         tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, half * (H / 2)), r[0]);
+        load_bias(0, half * (H / 2));
         tc::tmem_wait_ld();
 #pragma unroll
         for (int cc = 0; cc < kChunks; ++cc) {
             const int c0 = half * (H / 2) + cc * 32;
-            if (cc + 1 < kChunks) tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0 + 32), r[(cc + 1) & 1]);
+            if (cc + 1 < kChunks) {
+                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0 + 32), r[(cc + 1) & 1]);
+                load_bias((cc + 1) & 1, c0 + 32);
+            }
             const uint32_t* v = r[cc & 1];
+            const float4* b = bs[cc & 1];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                const float4 b0 = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 8 * j)
-                                            : __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j));
-                const float4 b1 = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4)
-                                            : __ldg(reinterpret_cast<const float4*>(bias + c0 + 8 * j + 4));
+                const float4 b0 = b[2 * j], b1 = b[2 * j + 1];
                 uint4 pk;
                 pk.x = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 0]) + b0.x, 0.f),
                                      fmaxf(__uint_as_float(v[8 * j + 1]) + b0.y, 0.f));

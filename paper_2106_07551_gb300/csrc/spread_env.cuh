@@ -83,13 +83,23 @@ __device__ __forceinline__ void spread_obs_dyn(const SpreadEnv<N>& s, int i, flo
     for (; k < XS; ++k) o[k] = 0.f;
 }
 
-__device__ __forceinline__ float dist2(float ax, float ay, float bx, float by) {
+
+__device__ __forceinline__ float sqdist(float ax, float ay, float bx, float by) {
     const float dx = __fsub_rn(ax, bx), dy = __fsub_rn(ay, by);
-    return __fsqrt_rn(__fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy)));
+    return __fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy));
 }
 
+// |p_i - p_j| < 0.3 (two radii of 0.15) with |.| the correctly rounded fp32
+// square root of the squared distance holds exactly when the squared distance
+// is below this threshold: the rounded square root is monotone, and the
+// smallest fp32 value whose rounded root reaches 0.3f is fp32(0.3f * 0.3f).
+constexpr float kCollideSq = 0x1.70a3d8p-4f;
+
 // Mass 1, dt 0.1, damping 0.25, unit force along the chosen axis; reward after
-// the move; collision when centres are closer than 2 x 0.15.
+// the move; collision when centres are closer than 2 x 0.15. The rounded
+// square root is monotone, so the minimum over agents of the rounded distances
+// to a landmark equals the rounded root of the minimum squared distance: one
+// root per landmark gives the same bits as one per (landmark, agent).
 template <int N>
 __device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N], float (&r)[N]) {
 #pragma unroll
@@ -104,22 +114,24 @@ __device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N]
     float cover = 0.f;
 #pragma unroll
     for (int l = 0; l < N; ++l) {
-        float best = dist2(s.px[0], s.py[0], s.lx[l], s.ly[l]);
+        float best = sqdist(s.px[0], s.py[0], s.lx[l], s.ly[l]);
 #pragma unroll
         for (int j = 1; j < N; ++j) {
-            const float d = dist2(s.px[j], s.py[j], s.lx[l], s.ly[l]);
+            const float d = sqdist(s.px[j], s.py[j], s.lx[l], s.ly[l]);
             best = d < best ? d : best;
         }
-        cover = __fadd_rn(cover, best);
+        cover = __fadd_rn(cover, __fsqrt_rn(best));
     }
+    int coll[N];
 #pragma unroll
-    for (int i = 0; i < N; ++i) {
-        int coll = 0;
+    for (int i = 0; i < N; ++i) coll[i] = 0;
 #pragma unroll
-        for (int j = 0; j < N; ++j)
-            if (j != i && dist2(s.px[i], s.py[i], s.px[j], s.py[j]) < 0.3f) ++coll;
-        r[i] = -__fadd_rn(cover, (float)coll);
-    }
+    for (int i = 0; i < N; ++i)
+#pragma unroll
+        for (int j = i + 1; j < N; ++j)
+            if (sqdist(s.px[i], s.py[i], s.px[j], s.py[j]) < kCollideSq) { ++coll[i]; ++coll[j]; }
+#pragma unroll
+    for (int i = 0; i < N; ++i) r[i] = -__fadd_rn(cover, (float)coll[i]);
 }
 
 }  // namespace malib
