@@ -9,10 +9,14 @@
 // then the fp32 biases b1 [H], b2 [H], b3 [NOUT] (staged with the image), then
 // one activation tile [128][H]. The observation tile X [128][K1] lives at the
 // start of that activation tile: every layer's A operand is the previous
-// layer's output, so X, h1 and h2 reuse the same 64 KB. One 256-column TMEM
-// accumulator is
-// reused by the three layers. Thread 0 issues the MMAs; the 8 warps split each
-// epilogue (warp w: TMEM lane quarter w % 4, column half w / 4).
+// layer's output, so X, h1 and h2 reuse the same 64 KB. Tensor memory holds
+// two 256-column accumulators: layer 1 writes D1 (columns 0..255), layer 2 D2
+// (256..511), layer 3 four 16-column partial sums over D1's first 64 columns.
+// Thread 0 issues the MMAs; the 8 warps split each epilogue (warp w: TMEM lane
+// quarter w % 4, 64 of the 128 columns of a half). Each layer's epilogue runs
+// in two column halves, and the next layer's MMAs over the first half's K
+// range are issued before the second half is produced, so the tensor core
+// works while the epilogue warps drain tensor memory.
 #pragma once
 
 #include <cstdint>
@@ -39,7 +43,7 @@ struct MlpTc {
     static constexpr uint32_t kActBytes = 128 * H * 2;
     static constexpr uint32_t kSmemBytes = kStageBytes + kActBytes;
     static_assert(kStageBytes % 16 == 0, "activation tile 16-byte aligned");
-    static constexpr uint32_t kTmemCols = 256;
+    static constexpr uint32_t kTmemCols = 512;    // D1 [0,256), D2 [256,512), D3 [0,64)
     static constexpr uint32_t kLboAct = (128 / 8) * 128;            // K-chunk stride, 128 rows
     static constexpr uint32_t kLboW = (H / 8) * 128;                // K-chunk stride, H rows
     static constexpr uint32_t kLboW3 = (NOUT / 8) * 128;
@@ -55,23 +59,26 @@ struct MlpTc {
         tc::fence_after_sync();
     }
 
-    // Issued by thread 0: D(tmem) = A(act tile, K) . B^T (B: n_rows x K image).
-    __device__ static void issue(uint32_t tbase, uint32_t act, uint32_t w, uint32_t lbo_w, int K,
-                                 uint32_t idesc) {
-        for (int s = 0; s < K / 16; ++s)
-            tc::mma_bf16(tbase, tc::smem_desc(act + 2u * s * kLboAct, kLboAct, 128),
-                         tc::smem_desc(w + 2u * s * lbo_w, lbo_w, 128), idesc, s > 0);
+    // Issued by thread 0: D(tmem) (+)= A(act tile, K steps [s0, s1)) . B^T, where
+    // B starts `w` (a row-group offset inside an image whose K-chunk stride is
+    // lbo_w). The first step overwrites D when `fresh`.
+    __device__ static void issue(uint32_t d, uint32_t act, uint32_t w, uint32_t lbo_w, int s0,
+                                 int s1, uint32_t idesc, bool fresh) {
+        for (int s = s0; s < s1; ++s)
+            tc::mma_bf16(d, tc::smem_desc(act + 2u * s * kLboAct, kLboAct, 128),
+                         tc::smem_desc(w + 2u * s * lbo_w, lbo_w, 128), idesc, !(fresh && s == s0));
     }
 
-    // D + bias -> relu -> bf16 into the activation tile (this thread: one row,
-    // one half of the H columns, in 32-column chunks; the next chunk's tensor
-    // memory load and bias loads are in flight while the current chunk is
-    // processed).
-    __device__ static void epilogue_hidden(uint8_t* act, const float* bias, uint32_t tbase) {
+    // Columns [c_begin, c_begin + 128) of a layer's output: D (TMEM column
+    // tcol + c) + bias -> relu -> bf16 into the activation tile. Warp w takes
+    // TMEM lane quarter w % 4 and columns c_begin + 64 (w / 4) .. +63 in two
+    // 32-column chunks; the second chunk's tensor-memory and bias loads are in
+    // flight while the first is processed.
+    __device__ static void epilogue_half(uint8_t* act, const float* bias, uint32_t tbase,
+                                         int tcol, int c_begin) {
         const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-        const int q = warp & 3, half = warp >> 2;
+        const int q = warp & 3, h = warp >> 2;
         const int row = 32 * q + lane;
-        constexpr int kChunks = H / 2 / 32;
         uint32_t r[2][32];
         float4 bs[2][8];
         auto load_bias = [&](int buf, int c0) {
@@ -80,18 +87,19 @@ struct MlpTc {
                 bs[buf][j] = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
                                        : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
         };
-        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, half * (H / 2)), r[0]);
-        load_bias(0, half * (H / 2));
+        const int cb = c_begin + 64 * h;
+        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb), r[0]);
+        load_bias(0, cb);
         tc::tmem_wait_ld();
 #pragma unroll
-        for (int cc = 0; cc < kChunks; ++cc) {
-            const int c0 = half * (H / 2) + cc * 32;
-            if (cc + 1 < kChunks) {
-                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, c0 + 32), r[(cc + 1) & 1]);
-                load_bias((cc + 1) & 1, c0 + 32);
+        for (int cc = 0; cc < 2; ++cc) {
+            const int c0 = cb + cc * 32;
+            if (cc == 0) {
+                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + c0 + 32), r[1]);
+                load_bias(1, c0 + 32);
             }
-            const uint32_t* v = r[cc & 1];
-            const float4* b = bs[cc & 1];
+            const uint32_t* v = r[cc];
+            const float4* b = bs[cc];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const float4 b0 = b[2 * j], b1 = b[2 * j + 1];
@@ -106,7 +114,7 @@ struct MlpTc {
                                      fmaxf(__uint_as_float(v[8 * j + 7]) + b1.w, 0.f));
                 *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
             }
-            if (cc + 1 < kChunks) tc::tmem_wait_ld();
+            if (cc == 0) tc::tmem_wait_ld();
         }
     }
 
@@ -140,29 +148,47 @@ struct MlpTc {
         } else {
             handoff();
         }
+        const uint32_t idesc_full = tc::instr_desc(128, H, 1);
+        const uint32_t idesc3 = tc::instr_desc(128, NOUT, 1);
+        const uint32_t d1 = tbase, d2 = tbase + 256;
+        constexpr int kS = H / 16;                      // K steps of layers 2 and 3
+        // layer 1 (N = 256, K = K1) into D1
         if (threadIdx.x == 0) {
-            issue(tbase, s_act, s_w1, kLboW, K1, tc::instr_desc(128, H, 1));
+            issue(d1, s_act, s_w1, kLboW, 0, K1 / 16, idesc_full, true);
             tc::mma_commit(bar);
         }
         wait_mma(bar, parity, err);
-        epilogue_hidden(act, bias, tbase);
+        // h1 columns 0..127, then layer-2 K steps 0..7 (N = 256) while h1
+        // columns 128..255 are produced, then K steps 8..15
+        epilogue_half(act, bias, tbase, 0, 0);
+        handoff();
+        if (threadIdx.x == 0) issue(d2, s_act, s_w2, kLboW, 0, kS / 2, idesc_full, true);
+        epilogue_half(act, bias, tbase, 0, H / 2);
         handoff();
         if (threadIdx.x == 0) {
-            issue(tbase, s_act, s_w2, kLboW, H, tc::instr_desc(128, H, 1));
+            issue(d2, s_act, s_w2, kLboW, kS / 2, kS, idesc_full, false);
             tc::mma_commit(bar);
         }
         wait_mma(bar, parity, err);
-        epilogue_hidden(act, bias + H, tbase);
+        // h2 columns 0..127, then layer-3 K steps 0..7 while h2 columns
+        // 128..255 are produced. Layer 3 runs as 4 chains of 4 MMAs into TMEM
+        // columns 16j (D1's columns, free once h1 is written).
+        epilogue_half(act, bias + H, tbase, 256, 0);
         handoff();
-        if (threadIdx.x == 0) {
-            // four independent accumulators (TMEM columns 16j..16j+15) over K
-            // quarters, so the 16 small MMAs form 4 short chains
-            const uint32_t idesc3 = tc::instr_desc(128, NOUT, 1);
-            for (int s = 0; s < H / 16; ++s)
-                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (H / 64))),
+        if (threadIdx.x == 0)
+            for (int s = 0; s < kS / 2; ++s)
+                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))),
                              tc::smem_desc(s_act + 2u * s * kLboAct, kLboAct, 128),
                              tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
-                             (s % (H / 64)) != 0);
+                             (s % (kS / 4)) != 0);
+        epilogue_half(act, bias + H, tbase, 256, H / 2);
+        handoff();
+        if (threadIdx.x == 0) {
+            for (int s = kS / 2; s < kS; ++s)
+                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))),
+                             tc::smem_desc(s_act + 2u * s * kLboAct, kLboAct, 128),
+                             tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
+                             (s % (kS / 4)) != 0);
             tc::mma_commit(bar);
         }
         wait_mma(bar, parity, err);
