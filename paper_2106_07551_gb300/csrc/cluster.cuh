@@ -48,6 +48,41 @@ __device__ __forceinline__ uint32_t atomic_add(uint32_t addr, uint32_t v) {
     return old;
 }
 
+// Asynchronous 16-byte store into a peer CTA's shared memory that, once the
+// data is written, completes 16 bytes of transaction count on the mbarrier at
+// `remote_bar` (both addresses from map(), in the same peer CTA).
+__device__ __forceinline__ void st_async_v4(uint32_t remote_addr, uint4 v, uint32_t remote_bar) {
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, "
+        "[%5];" ::"r"(remote_addr),
+        "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(remote_bar)
+        : "memory");
+}
+
+// Bounded wait (at most limit_ns) for the phase `parity` of a local mbarrier
+// whose transactions come from peer CTAs; acquires at cluster scope so the
+// peers' completed stores are visible. Returns false on expiry.
+__device__ __forceinline__ bool wait_cluster_bounded(uint64_t* bar, uint32_t parity,
+                                                     uint64_t limit_ns) {
+    auto try_once = [&]() {
+        uint32_t ok;
+        asm volatile(
+            "{\n .reg .pred p;\n"
+            " mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+            " selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(ok)
+            : "r"(smem_u32(bar)), "r"(parity)
+            : "memory");
+        return ok != 0;
+    };
+    if (try_once()) return true;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+        if (try_once()) return true;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
+    }
+}
+
 __device__ __forceinline__ void fence_cluster() {
     asm volatile("fence.acq_rel.cluster;" ::: "memory");
 }

@@ -103,15 +103,12 @@ struct MlpTc {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const float4 b0 = b[2 * j], b1 = b[2 * j + 1];
+                auto f = [&](int i) { return __uint_as_float(v[8 * j + i]); };
                 uint4 pk;
-                pk.x = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 0]) + b0.x, 0.f),
-                                     fmaxf(__uint_as_float(v[8 * j + 1]) + b0.y, 0.f));
-                pk.y = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 2]) + b0.z, 0.f),
-                                     fmaxf(__uint_as_float(v[8 * j + 3]) + b0.w, 0.f));
-                pk.z = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 4]) + b1.x, 0.f),
-                                     fmaxf(__uint_as_float(v[8 * j + 5]) + b1.y, 0.f));
-                pk.w = tc::pack_bf16(fmaxf(__uint_as_float(v[8 * j + 6]) + b1.z, 0.f),
-                                     fmaxf(__uint_as_float(v[8 * j + 7]) + b1.w, 0.f));
+                pk.x = tc::bias_relu_bf16x2(f(0), f(1), b0.x, b0.y);
+                pk.y = tc::bias_relu_bf16x2(f(2), f(3), b0.z, b0.w);
+                pk.z = tc::bias_relu_bf16x2(f(4), f(5), b1.x, b1.y);
+                pk.w = tc::bias_relu_bf16x2(f(6), f(7), b1.z, b1.w);
                 *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
             }
             if (cc == 0) tc::tmem_wait_ld();

@@ -6,11 +6,14 @@
 // CTA k keeps the policy of agent k resident in shared memory and every CTA
 // keeps a replica of all 128 environments' state in registers (one thread per
 // environment). Per step, CTA k builds agent k's observations as a 128-row
-// bf16 tile, runs it through the tensor-core MLP, draws agent k's actions and
-// broadcasts them to the other 7 CTAs through distributed shared memory; after
-// one bounded cluster synchronisation every CTA applies the same 8 actions to
-// its replica (identical IEEE operations, identical bits) and writes agent k's
-// trajectory (observation, action, reward; CTA 0 the done flags).
+// bf16 tile (the fp32 rows are staged in shared memory and leave as contiguous
+// stores), runs it through the tensor-core MLP and draws agent k's actions.
+// The 128 action bytes go to the 7 peers by asynchronous shared-memory stores
+// that complete transaction counts on each peer's mbarrier, so a CTA waits
+// only for the data it needs (bounded), with no cluster-wide barrier per step.
+// Every CTA then applies the same 8 actions to its replica (identical IEEE
+// operations, identical bits) and writes agent k's trajectory (observation,
+// action, reward; CTA 0 the done flags).
 #include "cluster.cuh"
 #include "device_common.cuh"
 #include "internal.h"
@@ -27,6 +30,9 @@ using Eng = MlpTc<kK1, 256, 16, false>;      // biases read through L1 (shared m
 constexpr int kThreads = 256;
 constexpr uint32_t kActs = Eng::kSmemBytes;                  // actions [parity][agent][env] u8
 constexpr uint32_t kSmem = kActs + 2 * kN * 128;
+constexpr uint32_t kStage = 128 * kK1 * 2;                   // fp32 obs rows, after X in the tile
+static_assert(kStage % 16 == 0 && kStage + 128 * kObsPad * 4 <= Eng::kActBytes, "obs staging fits");
+constexpr uint32_t kActTx = (kN - 1) * 128;                  // action bytes received per step
 
 __device__ __forceinline__ void cluster_barrier_all() {
     asm volatile("barrier.cluster.arrive.release.aligned;\n"
@@ -38,9 +44,8 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t stage_bar;
     __shared__ __align__(8) uint64_t mma_bar;
+    __shared__ __align__(8) uint64_t act_bar[2];   // peers' actions of steps with parity 0 / 1
     __shared__ uint32_t tmem_base;
-    __shared__ uint32_t flags[kN];
-    __shared__ uint32_t ok_slot;
 
     uint8_t* acts = smem + kActs;
     const uint32_t me = cl::rank();
@@ -49,8 +54,11 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     if (tid == 0) {
         mbar_init(&stage_bar, 1);
         mbar_init(&mma_bar, 1);
+        mbar_init(&act_bar[0], 1);
+        mbar_init(&act_bar[1], 1);
+        mbar_arrive_expect_tx(&act_bar[0], kActTx);      // armed for steps 0 and 1
+        mbar_arrive_expect_tx(&act_bar[1], kActTx);
     }
-    if (tid < kN) flags[tid] = 0;
     if (warp == 0) {
         tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
         tc::tmem_relinquish();
@@ -60,10 +68,11 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
-    cluster_barrier_all();
+    cluster_barrier_all();          // every peer's barriers exist before any remote store
     const uint32_t tbase = tmem_base;
 
-    uint32_t stage_par = 0, mma_par = 0, epoch = 0, step = 0;
+    uint32_t stage_par = 0, mma_par = 0, step = 0;
+    bool dead = false;              // a peer wait expired: stop waiting, results are flagged
     const int epp = (int)(a.n_envs / a.n_pairs);
     const int T = a.episode_len;
     const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
@@ -72,6 +81,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     const int64_t lo = cid * per, hi = min(items, lo + per);
     int staged = -1;
     const float* gbias = nullptr;
+    float* stage = reinterpret_cast<float*>(smem + Eng::kAct + kStage);
 
     for (int64_t it = lo; it < hi; ++it) {
         const int pair = (int)(it / a.n_episodes);
@@ -111,15 +121,16 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         for (int t = 0; t < T; ++t) {
             const uint32_t par = step & 1u;
             const int64_t ix = ((ep * T + t) * a.n_envs + env) * kN;
+            uint8_t* my_acts = acts + (par * kN + me) * 128;
             float u = 0.f;
             if (mine) {
                 u = u24(draw(g, (uint32_t)t, me, a.seed).x);      // ready before the logits
                 float o[kObsPad];
                 spread_obs_dyn<kN, kObsPad>(s, (int)me, o);
-                float4* dst = reinterpret_cast<float4*>(a.obs + (ix + me) * kObsPad);
+                float4* srow = reinterpret_cast<float4*>(stage + tid * kObsPad);
 #pragma unroll
                 for (int q = 0; q < kObsPad / 4; ++q)
-                    dst[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                    srow[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
                 uint32_t w[kK1 / 2];
 #pragma unroll
                 for (int i = 0; i < kK1 / 2; ++i)
@@ -129,25 +140,41 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     *reinterpret_cast<uint4*>(smem + Eng::kAct + Eng::act_offset(tid, 8 * c)) =
                         make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
             }
+            __syncthreads();
+            {   // observations of agent me: [ep][t][env][agent][obs_pad], 144-byte runs per env
+                const int64_t base = ((ep * T + t) * a.n_envs + (int64_t)pair * epp) * kN + me;
+                const float4* src = reinterpret_cast<const float4*>(stage);
+                for (int q = tid; q < epp * (kObsPad / 4); q += kThreads) {
+                    const int v = q / (kObsPad / 4), c = q - v * (kObsPad / 4);
+                    reinterpret_cast<float4*>(a.obs + (base + (int64_t)v * kN) * kObsPad)[c] = src[q];
+                }
+            }
             Eng::forward(smem, gbias, tbase, &mma_bar, mma_par, a.err, [&](int row, const float* lg) {
+                int act = 0;
                 if (row < epp) {
                     float l5[kA];
 #pragma unroll
                     for (int k = 0; k < kA; ++k) l5[k] = lg[k];
-                    const int act = sample_masked<kA>(l5, 0x1Fu, u);
+                    act = sample_masked<kA>(l5, 0x1Fu, u);
                     if (a.logits)
 #pragma unroll
                         for (int k = 0; k < kA; ++k) a.logits[(ix + me) * kA + k] = l5[k];
                     a.action[ix + me] = (uint8_t)act;
-                    const uint32_t off = (par * kN + me) * 128 + (uint32_t)row;
-#pragma unroll
-                    for (uint32_t r = 0; r < kN; ++r)
-                        asm volatile("st.shared::cluster.u8 [%0], %1;" ::"r"(cl::map(acts + off, r)),
-                                     "r"((uint32_t)act)
-                                     : "memory");
                 }
-            });
-            cl::sync(flags, ++epoch, kN, me, a.err, &ok_slot);
+                my_acts[row] = (uint8_t)act;
+            });   // its opening barrier also ends the staged rows' reads before h1 overwrites them
+            // forward ends with a CTA barrier: all 128 action bytes are in my_acts
+            if (tid < (kN - 1) * 8) {
+                const uint32_t c = (uint32_t)tid & 7u, j = (uint32_t)tid >> 3;
+                const uint32_t r = j < me ? j : j + 1;
+                const uint4 v = *reinterpret_cast<const uint4*>(my_acts + 16 * c);
+                cl::st_async_v4(cl::map(my_acts + 16 * c, r), v, cl::map(&act_bar[par], r));
+            }
+            if (!dead && !cl::wait_cluster_bounded(&act_bar[par], (step >> 1) & 1u, kWaitLimitNs)) {
+                dead = true;
+                atomicOr(a.err, ERRBIT_TIMEOUT);
+            }
+            if (tid == 0) mbar_arrive_expect_tx(&act_bar[par], kActTx);   // re-armed for step + 2
             if (mine) {
                 int act[kN];
 #pragma unroll
@@ -166,7 +193,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     }
     tc::fence_before_sync();
     __syncthreads();
-    cluster_barrier_all();
+    cluster_barrier_all();          // every remote store to this CTA was awaited before this
     if (warp == 0) tc::tmem_dealloc(tbase, Eng::kTmemCols);
 }
 

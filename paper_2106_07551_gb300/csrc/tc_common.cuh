@@ -161,5 +161,22 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     return r;
 }
 
+// bf16x2 of relu(x0 + b0) (low half) and relu(x1 + b1) (high half): one packed
+// fp32 add (each lane rounded to nearest, as a scalar add) and one conversion
+// that rounds to nearest-even and clamps negative results to zero. Rounding is
+// monotonic and keeps zero, so this equals rounding relu(x + b), up to the sign
+// of a zero result.
+__device__ __forceinline__ uint32_t bias_relu_bf16x2(float x0, float x1, float b0, float b1) {
+    uint32_t r;
+    asm("{\n .reg .b64 x, b, s;\n .reg .f32 lo, hi;\n"
+        " mov.b64 x, {%1, %2};\n mov.b64 b, {%3, %4};\n"
+        " add.rn.f32x2 s, x, b;\n"
+        " mov.b64 {lo, hi}, s;\n"
+        " cvt.rn.relu.bf16x2.f32 %0, hi, lo;\n}"
+        : "=r"(r)
+        : "f"(x0), "f"(x1), "f"(b0), "f"(b1));
+    return r;
+}
+
 }  // namespace tc
 }  // namespace malib
