@@ -7,12 +7,15 @@
 // owns 128 hands in flight. Rows 64 s .. 64 s + 63 of each CTA's 128-row tile
 // belong to the hands of CTA s. Each step, the hands of a CTA are ranked by
 // acting seat with warp ballots; the first 64 acting as seat r write their bf16
-// observation into rows of CTA r's tile through distributed shared memory (the
-// rest wait a step: a hand's randomness depends only on its own ids, so
-// deferral changes no result). Each CTA runs its tile through the tensor-core
-// MLP and returns every valid row's logits to the hand's CTA. Both CTAs take
-// the same pair segments and leave a segment together, when neither holds a
-// live hand.
+// observation into rows of CTA r's tile (the rest wait a step: a hand's
+// randomness depends only on its own ids, so deferral changes no result). Each
+// CTA runs its tile through the tensor-core MLP and returns every row's logits
+// to the row's CTA. Both directions use asynchronous stores into the peer's
+// shared memory that complete transaction counts on the receiver's mbarrier:
+// every slot is written each step (unused rows with zeros) plus a 16-byte
+// header (rows placed, live hands), so each receiver expects a fixed byte
+// count and waits (bounded) for its data alone. Both CTAs take the same pair
+// segments and leave a segment together, when neither holds a live hand.
 #include "cluster.cuh"
 #include "device_common.cuh"
 #include "eval_common.cuh"
@@ -28,8 +31,10 @@ using Eng = MlpTc<32, 256, 16>;
 constexpr int kSlots = 128;               // hands per CTA
 constexpr int kPart = 64;                 // tile rows per source CTA
 constexpr int kThreads = 256;
-constexpr uint32_t kLg = Eng::kSmemBytes;                 // logits [target][row][4] fp32
-constexpr uint32_t kSmem = kLg + 2 * 128 * 16;
+constexpr uint32_t kLg = Eng::kSmemBytes;                 // logits [target][rank][4] fp32
+constexpr uint32_t kSmem = kLg + 2 * kPart * 16;
+constexpr uint32_t kXTx = 2 * (kPart * 64 + 16);          // tile bytes + headers received per step
+constexpr uint32_t kLgTx = 2 * kPart * 16;                // logits bytes received per step
 constexpr int kMaxDec = 8;
 
 __device__ __forceinline__ void cluster_barrier_all() {
@@ -43,11 +48,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     __shared__ __align__(8) uint64_t stage_bar;
     __shared__ __align__(8) uint64_t mma_bar;
     __shared__ uint32_t tmem_base;
-    __shared__ uint32_t flags[2];
-    __shared__ uint32_t nrows[2];         // valid rows from each source CTA (this step)
-    __shared__ uint32_t live_of[2];       // live hands of each CTA (this step)
+    __shared__ __align__(8) uint64_t x_bar;        // tile rows and headers of this step
+    __shared__ __align__(8) uint64_t lg_bar;       // logits of this step
+    __shared__ __align__(16) uint4 hdr[2];         // from CTA s: {rows placed here, live hands}
+    __shared__ uint32_t dead_s, go_s;              // a peer wait expired; this step runs
     __shared__ int wcnt[2][8];
-    __shared__ uint32_t ok_slot;
     __shared__ unsigned long long next_k;
 
     float* lgbuf = reinterpret_cast<float*>(smem + kLg);
@@ -57,7 +62,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (tid == 0) {
         mbar_init(&stage_bar, 1);
         mbar_init(&mma_bar, 1);
-        flags[0] = flags[1] = 0;
+        dead_s = 0u;
+        mbar_init(&x_bar, 1);
+        mbar_init(&lg_bar, 1);
+        mbar_arrive_expect_tx(&x_bar, kXTx);       // armed for the first step
+        mbar_arrive_expect_tx(&lg_bar, kLgTx);
     }
     if (warp == 0) {
         tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
@@ -68,10 +77,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
-    cluster_barrier_all();          // peers' flags exist before any remote access
+    cluster_barrier_all();          // peers' barriers exist before any remote store
     const uint32_t tbase = tmem_base;
 
-    uint32_t stage_par = 0, mma_par = 0, epoch = 0, step = 0;
+    uint32_t stage_par = 0, mma_par = 0, x_par = 0, lg_par = 0, step = 0;
+
     const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
     const int64_t n_cl = gridDim.x / 2, cid = blockIdx.x / 2;
     const int64_t per = (total + n_cl - 1) / n_cl;
@@ -133,12 +143,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const unsigned mine = seat == 1 ? b1 : b0;
             const int rank = pre + __popc(mine & ((1u << lane) - 1u));
             const bool placed = live && rank < kPart;
-            const int row = (int)me * kPart + rank;
             float ob[17];
             float u = 0.f;
+            // Every (target CTA, row) slot of this CTA's part of both tiles is
+            // written each step: by its placed hand, else with zeros, so each
+            // target receives a fixed byte count.
             if (placed) {
                 u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);   // ready before the logits
-                const uint32_t target = (uint32_t)seat;
                 leduc_obs(h, ob);
                 uint32_t w[16];
 #pragma unroll
@@ -146,31 +157,63 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 w[8] = tc::pack_bf16(ob[16], 0.f);
 #pragma unroll
                 for (int i = 9; i < 16; ++i) w[i] = 0u;
+                const uint32_t bar = cl::map(&x_bar, (uint32_t)seat);
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
-                    cl::st_v4(cl::map(smem + Eng::kAct + Eng::act_offset(row, 8 * c), target),
-                              make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]));
-                asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+                    cl::st_async_v4(cl::map(smem + Eng::kAct + Eng::act_offset((int)me * kPart + rank, 8 * c),
+                                            (uint32_t)seat),
+                                    make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]), bar);
             }
-            if (tid < 2) {                  // thread s tells CTA s how many rows it got from us
+            if (tid < 2 * kPart) {
+                const int tgt = tid / kPart, rk = tid % kPart;
+                if (rk >= min(tgt == 0 ? c0 : c1, kPart)) {
+                    const uint32_t bar = cl::map(&x_bar, (uint32_t)tgt);
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        cl::st_async_v4(cl::map(smem + Eng::kAct + Eng::act_offset((int)me * kPart + rk, 8 * c),
+                                                (uint32_t)tgt),
+                                        make_uint4(0, 0, 0, 0), bar);
+                }
+            }
+            if (tid < 2) {                  // header to CTA tid: rows placed there, live hands here
                 const uint32_t n = (uint32_t)min(tid == 0 ? c0 : c1, kPart);
-                cl::st_u32(cl::map(&nrows[me], (uint32_t)tid), n);
-                cl::st_u32(cl::map(&live_of[me], (uint32_t)tid), (uint32_t)(c0 + c1));
+                cl::st_async_v4(cl::map(&hdr[me], (uint32_t)tid), make_uint4(n, (uint32_t)(c0 + c1), 0, 0),
+                                cl::map(&x_bar, (uint32_t)tid));
             }
-            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
-            if (live_of[0] == 0 && live_of[1] == 0) break;
+            // Thread 0 waits (bounded) and decides for the CTA; the barrier
+            // passes its view of the received data to every thread.
+            if (tid == 0) {
+                if (!dead_s && !cl::wait_cluster_bounded(&x_bar, x_par, kWaitLimitNs)) {
+                    dead_s = 1u;
+                    atomicOr(a.err, ERRBIT_TIMEOUT);
+                }
+                mbar_arrive_expect_tx(&x_bar, kXTx);                      // armed for the next step
+                go_s = (!dead_s && (hdr[0].y != 0 || hdr[1].y != 0)) ? 1u : 0u;
+            }
+            x_par ^= 1u;
+            __syncthreads();
+            if (!go_s) break;
+            // The tile rows arrived as generic-proxy stores; the MMA issuer
+            // orders them before the tensor core's reads (forward's opening fence).
             Eng::forward(smem, nullptr, tbase, &mma_bar, mma_par, a.err, [&](int r, const float* lg) {
                 const uint32_t src = (uint32_t)(r / kPart);
-                if ((uint32_t)(r % kPart) < nrows[src]) {
-                    const uint32_t dst = cl::map(lgbuf + (me * 128 + r) * 4, src);
-                    cl::st_f32(dst, lg[0]);
-                    cl::st_f32(dst + 4, lg[1]);
-                    cl::st_f32(dst + 8, lg[2]);
-                }
+                cl::st_async_v4(cl::map(lgbuf + (me * kPart + r % kPart) * 4, src),
+                                make_uint4(__float_as_uint(lg[0]), __float_as_uint(lg[1]),
+                                           __float_as_uint(lg[2]), 0u),
+                                cl::map(&lg_bar, src));
             }, /*x_published=*/true);
-            cl::sync(flags, ++epoch, 2, me, a.err, &ok_slot);
+            if (tid == 0) {
+                if (!dead_s && !cl::wait_cluster_bounded(&lg_bar, lg_par, kWaitLimitNs)) {
+                    dead_s = 1u;
+                    atomicOr(a.err, ERRBIT_TIMEOUT);
+                }
+                mbar_arrive_expect_tx(&lg_bar, kLgTx);
+            }
+            lg_par ^= 1u;
+            __syncthreads();
+            if (dead_s) break;
             if (placed) {
-                const float* lp = lgbuf + (seat * 128 + row) * 4;
+                const float* lp = lgbuf + (seat * kPart + rank) * 4;
                 float lg[3] = {lp[0], lp[1], lp[2]};
                 const unsigned legal = leduc_legal(h);
                 const int act = sample_masked<3>(lg, legal, u);
@@ -223,6 +266,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             ++step;
         }
         block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+        if (dead_s) break;          // uniform: written only before a barrier
     }
     tc::fence_before_sync();
     __syncthreads();
