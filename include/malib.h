@@ -42,7 +42,8 @@ typedef enum malib_status {
     MALIB_ECUDA = -3,         /* a CUDA runtime call failed */
     MALIB_ESTATE = -4,        /* no population loaded, or env/population mismatch */
     MALIB_ETIMEOUT = -5,      /* a bounded device-side wait expired */
-    MALIB_EUNSUPPORTED = -6   /* valid request outside the built kernels' shapes */
+    MALIB_EUNSUPPORTED = -6,  /* valid request outside the built kernels' shapes */
+    MALIB_ENOTCONVERGED = -7  /* an iterative solver reached its iteration limit */
 } malib_status;
 
 typedef enum malib_env_kind {
@@ -232,6 +233,52 @@ int malib_eval_payoff_ex(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pair
  */
 int malib_eval_payoff_noalloc(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pairs,
                               int64_t n_episodes, uint64_t seed, double* payoff_out);
+
+/* ---- meta-game solvers on payoff tables (Sec. 4.2, App. C.2) ----
+ *
+ * The PSRO loop of Sec. 4.2 turns the payoff table into a meta-strategy with a
+ * meta-solver (fictitious play; an exact LP solver is named as the
+ * alternative), and the training-loop listing of App. C.2 aggregates payoffs
+ * under that equilibrium. These calls solve G zero-sum matrix games at once,
+ * one CTA per game.
+ *
+ * Payoff layout (all calls): device fp64; element (g, i, j), seat 0's payoff
+ * when row policy i meets column policy j, is payoff[((g*m + i)*n + j)*stride].
+ * stride 1 reads a plain [G][m][n] table; stride 4 reads the mean column of
+ * malib_eval_payoff's [n_pairs][4] output when its pairs are the row-major
+ * Cartesian product of m rows and n columns. Entries must be finite.
+ * All outputs are caller-owned device fp64 buffers. Calls are asynchronous on
+ * the context's stream; EINVAL for host pointers or bad sizes, EUNSUPPORTED
+ * for dimensions above the stated limits. The context needs no population.
+ */
+
+/* Fictitious play: both seats play policy 0 first, then each plays the first
+ * (lowest-index) best response to the other's empirical play so far; the
+ * cumulative payoffs are fp64 sums in play order, so results are reproducible
+ * bit for bit. After iters >= 1 plays: x_out [G][m] and y_out [G][n] are the
+ * empirical mixtures (play counts / iters); bounds_out [G][2] = {min_j (x^T
+ * A)_j, max_i (A y)_i}, which bracket the game value (their difference is the
+ * mixtures' NashConv). 1 <= m, n <= 1024. */
+int malib_meta_fictitious_play(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
+                               int32_t n, int32_t stride, int64_t iters, double* x_out,
+                               double* y_out, double* bounds_out);
+
+/* Exact equilibrium by linear programming (simplex, Bland's rule): value_out
+ * [G] = the game value; x_out [G][m], y_out [G][n] one equilibrium (not unique
+ * in general). 1 <= m, n <= 512; tableaus larger than 200 KB live in
+ * context-owned device memory. A game that reaches the pivot limit raises
+ * MALIB_ENOTCONVERGED at the next malib_sync. */
+int malib_meta_lp_nash(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
+                       int32_t n, int32_t stride, double* x_out, double* y_out,
+                       double* value_out);
+
+/* Payoffs under mixtures x [G][m], y [G][n] (device fp64): row_payoff_out
+ * [G][m] = A y (what each row policy, e.g. a new best response, earns against
+ * the column mixture), col_payoff_out [G][n] = x^T A, value_out [G] = x^T A y
+ * (the equilibrium's expected payoff). */
+int malib_meta_aggregate(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
+                         int32_t n, int32_t stride, const double* x, const double* y,
+                         double* row_payoff_out, double* col_payoff_out, double* value_out);
 
 /* ---- measurement and self-test entry points (used by tests and the benchmark) ---- */
 

@@ -225,6 +225,37 @@ class Context:
         ms = self.lib.malib_main_kernel_ms(self.handle, C.byref(n), int(reset))
         return ms, n.value
 
+    # ---- meta-game solvers (device fp64 tensors; payoff [G][m][n] or [G][m][n][stride]) ----
+    @staticmethod
+    def _table(payoff, stride):
+        G, m, n = int(payoff.shape[0]), int(payoff.shape[1]), int(payoff.shape[2])
+        if not payoff.is_contiguous():
+            raise ValueError("payoff must be contiguous")
+        return G, m, n, int(stride)
+
+    def meta_fictitious_play(self, payoff, iters, x_out, y_out, bounds_out, stride=1):
+        """Fictitious play on G games: x_out [G][m], y_out [G][n], bounds_out [G][2]."""
+        G, m, n, st = self._table(payoff, stride)
+        _check(self.lib, self.handle,
+               self.lib.malib_meta_fictitious_play(self.handle, _ptr(payoff), G, m, n, st,
+                                                   int(iters), _ptr(x_out), _ptr(y_out),
+                                                   _ptr(bounds_out)))
+
+    def meta_lp_nash(self, payoff, x_out, y_out, value_out, stride=1):
+        """LP equilibrium of G games: x_out [G][m], y_out [G][n], value_out [G]."""
+        G, m, n, st = self._table(payoff, stride)
+        _check(self.lib, self.handle,
+               self.lib.malib_meta_lp_nash(self.handle, _ptr(payoff), G, m, n, st, _ptr(x_out),
+                                           _ptr(y_out), _ptr(value_out)))
+
+    def meta_aggregate(self, payoff, x, y, row_out, col_out, value_out, stride=1):
+        """A y -> row_out [G][m], x^T A -> col_out [G][n], x^T A y -> value_out [G]."""
+        G, m, n, st = self._table(payoff, stride)
+        _check(self.lib, self.handle,
+               self.lib.malib_meta_aggregate(self.handle, _ptr(payoff), G, m, n, st, _ptr(x),
+                                             _ptr(y), _ptr(row_out), _ptr(col_out),
+                                             _ptr(value_out)))
+
     def selftest_philox(self, ctr, seed, out):
         _check(self.lib, self.handle,
                self.lib.malib_selftest_philox(self.handle, _ptr(ctr), seed, _ptr(out),

@@ -28,7 +28,8 @@ EXPORTS = (
     "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "malib_eval_stats", "malib_launch_count",
     "malib_set_timing", "malib_main_kernel_ms",
     "malib_selftest_philox", "malib_selftest_det_expf", "malib_selftest_sample",
-    "malib_selftest_mma",
+    "malib_selftest_mma", "malib_meta_fictitious_play", "malib_meta_lp_nash",
+    "malib_meta_aggregate",
 )
 
 
@@ -90,6 +91,9 @@ def load(path: str | None = None):
             "malib_selftest_det_expf": (C.c_int, [P, P, P, i64]),
             "malib_selftest_sample": (C.c_int, [P, P, P, P, i32, P, i64]),
             "malib_selftest_mma": (C.c_int, [P, i32, P, P, P, i32, i32]),
+            "malib_meta_fictitious_play": (C.c_int, [P, P, i32, i32, i32, i32, i64, P, P, P]),
+            "malib_meta_lp_nash": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P]),
+            "malib_meta_aggregate": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P, P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)

@@ -12,6 +12,7 @@ constexpr int kMaxAgents = 16;
 enum : int {
     ERRBIT_BAD_PAIR = 1,      // an id in a device pair table is out of range / wrong seat
     ERRBIT_TIMEOUT = 2,       // a bounded mbarrier wait expired
+    ERRBIT_NOT_CONVERGED = 4, // an iterative solver reached its iteration limit
 };
 
 // fp32 MLP policy, kernel layout of one population member (floats, every
@@ -126,6 +127,22 @@ struct CtxView {
 bool ctx_view(const void* ctx, CtxView* v);
 int ctx_fail(void* ctx, int code, const char* msg);
 void ctx_count_launches(void* ctx, int n);
+// Device work space owned by the context, grown on its stream (cudaMallocAsync).
+int ctx_scratch(void* ctx, int64_t bytes, void** out);
+
+// Meta-game solvers (meta_solver.cu).
+cudaError_t launch_fictitious_play(const double* P, int32_t G, int32_t m, int32_t n, int32_t stride,
+                                   int64_t T, double* x, double* y, double* bounds, int n_sm,
+                                   cudaStream_t s);
+cudaError_t launch_aggregate(const double* P, int32_t G, int32_t m, int32_t n, int32_t stride,
+                             const double* x, const double* y, double* ay, double* xa, double* val,
+                             int n_sm, cudaStream_t s);
+int64_t lp_tableau_doubles(int32_t m, int32_t n);
+bool lp_on_chip(int32_t m, int32_t n);
+int lp_grid(int32_t n_games, int n_sm);
+cudaError_t launch_lp_nash(const double* P, int32_t G, int32_t m, int32_t n, int32_t stride,
+                           double* x, double* y, double* val, double* scratch, int* err, int n_sm,
+                           cudaStream_t s);
 
 bool leduc_f32_supported(int hidden);
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden);

@@ -55,6 +55,8 @@ struct malib_ctx {
     int64_t pairs_cap = 0;
     double* d_out = nullptr;
     int64_t out_cap = 0;
+    uint8_t* scratch = nullptr;        // solver work space (LP tableaus that do not fit on chip)
+    int64_t scratch_cap = 0;
 
     int64_t launches = 0;
     bool timing = false;
@@ -284,6 +286,8 @@ int read_device_errors(malib_ctx* c) {
             return fail(c, MALIB_ETIMEOUT, "a bounded device wait expired (staging copy)");
         if (h & ERRBIT_BAD_PAIR)
             return fail(c, MALIB_EINVAL, "a device pair table held an invalid policy id or seat");
+        if (h & ERRBIT_NOT_CONVERGED)
+            return fail(c, MALIB_ENOTCONVERGED, "the LP solver reached its pivot limit");
     }
     return MALIB_OK;
 }
@@ -342,6 +346,17 @@ int ctx_fail(void* ctx, int code, const char* msg) {
     return fail(static_cast<malib_ctx*>(ctx), code, "%s", msg);
 }
 
+int ctx_scratch(void* ctx, int64_t bytes, void** out) {
+    malib_ctx* c = static_cast<malib_ctx*>(ctx);
+    if (!c || !out || bytes < 0) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (!g.ok) return fail(c, MALIB_ECUDA, "cannot select the context's device");
+    const int r = ensure(c, c->scratch, c->scratch_cap, std::max<int64_t>(bytes, 1), "solver scratch");
+    if (r != MALIB_OK) return r;
+    *out = c->scratch;
+    return MALIB_OK;
+}
+
 void ctx_count_launches(void* ctx, int n) {
     if (ctx) static_cast<malib_ctx*>(ctx)->launches += n;
 }
@@ -390,6 +405,7 @@ void malib_destroy(malib_ctx* c) {
     cudaFree(c->d_err);
     cudaFree(c->d_pairs);
     cudaFree(c->d_out);
+    cudaFree(c->scratch);
     delete c;
 }
 
