@@ -46,7 +46,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "leduc_bf16", "spread8"],
+    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "leduc_bf16", "spread8",
+                                           "meta"],
                     default="leduc")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -422,10 +423,146 @@ def run_e2e(args, ctx, w, spec, dev, rollout):
             "d2h_bytes_per_step": int(d2h), "steps": n}
 
 
+# ----------------------------------------------------------------- meta-solver
+META_GAMES, META_M, META_N, META_PLAYS = 152, 100, 100, 10_000
+
+
+def run_meta(args):
+    """Fictitious play (the Sec. 4.2 meta-solver) on a batch of payoff tables of
+    the paper's largest PSRO population (100 x 100), one game per SM: a step
+    is META_PLAYS plays of every game. Also times the LP equilibrium and the
+    aggregation on the same tables (reported beside the main value)."""
+    import numpy as np
+    import torch
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2106_07551_gb300 import Context
+
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    ctx = Context(local, stream)
+    rng = np.random.default_rng(2106075516 + rank)
+    G, m, n, T = META_GAMES, META_M, META_N, META_PLAYS
+    tables = rng.normal(size=(G, m, n))
+    P = torch.from_numpy(tables).to(dev)
+    x = torch.empty((G, m), dtype=torch.float64, device=dev)
+    y = torch.empty((G, n), dtype=torch.float64, device=dev)
+    b = torch.empty((G, 2), dtype=torch.float64, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        ctx.meta_fictitious_play(P, T, x, y, b)
+    torch.cuda.synchronize(dev)
+    ctx.sync()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    launches0 = ctx.launch_count()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clocks:
+        for k in range(args.steps):
+            flush.zero_()
+            ev[k][0].record(stream)
+            ctx.meta_fictitious_play(P, T, x, y, b)
+            ev[k][1].record(stream)
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    launches = ctx.launch_count() - launches0
+    ctx.sync()
+    total_ms = sum(a.elapsed_time(c) for a, c in ev)
+    total_ms_max = max_over_ranks(total_ms, world, dev)
+    plays_all = sum_over_ranks(float(G * T * args.steps), world, dev)
+    value = plays_all / (total_ms_max / 1e3)
+    ns_per_play = total_ms / args.steps * 1e6 / T     # per CTA (all games run concurrently)
+
+    # LP and aggregation on the same tables
+    v = torch.empty((G,), dtype=torch.float64, device=dev)
+    ay = torch.empty((G, m), dtype=torch.float64, device=dev)
+    xa = torch.empty((G, n), dtype=torch.float64, device=dev)
+    ctx.meta_lp_nash(P, x, y, v)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    ctx.meta_lp_nash(P, x, y, v)
+    e1.record(stream)
+    ctx.meta_aggregate(P, x, y, ay, xa, v)
+    torch.cuda.synchronize(dev)
+    ctx.sync()
+    lp_ms = e0.elapsed_time(e1)
+
+    e2e = None
+    cpu = None
+    if rank == 0:
+        # e2e: tables from pinned host memory, mixtures and bounds back
+        h_tab = torch.from_numpy(tables).pin_memory()
+        h_x = torch.empty((G, m), dtype=torch.float64).pin_memory()
+        h_y = torch.empty((G, n), dtype=torch.float64).pin_memory()
+        h_b = torch.empty((G, 2), dtype=torch.float64).pin_memory()
+        reps = max(1, args.e2e_steps // 5)
+        t0 = 0.0
+        for k in range(reps + 1):
+            torch.cuda.synchronize(dev)
+            s0 = time.perf_counter()
+            P.copy_(h_tab, non_blocking=True)
+            ctx.meta_fictitious_play(P, T, x, y, b)
+            h_x.copy_(x, non_blocking=True)
+            h_y.copy_(y, non_blocking=True)
+            h_b.copy_(b, non_blocking=True)
+            torch.cuda.synchronize(dev)
+            if k > 0:
+                t0 += time.perf_counter() - s0
+        e2e = {"value": G * T * reps / t0, "unit": "plays/s",
+               "h2d_bytes_per_step": int(h_tab.numel() * 8),
+               "d2h_bytes_per_step": int((h_x.numel() + h_y.numel() + h_b.numel()) * 8),
+               "steps": reps}
+        if world == 1 and not args.no_cpu_baseline:
+            from oracle import meta_solver as ms
+            n_games, t_cpu = 0, 0.0
+            while t_cpu < 10.0 and n_games < G:
+                s0 = time.perf_counter()
+                ms.fictitious_play(tables[n_games], T)
+                t_cpu += time.perf_counter() - s0
+                n_games += 1
+            cpu = {"value": n_games * T / t_cpu, "unit": "plays/s", "cores": 1, "kind": "oracle",
+                   "sample": f"{n_games} of the {G} games, {T} plays each ({t_cpu:.1f} s, numpy)"}
+    clk = clocks.summary()
+    ctx.close()
+    if rank == 0:
+        line = {"metric": "fictitious-play plays/sec over a batch of payoff tables",
+                "value": value, "unit": "plays/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic",
+                "config": {"workload": f"fictitious_play_{G}games_{m}x{n}_{T}plays",
+                           "games": G, "rows": m, "cols": n, "plays": T,
+                           "l2": "flushed (256 MiB write) before every timed step"},
+                "roofline": {"bound": "latency", "achieved": ns_per_play, "peak": None,
+                             "unit": "ns per play per game", "frac": None, "traffic": None,
+                             "kernel": "fictitious_play_kernel",
+                             "note": "each play depends on the previous play's argmax: one CTA "
+                                     "barrier and two warp reductions per play bound it"},
+                "lp_nash_ms": lp_ms, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+                "gpu_launches": launches}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "meta":
+        return run_meta(args)
     return run_ours(args)
 
 

@@ -21,101 +21,126 @@ constexpr int kFpPer = 4;                       // rows (columns) per thread: m,
 constexpr int kFpMaxDim = kFpThreads * kFpPer;
 constexpr int kSmemLimit = 200 * 1024;          // bytes of payoff / tableau kept on chip
 
-struct ArgBest {
-    double v;
-    int i;
-};
-
-// Better of two candidates: larger (sign = +1) or smaller (sign = -1) value,
-// the lower index on equal values.
-__device__ __forceinline__ ArgBest better(ArgBest a, ArgBest b, double sign) {
-    const double av = sign * a.v, bv = sign * b.v;
-    if (b.i < 0) return a;
-    if (a.i < 0) return b;
-    if (bv > av || (bv == av && b.i < a.i)) return b;
-    return a;
+// Order-preserving integer key of a finite double (larger double, larger
+// key), and its inverse. The comparisons of a play run on these keys: fp64
+// arithmetic is a narrow pipe on this part, integer compares and shuffles are
+// not. The cumulative payoffs start at +0.0 and every sum with +0.0 is +0.0,
+// so -0.0 never occurs and key equality is value equality.
+__device__ __forceinline__ long long okey(double v) {
+    const long long b = __double_as_longlong(v);
+    return b >= 0 ? b : b ^ 0x7fffffffffffffffll;
+}
+__device__ __forceinline__ double okey_inv(long long k) {
+    return __longlong_as_double(k >= 0 ? k : k ^ 0x7fffffffffffffffll);
 }
 
-__device__ __forceinline__ ArgBest warp_best(ArgBest a, double sign) {
+struct Cand {
+    long long k;      // key to maximise; kNone for "no candidate"
+    int i;            // index; ties go to the lower one
+};
+constexpr long long kNone = (long long)0x8000000000000000ull;   // below every finite key
+
+// Branch-free: b replaces a when its key is larger, or equal with a lower index.
+__device__ __forceinline__ Cand pick(Cand a, Cand b) {
+    const bool take = (b.k > a.k) | ((b.k == a.k) & (b.i < a.i));
+    return Cand{take ? b.k : a.k, take ? b.i : a.i};
+}
+
+template <int kSteps>
+__device__ __forceinline__ Cand warp_pick(Cand a) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        ArgBest b;
-        b.v = __shfl_xor_sync(0xffffffffu, a.v, o);
+    for (int s = 0; s < kSteps; ++s) {
+        const int o = 1 << s;                   // butterfly over lane bits 0 .. kSteps-1
+        Cand b;
+        b.k = __shfl_xor_sync(0xffffffffu, a.k, o);
         b.i = __shfl_xor_sync(0xffffffffu, a.i, o);
-        a = better(a, b, sign);
+        a = pick(a, b);
     }
     return a;
 }
 
 // Simultaneous fictitious play: both play policy 0 first; then each plays the
 // first best response to the other's plays so far. u_row[i] = sum over plays
-// of A[i][j_s] and u_col[j] = sum of A[i_s][j] are fp64 sums in play order.
+// of A[i][j_s] and u_col[j] = sum of A[i_s][j] are fp64 sums in play order,
+// held in registers with the play counts (thread t owns rows and columns t,
+// t + blockDim, ...). One CTA barrier per play: every warp publishes its best
+// row and column into a buffer selected by the play's parity, and after the
+// barrier every warp reduces the published candidates itself, so all threads
+// know the next plays. The column player's argmin is the argmax of the
+// negated key.
+template <bool kOnChip>
 __global__ void __launch_bounds__(kFpThreads) fictitious_play_kernel(
     const double* __restrict__ P, int32_t n_games, int32_t m, int32_t n, int32_t stride,
     int64_t T, double* __restrict__ x_out, double* __restrict__ y_out,
-    double* __restrict__ bounds_out, int32_t on_chip) {
+    double* __restrict__ bounds_out) {
     extern __shared__ double sA[];              // [m][ld] when on chip
-    __shared__ ArgBest red[2][kFpThreads / 32];
-    __shared__ int play[2];
-    __shared__ long long cnt_row[kFpMaxDim], cnt_col[kFpMaxDim];
+    __shared__ Cand red[2][2][8];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nt = blockDim.x;
     const int ld = n | 1;                       // odd row stride: column reads hit distinct banks
 
     for (int g = blockIdx.x; g < n_games; g += gridDim.x) {
         const double* Pg = P + (int64_t)g * m * n * stride;
-        if (on_chip) {
-            for (int k = tid; k < m * n; k += kFpThreads) {
+        __syncthreads();                        // the previous game's readers are done
+        if (kOnChip) {
+            for (int k = tid; k < m * n; k += nt) {
                 const int i = k / n, j = k - i * n;
                 sA[i * ld + j] = Pg[(int64_t)k * stride];
             }
         }
-        for (int k = tid; k < kFpMaxDim; k += kFpThreads) { cnt_row[k] = 0; cnt_col[k] = 0; }
-        if (tid == 0) { play[0] = 0; play[1] = 0; }
+        if (tid < 32) {
+            const Cand none{kNone, 0x7fffffff};
+            (&red[0][0][0])[tid] = none;
+        }
         __syncthreads();
         auto a_at = [&](int i, int j) -> double {
-            return on_chip ? sA[i * ld + j] : __ldg(Pg + ((int64_t)i * n + j) * stride);
+            return kOnChip ? sA[i * ld + j] : __ldg(Pg + ((int64_t)i * n + j) * stride);
         };
         double ur[kFpPer], uc[kFpPer];
+        long long cr[kFpPer], cc[kFpPer];
 #pragma unroll
-        for (int k = 0; k < kFpPer; ++k) { ur[k] = 0.0; uc[k] = 0.0; }
-        ArgBest top{0.0, -1}, bot{0.0, -1};
+        for (int k = 0; k < kFpPer; ++k) { ur[k] = 0.0; uc[k] = 0.0; cr[k] = 0; cc[k] = 0; }
+        int it = 0, jt = 0;
+        Cand top{kNone, 0x7fffffff}, bot{kNone, 0x7fffffff};
         for (int64_t t = 0; t < T; ++t) {
-            const int it = play[0], jt = play[1];
-            if (tid == 0) { cnt_row[it] += 1; cnt_col[jt] += 1; }
-            ArgBest br{0.0, -1}, bc{0.0, -1};
+            const int par = (int)(t & 1);
+            Cand br{kNone, 0x7fffffff}, bc{kNone, 0x7fffffff};
 #pragma unroll
             for (int k = 0; k < kFpPer; ++k) {
-                const int i = tid + k * kFpThreads;
+                const int i = tid + k * nt;
                 if (i < m) {
+                    cr[k] += (i == it);
                     ur[k] += a_at(i, jt);
-                    br = better(br, ArgBest{ur[k], i}, 1.0);
+                    br = pick(br, Cand{okey(ur[k]), i});
                 }
                 if (i < n) {
+                    cc[k] += (i == jt);
                     uc[k] += a_at(it, i);
-                    bc = better(bc, ArgBest{uc[k], i}, -1.0);
+                    bc = pick(bc, Cand{-okey(uc[k]), i});
                 }
             }
-            br = warp_best(br, 1.0);
-            bc = warp_best(bc, -1.0);
-            if (lane == 0) { red[0][warp] = br; red[1][warp] = bc; }
-            __syncthreads();                    // also: every thread has read play[]
-            if (warp == 0) {
-                ArgBest r = lane < kFpThreads / 32 ? red[0][lane] : ArgBest{0.0, -1};
-                ArgBest c = lane < kFpThreads / 32 ? red[1][lane] : ArgBest{0.0, -1};
-                r = warp_best(r, 1.0);
-                c = warp_best(c, -1.0);
-                if (lane == 0) { play[0] = r.i; play[1] = c.i; top = r; bot = c; }
-            }
+            br = warp_pick<5>(br);
+            bc = warp_pick<5>(bc);
+            if (lane == 0) { red[par][0][warp] = br; red[par][1][warp] = bc; }
             __syncthreads();
+            // at most 8 published candidates (unused entries hold "none"); every
+            // group of 8 lanes holds all of them, reduced over lane bits 0..2
+            top = warp_pick<3>(red[par][0][lane & 7]);
+            bot = warp_pick<3>(red[par][1][lane & 7]);
+            it = top.i;
+            jt = bot.i;
         }
         const double Td = (double)T;
-        for (int i = tid; i < m; i += kFpThreads) x_out[(int64_t)g * m + i] = (double)cnt_row[i] / Td;
-        for (int j = tid; j < n; j += kFpThreads) y_out[(int64_t)g * n + j] = (double)cnt_col[j] / Td;
-        if (tid == 0) {
-            bounds_out[2 * g] = bot.v / Td;     // min_j (x^T A)_j
-            bounds_out[2 * g + 1] = top.v / Td; // max_i (A y)_i
+#pragma unroll
+        for (int k = 0; k < kFpPer; ++k) {
+            const int i = tid + k * nt;
+            if (i < m) x_out[(int64_t)g * m + i] = (double)cr[k] / Td;
+            if (i < n) y_out[(int64_t)g * n + i] = (double)cc[k] / Td;
         }
-        __syncthreads();
+        if (tid == 0) {
+            bounds_out[2 * g] = okey_inv(-bot.k) / Td;     // min_j (x^T A)_j
+            bounds_out[2 * g + 1] = okey_inv(top.k) / Td;  // max_i (A y)_i
+        }
     }
 }
 
@@ -160,11 +185,26 @@ __global__ void __launch_bounds__(256) aggregate_kernel(
 // column player's problem max sum(q) s.t. B q <= 1, q >= 0 has optimum
 // 1 / v_B; y = q v_B, and the row player's x = p v_B from the duals p (the
 // objective row under the slack columns). v_A = v_B + min(A) - 1.
-// Tableau rows 0..m-1: [B | I | 1]; row m: [-1 ... -1 | 0 | 0]. Bland's rule
-// (lowest entering index with a negative reduced cost; lowest basic index on
-// ratio ties) guarantees termination; a pivot limit guards regardless.
+// Tableau rows 0..m-1: [B | I | 1]; row m: [-1 ... -1 | 0 | 0].
+// Entering column: the most negative reduced cost (Dantzig); after 2 (m + n)
+// consecutive degenerate pivots the rule switches for good to Bland's (lowest
+// index with a negative reduced cost), which cannot cycle. Leaving row: the
+// minimum ratio, ties to the lowest basic variable index. A pivot limit
+// guards regardless. Comparisons run on the integer keys above; the tableau
+// arithmetic is fp64.
 // ---------------------------------------------------------------------------
 constexpr int kLpThreads = 512;
+constexpr int kLpWarps = kLpThreads / 32;
+
+// Reduction of one candidate per thread to the CTA's best (all threads get it).
+__device__ __forceinline__ Cand cta_pick(Cand c, Cand* red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    c = warp_pick<5>(c);
+    __syncthreads();                             // red's previous readers are done
+    if (lane == 0) red[warp] = c;
+    __syncthreads();
+    return warp_pick<4>(red[lane & 15]);
+}
 
 __global__ void __launch_bounds__(kLpThreads) lp_nash_kernel(
     const double* __restrict__ P, int32_t n_games, int32_t m, int32_t n, int32_t stride,
@@ -173,29 +213,22 @@ __global__ void __launch_bounds__(kLpThreads) lp_nash_kernel(
     extern __shared__ double smem_tab[];
     __shared__ double colq[1024 + 1];
     __shared__ int basis[1024];
-    __shared__ ArgBest red[kLpThreads / 32];
-    __shared__ int enter_s, leave_s;
-    __shared__ double amin_s;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    __shared__ Cand red[kLpWarps];
+    const int tid = threadIdx.x;
     const int W = n + m + 1;                     // tableau width; column W-1 is the right side
     const int H = m + 1;                         // rows; row m is the objective
+    const Cand none{kNone, 0x7fffffff};
+    const double eps = 1e-12;
+    const long long k_neg_eps = okey(-eps);
 
     for (int g = blockIdx.x; g < n_games; g += gridDim.x) {
         double* Tb = on_chip ? smem_tab : gscratch + (int64_t)blockIdx.x * H * W;
         const double* Pg = P + (int64_t)g * m * n * stride;
-        // min(A)
-        ArgBest lo{0.0, -1};
-        for (int k = tid; k < m * n; k += kLpThreads) lo = better(lo, ArgBest{Pg[(int64_t)k * stride], k}, -1.0);
-        lo = warp_best(lo, -1.0);
-        if (lane == 0) red[warp] = lo;
-        __syncthreads();
-        if (warp == 0) {
-            ArgBest r = lane < kLpThreads / 32 ? red[lane] : ArgBest{0.0, -1};
-            r = warp_best(r, -1.0);
-            if (lane == 0) amin_s = r.v;
-        }
-        __syncthreads();
-        const double shift = 1.0 - amin_s;
+        Cand lo = none;                          // min(A): the largest negated key
+        for (int k = tid; k < m * n; k += kLpThreads)
+            lo = pick(lo, Cand{-okey(Pg[(int64_t)k * stride]), k});
+        lo = cta_pick(lo, red);
+        const double shift = 1.0 - okey_inv(-lo.k);
         for (int k = tid; k < H * W; k += kLpThreads) {
             const int r = k / W, c = k - r * W;
             double v;
@@ -212,65 +245,33 @@ __global__ void __launch_bounds__(kLpThreads) lp_nash_kernel(
         __syncthreads();
 
         const int max_pivots = 50 * (m + n) + 1000;
-        bool done = false;
+        bool done = false, bland = false;
+        int degenerate = 0;
         for (int piv = 0; piv < max_pivots; ++piv) {
-            // entering column: lowest index with a negative reduced cost
-            const double eps = 1e-12;
-            int ent = 0x7fffffff;
-            for (int c = tid; c < n + m; c += kLpThreads)
-                if (Tb[(int64_t)m * W + c] < -eps) { ent = c; break; }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) ent = min(ent, __shfl_xor_sync(0xffffffffu, ent, o));
-            if (lane == 0) red[warp].i = ent;
-            __syncthreads();
-            if (tid == 0) {
-                int e = 0x7fffffff;
-                for (int w = 0; w < kLpThreads / 32; ++w) e = min(e, red[w].i);
-                enter_s = e;
+            // entering column
+            Cand ce = none;
+            for (int c = tid; c < n + m; c += kLpThreads) {
+                const long long k = okey(Tb[(int64_t)m * W + c]);
+                if (k < k_neg_eps) ce = pick(ce, Cand{bland ? 0ll : -k, c});
             }
-            __syncthreads();
-            const int q = enter_s;
-            if (q == 0x7fffffff) { done = true; break; }
-            // ratio test over rows with a positive pivot-column entry; ties to
-            // the lowest basic variable index
-            ArgBest best{0.0, -1};
-            int best_basis = 0x7fffffff;
+            ce = cta_pick(ce, red);
+            if (ce.k == kNone) { done = true; break; }
+            const int q = ce.i;
+            // leaving row: minimum ratio (ratios are >= 0), ties to the lowest
+            // basic index; the candidate index packs (basic index, row)
+            Cand cl = none;
             for (int r = tid; r < m; r += kLpThreads) {
                 const double a = Tb[(int64_t)r * W + q];
                 if (a > eps) {
                     const double ratio = Tb[(int64_t)r * W + W - 1] / a;
-                    if (best.i < 0 || ratio < best.v || (ratio == best.v && basis[r] < best_basis)) {
-                        best = ArgBest{ratio, r};
-                        best_basis = basis[r];
-                    }
+                    cl = pick(cl, Cand{-okey(ratio), basis[r] * 1024 + r});
                 }
             }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const double ov = __shfl_xor_sync(0xffffffffu, best.v, o);
-                const int oi = __shfl_xor_sync(0xffffffffu, best.i, o);
-                const int ob = __shfl_xor_sync(0xffffffffu, best_basis, o);
-                if (oi >= 0 && (best.i < 0 || ov < best.v || (ov == best.v && ob < best_basis))) {
-                    best = ArgBest{ov, oi};
-                    best_basis = ob;
-                }
-            }
-            if (lane == 0) red[warp] = best;
-            __syncthreads();
-            if (tid == 0) {
-                ArgBest b{0.0, -1};
-                int bb = 0x7fffffff;
-                for (int w = 0; w < kLpThreads / 32; ++w) {
-                    const ArgBest o = red[w];
-                    if (o.i < 0) continue;
-                    const int ob = basis[o.i];
-                    if (b.i < 0 || o.v < b.v || (o.v == b.v && ob < bb)) { b = o; bb = ob; }
-                }
-                leave_s = b.i;                   // -1: unbounded (cannot happen with B > 0)
-            }
-            __syncthreads();
-            const int p = leave_s;
-            if (p < 0) break;
+            cl = cta_pick(cl, red);
+            if (cl.k == kNone) break;            // unbounded: cannot happen with B > 0
+            const int p = cl.i & 1023;
+            degenerate = (okey_inv(-cl.k) == 0.0) ? degenerate + 1 : 0;
+            if (degenerate > 2 * (m + n)) bland = true;
             // pivot on (p, q)
             for (int r = tid; r < H; r += kLpThreads) colq[r] = Tb[(int64_t)r * W + q];
             __syncthreads();
@@ -310,13 +311,16 @@ cudaError_t launch_fictitious_play(const double* P, int32_t G, int32_t m, int32_
                                    cudaStream_t s) {
     const int ld = n | 1;
     const int64_t bytes = (int64_t)m * ld * 8;
-    const int on_chip = bytes <= kSmemLimit ? 1 : 0;
+    const bool on_chip = bytes <= kSmemLimit;
     const size_t dyn = on_chip ? (size_t)bytes : 0;
-    cudaError_t e = cudaFuncSetAttribute(fictitious_play_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    // one thread per row and column up to 256 of them (fewer warps, cheaper
+    // barriers), else 256 threads with up to kFpPer rows / columns each
+    const int mx = m > n ? m : n;
+    const int threads = mx <= kFpThreads ? ((mx + 31) / 32) * 32 : kFpThreads;
+    auto kern = on_chip ? fictitious_play_kernel<true> : fictitious_play_kernel<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
     if (e != cudaSuccess) return e;
-    fictitious_play_kernel<<<fp_grid(G, n_sm), kFpThreads, dyn, s>>>(P, G, m, n, stride, T, x, y,
-                                                                    bounds, on_chip);
+    kern<<<fp_grid(G, n_sm), threads, dyn, s>>>(P, G, m, n, stride, T, x, y, bounds);
     return cudaGetLastError();
 }
 
