@@ -280,6 +280,21 @@ int malib_meta_aggregate(malib_ctx* ctx, const double* payoff, int32_t n_games, 
                          int32_t n, int32_t stride, const double* x, const double* y,
                          double* row_payoff_out, double* col_payoff_out, double* value_out);
 
+/* Exploitability of a pair of seat mixtures (Sec. 4.2: PSRO's convergence is
+ * measured by exploitability). ids0 [n0] are seat-0 policy ids of the loaded
+ * population with weights x [n0], ids1 [n1] seat-1 ids with weights y [n1]
+ * (fp64; normally each sums to 1, e.g. a fictitious-play or LP mixture).
+ * out [3] = {b0, b1, (b0 + b1) / 2}: b0 is the best seat-0 strategy's expected
+ * payoff against the seat-1 mixture, b1 the best seat-1 strategy's against the
+ * seat-0 mixture; a best responder sees its card, the public card once dealt
+ * and the betting history. Kuhn (tabular) and Leduc (MLP 17-h1-h2-3 fp32 with
+ * h <= 256, or bf16 17-256-256-3) populations; 1 <= n0, n1 <= 256. Policy
+ * action probabilities: the fp64 softmax, over legal actions, of the logits of
+ * the policy's forward (fp32 FMA; bf16 operands for bf16 policies).
+ * Arguments may be host or device memory; the call waits for the result. */
+int malib_exploitability(malib_ctx* ctx, const int32_t* ids0, const double* x, int32_t n0,
+                         const int32_t* ids1, const double* y, int32_t n1, double* out);
+
 /* ---- measurement and self-test entry points (used by tests and the benchmark) ---- */
 
 /* Total decisions (env-steps: one decision by the acting seat) played by the

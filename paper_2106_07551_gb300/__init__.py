@@ -256,6 +256,18 @@ class Context:
                                              _ptr(y), _ptr(row_out), _ptr(col_out),
                                              _ptr(value_out)))
 
+    def exploitability(self, ids0, x, ids1, y):
+        """(b0, b1, exploitability) of the seat mixtures (ids with fp64 weights)."""
+        ids0 = np.ascontiguousarray(ids0, np.int32)
+        ids1 = np.ascontiguousarray(ids1, np.int32)
+        x = np.ascontiguousarray(x, np.float64)
+        y = np.ascontiguousarray(y, np.float64)
+        out = np.zeros(3, np.float64)
+        _check(self.lib, self.handle,
+               self.lib.malib_exploitability(self.handle, _ptr(ids0), _ptr(x), len(ids0),
+                                             _ptr(ids1), _ptr(y), len(ids1), _ptr(out)))
+        return float(out[0]), float(out[1]), float(out[2])
+
     def selftest_philox(self, ctr, seed, out):
         _check(self.lib, self.handle,
                self.lib.malib_selftest_philox(self.handle, _ptr(ctr), seed, _ptr(out),

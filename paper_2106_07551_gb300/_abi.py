@@ -29,7 +29,7 @@ EXPORTS = (
     "malib_set_timing", "malib_main_kernel_ms",
     "malib_selftest_philox", "malib_selftest_det_expf", "malib_selftest_sample",
     "malib_selftest_mma", "malib_meta_fictitious_play", "malib_meta_lp_nash",
-    "malib_meta_aggregate",
+    "malib_meta_aggregate", "malib_exploitability",
 )
 
 
@@ -94,6 +94,7 @@ def load(path: str | None = None):
             "malib_meta_fictitious_play": (C.c_int, [P, P, i32, i32, i32, i32, i64, P, P, P]),
             "malib_meta_lp_nash": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P]),
             "malib_meta_aggregate": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P, P, P]),
+            "malib_exploitability": (C.c_int, [P, P, P, i32, P, P, i32, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)

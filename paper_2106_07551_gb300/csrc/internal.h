@@ -123,6 +123,7 @@ struct CtxView {
     int32_t n_pol;
     int* err;
     bool tables_uploaded;
+    bool tc_layout;               // bf16 tensor-core images in the arena (else fp32 layouts)
 };
 bool ctx_view(const void* ctx, CtxView* v);
 int ctx_fail(void* ctx, int code, const char* msg);

@@ -339,6 +339,7 @@ bool ctx_view(const void* ctx, CtxView* v) {
     v->n_pol = (int32_t)c->pols.size();
     v->err = c->d_err;
     v->tables_uploaded = !c->tables_dirty;
+    v->tc_layout = c->tc_layout;
     return true;
 }
 
