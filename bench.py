@@ -498,8 +498,25 @@ def run_meta(args):
     ctx.sync()
     lp_ms = e0.elapsed_time(e1)
 
+    # exploitability of uniform mixtures over the whole Leduc 64 x 64 bf16 population
+    import workloads
+    from paper_2106_07551_gb300 import make_spec, policy_desc
+    w5 = workloads.config(5, n_episodes=16)
+    spec5 = make_spec(w5.env_kind, w5.n_agents, w5.obs_dim, w5.n_actions)
+    ctx.pop_load(spec5, [policy_desc(p.kind, p.dtype, p.seat, p.dims, p.params) for p in w5.policies])
+    ids0 = [i for i, p in enumerate(w5.policies) if p.seat == 0]
+    ids1 = [i for i, p in enumerate(w5.policies) if p.seat == 1]
+    ux, uy = np.full(len(ids0), 1.0 / len(ids0)), np.full(len(ids1), 1.0 / len(ids1))
+    expl = ctx.exploitability(ids0, ux, ids1, uy)
+    reps = 20
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        expl = ctx.exploitability(ids0, ux, ids1, uy)
+    expl_ms = (time.perf_counter() - t0) / reps * 1e3
+
     e2e = None
     cpu = None
+    expl_cpu_s = None
     if rank == 0:
         # e2e: tables from pinned host memory, mixtures and bounds back
         h_tab = torch.from_numpy(tables).pin_memory()
@@ -533,6 +550,12 @@ def run_meta(args):
                 n_games += 1
             cpu = {"value": n_games * T / t_cpu, "unit": "plays/s", "cores": 1, "kind": "oracle",
                    "sample": f"{n_games} of the {G} games, {T} plays each ({t_cpu:.1f} s, numpy)"}
+            from oracle import exploit as ex
+            P5 = [p.params for p in w5.policies]
+            t_ex = time.perf_counter()
+            ex.leduc_exploitability([P5[i] for i in ids0], ux, [P5[i] for i in ids1], uy,
+                                    w5.policies[0].dims, True)
+            expl_cpu_s = time.perf_counter() - t_ex
     clk = clocks.summary()
     ctx.close()
     if rank == 0:
@@ -549,7 +572,11 @@ def run_meta(args):
                              "kernel": "fictitious_play_kernel",
                              "note": "each play depends on the previous play's argmax: one CTA "
                                      "barrier and two warp reductions per play bound it"},
-                "lp_nash_ms": lp_ms, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+                "lp_nash_ms": lp_ms,
+                "exploitability": {"workload": "leduc 64x64 bf16 population, uniform mixtures",
+                                   "value": expl[2], "ms_per_call": expl_ms,
+                                   "oracle_s": expl_cpu_s},
+                "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
                 "gpu_launches": launches}
         print(json.dumps(line), flush=True)
     if world > 1:
