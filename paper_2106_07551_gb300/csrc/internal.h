@@ -4,6 +4,8 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include "malib.h"
+
 namespace malib {
 
 constexpr int kMaxAgents = 16;
@@ -42,6 +44,11 @@ struct F32Layout {
 inline bool tc_image_shape(const int* d) {
     return d[1] == 256 && d[2] == 256 && d[0] >= 1 && d[0] <= 48 && d[3] >= 1 && d[3] <= 16;
 }
+// Leduc's observation feature 15 (call/check legal) is 1 in every state: the
+// Leduc tensor-core image folds its weight column into b1 and drops the
+// feature, leaving 16 inputs (one bf16 K step).
+constexpr int kLeducConstFeature = 15;
+inline bool leduc_tc_fold(int env_kind, int in) { return env_kind == MALIB_ENV_LEDUC && in == 17; }
 inline int64_t tc_image_bytes(int in) {
     const int64_t k1 = (in + 15) / 16 * 16;
     return 256 * k1 * 2 + 256 * 256 * 2 + 16 * 256 * 2 + (256 + 256 + 16) * 4;

@@ -28,7 +28,10 @@ namespace malib {
 
 // kSmemBias: stage the biases with the weights (true) or read them from the
 // policy's global image through L1 (false, when shared memory is short).
-template <int K1, int H, int NOUT, bool kSmemBias = true>
+// kBarId: 0 - the whole CTA runs the engine (CTA barriers); otherwise the
+// engine runs on warps 0-7 alone and synchronises them with named barrier
+// kBarId (256 threads), leaving the CTA's other warps free for other work.
+template <int K1, int H, int NOUT, bool kSmemBias = true, int kBarId = 0>
 struct MlpTc {
     static_assert(K1 % 16 == 0 && H == 256 && NOUT == 16, "shapes built: K1 % 16, H 256, NOUT 16");
     static constexpr uint32_t kW1 = 0;
@@ -69,58 +72,74 @@ struct MlpTc {
                          tc::smem_desc(w + 2u * s * lbo_w, lbo_w, 128), idesc, !(fresh && s == s0));
     }
 
-    // Columns [c_begin, c_begin + 128) of a layer's output: D (TMEM column
-    // tcol + c) + bias -> relu -> bf16 into the activation tile. Warp w takes
-    // TMEM lane quarter w % 4 and columns c_begin + 64 (w / 4) .. +63 in two
-    // 32-column chunks; the second chunk's tensor-memory and bias loads are in
-    // flight while the first is processed.
-    __device__ static void epilogue_half(uint8_t* act, const float* bias, uint32_t tbase,
-                                         int tcol, int c_begin) {
-        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-        const int q = warp & 3, h = warp >> 2;
-        const int row = 32 * q + lane;
-        uint32_t r[2][32];
-        float4 bs[2][8];
-        auto load_bias = [&](int buf, int c0) {
+    // One 32-column chunk of a layer's output for this thread's row: D (already
+    // in registers) + bias -> relu -> bf16, stored into the activation tile.
+    __device__ static void store_chunk(uint8_t* act, const float* bias, int row, int c0,
+                                       const uint32_t (&v)[32]) {
+        float4 bs[8];
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-                bs[buf][j] = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
-                                       : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
-        };
-        const int cb = c_begin + 64 * h;
-        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb), r[0]);
-        load_bias(0, cb);
-        tc::tmem_wait_ld();
+        for (int j = 0; j < 8; ++j)
+            bs[j] = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
+                              : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
 #pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-            const int c0 = cb + cc * 32;
-            if (cc == 0) {
-                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + c0 + 32), r[1]);
-                load_bias(1, c0 + 32);
-            }
-            const uint32_t* v = r[cc];
-            const float4* b = bs[cc];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const float4 b0 = b[2 * j], b1 = b[2 * j + 1];
-                auto f = [&](int i) { return __uint_as_float(v[8 * j + i]); };
-                uint4 pk;
-                pk.x = tc::bias_relu_bf16x2(f(0), f(1), b0.x, b0.y);
-                pk.y = tc::bias_relu_bf16x2(f(2), f(3), b0.z, b0.w);
-                pk.z = tc::bias_relu_bf16x2(f(4), f(5), b1.x, b1.y);
-                pk.w = tc::bias_relu_bf16x2(f(6), f(7), b1.z, b1.w);
-                *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
-            }
-            if (cc == 0) tc::tmem_wait_ld();
+        for (int j = 0; j < 4; ++j) {
+            const float4 b0 = bs[2 * j], b1 = bs[2 * j + 1];
+            auto f = [&](int i) { return __uint_as_float(v[8 * j + i]); };
+            uint4 pk;
+            pk.x = tc::bias_relu_bf16x2(f(0), f(1), b0.x, b0.y);
+            pk.y = tc::bias_relu_bf16x2(f(2), f(3), b0.z, b0.w);
+            pk.z = tc::bias_relu_bf16x2(f(4), f(5), b1.x, b1.y);
+            pk.w = tc::bias_relu_bf16x2(f(6), f(7), b1.z, b1.w);
+            *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
         }
     }
 
-    // Makes this CTA's generic shared-memory writes visible to the tensor cores
-    // and orders tensor-memory reads before the next MMA (all threads call).
+    // A layer's output, D (TMEM columns tcol ..) + bias -> relu -> bf16 into the
+    // activation tile, in two column halves. Warp w takes TMEM lane quarter
+    // w % 4 and, in each half, the 64 columns 64 (w / 4) .. of that half. The
+    // first half is stored, then the second half's tensor-memory loads are
+    // issued and stay in flight across mid() (the hand-off that lets the next
+    // layer's MMAs start on the first half).
+    template <class Mid>
+    __device__ static void epilogue_layer(uint8_t* act, const float* bias, uint32_t tbase,
+                                          int tcol, Mid mid) {
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+        const int q = warp & 3, h = warp >> 2;
+        const int row = 32 * q + lane;
+        const int ca = 64 * h, cb = H / 2 + 64 * h;
+        {
+            uint32_t r0[32], r1[32];
+            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + ca), r0);
+            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + ca + 32), r1);
+            tc::tmem_wait_ld();
+            store_chunk(act, bias, row, ca, r0);
+            store_chunk(act, bias, row, ca + 32, r1);
+        }
+        uint32_t r2[32], r3[32];
+        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb), r2);
+        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb + 32), r3);
+        mid();
+        tc::tmem_wait_ld();
+        store_chunk(act, bias, row, cb, r2);
+        store_chunk(act, bias, row, cb + 32, r3);
+    }
+
+    // Barrier over the engine's threads.
+    __device__ static void sync() {
+        if (kBarId == 0) {
+            __syncthreads();
+        } else {
+            asm volatile("bar.sync %0, 256;" ::"n"(kBarId) : "memory");
+        }
+    }
+
+    // Makes the engine's generic shared-memory writes visible to the tensor
+    // cores and orders tensor-memory reads before the next MMA (all engine
+    // threads call).
     __device__ static void handoff() {
         fence_proxy_async_smem();
         tc::fence_before_sync();
-        __syncthreads();
+        sync();
         tc::fence_after_sync();
     }
 
@@ -131,9 +150,12 @@ struct MlpTc {
     // when kSmemBias is false). All threads call.
     // x_published: the caller's X writers already fenced (proxy) and the CTA
     // has synchronised since (e.g. a cluster sync), so MMA 1 issues at once.
+    // x_tile: shared-memory address of the observation tile [128][K1] (same
+    // core-matrix layout as the activation tile); 0 = the activation tile's start.
     template <class Out>
     __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bar,
-                                   uint32_t& parity, int* err, Out out, bool x_published = false) {
+                                   uint32_t& parity, int* err, Out out, bool x_published = false,
+                                   uint32_t x_tile = 0) {
         uint8_t* act = smem + kAct;
         const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
         const uint32_t s_act = smem_u32(act);
@@ -151,16 +173,16 @@ struct MlpTc {
         constexpr int kS = H / 16;                      // K steps of layers 2 and 3
         // layer 1 (N = 256, K = K1) into D1
         if (threadIdx.x == 0) {
-            issue(d1, s_act, s_w1, kLboW, 0, K1 / 16, idesc_full, true);
+            issue(d1, x_tile ? x_tile : s_act, s_w1, kLboW, 0, K1 / 16, idesc_full, true);
             tc::mma_commit(bar);
         }
         wait_mma(bar, parity, err);
         // h1 columns 0..127, then layer-2 K steps 0..7 (N = 256) while h1
         // columns 128..255 are produced, then K steps 8..15
-        epilogue_half(act, bias, tbase, 0, 0);
-        handoff();
-        if (threadIdx.x == 0) issue(d2, s_act, s_w2, kLboW, 0, kS / 2, idesc_full, true);
-        epilogue_half(act, bias, tbase, 0, H / 2);
+        epilogue_layer(act, bias, tbase, 0, [&] {
+            handoff();
+            if (threadIdx.x == 0) issue(d2, s_act, s_w2, kLboW, 0, kS / 2, idesc_full, true);
+        });
         handoff();
         if (threadIdx.x == 0) {
             issue(d2, s_act, s_w2, kLboW, kS / 2, kS, idesc_full, false);
@@ -170,22 +192,20 @@ struct MlpTc {
         // h2 columns 0..127, then layer-3 K steps 0..7 while h2 columns
         // 128..255 are produced. Layer 3 runs as 4 chains of 4 MMAs into TMEM
         // columns 16j (D1's columns, free once h1 is written).
-        epilogue_half(act, bias + H, tbase, 256, 0);
-        handoff();
-        if (threadIdx.x == 0)
-            for (int s = 0; s < kS / 2; ++s)
+        auto mma3 = [&](int s0, int s1) {
+            for (int s = s0; s < s1; ++s)
                 tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))),
                              tc::smem_desc(s_act + 2u * s * kLboAct, kLboAct, 128),
                              tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
                              (s % (kS / 4)) != 0);
-        epilogue_half(act, bias + H, tbase, 256, H / 2);
+        };
+        epilogue_layer(act, bias + H, tbase, 256, [&] {
+            handoff();
+            if (threadIdx.x == 0) mma3(0, kS / 2);
+        });
         handoff();
         if (threadIdx.x == 0) {
-            for (int s = kS / 2; s < kS; ++s)
-                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))),
-                             tc::smem_desc(s_act + 2u * s * kLboAct, kLboAct, 128),
-                             tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
-                             (s % (kS / 4)) != 0);
+            mma3(kS / 2, kS);
             tc::mma_commit(bar);
         }
         wait_mma(bar, parity, err);
@@ -208,7 +228,7 @@ struct MlpTc {
             out(row, v);
         }
         tc::fence_before_sync();
-        __syncthreads();
+        sync();
     }
 };
 

@@ -192,9 +192,15 @@ void to_f32_layout(const float* p, const int* d, float* out, int64_t size) {
 }
 
 // bf16 tensor-core image (internal.h) from the plain fp32 layout.
-void to_tc_image(const float* p, const int* d, float* out_floats) {
+// bf16 tensor-core image of one MLP (layout: tc_image_bytes). fold: the Leduc
+// image, whose observation feature 15 (call/check is legal) is 1 in every
+// state, so its W1 column is added to b1 (as the bf16 weight the product
+// would use) and the remaining 16 features fill one K step of 16: slot s holds
+// feature s for s < 15 and feature 16 in slot 15.
+void to_tc_image(const float* p, const int* d, float* out_floats, bool fold) {
     const int in = d[0], H = 256, A = d[3];
-    const int k1 = (in + 15) / 16 * 16;
+    const int in_img = fold ? in - 1 : in;
+    const int k1 = (in_img + 15) / 16 * 16;
     const float* W1 = p;
     const float* b1 = W1 + (int64_t)H * in;
     const float* W2 = b1 + H;
@@ -202,13 +208,19 @@ void to_tc_image(const float* p, const int* d, float* out_floats) {
     const float* W3 = b2 + H;
     const float* b3 = W3 + (int64_t)A * H;
     uint8_t* img = reinterpret_cast<uint8_t*>(out_floats);
-    const int64_t bytes = tc_image_bytes(in);
+    const int64_t bytes = tc_image_bytes(in_img);
     std::memset(img, 0, (size_t)bytes);
     auto bf = [](float x) -> uint16_t {
         uint32_t b;
         std::memcpy(&b, &x, 4);
         if ((b & 0x7F800000u) != 0x7F800000u) b += 0x7FFFu + ((b >> 16) & 1u);
         return (uint16_t)(b >> 16);
+    };
+    auto bf_value = [&](float x) -> float {
+        const uint32_t b = (uint32_t)bf(x) << 16;
+        float v;
+        std::memcpy(&v, &b, 4);
+        return v;
     };
     auto put = [&](uint8_t* base, int row, int k, int rows, float v) {
         const uint16_t h = bf(v);
@@ -219,12 +231,18 @@ void to_tc_image(const float* p, const int* d, float* out_floats) {
     uint8_t* w3 = w2 + (int64_t)H * H * 2;
     float* bias = reinterpret_cast<float*>(w3 + 16 * H * 2);
     for (int n = 0; n < H; ++n)
-        for (int k = 0; k < in; ++k) put(w1, n, k, H, W1[(int64_t)n * in + k]);
+        for (int s = 0; s < in_img; ++s) {
+            const int f = fold && s >= kLeducConstFeature ? s + 1 : s;
+            put(w1, n, s, H, W1[(int64_t)n * in + f]);
+        }
     for (int n = 0; n < H; ++n)
         for (int k = 0; k < H; ++k) put(w2, n, k, H, W2[(int64_t)n * H + k]);
     for (int n = 0; n < A; ++n)
         for (int k = 0; k < H; ++k) put(w3, n, k, 16, W3[(int64_t)n * H + k]);
-    for (int j = 0; j < H; ++j) { bias[j] = b1[j]; bias[H + j] = b2[j]; }
+    for (int j = 0; j < H; ++j) {
+        bias[j] = fold ? b1[j] + bf_value(W1[(int64_t)j * in + kLeducConstFeature]) : b1[j];
+        bias[H + j] = b2[j];
+    }
     for (int j = 0; j < A; ++j) bias[2 * H + j] = b3[j];
 }
 
@@ -499,8 +517,9 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
                                   (int64_t)d.dims[1] * d.dims[2] + d.dims[2] +
                                   (int64_t)d.dims[3] * d.dims[2] + d.dims[3] + 3) / 4 * 4;
             if (d.dtype == MALIB_BF16 && tc_image_shape(d.dims)) {
-                converted[i].assign((size_t)(tc_image_bytes(d.dims[0]) / 4), 0.f);
-                to_tc_image(plain.data(), d.dims, converted[i].data());
+                const bool fold = leduc_tc_fold(spec->env_kind, d.dims[0]);
+                converted[i].assign((size_t)(tc_image_bytes(fold ? d.dims[0] - 1 : d.dims[0]) / 4), 0.f);
+                to_tc_image(plain.data(), d.dims, converted[i].data(), fold);
                 recs[i] = rec;
                 continue;
             }
