@@ -224,7 +224,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 float ob[17];
                 float u = 0.f;
                 if (placed) {
-                    u = u24(draw(gid, (uint32_t)t, (uint32_t)seat, a.seed).x);
                     leduc_obs(h, ob);
                     uint32_t w[8];
 #pragma unroll
@@ -255,6 +254,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                     make_uint4(n, (uint32_t)(c0 + c1), 0, 0),
                                     cl::map(&x_bar[g], (uint32_t)lt));
                 }
+                // the decision's uniform, drawn while the engines work
+                if (placed) u = u24(draw(gid, (uint32_t)t, (uint32_t)seat, a.seed).x);
                 // logits (or the end of the segment) from both engines
                 if (lt == 0) {
                     if (!dead_s && !cl::wait_cluster_bounded(&lg_bar[g], lg_par, kWaitLimitNs)) {
