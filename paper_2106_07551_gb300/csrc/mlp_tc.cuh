@@ -12,11 +12,15 @@
 // layer's output, so X, h1 and h2 reuse the same 64 KB. Tensor memory holds
 // two 256-column accumulators: layer 1 writes D1 (columns 0..255), layer 2 D2
 // (256..511), layer 3 four 16-column partial sums over D1's first 64 columns.
-// Thread 0 issues the MMAs; the 8 warps split each epilogue (warp w: TMEM lane
-// quarter w % 4, 64 of the 128 columns of a half). Each layer's epilogue runs
-// in two column halves, and the next layer's MMAs over the first half's K
-// range are issued before the second half is produced, so the tensor core
-// works while the epilogue warps drain tensor memory.
+// D1 and D2 start each forward holding their layer's bias (written with
+// tcgen05.st while other work waits: b2 during layer 1's MMA, b1 after the
+// previous forward), so the MMAs accumulate onto it and the epilogues only
+// apply ReLU and bf16 rounding. Thread 0 issues the MMAs; the 8 warps split
+// each epilogue (warp w: TMEM lane quarter w % 4, 64 of the 128 columns of a
+// half). Each layer's epilogue runs in two column halves, and the next layer's
+// MMAs over the first half's K range are issued before the second half is
+// produced, so the tensor core works while the epilogue warps drain tensor
+// memory.
 #pragma once
 
 #include <cstdint>
@@ -73,36 +77,59 @@ struct MlpTc {
     }
 
     // One 32-column chunk of a layer's output for this thread's row: D (already
-    // in registers) + bias -> relu -> bf16, stored into the activation tile.
-    __device__ static void store_chunk(uint8_t* act, const float* bias, int row, int c0,
-                                       const uint32_t (&v)[32]) {
-        float4 bs[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-            bs[j] = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
-                              : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
+    // in registers, bias included) -> relu -> bf16, stored into the activation tile.
+    __device__ static void store_chunk(uint8_t* act, int row, int c0, const uint32_t (&v)[32]) {
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            const float4 b0 = bs[2 * j], b1 = bs[2 * j + 1];
             auto f = [&](int i) { return __uint_as_float(v[8 * j + i]); };
             uint4 pk;
-            pk.x = tc::bias_relu_bf16x2(f(0), f(1), b0.x, b0.y);
-            pk.y = tc::bias_relu_bf16x2(f(2), f(3), b0.z, b0.w);
-            pk.z = tc::bias_relu_bf16x2(f(4), f(5), b1.x, b1.y);
-            pk.w = tc::bias_relu_bf16x2(f(6), f(7), b1.z, b1.w);
+            pk.x = tc::relu_bf16x2(f(0), f(1));
+            pk.y = tc::relu_bf16x2(f(2), f(3));
+            pk.z = tc::relu_bf16x2(f(4), f(5));
+            pk.w = tc::relu_bf16x2(f(6), f(7));
             *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
         }
     }
 
-    // A layer's output, D (TMEM columns tcol ..) + bias -> relu -> bf16 into the
-    // activation tile, in two column halves. Warp w takes TMEM lane quarter
+    // Writes a layer's bias (H values) into every row of the accumulator at TMEM
+    // column tcol, so the layer's MMAs accumulate onto it: warp w writes its lane
+    // quarter w % 4, columns 128 (w / 4) .. +127. Waits for its stores.
+    __device__ static void prefill(const float* bias, uint32_t tbase, int tcol) {
+        const int warp = threadIdx.x >> 5;
+        const int q = warp & 3, h = warp >> 2;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+            const int c0 = 128 * h + 32 * c;
+            uint32_t r[32];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float4 b = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
+                                           : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
+                r[4 * j] = __float_as_uint(b.x);
+                r[4 * j + 1] = __float_as_uint(b.y);
+                r[4 * j + 2] = __float_as_uint(b.z);
+                r[4 * j + 3] = __float_as_uint(b.w);
+            }
+            tc::tmem_st32(tc::tmem_addr(tbase, 32 * q, tcol + c0), r);
+        }
+        tc::tmem_wait_st();
+    }
+
+    // Layer 1's bias into D1 before the first forward of a policy (after its
+    // weights and biases are staged). The caller orders it before the next MMA
+    // (tcgen05 fence before a barrier of the engine's threads).
+    __device__ static void prefill_d1(uint8_t* smem, const float* gbias, uint32_t tbase) {
+        prefill(kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias, tbase, 0);
+    }
+
+    // A layer's output, D (TMEM columns tcol .., bias included) -> relu -> bf16
+    // into the activation tile, in two column halves. Warp w takes TMEM lane quarter
     // w % 4 and, in each half, the 64 columns 64 (w / 4) .. of that half. The
     // first half is stored, then the second half's tensor-memory loads are
     // issued and stay in flight across mid() (the hand-off that lets the next
     // layer's MMAs start on the first half).
     template <class Mid>
-    __device__ static void epilogue_layer(uint8_t* act, const float* bias, uint32_t tbase,
-                                          int tcol, Mid mid) {
+    __device__ static void epilogue_layer(uint8_t* act, uint32_t tbase, int tcol, Mid mid) {
         const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
         const int q = warp & 3, h = warp >> 2;
         const int row = 32 * q + lane;
@@ -112,16 +139,16 @@ struct MlpTc {
             tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + ca), r0);
             tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + ca + 32), r1);
             tc::tmem_wait_ld();
-            store_chunk(act, bias, row, ca, r0);
-            store_chunk(act, bias, row, ca + 32, r1);
+            store_chunk(act, row, ca, r0);
+            store_chunk(act, row, ca + 32, r1);
         }
         uint32_t r2[32], r3[32];
         tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb), r2);
         tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb + 32), r3);
         mid();
         tc::tmem_wait_ld();
-        store_chunk(act, bias, row, cb, r2);
-        store_chunk(act, bias, row, cb + 32, r3);
+        store_chunk(act, row, cb, r2);
+        store_chunk(act, row, cb + 32, r3);
     }
 
     // Barrier over the engine's threads.
@@ -171,17 +198,18 @@ struct MlpTc {
         const uint32_t idesc3 = tc::instr_desc(128, NOUT, 1);
         const uint32_t d1 = tbase, d2 = tbase + 256;
         constexpr int kS = H / 16;                      // K steps of layers 2 and 3
-        // layer 1 (N = 256, K = K1) into D1
+        // layer 1 (N = 256, K = K1) onto D1 (holding b1); meanwhile b2 goes into D2
         if (threadIdx.x == 0) {
-            issue(d1, x_tile ? x_tile : s_act, s_w1, kLboW, 0, K1 / 16, idesc_full, true);
+            issue(d1, x_tile ? x_tile : s_act, s_w1, kLboW, 0, K1 / 16, idesc_full, false);
             tc::mma_commit(bar);
         }
+        prefill(bias + H, tbase, 256);
         wait_mma(bar, parity, err);
         // h1 columns 0..127, then layer-2 K steps 0..7 (N = 256) while h1
         // columns 128..255 are produced, then K steps 8..15
-        epilogue_layer(act, bias, tbase, 0, [&] {
+        epilogue_layer(act, tbase, 0, [&] {
             handoff();
-            if (threadIdx.x == 0) issue(d2, s_act, s_w2, kLboW, 0, kS / 2, idesc_full, true);
+            if (threadIdx.x == 0) issue(d2, s_act, s_w2, kLboW, 0, kS / 2, idesc_full, false);
         });
         handoff();
         if (threadIdx.x == 0) {
@@ -199,7 +227,7 @@ struct MlpTc {
                              tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
                              (s % (kS / 4)) != 0);
         };
-        epilogue_layer(act, bias + H, tbase, 256, [&] {
+        epilogue_layer(act, tbase, 256, [&] {
             handoff();
             if (threadIdx.x == 0) mma3(0, kS / 2);
         });
@@ -227,6 +255,9 @@ struct MlpTc {
             for (int i = 0; i < 16; ++i) v[i] += kSmemBias ? bias[2 * H + i] : __ldg(bias + 2 * H + i);
             out(row, v);
         }
+        // b1 into D1 for the next forward (each warp rewrites only columns of its
+        // own lane quarter, after its own reads of the layer-3 chains)
+        prefill(bias, tbase, 0);
         tc::fence_before_sync();
         sync();
     }
