@@ -259,15 +259,20 @@ struct MlpF32T8 {
             if (kk < kmax) {
                 const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(W + (k0 + kk) * H + c0);
                 const ulonglong2 wB = *reinterpret_cast<const ulonglong2*>(W + (k0 + kk) * H + c1);
+                // all 8 duplications first, then the packed FMAs column pair by
+                // column pair, so no FMA waits on the duplication just before it
+                u64 x2[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const float xv = kk == 0 ? xa[i].x : kk == 1 ? xa[i].y : kk == 2 ? xa[i].z : xa[i].w;
-                    const u64 x2 = f2_dup(xv);
-                    f2_fma(acc[i][0], x2, wA.x);
-                    f2_fma(acc[i][1], x2, wA.y);
-                    f2_fma(acc[i][2], x2, wB.x);
-                    f2_fma(acc[i][3], x2, wB.y);
-                }
+                for (int i = 0; i < 8; ++i)
+                    x2[i] = f2_dup(kk == 0 ? xa[i].x : kk == 1 ? xa[i].y : kk == 2 ? xa[i].z : xa[i].w);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][0], x2[i], wA.x);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][1], x2[i], wA.y);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][2], x2[i], wB.x);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][3], x2[i], wB.y);
             }
         }
     }
