@@ -60,12 +60,12 @@ def _L():
                 "orc_leduc_exact": (C.c_double, [P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int]),
                 "orc_leduc_eval": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, i32, i64,
                                           i64, u64, P, i64, P, P, P, P, P, P, P, P, C.c_int]),
-                "orc_spread_step": (None, [C.c_int, C.c_int, P, P, P]),
+                "orc_spread_step": (None, [C.c_int, C.c_int, P, P, P, C.c_float]),
                 "orc_spread_obs": (None, [C.c_int, C.c_int, P, C.c_int, P]),
                 "orc_spread_reset": (None, [C.c_int, C.c_int, u64, u64, P]),
                 "orc_spread_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                               C.c_int, C.c_int, C.c_int, i64, i64, i64, P, i32, i64,
-                                              u64, P, P, P, P, P, C.c_int]),
+                                              u64, P, P, P, P, P, C.c_int, C.c_float]),
             }
             for name, (res, args) in sig.items():
                 fn = getattr(lib, name)
@@ -206,11 +206,15 @@ def leduc_eval(params_list, dims, pairs, n_episodes, seed, bf16=False, n_rec=0,
 
 
 # ---------------------------------------------------------------- spread
-def spread_step(state: np.ndarray, N: int, L: int, actions) -> tuple[np.ndarray, np.ndarray]:
+def spread_step(state: np.ndarray, N: int, L: int, actions,
+                local_ratio=None) -> tuple[np.ndarray, np.ndarray]:
+    """One transition; local_ratio (None: the unweighted reward) weights the
+    shared cover term by 1 - local_ratio and the agent's collisions by it."""
     st = _c(state, np.float32).copy()
     act = _c(actions, np.int32)
     rew = np.zeros(N, np.float32)
-    _L().orc_spread_step(N, L, _p(st), _p(act), _p(rew))
+    _L().orc_spread_step(N, L, _p(st), _p(act), _p(rew),
+                         -1.0 if local_ratio is None else float(local_ratio))
     return st, rew
 
 
@@ -228,7 +232,7 @@ def spread_reset(N: int, L: int, g: int, seed: int) -> np.ndarray:
 
 
 def spread_rollout(params_list, dims, N, L, T, n_envs, pairs, n_episodes, seed, bf16=False,
-                   env_lo=0, env_hi=None, ext_logits=None, n_threads=0):
+                   env_lo=0, env_hi=None, ext_logits=None, n_threads=0, local_ratio=None):
     """Rollout over envs [env_lo, env_hi). Returns dict of obs [E][T][W][N][in],
     action int8 [E][T][W][N], reward [E][T][W][N], logits [E][T][W][N][A]."""
     env_hi = n_envs if env_hi is None else env_hi
@@ -244,6 +248,7 @@ def spread_rollout(params_list, dims, N, L, T, n_envs, pairs, n_episodes, seed, 
     _L().orc_spread_rollout(C.cast(tbl, C.c_void_p), i, h1, h2, A, int(bf16), N, L, T, n_envs,
                             env_lo, env_hi, _p(pairs), pairs.shape[0], n_episodes,
                             C.c_uint64(seed), _p(ext), _p(out["obs"]), _p(out["action"]),
-                            _p(out["reward"]), _p(out["logits"]), n_threads)
+                            _p(out["reward"]), _p(out["logits"]), n_threads,
+                            -1.0 if local_ratio is None else float(local_ratio))
     del arrs
     return out

@@ -526,7 +526,11 @@ float dist2d(float ax, float ay, float bx, float by) {
     return std::sqrt(sq);
 }
 
-void spread_step(Spread& s, const int* action, float* reward) {
+// local_ratio < 0: r_i = -(cover + collisions_i) (the workloads' reward);
+// otherwise the App. B.1 weighting of the shared and the local term:
+// r_i = -((1 - local_ratio) * cover + local_ratio * collisions_i), evaluated
+// as written (one rounding per operation, no contraction).
+void spread_step(Spread& s, const int* action, float* reward, float local_ratio) {
     for (int i = 0; i < s.N; ++i) {
         float fx = 0.0f, fy = 0.0f;
         switch (action[i]) {
@@ -558,7 +562,13 @@ void spread_step(Spread& s, const int* action, float* reward) {
             if (j == i) continue;
             if (dist2d(s.px[i], s.py[i], s.px[j], s.py[j]) < 0.3f) ++coll;
         }
-        reward[i] = -(cover + (float)coll);
+        if (local_ratio < 0.0f) {
+            reward[i] = -(cover + (float)coll);
+        } else {
+            const float shared = (1.0f - local_ratio) * cover;
+            const float local = local_ratio * (float)coll;
+            reward[i] = -(shared + local);
+        }
     }
 }
 
@@ -702,7 +712,8 @@ void orc_leduc_eval(const float* const* params, int in, int h1, int h2, int out,
 // ---- Spread ----
 // One transition from a given state (for hand-worked checks). state: px,py,vx,vy
 // for N agents then lx,ly for L landmarks (packed [4N + 2L]); updated in place.
-void orc_spread_step(int N, int L, float* state, const int32_t* action, float* reward) {
+void orc_spread_step(int N, int L, float* state, const int32_t* action, float* reward,
+                     float local_ratio) {
     Spread s;
     s.N = N; s.L = L;
     for (int i = 0; i < N; ++i) {
@@ -710,7 +721,7 @@ void orc_spread_step(int N, int L, float* state, const int32_t* action, float* r
         s.vx[i] = state[4 * i + 2]; s.vy[i] = state[4 * i + 3];
     }
     for (int l = 0; l < L; ++l) { s.lx[l] = state[4 * N + 2 * l]; s.ly[l] = state[4 * N + 2 * l + 1]; }
-    spread_step(s, action, reward);
+    spread_step(s, action, reward, local_ratio);
     for (int i = 0; i < N; ++i) {
         state[4 * i] = s.px[i]; state[4 * i + 1] = s.py[i];
         state[4 * i + 2] = s.vx[i]; state[4 * i + 3] = s.vy[i];
@@ -748,7 +759,7 @@ void orc_spread_rollout(const float* const* params, int in, int h1, int h2, int 
                         int N, int L, int T, int64_t n_envs, int64_t env_lo, int64_t env_hi,
                         const int32_t* pairs, int32_t n_pairs, int64_t n_episodes, uint64_t seed,
                         const float* ext_logits, float* obs, int8_t* action, float* reward,
-                        float* logits, int n_threads) {
+                        float* logits, int n_threads, float local_ratio) {
     int64_t per = n_envs / n_pairs;
     int64_t W = env_hi - env_lo;
     parallel_for(W * n_episodes, n_threads, [&](int64_t job) {
@@ -773,7 +784,7 @@ void orc_spread_rollout(const float* const* params, int in, int h1, int h2, int 
                 if (action) action[idx] = (int8_t)act[i];
             }
             float r[16];
-            spread_step(s, act, r);
+            spread_step(s, act, r, local_ratio);
             if (reward)
                 for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
         }

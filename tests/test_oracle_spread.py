@@ -124,3 +124,32 @@ def test_rollout_invariants_and_replay(orc):
     # a slice of envs equals the same envs of the full rollout
     sl = orc.spread_rollout(params, dims, 3, 3, 25, 64, w.pair_ids, 2, w.seed, env_lo=16, env_hi=40)
     np.testing.assert_array_equal(sl["reward"], out["reward"][:, :, 16:40])
+
+
+def test_local_ratio_weighting(orc):
+    """App. B.1's local_ratio weights the shared cover term by 1 - rho and the
+    agent's own collisions by rho. Fixed without retyping the formula: rho = 0
+    leaves the same cover reward to every agent, rho = 1 leaves minus the
+    collision count, rho = 1/2 halves the unweighted reward exactly (scaling by
+    a power of two commutes with rounding), and any rho interpolates between
+    the two ends."""
+    rng = np.random.default_rng(3)
+    for trial in range(40):
+        N = 3 if trial % 2 else 8
+        st = rng.uniform(-0.6, 0.6, 6 * N).astype(f32)
+        for i in range(N):
+            st[4 * i + 2:4 * i + 4] *= f32(0.1)
+        acts = rng.integers(0, 5, N)
+        _, r1 = orc.spread_step(st, N, N, acts)
+        _, r0 = orc.spread_step(st, N, N, acts, local_ratio=0.0)
+        _, rl = orc.spread_step(st, N, N, acts, local_ratio=1.0)
+        _, rh = orc.spread_step(st, N, N, acts, local_ratio=0.5)
+        assert np.all(r0 == r0[0]) and r0[0] <= 0
+        diff = r0 - r1                                 # (cover + coll) - cover, rounded twice
+        coll = np.round(diff)
+        assert np.all(np.abs(diff - coll) <= 4 * np.spacing(np.abs(r1))) and np.all(coll >= 0)
+        np.testing.assert_array_equal(rl, -coll)
+        np.testing.assert_array_equal(rh, r1 * f32(0.5))
+        _, rq = orc.spread_step(st, N, N, acts, local_ratio=0.25)
+        lo, hi = np.minimum(r0, rl), np.maximum(r0, rl)
+        assert np.all(rq >= lo - 1e-6) and np.all(rq <= hi + 1e-6)
