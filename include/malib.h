@@ -65,6 +65,7 @@ typedef enum malib_dtype {
 /* Flags of malib_env_spec.flags and malib_eval_payoff_ex(). */
 #define MALIB_DUMP_LOGITS 1u          /* record logits (and obs, actions) in a malib_traj */
 #define MALIB_EXACT_EXPECTATION 2u    /* Kuhn: exact enumeration instead of Monte Carlo */
+#define MALIB_SPREAD_LOCAL_RATIO 4u   /* SPREAD: weight the reward terms by local_ratio */
 
 typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
 
@@ -76,6 +77,13 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  *   SPREAD: n_agents = n_landmarks in [2, 16], obs_dim >= 4 + 4 n_agents - 2,
  *           n_actions 5 (noop, +x, -x, +y, -y), episode_len >= 1
  * n_envs is the number of parallel environments of a rollout (SPREAD).
+ * SPREAD reward of agent i after a step (App. B.1), with cover = sum over
+ * landmarks of the distance to the nearest agent and coll_i = the number of
+ * agents closer than 0.3 to agent i:
+ *   default:                        r_i = -(cover + coll_i)
+ *   flags & MALIB_SPREAD_LOCAL_RATIO: r_i = -((1 - local_ratio) cover + local_ratio coll_i)
+ * (the paper's local_ratio, 0 <= local_ratio <= 1; each operation rounded in
+ * fp32 in the order written).
  */
 typedef struct malib_env_spec {
     int32_t env_kind;
@@ -86,7 +94,7 @@ typedef struct malib_env_spec {
     int32_t episode_len;
     int64_t n_envs;
     uint32_t flags;
-    uint32_t reserved;
+    float local_ratio;        /* read only with MALIB_SPREAD_LOCAL_RATIO */
 } malib_env_spec;
 
 /*

@@ -47,9 +47,12 @@ def _ptr(x):
 
 
 def make_spec(env_kind, n_agents, obs_dim, n_actions, n_landmarks=0, episode_len=0, n_envs=0,
-              flags=0) -> EnvSpec:
+              flags=0, local_ratio=None) -> EnvSpec:
+    """Environment description; local_ratio (spread) weights the reward terms."""
+    if local_ratio is not None:
+        flags |= _abi.MALIB_SPREAD_LOCAL_RATIO
     return EnvSpec(env_kind, n_agents, n_landmarks, obs_dim, n_actions, episode_len, n_envs,
-                   flags, 0)
+                   flags, 0.0 if local_ratio is None else float(local_ratio))
 
 
 def policy_desc(kind, dtype, seat, dims, params) -> PolicyDesc:

@@ -19,7 +19,7 @@ STATUS_NAMES = {0: "OK", -1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ESTATE", 
 MALIB_ENV_KUHN, MALIB_ENV_LEDUC, MALIB_ENV_SPREAD = 1, 2, 3
 MALIB_POL_TABULAR, MALIB_POL_MLP = 1, 2
 MALIB_F32, MALIB_BF16 = 0, 1
-MALIB_DUMP_LOGITS, MALIB_EXACT_EXPECTATION = 1, 2
+MALIB_DUMP_LOGITS, MALIB_EXACT_EXPECTATION, MALIB_SPREAD_LOCAL_RATIO = 1, 2, 4
 
 # Every symbol include/malib.h declares.
 EXPORTS = (
@@ -36,7 +36,7 @@ EXPORTS = (
 class EnvSpec(C.Structure):
     _fields_ = [("env_kind", C.c_int32), ("n_agents", C.c_int32), ("n_landmarks", C.c_int32),
                 ("obs_dim", C.c_int32), ("n_actions", C.c_int32), ("episode_len", C.c_int32),
-                ("n_envs", C.c_int64), ("flags", C.c_uint32), ("reserved", C.c_uint32)]
+                ("n_envs", C.c_int64), ("flags", C.c_uint32), ("local_ratio", C.c_float)]
 
 
 class PolicyDesc(C.Structure):

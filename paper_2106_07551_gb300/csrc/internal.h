@@ -96,6 +96,7 @@ struct RolloutArgs {
     float* reward;
     uint8_t* done;
     float* logits;               // may be null
+    float local_ratio;           // < 0: r_i = -(cover + coll_i); else the weighted reward
 };
 
 // Launchers (return cudaGetLastError() of the launch). `grid_hint` = SM count.

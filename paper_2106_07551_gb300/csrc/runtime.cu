@@ -155,8 +155,14 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
         default:
             return fail(c, MALIB_EINVAL, "unknown env_kind %d", s->env_kind);
     }
-    if (s->flags & ~(MALIB_DUMP_LOGITS | MALIB_EXACT_EXPECTATION))
+    if (s->flags & ~(MALIB_DUMP_LOGITS | MALIB_EXACT_EXPECTATION | MALIB_SPREAD_LOCAL_RATIO))
         return fail(c, MALIB_EINVAL, "unknown flags 0x%x", s->flags);
+    if (s->flags & MALIB_SPREAD_LOCAL_RATIO) {
+        if (s->env_kind != MALIB_ENV_SPREAD)
+            return fail(c, MALIB_EINVAL, "MALIB_SPREAD_LOCAL_RATIO applies to SPREAD only");
+        if (!(s->local_ratio >= 0.0f && s->local_ratio <= 1.0f))
+            return fail(c, MALIB_EINVAL, "local_ratio must lie in [0, 1]");
+    }
     return MALIB_OK;
 }
 
@@ -748,6 +754,7 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     a.obs_dim = spec->obs_dim;
     a.obs_pad = (spec->obs_dim + 3) / 4 * 4;
     a.episode_len = spec->episode_len;
+    a.local_ratio = (spec->flags & MALIB_SPREAD_LOCAL_RATIO) ? spec->local_ratio : -1.0f;
     a.n_envs = spec->n_envs;
     a.n_episodes = n_episodes;
     a.seed = seed;

@@ -96,12 +96,15 @@ __device__ __forceinline__ float sqdist(float ax, float ay, float bx, float by) 
 constexpr float kCollideSq = 0x1.70a3d8p-4f;
 
 // Mass 1, dt 0.1, damping 0.25, unit force along the chosen axis; reward after
-// the move; collision when centres are closer than 2 x 0.15. The rounded
+// the move; collision when centres are closer than 2 x 0.15. local_ratio < 0:
+// r_i = -(cover + coll_i); otherwise -((1 - local_ratio) cover + local_ratio
+// coll_i), each operation rounded in the order written. The rounded
 // square root is monotone, so the minimum over agents of the rounded distances
 // to a landmark equals the rounded root of the minimum squared distance: one
 // root per landmark gives the same bits as one per (landmark, agent).
 template <int N>
-__device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N], float (&r)[N]) {
+__device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N], float (&r)[N],
+                                            float local_ratio) {
 #pragma unroll
     for (int i = 0; i < N; ++i) {
         const float fx = act[i] == 1 ? 1.f : (act[i] == 2 ? -1.f : 0.f);
@@ -131,7 +134,11 @@ __device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N]
         for (int j = i + 1; j < N; ++j)
             if (sqdist(s.px[i], s.py[i], s.px[j], s.py[j]) < kCollideSq) { ++coll[i]; ++coll[j]; }
 #pragma unroll
-    for (int i = 0; i < N; ++i) r[i] = -__fadd_rn(cover, (float)coll[i]);
+    for (int i = 0; i < N; ++i)
+        r[i] = local_ratio < 0.f
+                   ? -__fadd_rn(cover, (float)coll[i])
+                   : -__fadd_rn(__fmul_rn(__fsub_rn(1.f, local_ratio), cover),
+                                __fmul_rn(local_ratio, (float)coll[i]));
 }
 
 }  // namespace malib

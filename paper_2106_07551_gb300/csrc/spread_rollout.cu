@@ -139,7 +139,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 #pragma unroll
                         for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
                 }
-                spread_step<N>(s, act, r);
+                spread_step<N>(s, act, r, a.local_ratio);
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
                     a.action[ix + i] = (uint8_t)act[i];

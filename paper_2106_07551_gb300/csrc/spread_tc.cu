@@ -182,7 +182,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int i = 0; i < kN; ++i) act[i] = acts[(par * kN + i) * 128 + tid];
                 float r[kN];
-                spread_step<kN>(s, act, r);
+                spread_step<kN>(s, act, r, a.local_ratio);
                 float rm = 0.f;
 #pragma unroll
                 for (int i = 0; i < kN; ++i)

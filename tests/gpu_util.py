@@ -20,10 +20,10 @@ def context():
     return Context(0, torch.cuda.current_stream(0))
 
 
-def spec_of(w: workloads.Workload, flags: int = 0, n_envs: int | None = None):
+def spec_of(w: workloads.Workload, flags: int = 0, n_envs: int | None = None, local_ratio=None):
     from paper_2106_07551_gb300 import make_spec
     return make_spec(w.env_kind, w.n_agents, w.obs_dim, w.n_actions, w.n_landmarks,
-                     w.episode_len, w.n_envs if n_envs is None else n_envs, flags)
+                     w.episode_len, w.n_envs if n_envs is None else n_envs, flags, local_ratio)
 
 
 def load_population(ctx, w: workloads.Workload):

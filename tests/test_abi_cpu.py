@@ -68,3 +68,16 @@ def test_missing_library_fails_loudly(tmp_path):
             _abi.load(str(tmp_path / "nope.so"))
     finally:
         _abi._lib = saved
+
+
+def test_env_spec_layout_and_local_ratio_flag():
+    """The spec's last field is the spread reward's local_ratio (a float in the
+    slot of the same size); make_spec sets the flag only when it is given."""
+    import ctypes as C
+    from paper_2106_07551_gb300 import _abi, make_spec
+    assert C.sizeof(_abi.EnvSpec) == 40
+    assert _abi.EnvSpec.local_ratio.offset == 36
+    s = make_spec(3, 3, 18, 5, 3, 25, 4096)
+    assert s.flags & _abi.MALIB_SPREAD_LOCAL_RATIO == 0
+    s = make_spec(3, 3, 18, 5, 3, 25, 4096, local_ratio=0.25)
+    assert s.flags & _abi.MALIB_SPREAD_LOCAL_RATIO and abs(s.local_ratio - 0.25) < 1e-7

@@ -17,21 +17,21 @@ from paper_2106_07551_gb300 import MALIB_DUMP_LOGITS, MalibError, alloc_traj
 RTOL = 1e-5
 
 
-def rollout(ctx, w, n_eps, seed, n_envs=None):
-    spec = spec_of(w, MALIB_DUMP_LOGITS, n_envs)
+def rollout(ctx, w, n_eps, seed, n_envs=None, local_ratio=None):
+    spec = spec_of(w, MALIB_DUMP_LOGITS, n_envs, local_ratio)
     traj = alloc_traj(spec, n_eps, logits=True)
     ctx.rollout(spec, w.pair_ids, n_eps, seed, traj)
     ctx.sync()
     return {k: v.cpu().numpy() for k, v in traj.items()}
 
 
-def check(orc, w, g, n_eps, seed, env_lo, env_hi):
+def check(orc, w, g, n_eps, seed, env_lo, env_hi, local_ratio=None):
     params = [p.params for p in w.policies]
     dims = w.policies[0].dims
     sl = slice(env_lo, env_hi)
     ref = orc.spread_rollout(params, dims, w.n_agents, w.n_landmarks, w.episode_len, w.n_envs,
                              w.pair_ids, n_eps, seed, env_lo=env_lo, env_hi=env_hi,
-                             ext_logits=g["logits"][:, :, sl])
+                             ext_logits=g["logits"][:, :, sl], local_ratio=local_ratio)
     np.testing.assert_array_equal(g["obs"][:, :, sl, :, :w.obs_dim], ref["obs"])
     assert np.all(g["obs"][..., w.obs_dim:] == 0)
     np.testing.assert_array_equal(g["action"][:, :, sl].astype(np.int8), ref["action"])
@@ -54,6 +54,18 @@ def test_full_replay_parity(orc, n_envs, epp, n_eps):
     g2 = rollout(ctx, w, n_eps, 31337)
     for k in g:
         np.testing.assert_array_equal(g2[k], g[k])
+    ctx.close()
+
+
+@pytest.mark.parametrize("rho", [0.0, 0.3, 1.0])
+def test_local_ratio_replay_parity(orc, rho):
+    """App. B.1's local_ratio weighting of the reward: bit-exact under replay."""
+    need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=256, pop=4, envs_per_pair=64, with_bias=True, seed=77)
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 2, 4242, local_ratio=rho)
+    check(orc, w, g, 2, 4242, 0, 256, local_ratio=rho)
     ctx.close()
 
 

@@ -20,21 +20,21 @@ from paper_2106_07551_gb300 import MALIB_DUMP_LOGITS, alloc_traj
 RTOL = 2e-2
 
 
-def rollout(ctx, w, n_eps, seed):
-    spec = spec_of(w, MALIB_DUMP_LOGITS)
+def rollout(ctx, w, n_eps, seed, local_ratio=None):
+    spec = spec_of(w, MALIB_DUMP_LOGITS, None, local_ratio)
     traj = alloc_traj(spec, n_eps, logits=True)
     ctx.rollout(spec, w.pair_ids, n_eps, seed, traj)
     ctx.sync()
     return {k: v.cpu().numpy() for k, v in traj.items()}
 
 
-def check(orc, w, g, n_eps, seed, lo, hi):
+def check(orc, w, g, n_eps, seed, lo, hi, local_ratio=None):
     params = [p.params for p in w.policies]
     dims = w.policies[0].dims
     sl = slice(lo, hi)
     ref = orc.spread_rollout(params, dims, w.n_agents, w.n_landmarks, w.episode_len, w.n_envs,
                              w.pair_ids, n_eps, seed, bf16=True, env_lo=lo, env_hi=hi,
-                             ext_logits=g["logits"][:, :, sl])
+                             ext_logits=g["logits"][:, :, sl], local_ratio=local_ratio)
     np.testing.assert_array_equal(g["obs"][:, :, sl, :, :w.obs_dim], ref["obs"])
     assert np.all(g["obs"][..., w.obs_dim:] == 0)
     np.testing.assert_array_equal(g["action"][:, :, sl].astype(np.int8), ref["action"])
@@ -57,6 +57,18 @@ def test_full_replay_parity(orc, n_envs, epp, n_eps):
     g2 = rollout(ctx, w, n_eps, 4321)
     for k in g:
         np.testing.assert_array_equal(g2[k], g[k])
+    ctx.close()
+
+
+def test_local_ratio_replay_parity(orc):
+    """App. B.1's local_ratio weighting of the reward: bit-exact under replay."""
+    need_gpu()
+    w = workloads.spread(n_agents=8, n_envs=256, pop=4, hidden=256, dtype=workloads.BF16,
+                         envs_per_pair=128, with_bias=True, seed=91)
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 1, 777, local_ratio=0.3)
+    check(orc, w, g, 1, 777, 0, 256, local_ratio=0.3)
     ctx.close()
 
 
