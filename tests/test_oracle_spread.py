@@ -153,3 +153,23 @@ def test_local_ratio_weighting(orc):
         _, rq = orc.spread_step(st, N, N, acts, local_ratio=0.25)
         lo, hi = np.minimum(r0, rl), np.maximum(r0, rl)
         assert np.all(rq >= lo - 1e-6) and np.all(rq <= hi + 1e-6)
+
+
+def test_rollout_fixed_point_over_an_episode(orc):
+    """Logits that force the no-op in every step: resets start at rest, so the
+    whole 25-step episode stays at its reset state - observations and rewards
+    are the same at every step (a multi-step closed form of the rollout loop)."""
+    w = workloads.spread(n_agents=3, n_envs=32, pop=2, envs_per_pair=16, seed=5)
+    params = [p.params for p in w.policies]
+    dims = w.policies[0].dims
+    T = 25
+    ext = np.zeros((1, T, 32, 3, 5), np.float32)
+    ext[..., 0] = 100.0                                 # probability of the no-op ~ 1 - 4 e^-100
+    out = orc.spread_rollout(params, dims, 3, 3, T, 32, w.pair_ids, 1, w.seed, ext_logits=ext)
+    assert np.all(out["action"] == 0)
+    for env in (0, 7, 31):
+        st = orc.spread_reset(3, 3, env, w.seed)
+        _, r = orc.spread_step(st, 3, 3, [0, 0, 0])
+        for t in range(T):
+            np.testing.assert_array_equal(out["obs"][0, t, env], orc.spread_obs(st, 3, 3, 18))
+            np.testing.assert_array_equal(out["reward"][0, t, env], r)
