@@ -69,11 +69,19 @@ struct MlpTc {
     // Issued by thread 0: D(tmem) (+)= A(act tile, K steps [s0, s1)) . B^T, where
     // B starts `w` (a row-group offset inside an image whose K-chunk stride is
     // lbo_w). The first step overwrites D when `fresh`.
+    // Consecutive K steps advance the descriptors' start-address field (bits
+    // 0-13, address >> 4) by a constant; shared-memory addresses stay below
+    // 2^18, so the field never carries.
     __device__ static void issue(uint32_t d, uint32_t act, uint32_t w, uint32_t lbo_w, int s0,
                                  int s1, uint32_t idesc, bool fresh) {
-        for (int s = s0; s < s1; ++s)
-            tc::mma_bf16(d, tc::smem_desc(act + 2u * s * kLboAct, kLboAct, 128),
-                         tc::smem_desc(w + 2u * s * lbo_w, lbo_w, 128), idesc, !(fresh && s == s0));
+        uint64_t da = tc::smem_desc(act + 2u * s0 * kLboAct, kLboAct, 128);
+        uint64_t db = tc::smem_desc(w + 2u * s0 * lbo_w, lbo_w, 128);
+        const uint64_t step_a = (2u * kLboAct) >> 4, step_b = (2u * lbo_w) >> 4;
+        for (int s = s0; s < s1; ++s) {
+            tc::mma_bf16(d, da, db, idesc, !(fresh && s == s0));
+            da += step_a;
+            db += step_b;
+        }
     }
 
     // One 32-column chunk of a layer's output for this thread's row: D (already
@@ -221,11 +229,14 @@ struct MlpTc {
         // 128..255 are produced. Layer 3 runs as 4 chains of 4 MMAs into TMEM
         // columns 16j (D1's columns, free once h1 is written).
         auto mma3 = [&](int s0, int s1) {
-            for (int s = s0; s < s1; ++s)
-                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))),
-                             tc::smem_desc(s_act + 2u * s * kLboAct, kLboAct, 128),
-                             tc::smem_desc(s_w3 + 2u * s * kLboW3, kLboW3, 128), idesc3,
+            uint64_t da = tc::smem_desc(s_act + 2u * s0 * kLboAct, kLboAct, 128);
+            uint64_t db = tc::smem_desc(s_w3 + 2u * s0 * kLboW3, kLboW3, 128);
+            for (int s = s0; s < s1; ++s) {
+                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))), da, db, idesc3,
                              (s % (kS / 4)) != 0);
+                da += (2u * kLboAct) >> 4;
+                db += (2u * kLboW3) >> 4;
+            }
         };
         epilogue_layer(act, tbase, 256, [&] {
             handoff();
