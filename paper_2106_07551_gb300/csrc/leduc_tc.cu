@@ -3,7 +3,8 @@
 // policy combination).
 //
 // A cluster of two CTAs evaluates one pair at a time. CTA r keeps the policy of
-// seat r resident in shared memory (bf16 weight image and biases, ~146 KB).
+// seat r resident in shared memory (bf16 weight image and biases, ~146 KB);
+// the MLP's hidden activations stay in tensor memory.
 // Each CTA has 16 warps in three roles:
 //  * warps 0-7, the engine: runs 128-row tiles through the tensor-core MLP,
 //    alternating between two hand groups, and returns every row's logits;
@@ -41,7 +42,7 @@ constexpr int kEngineThreads = 256;
 constexpr int kGroups = 2;
 constexpr int kSlots = 128;               // hands per group per CTA
 constexpr int kPart = 64;                 // tile rows per source CTA
-constexpr uint32_t kXBytes = 128 * kK1 * 2;               // one group's observation tile
+constexpr uint32_t kXBytes = Eng::kXBytes;                // one group's observation tile
 constexpr uint32_t kX = Eng::kSmemBytes;                  // X tiles [group]
 constexpr uint32_t kLg = kX + kGroups * kXBytes;          // logits [group][target][rank][4] fp32
 constexpr uint32_t kSmem = kLg + kGroups * 2 * kPart * 16;
@@ -65,7 +66,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     leduc_eval_tc_kernel(EvalArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t stage_bar;
-    __shared__ __align__(8) uint64_t mma_bar;
+    __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t x_bar[kGroups];    // a group's rows and headers
     __shared__ __align__(8) uint64_t lg_bar[kGroups];   // a group's logits
     __shared__ __align__(16) uint4 hdr[kGroups][2];     // [group][source CTA]: {rows here, live}
@@ -84,7 +85,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (tid == 0) {
         dead_s = 0u;
         mbar_init(&stage_bar, 1);
-        mbar_init(&mma_bar, 1);
+        mbar_init(&mma_bar[0], 1);
+        mbar_init(&mma_bar[1], 1);
         for (int g = 0; g < kGroups; ++g) {
             mbar_init(&x_bar[g], 1);
             mbar_init(&lg_bar[g], 1);
@@ -96,8 +98,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
         tc::tmem_relinquish();
     }
-    for (uint32_t i = tid * 16; i < Eng::kActBytes; i += kThreads * 16)
-        *reinterpret_cast<uint4*>(smem + Eng::kAct + i) = make_uint4(0, 0, 0, 0);
+    for (uint32_t i = tid * 16; i < kGroups * kXBytes; i += kThreads * 16)
+        *reinterpret_cast<uint4*>(smem + kX + i) = make_uint4(0, 0, 0, 0);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
@@ -163,7 +165,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         }
                         continue;
                     }
-                    Eng::forward(smem, nullptr, tbase, &mma_bar, mma_par, a.err,
+                    Eng::forward(smem, nullptr, tbase, mma_bar, mma_par, a.err,
                                  [&](int r, const float* lg) {
                                      const uint32_t src = (uint32_t)(r / kPart);
                                      float* dst = lgbuf + ((g * 2 + (int)me) * kPart + r % kPart) * 4;
@@ -173,7 +175,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                                                 __float_as_uint(lg[2]), 0u),
                                                      cl::map(&lg_bar[g], src));
                                  },
-                                 /*x_published=*/true, smem_u32(smem + kX + g * kXBytes));
+                                 smem_u32(smem + kX + g * kXBytes), /*x_published=*/true);
                 }
             }
         }
@@ -235,7 +237,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                     const uint32_t bar = cl::map(&x_bar[g], (uint32_t)seat);
 #pragma unroll
                     for (int c = 0; c < 2; ++c)
-                        cl::st_async_v4(cl::map(xg + Eng::act_offset((int)me * kPart + rank, 8 * c),
+                        cl::st_async_v4(cl::map(xg + Eng::x_offset((int)me * kPart + rank, 8 * c),
                                                 (uint32_t)seat),
                                         make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]),
                                         bar);
@@ -246,7 +248,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         const uint32_t bar = cl::map(&x_bar[g], (uint32_t)tgt);
 #pragma unroll
                         for (int c = 0; c < 2; ++c)
-                            cl::st_async_v4(cl::map(xg + Eng::act_offset((int)me * kPart + rk, 8 * c),
+                            cl::st_async_v4(cl::map(xg + Eng::x_offset((int)me * kPart + rk, 8 * c),
                                                     (uint32_t)tgt),
                                             make_uint4(0, 0, 0, 0), bar);
                     }

@@ -6,21 +6,27 @@
 // Shared memory holds the policy's weight image (staged once by bulk copy):
 // W1 [H][K1], W2 [H][H], W3 [NOUT][H] in the core-matrix K-major layout of
 // tc_common.cuh (K1 = input width padded to 16, NOUT = actions padded to 16),
-// then the fp32 biases b1 [H], b2 [H], b3 [NOUT] (staged with the image), then
-// one activation tile [128][H]. The observation tile X [128][K1] lives at the
-// start of that activation tile: every layer's A operand is the previous
-// layer's output, so X, h1 and h2 reuse the same 64 KB. Tensor memory holds
-// two 256-column accumulators: layer 1 writes D1 (columns 0..255), layer 2 D2
-// (256..511), layer 3 four 16-column partial sums over D1's first 64 columns.
-// D1 and D2 start each forward holding their layer's bias (written with
-// tcgen05.st while other work waits: b2 during layer 1's MMA, b1 after the
-// previous forward), so the MMAs accumulate onto it and the epilogues only
-// apply ReLU and bf16 rounding. Thread 0 issues the MMAs; the 8 warps split
-// each epilogue (warp w: TMEM lane quarter w % 4, 64 of the 128 columns of a
-// half). Each layer's epilogue runs in two column halves, and the next layer's
-// MMAs over the first half's K range are issued before the second half is
-// produced, so the tensor core works while the epilogue warps drain tensor
-// memory.
+// then the fp32 biases b1 [H], b2 [H], b3 [NOUT] (staged with the image or read
+// from global memory). The caller's observation tile X [128][K1] (same layout)
+// is layer 1's A operand; the hidden activations never touch shared memory:
+// each layer's epilogue reads its fp32 accumulator from tensor memory, applies
+// ReLU, rounds to bf16 and writes the packed result back to tensor memory,
+// where the next layer's MMAs read it as their A operand (two bf16 per
+// 32-bit column, the lower k in the low half, row i in lane i).
+//
+// Tensor-memory columns (512 allocated):
+//   D1  [0, 256)    layer-1 accumulator (starts holding b1)
+//   H1  [256, 384)  h1, packed
+//   D2a [384, 512)  layer-2 accumulator, outputs 0..127 (starts holding b2)
+//   D2b [0, 128)    layer-2 accumulator, outputs 128..255 (D1's first half)
+//   H2  [128, 256)  h2, packed (D1's second half)
+//   D3  [384, 448)  layer 3 as four 16-column partial sums (D2a's first part)
+// Each layer's epilogue runs in two column halves. Layer 2's MMAs over h1's
+// first half are issued as soon as it is written, and layer 2 is split by
+// output halves so that the first half's epilogue starts while the tensor core
+// computes the second; layer 3 likewise follows h2's halves. Thread 0 issues
+// the MMAs; the engine's 8 warps split each epilogue (warp w: TMEM lane
+// quarter w % 4, 64 of the 128 columns of a half).
 #pragma once
 
 #include <cstdint>
@@ -46,68 +52,81 @@ struct MlpTc {
     static constexpr uint32_t kPolicyBytes = kImageBytes + kBiasFloats * 4;   // global image
     static constexpr uint32_t kStageBytes = kSmemBias ? kPolicyBytes : kImageBytes;
     static constexpr uint32_t kBias = kImageBytes;                  // biases (after the image)
-    static constexpr uint32_t kAct = kStageBytes;                   // activation tile offset
-    static constexpr uint32_t kActBytes = 128 * H * 2;
-    static constexpr uint32_t kSmemBytes = kStageBytes + kActBytes;
-    static_assert(kStageBytes % 16 == 0, "activation tile 16-byte aligned");
-    static constexpr uint32_t kTmemCols = 512;    // D1 [0,256), D2 [256,512), D3 [0,64)
-    static constexpr uint32_t kLboAct = (128 / 8) * 128;            // K-chunk stride, 128 rows
+    static constexpr uint32_t kSmemBytes = kStageBytes;             // the engine's shared memory
+    static_assert(kStageBytes % 16 == 0, "16-byte aligned image");
+    static constexpr uint32_t kXBytes = 128 * K1 * 2;               // one observation tile
+    static constexpr uint32_t kTmemCols = 512;
+    static constexpr int kD1 = 0, kH1 = 256, kD2a = 384, kD2b = 0, kH2 = 128, kD3 = 384;
+    static constexpr uint32_t kLboX = (128 / 8) * 128;              // K-chunk stride, 128 rows
     static constexpr uint32_t kLboW = (H / 8) * 128;                // K-chunk stride, H rows
     static constexpr uint32_t kLboW3 = (NOUT / 8) * 128;
 
-    // Byte offset, inside the activation tile, of the 8 bf16 columns k..k+7 of row.
-    __device__ static uint32_t act_offset(int row, int k) { return tc::cm_offset(row, k, 128, 2); }
+    // Byte offset, inside an observation tile, of the 8 bf16 columns k..k+7 of row.
+    __device__ static uint32_t x_offset(int row, int k) { return tc::cm_offset(row, k, 128, 2); }
 
-    // Waits for the MMA barrier's current phase (bounded); flips the parity.
-    __device__ static void wait_mma(uint64_t* bar, uint32_t& parity, int* err) {
-        if (!mbar_wait_bounded(bar, parity, kWaitLimitNs) && threadIdx.x == 0)
-            atomicOr(err, ERRBIT_TIMEOUT);
-        parity ^= 1u;
+    // Barrier over the engine's threads.
+    __device__ static void sync() {
+        if (kBarId == 0) {
+            __syncthreads();
+        } else {
+            asm volatile("bar.sync %0, 256;" ::"n"(kBarId) : "memory");
+        }
+    }
+
+    // Orders this thread's tensor-memory stores (and loads) before the next
+    // MMA, through a barrier of the engine's threads (all engine threads call).
+    __device__ static void handoff() {
+        tc::tmem_wait_st();
+        tc::fence_before_sync();
+        sync();
         tc::fence_after_sync();
     }
 
-    // Issued by thread 0: D(tmem) (+)= A(act tile, K steps [s0, s1)) . B^T, where
-    // B starts `w` (a row-group offset inside an image whose K-chunk stride is
-    // lbo_w). The first step overwrites D when `fresh`.
-    // Consecutive K steps advance the descriptors' start-address field (bits
-    // 0-13, address >> 4) by a constant; shared-memory addresses stay below
-    // 2^18, so the field never carries.
-    __device__ static void issue(uint32_t d, uint32_t act, uint32_t w, uint32_t lbo_w, int s0,
-                                 int s1, uint32_t idesc, bool fresh) {
-        uint64_t da = tc::smem_desc(act + 2u * s0 * kLboAct, kLboAct, 128);
+    // Waits (bounded) for the current phase of MMA barrier i (bars[i]); bit i
+    // of `parity` tracks that barrier's phase and is flipped. Two barriers: the
+    // two halves of layer 2 complete back to back, and a thread that looked late
+    // at one barrier whose next phase had already completed would miss it.
+    __device__ static void wait_mma(uint64_t* bars, int i, uint32_t& parity, int* err) {
+        if (!mbar_wait_bounded(bars + i, (parity >> i) & 1u, kWaitLimitNs) && threadIdx.x == 0)
+            atomicOr(err, ERRBIT_TIMEOUT);
+        parity ^= 1u << i;
+        tc::fence_after_sync();
+    }
+
+    // tcgen05.mma kind::f16 with the A operand in tensor memory.
+    __device__ static void mma_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc,
+                                  bool accumulate) {
+        asm volatile(
+            "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+            " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d_tmem),
+            "r"(a_tmem), "l"(b), "r"(idesc), "r"((uint32_t)accumulate)
+            : "memory");
+    }
+
+    // Issued by thread 0: D (+)= A(tensor memory, K steps [s0, s1), 8 columns
+    // per step from a_col) . B^T, B from the weight image at w (K-chunk stride
+    // lbo_w). Consecutive K steps advance the descriptor's start-address field
+    // (bits 0-13, address >> 4) by a constant; shared-memory addresses stay
+    // below 2^18, so the field never carries.
+    __device__ static void issue_ta(uint32_t d, uint32_t a_col, uint32_t w, uint32_t lbo_w, int s0,
+                                    int s1, uint32_t idesc, bool accumulate_first) {
         uint64_t db = tc::smem_desc(w + 2u * s0 * lbo_w, lbo_w, 128);
-        const uint64_t step_a = (2u * kLboAct) >> 4, step_b = (2u * lbo_w) >> 4;
         for (int s = s0; s < s1; ++s) {
-            tc::mma_bf16(d, da, db, idesc, !(fresh && s == s0));
-            da += step_a;
-            db += step_b;
+            mma_ta(d, a_col + 8u * s, db, idesc, accumulate_first || s != s0);
+            db += (2u * lbo_w) >> 4;
         }
     }
 
-    // One 32-column chunk of a layer's output for this thread's row: D (already
-    // in registers, bias included) -> relu -> bf16, stored into the activation tile.
-    __device__ static void store_chunk(uint8_t* act, int row, int c0, const uint32_t (&v)[32]) {
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            auto f = [&](int i) { return __uint_as_float(v[8 * j + i]); };
-            uint4 pk;
-            pk.x = tc::relu_bf16x2(f(0), f(1));
-            pk.y = tc::relu_bf16x2(f(2), f(3));
-            pk.z = tc::relu_bf16x2(f(4), f(5));
-            pk.w = tc::relu_bf16x2(f(6), f(7));
-            *reinterpret_cast<uint4*>(act + act_offset(row, c0 + 8 * j)) = pk;
-        }
-    }
-
-    // Writes a layer's bias (H values) into every row of the accumulator at TMEM
-    // column tcol, so the layer's MMAs accumulate onto it: warp w writes its lane
-    // quarter w % 4, columns 128 (w / 4) .. +127. Waits for its stores.
-    __device__ static void prefill(const float* bias, uint32_t tbase, int tcol) {
+    // Writes n bias values (starting at bias) into every row of the accumulator
+    // columns [tcol, tcol + n): warp w writes lane quarter w % 4, half w / 4 of
+    // the n columns (n = 128 or 256). Waits for its stores.
+    __device__ static void prefill(const float* bias, uint32_t tbase, int tcol, int n) {
         const int warp = threadIdx.x >> 5;
         const int q = warp & 3, h = warp >> 2;
+        const int per = n / 2;
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-            const int c0 = 128 * h + 32 * c;
+        for (int c = 0; c < per; c += 32) {
+            const int c0 = h * per + c;
             uint32_t r[32];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
@@ -127,136 +146,135 @@ struct MlpTc {
     // weights and biases are staged). The caller orders it before the next MMA
     // (tcgen05 fence before a barrier of the engine's threads).
     __device__ static void prefill_d1(uint8_t* smem, const float* gbias, uint32_t tbase) {
-        prefill(kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias, tbase, 0);
+        prefill(kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias, tbase, kD1, H);
     }
 
-    // A layer's output, D (TMEM columns tcol .., bias included) -> relu -> bf16
-    // into the activation tile, in two column halves. Warp w takes TMEM lane quarter
-    // w % 4 and, in each half, the 64 columns 64 (w / 4) .. of that half. The
-    // first half is stored, then the second half's tensor-memory loads are
-    // issued and stay in flight across mid() (the hand-off that lets the next
-    // layer's MMAs start on the first half).
-    template <class Mid>
-    __device__ static void epilogue_layer(uint8_t* act, uint32_t tbase, int tcol, Mid mid) {
-        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-        const int q = warp & 3, h = warp >> 2;
-        const int row = 32 * q + lane;
-        const int ca = 64 * h, cb = H / 2 + 64 * h;
-        {
-            uint32_t r0[32], r1[32];
-            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + ca), r0);
-            tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + ca + 32), r1);
-            tc::tmem_wait_ld();
-            store_chunk(act, row, ca, r0);
-            store_chunk(act, row, ca + 32, r1);
-        }
-        uint32_t r2[32], r3[32];
-        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb), r2);
-        tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * q, tcol + cb + 32), r3);
-        mid();
-        tc::tmem_wait_ld();
-        store_chunk(act, row, cb, r2);
-        store_chunk(act, row, cb + 32, r3);
-    }
-
-    // Barrier over the engine's threads.
-    __device__ static void sync() {
-        if (kBarId == 0) {
-            __syncthreads();
+    // One 32-column chunk of an accumulator (in registers) -> relu -> bf16 pairs
+    // -> 16 packed tensor-memory columns at taddr. With `bias`, the chunk's 32
+    // bias values are added first.
+    __device__ static void pack_chunk(const uint32_t (&v)[32], const float* bias, uint32_t taddr) {
+        uint32_t pk[16];
+        if (bias) {
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const float4 b = kSmemBias ? *reinterpret_cast<const float4*>(bias + 4 * j)
+                                           : __ldg(reinterpret_cast<const float4*>(bias + 4 * j));
+                pk[2 * j] = tc::bias_relu_bf16x2(__uint_as_float(v[4 * j]),
+                                                 __uint_as_float(v[4 * j + 1]), b.x, b.y);
+                pk[2 * j + 1] = tc::bias_relu_bf16x2(__uint_as_float(v[4 * j + 2]),
+                                                     __uint_as_float(v[4 * j + 3]), b.z, b.w);
+            }
         } else {
-            asm volatile("bar.sync %0, 256;" ::"n"(kBarId) : "memory");
+#pragma unroll
+            for (int j = 0; j < 16; ++j)
+                pk[j] = tc::relu_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
         }
+        tc::tmem_st16(taddr, pk);
     }
 
-    // Makes the engine's generic shared-memory writes visible to the tensor
-    // cores and orders tensor-memory reads before the next MMA (all engine
-    // threads call).
-    __device__ static void handoff() {
-        fence_proxy_async_smem();
-        tc::fence_before_sync();
-        sync();
-        tc::fence_after_sync();
+    // One 128-column half of a layer's output: accumulator columns
+    // [dcol, dcol + 128) -> packed activations at [hcol, hcol + 64). Warp w
+    // takes lane quarter w % 4 and columns 64 (w / 4) .. of the half. bias (or
+    // null when the accumulator already holds it) covers the half's columns.
+    __device__ static void epilogue_half(uint32_t tbase, int dcol, int hcol, const float* bias) {
+        const int warp = threadIdx.x >> 5;
+        const int q = warp & 3, h = warp >> 2;
+        const int c = 64 * h;
+        uint32_t r0[32], r1[32];
+        tc::tmem_ld32x2(tc::tmem_addr(tbase, 32 * q, dcol + c), tc::tmem_addr(tbase, 32 * q, dcol + c + 32),
+                        r0, r1);
+        pack_chunk(r0, bias ? bias + c : nullptr, tc::tmem_addr(tbase, 32 * q, hcol + c / 2));
+        pack_chunk(r1, bias ? bias + c + 32 : nullptr, tc::tmem_addr(tbase, 32 * q, hcol + c / 2 + 16));
     }
 
-    // Full forward of the 128-row tile whose X has been written (and published
-    // by the caller's synchronisation). out(row, logits[16]) is called by the
-    // threads of warps 0-3 (thread = row) for every row; the caller knows which
-    // rows hold observations. gbias: the policy's biases in global memory (used
-    // when kSmemBias is false). All threads call.
-    // x_published: the caller's X writers already fenced (proxy) and the CTA
-    // has synchronised since (e.g. a cluster sync), so MMA 1 issues at once.
-    // x_tile: shared-memory address of the observation tile [128][K1] (same
-    // core-matrix layout as the activation tile); 0 = the activation tile's start.
+    // Full forward of the 128-row observation tile at shared-memory address
+    // x_tile. bars: two mbarriers (count 1) for the MMA completions; parity:
+    // their phase bits, kept by the caller across forwards. out(row, logits[16]) is called by the threads of warps 0-3 (thread
+    // = row) for every row; the caller knows which rows hold observations.
+    // gbias: the policy's biases in global memory (used when kSmemBias is false).
+    // All engine threads call. D1 must hold b1 (prefill_d1 before the first
+    // forward of a policy; every forward leaves it so for the next one).
+    // x_published: the caller's X writers already fenced (proxy) and the engine
+    // has synchronised since, so MMA 1 issues at once; otherwise the forward
+    // fences and synchronises first.
     template <class Out>
-    __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bar,
-                                   uint32_t& parity, int* err, Out out, bool x_published = false,
-                                   uint32_t x_tile = 0) {
-        uint8_t* act = smem + kAct;
+    __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bars,
+                                   uint32_t& parity, int* err, Out out, uint32_t x_tile,
+                                   bool x_published = false) {
         const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
-        const uint32_t s_act = smem_u32(act);
         const uint32_t s_w1 = smem_u32(smem + kW1), s_w2 = smem_u32(smem + kW2);
         const uint32_t s_w3 = smem_u32(smem + kW3);
-        if (x_published) {
-            if (threadIdx.x == 0) fence_proxy_async_smem();
-            tc::fence_after_sync();
-        } else {
-            handoff();
+        if (!x_published) {
+            fence_proxy_async_smem();
+            tc::fence_before_sync();
+            sync();
         }
+        if (threadIdx.x == 0) fence_proxy_async_smem();
+        tc::fence_after_sync();
         const uint32_t idesc_full = tc::instr_desc(128, H, 1);
+        const uint32_t idesc_half = tc::instr_desc(128, H / 2, 1);
         const uint32_t idesc3 = tc::instr_desc(128, NOUT, 1);
-        const uint32_t d1 = tbase, d2 = tbase + 256;
         constexpr int kS = H / 16;                      // K steps of layers 2 and 3
-        // layer 1 (N = 256, K = K1) onto D1 (holding b1); meanwhile b2 goes into D2
+        // layer 1 (N = 256, K = K1) onto D1 (holding b1); meanwhile b2's first
+        // half goes into D2a
         if (threadIdx.x == 0) {
-            issue(d1, x_tile ? x_tile : s_act, s_w1, kLboW, 0, K1 / 16, idesc_full, false);
-            tc::mma_commit(bar);
+            uint64_t da = tc::smem_desc(x_tile, kLboX, 128);
+            uint64_t db = tc::smem_desc(s_w1, kLboW, 128);
+            for (int s = 0; s < K1 / 16; ++s) {
+                tc::mma_bf16(tbase + kD1, da, db, idesc_full, true);
+                da += (2u * kLboX) >> 4;
+                db += (2u * kLboW) >> 4;
+            }
+            tc::mma_commit(bars);
         }
-        prefill(bias + H, tbase, 256);
-        wait_mma(bar, parity, err);
-        // h1 columns 0..127, then layer-2 K steps 0..7 (N = 256) while h1
-        // columns 128..255 are produced, then K steps 8..15
-        epilogue_layer(act, tbase, 0, [&] {
-            handoff();
-            if (threadIdx.x == 0) issue(d2, s_act, s_w2, kLboW, 0, kS / 2, idesc_full, false);
-        });
+        prefill(bias + H, tbase, kD2a, H / 2);
+        wait_mma(bars, 0, parity, err);
+        // h1, first half; then layer 2's outputs 0..127 over h1's first half
+        epilogue_half(tbase, kD1, kH1, nullptr);
+        handoff();
+        if (threadIdx.x == 0)
+            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, true);
+        // h1, second half; then the rest of layer 2: outputs 0..127, then
+        // 128..255 into D2b (D1's first half, already read)
+        epilogue_half(tbase, kD1 + H / 2, kH1 + H / 4, nullptr);
         handoff();
         if (threadIdx.x == 0) {
-            issue(d2, s_act, s_w2, kLboW, kS / 2, kS, idesc_full, false);
-            tc::mma_commit(bar);
+            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, kS / 2, kS, idesc_half, true);
+            tc::mma_commit(bars);                           // D2a complete
+            issue_ta(tbase + kD2b, tbase + kH1, s_w2 + (H / 2 / 8) * 128, kLboW, 0, kS, idesc_half,
+                     false);
+            tc::mma_commit(bars + 1);                       // D2b complete
         }
-        wait_mma(bar, parity, err);
-        // h2 columns 0..127, then layer-3 K steps 0..7 while h2 columns
-        // 128..255 are produced. Layer 3 runs as 4 chains of 4 MMAs into TMEM
-        // columns 16j (D1's columns, free once h1 is written).
+        wait_mma(bars, 0, parity, err);                     // D2a
+        // h2, first half (into H2, D1's second half, already read); then layer 3
+        // over it: four chains of 4 K steps into D3 (D2a's columns, just read)
+        epilogue_half(tbase, kD2a, kH2, nullptr);
+        handoff();
         auto mma3 = [&](int s0, int s1) {
-            uint64_t da = tc::smem_desc(s_act + 2u * s0 * kLboAct, kLboAct, 128);
             uint64_t db = tc::smem_desc(s_w3 + 2u * s0 * kLboW3, kLboW3, 128);
             for (int s = s0; s < s1; ++s) {
-                tc::mma_bf16(tbase + (uint32_t)(16 * (s / (kS / 4))), da, db, idesc3,
-                             (s % (kS / 4)) != 0);
-                da += (2u * kLboAct) >> 4;
+                mma_ta(tbase + kD3 + (uint32_t)(16 * (s / (kS / 4))), tbase + kH2 + 8u * s, db,
+                       idesc3, (s % (kS / 4)) != 0);
                 db += (2u * kLboW3) >> 4;
             }
         };
-        epilogue_layer(act, tbase, 256, [&] {
-            handoff();
-            if (threadIdx.x == 0) mma3(0, kS / 2);
-        });
+        if (threadIdx.x == 0) mma3(0, kS / 2);
+        wait_mma(bars, 1, parity, err);                     // D2b
+        epilogue_half(tbase, kD2b, kH2 + H / 4, bias + H + H / 2);
         handoff();
         if (threadIdx.x == 0) {
             mma3(kS / 2, kS);
-            tc::mma_commit(bar);
+            tc::mma_commit(bars);
         }
-        wait_mma(bar, parity, err);
+        wait_mma(bars, 0, parity, err);
         const int warp = threadIdx.x >> 5;
         if (warp < 4) {
             const int row = threadIdx.x;
             float v[16];
             {
                 uint32_t r[32], r2[32];
-                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * warp, 0), r);
-                tc::tmem_ld32_nowait(tc::tmem_addr(tbase, 32 * warp, 32), r2);
-                tc::tmem_wait_ld();
+                tc::tmem_ld32x2(tc::tmem_addr(tbase, 32 * warp, kD3),
+                                tc::tmem_addr(tbase, 32 * warp, kD3 + 32), r, r2);
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
                     v[i] = (__uint_as_float(r[i]) + __uint_as_float(r[16 + i])) +
@@ -266,9 +284,10 @@ struct MlpTc {
             for (int i = 0; i < 16; ++i) v[i] += kSmemBias ? bias[2 * H + i] : __ldg(bias + 2 * H + i);
             out(row, v);
         }
-        // b1 into D1 for the next forward (each warp rewrites only columns of its
-        // own lane quarter, after its own reads of the layer-3 chains)
-        prefill(bias, tbase, 0);
+        // b1 into D1 for the next forward: D2b and H2, which share its columns,
+        // are consumed; each warp rewrites only its own lane quarter (the
+        // layer-3 chains it read live in other columns)
+        prefill(bias, tbase, kD1, H);
         tc::fence_before_sync();
         sync();
     }

@@ -28,10 +28,11 @@ constexpr int kN = 8;                        // agents = landmarks = cluster siz
 constexpr int kObs = 34, kObsPad = 36, kK1 = 48, kA = 5;
 using Eng = MlpTc<kK1, 256, 16, false>;      // biases read through L1 (shared memory is full)
 constexpr int kThreads = 256;
-constexpr uint32_t kActs = Eng::kSmemBytes;                  // actions [parity][agent][env] u8
+constexpr uint32_t kX = Eng::kSmemBytes;                     // observation tile (bf16)
+constexpr uint32_t kStage = kX + Eng::kXBytes;               // fp32 observation rows [128][36]
+constexpr uint32_t kActs = kStage + 128 * kObsPad * 4;       // actions [parity][agent][env] u8
 constexpr uint32_t kSmem = kActs + 2 * kN * 128;
-constexpr uint32_t kStage = 128 * kK1 * 2;                   // fp32 obs rows, after X in the tile
-static_assert(kStage % 16 == 0 && kStage + 128 * kObsPad * 4 <= Eng::kActBytes, "obs staging fits");
+static_assert(kX % 16 == 0 && kStage % 16 == 0 && kActs % 16 == 0, "16-byte aligned regions");
 constexpr uint32_t kActTx = (kN - 1) * 128;                  // action bytes received per step
 
 __device__ __forceinline__ void cluster_barrier_all() {
@@ -43,7 +44,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     spread_rollout_tc_kernel(RolloutArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t stage_bar;
-    __shared__ __align__(8) uint64_t mma_bar;
+    __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t act_bar[2];   // peers' actions of steps with parity 0 / 1
     __shared__ uint32_t tmem_base;
 
@@ -53,7 +54,8 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
 
     if (tid == 0) {
         mbar_init(&stage_bar, 1);
-        mbar_init(&mma_bar, 1);
+        mbar_init(&mma_bar[0], 1);
+        mbar_init(&mma_bar[1], 1);
         mbar_init(&act_bar[0], 1);
         mbar_init(&act_bar[1], 1);
         mbar_arrive_expect_tx(&act_bar[0], kActTx);      // armed for steps 0 and 1
@@ -63,8 +65,8 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
         tc::tmem_relinquish();
     }
-    for (uint32_t i = tid * 16; i < Eng::kActBytes; i += kThreads * 16)
-        *reinterpret_cast<uint4*>(smem + Eng::kAct + i) = make_uint4(0, 0, 0, 0);
+    for (uint32_t i = tid * 16; i < Eng::kXBytes; i += kThreads * 16)
+        *reinterpret_cast<uint4*>(smem + kX + i) = make_uint4(0, 0, 0, 0);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
@@ -81,7 +83,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     const int64_t lo = cid * per, hi = min(items, lo + per);
     int staged = -1;
     const float* gbias = nullptr;
-    float* stage = reinterpret_cast<float*>(smem + Eng::kAct + kStage);
+    float* stage = reinterpret_cast<float*>(smem + kStage);
 
     for (int64_t it = lo; it < hi; ++it) {
         const int pair = (int)(it / a.n_episodes);
@@ -139,7 +141,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     w[i] = 2 * i + 1 < kObs ? tc::pack_bf16(o[2 * i], o[2 * i + 1]) : 0u;
 #pragma unroll
                 for (int c = 0; c < kK1 / 8; ++c)
-                    *reinterpret_cast<uint4*>(smem + Eng::kAct + Eng::act_offset(tid, 8 * c)) =
+                    *reinterpret_cast<uint4*>(smem + kX + Eng::x_offset(tid, 8 * c)) =
                         make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]);
             }
             __syncthreads();
@@ -151,7 +153,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     reinterpret_cast<float4*>(a.obs + (base + (int64_t)v * kN) * kObsPad)[c] = src[q];
                 }
             }
-            Eng::forward(smem, gbias, tbase, &mma_bar, mma_par, a.err, [&](int row, const float* lg) {
+            Eng::forward(smem, gbias, tbase, mma_bar, mma_par, a.err, [&](int row, const float* lg) {
                 int act = 0;
                 if (row < epp) {
                     float l5[kA];
@@ -164,7 +166,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     a.action[ix + me] = (uint8_t)act;
                 }
                 my_acts[row] = (uint8_t)act;
-            });   // its opening barrier also ends the staged rows' reads before h1 overwrites them
+            }, smem_u32(smem + kX));
             // forward ends with a CTA barrier: all 128 action bytes are in my_acts
             if (tid < (kN - 1) * 8) {
                 const uint32_t c = (uint32_t)tid & 7u, j = (uint32_t)tid >> 3;
