@@ -67,6 +67,7 @@ struct EvalArgs {
     uint64_t seed;
     unsigned long long* acc;     // [n_pairs][2]
     unsigned long long* n_dec;   // total decisions (env-steps) of the call
+    unsigned long long* work;    // [n_pairs] hands claimed so far (zeroed per call)
     int* err;
     // optional dump of the first n_dump episodes of each pair
     int64_t n_dump;

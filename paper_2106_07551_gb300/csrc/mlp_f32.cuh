@@ -226,7 +226,8 @@ struct MlpF32 {
 // live in a buffer of its own (restaged per policy) while the small layers of
 // several policies stay resident. Layer 3 is folded into layer 2's epilogue
 // (shuffle reduction over the 16 column lanes of a row group, which share one
-// warp).
+// warp). NI (8 or 4) is the number of 16-row blocks a pass computes: NI = 4
+// covers rows 0..63 only, for passes whose compacted rows all lie there.
 template <int IN, int A>
 struct MlpF32T8 {
     static constexpr int H = 128;
@@ -244,14 +245,16 @@ struct MlpF32T8 {
     __device__ static int row_group() { return (threadIdx.x >> 5) * 2 + ((threadIdx.x >> 3) & 1); }
 
     // acc[i][p]: row i, column pair p (p 0,1: c0..c0+3; p 2,3: c1..c1+3)
+    template <int NI>
     __device__ static void init(u64 (&acc)[8][4], const float* __restrict__ b, int c0, int c1) {
         const ulonglong2 bA = *reinterpret_cast<const ulonglong2*>(b + c0);
         const ulonglong2 bB = *reinterpret_cast<const ulonglong2*>(b + c1);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) { acc[i][0] = bA.x; acc[i][1] = bA.y; acc[i][2] = bB.x; acc[i][3] = bB.y; }
+        for (int i = 0; i < NI; ++i) { acc[i][0] = bA.x; acc[i][1] = bA.y; acc[i][2] = bB.x; acc[i][3] = bB.y; }
     }
 
     // acc += rows' inputs [4 k from xa] x W rows k0..k0+3 (kk < kmax)
+    template <int NI>
     __device__ static void block(u64 (&acc)[8][4], const float4 (&xa)[8], const float* __restrict__ W,
                                  int k0, int kmax, int c0, int c1) {
 #pragma unroll
@@ -263,37 +266,38 @@ struct MlpF32T8 {
                 // column pair, so no FMA waits on the duplication just before it
                 u64 x2[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
+                for (int i = 0; i < NI; ++i)
                     x2[i] = f2_dup(kk == 0 ? xa[i].x : kk == 1 ? xa[i].y : kk == 2 ? xa[i].z : xa[i].w);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) f2_fma(acc[i][0], x2[i], wA.x);
+                for (int i = 0; i < NI; ++i) f2_fma(acc[i][0], x2[i], wA.x);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) f2_fma(acc[i][1], x2[i], wA.y);
+                for (int i = 0; i < NI; ++i) f2_fma(acc[i][1], x2[i], wA.y);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) f2_fma(acc[i][2], x2[i], wB.x);
+                for (int i = 0; i < NI; ++i) f2_fma(acc[i][2], x2[i], wB.x);
 #pragma unroll
-                for (int i = 0; i < 8; ++i) f2_fma(acc[i][3], x2[i], wB.y);
+                for (int i = 0; i < NI; ++i) f2_fma(acc[i][3], x2[i], wB.y);
             }
         }
     }
 
     // Layer 1 into H1 (rows of X [128][XS]). Ends with __syncthreads.
+    template <int NI = 8>
     __device__ static void layer1(const float* __restrict__ X, float* __restrict__ H1,
                                   const float* __restrict__ W1T, const float* __restrict__ b1) {
         const int tx = col_group(), ty = row_group();
         const int c0 = tx * 4, c1 = H / 2 + tx * 4;
         u64 acc[8][4];
-        init(acc, b1, c0, c1);
+        init<NI>(acc, b1, c0, c1);
 #pragma unroll
         for (int k0 = 0; k0 < IN; k0 += 4) {
             float4 xa[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < NI; ++i)
                 xa[i] = *reinterpret_cast<const float4*>(X + (ty + 16 * i) * XS + k0);
-            block(acc, xa, W1T, k0, IN - k0, c0, c1);
+            block<NI>(acc, xa, W1T, k0, IN - k0, c0, c1);
         }
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
+        for (int i = 0; i < NI; ++i) {
             float* hr = H1 + (ty + 16 * i) * HS;
             const float2 p0 = f2_split(acc[i][0]), p1 = f2_split(acc[i][1]);
             const float2 p2 = f2_split(acc[i][2]), p3 = f2_split(acc[i][3]);
@@ -306,20 +310,21 @@ struct MlpF32T8 {
     }
 
     // Layers 2 and 3: H1 -> logits rows of LG [128][LS]. Ends with __syncthreads.
+    template <int NI = 8>
     __device__ static void layer23(const float* __restrict__ H1, float* __restrict__ LG,
                                    const float* __restrict__ W2T, const float* __restrict__ b2,
                                    const float* __restrict__ W3, const float* __restrict__ b3) {
         const int tx = col_group(), ty = row_group();
         const int c0 = tx * 4, c1 = H / 2 + tx * 4;
         u64 acc[8][4];
-        init(acc, b2, c0, c1);
+        init<NI>(acc, b2, c0, c1);
 #pragma unroll 4
         for (int k0 = 0; k0 < H; k0 += 4) {
             float4 ha[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < NI; ++i)
                 ha[i] = *reinterpret_cast<const float4*>(H1 + (ty + 16 * i) * HS + k0);
-            block(acc, ha, W2T, k0, 4, c0, c1);
+            block<NI>(acc, ha, W2T, k0, 4, c0, c1);
         }
         float pl[8][A];
 #pragma unroll
@@ -327,7 +332,7 @@ struct MlpF32T8 {
             const float4 vA = *reinterpret_cast<const float4*>(W3 + a * H + c0);
             const float4 vB = *reinterpret_cast<const float4*>(W3 + a * H + c1);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
+            for (int i = 0; i < NI; ++i) {
                 const float2 p0 = f2_split(acc[i][0]), p1 = f2_split(acc[i][1]);
                 const float2 p2 = f2_split(acc[i][2]), p3 = f2_split(acc[i][3]);
                 float t = fmaxf(p0.x, 0.f) * vA.x;
@@ -345,13 +350,13 @@ struct MlpF32T8 {
         for (int o = 1; o <= 16; o <<= 1) {
             if (o == 8) continue;
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < NI; ++i)
 #pragma unroll
                 for (int a = 0; a < A; ++a) pl[i][a] += __shfl_xor_sync(0xffffffffu, pl[i][a], o);
         }
         if (tx == 0) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < NI; ++i)
 #pragma unroll
                 for (int a = 0; a < A; ++a) LG[(ty + 16 * i) * LS + a] = pl[i][a] + b3[a];
         }

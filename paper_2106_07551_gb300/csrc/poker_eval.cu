@@ -295,10 +295,23 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_kernel(EvalArgs a) {
 // seat order alternates each step, so W2 is restaged once per step by bulk copy,
 // overlapped with the second seat's layer 1. A seat with more than 128 acting
 // hands defers the rest to the next step (their results do not depend on it).
+//
+// Work distribution: every pair has a hand counter in global memory shared by
+// all CTAs that work on it. A CTA claims hands in chunks of kChunk and refills
+// its slots from them; when the pair has no unclaimed hands left and its own
+// hands have finished, it moves to the pair with the most unclaimed hands.
+// Games differ in length from pair to pair, so a fixed split of the hands
+// leaves CTAs with different numbers of steps; claiming keeps them finishing
+// together. A hand's result depends only on its (pair, hand) ids, so the
+// payoff sums do not depend on which CTA plays it.
 namespace t8 {
 using E = MlpF32T8<17, 3>;
 using L = F32Layout<17, 128, 3>;
 constexpr int kSlots = 248;
+constexpr int kChunk = 128;                                   // hands per claim
+constexpr int kRing = 8;                                      // claimed chunk starts kept
+// at a step's start the unconsumed claimed chunks number at most kSlots / kChunk + 2
+static_assert(kRing >= kSlots / kChunk + 3, "ring holds every chunk not yet handed out");
 constexpr int kSmall = L::kW2T + (L::kSize - L::kB2);        // W1T|b1 then b2|W3|b3
 constexpr int kOffSmall = 0;
 constexpr int kOffW2 = kOffSmall + 2 * kSmall;
@@ -308,6 +321,61 @@ constexpr int kOffLG = kOffH1 + E::kRows * E::HS;
 constexpr int kFloats = kOffLG + 2 * E::kRows * E::LS;
 constexpr size_t kBytes = (size_t)kFloats * 4;
 static_assert(kSmall % 4 == 0 && kOffW2 % 4 == 0 && kOffX % 4 == 0 && kOffH1 % 4 == 0, "16-B");
+
+struct Claims {
+    unsigned long long next;      // next slot number to hand out in this segment
+    unsigned long long n;         // chunks claimed in this segment
+    long long base[kRing];        // first hand of chunk c at base[c % kRing]
+    int done;                     // the pair has no unclaimed hands left
+};
+
+// One thread: claim chunks until slots [next, next + kSlots) are covered.
+__device__ __forceinline__ void top_up(Claims& c, unsigned long long* counter, int64_t n_episodes) {
+    while (!c.done && c.n * kChunk < c.next + kSlots) {
+        const unsigned long long s = atomicAdd(counter, (unsigned long long)kChunk);
+        if (s >= (unsigned long long)n_episodes) { c.done = 1; break; }
+        c.base[c.n % kRing] = (long long)s;
+        ++c.n;
+        if (s + kChunk >= (unsigned long long)n_episodes) c.done = 1;
+    }
+}
+
+// Hand of slot j, or -1 when the pair has none left for it.
+__device__ __forceinline__ int64_t slot_hand(const Claims& c, unsigned long long j, int64_t n_episodes) {
+    const unsigned long long ch = j / kChunk;
+    if (ch >= c.n) return -1;
+    const int64_t e = c.base[ch % kRing] + (int64_t)(j % kChunk);
+    return e < n_episodes ? e : -1;
+}
+
+// All threads: the pair with the most unclaimed hands (-1 when none has any).
+// Ends with a barrier; the result is uniform across the CTA.
+__device__ int pick_pair(const EvalArgs& a) {
+    __shared__ long long rem_w[8];
+    __shared__ int pair_w[8];
+    long long best = 0;
+    int bp = -1;
+    for (int p = threadIdx.x; p < a.n_pairs; p += blockDim.x) {
+        const unsigned long long w = *reinterpret_cast<volatile unsigned long long*>(a.work + p);
+        const long long rem = w >= (unsigned long long)a.n_episodes ? 0 : a.n_episodes - (long long)w;
+        if (rem > best) { best = rem; bp = p; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const long long ob = __shfl_xor_sync(0xffffffffu, best, o);
+        const int op = __shfl_xor_sync(0xffffffffu, bp, o);
+        if (ob > best || (ob == best && op >= 0 && (bp < 0 || op < bp))) { best = ob; bp = op; }
+    }
+    const int warp = threadIdx.x >> 5;
+    if ((threadIdx.x & 31) == 0) { rem_w[warp] = best; pair_w[warp] = bp; }
+    __syncthreads();
+    best = 0;
+    bp = -1;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w)
+        if (rem_w[w] > best) { best = rem_w[w]; bp = pair_w[w]; }
+    __syncthreads();
+    return bp;
+}
 }  // namespace t8
 
 __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
@@ -319,7 +387,7 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
     float* W2s = smem + kOffW2;
     __shared__ __align__(8) uint64_t bar;
     __shared__ int cnt[2][8];
-    __shared__ unsigned long long next_e;
+    __shared__ Claims cl;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     for (int i = tid; i < 2 * E::kRows * E::XS; i += blockDim.x) X[i] = 0.f;
@@ -327,19 +395,16 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
     __syncthreads();
     uint32_t parity = 0;
 
-    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
-    const int64_t per = (total + gridDim.x - 1) / gridDim.x;
-    const int64_t lo = (int64_t)blockIdx.x * per;
-    const int64_t hi = min(total, lo + per);
-
-    for (int64_t seg = lo; seg < hi;) {
-        const int pair = (int)(seg / a.n_episodes);
-        const int64_t e_lo = seg - (int64_t)pair * a.n_episodes;
-        const int64_t e_hi = min(a.n_episodes, e_lo + (hi - seg));
-        seg += e_hi - e_lo;
+    int pair = (int)(((int64_t)blockIdx.x * a.n_pairs) / gridDim.x);
+    while (pair >= 0) {
+        unsigned long long* counter = a.work + pair;
         const int pid[2] = {a.pairs[2 * pair], a.pairs[2 * pair + 1]};
         if (!pair_ok(a, pid[0], pid[1])) {
-            if (tid == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+            if (tid == 0) {
+                atomicOr(a.err, ERRBIT_BAD_PAIR);
+                atomicMax(counter, (unsigned long long)a.n_episodes);
+            }
+            pair = pick_pair(a);
             continue;
         }
         const float* pol0 = a.arena + a.pol_offset[pid[0]];
@@ -356,24 +421,31 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
             }
             bulk_g2s(W2s, pol0 + L::kW2T, 32768u, &bar);
             bulk_g2s(W2s + 8192, pol0 + L::kW2T + 8192, 32768u, &bar);
+            cl.next = 0;
+            cl.n = 0;
+            cl.done = 0;
+            top_up(cl, counter, a.n_episodes);
+            cl.next = kSlots;                           // slots 0..kSlots-1 go to threads 0..kSlots-1
         }
         if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs) && tid == 0) atomicOr(a.err, ERRBIT_TIMEOUT);
         parity ^= 1u;
+        __syncthreads();
 
         LeducHand h;
         bool live = false;
-        int64_t e = e_lo + tid;
+        int64_t e = tid < kSlots ? slot_hand(cl, (unsigned long long)tid, a.n_episodes) : -1;
         uint64_t g = 0;
         int t = 0;
         long long s1 = 0, s2 = 0, nd = 0;
-        if (tid < kSlots && e < e_hi) {
+        if (e >= 0) {
             live = true;
             g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
             leduc_deal(h, g, a.seed);
         }
-        if (tid == 0) next_e = (unsigned long long)(e_lo + kSlots);
 
         while (true) {
+            // claims for this step's refills; every reader of cl passed the last barrier
+            if (tid == 0) top_up(cl, counter, a.n_episodes);
             const int seat = live ? h.actor : -1;
             const unsigned b0 = __ballot_sync(0xffffffffu, seat == 0);
             const unsigned b1 = __ballot_sync(0xffffffffu, seat == 1);
@@ -403,9 +475,13 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
             const float* ss = smem + kOffSmall + second * kSmall;
             const int off_b2 = L::kW2T, off_w3 = L::kW2T + (L::kW3 - L::kB2),
                       off_b3 = L::kW2T + (L::kB3 - L::kB2);
-            if (c[first] > 0) {
-                E::layer1(X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
-                E::layer23(H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3, sf + off_b3);
+            // a pass whose placed rows all lie in 0..63 computes only those rows
+            if (c[first] > 64) {
+                E::layer1<8>(X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
+                E::layer23<8>(H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3, sf + off_b3);
+            } else if (c[first] > 0) {
+                E::layer1<4>(X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
+                E::layer23<4>(H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3, sf + off_b3);
             }
             if (c[second] > 0) {
                 const float* src = (second == 0 ? pol0 : pol1) + L::kW2T;
@@ -415,11 +491,16 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
                     bulk_g2s(W2s, src, 32768u, &bar);
                     bulk_g2s(W2s + 8192, src + 8192, 32768u, &bar);
                 }
-                E::layer1(X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
+                const bool full = c[second] > 64;
+                if (full) E::layer1<8>(X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
+                else E::layer1<4>(X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
                 if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs) && tid == 0)
                     atomicOr(a.err, ERRBIT_TIMEOUT);
                 parity ^= 1u;
-                E::layer23(H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3, ss + off_b3);
+                if (full)
+                    E::layer23<8>(H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3, ss + off_b3);
+                else
+                    E::layer23<4>(H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3, ss + off_b3);
                 res = second;
             }
             if (placed) {
@@ -464,8 +545,8 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
                             if (a.d_done) a.d_done[rb + k] = 1;
                         }
                     }
-                    e = (int64_t)atomicAdd(&next_e, 1ull);
-                    live = e < e_hi;
+                    e = slot_hand(cl, atomicAdd(&cl.next, 1ull), a.n_episodes);
+                    live = e >= 0;
                     if (live) {
                         g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
                         leduc_deal(h, g, a.seed);
@@ -476,6 +557,7 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
             __syncthreads();
         }
         block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+        pair = pick_pair(a);
     }
 }
 

@@ -672,12 +672,14 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
         time_end(c, e0, e1);
         c->launches += 1;
     } else {
-        if ((r = ensure(c, c->acc, c->acc_cap, (int64_t)n_pairs * 2 + 1, "payoff sums")) != MALIB_OK)
+        // [n_pairs][2] sums, the decision count, [n_pairs] hand-claim counters
+        if ((r = ensure(c, c->acc, c->acc_cap, (int64_t)n_pairs * 3 + 1, "payoff sums")) != MALIB_OK)
             return r;
         a.acc = c->acc;
         a.n_dec = c->acc + (int64_t)n_pairs * 2;
+        a.work = c->acc + (int64_t)n_pairs * 2 + 1;
         c->last_pairs = n_pairs;
-        CK(launch_zero_u64(c->acc, (int64_t)n_pairs * 2 + 1, c->stream), "zero kernel");
+        CK(launch_zero_u64(c->acc, (int64_t)n_pairs * 3 + 1, c->stream), "zero kernel");
         time_begin(c, &e0, &e1);
         if (kind == MALIB_ENV_KUHN) {
             CK(launch_kuhn_eval(a, c->n_sm, c->stream), "Kuhn eval kernel");

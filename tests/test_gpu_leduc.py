@@ -82,6 +82,21 @@ def test_small_and_ragged(orc, n_eps):
     ctx.close()
 
 
+@pytest.mark.parametrize("n_eps", [3, 1000])
+def test_claimed_hands_across_pairs(orc, n_eps):
+    """64 pairs: with 3 hands per pair one CTA walks every pair; with 1,000 more
+    CTAs than pairs share each pair's hands. Every hand is replayed."""
+    need_gpu()
+    w = workloads.leduc(pop=8, hidden=128, with_bias=True, seed=77)
+    ctx = context()
+    load_population(ctx, w)
+    res, d = run_dumped(ctx, w, n_eps, 31, n_eps)
+    check_replay(orc, w, res, d, n_eps, 31, n_eps, full=True)
+    res2, _ = run_dumped(ctx, w, n_eps, 31, n_eps)
+    np.testing.assert_array_equal(res2, res)
+    ctx.close()
+
+
 def test_full_workload_sampled_replay_and_exact_expectation(orc):
     """8x8 pairs x 65,536 hands in the benchmark's launch configuration."""
     need_gpu()
