@@ -20,8 +20,9 @@
 // complete transaction bytes on the receiver's mbarrier; every slot is written
 // every step (unused rows with zeros), so each receiver expects a fixed byte
 // count. A logits message whose flag is set tells a group that its hands of the
-// segment are finished in both CTAs. Both CTAs walk the same pair segments; the
-// engine restages weights when both groups have finished a segment.
+// segment are finished in both CTAs. Both CTAs walk the same pair segments
+// (cluster c takes every n_cl-th pair); the engine restages weights when both
+// groups have finished a segment.
 // Control decisions of a role are taken by one thread and handed to the role
 // through its own barrier, so every thread of a role takes the same path.
 #include "cluster.cuh"
@@ -106,20 +107,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     cluster_barrier_all();          // peers' barriers exist before any remote store
     const uint32_t tbase = tmem_base;
 
-    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
+    // Work units: a pair's hands, cut into `parts` pieces when there are fewer
+    // pairs than clusters. Cluster c takes units c, c + n_cl, ...: strided, so
+    // that its pairs come from every row and column of the table (neighbouring
+    // pairs share a policy and so have similar game lengths; contiguous ranges
+    // left clusters with 10 % more work than others).
     const int64_t n_cl = gridDim.x / 2, cid = blockIdx.x / 2;
-    const int64_t per = (total + n_cl - 1) / n_cl;
-    const int64_t lo = cid * per, hi = min(total, lo + per);
+    const int64_t parts = a.n_pairs >= n_cl ? 1 : (n_cl + a.n_pairs - 1) / a.n_pairs;
+    const int64_t chunk = (a.n_episodes + parts - 1) / parts;
+    const int64_t n_units = (int64_t)a.n_pairs * parts;
 
     if (warp < 8) {
         // ------------------------------------------------------------ engine
         uint32_t stage_par = 0, mma_par = 0, x_bits = 0;      // x_bar parity of group g: bit g
         bool stop = false;
-        for (int64_t seg = lo; seg < hi && !stop;) {
-            const int pair = (int)(seg / a.n_episodes);
-            const int64_t e_lo = seg - (int64_t)pair * a.n_episodes;
-            const int64_t e_hi = min(a.n_episodes, e_lo + (hi - seg));
-            seg += e_hi - e_lo;
+        for (int64_t u = cid; u < n_units && !stop; u += n_cl) {
+            const int pair = (int)(u % a.n_pairs);
+            const int64_t e_lo = (u / a.n_pairs) * chunk;
+            const int64_t e_hi = min(a.n_episodes, e_lo + chunk);
+            if (e_lo >= e_hi) continue;                     // the hand groups skip it too
             const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
             if (!pair_ok(a, p0, p1)) continue;             // the hand groups skip it too
             const float* policy = a.arena + a.pol_offset[me == 0 ? p0 : p1];
@@ -187,11 +193,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         uint32_t lg_par = 0;
         uint8_t* xg = smem + kX + g * kXBytes;
         bool stop = false;
-        for (int64_t seg = lo; seg < hi && !stop;) {
-            const int pair = (int)(seg / a.n_episodes);
-            const int64_t e_lo = seg - (int64_t)pair * a.n_episodes;
-            const int64_t e_hi = min(a.n_episodes, e_lo + (hi - seg));
-            seg += e_hi - e_lo;
+        for (int64_t u = cid; u < n_units && !stop; u += n_cl) {
+            const int pair = (int)(u % a.n_pairs);
+            const int64_t e_lo = (u / a.n_pairs) * chunk;
+            const int64_t e_hi = min(a.n_episodes, e_lo + chunk);
+            if (e_lo >= e_hi) continue;                 // same decision in every role of both CTAs
             const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
             if (!pair_ok(a, p0, p1)) {                  // same decision in every role of both CTAs
                 if (tid == kEngineThreads && me == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
