@@ -37,6 +37,12 @@ __device__ __forceinline__ float2 f2_split(unsigned long long v) {
     asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
     return make_float2(lo, hi);
 }
+__device__ __forceinline__ unsigned long long f2_relu(unsigned long long v) {
+    const float2 q = f2_split(v);
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(fmaxf(q.x, 0.f)), "f"(fmaxf(q.y, 0.f)));
+    return r;
+}
 
 template <int IN, int H, int A>
 struct MlpF32 {
@@ -326,39 +332,77 @@ struct MlpF32T8 {
                 ha[i] = *reinterpret_cast<const float4*>(H1 + (ty + 16 * i) * HS + k0);
             block<NI>(acc, ha, W2T, k0, 4, c0, c1);
         }
-        float pl[8][A];
+        // layer 3: ReLU once, then per row and action a packed dot product over
+        // the thread's 4 column pairs and the sum of its two halves
+        static_assert(A == 3, "the reduce-scatter below places 3 logits per row");
+#pragma unroll
+        for (int i = 0; i < NI; ++i)
+#pragma unroll
+            for (int p = 0; p < 4; ++p) acc[i][p] = f2_relu(acc[i][p]);
+        constexpr int V = NI * A;                 // partial logits of this thread
+        float v0[V];
 #pragma unroll
         for (int a = 0; a < A; ++a) {
-            const float4 vA = *reinterpret_cast<const float4*>(W3 + a * H + c0);
-            const float4 vB = *reinterpret_cast<const float4*>(W3 + a * H + c1);
+            const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(W3 + a * H + c0);
+            const ulonglong2 wB = *reinterpret_cast<const ulonglong2*>(W3 + a * H + c1);
 #pragma unroll
             for (int i = 0; i < NI; ++i) {
-                const float2 p0 = f2_split(acc[i][0]), p1 = f2_split(acc[i][1]);
-                const float2 p2 = f2_split(acc[i][2]), p3 = f2_split(acc[i][3]);
-                float t = fmaxf(p0.x, 0.f) * vA.x;
-                t = fmaf(fmaxf(p0.y, 0.f), vA.y, t);
-                t = fmaf(fmaxf(p1.x, 0.f), vA.z, t);
-                t = fmaf(fmaxf(p1.y, 0.f), vA.w, t);
-                t = fmaf(fmaxf(p2.x, 0.f), vB.x, t);
-                t = fmaf(fmaxf(p2.y, 0.f), vB.y, t);
-                t = fmaf(fmaxf(p3.x, 0.f), vB.z, t);
-                t = fmaf(fmaxf(p3.y, 0.f), vB.w, t);
-                pl[i][a] = t;
+                u64 t = 0ull;
+                f2_fma(t, acc[i][0], wA.x);
+                f2_fma(t, acc[i][1], wA.y);
+                f2_fma(t, acc[i][2], wB.x);
+                f2_fma(t, acc[i][3], wB.y);
+                const float2 q = f2_split(t);
+                v0[i * A + a] = q.x + q.y;
             }
         }
+        // Reduce-scatter over the 16 lanes of the row group (lane bits 4, 2, 1,
+        // 0): at each of the first levels a lane keeps the half of its values
+        // selected by its lane bit and adds the partner's copy of that half.
+        const int lane = threadIdx.x & 31;
+        const int l4 = (lane >> 4) & 1, l2 = (lane >> 2) & 1, l1 = (lane >> 1) & 1;
+        float v1[V / 2];
 #pragma unroll
-        for (int o = 1; o <= 16; o <<= 1) {
-            if (o == 8) continue;
-#pragma unroll
-            for (int i = 0; i < NI; ++i)
-#pragma unroll
-                for (int a = 0; a < A; ++a) pl[i][a] += __shfl_xor_sync(0xffffffffu, pl[i][a], o);
+        for (int j = 0; j < V / 2; ++j) {
+            const float keep = l4 ? v0[V / 2 + j] : v0[j];
+            const float send = l4 ? v0[j] : v0[V / 2 + j];
+            v1[j] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
         }
-        if (tx == 0) {
+        float v2[V / 4];
 #pragma unroll
-            for (int i = 0; i < NI; ++i)
+        for (int j = 0; j < V / 4; ++j) {
+            const float keep = l2 ? v1[V / 4 + j] : v1[j];
+            const float send = l2 ? v1[j] : v1[V / 4 + j];
+            v2[j] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+        }
+        float v3[A];
+        int i_own;
+        bool writer;
+        if constexpr (NI == 8) {
+            // 6 values: one more halving (lane bit 1), then lane bit 0 sums
+            // both copies; lanes with bit 0 clear hold row 4 l4 + 2 l2 + l1
 #pragma unroll
-                for (int a = 0; a < A; ++a) LG[(ty + 16 * i) * LS + a] = pl[i][a] + b3[a];
+            for (int j = 0; j < A; ++j) {
+                const float keep = l1 ? v2[A + j] : v2[j];
+                const float send = l1 ? v2[j] : v2[A + j];
+                v3[j] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+            }
+#pragma unroll
+            for (int j = 0; j < A; ++j) v3[j] += __shfl_xor_sync(0xffffffffu, v3[j], 1);
+            i_own = 4 * l4 + 2 * l2 + l1;
+            writer = (lane & 1) == 0;
+        } else {
+            // 3 values (row 2 l4 + l2): lane bits 1 and 0 sum all copies
+#pragma unroll
+            for (int j = 0; j < A; ++j) v3[j] = v2[j] + __shfl_xor_sync(0xffffffffu, v2[j], 2);
+#pragma unroll
+            for (int j = 0; j < A; ++j) v3[j] += __shfl_xor_sync(0xffffffffu, v3[j], 1);
+            i_own = 2 * l4 + l2;
+            writer = (lane & 3) == 0;
+        }
+        if (writer) {
+#pragma unroll
+            for (int j = 0; j < A; ++j) LG[(ty + 16 * i_own) * LS + j] = v3[j] + b3[j];
         }
         __syncthreads();
     }
