@@ -367,6 +367,19 @@ def run_ours(args):
                 "algorithmic": f"{flop_per_unit} flop per env-step (MLP forward, padding excluded)"}
     if clk.get("sm_mhz") and not tensor:
         roofline["frac_at_measured_clock"] = achieved / (peak_tflops * clk["sm_mhz"] / sm_max)
+    if args.workload == "kuhn":
+        # Kuhn's work is generator arithmetic: one Philox call per deal and one
+        # per decision; the ceiling is the measured rate of a Philox-only kernel
+        calls = (w.n_pairs * w.n_episodes * args.steps + decisions) / args.steps
+        rate = calls / (kern_ms / max(1, kern_n) / 1e3) if kern_n else 0.0
+        ceil = philox_ceiling(ctx, stream)
+        roofline = {"bound": "alu", "achieved": rate / 1e9, "peak": ceil / 1e9,
+                    "unit": "Gcall/s (Philox4x32-10)", "frac": rate / ceil,
+                    "traffic": None, "kernel": kname,
+                    "kernel_ms_per_launch": kern_ms / max(1, kern_n),
+                    "peak_basis": "measured: malib_philox_digest, 311,296 threads x 4,096 "
+                                  "calls per launch, best of 5 (CUDA events)",
+                    "algorithmic": "1 Philox4x32-10 call per deal + 1 per decision"}
 
     e2e = run_e2e(args, ctx, w, spec, dev, rollout) if rank == 0 else None
 
@@ -390,6 +403,26 @@ def run_ours(args):
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0
+
+
+def philox_ceiling(ctx, stream):
+    """Philox4x32-10 calls per second of the library's arithmetic-only digest
+    kernel: best of 5 launches after 3 warm-ups, timed with CUDA events on the
+    context's stream."""
+    import torch
+    n, calls = SM_COUNT_GB300 * 8 * 256, 4096
+    out = torch.empty(n, dtype=torch.int32, device=stream.device)
+    best = None
+    for k in range(8):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        ctx.philox_digest(0x5EED + k, calls, out)
+        b.record(stream)
+        b.synchronize()
+        if k >= 3:
+            ms = a.elapsed_time(b)
+            best = ms if best is None else min(best, ms)
+    return n * calls / (best / 1e3)
 
 
 def run_e2e(args, ctx, w, spec, dev, rollout):

@@ -325,6 +325,15 @@ double malib_main_kernel_ms(malib_ctx* ctx, int64_t* n_launches, int reset);
 int malib_selftest_philox(malib_ctx* ctx, const uint32_t* ctr, uint64_t seed, uint32_t* out,
                           int64_t n);
 
+/* Philox4x32-10 digest (the generator of Sec. 3.1's sampled rollouts, keyed as
+ * above): thread t < n XOR-folds the four output words of the calls
+ * i = 0..calls-1 at counter (t lo32, t hi32, i, 0) under key (seed lo32, seed
+ * hi32) into out[t] (device uint32 [n], caller-owned). Its work is generator
+ * arithmetic only, so its rate (calls per second) is the ALU ceiling of the Kuhn
+ * evaluation, whose per-hand work is Philox calls. EINVAL for n < 0, calls < 0
+ * or a host pointer; asynchronous on the context's stream. */
+int malib_philox_digest(malib_ctx* ctx, uint64_t seed, int64_t n, int32_t calls, uint32_t* out);
+
 /* The kernels' deterministic exp (Cody-Waite reduction, degree-7 Taylor) on n
  * device floats, and the masked inverse-CDF draw on n rows of A <= 8 logits
  * (device: logits [n][A], legal uint8 [n][A], u [n], out int32 [n]). */

@@ -276,6 +276,13 @@ class Context:
                self.lib.malib_selftest_philox(self.handle, _ptr(ctr), seed, _ptr(out),
                                               int(ctr.shape[0])))
 
+    def philox_digest(self, seed, calls, out):
+        """out[t] = XOR of the 4 words of Philox calls i < calls at counter
+        (t lo, t hi, i, 0) under seed (device uint32 tensor, one entry per t)."""
+        _check(self.lib, self.handle,
+               self.lib.malib_philox_digest(self.handle, seed, int(out.numel()), int(calls),
+                                            _ptr(out)))
+
     def selftest_det_expf(self, x, y):
         _check(self.lib, self.handle,
                self.lib.malib_selftest_det_expf(self.handle, _ptr(x), _ptr(y), int(x.numel())))

@@ -46,6 +46,23 @@ __global__ void philox_kernel(const uint32_t* ctr, uint64_t seed, uint32_t* out,
     }
 }
 
+// Philox throughput probe: thread t XOR-folds the four words of the calls
+// i = 0..calls-1 at counter (t lo, t hi, i, 0) into out[t]. One 4-byte store
+// per thread, so the time is the generator's arithmetic.
+__global__ void __launch_bounds__(256) philox_digest_kernel(uint64_t seed, int64_t n, int calls,
+                                                            uint32_t* out) {
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (t >= n) return;
+    const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+    uint32_t acc = 0u;
+#pragma unroll 4
+    for (int i = 0; i < calls; ++i) {
+        const U4 r = philox10((uint32_t)t, (uint32_t)(t >> 32), (uint32_t)i, 0u, k0, k1);
+        acc ^= r.x ^ r.y ^ r.z ^ r.w;
+    }
+    out[t] = acc;
+}
+
 __global__ void det_expf_kernel(const float* x, float* y, int64_t n) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x)
@@ -93,6 +110,15 @@ cudaError_t launch_selftest_philox(const uint32_t* ctr, uint64_t seed, uint32_t*
                                    cudaStream_t s) {
     if (n <= 0) return cudaSuccess;
     philox_kernel<<<grid_for(n, 256), 256, 0, s>>>(ctr, seed, out, n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_philox_digest(uint64_t seed, int64_t n, int calls, uint32_t* out,
+                                 cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    const int64_t blocks = (n + 255) / 256;
+    if (blocks > 0x7FFFFFFF) return cudaErrorInvalidValue;
+    philox_digest_kernel<<<(unsigned)blocks, 256, 0, s>>>(seed, n, calls, out);
     return cudaGetLastError();
 }
 

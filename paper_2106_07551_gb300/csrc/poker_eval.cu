@@ -24,28 +24,40 @@ namespace {
 // h = 1 when the seat faces a bet. Decision t uses counter (g, t, seat).
 struct KuhnHand { int n; int act[3]; float p[3]; int payoff; };
 
-__device__ __forceinline__ KuhnHand kuhn_play(const float* t0, const float* t1, uint64_t g,
+// Entry idx of a 6-entry register table without dynamic indexing.
+__device__ __forceinline__ float tab6(const float (&t)[6], int idx) {
+    float v = t[0];
+#pragma unroll
+    for (int i = 1; i < 6; ++i) v = idx == i ? t[i] : v;
+    return v;
+}
+
+// Seat 0 acts at decisions 0 and 2, seat 1 at decision 1, whatever the
+// actions, so the three decision draws (g, t, seat) are known before the hand
+// is played: they are drawn up front and the hand is resolved with selects, so
+// the threads of a warp never run the generator on divergent paths. The third
+// draw is used only after pass-bet.
+__device__ __forceinline__ KuhnHand kuhn_play(const float (&t0)[6], const float (&t1)[6], uint64_t g,
                                               uint64_t seed) {
     const U4 d = draw(g, 0, kChance, seed);
     const int c0 = (int)pick(d.x, 3);
     const int j = (int)pick(d.y, 2);
     const int c1 = j + (j >= c0 ? 1 : 0);
     const int sd = c0 > c1 ? 1 : -1;
+    const float u0 = u24(draw(g, 0, 0, seed).x);
+    const float u1 = u24(draw(g, 1, 1, seed).x);
+    const float u2 = u24(draw(g, 2, 0, seed).x);
     KuhnHand h;
-    h.n = 0;
-    auto decide = [&](int seat, float p) {
-        const float u = u24(draw(g, (uint32_t)h.n, (uint32_t)seat, seed).x);
-        const int a = u < p ? 1 : 0;
-        h.act[h.n] = a; h.p[h.n] = p; ++h.n;
-        return a;
-    };
-    if (decide(0, t0[c0 * 2])) {
-        h.payoff = decide(1, t1[c1 * 2 + 1]) ? 2 * sd : 1;
-    } else if (decide(1, t1[c1 * 2])) {
-        h.payoff = decide(0, t0[c0 * 2 + 1]) ? 2 * sd : -1;
-    } else {
-        h.payoff = sd;
-    }
+    h.p[0] = tab6(t0, c0 * 2);                                  // seat 0 opens: P(bet)
+    h.act[0] = u0 < h.p[0] ? 1 : 0;
+    h.p[1] = tab6(t1, c1 * 2 + h.act[0]);                       // seat 1: P(bet) or P(call)
+    h.act[1] = u1 < h.p[1] ? 1 : 0;
+    h.p[2] = tab6(t0, c0 * 2 + 1);                              // seat 0 facing a bet: P(call)
+    h.act[2] = u2 < h.p[2] ? 1 : 0;
+    const bool third = h.act[0] == 0 && h.act[1] == 1;          // pass, bet
+    h.n = third ? 3 : 2;
+    h.payoff = h.act[0] ? (h.act[1] ? 2 * sd : 1)
+                        : (h.act[1] ? (h.act[2] ? 2 * sd : -1) : sd);
     return h;
 }
 

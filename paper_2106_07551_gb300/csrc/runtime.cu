@@ -831,6 +831,16 @@ int malib_selftest_philox(malib_ctx* c, const uint32_t* ctr, uint64_t seed, uint
     return MALIB_OK;
 }
 
+int malib_philox_digest(malib_ctx* c, uint64_t seed, int64_t n, int32_t calls, uint32_t* out) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (n < 0 || calls < 0 || (n > 0 && (!out || !is_device_ptr(out))))
+        return fail(c, MALIB_EINVAL, "philox digest needs n >= 0, calls >= 0 and a device buffer");
+    CK(launch_philox_digest(seed, n, calls, out, c->stream), "philox digest kernel");
+    c->launches += n > 0;
+    return MALIB_OK;
+}
+
 int malib_selftest_det_expf(malib_ctx* c, const float* x, float* y, int64_t n) {
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);

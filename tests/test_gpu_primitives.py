@@ -33,6 +33,25 @@ def test_philox_bit_exact(ctx, orc, seed):
     np.testing.assert_array_equal(got, orc.philox(ctr, seed))
 
 
+@pytest.mark.parametrize("n,calls", [(1, 0), (1000, 7), (4099, 33)])
+def test_philox_digest(ctx, orc, n, calls):
+    """The throughput probe folds exactly the oracle's Philox words."""
+    torch = need_gpu()
+    seed = 0x0123456789ABCDEF
+    d_out = torch.zeros(n, dtype=torch.int32, device="cuda")
+    ctx.philox_digest(seed, calls, d_out)
+    ctx.sync()
+    got = d_out.cpu().numpy().view(np.uint32)
+    t = np.arange(n, dtype=np.uint64)
+    want = np.zeros(n, np.uint32)
+    for i in range(calls):
+        ctr = np.stack([(t & 0xFFFFFFFF).astype(np.uint32), (t >> 32).astype(np.uint32),
+                        np.full(n, i, np.uint32), np.zeros(n, np.uint32)], axis=1)
+        r = orc.philox(ctr, seed)
+        want ^= r[:, 0] ^ r[:, 1] ^ r[:, 2] ^ r[:, 3]
+    np.testing.assert_array_equal(got, want)
+
+
 def test_det_expf_bit_exact_and_near_expf(ctx, orc):
     torch = need_gpu()
     x = np.concatenate([np.linspace(-90, 89, 2_000_001, dtype=np.float32),
