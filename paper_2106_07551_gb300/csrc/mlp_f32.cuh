@@ -408,4 +408,156 @@ struct MlpF32T8 {
     }
 };
 
+// 256-row pass of one policy with H = 64 and 8x8 register tiles (256
+// threads): thread (tx, ty), tx = lane % 8 and ty = 4 warp + lane / 8,
+// computes rows ty + 32 i (i = 0..7) and columns {4tx..4tx+3} and
+// {32+4tx..32+4tx+3}, accumulating column pairs with packed fp32 FMAs. Per k
+// a thread issues 2 16-byte weight loads (4 column pairs), 8 duplications of
+// an input into a pair and 32 packed FMAs; its 8 inputs arrive as 2 16-byte
+// loads amortised over 4 k. A warp's 4 row groups are 4 consecutive rows,
+// which the bank-skewed strides (HS = 68, XS = 20 floats) put in different
+// banks; its 8 column groups read one 128-byte weight row. Layer 3 is folded
+// into layer 2's epilogue: packed dot products over the thread's column pairs,
+// then a reduce-scatter over the 8 lanes of a row group after which lane j
+// holds the logits of the group's row j.
+template <int IN, int A>
+struct MlpF32R8 {
+    static constexpr int H = 64;
+    static constexpr int kThreads = 256;
+    static constexpr int kRows = 256;
+    static constexpr int XS = (IN + 3) / 4 * 4;
+    static constexpr int HS = H + 4;
+    static constexpr int LS = (A + 3) / 4 * 4;
+    using u64 = unsigned long long;
+
+    __device__ static int col_group() { return threadIdx.x & 7; }
+    __device__ static int row_group() { return (threadIdx.x >> 5) * 4 + ((threadIdx.x >> 3) & 3); }
+
+    __device__ static void init(u64 (&acc)[8][4], const float* __restrict__ b, int c0, int c1) {
+        const ulonglong2 bA = *reinterpret_cast<const ulonglong2*>(b + c0);
+        const ulonglong2 bB = *reinterpret_cast<const ulonglong2*>(b + c1);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) { acc[i][0] = bA.x; acc[i][1] = bA.y; acc[i][2] = bB.x; acc[i][3] = bB.y; }
+    }
+
+    // acc += rows' inputs [4 k from xa] x W rows k0..k0+3 (kk < kmax)
+    __device__ static void block(u64 (&acc)[8][4], const float4 (&xa)[8], const float* __restrict__ W,
+                                 int k0, int kmax, int c0, int c1) {
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+            if (kk < kmax) {
+                const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(W + (k0 + kk) * H + c0);
+                const ulonglong2 wB = *reinterpret_cast<const ulonglong2*>(W + (k0 + kk) * H + c1);
+                u64 x2[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i)
+                    x2[i] = f2_dup(kk == 0 ? xa[i].x : kk == 1 ? xa[i].y : kk == 2 ? xa[i].z : xa[i].w);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][0], x2[i], wA.x);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][1], x2[i], wA.y);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][2], x2[i], wB.x);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) f2_fma(acc[i][3], x2[i], wB.y);
+            }
+        }
+    }
+
+    // Layer 1 into H1 (rows of X [256][XS]). Ends with __syncthreads.
+    __device__ static void layer1(const float* __restrict__ X, float* __restrict__ H1,
+                                  const float* __restrict__ W1T, const float* __restrict__ b1) {
+        const int tx = col_group(), ty = row_group();
+        const int c0 = tx * 4, c1 = H / 2 + tx * 4;
+        u64 acc[8][4];
+        init(acc, b1, c0, c1);
+#pragma unroll
+        for (int k0 = 0; k0 < IN; k0 += 4) {
+            float4 xa[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                xa[i] = *reinterpret_cast<const float4*>(X + (ty + 32 * i) * XS + k0);
+            block(acc, xa, W1T, k0, IN - k0, c0, c1);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            float* hr = H1 + (ty + 32 * i) * HS;
+            const u64 p0 = f2_relu(acc[i][0]), p1 = f2_relu(acc[i][1]);
+            const u64 p2 = f2_relu(acc[i][2]), p3 = f2_relu(acc[i][3]);
+            *reinterpret_cast<ulonglong2*>(hr + c0) = make_ulonglong2(p0, p1);
+            *reinterpret_cast<ulonglong2*>(hr + c1) = make_ulonglong2(p2, p3);
+        }
+        __syncthreads();
+    }
+
+    // Layers 2 and 3: H1 -> logits rows of LG [256][LS]. Ends with __syncthreads.
+    __device__ static void layer23(const float* __restrict__ H1, float* __restrict__ LG,
+                                   const float* __restrict__ W2T, const float* __restrict__ b2,
+                                   const float* __restrict__ W3, const float* __restrict__ b3) {
+        const int tx = col_group(), ty = row_group();
+        const int c0 = tx * 4, c1 = H / 2 + tx * 4;
+        u64 acc[8][4];
+        init(acc, b2, c0, c1);
+#pragma unroll 4
+        for (int k0 = 0; k0 < H; k0 += 4) {
+            float4 ha[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                ha[i] = *reinterpret_cast<const float4*>(H1 + (ty + 32 * i) * HS + k0);
+            block(acc, ha, W2T, k0, 4, c0, c1);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int p = 0; p < 4; ++p) acc[i][p] = f2_relu(acc[i][p]);
+        constexpr int V = 8 * A;                  // partial logits of this thread
+        float v0[V];
+#pragma unroll
+        for (int a = 0; a < A; ++a) {
+            const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(W3 + a * H + c0);
+            const ulonglong2 wB = *reinterpret_cast<const ulonglong2*>(W3 + a * H + c1);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                u64 t = 0ull;
+                f2_fma(t, acc[i][0], wA.x);
+                f2_fma(t, acc[i][1], wA.y);
+                f2_fma(t, acc[i][2], wB.x);
+                f2_fma(t, acc[i][3], wB.y);
+                const float2 q = f2_split(t);
+                v0[i * A + a] = q.x + q.y;
+            }
+        }
+        // Reduce-scatter over lane bits 2, 1, 0: at each level a lane keeps the
+        // half of its values selected by its lane bit and adds the partner's
+        // copy of that half; lane j ends with row j's A logits.
+        const int lane = threadIdx.x & 31;
+        const int l2 = (lane >> 2) & 1, l1 = (lane >> 1) & 1, l0 = lane & 1;
+        float v1[V / 2];
+#pragma unroll
+        for (int j = 0; j < V / 2; ++j) {
+            const float keep = l2 ? v0[V / 2 + j] : v0[j];
+            const float send = l2 ? v0[j] : v0[V / 2 + j];
+            v1[j] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+        }
+        float v2[V / 4];
+#pragma unroll
+        for (int j = 0; j < V / 4; ++j) {
+            const float keep = l1 ? v1[V / 4 + j] : v1[j];
+            const float send = l1 ? v1[j] : v1[V / 4 + j];
+            v2[j] = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+        }
+        float v3[A];
+#pragma unroll
+        for (int j = 0; j < A; ++j) {
+            const float keep = l0 ? v2[A + j] : v2[j];
+            const float send = l0 ? v2[j] : v2[A + j];
+            v3[j] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
+        }
+        float* lr = LG + (ty + 32 * (lane & 7)) * LS;
+#pragma unroll
+        for (int j = 0; j < A; ++j) lr[j] = v3[j] + b3[j];
+        __syncthreads();
+    }
+};
+
 }  // namespace malib

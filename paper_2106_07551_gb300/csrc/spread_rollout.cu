@@ -3,12 +3,13 @@
 // landmark to its closest agent, minus one per collision) under policy
 // combinations (Sec. 3.1: X ~ P(s, a, s' | a ~ Comb_t)), fp32 MLP policies.
 //
-// Work item = (combination, episode): the combination's block of
-// envs_per_pair environments for T steps. A persistent CTA takes a contiguous
-// range of items (combination-major, so the N policies are staged into shared
-// memory by bulk copy only when the combination changes). One thread steps one
-// environment with its state in registers; per step the N agents' observations
-// form N blocks of rows, each block one policy, run through the fp32 MLP
+// Work unit = (combination, episode pair): the combination's block of
+// envs_per_pair (<= 128) environments for T steps, in two episodes at once.
+// Each CTA takes a contiguous, equal-sized range of units (combination-major,
+// so the N policies are staged into shared memory by bulk copy only when the
+// combination changes). Thread t steps environment t % 128 of episode slot
+// t / 128 with its state in registers; per step agent i's observations of both
+// episodes form one 256-row pass of agent i's policy through the fp32 MLP
 // engine; trajectories leave as coalesced 16-byte stores.
 #include "device_common.cuh"
 #include "internal.h"
@@ -21,15 +22,17 @@ namespace {
 
 template <int N, int IN, int H>
 struct SpreadF32Smem {
-    using M = MlpF32<IN, H, 5>;
-    using L = typename M::L;
-    static constexpr int RPP = M::kRowsPerPass;
+    static_assert(H == 64, "the 256-row engine has 64 hidden units");
+    using M = MlpF32R8<IN, 5>;
+    using L = F32Layout<IN, H, 5>;
+    static constexpr int R = M::kRows;            // 2 episode slots x 128 envs
     static constexpr int kW = 0;
     static constexpr int kX = kW + N * L::kSize;
-    static constexpr int kH1 = kX + N * RPP * M::XS;
-    static constexpr int kLG = kH1 + RPP * M::HS;
-    static constexpr int kFloats = kLG + N * RPP * M::LS;
+    static constexpr int kH1 = kX + N * R * M::XS;
+    static constexpr int kLG = kH1 + R * M::HS;
+    static constexpr int kFloats = kLG + N * R * M::LS;
     static constexpr size_t kBytes = (size_t)kFloats * 4;
+    static_assert(kBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
 };
 
 template <int N, int IN, int H>
@@ -37,7 +40,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
     using SM = SpreadF32Smem<N, IN, H>;
     using M = typename SM::M;
     using L = typename SM::L;
-    constexpr int RPP = SM::RPP;
+    constexpr int R = SM::R;
     constexpr int XS = M::XS;           // == obs_pad
     extern __shared__ __align__(128) float smem[];
     float* Ws = smem + SM::kW;
@@ -47,22 +50,23 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
     __shared__ __align__(8) uint64_t bar;
 
     const int tid = threadIdx.x;
-    for (int i = tid; i < N * RPP * XS; i += blockDim.x) X[i] = 0.f;
+    const int slot = tid >> 7, v = tid & 127;        // episode slot, env of the combination
+    for (int i = tid; i < N * R * XS; i += blockDim.x) X[i] = 0.f;
     if (tid == 0) mbar_init(&bar, 1);
     __syncthreads();
     uint32_t parity = 0;
 
     const int epp = (int)(a.n_envs / a.n_pairs);
     const int T = a.episode_len;
-    const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
-    const int64_t per = (items + gridDim.x - 1) / gridDim.x;
-    const int64_t lo = (int64_t)blockIdx.x * per;
-    const int64_t hi = min(items, lo + per);
+    const int64_t upp = (a.n_episodes + 1) / 2;         // units (episode pairs) per combination
+    const int64_t units = (int64_t)a.n_pairs * upp;
+    const int64_t lo = units * blockIdx.x / gridDim.x;
+    const int64_t hi = units * (blockIdx.x + 1) / gridDim.x;
     int staged = -1;
 
-    for (int64_t it = lo; it < hi; ++it) {
-        const int pair = (int)(it / a.n_episodes);
-        const int64_t ep = it - (int64_t)pair * a.n_episodes;
+    for (int64_t u = lo; u < hi; ++u) {
+        const int pair = (int)(u / upp);
+        const int64_t ep0 = 2 * (u - (int64_t)pair * upp);
         if (pair != staged) {
             bool ok = true;
             for (int i = 0; i < N; ++i) {
@@ -90,8 +94,10 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
             staged = pair;
         }
 
-        const bool mine = tid < epp;
-        const int64_t env = (int64_t)pair * epp + tid;
+        const int64_t ep = ep0 + slot;
+        const int n_slots = ep0 + 1 < a.n_episodes ? 2 : 1;
+        const bool mine = slot < n_slots && v < epp;
+        const int64_t env = (int64_t)pair * epp + v;
         const uint64_t g = (uint64_t)ep * (uint64_t)a.n_envs + (uint64_t)env;
         SpreadEnv<N> s;
         if (mine) spread_reset<N>(s, g, a.seed);
@@ -102,7 +108,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                 for (int i = 0; i < N; ++i) {
                     float o[XS];
                     spread_obs<N, XS>(s, i, o);
-                    float4* xr = reinterpret_cast<float4*>(X + (i * RPP + tid) * XS);
+                    float4* xr = reinterpret_cast<float4*>(X + (i * R + tid) * XS);
 #pragma unroll
                     for (int q = 0; q < XS / 4; ++q)
                         xr[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
@@ -111,19 +117,24 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
             __syncthreads();
             // coalesced trajectory store of the observations: [ep][t][env][agent][XS]
             {
-                const int64_t row_base = ((ep * T + t) * a.n_envs + (int64_t)pair * epp) * N;
-                float4* dst = reinterpret_cast<float4*>(a.obs + row_base * XS);
-                const int n4 = epp * N * (XS / 4);
-                for (int q = tid; q < n4; q += blockDim.x) {
-                    const int v = q / (N * (XS / 4));
-                    const int rem = q - v * (N * (XS / 4));
+                constexpr int Q = N * (XS / 4);              // 16-byte chunks per env
+                const int n4 = epp * Q;
+                for (int q = tid; q < n_slots * n4; q += blockDim.x) {
+                    const int sl = q >= n4 ? 1 : 0;
+                    const int qq = q - sl * n4;
+                    const int ve = qq / Q;
+                    const int rem = qq - ve * Q;
                     const int i = rem / (XS / 4), c = rem - i * (XS / 4);
-                    dst[q] = *reinterpret_cast<const float4*>(X + (i * RPP + v) * XS + 4 * c);
+                    const int64_t row_base = (((ep0 + sl) * T + t) * a.n_envs + (int64_t)pair * epp) * N;
+                    reinterpret_cast<float4*>(a.obs + row_base * XS)[qq] =
+                        *reinterpret_cast<const float4*>(X + (i * R + sl * 128 + ve) * XS + 4 * c);
                 }
             }
-            for (int i = 0; i < N; ++i)
-                M::pass(X + i * RPP * XS, H1, LG + i * RPP * M::LS, Ws + i * L::kSize, 0,
-                        M::warp_first_row() < epp);
+            for (int i = 0; i < N; ++i) {
+                const float* w = Ws + i * L::kSize;
+                M::layer1(X + i * R * XS, H1, w + L::kW1T, w + L::kB1);
+                M::layer23(H1, LG + i * R * M::LS, w + L::kW2T, w + L::kB2, w + L::kW3, w + L::kB3);
+            }
             if (mine) {
                 int act[N];
                 float r[N];
@@ -132,9 +143,9 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                 for (int i = 0; i < N; ++i) {
                     float lg[5];
 #pragma unroll
-                    for (int k = 0; k < 5; ++k) lg[k] = LG[(i * RPP + tid) * M::LS + k];
-                    const float u = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
-                    act[i] = sample_masked<5>(lg, 0x1Fu, u);
+                    for (int k = 0; k < 5; ++k) lg[k] = LG[(i * R + tid) * M::LS + k];
+                    const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
+                    act[i] = sample_masked<5>(lg, 0x1Fu, uu);
                     if (a.logits)
 #pragma unroll
                         for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
@@ -160,8 +171,8 @@ cudaError_t launch_spread_nih(const RolloutArgs& a, int n_sm, cudaStream_t s) {
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SM::kBytes);
     if (err != cudaSuccess) return err;
-    const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
-    int64_t grid = items < n_sm ? items : n_sm;
+    const int64_t units = (int64_t)a.n_pairs * ((a.n_episodes + 1) / 2);
+    int64_t grid = units < n_sm ? units : n_sm;
     if (grid < 1) grid = 1;
     spread_rollout_f32_kernel<N, IN, H><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
     return cudaGetLastError();
