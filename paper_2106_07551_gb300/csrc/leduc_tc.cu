@@ -139,7 +139,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             if (!mbar_wait_bounded(&stage_bar, stage_par, kWaitLimitNs) && tid == 0)
                 atomicOr(a.err, ERRBIT_TIMEOUT);
             stage_par ^= 1u;
-            Eng::prefill_d1(smem, nullptr, tbase);          // the new policy's b1 into D1
             tc::fence_before_sync();
             Eng::sync();
             uint32_t done_bits = 0;

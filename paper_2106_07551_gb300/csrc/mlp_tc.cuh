@@ -15,9 +15,9 @@
 // 32-bit column, the lower k in the low half, row i in lane i).
 //
 // Tensor-memory columns (512 allocated):
-//   D1  [0, 256)    layer-1 accumulator (starts holding b1)
+//   D1  [0, 256)    layer-1 accumulator
 //   H1  [256, 384)  h1, packed
-//   D2a [384, 512)  layer-2 accumulator, outputs 0..127 (starts holding b2)
+//   D2a [384, 512)  layer-2 accumulator, outputs 0..127
 //   D2b [0, 128)    layer-2 accumulator, outputs 128..255 (D1's first half)
 //   H2  [128, 256)  h2, packed (D1's second half)
 //   D3  [384, 448)  layer 3 as four 16-column partial sums (D2a's first part)
@@ -26,7 +26,8 @@
 // output halves so that the first half's epilogue starts while the tensor core
 // computes the second; layer 3 likewise follows h2's halves. Thread 0 issues
 // the MMAs; the engine's 8 warps split each epilogue (warp w: TMEM lane
-// quarter w % 4, 64 of the 128 columns of a half).
+// quarter w % 4, 64 of the 128 columns of a half), which adds the layer's bias
+// (one packed add per pair of values) before ReLU and rounding.
 #pragma once
 
 #include <cstdint>
@@ -117,38 +118,6 @@ struct MlpTc {
         }
     }
 
-    // Writes n bias values (starting at bias) into every row of the accumulator
-    // columns [tcol, tcol + n): warp w writes lane quarter w % 4, half w / 4 of
-    // the n columns (n = 128 or 256). Waits for its stores.
-    __device__ static void prefill(const float* bias, uint32_t tbase, int tcol, int n) {
-        const int warp = threadIdx.x >> 5;
-        const int q = warp & 3, h = warp >> 2;
-        const int per = n / 2;
-#pragma unroll 1
-        for (int c = 0; c < per; c += 32) {
-            const int c0 = h * per + c;
-            uint32_t r[32];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const float4 b = kSmemBias ? *reinterpret_cast<const float4*>(bias + c0 + 4 * j)
-                                           : __ldg(reinterpret_cast<const float4*>(bias + c0 + 4 * j));
-                r[4 * j] = __float_as_uint(b.x);
-                r[4 * j + 1] = __float_as_uint(b.y);
-                r[4 * j + 2] = __float_as_uint(b.z);
-                r[4 * j + 3] = __float_as_uint(b.w);
-            }
-            tc::tmem_st32(tc::tmem_addr(tbase, 32 * q, tcol + c0), r);
-        }
-        tc::tmem_wait_st();
-    }
-
-    // Layer 1's bias into D1 before the first forward of a policy (after its
-    // weights and biases are staged). The caller orders it before the next MMA
-    // (tcgen05 fence before a barrier of the engine's threads).
-    __device__ static void prefill_d1(uint8_t* smem, const float* gbias, uint32_t tbase) {
-        prefill(kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias, tbase, kD1, H);
-    }
-
     // One 32-column chunk of an accumulator (in registers) -> relu -> bf16 pairs
     // -> 16 packed tensor-memory columns at taddr. With `bias`, the chunk's 32
     // bias values are added first.
@@ -173,9 +142,9 @@ struct MlpTc {
     }
 
     // One 128-column half of a layer's output: accumulator columns
-    // [dcol, dcol + 128) -> packed activations at [hcol, hcol + 64). Warp w
-    // takes lane quarter w % 4 and columns 64 (w / 4) .. of the half. bias (or
-    // null when the accumulator already holds it) covers the half's columns.
+    // [dcol, dcol + 128) plus bias -> packed activations at [hcol, hcol + 64).
+    // Warp w takes lane quarter w % 4 and columns 64 (w / 4) .. of the half;
+    // bias covers the half's columns.
     __device__ static void epilogue_half(uint32_t tbase, int dcol, int hcol, const float* bias) {
         const int warp = threadIdx.x >> 5;
         const int q = warp & 3, h = warp >> 2;
@@ -192,8 +161,7 @@ struct MlpTc {
     // their phase bits, kept by the caller across forwards. out(row, logits[16]) is called by the threads of warps 0-3 (thread
     // = row) for every row; the caller knows which rows hold observations.
     // gbias: the policy's biases in global memory (used when kSmemBias is false).
-    // All engine threads call. D1 must hold b1 (prefill_d1 before the first
-    // forward of a policy; every forward leaves it so for the next one).
+    // All engine threads call.
     // x_published: the caller's X writers already fenced (proxy) and the engine
     // has synchronised since, so MMA 1 issues at once; otherwise the forward
     // fences and synchronises first.
@@ -215,28 +183,26 @@ struct MlpTc {
         const uint32_t idesc_half = tc::instr_desc(128, H / 2, 1);
         const uint32_t idesc3 = tc::instr_desc(128, NOUT, 1);
         constexpr int kS = H / 16;                      // K steps of layers 2 and 3
-        // layer 1 (N = 256, K = K1) onto D1 (holding b1); meanwhile b2's first
-        // half goes into D2a
+        // layer 1 (N = 256, K = K1) into D1
         if (threadIdx.x == 0) {
             uint64_t da = tc::smem_desc(x_tile, kLboX, 128);
             uint64_t db = tc::smem_desc(s_w1, kLboW, 128);
             for (int s = 0; s < K1 / 16; ++s) {
-                tc::mma_bf16(tbase + kD1, da, db, idesc_full, true);
+                tc::mma_bf16(tbase + kD1, da, db, idesc_full, s != 0);
                 da += (2u * kLboX) >> 4;
                 db += (2u * kLboW) >> 4;
             }
             tc::mma_commit(bars);
         }
-        prefill(bias + H, tbase, kD2a, H / 2);
         wait_mma(bars, 0, parity, err);
         // h1, first half; then layer 2's outputs 0..127 over h1's first half
-        epilogue_half(tbase, kD1, kH1, nullptr);
+        epilogue_half(tbase, kD1, kH1, bias);
         handoff();
         if (threadIdx.x == 0)
-            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, true);
+            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, false);
         // h1, second half; then the rest of layer 2: outputs 0..127, then
         // 128..255 into D2b (D1's first half, already read)
-        epilogue_half(tbase, kD1 + H / 2, kH1 + H / 4, nullptr);
+        epilogue_half(tbase, kD1 + H / 2, kH1 + H / 4, bias + H / 2);
         handoff();
         if (threadIdx.x == 0) {
             issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, kS / 2, kS, idesc_half, true);
@@ -248,7 +214,7 @@ struct MlpTc {
         wait_mma(bars, 0, parity, err);                     // D2a
         // h2, first half (into H2, D1's second half, already read); then layer 3
         // over it: four chains of 4 K steps into D3 (D2a's columns, just read)
-        epilogue_half(tbase, kD2a, kH2, nullptr);
+        epilogue_half(tbase, kD2a, kH2, bias + H);
         handoff();
         auto mma3 = [&](int s0, int s1) {
             uint64_t db = tc::smem_desc(s_w3 + 2u * s0 * kLboW3, kLboW3, 128);
@@ -284,10 +250,8 @@ struct MlpTc {
             for (int i = 0; i < 16; ++i) v[i] += kSmemBias ? bias[2 * H + i] : __ldg(bias + 2 * H + i);
             out(row, v);
         }
-        // b1 into D1 for the next forward: D2b and H2, which share its columns,
-        // are consumed; each warp rewrites only its own lane quarter (the
-        // layer-3 chains it read live in other columns)
-        prefill(bias, tbase, kD1, H);
+        // the next forward's MMAs overwrite D1, D2b and H2's columns: every
+        // tensor-memory load of this one is complete before the barrier
         tc::fence_before_sync();
         sync();
     }

@@ -159,7 +159,6 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     atomicOr(a.err, ERRBIT_TIMEOUT);
                 stage_par ^= 1u;
                 staged = rd.pair;
-                Eng::prefill_d1(smem, gbias, tbase);   // the new policy's b1 into D1
                 tc::fence_before_sync();
                 Eng::sync();
             }
