@@ -32,7 +32,19 @@ FP32_LANES_PER_SM = 128
 # capture summarised under profiles/ (None until taken for the current kernel).
 # leduc_eval_f32_t8_kernel: profiles/leduc_eval_f32_t8_kernel_c2.md (the one-time
 # read of the population; independent of the hand count).
-NCU_TRAFFIC_PER_LAUNCH = {"leduc_eval_f32_t8_kernel": 1316096}
+# DRAM bytes (read + write) per launch of each workload's dominant kernel, from
+# ncu captures of small cases of the same kernels (profiles/*.md give the
+# commands). Trajectory writes grow with the episodes, so the spread figures are
+# scaled to the benchmark's episode counts (C3: 4 -> 100 episodes, C4: 1 -> 2);
+# the evaluation kernels' traffic is the staging of the population, which does
+# not grow with the hands per pair.
+NCU_TRAFFIC_PER_LAUNCH = {
+    "leduc_eval_f32_t8_kernel": 1351936 + 512,
+    "kuhn_eval_kernel": 13312,
+    "spread_rollout_f32_kernel<3,18,64>": (497920 + 43918080) * 25,
+    "leduc_eval_tc_kernel": 19300352 + 23296,
+    "spread_rollout_tc_kernel": (25526528 + 1919998000) * 2,
+}
 
 
 def mlp_flop(dims):
