@@ -11,8 +11,9 @@
 //  * warps 8-11 and 12-15, environment groups 0 and 1: two episodes of the
 //    combination in flight, one environment per thread. Every CTA keeps a
 //    replica of a group's 128 environments; per step a group builds agent k's
-//    observations (a bf16 tile for the engine, fp32 rows staged for contiguous
-//    trajectory stores), waits for the 8 agents' actions, applies them
+//    observations (a bf16 tile for the engine; each thread stores its fp32 row,
+//    one 144-byte run, to the trajectory), waits for the 8 agents' actions,
+//    applies them
 //    (identical IEEE operations in every CTA, identical bits) and writes agent
 //    k's trajectory (observation, action, reward; CTA 0 the done flags).
 // While the engine runs one group's tile, the other group steps its
@@ -33,17 +34,16 @@ namespace {
 
 constexpr int kN = 8;                        // agents = landmarks = cluster size
 constexpr int kObs = 34, kObsPad = 36, kK1 = 48, kA = 5;
-using Eng = MlpTc<kK1, 256, 16, false, /*kBarId=*/1>;   // biases read through L1
+using Eng = MlpTc<kK1, 256, 16, true, /*kBarId=*/1>;    // biases staged with the weights
 constexpr int kThreads = 512;
 constexpr int kEngineThreads = 256;
 constexpr int kGroups = 2;
 constexpr uint32_t kX = Eng::kSmemBytes;                          // observation tiles [group]
-constexpr uint32_t kStage = kX + kGroups * Eng::kXBytes;          // fp32 rows [group][128][36]
-constexpr uint32_t kActs = kStage + kGroups * 128 * kObsPad * 4;  // [group][parity][agent][env]
+constexpr uint32_t kActs = kX + kGroups * Eng::kXBytes;           // [group][parity][agent][env]
 constexpr uint32_t kSend = kActs + kGroups * 2 * kN * 128;        // this agent's actions [group][env]
 constexpr uint32_t kU = kSend + kGroups * 128;                    // decision uniforms [group][env]
 constexpr uint32_t kSmem = kU + kGroups * 128 * 4;
-static_assert(kX % 16 == 0 && kStage % 16 == 0 && kActs % 16 == 0 && kSend % 16 == 0 &&
+static_assert(kX % 16 == 0 && kActs % 16 == 0 && kSend % 16 == 0 &&
               kU % 16 == 0, "16-byte aligned regions");
 constexpr uint32_t kActTx = kN * 128;                             // action bytes received per step
 
@@ -136,7 +136,6 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ engine
         uint32_t stage_par = 0, mma_par = 0, x_bits = 0;
         int staged = -1;
-        const float* gbias = nullptr;
         for (int64_t it = lo; it < hi;) {
             const Round rd = round_at(it, hi, a.n_episodes);
             it = rd.next;
@@ -146,7 +145,6 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
             }
             if (rd.pair != staged) {
                 const float* policy = a.arena + a.pol_offset[a.pairs[rd.pair * kN + me]];
-                gbias = policy + Eng::kBias / 4;
                 Eng::sync();                 // the previous forwards are complete
                 if (tid == 0) {
                     fence_proxy_async_smem();
@@ -173,7 +171,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     const int64_t ep = rd.ep[g];
                     const float* u = ubuf + g * 128;
                     uint8_t* snd = send + g * 128;
-                    Eng::forward(smem, gbias, tbase, mma_bar, mma_par, a.err,
+                    Eng::forward(smem, nullptr, tbase, mma_bar, mma_par, a.err,
                                  [&](int row, const float* lg) {
                                      int act = 0;
                                      if (row < epp) {
@@ -208,7 +206,6 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         // ------------------------------------------------------------ environment groups
         const int g = (warp - 8) >> 2;
         const int e = tid - kEngineThreads - g * 128;     // environment within the block
-        float* stage = reinterpret_cast<float*>(smem + kStage) + g * 128 * kObsPad;
         uint8_t* xg = smem + kX + g * Eng::kXBytes;
         uint32_t act_bits = 0;                             // act_bar[g][p] phase: bit p
         for (int64_t it = lo; it < hi;) {
@@ -227,10 +224,12 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     ubuf[g * 128 + e] = u24(draw(gid, (uint32_t)t, me, a.seed).x);
                     float o[kObsPad];
                     spread_obs_dyn<kN, kObsPad>(s, (int)me, o);
-                    float4* srow = reinterpret_cast<float4*>(stage + e * kObsPad);
+                    // agent me's observation: [ep][t][env][agent][obs_pad], one 144-byte run
+                    float4* orow = reinterpret_cast<float4*>(
+                        a.obs + (((ep * T + t) * a.n_envs + env) * kN + me) * kObsPad);
 #pragma unroll
                     for (int q = 0; q < kObsPad / 4; ++q)
-                        srow[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                        orow[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
                     uint32_t w[kK1 / 2];
 #pragma unroll
                     for (int i = 0; i < kK1 / 2; ++i)
@@ -243,14 +242,6 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                 }
                 group_sync(g);
                 if (e == 0) mbar_arrive_release(&x_bar[g]);      // the tile goes to the engine
-                {   // observations of agent me: [ep][t][env][agent][obs_pad], 144-byte runs
-                    const int64_t base = ((ep * T + t) * a.n_envs + (int64_t)rd.pair * epp) * kN + me;
-                    const float4* src = reinterpret_cast<const float4*>(stage);
-                    for (int q = e; q < epp * (kObsPad / 4); q += 128) {
-                        const int v = q / (kObsPad / 4), c = q - v * (kObsPad / 4);
-                        reinterpret_cast<float4*>(a.obs + (base + (int64_t)v * kN) * kObsPad)[c] = src[q];
-                    }
-                }
                 // the 8 agents' actions of this step, from every engine of the cluster
                 if (!cl::wait_cluster_bounded(&act_bar[g][par], (act_bits >> par) & 1u, kWaitLimitNs) &&
                     e == 0)
@@ -272,7 +263,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                     a.reward[ix + me] = rm;
                     if (me == 0) a.done[(ep * T + t) * a.n_envs + env] = (t == T - 1) ? 1 : 0;
                 }
-                group_sync(g);       // the stage rows and tile are rewritten next step
+                group_sync(g);       // the tile is rewritten next step
             }
         }
     }
