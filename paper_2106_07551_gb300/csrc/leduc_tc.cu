@@ -322,7 +322,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                 if (a.d_done) a.d_done[rb + k] = 1;
                             }
                         }
-                        const int64_t k = (int64_t)atomicAdd(&next_k[g], 1ull);
+                    }
+                }
+                // finished hands take the group's next hands: one atomic per
+                // warp, ranks within the warp from a ballot
+                const bool need = placed && h.done;
+                const unsigned nm = __ballot_sync(0xffffffffu, need);
+                if (nm != 0u) {
+                    const int leader = __ffs(nm) - 1;
+                    unsigned long long base = 0ull;
+                    if (lane == leader) base = atomicAdd(&next_k[g], (unsigned long long)__popc(nm));
+                    base = __shfl_sync(0xffffffffu, base, leader);
+                    if (need) {
+                        const int64_t k = (int64_t)(base + (unsigned long long)__popc(nm & ((1u << lane) - 1u)));
                         e = e_lo + me + 2 * g + 4 * k;
                         live = e < e_hi;
                         if (live) {
