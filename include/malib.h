@@ -225,9 +225,10 @@ int malib_eval_payoff_ex(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pair
  * reserved the GPU's memory in its own caching pool, or a latency-critical loop
  * in which cudaMalloc/cudaFree would synchronise the device and stall other
  * streams. This call allocates nothing: it calls no cudaMalloc, cudaFree or
- * allocating library routine. Its scratch (per-pair payoff sums and a decision
- * counter) is a fixed file-scope device array of 128 KiB + 8 B that every GPU
- * loading the library holds until the process exits.
+ * allocating library routine. Its scratch (per-pair payoff sums, a decision
+ * counter and per-pair hand counters) is a fixed file-scope device array of
+ * 192 KiB + 8 B that every GPU loading the library holds until the process
+ * exits.
  *  - pair_ids and payoff_out must be DEVICE buffers (layouts as in
  *    malib_eval_payoff; no host staging). Host buffers give EINVAL.
  *  - n_pairs <= 8192 (the array's capacity); more gives EINVAL.

@@ -10,11 +10,12 @@
 // scratch (the per-pair payoff sums and the decision counter) lives in the
 // file-scope device array below instead of context-owned memory grown with
 // cudaMallocAsync, and it stages nothing (pair table and output must already
-// be device buffers).
+// be device buffers). The scratch also holds the per-pair hand counters from
+// which the fp32 Leduc kernel's CTAs claim hands.
 //
-// The array has room for kNoAllocMaxPairs pairs: (2 * 8192 + 1) x 8 bytes,
-// 128 KiB + 8 B, held by every GPU that loads the library until the process
-// exits. Every call shares it and it keeps the previous call's contents, so
+// The array has room for kNoAllocMaxPairs pairs: (3 * 8192 + 1) x 8 bytes
+// (sums, decision counter, hand counters), 192 KiB + 8 B, held by every GPU
+// that loads the library until the process exits. Every call shares it and it keeps the previous call's contents, so
 // each call clears it first; calls that overlap on the GPU (two streams, or two
 // contexts on one device) race on it and must be serialised by the caller.
 #include <cstdint>
@@ -30,7 +31,7 @@ namespace {
 constexpr int32_t kNoAllocMaxPairs = 8192;
 constexpr int kMaxDevices = 64;
 
-static __device__ __align__(256) unsigned long long g_noalloc_scratch[2 * kNoAllocMaxPairs + 1];
+static __device__ __align__(256) unsigned long long g_noalloc_scratch[3 * kNoAllocMaxPairs + 1];
 
 std::mutex g_mu;
 unsigned long long* g_scratch_addr[kMaxDevices] = {};
@@ -116,7 +117,8 @@ extern "C" int malib_eval_payoff_noalloc(malib_ctx* ctx, const int32_t* pair_ids
         a.seed = seed;
         a.acc = scratch;
         a.n_dec = scratch + 2 * (int64_t)n_pairs;
-        if ((e = launch_zero_u64(scratch, 2 * (int64_t)n_pairs + 1, v.stream)) == cudaSuccess)
+        a.work = scratch + 2 * (int64_t)n_pairs + 1;
+        if ((e = launch_zero_u64(scratch, 3 * (int64_t)n_pairs + 1, v.stream)) == cudaSuccess)
             e = v.env_kind == MALIB_ENV_KUHN ? launch_kuhn_eval(a, v.n_sm, v.stream)
                                              : launch_leduc_eval_f32(a, v.dims[1], v.n_sm, v.stream);
         if (e == cudaSuccess) e = launch_finalize(scratch, n_pairs, n_episodes, payoff_out, v.stream);

@@ -611,6 +611,7 @@ static cudaError_t launch_leduc_h(const EvalArgs& a, int n_sm, cudaStream_t s) {
 cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0) return cudaSuccess;
     if (hidden == 128) {
+        if (!a.work) return cudaErrorInvalidValue;       // the kernel claims hands from a.work
         cudaError_t err = cudaFuncSetAttribute(leduc_eval_f32_t8_kernel,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)t8::kBytes);
