@@ -464,7 +464,9 @@ struct MlpF32R8 {
         }
     }
 
-    // Layer 1 into H1 (rows of X [256][XS]). Ends with __syncthreads.
+    // Layer 1 into H1 (rows of X, XSTRIDE floats apart, 16-byte aligned). Ends
+    // with __syncthreads.
+    template <int XSTRIDE = XS>
     __device__ static void layer1(const float* __restrict__ X, float* __restrict__ H1,
                                   const float* __restrict__ W1T, const float* __restrict__ b1) {
         const int tx = col_group(), ty = row_group();
@@ -476,7 +478,7 @@ struct MlpF32R8 {
             float4 xa[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i)
-                xa[i] = *reinterpret_cast<const float4*>(X + (ty + 32 * i) * XS + k0);
+                xa[i] = *reinterpret_cast<const float4*>(X + (ty + 32 * i) * XSTRIDE + k0);
             block(acc, xa, W1T, k0, IN - k0, c0, c1);
         }
 #pragma unroll

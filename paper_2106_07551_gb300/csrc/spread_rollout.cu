@@ -10,7 +10,9 @@
 // combination changes). Thread t steps environment t % 128 of episode slot
 // t / 128 with its state in registers; per step agent i's observations of both
 // episodes form one 256-row pass of agent i's policy through the fp32 MLP
-// engine; trajectories leave as coalesced 16-byte stores.
+// engine. The observation tile is laid out [row][agent][obs_pad], the order of
+// the trajectory, so each episode's observations of a step leave shared memory
+// as one bulk copy; actions, rewards and done flags are stored per thread.
 #include "device_common.cuh"
 #include "internal.h"
 #include "mlp_f32.cuh"
@@ -51,7 +53,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 
     const int tid = threadIdx.x;
     const int slot = tid >> 7, v = tid & 127;        // episode slot, env of the combination
-    for (int i = tid; i < N * R * XS; i += blockDim.x) X[i] = 0.f;
+    for (int i = tid; i < R * N * XS; i += blockDim.x) X[i] = 0.f;
     if (tid == 0) mbar_init(&bar, 1);
     __syncthreads();
     uint32_t parity = 0;
@@ -86,7 +88,10 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                              (uint32_t)L::kSize * 4u, &bar);
             }
             if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs)) {
-                if (tid == 0) atomicOr(a.err, ERRBIT_TIMEOUT);
+                if (tid == 0) {
+                    atomicOr(a.err, ERRBIT_TIMEOUT);
+                    bulk_wait_all();
+                }
                 mbar_wait_bounded(&bar, parity, kWaitLimitNs);
                 return;
             }
@@ -108,31 +113,29 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                 for (int i = 0; i < N; ++i) {
                     float o[XS];
                     spread_obs<N, XS>(s, i, o);
-                    float4* xr = reinterpret_cast<float4*>(X + (i * R + tid) * XS);
+                    float4* xr = reinterpret_cast<float4*>(X + (tid * N + i) * XS);
 #pragma unroll
                     for (int q = 0; q < XS / 4; ++q)
                         xr[q] = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
                 }
+                fence_proxy_async_smem();                // the rows are read by bulk copies
             }
             __syncthreads();
-            // coalesced trajectory store of the observations: [ep][t][env][agent][XS]
-            {
-                constexpr int Q = N * (XS / 4);              // 16-byte chunks per env
-                const int n4 = epp * Q;
-                for (int q = tid; q < n_slots * n4; q += blockDim.x) {
-                    const int sl = q >= n4 ? 1 : 0;
-                    const int qq = q - sl * n4;
-                    const int ve = qq / Q;
-                    const int rem = qq - ve * Q;
-                    const int i = rem / (XS / 4), c = rem - i * (XS / 4);
+            // trajectory observations, [ep][t][env][agent][XS]: an episode's rows
+            // are contiguous in the tile and in the trajectory
+            if (tid == 0) {
+                for (int sl = 0; sl < n_slots; ++sl) {
                     const int64_t row_base = (((ep0 + sl) * T + t) * a.n_envs + (int64_t)pair * epp) * N;
-                    reinterpret_cast<float4*>(a.obs + row_base * XS)[qq] =
-                        *reinterpret_cast<const float4*>(X + (i * R + sl * 128 + ve) * XS + 4 * c);
+                    bulk_s2g(a.obs + row_base * XS, X + sl * 128 * N * XS, (uint32_t)(epp * N * XS * 4));
                 }
+                bulk_commit();
             }
             for (int i = 0; i < N; ++i) {
                 const float* w = Ws + i * L::kSize;
-                M::layer1(X + i * R * XS, H1, w + L::kW1T, w + L::kB1);
+                M::template layer1<N * XS>(X + i * XS, H1, w + L::kW1T, w + L::kB1);
+                // the copies have read the tile before the last pass's barrier;
+                // the tile is rewritten only after it
+                if (i == N - 1 && tid == 0) bulk_wait_read();
                 M::layer23(H1, LG + i * R * M::LS, w + L::kW2T, w + L::kB2, w + L::kW3, w + L::kB3);
             }
             if (mine) {
@@ -162,6 +165,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
             // LG is rewritten only after next step's first barrier.
         }
     }
+    if (tid == 0) bulk_wait_all();   // the trajectory copies have landed
 }
 
 template <int N, int IN, int H>
