@@ -41,9 +41,9 @@ FP32_LANES_PER_SM = 128
 NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1351936 + 512,
     "kuhn_eval_kernel": 13312,
-    "spread_rollout_f32_kernel<3,18,64>": (497920 + 43918080) * 25,
-    "leduc_eval_tc_kernel": 19300352 + 23296,
-    "spread_rollout_tc_kernel": (25526528 + 1919998000) * 2,
+    "spread_rollout_f32_kernel<3,18,64>": (428032 + 43692800) * 25,
+    "leduc_eval_tc_kernel": 19310848 + 25600,
+    "spread_rollout_tc_kernel": (18710272 + 1932523000) * 2,
 }
 
 
