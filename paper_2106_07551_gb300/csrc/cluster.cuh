@@ -59,6 +59,20 @@ __device__ __forceinline__ void st_async_v4(uint32_t remote_addr, uint4 v, uint3
         : "memory");
 }
 
+// One attempt at the phase `parity` of a local mbarrier whose transactions come
+// from peer CTAs (acquire at cluster scope); true when it has completed.
+__device__ __forceinline__ bool try_wait_cluster(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n"
+        " mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait (at most limit_ns) for the phase `parity` of a local mbarrier
 // whose transactions come from peer CTAs; acquires at cluster scope so the
 // peers' completed stores are visible. Returns false on expiry.

@@ -70,6 +70,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t x_bar[kGroups];    // a group's rows and headers
     __shared__ __align__(8) uint64_t lg_bar[kGroups];   // a group's logits
+    __shared__ __align__(8) uint64_t h1_bar[kGroups];   // h1 of a group's tile is in tensor memory
     __shared__ __align__(16) uint4 hdr[kGroups][2];     // [group][source CTA]: {rows here, live}
     __shared__ uint32_t tmem_base;
     __shared__ uint32_t dead_s;                         // a bounded wait expired
@@ -91,6 +92,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int g = 0; g < kGroups; ++g) {
             mbar_init(&x_bar[g], 1);
             mbar_init(&lg_bar[g], 1);
+            mbar_init(&h1_bar[g], 1);
             mbar_arrive_expect_tx(&x_bar[g], kXTx);         // armed for the first step
             mbar_arrive_expect_tx(&lg_bar[g], kLgTx);
         }
@@ -180,7 +182,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                                                 __float_as_uint(lg[2]), 0u),
                                                      cl::map(&lg_bar[g], src));
                                  },
-                                 smem_u32(smem + kX + g * kXBytes), /*x_published=*/true);
+                                 smem_u32(smem + kX + g * kXBytes), /*x_published=*/true, &h1_bar[g]);
                 }
             }
         }
@@ -189,7 +191,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const int g = (warp - 8) >> 2;                 // 0 or 1
         const int lt = tid - kEngineThreads - g * kSlots;
         const int gw = (warp - 8) & 3;                  // warp within the group
-        uint32_t lg_par = 0;
+        uint32_t lg_par = 0, h1_par = 0;
         uint8_t* xg = smem + kX + g * kXBytes;
         bool stop = false;
         for (int64_t u = cid; u < n_units && !stop; u += n_cl) {
@@ -266,11 +268,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 }
                 // the decision's uniform, drawn while the engines work
                 if (placed) u = u24(draw(gid, (uint32_t)t, (uint32_t)seat, a.seed).x);
-                // logits (or the end of the segment) from both engines
+                // logits (or the end of the segment) from both engines. While
+                // it waits, this group's leader issues the second output half of
+                // layer 2 of the group's tile in this CTA once the engine has h1
+                // in tensor memory (the engine's own MMA thread is then free for
+                // its epilogue share); a forward needs it before it can finish.
                 if (lt == 0) {
-                    if (!dead_s && !cl::wait_cluster_bounded(&lg_bar[g], lg_par, kWaitLimitNs)) {
-                        dead_s = 1u;
-                        atomicOr(a.err, ERRBIT_TIMEOUT);
+                    bool pend = true;
+                    const uint64_t t0 = globaltimer_ns();
+                    while (!dead_s) {
+                        if (pend && mbar_try_wait(&h1_bar[g], h1_par)) {
+                            h1_par ^= 1u;
+                            pend = false;
+                            tc::fence_after_sync();
+                            Eng::issue_layer2b(smem, tbase, &mma_bar[0]);
+                        }
+                        if (cl::try_wait_cluster(&lg_bar[g], lg_par)) break;
+                        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                            dead_s = 1u;
+                            atomicOr(a.err, ERRBIT_TIMEOUT);
+                        }
                     }
                     mbar_arrive_expect_tx(&lg_bar[g], kLgTx);
                     grp_flag[g] = dead_s ? 2u

@@ -156,6 +156,17 @@ struct MlpTc {
         pack_chunk(r1, bias ? bias + c + 32 : nullptr, tc::tmem_addr(tbase, 32 * q, hcol + c / 2 + 16));
     }
 
+    // The helper's part of a forward given h1_ready: layer 2's outputs
+    // 128..255 into D2b over all of h1, committed on bars[1]. Called by one
+    // thread after it has waited for h1_ready (and tcgen05-fenced after it).
+    // (Issuing layer 3 from the helper as well was slower: it sits on the
+    // forward's critical path, where the helper's response time shows.)
+    __device__ static void issue_layer2b(const uint8_t* smem, uint32_t tbase, uint64_t* bars) {
+        issue_ta(tbase + kD2b, tbase + kH1, smem_u32(smem + kW2) + (H / 2 / 8) * 128, kLboW, 0, H / 16,
+                 tc::instr_desc(128, H / 2, 1), false);
+        tc::mma_commit(bars + 1);
+    }
+
     // Full forward of the 128-row observation tile at shared-memory address
     // x_tile. bars: two mbarriers (count 1) for the MMA completions; parity:
     // their phase bits, kept by the caller across forwards. out(row, logits[16]) is called by the threads of warps 0-3 (thread
@@ -166,9 +177,13 @@ struct MlpTc {
     // has synchronised since, so MMA 1 issues at once; otherwise the forward
     // fences and synchronises first.
     template <class Out>
+    // h1_ready (optional, an mbarrier of count 1): instead of issuing layer
+    // 2's second output half itself, thread 0 arrives on it once h1 is complete
+    // and another, otherwise idle thread issues those MMAs (issue_layer2b), so
+    // that thread 0's warp is not held while the tensor core retires them.
     __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bars,
                                    uint32_t& parity, int* err, Out out, uint32_t x_tile,
-                                   bool x_published = false) {
+                                   bool x_published = false, uint64_t* h1_ready = nullptr) {
         const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
         const uint32_t s_w1 = smem_u32(smem + kW1), s_w2 = smem_u32(smem + kW2);
         const uint32_t s_w3 = smem_u32(smem + kW3);
@@ -207,9 +222,14 @@ struct MlpTc {
         if (threadIdx.x == 0) {
             issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, kS / 2, kS, idesc_half, true);
             tc::mma_commit(bars);                           // D2a complete
-            issue_ta(tbase + kD2b, tbase + kH1, s_w2 + (H / 2 / 8) * 128, kLboW, 0, kS, idesc_half,
-                     false);
-            tc::mma_commit(bars + 1);                       // D2b complete
+            if (h1_ready) {
+                tc::fence_before_sync();
+                mbar_arrive_release(h1_ready);              // D2b is issued by the helper
+            } else {
+                issue_ta(tbase + kD2b, tbase + kH1, s_w2 + (H / 2 / 8) * 128, kLboW, 0, kS, idesc_half,
+                         false);
+                tc::mma_commit(bars + 1);                   // D2b complete
+            }
         }
         wait_mma(bars, 0, parity, err);                     // D2a
         // h2, first half (into H2, D1's second half, already read); then layer 3
