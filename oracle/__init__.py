@@ -66,6 +66,11 @@ def _L():
                 "orc_spread_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                               C.c_int, C.c_int, C.c_int, i64, i64, i64, P, i32, i64,
                                               u64, P, P, P, P, P, C.c_int, C.c_float]),
+                "orc_adversary_reset": (None, [u64, u64, P]),
+                "orc_adversary_step": (None, [P, P, P]),
+                "orc_adversary_obs": (None, [P, P]),
+                "orc_adversary_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
+                                                 P, i32, i64, u64, P, P, P, P, P, C.c_int]),
             }
             for name, (res, args) in sig.items():
                 fn = getattr(lib, name)
@@ -250,5 +255,56 @@ def spread_rollout(params_list, dims, N, L, T, n_envs, pairs, n_episodes, seed, 
                             C.c_uint64(seed), _p(ext), _p(out["obs"]), _p(out["action"]),
                             _p(out["reward"]), _p(out["logits"]), n_threads,
                             -1.0 if local_ratio is None else float(local_ratio))
+    del arrs
+    return out
+
+
+# ---- simple adversary (App. B.1) ----
+# state: px,py,vx,vy of agents 0 (adversary), 1, 2; lx,ly of landmarks 0, 1;
+# then the target landmark's index (17 floats).
+ADV_N, ADV_L, ADV_OBS, ADV_STATE = 3, 2, 14, 17
+
+
+def adversary_reset(g: int, seed: int) -> np.ndarray:
+    st = np.zeros(ADV_STATE, np.float32)
+    _L().orc_adversary_reset(C.c_uint64(g), C.c_uint64(seed), _p(st))
+    return st
+
+
+def adversary_step(state: np.ndarray, actions) -> tuple[np.ndarray, np.ndarray]:
+    """One transition; rewards [adversary, good, good]."""
+    st = _c(state, np.float32).copy()
+    act = _c(actions, np.int32)
+    rew = np.zeros(ADV_N, np.float32)
+    _L().orc_adversary_step(_p(st), _p(act), _p(rew))
+    return st, rew
+
+
+def adversary_obs(state: np.ndarray) -> np.ndarray:
+    st = _c(state, np.float32)
+    out = np.zeros((ADV_N, ADV_OBS), np.float32)
+    _L().orc_adversary_obs(_p(st), _p(out))
+    return out
+
+
+def adversary_rollout(params_list, dims, T, n_envs, pairs, n_episodes, seed, bf16=False,
+                      env_lo=0, env_hi=None, ext_logits=None, n_threads=0):
+    """Rollout over envs [env_lo, env_hi) of the simple adversary (3 agents,
+    obs 14, 5 actions). Returns the arrays of spread_rollout."""
+    env_hi = n_envs if env_hi is None else env_hi
+    W = env_hi - env_lo
+    i, h1, h2, A = dims
+    assert i == ADV_OBS and A == 5
+    arrs, tbl = _param_table(params_list)
+    pairs = _c(pairs, np.int32).reshape(-1, ADV_N)
+    out = dict(obs=np.zeros((n_episodes, T, W, ADV_N, i), np.float32),
+               action=np.zeros((n_episodes, T, W, ADV_N), np.int8),
+               reward=np.zeros((n_episodes, T, W, ADV_N), np.float32),
+               logits=np.zeros((n_episodes, T, W, ADV_N, A), np.float32))
+    ext = None if ext_logits is None else _c(ext_logits, np.float32).reshape(n_episodes, T, W, ADV_N, A)
+    _L().orc_adversary_rollout(C.cast(tbl, C.c_void_p), h1, h2, int(bf16), T, n_envs, env_lo,
+                               env_hi, _p(pairs), pairs.shape[0], n_episodes, C.c_uint64(seed),
+                               _p(ext), _p(out["obs"]), _p(out["action"]), _p(out["reward"]),
+                               _p(out["logits"]), n_threads)
     del arrs
     return out

@@ -15,6 +15,10 @@
 //  * App. B.1 "Simple Spread": N agents cover N landmarks; reward is minus the
 //    sum over landmarks of the distance to the closest agent, minus one per
 //    collision.
+//  * App. B.1 "Simple Adversary": one adversary and two good agents, two
+//    landmarks of which one is the target; good agents are rewarded for being
+//    close to the target and for the adversary being far from it, the adversary
+//    (which is not told the target) for being close to it.
 // Kuhn and Leduc rules are not given in the paper; the textbook rules are used
 // (readings listed in the design doc, summarised at each function below).
 //
@@ -572,6 +576,75 @@ void spread_step(Spread& s, const int* action, float* reward, float local_ratio)
     }
 }
 
+// ---------------------------------------------------------------------------
+// Simple adversary (App. B.1; readings of its description, constants of the
+// spread scenario): agent 0 is the adversary, agents 1 and 2 the good agents,
+// two landmarks. Reset: agents and landmarks as for spread (same chance
+// counters), the target landmark = pick(x of the chance draw with step field
+// 0xC0000000, 2). Same dynamics as spread (no contact forces). Rewards after
+// the move, with d(.) the distance to the target:
+//   good agents: -min(d(p_1), d(p_2)) + d(p_0)      (shared)
+//   adversary:   -d(p_0)
+// each evaluated as written (one rounding per operation). Observation of agent
+// i (14 floats): velocity, position, target - p_i (zeros for the adversary,
+// which is not told the target), landmarks - p_i, other agents - p_i
+// (ascending j).
+// ---------------------------------------------------------------------------
+struct Adversary {
+    Spread s;
+    int target;
+};
+
+void adversary_reset(Adversary& a, uint64_t g, uint64_t seed) {
+    spread_reset(a.s, 3, 2, g, seed);
+    a.target = (int)pick(draw(g, 0xC0000000u, CHANCE, seed).x[0], 2);
+}
+
+void adversary_obs(const Adversary& a, int i, float* o) {
+    const Spread& s = a.s;
+    int k = 0;
+    o[k++] = s.vx[i]; o[k++] = s.vy[i];
+    o[k++] = s.px[i]; o[k++] = s.py[i];
+    if (i == 0) {
+        o[k++] = 0.0f; o[k++] = 0.0f;
+    } else {
+        o[k++] = s.lx[a.target] - s.px[i]; o[k++] = s.ly[a.target] - s.py[i];
+    }
+    for (int l = 0; l < 2; ++l) { o[k++] = s.lx[l] - s.px[i]; o[k++] = s.ly[l] - s.py[i]; }
+    for (int j = 0; j < 3; ++j) {
+        if (j == i) continue;
+        o[k++] = s.px[j] - s.px[i]; o[k++] = s.py[j] - s.py[i];
+    }
+}
+
+void adversary_step(Adversary& a, const int* action, float* reward) {
+    Spread& s = a.s;
+    for (int i = 0; i < 3; ++i) {
+        float fx = 0.0f, fy = 0.0f;
+        switch (action[i]) {
+            case 1: fx = 1.0f; break;
+            case 2: fx = -1.0f; break;
+            case 3: fy = 1.0f; break;
+            case 4: fy = -1.0f; break;
+            default: break;
+        }
+        s.vx[i] = s.vx[i] * 0.75f;
+        s.vy[i] = s.vy[i] * 0.75f;
+        s.vx[i] = s.vx[i] + fx * 0.1f;
+        s.vy[i] = s.vy[i] + fy * 0.1f;
+        s.px[i] = s.px[i] + s.vx[i] * 0.1f;
+        s.py[i] = s.py[i] + s.vy[i] * 0.1f;
+    }
+    const float tx = s.lx[a.target], ty = s.ly[a.target];
+    const float d_adv = dist2d(s.px[0], s.py[0], tx, ty);
+    const float d1 = dist2d(s.px[1], s.py[1], tx, ty);
+    const float d2 = dist2d(s.px[2], s.py[2], tx, ty);
+    const float d_good = d1 < d2 ? d1 : d2;
+    reward[0] = -d_adv;
+    reward[1] = -d_good + d_adv;
+    reward[2] = reward[1];
+}
+
 }  // namespace
 
 // ===========================================================================
@@ -785,6 +858,84 @@ void orc_spread_rollout(const float* const* params, int in, int h1, int h2, int 
             }
             float r[16];
             spread_step(s, act, r, local_ratio);
+            if (reward)
+                for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
+        }
+    });
+}
+
+// ---- Simple adversary ----
+// state: px,py,vx,vy of the 3 agents, lx,ly of the 2 landmarks, then the
+// target index as a float ([4*3 + 2*2 + 1] = 17 floats).
+static void adv_load(const float* state, Adversary& a) {
+    a.s.N = 3; a.s.L = 2;
+    for (int i = 0; i < 3; ++i) {
+        a.s.px[i] = state[4 * i]; a.s.py[i] = state[4 * i + 1];
+        a.s.vx[i] = state[4 * i + 2]; a.s.vy[i] = state[4 * i + 3];
+    }
+    for (int l = 0; l < 2; ++l) { a.s.lx[l] = state[12 + 2 * l]; a.s.ly[l] = state[12 + 2 * l + 1]; }
+    a.target = (int)state[16];
+}
+static void adv_store(const Adversary& a, float* state) {
+    for (int i = 0; i < 3; ++i) {
+        state[4 * i] = a.s.px[i]; state[4 * i + 1] = a.s.py[i];
+        state[4 * i + 2] = a.s.vx[i]; state[4 * i + 3] = a.s.vy[i];
+    }
+    for (int l = 0; l < 2; ++l) { state[12 + 2 * l] = a.s.lx[l]; state[12 + 2 * l + 1] = a.s.ly[l]; }
+    state[16] = (float)a.target;
+}
+
+void orc_adversary_reset(uint64_t g, uint64_t seed, float* state) {
+    Adversary a;
+    adversary_reset(a, g, seed);
+    adv_store(a, state);
+}
+
+void orc_adversary_step(float* state, const int32_t* action, float* reward) {
+    Adversary a;
+    adv_load(state, a);
+    adversary_step(a, action, reward);
+    adv_store(a, state);
+}
+
+void orc_adversary_obs(const float* state, float* obs /*[3][14]*/) {
+    Adversary a;
+    adv_load(state, a);
+    for (int i = 0; i < 3; ++i) adversary_obs(a, i, obs + i * 14);
+}
+
+// Rollout as orc_spread_rollout, for the simple adversary (N = 3, obs 14).
+void orc_adversary_rollout(const float* const* params, int h1, int h2, int bf16, int T,
+                           int64_t n_envs, int64_t env_lo, int64_t env_hi, const int32_t* pairs,
+                           int32_t n_pairs, int64_t n_episodes, uint64_t seed,
+                           const float* ext_logits, float* obs, int8_t* action, float* reward,
+                           float* logits, int n_threads) {
+    const int N = 3, in = 14, A = 5;
+    int64_t per = n_envs / n_pairs;
+    int64_t W = env_hi - env_lo;
+    parallel_for(W * n_episodes, n_threads, [&](int64_t job) {
+        int64_t ep = job / W, e = env_lo + job % W;
+        int64_t row = e / per;
+        Adversary adv;
+        uint64_t g = (uint64_t)ep * (uint64_t)n_envs + (uint64_t)e;
+        adversary_reset(adv, g, seed);
+        for (int t = 0; t < T; ++t) {
+            int act[3];
+            for (int i = 0; i < N; ++i) {
+                int64_t idx = ((ep * T + t) * W + (e - env_lo)) * N + i;
+                float o[14], lg[8];
+                adversary_obs(adv, i, o);
+                Mlp m{params[pairs[row * N + i]], in, h1, h2, A, bf16};
+                mlp_logits(m, o, lg);
+                uint8_t legal[8] = {1, 1, 1, 1, 1, 1, 1, 1};
+                float u = uniform24(draw(g, (uint32_t)t, (uint32_t)i, seed).x[0]);
+                act[i] = sample_masked(ext_logits ? ext_logits + idx * A : lg, legal, A, u);
+                if (obs) std::memcpy(obs + idx * in, o, sizeof(float) * in);
+                if (logits) std::memcpy(logits + idx * A, lg, sizeof(float) * A);
+                if (action) action[idx] = (int8_t)act[i];
+            }
+            float r[3];
+            adversary_step(adv, act, r);
             if (reward)
                 for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
         }
