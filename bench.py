@@ -58,7 +58,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "leduc_bf16", "spread8",
+    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "leduc_bf16", "spread8",
                                            "meta"],
                     default="leduc")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -171,6 +171,8 @@ def workload(name: str, rank: int, hands=None):
         w = workloads.config(1, **over)
     elif name == "spread8":
         w = workloads.config(4, **({"n_episodes": 2} if hands is None else over))
+    elif name == "adversary3":
+        w = workloads.adversary(n_envs=4096, pop=16, n_episodes=100 if hands is None else hands)
     else:
         w = workloads.config(3, **({"n_episodes": 100} if hands is None else over))
     return w
@@ -189,6 +191,10 @@ def config_of(w, name):
                 "l2": "flushed (256 MiB write) before every timed step"}
     if name == "spread8":
         return {"workload": f"spread_n8_65536env_mlp34-256-256-5_bf16_{w.n_episodes}episodes",
+                "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
+                "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
+    if name == "adversary3":
+        return {"workload": f"simple_adversary_4096env_mlp14-64-64-5_f32_{w.n_episodes}episodes",
                 "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
                 "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
     if name == "kuhn":
@@ -302,7 +308,7 @@ def run_ours(args):
     d_pairs = torch.from_numpy(w.pair_ids).to(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     seed0 = w.seed + 1_000_003 * rank
-    rollout = args.workload in ("spread3", "spread8")
+    rollout = args.workload in ("spread3", "spread8", "adversary3")
     if rollout:
         traj = alloc_traj(spec, w.n_episodes)
         steps_per_call = w.n_envs * w.episode_len * w.n_episodes
@@ -363,6 +369,7 @@ def run_ours(args):
         if kern_n else 0.0
     kname = {"leduc": "leduc_eval_f32_t8_kernel", "kuhn": "kuhn_eval_kernel",
              "spread3": "spread_rollout_f32_kernel<3,18,64>",
+             "adversary3": "spread_rollout_f32_kernel<3,14,64,true>",
              "leduc_bf16": "leduc_eval_tc_kernel",
              "spread8": "spread_rollout_tc_kernel"}[args.workload]
     basis = (f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"

@@ -49,7 +49,8 @@ typedef enum malib_status {
 typedef enum malib_env_kind {
     MALIB_ENV_KUHN = 1,       /* Kuhn poker: 3 cards, ante 1, one bet of 1, 2 seats */
     MALIB_ENV_LEDUC = 2,      /* Leduc hold'em: 6 cards, 2 rounds, raises 2 then 4 */
-    MALIB_ENV_SPREAD = 3      /* cooperative particle spread (App. B.1) */
+    MALIB_ENV_SPREAD = 3,     /* cooperative particle spread (App. B.1) */
+    MALIB_ENV_ADVERSARY = 4   /* simple adversary (App. B.1): 1 adversary, 2 good agents */
 } malib_env_kind;
 
 typedef enum malib_policy_kind {
@@ -76,7 +77,10 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  *   LEDUC:  n_agents 2, obs_dim 17, n_actions 3 (fold, call/check, raise)
  *   SPREAD: n_agents = n_landmarks in [2, 16], obs_dim >= 4 + 4 n_agents - 2,
  *           n_actions 5 (noop, +x, -x, +y, -y), episode_len >= 1
- * n_envs is the number of parallel environments of a rollout (SPREAD).
+ *   ADVERSARY: n_agents 3 (agent 0 the adversary, 1 and 2 the good agents),
+ *           n_landmarks 2, obs_dim 14, n_actions 5, episode_len >= 1
+ * n_envs is the number of parallel environments of a rollout (SPREAD,
+ * ADVERSARY).
  * SPREAD reward of agent i after a step (App. B.1), with cover = sum over
  * landmarks of the distance to the nearest agent and coll_i = the number of
  * agents closer than 0.3 to agent i:
@@ -84,6 +88,12 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  *   flags & MALIB_SPREAD_LOCAL_RATIO: r_i = -((1 - local_ratio) cover + local_ratio coll_i)
  * (the paper's local_ratio, 0 <= local_ratio <= 1; each operation rounded in
  * fp32 in the order written).
+ * ADVERSARY (App. B.1 simple adversary): the spread dynamics; at reset one of
+ * the two landmarks is drawn as the target. With d(.) the distance to the
+ * target after the step: adversary r_0 = -d(p_0); good agents r_1 = r_2 =
+ * -min(d(p_1), d(p_2)) + d(p_0). Observation of agent i: velocity, position,
+ * target - p_i (zeros for the adversary, which is not told the target), the two
+ * landmarks - p_i, the other agents - p_i (ascending).
  */
 typedef struct malib_env_spec {
     int32_t env_kind;

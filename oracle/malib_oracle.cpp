@@ -29,7 +29,9 @@
 //
 // Parity status: Philox, det_expf, Kuhn (exact enumeration), Leduc (tree
 // enumeration, hand-worked hands), spread (closed-form single steps and
-// invariants) are pinned by the CPU tests; spread episode returns beyond those
+// invariants) and the simple adversary (hand-worked geometry, the reward
+// identity against fp64, the spread dynamics and reset, symmetries) are pinned
+// by the CPU tests; episode returns of the particle scenarios beyond those
 // invariants are "parity unpinned" (no closed form exists).
 
 #include <algorithm>

@@ -16,7 +16,7 @@ MALIB_ESTATE, MALIB_ETIMEOUT, MALIB_EUNSUPPORTED = -4, -5, -6
 STATUS_NAMES = {0: "OK", -1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ESTATE", -5: "ETIMEOUT",
                 -6: "EUNSUPPORTED"}
 
-MALIB_ENV_KUHN, MALIB_ENV_LEDUC, MALIB_ENV_SPREAD = 1, 2, 3
+MALIB_ENV_KUHN, MALIB_ENV_LEDUC, MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY = 1, 2, 3, 4
 MALIB_POL_TABULAR, MALIB_POL_MLP = 1, 2
 MALIB_F32, MALIB_BF16 = 0, 1
 MALIB_DUMP_LOGITS, MALIB_EXACT_EXPECTATION, MALIB_SPREAD_LOCAL_RATIO = 1, 2, 4

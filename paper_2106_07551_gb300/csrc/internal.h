@@ -79,6 +79,7 @@ struct EvalArgs {
 };
 
 struct RolloutArgs {
+    int32_t env_kind;            // MALIB_ENV_SPREAD or MALIB_ENV_ADVERSARY
     const float* arena;
     const int64_t* pol_offset;
     int32_t n_pol;
@@ -158,5 +159,6 @@ cudaError_t launch_lp_nash(const double* P, int32_t G, int32_t m, int32_t n, int
 
 bool leduc_f32_supported(int hidden);
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden);
+bool adversary_f32_supported(int hidden);
 
 }  // namespace malib

@@ -152,6 +152,12 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
             if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
             break;
         }
+        case MALIB_ENV_ADVERSARY:
+            if (s->n_agents != 3 || s->n_landmarks != 2 || s->obs_dim != 14 || s->n_actions != 5)
+                return fail(c, MALIB_EINVAL,
+                            "adversary spec needs n_agents 3, n_landmarks 2, obs_dim 14, n_actions 5");
+            if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
+            break;
         default:
             return fail(c, MALIB_EINVAL, "unknown env_kind %d", s->env_kind);
     }
@@ -471,7 +477,7 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
     if (n < 0 || (n > 0 && (!pols || !ids_out))) return fail(c, MALIB_EINVAL, "bad policy list");
     if (c->has_pop && !same_env(c->spec, *spec))
         return fail(c, MALIB_ESTATE, "population was loaded for a different environment");
-    const bool poker = spec->env_kind != MALIB_ENV_SPREAD;
+    const bool poker = spec->env_kind == MALIB_ENV_KUHN || spec->env_kind == MALIB_ENV_LEDUC;
     std::vector<std::vector<float>> converted(n);
     std::vector<PolicyRec> recs(n);
     for (int i = 0; i < n; ++i) {
@@ -714,8 +720,9 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
     if (!same_env(c->spec, *spec))
         return fail(c, MALIB_ESTATE, "rollout spec differs from the population's environment");
-    if (spec->env_kind != MALIB_ENV_SPREAD)
-        return fail(c, MALIB_EUNSUPPORTED, "rollout is built for the particle spread environment");
+    const bool adv = spec->env_kind == MALIB_ENV_ADVERSARY;
+    if (spec->env_kind != MALIB_ENV_SPREAD && !adv)
+        return fail(c, MALIB_EUNSUPPORTED, "rollout is built for the particle environments");
     if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");
     if (spec->n_envs < 1 || spec->n_envs % n_pairs != 0)
         return fail(c, MALIB_EINVAL, "n_envs (%lld) must be a positive multiple of n_pairs (%d)",
@@ -732,10 +739,11 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
         if (((uintptr_t)p & 15u) != 0) return fail(c, MALIB_EINVAL, "trajectory buffers must be 16-byte aligned");
     }
     const int64_t epp = spec->n_envs / n_pairs;
-    const bool use_tc = c->tc_layout && spread_tc_supported(spec->n_agents, spec->obs_dim,
-                                                            spec->n_actions, epp);
-    if (!use_tc && (c->pol_dtype != MALIB_F32 || c->dims[1] != c->dims[2] ||
-                    !spread_f32_supported(spec->n_agents, spec->obs_dim, c->dims[1]) || epp > 128))
+    const bool use_tc = !adv && c->tc_layout && spread_tc_supported(spec->n_agents, spec->obs_dim,
+                                                                    spec->n_actions, epp);
+    const bool f32_ok = adv ? adversary_f32_supported(c->dims[1])
+                            : spread_f32_supported(spec->n_agents, spec->obs_dim, c->dims[1]);
+    if (!use_tc && (c->pol_dtype != MALIB_F32 || c->dims[1] != c->dims[2] || !f32_ok || epp > 128))
         return fail(c, MALIB_EUNSUPPORTED,
                     "no spread kernel for %s N=%d obs %d hidden %d with %lld envs per combination",
                     c->pol_dtype == MALIB_BF16 ? "bf16" : "fp32", spec->n_agents, spec->obs_dim,
@@ -747,6 +755,7 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
                          &dpairs)) != MALIB_OK)
         return r;
     RolloutArgs a{};
+    a.env_kind = spec->env_kind;
     a.arena = c->arena;
     a.pol_offset = c->d_off;
     a.n_pol = (int32_t)c->pols.size();

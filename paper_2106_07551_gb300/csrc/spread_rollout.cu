@@ -13,6 +13,9 @@
 // engine. The observation tile is laid out [row][agent][obs_pad], the order of
 // the trajectory, so each episode's observations of a step leave shared memory
 // as one bulk copy; actions, rewards and done flags are stored per thread.
+#include <type_traits>
+
+#include "adversary_env.cuh"
 #include "device_common.cuh"
 #include "internal.h"
 #include "mlp_f32.cuh"
@@ -37,8 +40,11 @@ struct SpreadF32Smem {
     static_assert(kBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
 };
 
-template <int N, int IN, int H>
+// kAdv: false - cooperative spread (N agents, N landmarks); true - the simple
+// adversary (N = 3, two landmarks, obs 14).
+template <int N, int IN, int H, bool kAdv = false>
 __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs a) {
+    static_assert(!kAdv || (N == 3 && IN == kAdvObs), "the simple adversary has 3 agents, obs 14");
     using SM = SpreadF32Smem<N, IN, H>;
     using M = typename SM::M;
     using L = typename SM::L;
@@ -104,15 +110,19 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
         const bool mine = slot < n_slots && v < epp;
         const int64_t env = (int64_t)pair * epp + v;
         const uint64_t g = (uint64_t)ep * (uint64_t)a.n_envs + (uint64_t)env;
-        SpreadEnv<N> s;
-        if (mine) spread_reset<N>(s, g, a.seed);
+        std::conditional_t<kAdv, AdvEnv, SpreadEnv<N>> s;
+        if (mine) {
+            if constexpr (kAdv) adv_reset(s, g, a.seed);
+            else spread_reset<N>(s, g, a.seed);
+        }
 
         for (int t = 0; t < T; ++t) {
             if (mine) {
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
                     float o[XS];
-                    spread_obs<N, XS>(s, i, o);
+                    if constexpr (kAdv) adv_obs<XS>(s, i, o);
+                    else spread_obs<N, XS>(s, i, o);
                     float4* xr = reinterpret_cast<float4*>(X + (tid * N + i) * XS);
 #pragma unroll
                     for (int q = 0; q < XS / 4; ++q)
@@ -153,7 +163,8 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 #pragma unroll
                         for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
                 }
-                spread_step<N>(s, act, r, a.local_ratio);
+                if constexpr (kAdv) adv_step(s, act, r);
+                else spread_step<N>(s, act, r, a.local_ratio);
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
                     a.action[ix + i] = (uint8_t)act[i];
@@ -168,21 +179,23 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
     if (tid == 0) bulk_wait_all();   // the trajectory copies have landed
 }
 
-template <int N, int IN, int H>
+template <int N, int IN, int H, bool kAdv = false>
 cudaError_t launch_spread_nih(const RolloutArgs& a, int n_sm, cudaStream_t s) {
     using SM = SpreadF32Smem<N, IN, H>;
-    cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H>,
+    cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H, kAdv>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SM::kBytes);
     if (err != cudaSuccess) return err;
     const int64_t units = (int64_t)a.n_pairs * ((a.n_episodes + 1) / 2);
     int64_t grid = units < n_sm ? units : n_sm;
     if (grid < 1) grid = 1;
-    spread_rollout_f32_kernel<N, IN, H><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
+    spread_rollout_f32_kernel<N, IN, H, kAdv><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
     return cudaGetLastError();
 }
 
 }  // namespace
+
+bool adversary_f32_supported(int hidden) { return hidden == 64; }
 
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden) {
     return n_agents == 3 && obs_dim == 18 && hidden == 64;
@@ -190,6 +203,10 @@ bool spread_f32_supported(int n_agents, int obs_dim, int hidden) {
 
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0 || a.n_episodes == 0) return cudaSuccess;
+    if (a.env_kind == MALIB_ENV_ADVERSARY) {
+        if (hidden == 64) return launch_spread_nih<3, kAdvObs, 64, true>(a, n_sm, s);
+        return cudaErrorInvalidValue;
+    }
     if (a.n_agents == 3 && a.obs_dim == 18 && hidden == 64) return launch_spread_nih<3, 18, 64>(a, n_sm, s);
     return cudaErrorInvalidValue;
 }
