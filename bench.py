@@ -35,14 +35,16 @@ FP32_LANES_PER_SM = 128
 # DRAM bytes (read + write) per launch of each workload's dominant kernel, from
 # ncu captures of small cases of the same kernels (profiles/*.md give the
 # commands). Trajectory writes grow with the episodes, so the spread figures are
-# scaled to the benchmark's episode counts (C3: 4 -> 100 episodes, C4: 1 -> 2);
+# scaled to the benchmark's episode counts (C3 and the simple adversary: 4 -> 100
+# episodes, C4: 1 -> 2);
 # the evaluation kernels' traffic is the staging of the population, which does
 # not grow with the hands per pair.
 NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1351936 + 512,
     "kuhn_eval_kernel": 13312,
     "spread_rollout_f32_kernel<3,18,64>": (428032 + 43692800) * 25,
-    "leduc_eval_tc_kernel": 19310848 + 25600,
+    "leduc_eval_tc_kernel": 19304960 + 28416,
+    "spread_rollout_f32_kernel<3,14,64,true>": (444160 + 24321792) * 25,
     "spread_rollout_tc_kernel": (18710272 + 1932523000) * 2,
 }
 
