@@ -345,6 +345,14 @@ int malib_selftest_philox(malib_ctx* ctx, const uint32_t* ctr, uint64_t seed, ui
  * or a host pointer; asynchronous on the context's stream. */
 int malib_philox_digest(malib_ctx* ctx, uint64_t seed, int64_t n, int32_t calls, uint32_t* out);
 
+/* Bounded-wait self-test: one device thread waits at most limit_ns
+ * (1 <= limit_ns <= 1e9) for an mbarrier phase; with arrive = 0 nothing
+ * completes it, the wait expires and the kernel records a timeout, which the
+ * next malib_sync reports as MALIB_ETIMEOUT (the context stays usable); with
+ * arrive != 0 the thread completes the phase itself first and no error is
+ * recorded. Every wait of the library's kernels is bounded the same way. */
+int malib_selftest_wait(malib_ctx* ctx, int32_t arrive, int64_t limit_ns);
+
 /* The kernels' deterministic exp (Cody-Waite reduction, degree-7 Taylor) on n
  * device floats, and the masked inverse-CDF draw on n rows of A <= 8 logits
  * (device: logits [n][A], legal uint8 [n][A], u [n], out int32 [n]). */

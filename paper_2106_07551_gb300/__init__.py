@@ -283,6 +283,12 @@ class Context:
                self.lib.malib_philox_digest(self.handle, seed, int(out.numel()), int(calls),
                                             _ptr(out)))
 
+    def selftest_wait(self, arrive, limit_ns):
+        """A bounded device wait that expires (arrive False) or completes (True);
+        the outcome is reported by the next sync()."""
+        _check(self.lib, self.handle, self.lib.malib_selftest_wait(self.handle, int(bool(arrive)),
+                                                                   int(limit_ns)))
+
     def selftest_det_expf(self, x, y):
         _check(self.lib, self.handle,
                self.lib.malib_selftest_det_expf(self.handle, _ptr(x), _ptr(y), int(x.numel())))

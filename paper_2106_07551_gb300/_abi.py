@@ -27,7 +27,7 @@ EXPORTS = (
     "malib_pop_load", "malib_pop_reset", "malib_rollout", "malib_eval_payoff",
     "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "malib_eval_stats", "malib_launch_count",
     "malib_set_timing", "malib_main_kernel_ms",
-    "malib_selftest_philox", "malib_philox_digest", "malib_selftest_det_expf",
+    "malib_selftest_philox", "malib_philox_digest", "malib_selftest_wait", "malib_selftest_det_expf",
     "malib_selftest_sample",
     "malib_selftest_mma", "malib_meta_fictitious_play", "malib_meta_lp_nash",
     "malib_meta_aggregate", "malib_exploitability",
@@ -90,6 +90,7 @@ def load(path: str | None = None):
             "malib_main_kernel_ms": (C.c_double, [P, C.POINTER(C.c_int64), C.c_int]),
             "malib_selftest_philox": (C.c_int, [P, P, u64, P, i64]),
             "malib_philox_digest": (C.c_int, [P, u64, i64, i32, P]),
+            "malib_selftest_wait": (C.c_int, [P, i32, i64]),
             "malib_selftest_det_expf": (C.c_int, [P, P, P, i64]),
             "malib_selftest_sample": (C.c_int, [P, P, P, P, i32, P, i64]),
             "malib_selftest_mma": (C.c_int, [P, i32, P, P, P, i32, i32]),

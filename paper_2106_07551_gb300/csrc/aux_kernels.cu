@@ -63,6 +63,17 @@ __global__ void __launch_bounds__(256) philox_digest_kernel(uint64_t seed, int64
     out[t] = acc;
 }
 
+// Bounded-wait self-test: one thread waits at most limit_ns for the first
+// phase of an mbarrier of count 1 that it arrives on itself (arrive) or that
+// nothing arrives on; an expired wait sets ERRBIT_TIMEOUT and the kernel ends.
+__global__ void wait_selftest_kernel(bool arrive, uint64_t limit_ns, int* err) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x != 0) return;
+    mbar_init(&bar, 1);
+    if (arrive) mbar_arrive_release(&bar);
+    if (!mbar_wait_bounded(&bar, 0, limit_ns)) atomicOr(err, ERRBIT_TIMEOUT);
+}
+
 __global__ void det_expf_kernel(const float* x, float* y, int64_t n) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x)
@@ -119,6 +130,11 @@ cudaError_t launch_philox_digest(uint64_t seed, int64_t n, int calls, uint32_t* 
     const int64_t blocks = (n + 255) / 256;
     if (blocks > 0x7FFFFFFF) return cudaErrorInvalidValue;
     philox_digest_kernel<<<(unsigned)blocks, 256, 0, s>>>(seed, n, calls, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_selftest_wait(bool arrive, uint64_t limit_ns, int* err, cudaStream_t s) {
+    wait_selftest_kernel<<<1, 32, 0, s>>>(arrive, limit_ns, err);
     return cudaGetLastError();
 }
 

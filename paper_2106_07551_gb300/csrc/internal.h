@@ -112,6 +112,7 @@ bool spread_tc_supported(int n_agents, int obs_dim, int n_actions, int64_t envs_
 cudaError_t launch_zero_u64(unsigned long long* p, int64_t n, cudaStream_t s);
 cudaError_t launch_finalize(const unsigned long long* acc, int32_t n_pairs, int64_t n_episodes,
                             double* out, cudaStream_t s);
+cudaError_t launch_selftest_wait(bool arrive, uint64_t limit_ns, int* err, cudaStream_t s);
 cudaError_t launch_philox_digest(uint64_t seed, int64_t n, int calls, uint32_t* out,
                                  cudaStream_t s);
 cudaError_t launch_selftest_philox(const uint32_t* ctr, uint64_t seed, uint32_t* out, int64_t n,

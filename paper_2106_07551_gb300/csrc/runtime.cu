@@ -313,7 +313,7 @@ int read_device_errors(malib_ctx* c) {
     if (h) {
         CK(cudaMemsetAsync(c->d_err, 0, 4, c->stream), "error flag");
         if (h & ERRBIT_TIMEOUT)
-            return fail(c, MALIB_ETIMEOUT, "a bounded device wait expired (staging copy)");
+            return fail(c, MALIB_ETIMEOUT, "a bounded device wait expired");
         if (h & ERRBIT_BAD_PAIR)
             return fail(c, MALIB_EINVAL, "a device pair table held an invalid policy id or seat");
         if (h & ERRBIT_NOT_CONVERGED)
@@ -847,6 +847,16 @@ int malib_philox_digest(malib_ctx* c, uint64_t seed, int64_t n, int32_t calls, u
         return fail(c, MALIB_EINVAL, "philox digest needs n >= 0, calls >= 0 and a device buffer");
     CK(launch_philox_digest(seed, n, calls, out, c->stream), "philox digest kernel");
     c->launches += n > 0;
+    return MALIB_OK;
+}
+
+int malib_selftest_wait(malib_ctx* c, int32_t arrive, int64_t limit_ns) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (limit_ns < 1 || limit_ns > 1000000000)
+        return fail(c, MALIB_EINVAL, "limit_ns must lie in [1, 1e9]");
+    CK(launch_selftest_wait(arrive != 0, (uint64_t)limit_ns, c->d_err, c->stream), "wait self-test kernel");
+    c->launches += 1;
     return MALIB_OK;
 }
 
