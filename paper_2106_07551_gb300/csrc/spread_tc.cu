@@ -6,14 +6,15 @@
 // CTA k keeps the policy of agent k resident in shared memory. Each CTA has 16
 // warps in three roles:
 //  * warps 0-7, the engine: runs agent k's 128-row observation tiles through
-//    the tensor-core MLP (hidden activations in tensor memory), draws agent k's
-//    actions and sends them to all 8 CTAs;
+//    the tensor-core MLP (hidden activations in tensor memory) and hands the
+//    logits to the tile's group through shared memory and a local mbarrier;
 //  * warps 8-11 and 12-15, environment groups 0 and 1: two episodes of the
 //    combination in flight, one environment per thread. Every CTA keeps a
 //    replica of a group's 128 environments; per step a group builds agent k's
 //    observations (a bf16 tile for the engine; each thread stores its fp32 row,
-//    one 144-byte run, to the trajectory), waits for the 8 agents' actions,
-//    applies them
+//    one 144-byte run, to the trajectory), draws agent k's actions from the
+//    engine's logits and sends them to all 8 CTAs, waits for the 8 agents'
+//    actions, applies them
 //    (identical IEEE operations in every CTA, identical bits) and writes agent
 //    k's trajectory (observation, action, reward; CTA 0 the done flags).
 // While the engine runs one group's tile, the other group steps its
@@ -41,10 +42,10 @@ constexpr int kGroups = 2;
 constexpr uint32_t kX = Eng::kSmemBytes;                          // observation tiles [group]
 constexpr uint32_t kActs = kX + kGroups * Eng::kXBytes;           // [group][parity][agent][env]
 constexpr uint32_t kSend = kActs + kGroups * 2 * kN * 128;        // this agent's actions [group][env]
-constexpr uint32_t kU = kSend + kGroups * 128;                    // decision uniforms [group][env]
-constexpr uint32_t kSmem = kU + kGroups * 128 * 4;
+constexpr uint32_t kLgs = kSend + kGroups * 128;                  // logits [group][env][8] fp32
+constexpr uint32_t kSmem = kLgs + kGroups * 128 * 8 * 4;
 static_assert(kX % 16 == 0 && kActs % 16 == 0 && kSend % 16 == 0 &&
-              kU % 16 == 0, "16-byte aligned regions");
+              kLgs % 16 == 0, "16-byte aligned regions");
 constexpr uint32_t kActTx = kN * 128;                             // action bytes received per step
 
 __device__ __forceinline__ void cluster_barrier_all() {
@@ -93,11 +94,12 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
     __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t act_bar[kGroups][2];   // actions of a group's steps, by parity
     __shared__ __align__(8) uint64_t x_bar[kGroups];        // a group's tile is ready
+    __shared__ __align__(8) uint64_t lg_bar[kGroups];       // a group's logits are ready
     __shared__ uint32_t tmem_base;
 
     uint8_t* acts = smem + kActs;
     uint8_t* send = smem + kSend;
-    float* ubuf = reinterpret_cast<float*>(smem + kU);
+    float* lgs = reinterpret_cast<float*>(smem + kLgs);
     const uint32_t me = cl::rank();
     const int tid = threadIdx.x, warp = tid >> 5;
 
@@ -107,6 +109,7 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         mbar_init(&mma_bar[1], 1);
         for (int g = 0; g < kGroups; ++g) {
             mbar_init(&x_bar[g], 1);
+            mbar_init(&lg_bar[g], 1);
             for (int p = 0; p < 2; ++p) {
                 mbar_init(&act_bar[g][p], 1);
                 mbar_arrive_expect_tx(&act_bar[g][p], kActTx);   // armed for steps 0 and 1
@@ -168,37 +171,16 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                         atomicOr(a.err, ERRBIT_TIMEOUT);
                     x_bits ^= 1u << g;
                     Eng::sync();
-                    const int64_t ep = rd.ep[g];
-                    const float* u = ubuf + g * 128;
-                    uint8_t* snd = send + g * 128;
+                    float* lgg = lgs + g * 128 * 8;
                     Eng::forward(smem, nullptr, tbase, mma_bar, mma_par, a.err,
                                  [&](int row, const float* lg) {
-                                     int act = 0;
-                                     if (row < epp) {
-                                         const int64_t ix =
-                                             ((ep * T + t) * a.n_envs + (int64_t)rd.pair * epp + row) * kN;
-                                         float l5[kA];
-#pragma unroll
-                                         for (int k = 0; k < kA; ++k) l5[k] = lg[k];
-                                         act = sample_masked<kA>(l5, 0x1Fu, u[row]);
-                                         if (a.logits)
-#pragma unroll
-                                             for (int k = 0; k < kA; ++k)
-                                                 a.logits[(ix + me) * kA + k] = l5[k];
-                                         a.action[ix + me] = (uint8_t)act;
-                                     }
-                                     snd[row] = (uint8_t)act;
+                                     float4* d = reinterpret_cast<float4*>(lgg + row * 8);
+                                     d[0] = make_float4(lg[0], lg[1], lg[2], lg[3]);
+                                     d[1] = make_float4(lg[4], 0.f, 0.f, 0.f);
                                  },
                                  smem_u32(smem + kX + g * Eng::kXBytes), /*x_published=*/true);
-                    // the forward ends with an engine barrier: all 128 bytes are in snd
-                    if (tid < kN * 8) {
-                        const uint32_t c = (uint32_t)tid & 7u, r = (uint32_t)tid >> 3;
-                        const uint32_t par = (uint32_t)t & 1u;
-                        uint8_t* dst = acts + ((g * 2 + par) * kN + me) * 128 + 16 * c;
-                        cl::st_async_v4(cl::map(dst, r),
-                                        *reinterpret_cast<const uint4*>(snd + 16 * c),
-                                        cl::map(&act_bar[g][par], r));
-                    }
+                    // the forward ends with an engine barrier: every row's logits are stored
+                    if (tid == 0) mbar_arrive_release(&lg_bar[g]);
                 }
             }
         }
@@ -208,6 +190,9 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
         const int e = tid - kEngineThreads - g * 128;     // environment within the block
         uint8_t* xg = smem + kX + g * Eng::kXBytes;
         uint32_t act_bits = 0;                             // act_bar[g][p] phase: bit p
+        uint32_t lg_par = 0;
+        const float* lgg = lgs + g * 128 * 8;
+        uint8_t* snd = send + g * 128;
         for (int64_t it = lo; it < hi;) {
             const Round rd = round_at(it, hi, a.n_episodes);
             it = rd.next;
@@ -220,8 +205,9 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
             if (mine) spread_reset<kN>(s, gid, a.seed);
             for (int t = 0; t < T; ++t) {
                 const uint32_t par = (uint32_t)t & 1u;
+                float u = 0.f;
                 if (mine) {
-                    ubuf[g * 128 + e] = u24(draw(gid, (uint32_t)t, me, a.seed).x);
+                    u = u24(draw(gid, (uint32_t)t, me, a.seed).x);
                     float o[kObsPad];
                     spread_obs_dyn<kN, kObsPad>(s, (int)me, o);
                     // agent me's observation: [ep][t][env][agent][obs_pad], one 144-byte run
@@ -242,6 +228,31 @@ __global__ void __cluster_dims__(8, 1, 1) __launch_bounds__(kThreads, 1)
                 }
                 group_sync(g);
                 if (e == 0) mbar_arrive_release(&x_bar[g]);      // the tile goes to the engine
+                // agent me's logits from the engine; its actions to every CTA
+                if (!mbar_wait_bounded(&lg_bar[g], lg_par, kWaitLimitNs) && e == 0)
+                    atomicOr(a.err, ERRBIT_TIMEOUT);
+                lg_par ^= 1u;
+                {
+                    int act = 0;
+                    if (mine) {
+                        const float4 l0 = *reinterpret_cast<const float4*>(lgg + e * 8);
+                        float l5[kA] = {l0.x, l0.y, l0.z, l0.w, lgg[e * 8 + 4]};
+                        act = sample_masked<kA>(l5, 0x1Fu, u);
+                        const int64_t ix = ((ep * T + t) * a.n_envs + env) * kN;
+                        if (a.logits)
+#pragma unroll
+                            for (int k = 0; k < kA; ++k) a.logits[(ix + me) * kA + k] = l5[k];
+                        a.action[ix + me] = (uint8_t)act;
+                    }
+                    snd[e] = (uint8_t)act;
+                }
+                group_sync(g);
+                if (e < kN * 8) {
+                    const uint32_t c = (uint32_t)e & 7u, r = (uint32_t)e >> 3;
+                    uint8_t* dst = acts + ((g * 2 + par) * kN + me) * 128 + 16 * c;
+                    cl::st_async_v4(cl::map(dst, r), *reinterpret_cast<const uint4*>(snd + 16 * c),
+                                    cl::map(&act_bar[g][par], r));
+                }
                 // the 8 agents' actions of this step, from every engine of the cluster
                 if (!cl::wait_cluster_bounded(&act_bar[g][par], (act_bits >> par) & 1u, kWaitLimitNs) &&
                     e == 0)
