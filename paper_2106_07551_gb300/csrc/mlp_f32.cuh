@@ -232,8 +232,8 @@ struct MlpF32 {
 // live in a buffer of its own (restaged per policy) while the small layers of
 // several policies stay resident. Layer 3 is folded into layer 2's epilogue
 // (shuffle reduction over the 16 column lanes of a row group, which share one
-// warp). NI (8 or 4) is the number of 16-row blocks a pass computes: NI = 4
-// covers rows 0..63 only, for passes whose compacted rows all lie there.
+// warp). NI (1..8) is the number of 16-row blocks a pass computes: rows
+// 0 .. 16 NI - 1, for passes whose compacted rows all lie there.
 template <int IN, int A>
 struct MlpF32T8 {
     static constexpr int H = 128;
@@ -335,12 +335,18 @@ struct MlpF32T8 {
         // layer 3: ReLU once, then per row and action a packed dot product over
         // the thread's 4 column pairs and the sum of its two halves
         static_assert(A == 3, "the reduce-scatter below places 3 logits per row");
+        static_assert(NI >= 1 && NI <= 8, "1 to 8 row blocks");
 #pragma unroll
         for (int i = 0; i < NI; ++i)
 #pragma unroll
             for (int p = 0; p < 4; ++p) acc[i][p] = f2_relu(acc[i][p]);
-        constexpr int V = NI * A;                 // partial logits of this thread
+        // the reduce-scatter runs on 8 (NI > 4) or 4 row blocks; blocks beyond
+        // NI enter it as zeros and their rows hold no hand
+        constexpr int NR = NI > 4 ? 8 : 4;
+        constexpr int V = NR * A;                 // partial logits of this thread
         float v0[V];
+#pragma unroll
+        for (int j = NI * A; j < V; ++j) v0[j] = 0.f;
 #pragma unroll
         for (int a = 0; a < A; ++a) {
             const ulonglong2 wA = *reinterpret_cast<const ulonglong2*>(W3 + a * H + c0);
@@ -378,7 +384,7 @@ struct MlpF32T8 {
         float v3[A];
         int i_own;
         bool writer;
-        if constexpr (NI == 8) {
+        if constexpr (NR == 8) {
             // 6 values: one more halving (lane bit 1), then lane bit 0 sums
             // both copies; lanes with bit 0 clear hold row 4 l4 + 2 l2 + l1
 #pragma unroll

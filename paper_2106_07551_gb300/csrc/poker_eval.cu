@@ -388,6 +388,34 @@ __device__ int pick_pair(const EvalArgs& a) {
     __syncthreads();
     return bp;
 }
+// 16-row blocks a pass of c placed rows (compacted into rows 0 .. c - 1)
+// computes: ceil(c / 16), at least 4.
+__device__ __forceinline__ int blocks_for(int c) { return c <= 64 ? 4 : (c + 15) >> 4; }
+
+template <class Eng>
+__device__ __forceinline__ void layer1_n(int nb, const float* X, float* H1, const float* W1T,
+                                         const float* b1) {
+    switch (nb) {
+        case 4: Eng::template layer1<4>(X, H1, W1T, b1); break;
+        case 5: Eng::template layer1<5>(X, H1, W1T, b1); break;
+        case 6: Eng::template layer1<6>(X, H1, W1T, b1); break;
+        case 7: Eng::template layer1<7>(X, H1, W1T, b1); break;
+        default: Eng::template layer1<8>(X, H1, W1T, b1); break;
+    }
+}
+
+template <class Eng>
+__device__ __forceinline__ void layer23_n(int nb, const float* H1, float* LG, const float* W2T,
+                                          const float* b2, const float* W3, const float* b3) {
+    switch (nb) {
+        case 4: Eng::template layer23<4>(H1, LG, W2T, b2, W3, b3); break;
+        case 5: Eng::template layer23<5>(H1, LG, W2T, b2, W3, b3); break;
+        case 6: Eng::template layer23<6>(H1, LG, W2T, b2, W3, b3); break;
+        case 7: Eng::template layer23<7>(H1, LG, W2T, b2, W3, b3); break;
+        default: Eng::template layer23<8>(H1, LG, W2T, b2, W3, b3); break;
+    }
+}
+
 }  // namespace t8
 
 __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
@@ -487,13 +515,13 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
             const float* ss = smem + kOffSmall + second * kSmall;
             const int off_b2 = L::kW2T, off_w3 = L::kW2T + (L::kW3 - L::kB2),
                       off_b3 = L::kW2T + (L::kB3 - L::kB2);
-            // a pass whose placed rows all lie in 0..63 computes only those rows
-            if (c[first] > 64) {
-                E::layer1<8>(X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
-                E::layer23<8>(H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3, sf + off_b3);
-            } else if (c[first] > 0) {
-                E::layer1<4>(X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
-                E::layer23<4>(H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3, sf + off_b3);
+            // a pass computes the 16-row blocks that hold its placed rows (at
+            // least 4)
+            if (c[first] > 0) {
+                const int nb = t8::blocks_for(c[first]);
+                t8::layer1_n<E>(nb, X + first * E::kRows * E::XS, H1, sf, sf + L::kB1);
+                t8::layer23_n<E>(nb, H1, LG + first * E::kRows * E::LS, W2s, sf + off_b2, sf + off_w3,
+                                 sf + off_b3);
             }
             if (c[second] > 0) {
                 const float* src = (second == 0 ? pol0 : pol1) + L::kW2T;
@@ -503,16 +531,13 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
                     bulk_g2s(W2s, src, 32768u, &bar);
                     bulk_g2s(W2s + 8192, src + 8192, 32768u, &bar);
                 }
-                const bool full = c[second] > 64;
-                if (full) E::layer1<8>(X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
-                else E::layer1<4>(X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
+                const int nb = t8::blocks_for(c[second]);
+                t8::layer1_n<E>(nb, X + second * E::kRows * E::XS, H1, ss, ss + L::kB1);
                 if (!mbar_wait_bounded(&bar, parity, kWaitLimitNs) && tid == 0)
                     atomicOr(a.err, ERRBIT_TIMEOUT);
                 parity ^= 1u;
-                if (full)
-                    E::layer23<8>(H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3, ss + off_b3);
-                else
-                    E::layer23<4>(H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3, ss + off_b3);
+                t8::layer23_n<E>(nb, H1, LG + second * E::kRows * E::LS, W2s, ss + off_b2, ss + off_w3,
+                                 ss + off_b3);
                 res = second;
             }
             if (placed) {
