@@ -175,8 +175,12 @@ int malib_set_stream(malib_ctx* ctx, void* cuda_stream);
 /*
  * malib_pop_load - add policies to the population (Sec. 3.1: policy pools
  * P = {P_i}, extended as PSRO adds best responses, App. C.2 main loop).
- * Copies and converts the parameters into the context's device arena; the
- * caller may free `pols[i].params` when the call returns. All policies of one
+ * Copies and converts the parameters into the context's device arena: the
+ * plain fp32 parameters (host or device memory) are copied into a device
+ * staging buffer and one kernel writes every policy's kernel image (fp32
+ * layout, bf16-rounded weights, or the bf16 tensor-core image). The call waits
+ * for its copies and the conversion on the context's stream, so the caller may
+ * free `pols[i].params` when it returns. All policies of one
  * context share env kind, kind, dtype and dims; the first call fixes them and
  * `spec`. ids_out[n] receives the new policies' ids (consecutive, from 0).
  * Errors: EINVAL (shape or size mismatch with spec), ESTATE (different spec

@@ -113,6 +113,22 @@ cudaError_t launch_zero_u64(unsigned long long* p, int64_t n, cudaStream_t s);
 cudaError_t launch_finalize(const unsigned long long* acc, int32_t n_pairs, int64_t n_episodes,
                             double* out, cudaStream_t s);
 cudaError_t launch_selftest_wait(bool arrive, uint64_t limit_ns, int* err, cudaStream_t s);
+// One policy of a population load: its plain fp32 parameters at stage + src
+// (row-major W[out][in] then b[out], per layer) become its kernel image at
+// arena + dst, `size` 32-bit words (pop_convert.cu).
+constexpr int32_t kConvTable = 0, kConvF32 = 1, kConvTc = 2;   // kind
+constexpr int32_t kConvRound = 1, kConvFold = 2;               // flags
+struct ConvJob {
+    int64_t src;        // float offset in the staging buffer
+    int64_t dst;        // float offset in the arena
+    int64_t size;       // image words
+    int32_t kind;
+    int32_t flags;      // kConvRound: weights to bf16 (fp32 layout); kConvFold: Leduc feature 15
+    int32_t dims[4];
+};
+cudaError_t launch_pop_convert(const ConvJob* jobs, int n_jobs, int64_t max_size, const float* stage,
+                               float* arena, cudaStream_t s);
+
 cudaError_t launch_philox_digest(uint64_t seed, int64_t n, int calls, uint32_t* out,
                                  cudaStream_t s);
 cudaError_t launch_selftest_philox(const uint32_t* ctr, uint64_t seed, uint32_t* out, int64_t n,

@@ -38,9 +38,13 @@ struct malib_ctx {
     int dims[4] = {0, 0, 0, 0};
     bool tc_layout = false;            // bf16 tensor-core images in the arena
     std::vector<PolicyRec> pols;
-    std::vector<float> host_arena;     // mirror of the device arena
     float* arena = nullptr;
     int64_t arena_cap = 0;             // floats
+    int64_t arena_used = 0;            // floats
+    float* d_stage = nullptr;          // plain parameters of a load, before conversion
+    int64_t stage_cap = 0;
+    ConvJob* d_jobs = nullptr;
+    int64_t jobs_cap = 0;
     int64_t* d_off = nullptr;
     int32_t* d_seat = nullptr;
     int64_t tbl_cap = 0;
@@ -175,87 +179,6 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
 bool same_env(const malib_env_spec& a, const malib_env_spec& b) {
     return a.env_kind == b.env_kind && a.n_agents == b.n_agents &&
            a.n_landmarks == b.n_landmarks && a.obs_dim == b.obs_dim && a.n_actions == b.n_actions;
-}
-
-// fp32 kernel layout (internal.h F32Layout) from the plain layout.
-void to_f32_layout(const float* p, const int* d, float* out, int64_t size) {
-    const int in = d[0], h1 = d[1], h2 = d[2], a = d[3];
-    const float* W1 = p;
-    const float* b1 = W1 + (int64_t)h1 * in;
-    const float* W2 = b1 + h1;
-    const float* b2 = W2 + (int64_t)h2 * h1;
-    const float* W3 = b2 + h2;
-    const float* b3 = W3 + (int64_t)a * h2;
-    std::memset(out, 0, (size_t)size * 4);
-    float* o = out;
-    for (int k = 0; k < in; ++k)
-        for (int j = 0; j < h1; ++j) o[(int64_t)k * h1 + j] = W1[(int64_t)j * in + k];
-    o += (int64_t)in * h1;
-    for (int j = 0; j < h1; ++j) o[j] = b1[j];
-    o += h1;
-    for (int k = 0; k < h1; ++k)
-        for (int j = 0; j < h2; ++j) o[(int64_t)k * h2 + j] = W2[(int64_t)j * h1 + k];
-    o += (int64_t)h1 * h2;
-    for (int j = 0; j < h2; ++j) o[j] = b2[j];
-    o += h2;
-    for (int i = 0; i < a * h2; ++i) o[i] = W3[i];
-    o += (int64_t)a * h2;
-    for (int j = 0; j < a; ++j) o[j] = b3[j];
-}
-
-// bf16 tensor-core image (internal.h) from the plain fp32 layout.
-// bf16 tensor-core image of one MLP (layout: tc_image_bytes). fold: the Leduc
-// image, whose observation feature 15 (call/check is legal) is 1 in every
-// state, so its W1 column is added to b1 (as the bf16 weight the product
-// would use) and the remaining 16 features fill one K step of 16: slot s holds
-// feature s for s < 15 and feature 16 in slot 15.
-void to_tc_image(const float* p, const int* d, float* out_floats, bool fold) {
-    const int in = d[0], H = 256, A = d[3];
-    const int in_img = fold ? in - 1 : in;
-    const int k1 = (in_img + 15) / 16 * 16;
-    const float* W1 = p;
-    const float* b1 = W1 + (int64_t)H * in;
-    const float* W2 = b1 + H;
-    const float* b2 = W2 + (int64_t)H * H;
-    const float* W3 = b2 + H;
-    const float* b3 = W3 + (int64_t)A * H;
-    uint8_t* img = reinterpret_cast<uint8_t*>(out_floats);
-    const int64_t bytes = tc_image_bytes(in_img);
-    std::memset(img, 0, (size_t)bytes);
-    auto bf = [](float x) -> uint16_t {
-        uint32_t b;
-        std::memcpy(&b, &x, 4);
-        if ((b & 0x7F800000u) != 0x7F800000u) b += 0x7FFFu + ((b >> 16) & 1u);
-        return (uint16_t)(b >> 16);
-    };
-    auto bf_value = [&](float x) -> float {
-        const uint32_t b = (uint32_t)bf(x) << 16;
-        float v;
-        std::memcpy(&v, &b, 4);
-        return v;
-    };
-    auto put = [&](uint8_t* base, int row, int k, int rows, float v) {
-        const uint16_t h = bf(v);
-        std::memcpy(base + tc::cm_offset(row, k, rows, 2), &h, 2);
-    };
-    uint8_t* w1 = img;
-    uint8_t* w2 = w1 + (int64_t)H * k1 * 2;
-    uint8_t* w3 = w2 + (int64_t)H * H * 2;
-    float* bias = reinterpret_cast<float*>(w3 + 16 * H * 2);
-    for (int n = 0; n < H; ++n)
-        for (int s = 0; s < in_img; ++s) {
-            const int f = fold && s >= kLeducConstFeature ? s + 1 : s;
-            put(w1, n, s, H, W1[(int64_t)n * in + f]);
-        }
-    for (int n = 0; n < H; ++n)
-        for (int k = 0; k < H; ++k) put(w2, n, k, H, W2[(int64_t)n * H + k]);
-    for (int n = 0; n < A; ++n)
-        for (int k = 0; k < H; ++k) put(w3, n, k, 16, W3[(int64_t)n * H + k]);
-    for (int j = 0; j < H; ++j) {
-        bias[j] = fold ? b1[j] + bf_value(W1[(int64_t)j * in + kLeducConstFeature]) : b1[j];
-        bias[H + j] = b2[j];
-    }
-    for (int j = 0; j < A; ++j) bias[2 * H + j] = b3[j];
 }
 
 int upload_tables(malib_ctx* c) {
@@ -437,6 +360,8 @@ void malib_destroy(malib_ctx* c) {
     cudaFree(c->d_pairs);
     cudaFree(c->d_out);
     cudaFree(c->scratch);
+    cudaFree(c->d_stage);
+    cudaFree(c->d_jobs);
     delete c;
 }
 
@@ -462,7 +387,7 @@ int malib_pop_reset(malib_ctx* c) {
     DeviceGuard g(c->device);
     CK(cudaStreamSynchronize(c->stream), "stream");
     c->pols.clear();
-    c->host_arena.clear();
+    c->arena_used = 0;
     c->has_pop = false;
     c->tables_dirty = true;
     return MALIB_OK;
@@ -478,8 +403,9 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
     if (c->has_pop && !same_env(c->spec, *spec))
         return fail(c, MALIB_ESTATE, "population was loaded for a different environment");
     const bool poker = spec->env_kind == MALIB_ENV_KUHN || spec->env_kind == MALIB_ENV_LEDUC;
-    std::vector<std::vector<float>> converted(n);
+    std::vector<ConvJob> jobs(n);
     std::vector<PolicyRec> recs(n);
+    int64_t stage_floats = 0, image_floats = 0, max_size = 0;
     for (int i = 0; i < n; ++i) {
         const malib_policy_desc& d = pols[i];
         PolicyRec rec{};
@@ -515,82 +441,70 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
         const int ref_dtype = first ? d.dtype : (c->has_pop ? c->pol_dtype : pols[0].dtype);
         if (d.kind != ref_kind || d.dtype != ref_dtype || std::memcmp(d.dims, ref_dims, 16) != 0)
             return fail(c, MALIB_EINVAL, "policy %d: every policy of a population shares kind, dtype and dims", i);
-        std::vector<float> plain(count);
-        if (is_device_ptr(d.params)) {
-            CK(cudaMemcpy(plain.data(), d.params, count * 4, cudaMemcpyDeviceToHost), "params");
-        } else {
-            std::memcpy(plain.data(), d.params, count * 4);
-        }
+        ConvJob& jb = jobs[i];
+        std::memcpy(jb.dims, d.dims, sizeof jb.dims);
+        jb.flags = 0;
         if (d.kind == MALIB_POL_TABULAR) {
-            converted[i].assign(8, 0.f);
-            for (int k = 0; k < 6; ++k) converted[i][k] = plain[k];
+            jb.kind = kConvTable;
+            jb.size = 8;
+        } else if (d.dtype == MALIB_BF16 && tc_image_shape(d.dims)) {
+            const bool fold = leduc_tc_fold(spec->env_kind, d.dims[0]);
+            jb.kind = kConvTc;
+            jb.flags = fold ? kConvFold : 0;
+            jb.size = tc_image_bytes(fold ? d.dims[0] - 1 : d.dims[0]) / 4;
         } else {
-            const int64_t size = ((int64_t)d.dims[0] * d.dims[1] + d.dims[1] +
-                                  (int64_t)d.dims[1] * d.dims[2] + d.dims[2] +
-                                  (int64_t)d.dims[3] * d.dims[2] + d.dims[3] + 3) / 4 * 4;
-            if (d.dtype == MALIB_BF16 && tc_image_shape(d.dims)) {
-                const bool fold = leduc_tc_fold(spec->env_kind, d.dims[0]);
-                converted[i].assign((size_t)(tc_image_bytes(fold ? d.dims[0] - 1 : d.dims[0]) / 4), 0.f);
-                to_tc_image(plain.data(), d.dims, converted[i].data(), fold);
-                recs[i] = rec;
-                continue;
-            }
-            if (d.dtype == MALIB_BF16) {
-                // weights rounded to bf16 (nearest even); biases stay fp32
-                auto rne = [](float x) {
-                    uint32_t b;
-                    std::memcpy(&b, &x, 4);
-                    if ((b & 0x7F800000u) != 0x7F800000u) {
-                        b += 0x7FFFu + ((b >> 16) & 1u);
-                        b &= 0xFFFF0000u;
-                    }
-                    float y;
-                    std::memcpy(&y, &b, 4);
-                    return y;
-                };
-                const int* D = d.dims;
-                int64_t k = 0;
-                for (int layer = 0; layer < 3; ++layer) {
-                    const int fi = D[layer], fo = D[layer + 1];
-                    for (int64_t q = 0; q < (int64_t)fi * fo; ++q, ++k) plain[k] = rne(plain[k]);
-                    k += fo;
-                }
-            }
-            converted[i].resize(size);
-            to_f32_layout(plain.data(), d.dims, converted[i].data(), size);
+            jb.kind = kConvF32;
+            jb.flags = d.dtype == MALIB_BF16 ? kConvRound : 0;   // bf16 weights, fp32 biases
+            jb.size = ((int64_t)d.dims[0] * d.dims[1] + d.dims[1] + (int64_t)d.dims[1] * d.dims[2] +
+                       d.dims[2] + (int64_t)d.dims[3] * d.dims[2] + d.dims[3] + 3) / 4 * 4;
         }
+        jb.src = stage_floats;
+        jb.dst = c->arena_used + image_floats;
+        rec.offset = jb.dst;
+        stage_floats += (count + 3) / 4 * 4;            // 16-byte aligned sources
+        image_floats += jb.size;
+        max_size = std::max(max_size, jb.size);
         recs[i] = rec;
     }
-    // append to the arena
-    int64_t add = 0;
-    for (int i = 0; i < n; ++i) add += (int64_t)converted[i].size();
-    const int64_t base = (int64_t)c->host_arena.size();
-    c->host_arena.resize(base + add);
-    int64_t off = base;
-    for (int i = 0; i < n; ++i) {
-        std::memcpy(c->host_arena.data() + off, converted[i].data(), converted[i].size() * 4);
-        recs[i].offset = off;
-        off += (int64_t)converted[i].size();
-    }
-    const int64_t need = (int64_t)c->host_arena.size();
-    if (need > c->arena_cap) {
-        int64_t cap = c->arena_cap > 0 ? c->arena_cap : 1 << 16;
-        while (cap < need) cap *= 2;
-        float* na = nullptr;
-        cudaError_t e = cudaMalloc((void**)&na, (size_t)cap * 4);
-        if (e != cudaSuccess) {
-            c->host_arena.resize(base);
-            return cuda_fail(c, e, "population arena");
+    if (n > 0) {
+        // the arena grows by a device copy of what it holds
+        const int64_t need = c->arena_used + image_floats;
+        if (need > c->arena_cap) {
+            int64_t cap = c->arena_cap > 0 ? c->arena_cap : 1 << 16;
+            while (cap < need) cap *= 2;
+            float* na = nullptr;
+            CK(cudaMalloc((void**)&na, (size_t)cap * 4), "population arena");
+            if (c->arena_used > 0) {
+                const cudaError_t e = cudaMemcpyAsync(na, c->arena, c->arena_used * 4,
+                                                      cudaMemcpyDeviceToDevice, c->stream);
+                if (e != cudaSuccess) {
+                    cudaFree(na);
+                    return cuda_fail(c, e, "arena copy");
+                }
+            }
+            CK(cudaStreamSynchronize(c->stream), "arena copy");
+            cudaFree(c->arena);
+            c->arena = na;
+            c->arena_cap = cap;
         }
-        cudaStreamSynchronize(c->stream);
-        cudaFree(c->arena);
-        c->arena = na;
-        c->arena_cap = cap;
-        CK(cudaMemcpyAsync(c->arena, c->host_arena.data(), need * 4, cudaMemcpyHostToDevice,
-                           c->stream), "arena upload");
-    } else if (add > 0) {
-        CK(cudaMemcpyAsync(c->arena + base, c->host_arena.data() + base, add * 4,
-                           cudaMemcpyHostToDevice, c->stream), "arena upload");
+        if ((r = ensure(c, c->d_stage, c->stage_cap, stage_floats, "parameter staging")) != MALIB_OK)
+            return r;
+        if ((r = ensure(c, c->d_jobs, c->jobs_cap, (int64_t)n, "conversion jobs")) != MALIB_OK)
+            return r;
+        // plain parameters from host or device memory (cudaMemcpyDefault: unified addressing)
+        for (int i = 0; i < n; ++i)
+            CK(cudaMemcpyAsync(c->d_stage + jobs[i].src, pols[i].params, pols[i].nbytes,
+                               cudaMemcpyDefault, c->stream), "parameter upload");
+        CK(cudaMemcpyAsync(c->d_jobs, jobs.data(), (size_t)n * sizeof(ConvJob), cudaMemcpyHostToDevice,
+                           c->stream), "conversion jobs");
+        for (int j0 = 0; j0 < n; j0 += 65535) {
+            CK(launch_pop_convert(c->d_jobs + j0, std::min(65535, n - j0), max_size, c->d_stage,
+                                  c->arena, c->stream), "population conversion kernel");
+            c->launches += 1;
+        }
+        // the caller may free or reuse its parameter buffers once this returns
+        CK(cudaStreamSynchronize(c->stream), "population load");
+        c->arena_used = need;
     }
     for (int i = 0; i < n; ++i) {
         ids_out[i] = (int32_t)c->pols.size();
