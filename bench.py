@@ -448,12 +448,13 @@ def philox_ceiling(ctx, stream):
 
 def run_e2e(args, ctx, w, spec, dev, rollout):
     """The same metric through the public API with host buffers: population
-    upload from pinned host memory, pair table in, payoff table back."""
+    upload from pinned host memory and the pair (or combination) table in; the
+    payoff table (evaluation) or the trajectory's rewards (rollout) back."""
     import numpy as np
     import torch
     from paper_2106_07551_gb300 import policy_desc
     if rollout:
-        return None
+        return run_e2e_rollout(args, ctx, w, spec, dev)
     h_params = [torch.from_numpy(p.params).pin_memory() for p in w.policies]
     h_pairs = torch.from_numpy(w.pair_ids).pin_memory()
     h_out = torch.empty((w.n_pairs, 4), dtype=torch.float64).pin_memory()
@@ -474,6 +475,39 @@ def run_e2e(args, ctx, w, spec, dev, rollout):
             tot += t1 - t0
             dec += d
     return {"value": dec / tot, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "steps": n}
+
+
+def run_e2e_rollout(args, ctx, w, spec, dev):
+    """Rollout end to end: population and combination table from pinned host
+    memory, the rollout into device trajectory buffers (where a learner on the
+    GPU reads them), and every agent-step's reward copied back to pinned host
+    memory as the step's result."""
+    import torch
+    from paper_2106_07551_gb300 import alloc_traj, policy_desc
+    h_params = [torch.from_numpy(p.params).pin_memory() for p in w.policies]
+    h_pairs = torch.from_numpy(w.pair_ids).pin_memory()
+    descs = [policy_desc(p.kind, p.dtype, p.seat, p.dims, h) for p, h in zip(w.policies, h_params)]
+    traj = alloc_traj(spec, w.n_episodes)
+    h_rew = torch.empty(traj["reward"].shape, dtype=torch.float32).pin_memory()
+    h2d = sum(h.numel() * 4 for h in h_params) + h_pairs.numel() * 4
+    d2h = h_rew.numel() * 4
+    steps_per_call = w.n_envs * w.episode_len * w.n_episodes
+    n = max(1, args.e2e_steps)
+    tot = 0.0
+    for k in range(n + 1):
+        torch.cuda.synchronize(dev)
+        t0 = time.perf_counter()
+        ctx.pop_reset()
+        ctx.pop_load(spec, descs)
+        ctx.rollout(spec, h_pairs, w.n_episodes, w.seed + 777 + k, traj)
+        h_rew.copy_(traj["reward"], non_blocking=True)
+        ctx.sync()
+        torch.cuda.synchronize(dev)
+        t1 = time.perf_counter()
+        if k > 0:            # first call warms the host path
+            tot += t1 - t0
+    return {"value": steps_per_call * n / tot, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "steps": n}
 
 
