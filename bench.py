@@ -236,6 +236,76 @@ def oracle_leduc_sample(w, target_s: float, threads: int):
     return dec / dt, f"first {n} hands of each of the {w.n_pairs} pairs ({dec} decisions, {dt:.1f} s)"
 
 
+def oracle_rollout_sample(w, name, target_s: float, threads: int):
+    """Times the oracle's rollout (one episode) on the first n environments, n
+    sized so that the run takes about target_s seconds. Returns (env-steps/s,
+    sample text)."""
+    import oracle
+    params = [p.params for p in w.policies]
+    dims = w.policies[0].dims
+    bf16 = w.policies[0].dtype == 1
+
+    def run(n, eps=1):
+        t0 = time.perf_counter()
+        if name == "adversary3":
+            oracle.adversary_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, eps, w.seed,
+                                     env_lo=0, env_hi=n, n_threads=threads)
+        else:
+            oracle.spread_rollout(params, dims, w.n_agents, w.n_landmarks, w.episode_len, w.n_envs,
+                                  w.pair_ids, eps, w.seed, bf16=bf16, env_lo=0, env_hi=n,
+                                  n_threads=threads)
+        return time.perf_counter() - t0
+
+    n = threads
+    dt = run(n)
+    while dt < 0.5 and n < w.n_envs:
+        n = min(w.n_envs, n * 4)
+        dt = run(n)
+    eps = 1
+    n2 = max(1, min(w.n_envs, int(n * target_s / max(dt, 1e-6))))
+    if n2 == w.n_envs and n == w.n_envs:
+        # every environment fits: add episodes, the oracle's output kept under 512 MB
+        per_ep = w.n_envs * w.episode_len * w.n_agents * (w.obs_dim + 8) * 4
+        eps = max(1, min(w.n_episodes, int(target_s / max(dt, 1e-6)), (512 << 20) // per_ep))
+    if n2 != n or eps != 1:
+        dt = run(n2, eps)
+        n = n2
+    steps = n * w.episode_len * eps
+    return steps / dt, (f"first {n} of the {w.n_envs} environments, {eps} episode(s) of "
+                        f"{w.episode_len} steps ({steps} env-steps, {dt:.1f} s)")
+
+
+def oracle_kuhn_sample(w, target_s: float, threads: int):
+    """Times the oracle's Kuhn evaluation on the first n hands of every pair."""
+    import numpy as np
+    import oracle
+    tables = np.stack([p.params for p in w.policies])
+
+    def run(n):
+        t0 = time.perf_counter()
+        oracle.kuhn_eval(tables, w.pair_ids, n, w.seed, n_threads=threads)
+        return time.perf_counter() - t0
+
+    n = 1000
+    dt = run(n)
+    while dt < 0.5 and n < (1 << 26):
+        n *= 4
+        dt = run(n)
+    n2 = max(1, int(n * target_s / max(dt, 1e-6)))
+    if n2 != n:
+        dt = run(n2)
+        n = n2
+    # decisions per hand, exactly: 2, plus a third when seat 0 passes (infoset
+    # card * 2) and seat 1 then bets (infoset card * 2), over the 6 deals
+    deals = [(a, b) for a in range(3) for b in range(3) if a != b]
+    dec = 0.0
+    for i, j in w.pair_ids:
+        p0, p1 = tables[i].astype(np.float64), tables[j].astype(np.float64)
+        dec += n * (2.0 + sum((1.0 - p0[2 * a]) * p1[2 * b] for a, b in deals) / 6.0)
+    return dec / dt, (f"first {n} hands of each of the {w.n_pairs} pairs ({dt:.1f} s; decisions "
+                      f"counted by their exact expectation per pair)")
+
+
 def cpu_count():
     try:
         return len(os.sched_getaffinity(0))
@@ -405,9 +475,13 @@ def run_ours(args):
     e2e = run_e2e(args, ctx, w, spec, dev, rollout) if rank == 0 else None
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload in ("leduc",
-                                                                                 "leduc_bf16"):
-        rate, sample = oracle_leduc_sample(w, 12.0, cpu_count())
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and args.workload != "meta":
+        if args.workload in ("leduc", "leduc_bf16"):
+            rate, sample = oracle_leduc_sample(w, 12.0, cpu_count())
+        elif args.workload == "kuhn":
+            rate, sample = oracle_kuhn_sample(w, 12.0, cpu_count())
+        else:
+            rate, sample = oracle_rollout_sample(w, args.workload, 12.0, cpu_count())
         cpu = {"value": rate, "unit": UNIT, "cores": cpu_count(), "kind": "oracle",
                "sample": sample}
     ctx.close()
