@@ -488,7 +488,8 @@ def run_ours(args):
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
-                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "bf16" if tensor else "f32",
                 "data": "synthetic", "config": config_of(w, args.workload),
                 "payoff_entries_per_s": entries if not rollout else None,
                 "env_steps_per_step": decisions / args.steps,
