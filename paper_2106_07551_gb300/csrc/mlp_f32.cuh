@@ -324,7 +324,7 @@ struct MlpF32T8 {
         const int c0 = tx * 4, c1 = H / 2 + tx * 4;
         u64 acc[8][4];
         init<NI>(acc, b2, c0, c1);
-#pragma unroll 4
+#pragma unroll 2
         for (int k0 = 0; k0 < H; k0 += 4) {
             float4 ha[8];
 #pragma unroll
