@@ -40,7 +40,7 @@ FP32_LANES_PER_SM = 128
 # the evaluation kernels' traffic is the staging of the population, which does
 # not grow with the hands per pair.
 NCU_TRAFFIC_PER_LAUNCH = {
-    "leduc_eval_f32_t8_kernel": 1477632 + 512,
+    "leduc_eval_f32_t8_kernel": 1441536 + 512,
     "kuhn_eval_kernel": 13312,
     "spread_rollout_f32_kernel<3,18,64>": (428032 + 43692800) * 25,
     "leduc_eval_tc_kernel": 19304960 + 28416,
