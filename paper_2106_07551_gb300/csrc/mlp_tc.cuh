@@ -181,9 +181,14 @@ struct MlpTc {
     // 2's second output half itself, thread 0 arrives on it once h1 is complete
     // and another, otherwise idle thread issues those MMAs (issue_layer2b), so
     // that thread 0's warp is not held while the tensor core retires them.
+    // w2_ready (optional, with its phase parity): an mbarrier whose phase
+    // completes when W2 and W3 have landed in shared memory; thread 0 waits
+    // on it (bounded) before the first layer-2 MMA, so that a restage of
+    // those weights overlaps layer 1 and its epilogue.
     __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bars,
                                    uint32_t& parity, int* err, Out out, uint32_t x_tile,
-                                   bool x_published = false, uint64_t* h1_ready = nullptr) {
+                                   bool x_published = false, uint64_t* h1_ready = nullptr,
+                                   uint64_t* w2_ready = nullptr, uint32_t w2_parity = 0) {
         const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
         const uint32_t s_w1 = smem_u32(smem + kW1), s_w2 = smem_u32(smem + kW2);
         const uint32_t s_w3 = smem_u32(smem + kW3);
@@ -213,8 +218,11 @@ struct MlpTc {
         // h1, first half; then layer 2's outputs 0..127 over h1's first half
         epilogue_half(tbase, kD1, kH1, bias);
         handoff();
-        if (threadIdx.x == 0)
+        if (threadIdx.x == 0) {
+            if (w2_ready && !mbar_wait_bounded(w2_ready, w2_parity, kWaitLimitNs))
+                atomicOr(err, ERRBIT_TIMEOUT);
             issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, false);
+        }
         // h1, second half; then the rest of layer 2: outputs 0..127, then
         // 128..255 into D2b (D1's first half, already read)
         epilogue_half(tbase, kD1 + H / 2, kH1 + H / 4, bias + H / 2);

@@ -84,7 +84,8 @@ __device__ __forceinline__ bool pair_valid(const RolloutArgs& a, int pair) {
 
 __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ __align__(8) uint64_t stage_bar;
+    __shared__ __align__(8) uint64_t stage_bar;             // W1 and the biases staged
+    __shared__ __align__(8) uint64_t w2_bar;                // W2 and W3 staged
     __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t x_full[kGroups][2];    // a group's tile in buffer b is ready
     __shared__ __align__(8) uint64_t lg_full[kGroups][2];   // the logits of that tile are ready
@@ -97,6 +98,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
 
     if (tid == 0) {
         mbar_init(&stage_bar, 1);
+        mbar_init(&w2_bar, 1);
         mbar_init(&mma_bar[0], 1);
         mbar_init(&mma_bar[1], 1);
         for (int g = 0; g < kGroups; ++g) {
@@ -141,13 +143,19 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
                     const int pol = a.pairs[rd.pair * kN + k];
                     if (pol != staged) {
                         // the forwards of the previous agent are complete (each ends
-                        // with an engine barrier): restage
+                        // with an engine barrier): restage, W1 and the biases on
+                        // stage_bar, which every engine thread waits for, W2 and W3
+                        // on w2_bar, which only the MMA thread waits for, before
+                        // layer 2 of the next forward
                         if (tid == 0) {
                             fence_proxy_async_smem();
-                            mbar_arrive_expect_tx(&stage_bar, Eng::kStageBytes);
                             const uint8_t* src = reinterpret_cast<const uint8_t*>(a.arena + a.pol_offset[pol]);
-                            for (uint32_t off = 0; off < Eng::kStageBytes; off += 32768u)
-                                bulk_g2s(smem + off, src + off, min(32768u, Eng::kStageBytes - off), &stage_bar);
+                            mbar_arrive_expect_tx(&stage_bar, Eng::kW2 + (Eng::kStageBytes - Eng::kBias));
+                            bulk_g2s(smem, src, Eng::kW2, &stage_bar);
+                            bulk_g2s(smem + Eng::kBias, src + Eng::kBias, Eng::kStageBytes - Eng::kBias, &stage_bar);
+                            mbar_arrive_expect_tx(&w2_bar, Eng::kBias - Eng::kW2);
+                            for (uint32_t off = Eng::kW2; off < Eng::kBias; off += 32768u)
+                                bulk_g2s(smem + off, src + off, min(32768u, Eng::kBias - off), &w2_bar);
                         }
                         if (!mbar_wait_bounded(&stage_bar, stage_par, kWaitLimitNs) && tid == 0)
                             atomicOr(a.err, ERRBIT_TIMEOUT);
@@ -172,7 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
                                          for (int j = 0; j < kA; ++j) lgg[row * kLgStride + j] = lg[j];
                                      },
                                      smem_u32(smem + kX + (g * 2 + b) * Eng::kXBytes), /*x_published=*/true,
-                                     &h1_bar[g]);
+                                     &h1_bar[g], &w2_bar, stage_par ^ 1u);
                         // the forward ends with an engine barrier: every row's logits are stored
                         if (tid == 0) mbar_arrive_release(&lg_full[g][b]);
                     }
