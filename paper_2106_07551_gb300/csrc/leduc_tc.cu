@@ -70,7 +70,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t x_bar[kGroups];    // a group's rows and headers
     __shared__ __align__(8) uint64_t lg_bar[kGroups];   // a group's logits
-    __shared__ __align__(8) uint64_t h1_bar[kGroups];   // h1 of a group's tile is in tensor memory
+    __shared__ __align__(8) uint64_t h1_bar[kGroups][2];  // h1 of a group's tile stored ([0] used)
     __shared__ __align__(16) uint4 hdr[kGroups][2];     // [group][source CTA]: {rows here, live}
     __shared__ uint32_t tmem_base;
     __shared__ uint32_t dead_s;                         // a bounded wait expired
@@ -92,7 +92,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int g = 0; g < kGroups; ++g) {
             mbar_init(&x_bar[g], 1);
             mbar_init(&lg_bar[g], 1);
-            mbar_init(&h1_bar[g], 1);
+            mbar_init(&h1_bar[g][0], 1);
+            mbar_init(&h1_bar[g][1], 1);
             mbar_arrive_expect_tx(&x_bar[g], kXTx);         // armed for the first step
             mbar_arrive_expect_tx(&lg_bar[g], kLgTx);
         }
@@ -182,7 +183,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                                                                 __float_as_uint(lg[2]), 0u),
                                                      cl::map(&lg_bar[g], src));
                                  },
-                                 smem_u32(smem + kX + g * kXBytes), /*x_published=*/true, &h1_bar[g]);
+                                 smem_u32(smem + kX + g * kXBytes), /*x_published=*/true, h1_bar[g]);
                 }
             }
         }
@@ -273,11 +274,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 // layer 2 of the group's tile in this CTA once the engine has h1
                 // in tensor memory (the engine's own MMA thread is then free for
                 // its epilogue share); a forward needs it before it can finish.
+                // (Issuing all of layer 2 from here measured 52.4 ms against
+                // 49.4: the helper's response then delays layer 2's start.)
                 if (lt == 0) {
                     bool pend = true;
                     const uint64_t t0 = globaltimer_ns();
                     while (!dead_s) {
-                        if (pend && mbar_try_wait(&h1_bar[g], h1_par)) {
+                        if (pend && mbar_try_wait(&h1_bar[g][0], h1_par)) {
                             h1_par ^= 1u;
                             pend = false;
                             tc::fence_after_sync();

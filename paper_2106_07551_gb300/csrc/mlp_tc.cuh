@@ -156,15 +156,34 @@ struct MlpTc {
         pack_chunk(r1, bias ? bias + c + 32 : nullptr, tc::tmem_addr(tbase, 32 * q, hcol + c / 2 + 16));
     }
 
-    // The helper's part of a forward given h1_ready: layer 2's outputs
-    // 128..255 into D2b over all of h1, committed on bars[1]. Called by one
-    // thread after it has waited for h1_ready (and tcgen05-fenced after it).
+    // The helper's part of a forward given h1_ready, called by one thread after
+    // the phase of h1_ready[part] (and tcgen05-fenced after it), in order: part 0
+    // (h1's first half stored) issues layer 2's outputs 0..127 over it; part 1
+    // (all of h1 stored) the rest of those outputs, committed on bars[0], then
+    // outputs 128..255 into D2b over all of h1, committed on bars[1]. One
+    // thread issues every layer-2 MMA, so they execute in order.
     // (Issuing layer 3 from the helper as well was slower: it sits on the
     // forward's critical path, where the helper's response time shows.)
+    // The helper's part of a forward when only layer 2's second output half is
+    // delegated (helper_all false): after the phase of h1_ready[0], outputs
+    // 128..255 into D2b over all of h1, committed on bars[1].
     __device__ static void issue_layer2b(const uint8_t* smem, uint32_t tbase, uint64_t* bars) {
         issue_ta(tbase + kD2b, tbase + kH1, smem_u32(smem + kW2) + (H / 2 / 8) * 128, kLboW, 0, H / 16,
                  tc::instr_desc(128, H / 2, 1), false);
         tc::mma_commit(bars + 1);
+    }
+
+    __device__ static void issue_layer2(const uint8_t* smem, uint32_t tbase, uint64_t* bars, int part) {
+        const uint32_t s_w2 = smem_u32(smem + kW2), idesc_half = tc::instr_desc(128, H / 2, 1);
+        constexpr int kS = H / 16;
+        if (part == 0) {
+            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, false);
+            return;
+        }
+        issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, kS / 2, kS, idesc_half, true);
+        tc::mma_commit(bars);                               // D2a complete
+        issue_ta(tbase + kD2b, tbase + kH1, s_w2 + (H / 2 / 8) * 128, kLboW, 0, kS, idesc_half, false);
+        tc::mma_commit(bars + 1);                           // D2b complete
     }
 
     // Full forward of the 128-row observation tile at shared-memory address
@@ -177,10 +196,17 @@ struct MlpTc {
     // has synchronised since, so MMA 1 issues at once; otherwise the forward
     // fences and synchronises first.
     template <class Out>
-    // h1_ready (optional, an mbarrier of count 1): instead of issuing layer
-    // 2's second output half itself, thread 0 arrives on it once h1 is complete
-    // and another, otherwise idle thread issues those MMAs (issue_layer2b), so
-    // that thread 0's warp is not held while the tensor core retires them.
+    // h1_ready (optional, two mbarriers of count 1): part of layer 2 is issued
+    // by another, otherwise idle thread, so that thread 0's warp is not held
+    // while the tensor core retires those MMAs. helper_all false: thread 0
+    // issues outputs 0..127 and arrives on h1_ready[0] once h1 is complete;
+    // the helper issues outputs 128..255 (issue_layer2b). helper_all true:
+    // thread 0 arrives on h1_ready[0] when h1's first half is stored and on
+    // h1_ready[1] when all of h1 is; the helper issues all of layer 2
+    // (issue_layer2). Two barriers, because both arrivals may land before the
+    // helper looks: on one barrier the second would return its phase parity to
+    // the value the helper waits for. No barrier can run a phase ahead, since
+    // the next forward needs this one's layer 2.
     // w2_ready (optional, with its phase parity): an mbarrier whose phase
     // completes when W2 and W3 have landed in shared memory; thread 0 waits
     // on it (bounded) before the first layer-2 MMA, so that a restage of
@@ -188,7 +214,9 @@ struct MlpTc {
     __device__ static void forward(uint8_t* smem, const float* gbias, uint32_t tbase, uint64_t* bars,
                                    uint32_t& parity, int* err, Out out, uint32_t x_tile,
                                    bool x_published = false, uint64_t* h1_ready = nullptr,
-                                   uint64_t* w2_ready = nullptr, uint32_t w2_parity = 0) {
+                                   uint64_t* w2_ready = nullptr, uint32_t w2_parity = 0,
+                                   bool helper_all = false) {
+        uint64_t* const h1_all = helper_all ? h1_ready : nullptr;   // the helper issues all of layer 2
         const float* bias = kSmemBias ? reinterpret_cast<const float*>(smem + kBias) : gbias;
         const uint32_t s_w1 = smem_u32(smem + kW1), s_w2 = smem_u32(smem + kW2);
         const uint32_t s_w3 = smem_u32(smem + kW3);
@@ -219,24 +247,36 @@ struct MlpTc {
         epilogue_half(tbase, kD1, kH1, bias);
         handoff();
         if (threadIdx.x == 0) {
+            // the W2 wait comes first: with a helper, its acquire reaches the
+            // helper through the release of the arrival below
             if (w2_ready && !mbar_wait_bounded(w2_ready, w2_parity, kWaitLimitNs))
                 atomicOr(err, ERRBIT_TIMEOUT);
-            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, false);
+            if (h1_all) {
+                tc::fence_before_sync();
+                mbar_arrive_release(h1_all);                // part 0 is issued by the helper
+            } else {
+                issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, 0, kS / 2, idesc_half, false);
+            }
         }
         // h1, second half; then the rest of layer 2: outputs 0..127, then
         // 128..255 into D2b (D1's first half, already read)
         epilogue_half(tbase, kD1 + H / 2, kH1 + H / 4, bias + H / 2);
         handoff();
         if (threadIdx.x == 0) {
-            issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, kS / 2, kS, idesc_half, true);
-            tc::mma_commit(bars);                           // D2a complete
-            if (h1_ready) {
+            if (h1_all) {
                 tc::fence_before_sync();
-                mbar_arrive_release(h1_ready);              // D2b is issued by the helper
+                mbar_arrive_release(h1_all + 1);            // part 1 is issued by the helper
             } else {
-                issue_ta(tbase + kD2b, tbase + kH1, s_w2 + (H / 2 / 8) * 128, kLboW, 0, kS, idesc_half,
-                         false);
-                tc::mma_commit(bars + 1);                   // D2b complete
+                issue_ta(tbase + kD2a, tbase + kH1, s_w2, kLboW, kS / 2, kS, idesc_half, true);
+                tc::mma_commit(bars);                       // D2a complete
+                if (h1_ready) {
+                    tc::fence_before_sync();
+                    mbar_arrive_release(h1_ready);          // D2b is issued by the helper
+                } else {
+                    issue_ta(tbase + kD2b, tbase + kH1, s_w2 + (H / 2 / 8) * 128, kLboW, 0, kS,
+                             idesc_half, false);
+                    tc::mma_commit(bars + 1);               // D2b complete
+                }
             }
         }
         wait_mma(bars, 0, parity, err);                     // D2a

@@ -12,8 +12,8 @@
 //  * warps 0-7, the engine: for each agent, the tiles of both episodes
 //    through the tensor-core MLP (hidden activations in tensor memory); each
 //    row's 5 logits go to shared memory, announced on a per-buffer mbarrier.
-//    Layer 2's second output half is issued by the tile's group's first
-//    thread, which waits for those logits anyway;
+//    Layer 2 is issued by the tile's group's first thread, which waits for
+//    those logits anyway;
 //  * warps 8-11 and 12-15, environment groups 0 and 1: two episodes of the
 //    combination in flight, one environment per thread, state in registers.
 //    For each agent a group builds its observations (a bf16 tile in one of two
@@ -89,7 +89,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
     __shared__ __align__(8) uint64_t mma_bar[2];
     __shared__ __align__(8) uint64_t x_full[kGroups][2];    // a group's tile in buffer b is ready
     __shared__ __align__(8) uint64_t lg_full[kGroups][2];   // the logits of that tile are ready
-    __shared__ __align__(8) uint64_t h1_bar[kGroups];       // h1 of a group's tile is in tensor memory
+    __shared__ __align__(8) uint64_t h1_bar[kGroups][2];    // h1 halves of a group's tile stored
     __shared__ uint32_t tmem_base;
 
     float* lgs = reinterpret_cast<float*>(smem + kLgs);
@@ -102,7 +102,8 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
         mbar_init(&mma_bar[0], 1);
         mbar_init(&mma_bar[1], 1);
         for (int g = 0; g < kGroups; ++g) {
-            mbar_init(&h1_bar[g], 1);
+            mbar_init(&h1_bar[g][0], 1);
+            mbar_init(&h1_bar[g][1], 1);
             for (int b = 0; b < 2; ++b) {
                 mbar_init(&x_full[g][b], 1);
                 mbar_init(&lg_full[g][b], 1);
@@ -180,7 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
                                          for (int j = 0; j < kA; ++j) lgg[row * kLgStride + j] = lg[j];
                                      },
                                      smem_u32(smem + kX + (g * 2 + b) * Eng::kXBytes), /*x_published=*/true,
-                                     &h1_bar[g], &w2_bar, stage_par ^ 1u);
+                                     h1_bar[g], &w2_bar, stage_par ^ 1u, /*helper_all=*/true);
                         // the forward ends with an engine barrier: every row's logits are stored
                         if (tid == 0) mbar_arrive_release(&lg_full[g][b]);
                     }
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
         const int g = (warp - 8) >> 2;
         const int e = tid - kEngineThreads - g * 128;     // environment within the block
         uint32_t lg_bits = 0;                              // lg_full[g][b] phase: bit b
-        uint32_t h1_par = 0;
+        uint32_t h1_par = 0, h1_part = 0;
         uint8_t* ag = acts + g * kN * 128;
         for (int64_t it = lo; it < hi;) {
             const Round rd = round_at(it, hi, a.n_episodes);
@@ -212,17 +213,18 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
                     const int bj = j & 1;
                     const uint32_t par = (lg_bits >> bj) & 1u;
                     if (e == 0) {
-                        // while it waits, the group's first thread issues the second
-                        // output half of layer 2 of the group's tile once the engine
-                        // has its h1 in tensor memory (the engine's MMA thread is then
+                        // while it waits, the group's first thread issues layer 2 of
+                        // the group's tile, in two parts as the engine stores h1's
+                        // halves in tensor memory (the engine's MMA thread is then
                         // free for its epilogue share); the forward needs it to finish
                         const uint64_t t0 = globaltimer_ns();
                         bool done = false;
                         while (!done) {
-                            if (mbar_try_wait(&h1_bar[g], h1_par)) {
-                                h1_par ^= 1u;
+                            if (mbar_try_wait(&h1_bar[g][h1_part], (h1_par >> h1_part) & 1u)) {
+                                h1_par ^= 1u << h1_part;
                                 tc::fence_after_sync();
-                                Eng::issue_layer2b(smem, tbase, &mma_bar[0]);
+                                Eng::issue_layer2(smem, tbase, &mma_bar[0], (int)h1_part);
+                                h1_part ^= 1u;
                             }
                             done = mbar_try_wait(&lg_full[g][bj], par);
                             if (!done && globaltimer_ns() - t0 > kWaitLimitNs) {
