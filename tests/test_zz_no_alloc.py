@@ -72,3 +72,37 @@ def test_noalloc_refuses_oversize_and_host_buffers():
                                          10, 0, h_out.ctypes.data_as(C.c_void_p))
     assert code == _abi.MALIB_EINVAL
     ctx.close()
+
+
+@pytest.mark.parametrize("kind", ["kuhn", "leduc"])
+def test_noalloc_captured_in_a_cuda_graph(kind):
+    """The allocation-free call can be captured into a CUDA graph (zero, main
+    and finalize kernels as graph nodes) and replayed: every replay gives the
+    table of the ordinary entry point."""
+    torch = need_gpu()
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2106_07551_gb300 import Context
+    w = (workloads.leduc(pop=3, with_bias=True, seed=78) if kind == "leduc" else workloads.kuhn())
+    n_eps = 2000 if kind == "leduc" else 10_000
+    s = torch.cuda.Stream()
+    ctx = Context(0, s)                      # every call of this context is ordered on s
+    load_population(ctx, w)
+    ref = ctx.eval_payoff(w.pair_ids, n_eps, 12)
+    d_pairs = torch.from_numpy(w.pair_ids).cuda()
+    out = torch.zeros((w.n_pairs, 4), dtype=torch.float64, device="cuda")
+    with torch.cuda.stream(s):               # warm-up outside the capture
+        assert _noalloc(ctx, d_pairs, n_eps, 12, out) == 0, ctx.last_error()
+    s.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        assert _noalloc(ctx, d_pairs, n_eps, 12, out) == 0, ctx.last_error()
+    for _ in range(3):
+        out.fill_(-1.0)
+        g.replay()
+        torch.cuda.synchronize()
+        got = out.cpu().numpy()
+        np.testing.assert_array_equal(got[:, 2:], ref[:, 2:])
+        np.testing.assert_allclose(got[:, :2], ref[:, :2], rtol=1e-12, atol=1e-15)
+    ctx.sync()
+    ctx.close()
