@@ -74,7 +74,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     __shared__ __align__(16) uint4 hdr[kGroups][2];     // [group][source CTA]: {rows here, live}
     __shared__ uint32_t tmem_base;
     __shared__ uint32_t dead_s;                         // a bounded wait expired
-    __shared__ uint32_t eng_flag;                       // engine: 0 run, 1 group done, 2 stop
+    __shared__ uint32_t eng_flag[2];                    // engine: 0 run, 1 group done, 2 stop
+                                                        // (two slots, used alternately)
     __shared__ uint32_t grp_flag[kGroups];              // group: 0 logits, 1 segment done, 2 stop
     __shared__ int wcnt[kGroups][2][4];                 // [group][seat][warp of the group]
     __shared__ unsigned long long next_k[kGroups];
@@ -144,7 +145,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             stage_par ^= 1u;
             tc::fence_before_sync();
             Eng::sync();
-            uint32_t done_bits = 0;
+            uint32_t done_bits = 0, fslot = 0;
             while (done_bits != 3u && !stop) {
                 for (int g = 0; g < kGroups && !stop; ++g) {
                     if (done_bits & (1u << g)) continue;
@@ -155,12 +156,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                             atomicOr(a.err, ERRBIT_TIMEOUT);
                         }
                         mbar_arrive_expect_tx(&x_bar[g], kXTx);   // armed for the group's next step
-                        eng_flag = dead_s ? 2u : ((hdr[g][0].y | hdr[g][1].y) == 0 ? 1u : 0u);
+                        eng_flag[fslot] = dead_s ? 2u : ((hdr[g][0].y | hdr[g][1].y) == 0 ? 1u : 0u);
                     }
                     x_bits ^= 1u << g;
                     Eng::sync();
-                    const uint32_t f = eng_flag;
-                    Eng::sync();                                  // eng_flag read by all
+                    // a slot is rewritten two decisions later, after the next one's
+                    // barrier, which every thread passes only once it has read it
+                    const uint32_t f = eng_flag[fslot];
+                    fslot ^= 1u;
                     if (f == 2u) { stop = true; break; }
                     if (f == 1u) {
                         // no live hand of the group in either CTA: tell both sources
