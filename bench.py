@@ -43,7 +43,7 @@ NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1441536 + 512,
     "kuhn_eval_kernel": 13312,
     "spread_rollout_f32_kernel<3,18,64>": (428032 + 43692800) * 25,
-    "leduc_eval_tc_kernel": 19302400 + 26624,
+    "leduc_eval_tc_kernel": 19302400 + 24576,
     "spread_rollout_f32_kernel<3,14,64,true>": (444160 + 24321792) * 25,
     "spread_rollout_tc_kernel": (20857088 + 1914217984) * 2,
 }
