@@ -66,6 +66,11 @@ def _L():
                 "orc_spread_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                               C.c_int, C.c_int, C.c_int, i64, i64, i64, P, i32, i64,
                                               u64, P, P, P, P, P, C.c_int, C.c_float]),
+                "orc_sl_reset": (None, [u64, u64, P]),
+                "orc_sl_step": (None, [P, P, P]),
+                "orc_sl_obs": (None, [P, P]),
+                "orc_sl_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
+                                          P, i32, i64, u64, P, P, P, P, P, C.c_int]),
                 "orc_adversary_reset": (None, [u64, u64, P]),
                 "orc_adversary_step": (None, [P, P, P]),
                 "orc_adversary_obs": (None, [P, P]),
@@ -263,6 +268,56 @@ def spread_rollout(params_list, dims, N, L, T, n_envs, pairs, n_episodes, seed, 
 # state: px,py,vx,vy of agents 0 (adversary), 1, 2; lx,ly of landmarks 0, 1;
 # then the target landmark's index (17 floats).
 ADV_N, ADV_L, ADV_OBS, ADV_STATE = 3, 2, 14, 17
+
+
+SL_N, SL_L, SL_OBS, SL_STATE = 2, 3, 11, 16
+
+
+def sl_reset(g: int, seed: int) -> np.ndarray:
+    """Simple speaker listener: state [px,py,vx,vy] x 2, [lx,ly] x 3, target, message."""
+    st = np.zeros(SL_STATE, np.float32)
+    _L().orc_sl_reset(C.c_uint64(g), C.c_uint64(seed), _p(st))
+    return st
+
+
+def sl_step(state: np.ndarray, actions) -> tuple[np.ndarray, np.ndarray]:
+    """One transition; actions [message, move]; rewards [speaker, listener]."""
+    st = _c(state, np.float32).copy()
+    act = _c(actions, np.int32)
+    rew = np.zeros(SL_N, np.float32)
+    _L().orc_sl_step(_p(st), _p(act), _p(rew))
+    return st, rew
+
+
+def sl_obs(state: np.ndarray) -> np.ndarray:
+    st = _c(state, np.float32)
+    out = np.zeros((SL_N, SL_OBS), np.float32)
+    _L().orc_sl_obs(_p(st), _p(out))
+    return out
+
+
+def sl_rollout(params_list, dims, T, n_envs, pairs, n_episodes, seed, bf16=False,
+               env_lo=0, env_hi=None, ext_logits=None, n_threads=0):
+    """Rollout over envs [env_lo, env_hi) of the simple speaker listener (2
+    agents, obs 11, 5 actions, the speaker's 3 and 4 illegal). Returns the
+    arrays of spread_rollout."""
+    env_hi = n_envs if env_hi is None else env_hi
+    W = env_hi - env_lo
+    i, h1, h2, A = dims
+    assert i == SL_OBS and A == 5
+    arrs, tbl = _param_table(params_list)
+    pairs = _c(pairs, np.int32).reshape(-1, SL_N)
+    out = dict(obs=np.zeros((n_episodes, T, W, SL_N, i), np.float32),
+               action=np.zeros((n_episodes, T, W, SL_N), np.int8),
+               reward=np.zeros((n_episodes, T, W, SL_N), np.float32),
+               logits=np.zeros((n_episodes, T, W, SL_N, A), np.float32))
+    ext = None if ext_logits is None else _c(ext_logits, np.float32).reshape(n_episodes, T, W, SL_N, A)
+    _L().orc_sl_rollout(C.cast(tbl, C.c_void_p), h1, h2, int(bf16), T, n_envs, env_lo, env_hi,
+                        _p(pairs), pairs.shape[0], n_episodes, C.c_uint64(seed), _p(ext),
+                        _p(out["obs"]), _p(out["action"]), _p(out["reward"]), _p(out["logits"]),
+                        n_threads)
+    del arrs
+    return out
 
 
 def adversary_reset(g: int, seed: int) -> np.ndarray:

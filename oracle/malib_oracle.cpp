@@ -15,6 +15,9 @@
 //  * App. B.1 "Simple Spread": N agents cover N landmarks; reward is minus the
 //    sum over landmarks of the distance to the closest agent, minus one per
 //    collision.
+//  * App. B.1 "Simple Speaker Listener": a speaker that cannot move sends one of
+//    three messages naming the target landmark; the listener, which cannot
+//    speak, navigates to it; both are rewarded by the listener's distance.
 //  * App. B.1 "Simple Adversary": one adversary and two good agents, two
 //    landmarks of which one is the target; good agents are rewarded for being
 //    close to the target and for the adversary being far from it, the adversary
@@ -29,9 +32,11 @@
 //
 // Parity status: Philox, det_expf, Kuhn (exact enumeration), Leduc (tree
 // enumeration, hand-worked hands), spread (closed-form single steps and
-// invariants) and the simple adversary (hand-worked geometry, the reward
-// identity against fp64, the spread dynamics and reset, symmetries) are pinned
-// by the CPU tests; episode returns of the particle scenarios beyond those
+// invariants), the simple adversary (hand-worked geometry, the reward
+// identity against fp64, the spread dynamics and reset, symmetries) and the
+// simple speaker listener (hand-worked geometry, the one-step message delay,
+// the immobile speaker, the spread dynamics and reset, the target draw) are
+// pinned by the CPU tests; episode returns of the particle scenarios beyond those
 // invariants are "parity unpinned" (no closed form exists).
 
 #include <algorithm>
@@ -647,6 +652,67 @@ void adversary_step(Adversary& a, const int* action, float* reward) {
     reward[2] = reward[1];
 }
 
+// ---------------------------------------------------------------------------
+// Simple speaker listener (App. B.1; readings of its description and of the
+// simple reference scenario it is said to resemble, constants of the spread
+// scenario): agent 0 is the speaker, which does not move and whose action
+// 0..2 is the message it sends (actions 3 and 4 are not legal for it); agent 1
+// the listener, which moves with the spread dynamics and cannot speak; three
+// landmarks, one of them the target. Reset: agents and landmarks as for spread
+// (same chance counters), the target = pick(x of the chance draw with step
+// field 0xC0000000, 3), no message yet. The listener observes the message the
+// speaker sent at the previous step. Reward after the move, shared by both
+// agents: -d(p_1, target). Observations (11 floats): speaker - one-hot of the
+// target, zeros; listener - velocity, landmarks - p_1 (ascending), one-hot of
+// the last message (zeros before the first).
+// ---------------------------------------------------------------------------
+struct SpeakerListener {
+    Spread s;
+    int target;
+    int msg;            // -1: none yet
+};
+
+void sl_reset(SpeakerListener& a, uint64_t g, uint64_t seed) {
+    spread_reset(a.s, 2, 3, g, seed);
+    a.target = (int)pick(draw(g, 0xC0000000u, CHANCE, seed).x[0], 3);
+    a.msg = -1;
+}
+
+void sl_obs(const SpeakerListener& a, int i, float* o) {
+    for (int k = 0; k < 11; ++k) o[k] = 0.0f;
+    const Spread& s = a.s;
+    if (i == 0) {
+        o[a.target] = 1.0f;
+        return;
+    }
+    int k = 0;
+    o[k++] = s.vx[1]; o[k++] = s.vy[1];
+    for (int l = 0; l < 3; ++l) { o[k++] = s.lx[l] - s.px[1]; o[k++] = s.ly[l] - s.py[1]; }
+    if (a.msg >= 0) o[k + a.msg] = 1.0f;
+}
+
+void sl_step(SpeakerListener& a, const int* action, float* reward) {
+    Spread& s = a.s;
+    a.msg = action[0];
+    float fx = 0.0f, fy = 0.0f;
+    switch (action[1]) {
+        case 1: fx = 1.0f; break;
+        case 2: fx = -1.0f; break;
+        case 3: fy = 1.0f; break;
+        case 4: fy = -1.0f; break;
+        default: break;
+    }
+    s.vx[1] = s.vx[1] * 0.75f;
+    s.vy[1] = s.vy[1] * 0.75f;
+    s.vx[1] = s.vx[1] + fx * 0.1f;
+    s.vy[1] = s.vy[1] + fy * 0.1f;
+    s.px[1] = s.px[1] + s.vx[1] * 0.1f;
+    s.py[1] = s.py[1] + s.vy[1] * 0.1f;
+    const float d = dist2d(s.px[1], s.py[1], s.lx[a.target], s.ly[a.target]);
+    reward[0] = -d;
+    reward[1] = -d;
+}
+
 }  // namespace
 
 // ===========================================================================
@@ -938,6 +1004,87 @@ void orc_adversary_rollout(const float* const* params, int h1, int h2, int bf16,
             }
             float r[3];
             adversary_step(adv, act, r);
+            if (reward)
+                for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
+        }
+    });
+}
+
+// ---- Simple speaker listener ----
+// state: px,py,vx,vy of the 2 agents, lx,ly of the 3 landmarks, the target
+// index and the last message (-1: none) as floats ([4*2 + 2*3 + 2] = 16).
+static void sl_load(const float* state, SpeakerListener& a) {
+    a.s.N = 2; a.s.L = 3;
+    for (int i = 0; i < 2; ++i) {
+        a.s.px[i] = state[4 * i]; a.s.py[i] = state[4 * i + 1];
+        a.s.vx[i] = state[4 * i + 2]; a.s.vy[i] = state[4 * i + 3];
+    }
+    for (int l = 0; l < 3; ++l) { a.s.lx[l] = state[8 + 2 * l]; a.s.ly[l] = state[8 + 2 * l + 1]; }
+    a.target = (int)state[14];
+    a.msg = (int)state[15];
+}
+static void sl_store(const SpeakerListener& a, float* state) {
+    for (int i = 0; i < 2; ++i) {
+        state[4 * i] = a.s.px[i]; state[4 * i + 1] = a.s.py[i];
+        state[4 * i + 2] = a.s.vx[i]; state[4 * i + 3] = a.s.vy[i];
+    }
+    for (int l = 0; l < 3; ++l) { state[8 + 2 * l] = a.s.lx[l]; state[8 + 2 * l + 1] = a.s.ly[l]; }
+    state[14] = (float)a.target;
+    state[15] = (float)a.msg;
+}
+
+void orc_sl_reset(uint64_t g, uint64_t seed, float* state) {
+    SpeakerListener a;
+    sl_reset(a, g, seed);
+    sl_store(a, state);
+}
+
+void orc_sl_step(float* state, const int32_t* action, float* reward) {
+    SpeakerListener a;
+    sl_load(state, a);
+    sl_step(a, action, reward);
+    sl_store(a, state);
+}
+
+void orc_sl_obs(const float* state, float* obs /*[2][11]*/) {
+    SpeakerListener a;
+    sl_load(state, a);
+    for (int i = 0; i < 2; ++i) sl_obs(a, i, obs + i * 11);
+}
+
+// Rollout as orc_spread_rollout, for the simple speaker listener (N = 2, obs
+// 11, 5 actions of which the speaker may take 0..2).
+void orc_sl_rollout(const float* const* params, int h1, int h2, int bf16, int T, int64_t n_envs,
+                    int64_t env_lo, int64_t env_hi, const int32_t* pairs, int32_t n_pairs,
+                    int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
+                    int8_t* action, float* reward, float* logits, int n_threads) {
+    const int N = 2, in = 11, A = 5;
+    int64_t per = n_envs / n_pairs;
+    int64_t W = env_hi - env_lo;
+    parallel_for(W * n_episodes, n_threads, [&](int64_t job) {
+        int64_t ep = job / W, e = env_lo + job % W;
+        int64_t row = e / per;
+        SpeakerListener sl;
+        uint64_t g = (uint64_t)ep * (uint64_t)n_envs + (uint64_t)e;
+        sl_reset(sl, g, seed);
+        for (int t = 0; t < T; ++t) {
+            int act[2];
+            for (int i = 0; i < N; ++i) {
+                int64_t idx = ((ep * T + t) * W + (e - env_lo)) * N + i;
+                float o[11], lg[8];
+                sl_obs(sl, i, o);
+                Mlp m{params[pairs[row * N + i]], in, h1, h2, A, bf16};
+                mlp_logits(m, o, lg);
+                uint8_t legal[8] = {1, 1, 1, 1, 1, 1, 1, 1};
+                if (i == 0) legal[3] = legal[4] = 0;          // the speaker only speaks
+                float u = uniform24(draw(g, (uint32_t)t, (uint32_t)i, seed).x[0]);
+                act[i] = sample_masked(ext_logits ? ext_logits + idx * A : lg, legal, A, u);
+                if (obs) std::memcpy(obs + idx * in, o, sizeof(float) * in);
+                if (logits) std::memcpy(logits + idx * A, lg, sizeof(float) * A);
+                if (action) action[idx] = (int8_t)act[i];
+            }
+            float r[2];
+            sl_step(sl, act, r);
             if (reward)
                 for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
         }
