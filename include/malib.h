@@ -50,7 +50,8 @@ typedef enum malib_env_kind {
     MALIB_ENV_KUHN = 1,       /* Kuhn poker: 3 cards, ante 1, one bet of 1, 2 seats */
     MALIB_ENV_LEDUC = 2,      /* Leduc hold'em: 6 cards, 2 rounds, raises 2 then 4 */
     MALIB_ENV_SPREAD = 3,     /* cooperative particle spread (App. B.1) */
-    MALIB_ENV_ADVERSARY = 4   /* simple adversary (App. B.1): 1 adversary, 2 good agents */
+    MALIB_ENV_ADVERSARY = 4,  /* simple adversary (App. B.1): 1 adversary, 2 good agents */
+    MALIB_ENV_SPEAKER_LISTENER = 5  /* simple speaker listener (App. B.1): speaker, listener */
 } malib_env_kind;
 
 typedef enum malib_policy_kind {
@@ -79,8 +80,10 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  *           n_actions 5 (noop, +x, -x, +y, -y), episode_len >= 1
  *   ADVERSARY: n_agents 3 (agent 0 the adversary, 1 and 2 the good agents),
  *           n_landmarks 2, obs_dim 14, n_actions 5, episode_len >= 1
+ *   SPEAKER_LISTENER: n_agents 2 (agent 0 the speaker, 1 the listener),
+ *           n_landmarks 3, obs_dim 11, n_actions 5, episode_len >= 1
  * n_envs is the number of parallel environments of a rollout (SPREAD,
- * ADVERSARY).
+ * ADVERSARY, SPEAKER_LISTENER).
  * SPREAD reward of agent i after a step (App. B.1), with cover = sum over
  * landmarks of the distance to the nearest agent and coll_i = the number of
  * agents closer than 0.3 to agent i:
@@ -94,6 +97,13 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  * -min(d(p_1), d(p_2)) + d(p_0). Observation of agent i: velocity, position,
  * target - p_i (zeros for the adversary, which is not told the target), the two
  * landmarks - p_i, the other agents - p_i (ascending).
+ * SPEAKER_LISTENER (App. B.1 simple speaker listener): at reset one of the
+ * three landmarks is drawn as the target. The speaker does not move; its action
+ * 0..2 is a message (actions 3 and 4 are never drawn for it). The listener
+ * moves with the spread dynamics and observes the message sent at the previous
+ * step. Both agents get r = -d(p_1, target) after the step. Observations (11
+ * floats): speaker - one-hot of the target, zeros; listener - velocity, the
+ * three landmarks - p_1, one-hot of the last message (zeros before the first).
  */
 typedef struct malib_env_spec {
     int32_t env_kind;

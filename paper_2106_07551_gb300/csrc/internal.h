@@ -79,7 +79,7 @@ struct EvalArgs {
 };
 
 struct RolloutArgs {
-    int32_t env_kind;            // MALIB_ENV_SPREAD or MALIB_ENV_ADVERSARY
+    int32_t env_kind;            // MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY or MALIB_ENV_SPEAKER_LISTENER
     const float* arena;
     const int64_t* pol_offset;
     int32_t n_pol;
@@ -176,6 +176,7 @@ cudaError_t launch_lp_nash(const double* P, int32_t G, int32_t m, int32_t n, int
 
 bool leduc_f32_supported(int hidden);
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden);
-bool adversary_f32_supported(int hidden);
+// The simple adversary and simple speaker listener scenarios (hidden width 64).
+bool scenario_f32_supported(int hidden);
 
 }  // namespace malib

@@ -162,6 +162,12 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
                             "adversary spec needs n_agents 3, n_landmarks 2, obs_dim 14, n_actions 5");
             if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
             break;
+        case MALIB_ENV_SPEAKER_LISTENER:
+            if (s->n_agents != 2 || s->n_landmarks != 3 || s->obs_dim != 11 || s->n_actions != 5)
+                return fail(c, MALIB_EINVAL,
+                            "speaker-listener spec needs n_agents 2, n_landmarks 3, obs_dim 11, n_actions 5");
+            if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
+            break;
         default:
             return fail(c, MALIB_EINVAL, "unknown env_kind %d", s->env_kind);
     }
@@ -634,8 +640,10 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
     if (!same_env(c->spec, *spec))
         return fail(c, MALIB_ESTATE, "rollout spec differs from the population's environment");
-    const bool adv = spec->env_kind == MALIB_ENV_ADVERSARY;
-    if (spec->env_kind != MALIB_ENV_SPREAD && !adv)
+    // scenarios of the fp32 rollout kernel other than spread (one policy width, hidden 64)
+    const bool other = spec->env_kind == MALIB_ENV_ADVERSARY ||
+                       spec->env_kind == MALIB_ENV_SPEAKER_LISTENER;
+    if (spec->env_kind != MALIB_ENV_SPREAD && !other)
         return fail(c, MALIB_EUNSUPPORTED, "rollout is built for the particle environments");
     if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");
     if (spec->n_envs < 1 || spec->n_envs % n_pairs != 0)
@@ -653,9 +661,9 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
         if (((uintptr_t)p & 15u) != 0) return fail(c, MALIB_EINVAL, "trajectory buffers must be 16-byte aligned");
     }
     const int64_t epp = spec->n_envs / n_pairs;
-    const bool use_tc = !adv && c->tc_layout && spread_tc_supported(spec->n_agents, spec->obs_dim,
+    const bool use_tc = !other && c->tc_layout && spread_tc_supported(spec->n_agents, spec->obs_dim,
                                                                     spec->n_actions, epp);
-    const bool f32_ok = adv ? adversary_f32_supported(c->dims[1])
+    const bool f32_ok = other ? scenario_f32_supported(c->dims[1])
                             : spread_f32_supported(spec->n_agents, spec->obs_dim, c->dims[1]);
     if (!use_tc && (c->pol_dtype != MALIB_F32 || c->dims[1] != c->dims[2] || !f32_ok || epp > 128))
         return fail(c, MALIB_EUNSUPPORTED,

@@ -13,9 +13,10 @@
 // engine. The observation tile is laid out [row][agent][obs_pad], the order of
 // the trajectory, so each episode's observations of a step leave shared memory
 // as one bulk copy; actions, rewards and done flags are stored per thread.
-#include <type_traits>
-
+// The same kernel, templated on the scenario, runs the simple adversary and the
+// simple speaker listener (App. B.1) with their own environment code.
 #include "adversary_env.cuh"
+#include "sl_env.cuh"
 #include "device_common.cuh"
 #include "internal.h"
 #include "mlp_f32.cuh"
@@ -40,11 +41,30 @@ struct SpreadF32Smem {
     static_assert(kBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
 };
 
-// kAdv: false - cooperative spread (N agents, N landmarks); true - the simple
-// adversary (N = 3, two landmarks, obs 14).
-template <int N, int IN, int H, bool kAdv = false>
+// kScen: kSpread - cooperative spread (N agents, N landmarks); kAdversary - the
+// simple adversary (N = 3, two landmarks, obs 14); kSpeakerListener - the simple
+// speaker listener (N = 2, three landmarks, obs 11; the speaker may take
+// actions 0..2 only).
+constexpr int kSpread = 0, kAdversary = 1, kSpeakerListener = 2;
+
+template <int kScen, int N>
+struct ScenarioEnv {
+    using type = SpreadEnv<N>;
+};
+template <int N>
+struct ScenarioEnv<kAdversary, N> {
+    using type = AdvEnv;
+};
+template <int N>
+struct ScenarioEnv<kSpeakerListener, N> {
+    using type = SlEnv;
+};
+
+template <int N, int IN, int H, int kScen = kSpread>
 __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs a) {
-    static_assert(!kAdv || (N == 3 && IN == kAdvObs), "the simple adversary has 3 agents, obs 14");
+    static_assert(kScen != kAdversary || (N == 3 && IN == kAdvObs), "the simple adversary has 3 agents, obs 14");
+    static_assert(kScen != kSpeakerListener || (N == 2 && IN == kSlObs),
+                  "the simple speaker listener has 2 agents, obs 11");
     using SM = SpreadF32Smem<N, IN, H>;
     using M = typename SM::M;
     using L = typename SM::L;
@@ -110,9 +130,10 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
         const bool mine = slot < n_slots && v < epp;
         const int64_t env = (int64_t)pair * epp + v;
         const uint64_t g = (uint64_t)ep * (uint64_t)a.n_envs + (uint64_t)env;
-        std::conditional_t<kAdv, AdvEnv, SpreadEnv<N>> s;
+        typename ScenarioEnv<kScen, N>::type s;
         if (mine) {
-            if constexpr (kAdv) adv_reset(s, g, a.seed);
+            if constexpr (kScen == kAdversary) adv_reset(s, g, a.seed);
+            else if constexpr (kScen == kSpeakerListener) sl_reset(s, g, a.seed);
             else spread_reset<N>(s, g, a.seed);
         }
 
@@ -121,7 +142,8 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
                     float o[XS];
-                    if constexpr (kAdv) adv_obs<XS>(s, i, o);
+                    if constexpr (kScen == kAdversary) adv_obs<XS>(s, i, o);
+                    else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, i, o);
                     else spread_obs<N, XS>(s, i, o);
                     float4* xr = reinterpret_cast<float4*>(X + (tid * N + i) * XS);
 #pragma unroll
@@ -158,12 +180,14 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 #pragma unroll
                     for (int k = 0; k < 5; ++k) lg[k] = LG[(i * R + tid) * M::LS + k];
                     const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
-                    act[i] = sample_masked<5>(lg, 0x1Fu, uu);
+                    const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : 0x1Fu;
+                    act[i] = sample_masked<5>(lg, legal, uu);
                     if (a.logits)
 #pragma unroll
                         for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
                 }
-                if constexpr (kAdv) adv_step(s, act, r);
+                if constexpr (kScen == kAdversary) adv_step(s, act, r);
+                else if constexpr (kScen == kSpeakerListener) sl_step(s, act, r);
                 else spread_step<N>(s, act, r, a.local_ratio);
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
@@ -179,23 +203,23 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
     if (tid == 0) bulk_wait_all();   // the trajectory copies have landed
 }
 
-template <int N, int IN, int H, bool kAdv = false>
+template <int N, int IN, int H, int kScen = kSpread>
 cudaError_t launch_spread_nih(const RolloutArgs& a, int n_sm, cudaStream_t s) {
     using SM = SpreadF32Smem<N, IN, H>;
-    cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H, kAdv>,
+    cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H, kScen>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SM::kBytes);
     if (err != cudaSuccess) return err;
     const int64_t units = (int64_t)a.n_pairs * ((a.n_episodes + 1) / 2);
     int64_t grid = units < n_sm ? units : n_sm;
     if (grid < 1) grid = 1;
-    spread_rollout_f32_kernel<N, IN, H, kAdv><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
+    spread_rollout_f32_kernel<N, IN, H, kScen><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-bool adversary_f32_supported(int hidden) { return hidden == 64; }
+bool scenario_f32_supported(int hidden) { return hidden == 64; }
 
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden) {
     return n_agents == 3 && obs_dim == 18 && hidden == 64;
@@ -204,7 +228,11 @@ bool spread_f32_supported(int n_agents, int obs_dim, int hidden) {
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0 || a.n_episodes == 0) return cudaSuccess;
     if (a.env_kind == MALIB_ENV_ADVERSARY) {
-        if (hidden == 64) return launch_spread_nih<3, kAdvObs, 64, true>(a, n_sm, s);
+        if (hidden == 64) return launch_spread_nih<3, kAdvObs, 64, kAdversary>(a, n_sm, s);
+        return cudaErrorInvalidValue;
+    }
+    if (a.env_kind == MALIB_ENV_SPEAKER_LISTENER) {
+        if (hidden == 64) return launch_spread_nih<2, kSlObs, 64, kSpeakerListener>(a, n_sm, s);
         return cudaErrorInvalidValue;
     }
     if (a.n_agents == 3 && a.obs_dim == 18 && hidden == 64) return launch_spread_nih<3, 18, 64>(a, n_sm, s);

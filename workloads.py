@@ -26,6 +26,7 @@ import numpy as np
 SEED_BASE = 2106075510
 
 ENV_KUHN, ENV_LEDUC, ENV_SPREAD, ENV_ADVERSARY = 1, 2, 3, 4
+ENV_SPEAKER_LISTENER = 5
 POL_TABULAR, POL_MLP = 1, 2
 F32, BF16 = 0, 1
 
@@ -155,6 +156,24 @@ def adversary(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_episodes: i
         w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
     n_pairs = max(1, n_envs // envs_per_pair)
     w.pair_ids = rng.integers(0, pop, size=(n_pairs, 3)).astype(np.int32)
+    return w
+
+
+def speaker_listener(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_episodes: int = 1,
+                     episode_len: int = 25, envs_per_pair: int = 128, seed: int = SEED_BASE + 7,
+                     with_bias: bool = False, name: str | None = None) -> Workload:
+    """Simple speaker listener (App. B.1): agent 0 the speaker, agent 1 the
+    listener, three landmarks; MLP 11-hidden-hidden-5 fp32 policies from one
+    shared pool, assigned by the seed per (block of envs_per_pair envs, agent
+    slot)."""
+    rng = np.random.default_rng(seed)
+    dims = (11, hidden, hidden, 5)
+    w = Workload(name or f"speaker_listener_{n_envs}env_mlp{hidden}_f32", ENV_SPEAKER_LISTENER, 2, 3,
+                 11, 5, episode_len, n_envs, n_episodes=n_episodes, seed=seed)
+    for _ in range(pop):
+        w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
+    n_pairs = max(1, n_envs // envs_per_pair)
+    w.pair_ids = rng.integers(0, pop, size=(n_pairs, 2)).astype(np.int32)
     return w
 
 
