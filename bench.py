@@ -28,23 +28,22 @@ METRIC = "env-steps/sec incl. policy inference and payoff entries/sec on 1 GB300
 UNIT = "env-steps/s"
 SM_COUNT_GB300 = 152
 FP32_LANES_PER_SM = 128
-# dram bytes (read + write) of one launch of the dominant kernel from the ncu
-# capture summarised under profiles/ (None until taken for the current kernel).
-# leduc_eval_f32_t8_kernel: profiles/leduc_eval_f32_t8_kernel_c2.md (the one-time
-# read of the population; independent of the hand count).
 # DRAM bytes (read + write) per launch of each workload's dominant kernel, from
-# ncu captures of small cases of the same kernels (profiles/*.md give the
-# commands). Trajectory writes grow with the episodes, so the spread figures are
-# scaled to the benchmark's episode counts (C3 and the simple adversary: 4 -> 100
-# episodes, C4: 1 -> 2);
+# ncu (profiles/*.md give the commands). The fp32 rollout kernels were captured
+# on the benchmark's own workload with the two dram counters alone (one pass);
+# about 62 MB of trajectory lines are still dirty in L2 when such a kernel ends,
+# so their writes fall that much short of the bytes stored. The spread N=8 bf16
+# figure is a one-episode capture x 2 (65,536 environments: one episode's output
+# is 15x the L2, so the traffic grows in proportion);
 # the evaluation kernels' traffic is the staging of the population, which does
 # not grow with the hands per pair.
 NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1441536 + 512,
     "kuhn_eval_kernel": 13312,
-    "spread_rollout_f32_kernel<3,18,64>": (428032 + 43692800) * 25,
+    "spread_rollout_f32_kernel<3,18,64,0>": 1373184 + 2559883520,
     "leduc_eval_tc_kernel": 19302400 + 24576,
-    "spread_rollout_f32_kernel<3,14,64,true>": (444160 + 24321792) * 25,
+    "spread_rollout_f32_kernel<3,14,64,1>": 1683968 + 2068428800,
+    "spread_rollout_f32_kernel<2,11,64,2>": 1547520 + 1034004736,
     "spread_rollout_tc_kernel": (20857088 + 1914217984) * 2,
 }
 
@@ -60,8 +59,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "leduc_bf16", "spread8",
-                                           "meta"],
+    ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "speaker_listener",
+                                           "leduc_bf16", "spread8", "meta"],
                     default="leduc")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -175,6 +174,8 @@ def workload(name: str, rank: int, hands=None):
         w = workloads.config(4, **({"n_episodes": 2} if hands is None else over))
     elif name == "adversary3":
         w = workloads.adversary(n_envs=4096, pop=16, n_episodes=100 if hands is None else hands)
+    elif name == "speaker_listener":
+        w = workloads.speaker_listener(n_envs=4096, pop=16, n_episodes=100 if hands is None else hands)
     else:
         w = workloads.config(3, **({"n_episodes": 100} if hands is None else over))
     return w
@@ -197,6 +198,10 @@ def config_of(w, name):
                 "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
     if name == "adversary3":
         return {"workload": f"simple_adversary_4096env_mlp14-64-64-5_f32_{w.n_episodes}episodes",
+                "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
+                "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
+    if name == "speaker_listener":
+        return {"workload": f"simple_speaker_listener_4096env_mlp11-64-64-5_f32_{w.n_episodes}episodes",
                 "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
                 "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
     if name == "kuhn":
@@ -250,6 +255,9 @@ def oracle_rollout_sample(w, name, target_s: float, threads: int):
         if name == "adversary3":
             oracle.adversary_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, eps, w.seed,
                                      env_lo=0, env_hi=n, n_threads=threads)
+        elif name == "speaker_listener":
+            oracle.sl_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, eps, w.seed,
+                              env_lo=0, env_hi=n, n_threads=threads)
         else:
             oracle.spread_rollout(params, dims, w.n_agents, w.n_landmarks, w.episode_len, w.n_envs,
                                   w.pair_ids, eps, w.seed, bf16=bf16, env_lo=0, env_hi=n,
@@ -380,7 +388,7 @@ def run_ours(args):
     d_pairs = torch.from_numpy(w.pair_ids).to(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     seed0 = w.seed + 1_000_003 * rank
-    rollout = args.workload in ("spread3", "spread8", "adversary3")
+    rollout = args.workload in ("spread3", "spread8", "adversary3", "speaker_listener")
     if rollout:
         traj = alloc_traj(spec, w.n_episodes)
         steps_per_call = w.n_envs * w.episode_len * w.n_episodes
@@ -440,8 +448,9 @@ def run_ours(args):
     achieved = (decisions * flop_per_unit / args.steps) / (kern_ms / kern_n / 1e3) / 1e12 \
         if kern_n else 0.0
     kname = {"leduc": "leduc_eval_f32_t8_kernel", "kuhn": "kuhn_eval_kernel",
-             "spread3": "spread_rollout_f32_kernel<3,18,64>",
-             "adversary3": "spread_rollout_f32_kernel<3,14,64,true>",
+             "spread3": "spread_rollout_f32_kernel<3,18,64,0>",
+             "adversary3": "spread_rollout_f32_kernel<3,14,64,1>",
+             "speaker_listener": "spread_rollout_f32_kernel<2,11,64,2>",
              "leduc_bf16": "leduc_eval_tc_kernel",
              "spread8": "spread_rollout_tc_kernel"}[args.workload]
     basis = (f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"

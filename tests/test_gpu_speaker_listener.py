@@ -82,4 +82,13 @@ def test_invalid_speaker_listener_arguments():
     with pytest.raises(MalibError, match="EINVAL"):      # local_ratio is a spread option
         spec = spec_of(w, local_ratio=0.5)
         ctx.rollout(spec, w.pair_ids, 1, 0, alloc_traj(spec, 1))
+    from paper_2106_07551_gb300 import make_spec
+    bad = [dict(n_agents=3), dict(n_landmarks=2), dict(obs_dim=12), dict(n_envs=62)]
+    for over in bad:                                     # App. B.1's 2 agents, 3 landmarks
+        kw = dict(n_agents=2, obs_dim=11, n_landmarks=3, n_envs=64) | over
+        spec = make_spec(w.env_kind, kw["n_agents"], kw["obs_dim"], w.n_actions, kw["n_landmarks"],
+                         w.episode_len, kw["n_envs"], 0, None)
+        with pytest.raises(MalibError, match="EINVAL"):
+            ctx.rollout(spec, w.pair_ids, 1, 0, alloc_traj(spec, 1))
+    ctx.sync()
     ctx.close()
