@@ -55,6 +55,7 @@ def _L():
                 "orc_mlp_forward": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, i64, P]),
                 "orc_kuhn_exact": (C.c_double, [P, P]),
                 "orc_kuhn_eval": (None, [P, P, i32, i64, u64, P, P, i64, C.c_int]),
+                "orc_kuhn_hands": (None, [P, P, u64, i64, u64, P]),
                 "orc_leduc_deal": (None, [u64, u64, P]),
                 "orc_leduc_play": (C.c_int, [C.c_int, C.c_int, C.c_int, P, C.c_int, P, P, P, P, P, P]),
                 "orc_leduc_exact": (C.c_double, [P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int]),
@@ -149,6 +150,14 @@ def kuhn_eval(tables: np.ndarray, pairs: np.ndarray, n_episodes: int, seed: int,
     _L().orc_kuhn_eval(_p(tables), _p(pairs), n, n_episodes, C.c_uint64(seed), _p(res),
                        _p(trace), n_trace, n_threads)
     return res, trace
+
+
+def kuhn_hands(pol0: np.ndarray, pol1: np.ndarray, g0: int, n: int, seed: int) -> np.ndarray:
+    """Traces int32 [n][8] (as kuhn_eval's) of the hands with global ids g0 .. g0 + n - 1."""
+    a, b = _c(pol0, np.float32), _c(pol1, np.float32)
+    trace = np.zeros((n, 8), dtype=np.int32)
+    _L().orc_kuhn_hands(_p(a), _p(b), C.c_uint64(g0), n, C.c_uint64(seed), _p(trace))
+    return trace
 
 
 # ---------------------------------------------------------------- Leduc

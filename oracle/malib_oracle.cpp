@@ -771,6 +771,22 @@ void orc_kuhn_eval(const float* pol, const int32_t* pairs, int32_t n_pairs, int6
     });
 }
 
+// Plays n hands with global episode ids g0 .. g0 + n - 1 (Sec. 4.2's simulations
+// indexed as in orc_kuhn_eval), for checking records of hands whose id is
+// too far into a long evaluation for the whole evaluation to be replayed.
+// trace [n][8] as in orc_kuhn_eval.
+void orc_kuhn_hands(const float* pol0, const float* pol1, uint64_t g0, int64_t n, uint64_t seed,
+                    int32_t* trace) {
+    for (int64_t e = 0; e < n; ++e) {
+        KuhnTrace tr;
+        kuhn_episode(pol0, pol1, g0 + (uint64_t)e, seed, &tr);
+        int32_t* t = trace + e * 8;
+        t[0] = tr.card0; t[1] = tr.card1; t[2] = tr.n_dec;
+        for (int k = 0; k < 3; ++k) t[3 + k] = k < tr.n_dec ? tr.action[k] : -1;
+        t[6] = tr.payoff0; t[7] = 0;
+    }
+}
+
 // ---- Leduc ----
 void orc_leduc_deal(uint64_t g, uint64_t seed, int32_t* cards3) {
     int a, b, c;

@@ -122,3 +122,38 @@ def test_invalid_arguments(kuhn_ctx):
     with pytest.raises(MalibError, match="EINVAL"):
         ctx.sync()
     ctx.sync()   # cleared
+
+
+def test_hand_ids_beyond_32_bits_and_64_bit_sums(kuhn_ctx, orc):
+    """3 pairs x 2.2e9 hands: the third pair's hand ids start at 4.4e9 > 2^32 and
+    every pair's sum of r^2 passes 2^31. The first 256 records of every pair
+    equal the oracle's hands at the same global ids; the integer sums are
+    consistent with payoffs in {+-1, +-2}; the means lie within 4 SE of the
+    exact values."""
+    need_gpu()
+    ctx, w = kuhn_ctx
+    n, n_dump, seed = 2_200_000_000, 256, 5
+    pairs = np.ascontiguousarray(w.pair_ids[:3])
+    dump = alloc_eval_dump(MALIB_ENV_KUHN, 3, n_dump)
+    got = ctx.eval_payoff_ex(pairs, n, seed, MALIB_DUMP_LOGITS, dump=dump, n_dump=n_dump)
+    act = dump["action"].cpu().numpy().astype(np.int32)
+    act[act == 255] = -1
+    rew = dump["reward"].cpu().numpy()
+    T = tables(w)
+    for k, (i, j) in enumerate(pairs):
+        ref = orc.kuhn_hands(T[i], T[j], k * n, n_dump, seed)
+        np.testing.assert_array_equal(act[k], ref[:, 3:6])
+        np.testing.assert_array_equal(rew[k].sum(axis=1), ref[:, 6])
+    s1, s2 = got[:, 2], got[:, 3]
+    assert np.all(s2 >= n) and np.all(s2 <= 4 * n) and np.all(np.abs(s1) <= s2)
+    ex = np.array([orc.kuhn_exact(T[i], T[j]) for i, j in pairs])
+    n_out, zmax = four_se_rule(got[:, 0], got[:, 1], ex)
+    assert n_out == 0 and zmax < 4.5, (n_out, zmax)
+
+
+def test_evaluation_size_limit(kuhn_ctx):
+    need_gpu()
+    ctx, w = kuhn_ctx
+    with pytest.raises(MalibError, match="EINVAL"):            # 2 x (2^39 + 1) > 2^40 hands
+        ctx.eval_payoff(np.ascontiguousarray(w.pair_ids[:2]), (1 << 39) + 1, 0)
+    ctx.sync()

@@ -131,3 +131,19 @@ def test_kuhn_entry_statistics(orc):
     assert res[0, 3] == (r ** 2).sum()
     assert abs(res[0, 0] - r.mean()) < 1e-15
     assert abs(res[0, 1] - r.std(ddof=1) / np.sqrt(n)) < 1e-12
+
+
+def test_kuhn_hands_at_any_id_match_the_evaluation(orc):
+    """The per-id helper replays the evaluation's hands: pair k's hand e is the
+    hand with global id k * n_episodes + e, and its payoffs sum to the entry's."""
+    w = workloads.kuhn(n_episodes=500)
+    tables = np.stack([p.params for p in w.policies])
+    res, tr = orc.kuhn_eval(tables, w.pair_ids[:3], 500, 11, n_trace=500)
+    for k in range(3):
+        i, j = w.pair_ids[k]
+        got = orc.kuhn_hands(tables[i], tables[j], k * 500, 500, 11)
+        np.testing.assert_array_equal(got, tr[k])
+        assert got[:, 6].sum() == res[k, 2]
+    far = orc.kuhn_hands(tables[0], tables[1], (1 << 33) + 5, 64, 11)
+    assert set(np.unique(far[:, 6])) <= {-2, -1, 1, 2}
+    assert not np.array_equal(far, orc.kuhn_hands(tables[0], tables[1], 5, 64, 11))
