@@ -6,8 +6,10 @@ simple spread) in ``malib_oracle.cpp``, wrapped here with ctypes + numpy.
 Only the tests, the smoke check and the benchmark's CPU-baseline leg may use
 it; the GPU path never imports it and shares no code with it.
 
-Parity pins live in ``tests/test_oracle_*.py``. The spread episode return has
-no closed form: beyond single-step and invariant checks it is "parity unpinned".
+Parity pins live in ``tests/test_oracle_*.py``. The spread episode return under
+sampled policies has no closed form: beyond single steps, invariants and two
+forced-action episodes (at rest; under a constant force) it is "parity
+unpinned".
 """
 from __future__ import annotations
 

@@ -36,8 +36,10 @@
 // identity against fp64, the spread dynamics and reset, symmetries) and the
 // simple speaker listener (hand-worked geometry, the one-step message delay,
 // the immobile speaker, the spread dynamics and reset, the target draw) are
-// pinned by the CPU tests; episode returns of the particle scenarios beyond those
-// invariants are "parity unpinned" (no closed form exists).
+// pinned by the CPU tests, and whole spread episodes under forced actions (at
+// rest; a constant force from rest) match closed forms; episode returns of the
+// particle scenarios under sampled policies beyond those are "parity unpinned"
+// (no closed form exists).
 
 #include <algorithm>
 #include <cmath>

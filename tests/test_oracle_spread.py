@@ -1,7 +1,8 @@
 """Pins for the oracle's particle spread: closed-form single steps, velocity
 damping, exact distances on 3-4-5 triangles, collision counting and the
-observation layout. The episode return has no closed form ("parity unpinned"
-beyond these invariants)."""
+observation layout, and two forced-action episodes with closed forms (at rest;
+under a constant force). The return under sampled policies has no closed form
+("parity unpinned" beyond these)."""
 import numpy as np
 
 import workloads
@@ -173,3 +174,42 @@ def test_rollout_fixed_point_over_an_episode(orc):
         for t in range(T):
             np.testing.assert_array_equal(out["obs"][0, t, env], orc.spread_obs(st, 3, 3, 18))
             np.testing.assert_array_equal(out["reward"][0, t, env], r)
+
+
+def test_rollout_constant_force_closed_form(orc):
+    """Logits that force action 1 (+x) in every step. From rest, after k moves
+    v_k = 0.4 (1 - 0.75^k) and p_k = p_0 + 0.04 (k - 3 (1 - 0.75^k)) along x,
+    with y fixed (Sec. 3.1's rollout over the dynamics of App. B.1). All agents
+    drift together, so their collision counts stay those of the reset, and the
+    cover term follows from the closed-form positions. The 25-step rollout must
+    agree with the fp64 closed form to within fp32 rounding."""
+    V, T = 32, 25
+    w = workloads.spread(n_agents=3, n_envs=V, pop=2, envs_per_pair=16, seed=6)
+    params = [p.params for p in w.policies]
+    ext = np.zeros((1, T, V, 3, 5), np.float32)
+    ext[..., 1] = 100.0
+    out = orc.spread_rollout(params, w.policies[0].dims, 3, 3, T, V, w.pair_ids, 1, w.seed,
+                             ext_logits=ext)
+    assert np.all(out["action"] == 1)
+    checked = 0
+    for env in range(V):
+        st = orc.spread_reset(3, 3, env, w.seed).astype(np.float64)
+        p0 = st[:12].reshape(3, 4)[:, :2]
+        lm = st[12:18].reshape(3, 2)
+        d = np.hypot(*(p0[:, None, :] - p0[None, :, :]).transpose(2, 0, 1))
+        if np.any(np.abs(d - 0.3) < 1e-3):
+            continue                                      # too close to the collision radius
+        coll = (d < 0.3).sum(axis=1) - 1
+        for t in range(T):
+            v = 0.4 * (1 - 0.75 ** t)
+            dx = 0.04 * (t - 3 * (1 - 0.75 ** t))
+            obs = out["obs"][0, t, env]
+            np.testing.assert_allclose(obs[:, 0], v, atol=1e-6)
+            np.testing.assert_array_equal(obs[:, 1], 0.0)
+            np.testing.assert_allclose(obs[:, 2:4], p0 + [dx, 0.0], atol=5e-6)
+            k = t + 1                                     # the reward follows the step's move
+            p = p0 + [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0]
+            cover = sum(min(np.hypot(*(p[a] - lm[l])) for a in range(3)) for l in range(3))
+            np.testing.assert_allclose(out["reward"][0, t, env], -(cover + coll), atol=5e-5)
+        checked += 1
+    assert checked >= 24
