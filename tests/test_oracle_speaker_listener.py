@@ -12,6 +12,7 @@ import numpy as np
 import pytest
 
 import oracle
+import workloads
 
 pytestmark = pytest.mark.filterwarnings("ignore")
 
@@ -116,3 +117,34 @@ def test_rollout_replays_the_step_function():
                 np.testing.assert_array_equal(out["obs"][ep, t, e], oracle.sl_obs(st))
                 st, r = oracle.sl_step(st, out["action"][ep, t, e].astype(np.int32))
                 np.testing.assert_array_equal(out["reward"][ep, t, e], r)
+
+
+def test_forced_episode_closed_form(orc):
+    """A whole 25-step episode with forced actions: the speaker always sends
+    message 2 and the listener always pushes +x. The speaker sees the target's
+    one-hot at every step; from rest the listener follows v_k = 0.4 (1 - 0.75^k),
+    p_k = p_0 + 0.04 (k - 3 (1 - 0.75^k)) along x; both rewards equal minus
+    the listener's fp64 distance to the target; the listener sees no message
+    at the first step and message 2 from then on."""
+    V, T = 16, 25
+    w = workloads.speaker_listener(n_envs=V, pop=2, envs_per_pair=8, seed=4)
+    params = [p.params for p in w.policies]
+    ext = np.zeros((1, T, V, 2, 5), np.float32)
+    ext[:, :, :, 0, 2] = 100.0
+    ext[:, :, :, 1, 1] = 100.0
+    out = orc.sl_rollout(params, w.policies[0].dims, T, V, w.pair_ids, 1, w.seed, ext_logits=ext)
+    np.testing.assert_array_equal(out["action"][0, :, :, 0], 2)
+    np.testing.assert_array_equal(out["action"][0, :, :, 1], 1)
+    for env in range(V):
+        st = orc.sl_reset(env, w.seed).astype(np.float64)
+        p1 = st[4:6]
+        target = st[8 + 2 * int(st[14]): 10 + 2 * int(st[14])]
+        for t in range(T):
+            obs = out["obs"][0, t, env]
+            np.testing.assert_array_equal(obs[0], np.eye(11)[int(st[14])])
+            np.testing.assert_allclose(obs[1, 0], 0.4 * (1 - 0.75 ** t), atol=1e-6)
+            assert obs[1, 1] == 0.0
+            np.testing.assert_array_equal(obs[1, 8:11], [0, 0, 0] if t == 0 else [0, 0, 1])
+            k = t + 1
+            p = p1 + [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0]
+            np.testing.assert_allclose(out["reward"][0, t, env], -np.hypot(*(p - target)), atol=2e-5)
