@@ -13,6 +13,7 @@ import numpy as np
 import pytest
 
 import oracle
+import workloads
 
 pytestmark = pytest.mark.filterwarnings("ignore")
 
@@ -150,3 +151,30 @@ def test_rollout_replays_the_step_function():
                 np.testing.assert_array_equal(out["obs"][ep, t, e], oracle.adversary_obs(st))
                 st, r = oracle.adversary_step(st, out["action"][ep, t, e].astype(np.int32))
                 np.testing.assert_array_equal(out["reward"][ep, t, e], r)
+
+
+def test_forced_episode_closed_form(orc):
+    """A whole 25-step episode in which every agent pushes +x. From rest all
+    three follow v_k = 0.4 (1 - 0.75^k), p_k = p_0 + 0.04 (k - 3 (1 - 0.75^k))
+    along x; the rewards, recomputed in fp64 from those positions, are
+    -d(p_0) for the adversary and -min(d(p_1), d(p_2)) + d(p_0) for both good
+    agents, d the distance to the target landmark."""
+    V, T = 16, 25
+    w = workloads.adversary(n_envs=V, pop=2, envs_per_pair=8, seed=3)
+    params = [p.params for p in w.policies]
+    ext = np.zeros((1, T, V, 3, 5), np.float32)
+    ext[..., 1] = 100.0
+    out = orc.adversary_rollout(params, w.policies[0].dims, T, V, w.pair_ids, 1, w.seed,
+                                ext_logits=ext)
+    assert np.all(out["action"] == 1)
+    for env in range(V):
+        st = orc.adversary_reset(env, w.seed).astype(np.float64)
+        p0 = st[:12].reshape(3, 4)[:, :2]
+        target = st[12 + 2 * int(st[16]): 14 + 2 * int(st[16])]
+        for t in range(T):
+            np.testing.assert_allclose(out["obs"][0, t, env, :, 0], 0.4 * (1 - 0.75 ** t), atol=1e-6)
+            k = t + 1
+            p = p0 + [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0]
+            d = np.hypot(*(p - target).T)
+            want = [-d[0], -min(d[1], d[2]) + d[0], -min(d[1], d[2]) + d[0]]
+            np.testing.assert_allclose(out["reward"][0, t, env], want, atol=5e-5)
