@@ -104,3 +104,42 @@ def test_invalid_rollout_arguments():
         ctx.rollout(big, w.pair_ids, 1, 0, alloc_traj(big, 1))
     ctx.rollout(spec, w.pair_ids, 0, 0, traj)              # zero episodes: no-op
     ctx.close()
+
+
+def test_forced_episode_closed_form(orc):
+    """Policies with zero weights and b3 = (0, 100, 0, 0, 0) push every agent +x
+    in every step. From rest, after k moves v_k = 0.4 (1 - 0.75^k) and
+    p_k = p_0 + 0.04 (k - 3 (1 - 0.75^k)) along x; the GPU's observations and
+    rewards must follow that closed form (rewards recomputed in fp64; the
+    agents keep their reset distances, hence their collision counts)."""
+    need_gpu()
+    V, T = 64, 25
+    w = workloads.spread(n_agents=3, n_envs=V, pop=2, envs_per_pair=16, seed=6)
+    for p in w.policies:
+        p.params[:] = 0.0
+        p.params[-4] = 100.0                              # b3[1]: action 1, +x
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 1, w.seed)
+    ctx.close()
+    assert np.all(g["action"] == 1)
+    checked = 0
+    for env in range(V):
+        st = orc.spread_reset(3, 3, env, w.seed).astype(np.float64)
+        p0 = st[:12].reshape(3, 4)[:, :2]
+        lm = st[12:18].reshape(3, 2)
+        d = np.hypot(*(p0[:, None, :] - p0[None, :, :]).transpose(2, 0, 1))
+        if np.any(np.abs(d - 0.3) < 1e-3):
+            continue                                      # too close to the collision radius
+        coll = (d < 0.3).sum(axis=1) - 1
+        for t in range(T):
+            obs = g["obs"][0, t, env]
+            np.testing.assert_allclose(obs[:, 0], 0.4 * (1 - 0.75 ** t), atol=1e-6)
+            np.testing.assert_allclose(obs[:, 2:4], p0 + [0.04 * (t - 3 * (1 - 0.75 ** t)), 0.0],
+                                       atol=5e-6)
+            k = t + 1
+            p = p0 + [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0]
+            cover = sum(min(np.hypot(*(p[a] - lm[l])) for a in range(3)) for l in range(3))
+            np.testing.assert_allclose(g["reward"][0, t, env], -(cover + coll), atol=5e-5)
+        checked += 1
+    assert checked >= 40
