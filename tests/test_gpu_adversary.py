@@ -81,3 +81,32 @@ def test_invalid_adversary_arguments():
         spec = spec_of(w, local_ratio=0.5)
         ctx.rollout(spec, w.pair_ids, 1, 0, alloc_traj(spec, 1))
     ctx.close()
+
+
+def test_forced_episode_closed_form(orc):
+    """Policies with zero weights and b3 = (0, 100, 0, 0, 0) push every agent +x
+    in every step. From rest all three follow v_k = 0.4 (1 - 0.75^k),
+    p_k = p_0 + 0.04 (k - 3 (1 - 0.75^k)) along x; the GPU's rewards must equal
+    -d(p_0) for the adversary and -min(d(p_1), d(p_2)) + d(p_0) for both good
+    agents, recomputed in fp64 from those positions."""
+    need_gpu()
+    V, T = 64, 25
+    w = workloads.adversary(n_envs=V, pop=2, envs_per_pair=16, seed=3)
+    for p in w.policies:
+        p.params[:] = 0.0
+        p.params[-4] = 100.0                              # b3[1]: action 1, +x
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 1, w.seed)
+    ctx.close()
+    assert np.all(g["action"] == 1)
+    for env in range(V):
+        st = orc.adversary_reset(env, w.seed).astype(np.float64)
+        p0 = st[:12].reshape(3, 4)[:, :2]
+        target = st[12 + 2 * int(st[16]): 14 + 2 * int(st[16])]
+        for t in range(T):
+            np.testing.assert_allclose(g["obs"][0, t, env, :, 0], 0.4 * (1 - 0.75 ** t), atol=1e-6)
+            k = t + 1
+            d = np.hypot(*(p0 + [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0] - target).T)
+            good = -min(d[1], d[2]) + d[0]
+            np.testing.assert_allclose(g["reward"][0, t, env], [-d[0], good, good], atol=5e-5)

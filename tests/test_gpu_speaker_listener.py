@@ -92,3 +92,34 @@ def test_invalid_speaker_listener_arguments():
             ctx.rollout(spec, w.pair_ids, 1, 0, alloc_traj(spec, 1))
     ctx.sync()
     ctx.close()
+
+
+def test_forced_episode_closed_form(orc):
+    """Every policy with zero weights and b3 = (0, 0, 100, 0, 0): the speaker
+    sends message 2 and the listener pushes -x in every step. From rest the
+    listener follows v_k = -0.4 (1 - 0.75^k), p_k = p_0 - 0.04 (k - 3 (1 - 0.75^k))
+    along x; the GPU's observations and rewards must follow that closed form
+    (rewards: minus the listener's fp64 distance to the target)."""
+    need_gpu()
+    V, T = 64, 25
+    w = workloads.speaker_listener(n_envs=V, pop=2, envs_per_pair=16, seed=4)
+    for p in w.policies:
+        p.params[:] = 0.0
+        p.params[-3] = 100.0                              # b3[2]: message 2 / move -x
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 1, w.seed)
+    ctx.close()
+    assert np.all(g["action"] == 2)
+    for env in range(V):
+        st = orc.sl_reset(env, w.seed).astype(np.float64)
+        tgt = int(st[14])
+        for t in range(T):
+            obs = g["obs"][0, t, env]
+            np.testing.assert_array_equal(obs[0, :11], np.eye(11)[tgt])
+            np.testing.assert_allclose(obs[1, 0], -0.4 * (1 - 0.75 ** t), atol=1e-6)
+            np.testing.assert_array_equal(obs[1, 8:11], [0, 0, 0] if t == 0 else [0, 0, 1])
+            k = t + 1
+            p = st[4:6] - [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0]
+            d = np.hypot(*(p - st[8 + 2 * tgt: 10 + 2 * tgt]))
+            np.testing.assert_allclose(g["reward"][0, t, env], [-d, -d], atol=2e-5)
