@@ -83,3 +83,44 @@ def test_full_workload_sampled_envs(orc):
         check(orc, w, g, 1, w.seed, lo, hi)
     assert np.all(g["reward"] <= 0)
     ctx.close()
+
+
+def test_forced_episode_closed_form(orc):
+    """bf16 policies with zero weights and b3 = (0, 100, 0, 0, 0) push all 8
+    agents +x in every step (the tensor-core forward then yields exactly b3).
+    From rest, after k moves v_k = 0.4 (1 - 0.75^k) and
+    p_k = p_0 + 0.04 (k - 3 (1 - 0.75^k)) along x; the GPU's observations and
+    rewards must follow that closed form (rewards recomputed in fp64; the
+    agents keep their reset distances, hence their collision counts)."""
+    need_gpu()
+    V, T, N = 128, 25, 8
+    w = workloads.spread(n_agents=N, n_envs=V, pop=3, hidden=256, dtype=workloads.BF16,
+                         envs_per_pair=128, seed=9)
+    for p in w.policies:
+        p.params[:] = 0.0
+        p.params[-4] = 100.0                              # b3[1]: action 1, +x
+    ctx = context()
+    load_population(ctx, w)
+    g = rollout(ctx, w, 1, w.seed)
+    ctx.close()
+    assert np.all(g["action"] == 1)
+    checked = 0
+    for env in range(V):
+        st = orc.spread_reset(N, N, env, w.seed).astype(np.float64)
+        p0 = st[:4 * N].reshape(N, 4)[:, :2]
+        lm = st[4 * N:6 * N].reshape(N, 2)
+        d = np.hypot(*(p0[:, None, :] - p0[None, :, :]).transpose(2, 0, 1))
+        if np.any(np.abs(d - 0.3) < 1e-3):
+            continue                                      # too close to the collision radius
+        coll = (d < 0.3).sum(axis=1) - 1
+        for t in range(T):
+            obs = g["obs"][0, t, env]
+            np.testing.assert_allclose(obs[:, 0], 0.4 * (1 - 0.75 ** t), atol=1e-6)
+            np.testing.assert_allclose(obs[:, 2:4], p0 + [0.04 * (t - 3 * (1 - 0.75 ** t)), 0.0],
+                                       atol=5e-6)
+            k = t + 1
+            p = p0 + [0.04 * (k - 3 * (1 - 0.75 ** k)), 0.0]
+            cover = sum(min(np.hypot(*(p[a] - lm[l])) for a in range(N)) for l in range(N))
+            np.testing.assert_allclose(g["reward"][0, t, env], -(cover + coll), atol=1e-4)
+        checked += 1
+    assert checked >= 64
