@@ -1,12 +1,14 @@
 #!/usr/bin/env python
 """Benchmark of the rollout / payoff-evaluation path on GB300.
 
-Default workload (one "step"): the empirical payoff table of Leduc hold'em for
-an 8 x 8 population of fp32 MLP policies 17-128-128-3, 65,536 Monte-Carlo
-hands per pair (64 pairs, ~14 M decisions): deal, observation, policy forward
-of the acting seat, masked softmax + Philox draw, transition, payoff reduction
-(malib_eval_payoff). Inputs (population, pair table) are resident in HBM; L2 is
-flushed (256 MiB write) before every timed step; each step uses a new seed.
+Default workload (one "step"): the PSRO payoff-table sweep on Leduc hold'em,
+the largest of the five workloads: a 64 x 64 population of bf16 MLP policies
+17-256-256-3 (fp32 accumulation on the tensor cores), 16,384 Monte-Carlo hands
+per pair (4,096 pairs, ~67 M hands, ~300 M decisions): deal, observation,
+policy forward of the acting seat, masked softmax + Philox draw, transition,
+payoff reduction (malib_eval_payoff). Inputs (population, pair table) are
+resident in HBM; L2 is flushed (256 MiB write) before every timed step; each
+step uses a new seed. --workload selects another of the workloads.
 
 Prints ONE JSON line (rank 0). --impl reference times the CPU oracle on a
 bounded sample of the same workload instead.
@@ -26,10 +28,9 @@ sys.path.insert(0, ROOT)
 
 METRIC = "env-steps/sec incl. policy inference and payoff entries/sec on 1 GB300; % of roofline"
 UNIT = "env-steps/s"
-SM_COUNT_GB300 = 152
 FP32_LANES_PER_SM = 128
 # DRAM bytes (read + write) per launch of each workload's dominant kernel, from
-# ncu (profiles/*.md give the commands). The fp32 rollout kernels were captured
+# ncu (dram__bytes_read.sum + dram__bytes_write.sum). The fp32 rollout kernels were captured
 # on the benchmark's own workload with the two dram counters alone (one pass);
 # about 62 MB of trajectory lines are still dirty in L2 when such a kernel ends,
 # so their writes fall that much short of the bytes stored. The spread N=8 bf16
@@ -61,7 +62,7 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "speaker_listener",
                                            "leduc_bf16", "spread8", "meta"],
-                    default="leduc")
+                    default="leduc_bf16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--hands", type=int, default=None,
@@ -321,40 +322,89 @@ def cpu_count():
         return os.cpu_count() or 1
 
 
+def oracle_step_fn(w, name, threads, per_step):
+    """One bounded step of the oracle on workload `w`, sized once so that it
+    takes about per_step seconds: returns (step(seed) -> units done, sample
+    text). Units are the workload's metric unit (decisions or env-steps)."""
+    import numpy as np
+    import oracle
+    params = [p.params for p in w.policies]
+    dims = w.policies[0].dims
+    if name in ("leduc", "leduc_bf16"):
+        bf16 = w.policies[0].dtype == 1
+        _, sample = oracle_leduc_sample(w, per_step, threads)
+        n = int(sample.split()[1])
+
+        def step(seed):
+            dec = np.zeros(w.n_pairs, np.int64)
+            oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, seed, n_sim=n,
+                              decisions=dec, n_threads=threads, bf16=bf16)
+            return int(dec.sum())
+        return step, f"per step: first {n} hands of each of the {w.n_pairs} pairs"
+    if name == "kuhn":
+        rate, sample = oracle_kuhn_sample(w, per_step, threads)
+        n = int(sample.split()[1])
+        tables = np.stack([p.params for p in w.policies])
+        deals = [(a, b) for a in range(3) for b in range(3) if a != b]
+        dec = 0.0
+        for i, j in w.pair_ids:
+            p0, p1 = tables[i].astype(np.float64), tables[j].astype(np.float64)
+            dec += n * (2.0 + sum((1.0 - p0[2 * a]) * p1[2 * b] for a, b in deals) / 6.0)
+
+        def step(seed):
+            oracle.kuhn_eval(tables, w.pair_ids, n, seed, n_threads=threads)
+            return dec
+        return step, (f"per step: first {n} hands of each of the {w.n_pairs} pairs (decisions "
+                      "counted by their exact expectation per pair)")
+    # rollouts: the first n environments, one episode
+    _, sample = oracle_rollout_sample(w, name, per_step, threads)
+    n = int(sample.split()[1])
+    bf16 = w.policies[0].dtype == 1
+
+    def step(seed):
+        if name == "adversary3":
+            oracle.adversary_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, 1, seed,
+                                     env_lo=0, env_hi=n, n_threads=threads)
+        elif name == "speaker_listener":
+            oracle.sl_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, 1, seed,
+                              env_lo=0, env_hi=n, n_threads=threads)
+        else:
+            oracle.spread_rollout(params, dims, w.n_agents, w.n_landmarks, w.episode_len, w.n_envs,
+                                  w.pair_ids, 1, seed, bf16=bf16, env_lo=0, env_hi=n,
+                                  n_threads=threads)
+        return n * w.episode_len
+    return step, (f"per step: first {n} of the {w.n_envs} environments, one episode of "
+                  f"{w.episode_len} steps")
+
+
 def run_reference(args):
+    """The reference arm: the CPU oracle, as it stands, on the host cores, on a
+    bounded sample of the same workload as the GPU arm (rank 0 only)."""
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
     import oracle
     oracle.build()
-    w = workload("leduc", 0)
+    name = "leduc_bf16" if args.workload == "meta" else args.workload
+    w = workload(name, 0, args.hands)
     threads = cpu_count()
     per_step = max(0.2, min(5.0, 150.0 / max(1, args.steps + args.warmup)))
-    import numpy as np
-    params = [p.params for p in w.policies]
-    dims = w.policies[0].dims
-    # size one step
-    rate, sample = oracle_leduc_sample(w, per_step, threads)
-    n = int(sample.split()[1])
-    for _ in range(args.warmup):
-        oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, w.seed, n_sim=n,
-                          n_threads=threads)
-    tot_dec, tot_t = 0, 0.0
+    step, sample = oracle_step_fn(w, name, threads, per_step)
+    for k in range(args.warmup):
+        step(w.seed + 10_000 + k)
+    tot_units, tot_t = 0.0, 0.0
     for k in range(args.steps):
-        dec = np.zeros(w.n_pairs, np.int64)
         t0 = time.perf_counter()
-        oracle.leduc_eval(params, dims, w.pair_ids, w.n_episodes, w.seed + k, n_sim=n,
-                          decisions=dec, n_threads=threads)
+        tot_units += step(w.seed + k)
         tot_t += time.perf_counter() - t0
-        tot_dec += int(dec.sum())
-    value = tot_dec / tot_t
+    value = tot_units / tot_t
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * tot_t / max(1, args.steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": config_of(w, "leduc"),
+            "config": config_of(w, name),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                             "sample": f"per step: first {n} hands of each of the 64 pairs"},
+                             "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -444,7 +494,8 @@ def run_ours(args):
 
     peaks = load_peaks()
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
-    peak_tflops = SM_COUNT_GB300 * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak_tflops = n_sm * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
     achieved = (decisions * flop_per_unit / args.steps) / (kern_ms / kern_n / 1e3) / 1e12 \
         if kern_n else 0.0
     kname = {"leduc": "leduc_eval_f32_t8_kernel", "kuhn": "kuhn_eval_kernel",
@@ -453,11 +504,17 @@ def run_ours(args):
              "speaker_listener": "spread_rollout_f32_kernel<2,11,64,2>",
              "leduc_bf16": "leduc_eval_tc_kernel",
              "spread8": "spread_rollout_tc_kernel"}[args.workload]
-    basis = (f"fp32 FMA: {SM_COUNT_GB300} SMs x {FP32_LANES_PER_SM} lanes x 2 flop"
+    basis = (f"fp32 FMA: {n_sm} SMs (queried) x {FP32_LANES_PER_SM} lanes x 2 flop"
              f" x {sm_max:.0f} MHz (max SM clock of MEASURED_PEAKS.json)")
     if tensor:
-        peak_tflops = float(peaks.get("bf16_tflops_sustained", 1700.0))
-        basis = "measured cuBLAS bf16 dense, sustained (MEASURED_PEAKS.json bf16_tflops_sustained)"
+        # the kernel is timed alone, launch by launch, with CUDA events: the
+        # burst figure of the measured cuBLAS bf16 GEMM is its peak
+        if "bf16_tflops" in peaks:
+            peak_tflops = float(peaks["bf16_tflops"])
+            basis = "measured cuBLAS bf16 dense GEMM, burst (MEASURED_PEAKS.json bf16_tflops), of measured"
+        else:
+            peak_tflops = 1900.0
+            basis = "fallback bf16 dense burst 1.9 PFLOP/s (no MEASURED_PEAKS.json), of fallback"
     roofline = {"bound": "tensor" if tensor else "alu", "achieved": achieved,
                 "peak": peak_tflops, "unit": "TFLOP/s",
                 "frac": achieved / peak_tflops if peak_tflops else None,
@@ -472,13 +529,13 @@ def run_ours(args):
         # per decision; the ceiling is the measured rate of a Philox-only kernel
         calls = (w.n_pairs * w.n_episodes * args.steps + decisions) / args.steps
         rate = calls / (kern_ms / max(1, kern_n) / 1e3) if kern_n else 0.0
-        ceil = philox_ceiling(ctx, stream)
+        ceil = philox_ceiling(ctx, stream, n_sm)
         roofline = {"bound": "alu", "achieved": rate / 1e9, "peak": ceil / 1e9,
                     "unit": "Gcall/s (Philox4x32-10)", "frac": rate / ceil,
                     "traffic": None, "kernel": kname,
                     "kernel_ms_per_launch": kern_ms / max(1, kern_n),
-                    "peak_basis": "measured: malib_philox_digest, 311,296 threads x 4,096 "
-                                  "calls per launch, best of 5 (CUDA events)",
+                    "peak_basis": f"measured: malib_philox_digest, {n_sm * 8 * 256} threads x "
+                                  "4,096 calls per launch, best of 5 (CUDA events)",
                     "algorithmic": "1 Philox4x32-10 call per deal + 1 per decision"}
 
     e2e = run_e2e(args, ctx, w, spec, dev, rollout) if rank == 0 else None
@@ -510,12 +567,12 @@ def run_ours(args):
     return 0
 
 
-def philox_ceiling(ctx, stream):
+def philox_ceiling(ctx, stream, n_sm):
     """Philox4x32-10 calls per second of the library's arithmetic-only digest
     kernel: best of 5 launches after 3 warm-ups, timed with CUDA events on the
     context's stream."""
     import torch
-    n, calls = SM_COUNT_GB300 * 8 * 256, 4096
+    n, calls = n_sm * 8 * 256, 4096
     out = torch.empty(n, dtype=torch.int32, device=stream.device)
     best = None
     for k in range(8):

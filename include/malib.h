@@ -205,12 +205,15 @@ int malib_pop_reset(malib_ctx* ctx);
 /*
  * malib_rollout - batched multi-agent rollout (Sec. 3.1, X(theta) ~ P(s, a, s'
  * | a ~ Comb_t); the Actor with k environments of the architecture figure).
- * SPREAD only. pair_ids (host or device) int32 [n_pairs][n_agents] holds one
+ * SPREAD, ADVERSARY and SPEAKER_LISTENER (App. B.1 particle scenarios).
+ * pair_ids (host or device) int32 [n_pairs][n_agents] holds one
  * policy id per agent for each combination; the n_envs environments are split
  * evenly and contiguously over the combinations (n_envs % n_pairs == 0).
  * Environment v of episode e uses global episode id g = e * n_envs + v; all
  * randomness is Philox4x32-10 keyed by seed with counter (g, step, agent).
- * traj_out (device buffers, layout above) receives n_episodes episodes per env.
+ * traj_out (device buffers of the context's device, layout above) receives
+ * n_episodes episodes per env. A device pair table or output on another GPU
+ * gives EINVAL.
  * Errors: EINVAL, ESTATE, EUNSUPPORTED (a policy shape without a kernel).
  */
 int malib_rollout(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pair_ids,
@@ -225,7 +228,8 @@ int malib_rollout(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pai
  * receives, for the seat-0 payoff (seat 1 gets its negation):
  *   mean, standard error of the mean (sample variance / n, 0 if n < 2),
  *   sum, sum of squares (exact integers).
- * n_pairs == 0 is a no-op. Errors: EINVAL, ESTATE, EUNSUPPORTED.
+ * n_pairs == 0 is a no-op. Device buffers must belong to the context's device
+ * (EINVAL otherwise). Errors: EINVAL, ESTATE, EUNSUPPORTED.
  */
 int malib_eval_payoff(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pairs,
                       int64_t n_episodes, uint64_t seed, double* payoff_out);
@@ -253,11 +257,14 @@ int malib_eval_payoff_ex(malib_ctx* ctx, const int32_t* pair_ids, int32_t n_pair
  * counter and per-pair hand counters) is a fixed file-scope device array of
  * 192 KiB + 8 B that every GPU loading the library holds until the process
  * exits.
- *  - pair_ids and payoff_out must be DEVICE buffers (layouts as in
- *    malib_eval_payoff; no host staging). Host buffers give EINVAL.
+ *  - pair_ids and payoff_out must be DEVICE buffers of the context's device
+ *    (layouts as in malib_eval_payoff; no host staging). Host buffers, or
+ *    buffers on another GPU, give EINVAL.
  *  - n_pairs <= 8192 (the array's capacity); more gives EINVAL.
  *  - The population must already be loaded (malib_pop_load), MC mode only,
- *    no dump; same results as malib_eval_payoff for the same arguments.
+ *    no dump. Kuhn populations and fp32 Leduc populations are served, with the
+ *    same results as malib_eval_payoff for the same arguments; bf16 Leduc
+ *    populations (tensor-core images) give MALIB_EUNSUPPORTED.
  *    malib_eval_stats does not report its decision count.
  *  - The first call on a device looks the array's device address up
  *    (cudaGetSymbolAddress); make that first call before any stream capture.
@@ -304,6 +311,16 @@ int malib_meta_fictitious_play(malib_ctx* ctx, const double* payoff, int32_t n_g
 int malib_meta_lp_nash(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
                        int32_t n, int32_t stride, double* x_out, double* y_out,
                        double* value_out);
+
+/* malib_meta_lp_nash with the pivot limit chosen by the caller: max_pivots > 0
+ * caps the pivots of every game at that number; 0 keeps the default limit of
+ * 50 (m + n) + 1000. A game that needs more pivots than the limit leaves its
+ * outputs at the last tableau (not an equilibrium) and raises
+ * MALIB_ENOTCONVERGED at the next malib_sync, which clears it; the context
+ * stays usable. EINVAL for max_pivots < 0. */
+int malib_meta_lp_nash_ex(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
+                          int32_t n, int32_t stride, int32_t max_pivots, double* x_out,
+                          double* y_out, double* value_out);
 
 /* Payoffs under mixtures x [G][m], y [G][n] (device fp64): row_payoff_out
  * [G][m] = A y (what each row policy, e.g. a new best response, earns against

@@ -22,8 +22,8 @@
 //    landmarks of which one is the target; good agents are rewarded for being
 //    close to the target and for the adversary being far from it, the adversary
 //    (which is not told the target) for being close to it.
-// Kuhn and Leduc rules are not given in the paper; the textbook rules are used
-// (readings listed in the design doc, summarised at each function below).
+// Kuhn and Leduc rules are not given in the paper; the textbook rules are used,
+// each reading stated at the function that takes it below.
 //
 // Numerics: fp32 where the method is defined in fp32 (environment dynamics,
 // sampling); policy forward accumulated in fp64 and rounded to fp32 logits;
@@ -455,11 +455,30 @@ int leduc_episode(const Mlp& m0, const Mlp& m1, uint64_t g, uint64_t seed, const
 // Exact expected seat-0 payoff of a pair: every ordered deal of the 6 cards
 // (6*5*4 = 120, equally likely) times the betting tree, with the policy's
 // action probabilities = fp64 softmax of its fp32 logits over legal actions.
-double leduc_tree(const Mlp& m0, const Mlp& m1, const Leduc& s) {
+// A seat's logits depend only on its observation, so each walk keeps the
+// logits of the observations it has met (at most 144 per seat) and looks them
+// up instead of running the MLP again: a memo of a pure function, the values
+// are the same bits.
+struct LogitMemo {
+    std::vector<float> obs[2], lg[2];          // per seat: [n][17], [n][3]
+    void get(const Mlp& m, int seat, const float* o, float* out) {
+        const std::vector<float>& ob = obs[seat];
+        for (size_t i = 0; i < ob.size(); i += 17)
+            if (std::memcmp(ob.data() + i, o, 17 * sizeof(float)) == 0) {
+                std::memcpy(out, lg[seat].data() + i / 17 * 3, 3 * sizeof(float));
+                return;
+            }
+        mlp_logits(m, o, out);
+        obs[seat].insert(obs[seat].end(), o, o + 17);
+        lg[seat].insert(lg[seat].end(), out, out + 3);
+    }
+};
+
+double leduc_tree(const Mlp& m0, const Mlp& m1, const Leduc& s, LogitMemo& memo) {
     if (s.done) return (double)s.payoff0;
     float o[17], lg[3];
     leduc_obs(s, o);
-    mlp_logits(s.actor == 0 ? m0 : m1, o, lg);
+    memo.get(s.actor == 0 ? m0 : m1, s.actor, o, lg);
     uint8_t legal[3];
     leduc_legal(s, legal);
     double mx = -1e300;
@@ -471,12 +490,13 @@ double leduc_tree(const Mlp& m0, const Mlp& m1, const Leduc& s) {
         if (!legal[a]) continue;
         Leduc n = s;
         leduc_apply(n, a);
-        v += (pr[a] / z) * leduc_tree(m0, m1, n);
+        v += (pr[a] / z) * leduc_tree(m0, m1, n, memo);
     }
     return v;
 }
 
 double leduc_exact(const Mlp& m0, const Mlp& m1) {
+    LogitMemo memo;
     double total = 0.0;
     for (int c0 = 0; c0 < 6; ++c0)
         for (int c1 = 0; c1 < 6; ++c1)
@@ -484,7 +504,7 @@ double leduc_exact(const Mlp& m0, const Mlp& m1) {
                 if (c0 == c1 || p == c0 || p == c1) continue;
                 Leduc s;
                 leduc_init(s, c0, c1, p);
-                total += leduc_tree(m0, m1, s) / 120.0;
+                total += leduc_tree(m0, m1, s, memo) / 120.0;
             }
     return total;
 }

@@ -14,15 +14,16 @@ import ctypes as C
 import numpy as np
 
 from . import _abi
-from ._abi import (MALIB_BF16, MALIB_DUMP_LOGITS, MALIB_ENV_KUHN, MALIB_ENV_LEDUC,
-                   MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY, MALIB_ENV_SPEAKER_LISTENER, MALIB_EXACT_EXPECTATION, MALIB_F32, MALIB_POL_MLP,
-                   MALIB_POL_TABULAR, EnvSpec, PolicyDesc, Traj)
+from ._abi import (MALIB_BF16, MALIB_DUMP_LOGITS, MALIB_ENOTCONVERGED, MALIB_ENV_KUHN,
+                   MALIB_ENV_LEDUC, MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY, MALIB_ENV_SPEAKER_LISTENER,
+                   MALIB_EXACT_EXPECTATION, MALIB_F32, MALIB_POL_MLP, MALIB_POL_TABULAR, EnvSpec,
+                   PolicyDesc, Traj)
 
 __all__ = ["MalibError", "Context", "EnvSpec", "make_spec", "policy_desc", "alloc_traj",
            "alloc_eval_dump", "malib_create", "malib_pop_load", "malib_rollout",
            "malib_eval_payoff", "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "MALIB_ENV_KUHN", "MALIB_ENV_LEDUC",
            "MALIB_ENV_SPREAD", "MALIB_ENV_ADVERSARY", "MALIB_ENV_SPEAKER_LISTENER", "MALIB_POL_TABULAR", "MALIB_POL_MLP", "MALIB_F32", "MALIB_BF16",
-           "MALIB_DUMP_LOGITS", "MALIB_EXACT_EXPECTATION"]
+           "MALIB_DUMP_LOGITS", "MALIB_EXACT_EXPECTATION", "MALIB_ENOTCONVERGED"]
 
 
 class MalibError(RuntimeError):
@@ -244,12 +245,19 @@ class Context:
                                                    int(iters), _ptr(x_out), _ptr(y_out),
                                                    _ptr(bounds_out)))
 
-    def meta_lp_nash(self, payoff, x_out, y_out, value_out, stride=1):
-        """LP equilibrium of G games: x_out [G][m], y_out [G][n], value_out [G]."""
+    def meta_lp_nash(self, payoff, x_out, y_out, value_out, stride=1, max_pivots=None):
+        """LP equilibrium of G games: x_out [G][m], y_out [G][n], value_out [G].
+        max_pivots caps the simplex pivots per game (None: the library's default
+        limit); a game over the cap raises ENOTCONVERGED at the next sync()."""
         G, m, n, st = self._table(payoff, stride)
-        _check(self.lib, self.handle,
-               self.lib.malib_meta_lp_nash(self.handle, _ptr(payoff), G, m, n, st, _ptr(x_out),
-                                           _ptr(y_out), _ptr(value_out)))
+        if max_pivots is None:
+            rc = self.lib.malib_meta_lp_nash(self.handle, _ptr(payoff), G, m, n, st, _ptr(x_out),
+                                             _ptr(y_out), _ptr(value_out))
+        else:
+            rc = self.lib.malib_meta_lp_nash_ex(self.handle, _ptr(payoff), G, m, n, st,
+                                                int(max_pivots), _ptr(x_out), _ptr(y_out),
+                                                _ptr(value_out))
+        _check(self.lib, self.handle, rc)
 
     def meta_aggregate(self, payoff, x, y, row_out, col_out, value_out, stride=1):
         """A y -> row_out [G][m], x^T A -> col_out [G][n], x^T A y -> value_out [G]."""

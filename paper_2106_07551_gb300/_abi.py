@@ -13,8 +13,9 @@ from . import build as _build
 
 MALIB_OK, MALIB_EINVAL, MALIB_ENOMEM, MALIB_ECUDA = 0, -1, -2, -3
 MALIB_ESTATE, MALIB_ETIMEOUT, MALIB_EUNSUPPORTED = -4, -5, -6
+MALIB_ENOTCONVERGED = -7
 STATUS_NAMES = {0: "OK", -1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ESTATE", -5: "ETIMEOUT",
-                -6: "EUNSUPPORTED"}
+                -6: "EUNSUPPORTED", -7: "ENOTCONVERGED"}
 
 MALIB_ENV_KUHN, MALIB_ENV_LEDUC, MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY = 1, 2, 3, 4
 MALIB_ENV_SPEAKER_LISTENER = 5
@@ -31,6 +32,7 @@ EXPORTS = (
     "malib_selftest_philox", "malib_philox_digest", "malib_selftest_wait", "malib_selftest_det_expf",
     "malib_selftest_sample",
     "malib_selftest_mma", "malib_meta_fictitious_play", "malib_meta_lp_nash",
+    "malib_meta_lp_nash_ex",
     "malib_meta_aggregate", "malib_exploitability",
 )
 
@@ -97,6 +99,7 @@ def load(path: str | None = None):
             "malib_selftest_mma": (C.c_int, [P, i32, P, P, P, i32, i32]),
             "malib_meta_fictitious_play": (C.c_int, [P, P, i32, i32, i32, i32, i64, P, P, P]),
             "malib_meta_lp_nash": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P]),
+            "malib_meta_lp_nash_ex": (C.c_int, [P, P, i32, i32, i32, i32, i32, P, P, P]),
             "malib_meta_aggregate": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P, P, P]),
             "malib_exploitability": (C.c_int, [P, P, P, i32, P, P, i32, P]),
         }

@@ -155,6 +155,11 @@ struct CtxView {
     bool tc_layout;               // bf16 tensor-core images in the arena (else fp32 layouts)
 };
 bool ctx_view(const void* ctx, CtxView* v);
+// Where a pointer lives, by cudaPointerGetAttributes: host memory (pageable,
+// pinned or unknown), device memory of `device` (or managed memory), or device
+// memory of another GPU, which no kernel of a context on `device` may touch.
+enum : int { kPtrHost = 0, kPtrHere = 1, kPtrOther = -1 };
+int ptr_where(const void* p, int device);
 int ctx_fail(void* ctx, int code, const char* msg);
 void ctx_count_launches(void* ctx, int n);
 // Device work space owned by the context, grown on its stream (cudaMallocAsync).
@@ -171,8 +176,8 @@ int64_t lp_tableau_doubles(int32_t m, int32_t n);
 bool lp_on_chip(int32_t m, int32_t n);
 int lp_grid(int32_t n_games, int n_sm);
 cudaError_t launch_lp_nash(const double* P, int32_t G, int32_t m, int32_t n, int32_t stride,
-                           double* x, double* y, double* val, double* scratch, int* err, int n_sm,
-                           cudaStream_t s);
+                           double* x, double* y, double* val, double* scratch, int32_t pivot_limit,
+                           int* err, int n_sm, cudaStream_t s);
 
 bool leduc_f32_supported(int hidden);
 bool spread_f32_supported(int n_agents, int obs_dim, int hidden);

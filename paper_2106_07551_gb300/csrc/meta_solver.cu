@@ -189,7 +189,8 @@ __global__ void __launch_bounds__(256) aggregate_kernel(
 // Entering column: the most negative reduced cost (Dantzig); after 2 (m + n)
 // consecutive degenerate pivots the rule switches for good to Bland's (lowest
 // index with a negative reduced cost), which cannot cycle. Leaving row: the
-// minimum ratio, ties to the lowest basic variable index. A pivot limit
+// minimum ratio, ties to the lowest basic variable index. A pivot limit (at
+// most that many pivots; optimality is still recognised after the last one)
 // guards regardless. Comparisons run on the integer keys above; the tableau
 // arithmetic is fp64.
 // ---------------------------------------------------------------------------
@@ -209,7 +210,7 @@ __device__ __forceinline__ Cand cta_pick(Cand c, Cand* red) {
 __global__ void __launch_bounds__(kLpThreads) lp_nash_kernel(
     const double* __restrict__ P, int32_t n_games, int32_t m, int32_t n, int32_t stride,
     double* __restrict__ x_out, double* __restrict__ y_out, double* __restrict__ val_out,
-    double* __restrict__ gscratch, int32_t on_chip, int* __restrict__ err) {
+    double* __restrict__ gscratch, int32_t on_chip, int32_t pivot_limit, int* __restrict__ err) {
     extern __shared__ double smem_tab[];
     __shared__ double colq[1024 + 1];
     __shared__ int basis[1024];
@@ -244,10 +245,10 @@ __global__ void __launch_bounds__(kLpThreads) lp_nash_kernel(
         for (int r = tid; r < m; r += kLpThreads) basis[r] = n + r;
         __syncthreads();
 
-        const int max_pivots = 50 * (m + n) + 1000;
+        const int max_pivots = pivot_limit > 0 ? pivot_limit : 50 * (m + n) + 1000;
         bool done = false, bland = false;
         int degenerate = 0;
-        for (int piv = 0; piv < max_pivots; ++piv) {
+        for (int piv = 0;; ++piv) {
             // entering column
             Cand ce = none;
             for (int c = tid; c < n + m; c += kLpThreads) {
@@ -256,6 +257,7 @@ __global__ void __launch_bounds__(kLpThreads) lp_nash_kernel(
             }
             ce = cta_pick(ce, red);
             if (ce.k == kNone) { done = true; break; }
+            if (piv == max_pivots) break;        // another pivot is needed: limit reached
             const int q = ce.i;
             // leaving row: minimum ratio (ratios are >= 0), ties to the lowest
             // basic index; the candidate index packs (basic index, row)
@@ -338,15 +340,15 @@ bool lp_on_chip(int32_t m, int32_t n) { return lp_tableau_doubles(m, n) * 8 <= k
 int lp_grid(int32_t n_games, int n_sm) { return n_games < n_sm ? n_games : n_sm; }
 
 cudaError_t launch_lp_nash(const double* P, int32_t G, int32_t m, int32_t n, int32_t stride,
-                           double* x, double* y, double* val, double* scratch, int* err, int n_sm,
-                           cudaStream_t s) {
+                           double* x, double* y, double* val, double* scratch, int32_t pivot_limit,
+                           int* err, int n_sm, cudaStream_t s) {
     const int on_chip = lp_on_chip(m, n) ? 1 : 0;
     const size_t dyn = on_chip ? (size_t)lp_tableau_doubles(m, n) * 8 : 0;
     cudaError_t e = cudaFuncSetAttribute(lp_nash_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)dyn);
     if (e != cudaSuccess) return e;
     lp_nash_kernel<<<lp_grid(G, n_sm), kLpThreads, dyn, s>>>(P, G, m, n, stride, x, y, val, scratch,
-                                                             on_chip, err);
+                                                             on_chip, pivot_limit, err);
     return cudaGetLastError();
 }
 
@@ -359,15 +361,8 @@ using namespace malib;
 
 namespace {
 
-bool dev_ptr(const void* p) {
-    if (!p) return false;
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-        cudaGetLastError();
-        return false;
-    }
-    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
-}
+// Device memory of the context's own device.
+bool dev_ptr(int device, const void* p) { return p && ptr_where(p, device) == kPtrHere; }
 
 struct DevSel {
     int prev = -1;
@@ -381,7 +376,7 @@ struct DevSel {
     }
 };
 
-int check_table(malib_ctx* ctx, const double* payoff, int32_t G, int32_t m, int32_t n,
+int check_table(malib_ctx* ctx, int device, const double* payoff, int32_t G, int32_t m, int32_t n,
                 int32_t stride, int32_t max_dim) {
     if (G < 0) return ctx_fail(ctx, MALIB_EINVAL, "n_games < 0");
     if (m < 1 || n < 1 || m > max_dim || n > max_dim)
@@ -390,7 +385,7 @@ int check_table(malib_ctx* ctx, const double* payoff, int32_t G, int32_t m, int3
     if (stride < 1) return ctx_fail(ctx, MALIB_EINVAL, "stride < 1");
     if ((int64_t)G * m * n * stride > ((int64_t)1 << 40))
         return ctx_fail(ctx, MALIB_EINVAL, "payoff table too large");
-    if (G > 0 && !dev_ptr(payoff)) return ctx_fail(ctx, MALIB_EINVAL, "payoff must be device memory");
+    if (G > 0 && !dev_ptr(device, payoff)) return ctx_fail(ctx, MALIB_EINVAL, "payoff must be device memory of the context's device");
     return MALIB_OK;
 }
 
@@ -407,12 +402,12 @@ extern "C" int malib_meta_fictitious_play(malib_ctx* ctx, const double* payoff, 
                                           double* x_out, double* y_out, double* bounds_out) {
     CtxView v;
     if (!ctx_view(ctx, &v)) return MALIB_EINVAL;
-    int r = check_table(ctx, payoff, n_games, m, n, stride, kFpMaxDim);
+    int r = check_table(ctx, v.device, payoff, n_games, m, n, stride, kFpMaxDim);
     if (r != MALIB_OK) return r;
     if (iters < 1) return ctx_fail(ctx, MALIB_EINVAL, "iters must be >= 1");
     if (n_games == 0) return MALIB_OK;
-    if (!dev_ptr(x_out) || !dev_ptr(y_out) || !dev_ptr(bounds_out))
-        return ctx_fail(ctx, MALIB_EINVAL, "x_out, y_out and bounds_out must be device memory");
+    if (!dev_ptr(v.device, x_out) || !dev_ptr(v.device, y_out) || !dev_ptr(v.device, bounds_out))
+        return ctx_fail(ctx, MALIB_EINVAL, "x_out, y_out and bounds_out must be device memory of the context's device");
     DevSel d(v.device);
     if (!d.ok) return ctx_fail(ctx, MALIB_ECUDA, "cannot select the context's device");
     return launched(ctx, launch_fictitious_play(payoff, n_games, m, n, stride, iters, x_out, y_out,
@@ -425,28 +420,29 @@ extern "C" int malib_meta_aggregate(malib_ctx* ctx, const double* payoff, int32_
                                     double* col_payoff_out, double* value_out) {
     CtxView v;
     if (!ctx_view(ctx, &v)) return MALIB_EINVAL;
-    int r = check_table(ctx, payoff, n_games, m, n, stride, 1 << 20);
+    int r = check_table(ctx, v.device, payoff, n_games, m, n, stride, 1 << 20);
     if (r != MALIB_OK) return r;
     if (n_games == 0) return MALIB_OK;
-    if (!dev_ptr(x) || !dev_ptr(y) || !dev_ptr(row_payoff_out) || !dev_ptr(col_payoff_out) ||
-        !dev_ptr(value_out))
-        return ctx_fail(ctx, MALIB_EINVAL, "mixtures and outputs must be device memory");
+    if (!dev_ptr(v.device, x) || !dev_ptr(v.device, y) || !dev_ptr(v.device, row_payoff_out) ||
+        !dev_ptr(v.device, col_payoff_out) || !dev_ptr(v.device, value_out))
+        return ctx_fail(ctx, MALIB_EINVAL, "mixtures and outputs must be device memory of the context's device");
     DevSel d(v.device);
     if (!d.ok) return ctx_fail(ctx, MALIB_ECUDA, "cannot select the context's device");
     return launched(ctx, launch_aggregate(payoff, n_games, m, n, stride, x, y, row_payoff_out,
                                           col_payoff_out, value_out, v.n_sm, v.stream), 1);
 }
 
-extern "C" int malib_meta_lp_nash(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
-                                  int32_t n, int32_t stride, double* x_out, double* y_out,
-                                  double* value_out) {
+extern "C" int malib_meta_lp_nash_ex(malib_ctx* ctx, const double* payoff, int32_t n_games,
+                                     int32_t m, int32_t n, int32_t stride, int32_t max_pivots,
+                                     double* x_out, double* y_out, double* value_out) {
     CtxView v;
     if (!ctx_view(ctx, &v)) return MALIB_EINVAL;
-    int r = check_table(ctx, payoff, n_games, m, n, stride, 512);
+    int r = check_table(ctx, v.device, payoff, n_games, m, n, stride, 512);
     if (r != MALIB_OK) return r;
+    if (max_pivots < 0) return ctx_fail(ctx, MALIB_EINVAL, "max_pivots < 0");
     if (n_games == 0) return MALIB_OK;
-    if (!dev_ptr(x_out) || !dev_ptr(y_out) || !dev_ptr(value_out))
-        return ctx_fail(ctx, MALIB_EINVAL, "x_out, y_out and value_out must be device memory");
+    if (!dev_ptr(v.device, x_out) || !dev_ptr(v.device, y_out) || !dev_ptr(v.device, value_out))
+        return ctx_fail(ctx, MALIB_EINVAL, "x_out, y_out and value_out must be device memory of the context's device");
     DevSel d(v.device);
     if (!d.ok) return ctx_fail(ctx, MALIB_ECUDA, "cannot select the context's device");
     double* scratch = nullptr;
@@ -457,5 +453,11 @@ extern "C" int malib_meta_lp_nash(malib_ctx* ctx, const double* payoff, int32_t 
         scratch = static_cast<double*>(p);
     }
     return launched(ctx, launch_lp_nash(payoff, n_games, m, n, stride, x_out, y_out, value_out,
-                                        scratch, v.err, v.n_sm, v.stream), 1);
+                                        scratch, max_pivots, v.err, v.n_sm, v.stream), 1);
+}
+
+extern "C" int malib_meta_lp_nash(malib_ctx* ctx, const double* payoff, int32_t n_games, int32_t m,
+                                  int32_t n, int32_t stride, double* x_out, double* y_out,
+                                  double* value_out) {
+    return malib_meta_lp_nash_ex(ctx, payoff, n_games, m, n, stride, 0, x_out, y_out, value_out);
 }

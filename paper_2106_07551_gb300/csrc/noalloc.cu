@@ -51,15 +51,6 @@ cudaError_t scratch_address(int device, unsigned long long** out) {
     return cudaSuccess;
 }
 
-bool on_device(const void* p) {
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-        cudaGetLastError();
-        return false;
-    }
-    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
-}
-
 }  // namespace
 
 }  // namespace malib
@@ -98,10 +89,10 @@ extern "C" int malib_eval_payoff_noalloc(malib_ctx* ctx, const int32_t* pair_ids
     int code = MALIB_OK;
     unsigned long long* scratch = nullptr;
     cudaError_t e;
-    if (!on_device(pair_ids) || !on_device(payoff_out)) {
+    if (ptr_where(pair_ids, v.device) != kPtrHere || ptr_where(payoff_out, v.device) != kPtrHere) {
         code = ctx_fail(ctx, MALIB_EINVAL,
-                        "malib_eval_payoff_noalloc needs device pair_ids and payoff_out "
-                        "(host buffers would need a staging allocation)");
+                        "malib_eval_payoff_noalloc needs pair_ids and payoff_out in device memory "
+                        "of the context's device (host buffers would need a staging allocation)");
     } else if ((e = scratch_address(v.device, &scratch)) != cudaSuccess) {
         code = ctx_fail(ctx, MALIB_ECUDA, cudaGetErrorString(e));
     } else {

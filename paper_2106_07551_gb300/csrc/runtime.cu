@@ -108,14 +108,8 @@ int cuda_fail(malib_ctx* c, cudaError_t e, const char* what) {
         if (e_ != cudaSuccess) return cuda_fail(c, e_, what); \
     } while (0)
 
-bool is_device_ptr(const void* p) {
-    cudaPointerAttributes at;
-    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-        cudaGetLastError();
-        return false;
-    }
-    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
-}
+// Device memory of the context's own device (or managed memory).
+bool is_device_ptr(const malib_ctx* c, const void* p) { return ptr_where(p, c->device) == kPtrHere; }
 
 template <class T>
 int ensure(malib_ctx* c, T*& p, int64_t& cap, int64_t need, const char* what) {
@@ -207,7 +201,10 @@ int upload_tables(malib_ctx* c) {
 
 int stage_pairs(malib_ctx* c, const int32_t* pair_ids, int64_t n_ints, int width, bool poker,
                 const int32_t** dev_pairs) {
-    if (is_device_ptr(pair_ids)) {
+    const int where = ptr_where(pair_ids, c->device);
+    if (where == kPtrOther)
+        return fail(c, MALIB_EINVAL, "pair_ids lives on another device than the context's");
+    if (where == kPtrHere) {
         *dev_pairs = pair_ids;      // validated by the kernels
         return MALIB_OK;
     }
@@ -281,6 +278,17 @@ EvalArgs eval_args(malib_ctx* c) {
 }  // namespace
 
 namespace malib {
+
+int ptr_where(const void* p, int device) {
+    cudaPointerAttributes at;
+    if (!p || cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return kPtrHost;
+    }
+    if (at.type == cudaMemoryTypeManaged) return kPtrHere;
+    if (at.type == cudaMemoryTypeDevice) return at.device == device ? kPtrHere : kPtrOther;
+    return kPtrHost;
+}
 
 bool ctx_view(const void* ctx, CtxView* v) {
     const malib_ctx* c = static_cast<const malib_ctx*>(ctx);
@@ -558,7 +566,8 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
         if (n_dump < 0 || n_dump > n_episodes) return fail(c, MALIB_EINVAL, "n_dump out of range");
         const void* ptrs[5] = {dump->obs, dump->action, dump->reward, dump->done, dump->logits};
         for (const void* p : ptrs)
-            if (p && !is_device_ptr(p)) return fail(c, MALIB_EINVAL, "dump buffers must be device memory");
+            if (p && !is_device_ptr(c, p))
+                return fail(c, MALIB_EINVAL, "dump buffers must be device memory of the context's device");
     }
     const bool leduc_tc = kind == MALIB_ENV_LEDUC && c->tc_layout && c->dims[0] == 17 &&
                           c->dims[3] == 3;
@@ -571,7 +580,10 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
     if ((r = upload_tables(c)) != MALIB_OK) return r;
     const int32_t* dpairs = nullptr;
     if ((r = stage_pairs(c, pair_ids, (int64_t)n_pairs * 2, 2, true, &dpairs)) != MALIB_OK) return r;
-    const bool host_out = !is_device_ptr(payoff_out);
+    const int out_where = ptr_where(payoff_out, c->device);
+    if (out_where == kPtrOther)
+        return fail(c, MALIB_EINVAL, "payoff_out lives on another device than the context's");
+    const bool host_out = out_where == kPtrHost;
     double* dout = payoff_out;
     if (host_out) {
         if ((r = ensure(c, c->d_out, c->out_cap, (int64_t)n_pairs * 4, "output staging")) != MALIB_OK)
@@ -657,7 +669,8 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     const void* ptrs[5] = {traj->obs, traj->action, traj->reward, traj->done,
                            want_logits ? traj->logits : traj->obs};
     for (const void* p : ptrs) {
-        if (!is_device_ptr(p)) return fail(c, MALIB_EINVAL, "trajectory buffers must be device memory");
+        if (!is_device_ptr(c, p))
+            return fail(c, MALIB_EINVAL, "trajectory buffers must be device memory of the context's device");
         if (((uintptr_t)p & 15u) != 0) return fail(c, MALIB_EINVAL, "trajectory buffers must be 16-byte aligned");
     }
     const int64_t epp = spec->n_envs / n_pairs;
@@ -755,7 +768,7 @@ int malib_selftest_philox(malib_ctx* c, const uint32_t* ctr, uint64_t seed, uint
                           int64_t n) {
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);
-    if (n < 0 || (n > 0 && (!ctr || !out || !is_device_ptr(ctr) || !is_device_ptr(out))))
+    if (n < 0 || (n > 0 && (!ctr || !out || !is_device_ptr(c, ctr) || !is_device_ptr(c, out))))
         return fail(c, MALIB_EINVAL, "philox self-test needs device buffers");
     CK(launch_selftest_philox(ctr, seed, out, n, c->stream), "philox kernel");
     c->launches += n > 0;
@@ -765,7 +778,7 @@ int malib_selftest_philox(malib_ctx* c, const uint32_t* ctr, uint64_t seed, uint
 int malib_philox_digest(malib_ctx* c, uint64_t seed, int64_t n, int32_t calls, uint32_t* out) {
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);
-    if (n < 0 || calls < 0 || (n > 0 && (!out || !is_device_ptr(out))))
+    if (n < 0 || calls < 0 || (n > 0 && (!out || !is_device_ptr(c, out))))
         return fail(c, MALIB_EINVAL, "philox digest needs n >= 0, calls >= 0 and a device buffer");
     CK(launch_philox_digest(seed, n, calls, out, c->stream), "philox digest kernel");
     c->launches += n > 0;
@@ -785,7 +798,7 @@ int malib_selftest_wait(malib_ctx* c, int32_t arrive, int64_t limit_ns) {
 int malib_selftest_det_expf(malib_ctx* c, const float* x, float* y, int64_t n) {
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);
-    if (n < 0 || (n > 0 && (!x || !y || !is_device_ptr(x) || !is_device_ptr(y))))
+    if (n < 0 || (n > 0 && (!x || !y || !is_device_ptr(c, x) || !is_device_ptr(c, y))))
         return fail(c, MALIB_EINVAL, "det_expf self-test needs device buffers");
     CK(launch_selftest_det_expf(x, y, n, c->stream), "det_expf kernel");
     c->launches += n > 0;
@@ -797,8 +810,8 @@ int malib_selftest_sample(malib_ctx* c, const float* logits, const uint8_t* lega
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);
     if (A < 2 || A > 8) return fail(c, MALIB_EINVAL, "A must be in [2, 8]");
-    if (n < 0 || (n > 0 && (!logits || !legal || !u || !out || !is_device_ptr(logits) ||
-                            !is_device_ptr(legal) || !is_device_ptr(u) || !is_device_ptr(out))))
+    if (n < 0 || (n > 0 && (!logits || !legal || !u || !out || !is_device_ptr(c, logits) ||
+                            !is_device_ptr(c, legal) || !is_device_ptr(c, u) || !is_device_ptr(c, out))))
         return fail(c, MALIB_EINVAL, "sample self-test needs device buffers");
     CK(launch_selftest_sample(logits, legal, u, A, out, n, c->stream), "sample kernel");
     c->launches += n > 0;

@@ -11,18 +11,26 @@ import pytest
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
-def test_reference_arm_json_line():
-    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
-                        "--steps", "2", "--warmup", "1"], capture_output=True, text=True,
-                       timeout=600, cwd=ROOT)
+@pytest.mark.parametrize("workload,prefix", [(None, "leduc_holdem_64x64"),
+                                              ("kuhn", "kuhn_4x4"),
+                                              ("spread3", "spread_n3_4096env")])
+def test_reference_arm_json_line(workload, prefix):
+    """The reference arm times the oracle on the GPU arm's own workload (the
+    default is the 64 x 64 bf16 Leduc sweep) and prints one JSON line."""
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+           "--steps", "2", "--warmup", "1"]
+    if workload:
+        cmd += ["--workload", workload]
+    r = subprocess.run(cmd, capture_output=True, text=True, timeout=600, cwd=ROOT)
     assert r.returncode == 0, r.stderr[-2000:]
     lines = [l for l in r.stdout.splitlines() if l.strip().startswith("{")]
     assert len(lines) == 1
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
-    assert d["e2e"]["h2d_bytes_per_step"] == 0
-    assert d["config"]["workload"].startswith("leduc_holdem_8x8")
+    assert d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
+    assert d["config"]["workload"].startswith(prefix)
 
 
 def _worker(rank, world, port, q):

@@ -1,0 +1,58 @@
+"""The library's two quick-start uses, written as a user would: a Leduc payoff
+table between 8 + 8 fp32 MLP policies, and a particle-spread rollout of 3
+agents over 4,096 environments in 32 blocks of 128 with their own policy
+combinations. Checks the shapes and invariants of what comes back."""
+import numpy as np
+import pytest
+
+from gpu_util import need_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+def _mlp(rng, dims):
+    """Row-major W[out][in] then b[out], per layer, fp32."""
+    parts = []
+    for fi, fo in zip(dims[:-1], dims[1:]):
+        parts += [rng.normal(0, fi ** -0.5, (fo, fi)).astype(np.float32).ravel(),
+                  np.zeros(fo, np.float32)]
+    return np.concatenate(parts)
+
+
+def test_quick_start_payoff_table_and_rollout():
+    need_gpu()
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2106_07551_gb300 import (MALIB_ENV_LEDUC, MALIB_ENV_SPREAD, MALIB_F32,
+                                        MALIB_POL_MLP, Context, alloc_traj, make_spec,
+                                        policy_desc)
+    rng = np.random.default_rng(0)
+    dims = (17, 128, 128, 3)
+    params = [_mlp(rng, dims) for _ in range(16)]
+    seats = [0] * 8 + [1] * 8
+    spec = make_spec(MALIB_ENV_LEDUC, 2, 17, 3)
+    with Context(0) as ctx:
+        ids = ctx.pop_load(spec, [policy_desc(MALIB_POL_MLP, MALIB_F32, s, dims, p)
+                                  for s, p in zip(seats, params)])
+        pairs = np.array([[i, j] for i in ids[:8] for j in ids[8:]], np.int32)
+        table = ctx.eval_payoff(pairs, 65536, 1)
+    assert table.shape == (64, 4)
+    assert np.all(np.isfinite(table)) and np.all(table[:, 1] > 0)
+    assert np.all(np.abs(table[:, 0]) <= 13)
+
+    dims = (18, 64, 64, 5)
+    params = [_mlp(rng, dims) for _ in range(16)]
+    spec = make_spec(MALIB_ENV_SPREAD, 3, 18, 5, n_landmarks=3, episode_len=25, n_envs=4096)
+    with Context(0) as ctx:
+        ids = ctx.pop_load(spec, [policy_desc(MALIB_POL_MLP, MALIB_F32, -1, dims, p)
+                                  for p in params])
+        combos = rng.integers(0, 16, (32, 3)).astype(np.int32)
+        traj = alloc_traj(spec, 2)
+        ctx.rollout(spec, combos, 2, 7, traj)
+        ctx.sync()
+    obs = traj["obs"].cpu().numpy()
+    assert obs.shape == (2, 25, 4096, 3, 20)
+    assert traj["action"].cpu().numpy().max() <= 4
+    done = traj["done"].cpu().numpy()
+    assert np.all(done[:, -1] == 1) and np.all(done[:, :-1] == 0)
+    assert np.all(traj["reward"].cpu().numpy() <= 0)

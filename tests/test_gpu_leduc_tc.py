@@ -1,14 +1,15 @@
 """GPU parity for Leduc hold'em evaluation with bf16 MLP policies
-17-256-256-3 on the tensor cores (2-CTA clusters, one seat's policy per CTA).
+17-256-256-3 on the tensor cores.
 
 Every dumped hand is replayed by the oracle (bf16 emulation: weights and layer
 inputs rounded to bf16, fp64 sums) with the GPU's logits: observations,
 actions, payoffs and the integer payoff sums must match exactly, and the GPU
 logits must match the oracle's within 2e-2 relative (|g - o| <= 2e-2 max(|o|,
-rms of the row)). At the full 64x64 x 16,384 workload, sampled hands are
-replayed and 64 sampled entries are checked against the exact tree
-expectation (4-SE rule)."""
+rms of the row)). At the full 64x64 x 16,384 workload, the first 16 hands of
+every pair are replayed and every one of the 4,096 entries is checked against
+the exact tree expectation (at most 3 beyond 4 SE, none beyond 5)."""
 import concurrent.futures as cf
+import os
 
 import numpy as np
 import pytest
@@ -64,24 +65,24 @@ def test_full_replay_parity(orc, n_eps):
     ctx.close()
 
 
-def test_full_workload_sampled(orc):
-    """64x64 pairs x 16,384 hands: 4 hands per pair replayed; 64 entries vs exact."""
+def test_full_workload_every_cell(orc):
+    """64x64 pairs x 16,384 hands: 16 hands of every pair replayed; all 4,096
+    entries against the exact tree expectation."""
     need_gpu()
     w = workloads.config(5)
     ctx = context()
     load_population(ctx, w)
-    res, d = run(ctx, w, w.n_episodes, w.seed, 4)
-    replay(orc, w, res, d, w.n_episodes, w.seed, 4, full=False)
+    res, d = run(ctx, w, w.n_episodes, w.seed, 16)
+    replay(orc, w, res, d, w.n_episodes, w.seed, 16, full=False)
     plain = ctx.eval_payoff(w.pair_ids, w.n_episodes, w.seed)
     np.testing.assert_array_equal(plain, res)
+    ctx.close()
     params = [p.params for p in w.policies]
     dims = w.policies[0].dims
-    rng = np.random.default_rng(0)
-    pick = rng.choice(w.n_pairs, 64, replace=False)
-    with cf.ThreadPoolExecutor(16) as ex:
+    with cf.ThreadPoolExecutor(os.cpu_count() or 4) as ex:
         exact = np.array(list(ex.map(
             lambda k: orc.leduc_exact(params[w.pair_ids[k][0]], params[w.pair_ids[k][1]], dims,
-                                      bf16=True), pick)))
-    n_out, zmax = four_se_rule(res[pick, 0], res[pick, 1], exact)
+                                      bf16=True), range(w.n_pairs))))
+    assert np.all(res[:, 2] == np.round(res[:, 0] * w.n_episodes))
+    n_out, zmax = four_se_rule(res[:, 0], res[:, 1], exact)
     assert n_out <= 3 and zmax < 5, (n_out, zmax)
-    ctx.close()

@@ -142,6 +142,36 @@ def test_lp_off_chip(ctx):
     check_lp(tables, *run_lp(ctx, tables))
 
 
+def test_lp_pivot_limit_reports_not_converged(ctx):
+    """A game that needs more simplex pivots than the caller's limit raises
+    ENOTCONVERGED at the next sync; the flag is cleared once read and the
+    context stays usable. Rock-paper-scissors needs at least 3 pivots (its
+    optimal basis holds all 3 columns, one enters per pivot); a 1 x 1 game
+    needs exactly 1, so a limit of 1 still converges."""
+    torch = need_gpu()
+    from paper_2106_07551_gb300 import MALIB_ENOTCONVERGED, MalibError
+    rps = np.array([[[0, -1, 1], [1, 0, -1], [-1, 1, 0]]], float)
+    P = torch.from_numpy(rps).cuda()
+    x = torch.empty((1, 3), dtype=torch.float64, device="cuda")
+    y = torch.empty((1, 3), dtype=torch.float64, device="cuda")
+    v = torch.empty((1,), dtype=torch.float64, device="cuda")
+    ctx.meta_lp_nash(P, x, y, v, max_pivots=2)
+    with pytest.raises(MalibError) as e:
+        ctx.sync()
+    assert e.value.code == MALIB_ENOTCONVERGED and "ENOTCONVERGED" in str(e.value)
+    ctx.sync()                                       # cleared once reported
+    ctx.meta_lp_nash(P, x, y, v, max_pivots=3 * 6)
+    ctx.sync()
+    check_lp(rps, x.cpu().numpy(), y.cpu().numpy(), v.cpu().numpy())
+    one = torch.full((1, 1, 1), 0.5, dtype=torch.float64, device="cuda")
+    x1 = torch.empty((1, 1), dtype=torch.float64, device="cuda")
+    ctx.meta_lp_nash(one, x1, x1.clone(), v, max_pivots=1)
+    ctx.sync()
+    assert abs(float(v[0]) - 0.5) < 1e-15
+    with pytest.raises(MalibError):
+        ctx.meta_lp_nash(P, x, y, v, max_pivots=-1)
+
+
 def test_aggregate(ctx):
     torch = need_gpu()
     rng = np.random.default_rng(13)

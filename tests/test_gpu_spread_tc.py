@@ -1,12 +1,13 @@
 """GPU parity for the particle-spread rollout with N = 8 agents and bf16 MLP
-policies 34-256-256-5 on the tensor cores (8-CTA clusters, one agent's policy
-per CTA, actions exchanged through distributed shared memory).
+policies 34-256-256-5 on the tensor cores.
 
 The oracle replays the same environments with the GPU's logits (bf16
 emulation for its own logits): observations (with zero padding), actions,
 rewards and done flags must match bit for bit, and the GPU logits must match
-the oracle's within 2e-2 relative. The full 65,536-env workload is checked on
-sampled env slices."""
+the oracle's within 2e-2 relative. The full 65,536-env workload is checked in
+the benchmark's launch (two episodes per environment) on slices of 16
+environments from 8 combinations spread across the combination table (first,
+middle and last environments of a combination among them)."""
 import numpy as np
 import pytest
 
@@ -73,15 +74,35 @@ def test_local_ratio_replay_parity(orc):
 
 
 def test_full_workload_sampled_envs(orc):
-    """65,536 envs, 512 combinations of 128 envs, population 32, one episode."""
+    """65,536 envs, 512 combinations of 128 envs, population 32, two episodes."""
     need_gpu()
     w = workloads.config(4)
+    n_eps = 2
     ctx = context()
     load_population(ctx, w)
-    g = rollout(ctx, w, 1, w.seed)
-    for lo, hi in ((0, 24), (30000, 30010), (65530, 65536)):
-        check(orc, w, g, 1, w.seed, lo, hi)
-    assert np.all(g["reward"] <= 0)
+    spec = spec_of(w, MALIB_DUMP_LOGITS)
+    traj = alloc_traj(spec, n_eps, logits=True)
+    ctx.rollout(spec, w.pair_ids, n_eps, w.seed, traj)
+    ctx.sync()
+    assert bool((traj["reward"] <= 0).all())
+    epp = w.n_envs // w.n_pairs
+    combos = [0, 37, 101, 178, 255, 300, 433, w.n_pairs - 1]
+    offs = [(0, 16), (56, 72), (112, 128)]
+    for j, c in enumerate(combos):
+        a, b = offs[j % len(offs)]
+        lo, hi = c * epp + a, c * epp + b
+        g = {k: v[:, :, lo:hi].cpu().numpy() for k, v in traj.items()}
+        params = [p.params for p in w.policies]
+        ref = orc.spread_rollout(params, w.policies[0].dims, w.n_agents, w.n_landmarks,
+                                 w.episode_len, w.n_envs, w.pair_ids, n_eps, w.seed, bf16=True,
+                                 env_lo=lo, env_hi=hi, ext_logits=g["logits"])
+        np.testing.assert_array_equal(g["obs"][..., :w.obs_dim], ref["obs"])
+        assert np.all(g["obs"][..., w.obs_dim:] == 0)
+        np.testing.assert_array_equal(g["action"].astype(np.int8), ref["action"])
+        np.testing.assert_array_equal(g["reward"], ref["reward"])
+        assert np.all(g["done"][:, -1] == 1) and np.all(g["done"][:, :-1] == 0)
+        n_bad, worst = logits_close(g["logits"], ref["logits"], RTOL)
+        assert n_bad == 0, (c, n_bad, worst)
     ctx.close()
 
 

@@ -6,8 +6,10 @@ latency-critical loop where cudaMalloc / cudaFree would synchronise the device.
 Its scratch is a fixed device array inside the library, so this test checks,
 through the C ABI, that two calls in a row give exactly the table of the
 ordinary allocating entry point (integer sums bit-exact, mean and SE to 1e-12),
-that the shared scratch is cleared between calls, and that sizes beyond the
-array's capacity and host buffers are refused. This file is collected last.
+that the shared scratch is cleared between calls, that the call leaves the
+device's free memory unchanged on a context that has never evaluated, that
+exactly 8192 pairs are served while more, host buffers and bf16 (tensor-core)
+Leduc populations are refused. This file is collected last.
 """
 import ctypes as C
 
@@ -61,16 +63,67 @@ def test_noalloc_refuses_oversize_and_host_buffers():
     w = workloads.kuhn()
     ctx = context()
     load_population(ctx, w)
-    big = torch.from_numpy(np.tile(w.pair_ids, (8193 // w.n_pairs + 1, 1))[:8193].copy()).cuda()
+    tiled = np.tile(w.pair_ids, (8193 // w.n_pairs + 1, 1))
+    big = torch.from_numpy(tiled[:8193].copy()).cuda()
     out = torch.zeros((8193, 4), dtype=torch.float64, device="cuda")
     assert _noalloc(ctx, big, 10, 0, out) == _abi.MALIB_EINVAL
     assert "8192" in ctx.last_error()
+    # exactly the capacity is served, with the ordinary entry point's table
+    edge = torch.from_numpy(tiled[:8192].copy()).cuda()
+    out = torch.full((8192, 4), -1.0, dtype=torch.float64, device="cuda")
+    assert _noalloc(ctx, edge, 10, 3, out) == 0, ctx.last_error()
+    ctx.sync()
+    ref = ctx.eval_payoff(tiled[:8192].copy(), 10, 3)
+    np.testing.assert_array_equal(out.cpu().numpy()[:, 2:], ref[:, 2:])
     lib = _abi.load()
     h_out = np.zeros((w.n_pairs, 4), np.float64)
     d_pairs = torch.from_numpy(w.pair_ids).cuda()
     code = lib.malib_eval_payoff_noalloc(ctx.handle, C.c_void_p(d_pairs.data_ptr()), w.n_pairs,
                                          10, 0, h_out.ctypes.data_as(C.c_void_p))
     assert code == _abi.MALIB_EINVAL
+    ctx.close()
+    # bf16 Leduc populations run on the tensor-core kernel, which this entry
+    # point does not serve
+    wb = workloads.leduc(pop=2, hidden=256, dtype=workloads.BF16, seed=79)
+    ctx = context()
+    load_population(ctx, wb)
+    d_pairs = torch.from_numpy(wb.pair_ids).cuda()
+    out = torch.zeros((wb.n_pairs, 4), dtype=torch.float64, device="cuda")
+    assert _noalloc(ctx, d_pairs, 10, 0, out) == _abi.MALIB_EUNSUPPORTED
+    ctx.close()
+
+
+@pytest.mark.parametrize("kind", ["kuhn", "leduc"])
+def test_noalloc_leaves_free_memory_unchanged(kind):
+    """On a context that has never evaluated (so none of its evaluation
+    buffers exists), two calls change the device's free memory by nothing. The
+    kernels and the library's scratch array are loaded first on another
+    context, so lazy module loading does not count."""
+    torch = need_gpu()
+    w = (workloads.leduc(pop=3, with_bias=True, seed=80) if kind == "leduc" else workloads.kuhn())
+    n_eps = 2000 if kind == "leduc" else 10_000
+    d_pairs = torch.from_numpy(w.pair_ids).cuda()
+    out = torch.zeros((w.n_pairs, 4), dtype=torch.float64, device="cuda")
+    warm = context()
+    load_population(warm, w)
+    ref = warm.eval_payoff(w.pair_ids, n_eps, 4)
+    assert _noalloc(warm, d_pairs, n_eps, 4, out) == 0, warm.last_error()
+    warm.sync()
+    warm.close()
+    out.fill_(-1.0)                            # torch's own kernel loaded before the window
+    ctx = context()
+    load_population(ctx, w)
+    ctx.sync()
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    for _ in range(2):
+        out.fill_(-1.0)
+        assert _noalloc(ctx, d_pairs, n_eps, 4, out) == 0, ctx.last_error()
+        ctx.sync()
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0, (free0, free1)
+    np.testing.assert_array_equal(out.cpu().numpy()[:, 2:], ref[:, 2:])
     ctx.close()
 
 
