@@ -400,6 +400,20 @@ int malib_selftest_sample(malib_ctx* ctx, const float* logits, const uint8_t* le
 int malib_selftest_mma(malib_ctx* ctx, int32_t dtype, const void* A, const void* B, float* D,
                        int32_t N, int32_t K);
 
+/* Policy forward (Sec. 3.1: the policy's action distribution for an
+ * observation; a3 of the rollout) on the pipelined tensor-core engine alone:
+ * logits_out [n_rows][A] = the MLP of policy `policy_id` of the loaded bf16
+ * population on the fp32 observation rows x [n_rows][in] (bf16 weights and
+ * layer inputs, fp32 accumulation; layer 3 on the CUDA cores). Built for the
+ * 17-256-256-3 Leduc populations (observation feature 15 must be 1, as every
+ * Leduc state has it) and 34-256-256-5 populations; other shapes give
+ * EUNSUPPORTED. reps >= 1 repeats the whole set (the same logits are written
+ * again) so that the engine's rate can be measured on resident inputs. x and
+ * logits_out are device buffers of the context's device; asynchronous on the
+ * context's stream. */
+int malib_selftest_mlp_tc(malib_ctx* ctx, int32_t policy_id, const float* x, int64_t n_rows,
+                          int32_t reps, float* logits_out);
+
 #ifdef __cplusplus
 }
 #endif

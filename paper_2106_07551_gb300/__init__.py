@@ -307,6 +307,13 @@ class Context:
         _check(self.lib, self.handle,
                self.lib.malib_selftest_mma(self.handle, dtype, _ptr(A), _ptr(B), _ptr(D), N, K))
 
+    def selftest_mlp_tc(self, policy_id, x, out, reps=1):
+        """logits out [n][A] of policy policy_id on rows x [n][in] (device fp32)
+        through the pipelined tensor-core engine."""
+        _check(self.lib, self.handle,
+               self.lib.malib_selftest_mlp_tc(self.handle, int(policy_id), _ptr(x), int(x.shape[0]),
+                                              int(reps), _ptr(out)))
+
     def selftest_sample(self, logits, legal, u, out):
         n, A = logits.shape
         _check(self.lib, self.handle,

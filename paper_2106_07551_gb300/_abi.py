@@ -31,7 +31,7 @@ EXPORTS = (
     "malib_set_timing", "malib_main_kernel_ms",
     "malib_selftest_philox", "malib_philox_digest", "malib_selftest_wait", "malib_selftest_det_expf",
     "malib_selftest_sample",
-    "malib_selftest_mma", "malib_meta_fictitious_play", "malib_meta_lp_nash",
+    "malib_selftest_mma", "malib_selftest_mlp_tc", "malib_meta_fictitious_play", "malib_meta_lp_nash",
     "malib_meta_lp_nash_ex",
     "malib_meta_aggregate", "malib_exploitability",
 )
@@ -97,6 +97,7 @@ def load(path: str | None = None):
             "malib_selftest_det_expf": (C.c_int, [P, P, P, i64]),
             "malib_selftest_sample": (C.c_int, [P, P, P, P, i32, P, i64]),
             "malib_selftest_mma": (C.c_int, [P, i32, P, P, P, i32, i32]),
+            "malib_selftest_mlp_tc": (C.c_int, [P, i32, P, i64, i32, P]),
             "malib_meta_fictitious_play": (C.c_int, [P, P, i32, i32, i32, i32, i64, P, P, P]),
             "malib_meta_lp_nash": (C.c_int, [P, P, i32, i32, i32, i32, P, P, P]),
             "malib_meta_lp_nash_ex": (C.c_int, [P, P, i32, i32, i32, i32, i32, P, P, P]),

@@ -39,7 +39,8 @@ struct F32Layout {
 
 // bf16 tensor-core policy image (bytes): W1 [256][K1], W2 [256][256], W3 [16][256]
 // as bf16 in the core-matrix K-major layout (K1 = input width rounded up to
-// 16, rows past the output width zero), then fp32 b1[256], b2[256], b3[16].
+// 16, rows past the output width zero), then fp32 b1[256], b2[256], b3[16], then
+// fp32 W3 [16][256] with the bf16-rounded weights (for a CUDA-core layer 3).
 // Built for populations with h1 = h2 = 256, input <= 48, output <= 16.
 inline bool tc_image_shape(const int* d) {
     return d[1] == 256 && d[2] == 256 && d[0] >= 1 && d[0] <= 48 && d[3] >= 1 && d[3] <= 16;
@@ -51,7 +52,7 @@ constexpr int kLeducConstFeature = 15;
 inline bool leduc_tc_fold(int env_kind, int in) { return env_kind == MALIB_ENV_LEDUC && in == 17; }
 inline int64_t tc_image_bytes(int in) {
     const int64_t k1 = (in + 15) / 16 * 16;
-    return 256 * k1 * 2 + 256 * 256 * 2 + 16 * 256 * 2 + (256 + 256 + 16) * 4;
+    return 256 * k1 * 2 + 256 * 256 * 2 + 16 * 256 * 2 + (256 + 256 + 16) * 4 + 16 * 256 * 4;
 }
 
 // Output sums of the payoff reduction: per pair {sum r, sum r^2} as 64-bit
