@@ -27,8 +27,8 @@
 // Roles: each slot has its own epilogue team of 8 warps (warps 0-7 slot 0,
 // warps 8-15 slot 1; in a team, warp w: lane quarter q = w % 4, half
 // p = (w / 4) % 2 of the columns: [64p, 64p + 64)), so the two slots'
-// epilogues run concurrently; the first thread of warp 16 issues every MMA,
-// each slot's next group as soon as it is ready. The kernel supplies the tiles
+// epilogues run concurrently; the first thread of warp 16 + s issues slot s's
+// MMAs, each group as soon as it is ready. The kernel supplies the tiles
 // (producers: X(t) into buffer t % kNX, then one arrival on x_full) and takes
 // the results (consumers: after p_full of slot t % 2, partial logits
 // [2][128][A] fp32, then one arrival on p_free). Each mbarrier is waited on in
@@ -82,7 +82,7 @@ struct Eng2 {
     static constexpr uint32_t kTmemCols = 512;
     static constexpr int kEpiWarps = 16;                        // two teams of 8
     static constexpr int kTeamThreads = 256;
-    static constexpr int kIssuerWarp = kEpiWarps;
+    static constexpr int kIssuerWarp = kEpiWarps;               // warps 16 and 17
     static constexpr int kOps = 3;                              // MMA groups per tile
 
     // Shared-memory state of the engine (the kernel places one instance in
@@ -95,7 +95,7 @@ struct Eng2 {
         uint64_t x_free[NX];          // tile's layer 1 complete (tcgen05.commit)
         uint64_t p_full[2];           // slot's partial logits written (one arrival per team warp)
         uint64_t p_free[2];           // slot's partials read by the consumers (1 arrival)
-        uint64_t drained;             // every MMA issued so far complete (tcgen05.commit)
+        uint64_t drained[2];          // every MMA a slot's thread issued complete (tcgen05.commit)
         uint32_t dead;                // a bounded wait expired: nobody waits any more
         __device__ void init() {
             mbar_init(&stage, 1);
@@ -109,7 +109,8 @@ struct Eng2 {
                 mbar_init(&x_full[b], 1);
                 mbar_init(&x_free[b], 1);
             }
-            mbar_init(&drained, 1);
+            mbar_init(&drained[0], 1);
+            mbar_init(&drained[1], 1);
             dead = 0u;
         }
     };
@@ -173,15 +174,25 @@ struct Eng2 {
     };
 
     // ------------------------------------------------------------------ issuer
-    // The MMA-issuing thread. Tiles are numbered t = 0, 1, ... over the whole
-    // kernel; run(n) issues every group of the next n tiles.
+    // The MMA-issuing thread of slot S (the first thread of warp 16 + S). A
+    // thread that issues tcgen05.mma is held until its MMAs have nearly
+    // completed, so each slot has its own: while one is held by its group, the
+    // other's next group is already queued on the tensor pipe, and each
+    // thread's commits track only its own MMAs. Tiles are numbered t = 0, 1,
+    // ... over the whole kernel; run(n) issues the slot's groups of tiles
+    // t .. t + n - 1 (those of its parity).
+    template <int S>
     struct Issuer {
         uint32_t t = 0;               // first tile of the next run
-        Slot sl0, sl1;
+        Slot sl;
 
-        template <int S>
-        __device__ void issue(uint8_t* smem, uint32_t x_base, uint32_t tbase, Bars& b, uint32_t tt,
-                              int op) {
+        // Group `op` of tile tt once the slot's previous group has been
+        // converted by its epilogue team and, for a tile's first group, the
+        // tile's observations are written.
+        __device__ bool group(uint8_t* smem, uint32_t x_base, uint32_t tbase, Bars& b, uint32_t tt,
+                              int op, int* err) {
+            if (sl.total > 0 && !spin(b, &b.ep_done[S], (sl.total - 1) & 1u, err)) return false;
+            if (op == 0 && !spin(b, &b.x_full[tt % NX], (tt / NX) & 1u, err)) return false;
             const uint32_t h = tbase + 256u * S, acc = h + 128u;
             const uint32_t idesc = tc::instr_desc(128, 128, 1);
             tc::fence_after_sync();
@@ -202,62 +213,33 @@ struct Eng2 {
                 tc::mma_commit(&b.x_free[buf]);                  // X(tt) is no longer read
             } else {
                 uint64_t db = tc::smem_desc(smem_u32(smem + kW2) + 2048u * (op - 1), kLboW, 128);
-#pragma unroll 4
+#pragma unroll
                 for (int k = 0; k < 16; ++k) {
                     mma_ts(acc, h + h1_col(k), db, idesc, k != 0);
                     db += (2u * kLboW) >> 4;
                 }
                 tc::mma_commit(&b.acc_full[S]);
             }
-        }
-
-        // Issues slot S's next group (op of tile tt) if it is ready: the
-        // slot's previous group has been converted by its epilogue team and,
-        // for a tile's first group, the tile's observations are written.
-        template <int S>
-        __device__ bool try_issue(uint8_t* smem, uint32_t x_base, uint32_t tbase, Bars& b, Slot& sl,
-                                  uint32_t tt, int op) {
-            if (sl.total > 0 && !mbar_test_wait(&b.ep_done[S], (sl.total - 1) & 1u)) return false;
-            if (op == 0 && !mbar_test_wait(&b.x_full[tt % NX], (tt / NX) & 1u)) return false;
-            issue<S>(smem, x_base, tbase, b, tt, op);
             ++sl.total;
             return true;
         }
 
-        // Issues every group of tiles t .. t + n - 1: slot s takes the tiles
-        // of its parity, groups 0, 1, 2 of each in order; the two slots
-        // advance independently, each as soon as its next group is ready.
         __device__ void run(uint8_t* smem, uint32_t x_base, uint32_t tbase, Bars& b, uint32_t n,
                             int* err) {
-            uint32_t tile0 = t + ((t & 1u) ? 1u : 0u), tile1 = t + ((t & 1u) ? 0u : 1u);
             const uint32_t end = t + n;
-            int op0 = 0, op1 = 0;
-            uint64_t t0 = globaltimer_ns();
-            while (tile0 < end || tile1 < end) {
-                bool any = false;
-                if (tile0 < end && try_issue<0>(smem, x_base, tbase, b, sl0, tile0, op0)) {
-                    any = true;
-                    if (++op0 == kOps) { op0 = 0; tile0 += 2; }
-                }
-                if (tile1 < end && try_issue<1>(smem, x_base, tbase, b, sl1, tile1, op1)) {
-                    any = true;
-                    if (++op1 == kOps) { op1 = 0; tile1 += 2; }
-                }
-                if (any) {
-                    t0 = globaltimer_ns();
-                } else if (is_dead(b)) {
-                    break;
-                } else if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                    mark_dead(b, err);
-                    break;
-                }
-            }
-            t += n;
+            for (uint32_t tt = t + ((t & 1u) == (uint32_t)S ? 0u : 1u); tt < end; tt += 2)
+                for (int op = 0; op < kOps; ++op)
+                    if (!group(smem, x_base, tbase, b, tt, op, err)) {
+                        t = end;
+                        return;
+                    }
+            t = end;
         }
-        // Before the tensor memory is released: every MMA issued has completed.
+        // Before the tensor memory is released: every MMA this thread issued
+        // has completed.
         __device__ void finish(Bars& b, int* err) {
-            tc::mma_commit(&b.drained);
-            if (!mbar_wait_bounded(&b.drained, 0u, kWaitLimitNs)) atomicOr(err, ERRBIT_TIMEOUT);
+            tc::mma_commit(&b.drained[S]);
+            if (!mbar_wait_bounded(&b.drained[S], 0u, kWaitLimitNs)) atomicOr(err, ERRBIT_TIMEOUT);
             tc::fence_after_sync();
         }
     };

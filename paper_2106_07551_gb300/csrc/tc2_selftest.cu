@@ -5,7 +5,7 @@
 //
 // One persistent CTA per SM, tiles of 128 rows dealt round robin; `reps`
 // repeats the row set (the same logits are written again), so a small input
-// gives a long, compute-only run. Warps 0-16 are the engine; warps 17-20
+// gives a long, compute-only run. Warps 0-17 are the engine; warps 18-21
 // convert rows to a bf16 observation tile (one row per thread) and, two tiles
 // behind, add each row's two partial logits and b3 and store them.
 #include "device_common.cuh"
@@ -17,8 +17,8 @@ namespace malib {
 
 namespace {
 
-constexpr int kThreads = 21 * 32;
-constexpr int kIoWarp = 17;
+constexpr int kThreads = 22 * 32;
+constexpr int kIoWarp = 18;
 constexpr uint32_t kLag = 2;                 // results of tile i are taken after producing tile i + 2
 
 template <int K1, int A>
@@ -72,7 +72,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ep.run(smem, tbase, bars, n, err);
     } else if (warp == E::kIssuerWarp) {
         if ((tid & 31) == 0) {
-            typename E::Issuer is;
+            typename E::template Issuer<0> is;
+            E::wait(bars, &bars.stage, 0u, err);
+            is.run(smem, smem_u32(smem + L::kX), tbase, bars, n, err);
+            is.finish(bars, err);
+        }
+    } else if (warp == E::kIssuerWarp + 1) {
+        if ((tid & 31) == 0) {
+            typename E::template Issuer<1> is;
             E::wait(bars, &bars.stage, 0u, err);
             is.run(smem, smem_u32(smem + L::kX), tbase, bars, n, err);
             is.finish(bars, err);
@@ -88,7 +95,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int buf = (int)(i % E::kNX);
                 if (i >= (uint32_t)E::kNX) E::wait(bars, &bars.x_free[buf], ((i / E::kNX) - 1) & 1u, err);
                 uint8_t* xt = smem + L::kX + buf * E::kXBytes;
-#pragma unroll 1
+#pragma unroll
                 for (int c = 0; c < K1 / 8; ++c) {
                     uint32_t w[4];
 #pragma unroll
