@@ -39,8 +39,7 @@ struct F32Layout {
 
 // bf16 tensor-core policy image (bytes): W1 [256][K1], W2 [256][256], W3 [16][256]
 // as bf16 in the core-matrix K-major layout (K1 = input width rounded up to
-// 16, rows past the output width zero), then fp32 b1[256], b2[256], b3[16], then
-// fp32 W3 [16][256] with the bf16-rounded weights (for a CUDA-core layer 3).
+// 16, rows past the output width zero), then fp32 b1[256], b2[256], b3[16].
 // Built for populations with h1 = h2 = 256, input <= 48, output <= 16.
 inline bool tc_image_shape(const int* d) {
     return d[1] == 256 && d[2] == 256 && d[0] >= 1 && d[0] <= 48 && d[3] >= 1 && d[3] <= 16;
@@ -52,7 +51,7 @@ constexpr int kLeducConstFeature = 15;
 inline bool leduc_tc_fold(int env_kind, int in) { return env_kind == MALIB_ENV_LEDUC && in == 17; }
 inline int64_t tc_image_bytes(int in) {
     const int64_t k1 = (in + 15) / 16 * 16;
-    return 256 * k1 * 2 + 256 * 256 * 2 + 16 * 256 * 2 + (256 + 256 + 16) * 4 + 16 * 256 * 4;
+    return 256 * k1 * 2 + 256 * 256 * 2 + 16 * 256 * 2 + (256 + 256 + 16) * 4;
 }
 
 // Output sums of the payoff reduction: per pair {sum r, sum r^2} as 64-bit
@@ -106,7 +105,18 @@ struct RolloutArgs {
 cudaError_t launch_kuhn_eval(const EvalArgs& a, int n_sm, cudaStream_t s);
 cudaError_t launch_kuhn_exact(const EvalArgs& a, double* out, cudaStream_t s);
 cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaStream_t s);
-cudaError_t launch_leduc_eval_tc(const EvalArgs& a, int n_sm, cudaStream_t s);
+// Work space of the tensor-core Leduc evaluation: per CTA, the state of up to
+// max_hands hands (two words each) and four queues of hand slots.
+constexpr int kLeducTcMaxHands = 16384;
+struct LeducWork {
+    uint2* hands;                // [grid][max_hands]
+    uint16_t* queues;            // [grid][2 seats][2 queues][max_hands]
+    int32_t max_hands;
+    int64_t n_seg;               // segments per pair (set by the launcher)
+};
+// Units (pair, segment) of a call and the segments per pair.
+int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n_seg_out);
+cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s);
 bool spread_tc_supported(int n_agents, int obs_dim, int n_actions, int64_t envs_per_pair);

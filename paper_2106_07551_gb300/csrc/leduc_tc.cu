@@ -2,320 +2,341 @@
 // tensor cores (Sec. 3.2 payoff table, Sec. 4.2 Monte-Carlo simulations per
 // policy combination).
 //
-// A cluster of two CTAs evaluates one pair at a time. CTA r keeps the policy of
-// seat r resident in shared memory (bf16 weight image and biases, ~146 KB);
-// the MLP's hidden activations stay in tensor memory.
-// Each CTA has 16 warps in three roles:
-//  * warps 0-7, the engine: runs 128-row tiles through the tensor-core MLP,
-//    alternating between two hand groups, and returns every row's logits;
-//  * warps 8-11 and 12-15, hand groups 0 and 1, 128 hands each. While the
-//    engine works on one group's tile, the other group samples its actions,
-//    applies them, deals new hands and publishes its next observations, so the
-//    environment work overlaps the tensor-core forward.
-// Rows 64 s .. 64 s + 63 of a group's tile in CTA r hold observations of CTA s's
-// hands acting as seat r, ranked with warp ballots (a hand beyond 64 waits a
-// step; its randomness depends only on its own ids, so deferral changes no
-// result). Observations (with a 16-byte header: rows placed, live hands) and
-// logits travel as asynchronous stores into the peer's shared memory that
-// complete transaction bytes on the receiver's mbarrier; every slot is written
-// every step (unused rows with zeros), so each receiver expects a fixed byte
-// count. A logits message whose flag is set tells a group that its hands of the
-// segment are finished in both CTAs. Both CTAs walk the same pair segments
-// (cluster c takes every n_cl-th pair); the engine restages weights when both
-// groups have finished a segment.
-// Control decisions of a role are taken by one thread and handed to the role
-// through its own barrier, so every thread of a role takes the same path.
-#include "cluster.cuh"
+// Work units are (pair, segment of at most kMaxHands hands), claimed by the
+// CTAs from a counter. A CTA plays a unit's hands all at once, in phases: in a
+// phase every live hand whose acting seat is s makes one decision, through
+// seat s's policy, which is the only policy in shared memory; phases alternate
+// between the seats (a phase without hands is skipped), and the policy is
+// restaged between them. So every tile of the tensor-core forward holds 128
+// decisions of one policy, and one policy at a time fits the shared memory
+// with the pipelined engine's buffers.
+// Hands live in global memory (a state word pair per hand, in the CTA's part
+// of the context's work space); each seat has two queues of hand slots: the
+// phase of seat s takes the current queue of s whole, hands that act next as
+// the other seat join its current queue, hands that act again as s join the
+// other queue of s, which becomes current when the phase ends (queues never
+// change while they are read). The phase of a unit's first decisions deals the
+// hands from their Philox keys.
+// Warps (7 warpgroups; setmaxnreg moves registers between them):
+//  * 0-15: the engine's epilogue teams (mlp_tc2.cuh), 16-17: its MMA threads,
+//    18-19 idle;
+//  * 20-23 producers: one row per thread, the hand's observation into a bf16
+//    tile (feature 15, constant 1, is folded into b1);
+//  * 24-27 consumers: one row per thread, the logits (two partials + b3), the
+//    masked softmax draw keyed by (episode, decision, seat), the transition,
+//    the payoff sums of finished hands, the queue of the next acting seat.
+// Every wait is bounded.
 #include "device_common.cuh"
 #include "eval_common.cuh"
 #include "internal.h"
 #include "leduc_env.cuh"
-#include "mlp_tc.cuh"
+#include "mlp_tc2.cuh"
 
 namespace malib {
 
 namespace {
 
 constexpr int kK1 = 16;                    // observation inputs after folding feature 15
-using Eng = MlpTc<kK1, 256, 16, true, /*kBarId=*/1>;
-constexpr int kThreads = 512;
-constexpr int kEngineThreads = 256;
-constexpr int kGroups = 2;
-constexpr int kSlots = 128;               // hands per group per CTA
-constexpr int kPart = 64;                 // tile rows per source CTA
-constexpr uint32_t kXBytes = Eng::kXBytes;                // one group's observation tile
-constexpr uint32_t kX = Eng::kSmemBytes;                  // X tiles [group]
-constexpr uint32_t kLg = kX + kGroups * kXBytes;          // logits [group][target][rank][4] fp32
-constexpr uint32_t kSmem = kLg + kGroups * 2 * kPart * 16;
-constexpr uint32_t kXTx = 2 * (kPart * kK1 * 2 + 16);     // rows + headers received per step
-constexpr uint32_t kLgTx = 2 * kPart * 16;                // logits received per step
-constexpr uint32_t kDoneFlag = 0x3f800000u;               // 1.0f in a logits row's 4th word
+using E = Eng2<kK1, 3, 3, 8>;
+constexpr int kWarps = 28;
+constexpr int kThreads = 32 * kWarps;
+constexpr int kProdWarp = 20, kConsWarp = 24;
 constexpr int kMaxDec = 8;
-static_assert(kX % 16 == 0 && kLg % 16 == 0, "16-byte aligned tiles");
+constexpr uint32_t kX = (E::kImage + 1023u) / 1024u * 1024u;     // X tiles
+constexpr uint32_t kP = kX + E::kNX * E::kXBytes;                  // partial logits
+constexpr uint32_t kSmem = kP + 2 * E::kPBytes;
+static_assert(kSmem <= 227 * 1024, "fits one CTA's shared memory");
 
-__device__ __forceinline__ void cluster_barrier_all() {
-    asm volatile("barrier.cluster.arrive.release.aligned;\n"
-                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+// A hand in global memory: cards, round, raises, actions this round, actor,
+// decisions so far (x) and both contributions (y).
+__device__ __forceinline__ uint2 pack(const LeducHand& h, int t) {
+    uint2 w;
+    w.x = (uint32_t)h.c0 | ((uint32_t)h.c1 << 4) | ((uint32_t)h.pub << 8) | ((uint32_t)h.round << 12) |
+          ((uint32_t)h.raises << 13) | ((uint32_t)h.nact << 15) | ((uint32_t)h.actor << 17) |
+          ((uint32_t)t << 18);
+    w.y = (uint32_t)h.con0 | ((uint32_t)h.con1 << 8);
+    return w;
+}
+__device__ __forceinline__ void unpack(uint2 w, LeducHand& h, int& t) {
+    h.c0 = (int)(w.x & 15u);
+    h.c1 = (int)((w.x >> 4) & 15u);
+    h.pub = (int)((w.x >> 8) & 15u);
+    h.round = (int)((w.x >> 12) & 1u);
+    h.raises = (int)((w.x >> 13) & 3u);
+    h.nact = (int)((w.x >> 15) & 3u);
+    h.actor = (int)((w.x >> 17) & 1u);
+    t = (int)((w.x >> 18) & 15u);
+    h.con0 = (int)(w.y & 255u);
+    h.con1 = (int)((w.y >> 8) & 255u);
+    h.done = 0;
+    h.payoff = 0;
 }
 
-__device__ __forceinline__ void group_sync(int g) {
-    if (g == 0) asm volatile("bar.sync 2, 128;" ::: "memory");
-    else asm volatile("bar.sync 3, 128;" ::: "memory");
+struct Ctl {                   // per-CTA control words (shared memory)
+    int64_t unit;              // claimed unit, or -1 when none is left
+    int pair, p0, p1, ok;
+    int64_t e_lo;              // first hand of the unit
+    int n;                     // hands of the unit
+    int cur[2];                // current queue of each seat (0 or 1)
+    int len[2][2];             // [seat][queue] entries
+    int seat;                  // seat of the current phase
+    int first;                 // 1 in the unit's first phase (hands are dealt)
+    int staged;                // policy id in shared memory (-1: none)
+    uint32_t stagings;         // policies staged so far (stage barrier phase)
+};
+
+// What every role needs of the current phase.
+struct Phase {
+    int pair, s, n;
+    int64_t e_lo;
+    uint32_t tile;             // the phase's first tile (over the whole kernel)
+    uint32_t nt;               // tiles of the phase
+    bool first;                // hands are dealt in this phase
+    const uint16_t* qin;       // queue read by the phase (not used when first)
+};
+
+// The unit and phase loop, run by every role in its own copy (each copy
+// compiled within its warpgroup's register budget); all copies pass the same
+// CTA barriers in the same order. on_phase(ph) does the role's share of a
+// phase, on_stage() its work after a new policy has landed, on_unit(sums)
+// adds the unit's payoff sums (consumers hold them; the others add zeros).
+template <class OnPhase, class OnStage>
+__device__ __forceinline__ void drive(const EvalArgs& a, const LeducWork& w, E::Bars& bars, Ctl& ctl,
+                                      uint8_t* smem, OnPhase&& on_phase, OnStage&& on_stage,
+                                      long long* sums) {
+    const int tid = threadIdx.x;
+    const int64_t n_seg = w.n_seg;
+    const int64_t n_units = (int64_t)a.n_pairs * n_seg;
+    uint16_t* q_base = w.queues + (size_t)blockIdx.x * 4 * w.max_hands;   // [seat][queue][max_hands]
+    uint32_t tile = 0;
+    while (true) {
+        __syncthreads();                         // ctl of the previous unit is read by all
+        if (tid == 0) {
+            const int64_t u = (int64_t)atomicAdd(a.work, 1ull);
+            ctl.unit = u < n_units ? u : -1;
+            if (u < n_units) {
+                const int pair = (int)(u / n_seg);
+                const int64_t seg = u % n_seg;
+                const int64_t per = (a.n_episodes + n_seg - 1) / n_seg;
+                ctl.pair = pair;
+                ctl.e_lo = seg * per;
+                const int64_t hi = min(a.n_episodes, ctl.e_lo + per);
+                ctl.n = (int)max((int64_t)0, hi - ctl.e_lo);
+                ctl.p0 = a.pairs[2 * pair];
+                ctl.p1 = a.pairs[2 * pair + 1];
+                ctl.ok = pair_ok(a, ctl.p0, ctl.p1) ? 1 : 0;
+                if (!ctl.ok && seg == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
+                ctl.cur[0] = ctl.cur[1] = 0;
+                ctl.len[0][0] = ctl.n;          // seat 0 acts first in every hand
+                ctl.len[0][1] = ctl.len[1][0] = ctl.len[1][1] = 0;
+                ctl.seat = 0;
+                ctl.first = 1;
+            }
+        }
+        __syncthreads();
+        if (ctl.unit < 0) break;
+        if (!ctl.ok || ctl.n == 0) continue;
+        sums[0] = sums[1] = sums[2] = 0;
+        while (true) {
+            const int s = ctl.seat;
+            const int n = ctl.len[s][ctl.cur[s]];
+            if (n == 0 && ctl.len[s ^ 1][ctl.cur[s ^ 1]] == 0) break;   // the unit is done
+            const int pol = s == 0 ? ctl.p0 : ctl.p1;
+            const bool restage = n > 0 && pol != ctl.staged;
+            if (restage) {
+                // every MMA and epilogue read of the previous policy is done (the
+                // previous phase ended with a CTA barrier); ctl is written again
+                // only after the next CTA barrier
+                if (tid == 0) E::stage(smem, reinterpret_cast<const uint8_t*>(a.arena + a.pol_offset[pol]), bars);
+                E::wait(bars, &bars.stage, ctl.stagings & 1u, a.err);
+                on_stage();
+            }
+            if (n > 0) {
+                Phase ph;
+                ph.pair = ctl.pair;
+                ph.s = s;
+                ph.n = n;
+                ph.e_lo = ctl.e_lo;
+                ph.tile = tile;
+                ph.nt = (uint32_t)((n + 127) / 128);
+                ph.first = ctl.first != 0;
+                ph.qin = q_base + (size_t)(2 * s + ctl.cur[s]) * w.max_hands;
+                on_phase(ph);
+                tile += ph.nt;
+            }
+            __syncthreads();                     // every role has finished the phase
+            if (tid == 0) {
+                if (restage) {
+                    ctl.staged = pol;
+                    ++ctl.stagings;
+                }
+                if (n > 0) {
+                    ctl.len[s][ctl.cur[s]] = 0;  // the queue just read is empty
+                    ctl.cur[s] ^= 1;             // hands that act again as s
+                    ctl.first = 0;
+                }
+                ctl.seat = s ^ 1;
+            }
+            __syncthreads();
+            if (E::is_dead(bars)) break;
+        }
+        block_add_sums(sums[0], sums[1], sums[2], a.acc + 2 * ctl.pair, a.n_dec);
+        if (E::is_dead(bars)) break;
+    }
 }
 
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-    leduc_eval_tc_kernel(EvalArgs a) {
-    extern __shared__ __align__(128) uint8_t smem[];
-    __shared__ __align__(8) uint64_t stage_bar;
-    __shared__ __align__(8) uint64_t mma_bar[2];
-    __shared__ __align__(8) uint64_t x_bar[kGroups];    // a group's rows and headers
-    __shared__ __align__(8) uint64_t lg_bar[kGroups];   // a group's logits
-    __shared__ __align__(8) uint64_t h1_bar[kGroups][2];  // h1 of a group's tile stored ([0] used)
-    __shared__ __align__(16) uint4 hdr[kGroups][2];     // [group][source CTA]: {rows here, live}
+// The CTA's last barrier (every MMA has completed: the MMA threads waited for
+// their last commits), then warp 0 releases the tensor memory. Called at the
+// end of every role's branch, inside its register budget.
+__device__ __forceinline__ void end_cta(uint32_t tbase) {
+    tc::fence_before_sync();
+    __syncthreads();
+    if ((threadIdx.x >> 5) == 0) tc::tmem_dealloc(tbase, E::kTmemCols);
+}
+
+__global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, LeducWork w) {
+    extern __shared__ __align__(1024) uint8_t smem[];
+    __shared__ E::Bars bars;
+    __shared__ Ctl ctl;
     __shared__ uint32_t tmem_base;
-    __shared__ uint32_t dead_s;                         // a bounded wait expired
-    __shared__ uint32_t eng_flag[2];                    // engine: 0 run, 1 group done, 2 stop
-                                                        // (two slots, used alternately)
-    __shared__ uint32_t grp_flag[kGroups];              // group: 0 logits, 1 segment done, 2 stop
-    __shared__ int wcnt[kGroups][2][4];                 // [group][seat][warp of the group]
-    __shared__ unsigned long long next_k[kGroups];
-    __shared__ long long red[kGroups][3][4];
-
-    float* lgbuf = reinterpret_cast<float*>(smem + kLg);
-    const uint32_t me = cl::rank();
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wg = warp >> 2;
 
     if (tid == 0) {
-        dead_s = 0u;
-        mbar_init(&stage_bar, 1);
-        mbar_init(&mma_bar[0], 1);
-        mbar_init(&mma_bar[1], 1);
-        for (int g = 0; g < kGroups; ++g) {
-            mbar_init(&x_bar[g], 1);
-            mbar_init(&lg_bar[g], 1);
-            mbar_init(&h1_bar[g][0], 1);
-            mbar_init(&h1_bar[g][1], 1);
-            mbar_arrive_expect_tx(&x_bar[g], kXTx);         // armed for the first step
-            mbar_arrive_expect_tx(&lg_bar[g], kLgTx);
-        }
+        bars.init();
+        ctl.staged = -1;
+        ctl.stagings = 0;
     }
     if (warp == 0) {
-        tc::tmem_alloc(&tmem_base, Eng::kTmemCols);
+        tc::tmem_alloc(&tmem_base, E::kTmemCols);
         tc::tmem_relinquish();
     }
-    for (uint32_t i = tid * 16; i < kGroups * kXBytes; i += kThreads * 16)
-        *reinterpret_cast<uint4*>(smem + kX + i) = make_uint4(0, 0, 0, 0);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
-    cluster_barrier_all();          // peers' barriers exist before any remote store
     const uint32_t tbase = tmem_base;
+    long long sums[3] = {0, 0, 0};
+    auto nothing = [] {};
 
-    // Work units: a pair's hands, cut into `parts` pieces when there are fewer
-    // pairs than clusters. Cluster c takes units c, c + n_cl, ...: strided, so
-    // that its pairs come from every row and column of the table (neighbouring
-    // pairs share a policy and so have similar game lengths; contiguous ranges
-    // left clusters with 10 % more work than others).
-    const int64_t n_cl = gridDim.x / 2, cid = blockIdx.x / 2;
-    const int64_t parts = a.n_pairs >= n_cl ? 1 : (n_cl + a.n_pairs - 1) / a.n_pairs;
-    const int64_t chunk = (a.n_episodes + parts - 1) / parts;
-    const int64_t n_units = (int64_t)a.n_pairs * parts;
-
-    if (warp < 8) {
-        // ------------------------------------------------------------ engine
-        uint32_t stage_par = 0, mma_par = 0, x_bits = 0;      // x_bar parity of group g: bit g
-        bool stop = false;
-        for (int64_t u = cid; u < n_units && !stop; u += n_cl) {
-            const int pair = (int)(u % a.n_pairs);
-            const int64_t e_lo = (u / a.n_pairs) * chunk;
-            const int64_t e_hi = min(a.n_episodes, e_lo + chunk);
-            if (e_lo >= e_hi) continue;                     // the hand groups skip it too
-            const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
-            if (!pair_ok(a, p0, p1)) continue;             // the hand groups skip it too
-            const float* policy = a.arena + a.pol_offset[me == 0 ? p0 : p1];
-            if (tid == 0) {
-                fence_proxy_async_smem();
-                mbar_arrive_expect_tx(&stage_bar, Eng::kStageBytes);
-                for (uint32_t off = 0; off < Eng::kStageBytes; off += 32768u)
-                    bulk_g2s(smem + off, reinterpret_cast<const uint8_t*>(policy) + off,
-                             min(32768u, Eng::kStageBytes - off), &stage_bar);
-            }
-            if (!mbar_wait_bounded(&stage_bar, stage_par, kWaitLimitNs) && tid == 0)
-                atomicOr(a.err, ERRBIT_TIMEOUT);
-            stage_par ^= 1u;
-            tc::fence_before_sync();
-            Eng::sync();
-            uint32_t done_bits = 0, fslot = 0;
-            while (done_bits != 3u && !stop) {
-                for (int g = 0; g < kGroups && !stop; ++g) {
-                    if (done_bits & (1u << g)) continue;
-                    if (tid == 0) {
-                        if (!dead_s && !cl::wait_cluster_bounded(&x_bar[g], (x_bits >> g) & 1u,
-                                                                 kWaitLimitNs)) {
-                            dead_s = 1u;
-                            atomicOr(a.err, ERRBIT_TIMEOUT);
-                        }
-                        mbar_arrive_expect_tx(&x_bar[g], kXTx);   // armed for the group's next step
-                        eng_flag[fslot] = dead_s ? 2u : ((hdr[g][0].y | hdr[g][1].y) == 0 ? 1u : 0u);
-                    }
-                    x_bits ^= 1u << g;
-                    Eng::sync();
-                    // a slot is rewritten two decisions later, after the next one's
-                    // barrier, which every thread passes only once it has read it
-                    const uint32_t f = eng_flag[fslot];
-                    fslot ^= 1u;
-                    if (f == 2u) { stop = true; break; }
-                    if (f == 1u) {
-                        // no live hand of the group in either CTA: tell both sources
-                        done_bits |= 1u << g;
-                        if (tid < 128) {
-                            const uint32_t src = (uint32_t)(tid / kPart);
-                            float* dst = lgbuf + ((g * 2 + (int)me) * kPart + tid % kPart) * 4;
-                            cl::st_async_v4(cl::map(dst, src), make_uint4(0, 0, 0, kDoneFlag),
-                                            cl::map(&lg_bar[g], src));
-                        }
-                        continue;
-                    }
-                    Eng::forward(smem, nullptr, tbase, mma_bar, mma_par, a.err,
-                                 [&](int r, const float* lg) {
-                                     const uint32_t src = (uint32_t)(r / kPart);
-                                     float* dst = lgbuf + ((g * 2 + (int)me) * kPart + r % kPart) * 4;
-                                     cl::st_async_v4(cl::map(dst, src),
-                                                     make_uint4(__float_as_uint(lg[0]),
-                                                                __float_as_uint(lg[1]),
-                                                                __float_as_uint(lg[2]), 0u),
-                                                     cl::map(&lg_bar[g], src));
-                                 },
-                                 smem_u32(smem + kX + g * kXBytes), /*x_published=*/true, h1_bar[g]);
-                }
-            }
+    if (wg < 4) {
+        // ---- epilogue teams (warps 0-7 slot 0, 8-15 slot 1)
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 80;" ::: "memory");
+        if (warp < 8) {
+            E::Epilogue<0> ep;
+            ep.p_base_off = kP;
+            drive(a, w, bars, ctl, smem, [&](const Phase& ph) { ep.run(smem, tbase, bars, ph.nt, a.err); },
+                  [&] { ep.init(smem); }, sums);
+        } else {
+            E::Epilogue<1> ep;
+            ep.p_base_off = kP;
+            drive(a, w, bars, ctl, smem, [&](const Phase& ph) { ep.run(smem, tbase, bars, ph.nt, a.err); },
+                  [&] { ep.init(smem); }, sums);
         }
-    } else {
-        // ------------------------------------------------------------ hand groups
-        const int g = (warp - 8) >> 2;                 // 0 or 1
-        const int lt = tid - kEngineThreads - g * kSlots;
-        const int gw = (warp - 8) & 3;                  // warp within the group
-        uint32_t lg_par = 0, h1_par = 0;
-        uint8_t* xg = smem + kX + g * kXBytes;
-        bool stop = false;
-        for (int64_t u = cid; u < n_units && !stop; u += n_cl) {
-            const int pair = (int)(u % a.n_pairs);
-            const int64_t e_lo = (u / a.n_pairs) * chunk;
-            const int64_t e_hi = min(a.n_episodes, e_lo + chunk);
-            if (e_lo >= e_hi) continue;                 // same decision in every role of both CTAs
-            const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
-            if (!pair_ok(a, p0, p1)) {                  // same decision in every role of both CTAs
-                if (tid == kEngineThreads && me == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
-                continue;
-            }
-            // this group's hands: e = e_lo + me + 2 g + 4 k
-            LeducHand h;
-            int64_t e = e_lo + me + 2 * g + 4 * (int64_t)lt;
-            bool live = e < e_hi;
-            uint64_t gid = 0;
-            int t = 0;
-            long long s1 = 0, s2 = 0, nd = 0;
-            if (live) {
-                gid = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
-                leduc_deal(h, gid, a.seed);
-            }
-            if (lt == 0) next_k[g] = kSlots;
-            while (true) {
-                // rank this group's live hands by acting seat
-                const int seat = live ? h.actor : -1;
-                const unsigned b0 = __ballot_sync(0xffffffffu, seat == 0);
-                const unsigned b1 = __ballot_sync(0xffffffffu, seat == 1);
-                if (lane == 0) { wcnt[g][0][gw] = __popc(b0); wcnt[g][1][gw] = __popc(b1); }
-                group_sync(g);
-                int pre = 0, c0 = 0, c1 = 0;
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    c0 += wcnt[g][0][w];
-                    c1 += wcnt[g][1][w];
-                    if (w < gw) pre += seat == 1 ? wcnt[g][1][w] : wcnt[g][0][w];
-                }
-                const unsigned mine = seat == 1 ? b1 : b0;
-                const int rank = pre + __popc(mine & ((1u << lane) - 1u));
-                const bool placed = live && rank < kPart;
-                float ob[17];
-                float u = 0.f;
-                if (placed) {
+        end_cta(tbase);
+    } else if (wg == 4) {
+        // ---- the MMA threads (warps 16, 17); warps 18-19 idle
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 56;" ::: "memory");
+        if (warp == 16) {
+            E::Issuer<0> is;
+            drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
+                if (lane == 0) is.run(smem, smem_u32(smem + kX), tbase, bars, ph.nt, a.err);
+            }, nothing, sums);
+            if (lane == 0) is.finish(bars, a.err);
+        } else if (warp == 17) {
+            E::Issuer<1> is;
+            drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
+                if (lane == 0) is.run(smem, smem_u32(smem + kX), tbase, bars, ph.nt, a.err);
+            }, nothing, sums);
+            if (lane == 0) is.finish(bars, a.err);
+        } else {
+            drive(a, w, bars, ctl, smem, [](const Phase&) {}, nothing, sums);
+        }
+        end_cta(tbase);
+    } else if (wg == 5) {
+        // ---- producers: observation rows, one per thread
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 48;" ::: "memory");
+        const int r = tid - kProdWarp * 32;
+        const uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
+        drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
+            for (uint32_t i = 0; i < ph.nt; ++i) {
+                const uint32_t T = ph.tile + i;
+                const int buf = (int)(T % E::kNX);
+                if (T >= (uint32_t)E::kNX) E::wait(bars, &bars.x_free[buf], ((T / E::kNX) - 1) & 1u, a.err);
+                uint8_t* xt = smem + kX + buf * E::kXBytes;
+                const int idx = (int)i * 128 + r;
+                uint32_t wv[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+                if (idx < ph.n) {
+                    const int slot = ph.first ? idx : (int)ph.qin[idx];
+                    LeducHand h;
+                    int t;
+                    if (ph.first) {
+                        leduc_deal(h, (uint64_t)ph.pair * (uint64_t)a.n_episodes + (uint64_t)(ph.e_lo + slot), a.seed);
+                        t = 0;
+                    } else {
+                        unpack(hands[slot], h, t);
+                    }
+                    float ob[17];
                     leduc_obs(h, ob);
-                    uint32_t w[8];
 #pragma unroll
-                    for (int i = 0; i < 7; ++i) w[i] = tc::pack_bf16(ob[2 * i], ob[2 * i + 1]);
-                    w[7] = tc::pack_bf16(ob[14], ob[16]);   // feature 15 is folded into b1
-                    const uint32_t bar = cl::map(&x_bar[g], (uint32_t)seat);
-#pragma unroll
-                    for (int c = 0; c < 2; ++c)
-                        cl::st_async_v4(cl::map(xg + Eng::x_offset((int)me * kPart + rank, 8 * c),
-                                                (uint32_t)seat),
-                                        make_uint4(w[4 * c], w[4 * c + 1], w[4 * c + 2], w[4 * c + 3]),
-                                        bar);
+                    for (int q = 0; q < 7; ++q) wv[q] = tc::pack_bf16(ob[2 * q], ob[2 * q + 1]);
+                    wv[7] = tc::pack_bf16(ob[14], ob[16]);   // feature 15 is folded into b1
                 }
-                {   // every unused slot of this CTA's part of both tiles gets zeros
-                    const int tgt = lt / kPart, rk = lt % kPart;
-                    if (rk >= min(tgt == 0 ? c0 : c1, kPart)) {
-                        const uint32_t bar = cl::map(&x_bar[g], (uint32_t)tgt);
+                *reinterpret_cast<uint4*>(xt + E::x_offset(r, 0)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                *reinterpret_cast<uint4*>(xt + E::x_offset(r, 8)) = make_uint4(wv[4], wv[5], wv[6], wv[7]);
+                fence_proxy_async_smem();
+                asm volatile("bar.sync 2, 128;" ::: "memory");
+                if (r == 0) mbar_arrive_release(&bars.x_full[buf]);
+            }
+        }, nothing, sums);
+        end_cta(tbase);
+    } else {
+        // ---- consumers: draw, transition, sums, next queue; one row per thread
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 80;" ::: "memory");
+        const int r = tid - kConsWarp * 32;
+        uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
+        uint16_t* q_base = w.queues + (size_t)blockIdx.x * 4 * w.max_hands;
+        drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
+            const float* b3 = reinterpret_cast<const float*>(smem + E::kB3);
+            const int s = ph.s;
+            for (uint32_t i = 0; i < ph.nt; ++i) {
+                const uint32_t T = ph.tile + i;
+                const int sl = (int)(T & 1u);
+                E::wait(bars, &bars.p_full[sl], (T >> 1) & 1u, a.err);
+                const float* pp = reinterpret_cast<const float*>(smem + kP + sl * E::kPBytes);
+                const int idx = (int)i * 128 + r;
+                float lg[3] = {0.f, 0.f, 0.f};
+                if (idx < ph.n) {
 #pragma unroll
-                        for (int c = 0; c < 2; ++c)
-                            cl::st_async_v4(cl::map(xg + Eng::x_offset((int)me * kPart + rk, 8 * c),
-                                                    (uint32_t)tgt),
-                                            make_uint4(0, 0, 0, 0), bar);
+                    for (int q = 0; q < 3; ++q)
+                        lg[q] = __fadd_rn(__fadd_rn(pp[r * 3 + q], pp[(128 + r) * 3 + q]), b3[q]);
+                }
+                asm volatile("bar.sync 3, 128;" ::: "memory");
+                if (r == 0) mbar_arrive_release(&bars.p_free[sl]);
+                int next = -1, slot = 0;
+                if (idx < ph.n) {
+                    slot = ph.first ? idx : (int)ph.qin[idx];
+                    LeducHand h;
+                    int t;
+                    const int64_t e = ph.e_lo + slot;
+                    const uint64_t gid = (uint64_t)ph.pair * (uint64_t)a.n_episodes + (uint64_t)e;
+                    if (ph.first) {
+                        leduc_deal(h, gid, a.seed);
+                        t = 0;
+                    } else {
+                        unpack(hands[slot], h, t);
                     }
-                }
-                if (lt < 2) {                                   // header to CTA lt
-                    const uint32_t n = (uint32_t)min(lt == 0 ? c0 : c1, kPart);
-                    cl::st_async_v4(cl::map(&hdr[g][me], (uint32_t)lt),
-                                    make_uint4(n, (uint32_t)(c0 + c1), 0, 0),
-                                    cl::map(&x_bar[g], (uint32_t)lt));
-                }
-                // the decision's uniform, drawn while the engines work
-                if (placed) u = u24(draw(gid, (uint32_t)t, (uint32_t)seat, a.seed).x);
-                // logits (or the end of the segment) from both engines. While
-                // it waits, this group's leader issues the second output half of
-                // layer 2 of the group's tile in this CTA once the engine has h1
-                // in tensor memory (the engine's own MMA thread is then free for
-                // its epilogue share); a forward needs it before it can finish.
-                // (Issuing all of layer 2 from here measured 52.4 ms against
-                // 49.4: the helper's response then delays layer 2's start.)
-                if (lt == 0) {
-                    bool pend = true;
-                    const uint64_t t0 = globaltimer_ns();
-                    while (!dead_s) {
-                        if (pend && mbar_try_wait(&h1_bar[g][0], h1_par)) {
-                            h1_par ^= 1u;
-                            pend = false;
-                            tc::fence_after_sync();
-                            Eng::issue_layer2b(smem, tbase, &mma_bar[0]);
-                        }
-                        if (cl::try_wait_cluster(&lg_bar[g], lg_par)) break;
-                        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                            dead_s = 1u;
-                            atomicOr(a.err, ERRBIT_TIMEOUT);
-                        }
-                    }
-                    mbar_arrive_expect_tx(&lg_bar[g], kLgTx);
-                    grp_flag[g] = dead_s ? 2u
-                                         : (__float_as_uint(lgbuf[(g * 2) * kPart * 4 + 3]) == kDoneFlag
-                                                ? 1u : 0u);
-                }
-                lg_par ^= 1u;
-                group_sync(g);
-                const uint32_t f = grp_flag[g];
-                if (f != 0u) { stop = f == 2u; break; }
-                if (placed) {
-                    const float* lp = lgbuf + ((g * 2 + seat) * kPart + rank) * 4;
-                    float lg[3] = {lp[0], lp[1], lp[2]};
+                    const float u = u24(draw(gid, (uint32_t)t, (uint32_t)s, a.seed).x);
                     const unsigned legal = leduc_legal(h);
                     const int act = sample_masked<3>(lg, legal, u);
                     const bool rec = e < a.n_dump;
-                    const int64_t rb = ((int64_t)pair * a.n_dump + e) * kMaxDec;
+                    const int64_t rb = ((int64_t)ph.pair * a.n_dump + e) * kMaxDec;
                     if (rec) {
                         if (a.d_obs) {
+                            float ob[17];
+                            leduc_obs(h, ob);
                             float* o = a.d_obs + (rb + t) * 20;
 #pragma unroll
-                            for (int i = 0; i < 17; ++i) o[i] = ob[i];
+                            for (int q = 0; q < 17; ++q) o[q] = ob[q];
                             o[17] = 0.f; o[18] = 0.f; o[19] = 0.f;
                         }
                         if (a.d_logits) {
@@ -330,79 +351,68 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                         if (a.d_done) a.d_done[rb + t] = h.done ? 1 : 0;
                     }
                     ++t;
-                    ++nd;
+                    ++sums[2];
                     if (h.done) {
-                        s1 += h.payoff;
-                        s2 += (long long)h.payoff * h.payoff;
+                        sums[0] += h.payoff;
+                        sums[1] += (long long)h.payoff * h.payoff;
                         if (rec) {
                             for (int k = t; k < kMaxDec; ++k) {
                                 if (a.d_obs)
-                                    for (int i = 0; i < 20; ++i) a.d_obs[(rb + k) * 20 + i] = 0.f;
+                                    for (int q = 0; q < 20; ++q) a.d_obs[(rb + k) * 20 + q] = 0.f;
                                 if (a.d_logits)
-                                    for (int i = 0; i < 3; ++i) a.d_logits[(rb + k) * 3 + i] = 0.f;
+                                    for (int q = 0; q < 3; ++q) a.d_logits[(rb + k) * 3 + q] = 0.f;
                                 if (a.d_action) a.d_action[rb + k] = 255;
                                 if (a.d_reward) a.d_reward[rb + k] = 0.f;
                                 if (a.d_done) a.d_done[rb + k] = 1;
                             }
                         }
+                    } else {
+                        hands[slot] = pack(h, t);
+                        next = h.actor;
                     }
                 }
-                // finished hands take the group's next hands: one atomic per
-                // warp, ranks within the warp from a ballot
-                const bool need = placed && h.done;
-                const unsigned nm = __ballot_sync(0xffffffffu, need);
-                if (nm != 0u) {
-                    const int leader = __ffs(nm) - 1;
-                    unsigned long long base = 0ull;
-                    if (lane == leader) base = atomicAdd(&next_k[g], (unsigned long long)__popc(nm));
+                // the hand joins the queue of its next acting seat: the other
+                // seat's current queue, or this seat's other queue
+#pragma unroll
+                for (int ns = 0; ns < 2; ++ns) {
+                    const unsigned m = __ballot_sync(0xffffffffu, next == ns);
+                    if (m == 0u) continue;
+                    const int qi = ns == s ? (ctl.cur[s] ^ 1) : ctl.cur[ns];
+                    const int leader = __ffs(m) - 1;
+                    int base = 0;
+                    if (lane == leader) base = atomicAdd(&ctl.len[ns][qi], __popc(m));
                     base = __shfl_sync(0xffffffffu, base, leader);
-                    if (need) {
-                        const int64_t k = (int64_t)(base + (unsigned long long)__popc(nm & ((1u << lane) - 1u)));
-                        e = e_lo + me + 2 * g + 4 * k;
-                        live = e < e_hi;
-                        if (live) {
-                            gid = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
-                            leduc_deal(h, gid, a.seed);
-                            t = 0;
-                        }
-                    }
+                    if (next == ns)
+                        q_base[(size_t)(2 * ns + qi) * w.max_hands + base + __popc(m & ((1u << lane) - 1u))] =
+                            (uint16_t)slot;
                 }
             }
-            // the group's payoff sums: warp shuffles, then one atomic per sum
-            s1 = warp_sum_ll(s1);
-            s2 = warp_sum_ll(s2);
-            nd = warp_sum_ll(nd);
-            if (lane == 0) { red[g][0][gw] = s1; red[g][1][gw] = s2; red[g][2][gw] = nd; }
-            group_sync(g);
-            if (lt == 0) {
-                long long t1 = 0, t2 = 0, t3 = 0;
-                for (int w = 0; w < 4; ++w) { t1 += red[g][0][w]; t2 += red[g][1][w]; t3 += red[g][2][w]; }
-                atomicAdd(a.acc + 2 * pair, (unsigned long long)t1);
-                atomicAdd(a.acc + 2 * pair + 1, (unsigned long long)t2);
-                atomicAdd(a.n_dec, (unsigned long long)t3);
-            }
-            group_sync(g);
-        }
+        }, nothing, sums);
+        end_cta(tbase);
     }
-    tc::fence_before_sync();
-    __syncthreads();
-    cluster_barrier_all();          // no peer touches this CTA's shared memory after this
-    if (warp == 0) tc::tmem_dealloc(tbase, Eng::kTmemCols);
 }
 
 }  // namespace
 
-cudaError_t launch_leduc_eval_tc(const EvalArgs& a, int n_sm, cudaStream_t s) {
+int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n_seg_out) {
+    int64_t n_seg = (n_episodes + kLeducTcMaxHands - 1) / kLeducTcMaxHands;
+    // enough units for every SM when pairs are few
+    while ((int64_t)n_pairs * n_seg < n_sm && (n_episodes + n_seg - 1) / n_seg > 256) ++n_seg;
+    *n_seg_out = n_seg;
+    return (int64_t)n_pairs * n_seg;
+}
+
+cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0) return cudaSuccess;
     cudaError_t err = cudaFuncSetAttribute(leduc_eval_tc_kernel,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (err != cudaSuccess) return err;
-    const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
-    int64_t clusters = (total + 2 * kGroups * kSlots - 1) / (2 * kGroups * kSlots);
-    const int64_t max_clusters = n_sm / 2;
-    if (clusters > max_clusters) clusters = max_clusters;
-    if (clusters < 1) clusters = 1;
-    leduc_eval_tc_kernel<<<(unsigned)(2 * clusters), kThreads, kSmem, s>>>(a);
+    int64_t n_seg = 0;
+    const int64_t units = leduc_tc_units(a.n_pairs, a.n_episodes, n_sm, &n_seg);
+    const int64_t grid = units < n_sm ? units : n_sm;
+    LeducWork ww = w;
+    ww.n_seg = n_seg;
+    leduc_eval_tc_kernel<<<(unsigned)grid, kThreads, kSmem, s>>>(a, ww);
     return cudaGetLastError();
 }
 

@@ -18,20 +18,20 @@
 //       ep: h2 = bf16(relu(ACC + b2)) is read in the mma.sync fragment layout
 //       (tcgen05.ld 16x256b) and layer 3 runs on it as warp-level MMAs
 //       (m16n8k16, W3 as the B operand, actions padded to 8), accumulating each
-//       warp's partial logits over its 128 neurons in registers; after G2 the
-//       two partials of a row go to shared memory, where the consumer adds
-//       them and b3.
+//       warp's partial logits over its neurons in registers; after G2 the
+//       partials of a row (one per warp of its lane quarter) go to shared
+//       memory, where the consumer adds them and b3.
 // Layer 3 is 0.4 % of the flops; as tcgen05 MMAs of N = 16 it cost as much
 // tensor-pipe time as half of layer 2, so it runs on the warp-level path.
 //
-// Roles: each slot has its own epilogue team of 8 warps (warps 0-7 slot 0,
-// warps 8-15 slot 1; in a team, warp w: lane quarter q = w % 4, half
-// p = (w / 4) % 2 of the columns: [64p, 64p + 64)), so the two slots'
-// epilogues run concurrently; the first thread of warp 16 + s issues slot s's
-// MMAs, each group as soon as it is ready. The kernel supplies the tiles
-// (producers: X(t) into buffer t % kNX, then one arrival on x_full) and takes
-// the results (consumers: after p_full of slot t % 2, partial logits
-// [2][128][A] fp32, then one arrival on p_free). Each mbarrier is waited on in
+// Roles: each slot has its own epilogue team of TW warps (warps TW s .. TW s +
+// TW - 1; in a team, warp w handles lane quarter w % 4 and, with TW = 8, half
+// w / 4 of the columns), so the two slots' epilogues run concurrently; the
+// first thread of warp 2 TW + s issues slot s's MMAs, each group as soon as it
+// is ready. The kernel supplies the tiles (producers: X(t) into buffer
+// t % kNX, then one arrival on x_full) and takes the results (consumers: after
+// p_full of slot t % 2, partial logits [TW / 4][128][A] fp32, then one arrival
+// on p_free). Each mbarrier is waited on in
 // strict phase order, so parities are counted, never guessed; every wait is
 // bounded (a timeout raises ERRBIT_TIMEOUT and marks the engine dead, after
 // which no role waits again).
@@ -62,9 +62,10 @@ __device__ __forceinline__ void mma_m16n8k16(float (&d)[4], const uint32_t (&a)[
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
-template <int K1, int A, int NX = 3>
+template <int K1, int A, int NX = 3, int TW = 8>
 struct Eng2 {
     static_assert(K1 % 16 == 0 && K1 <= 48 && A >= 1 && A <= 8, "shapes built");
+    static_assert(TW == 4 || TW == 8, "epilogue team of 4 or 8 warps");
     // ---- the policy in shared memory: the leading part of its global image
     // (tc_image_bytes layout), staged once
     static constexpr uint32_t kW1 = 0;                          // bf16 [256][K1], core-matrix K-major
@@ -75,14 +76,16 @@ struct Eng2 {
     static constexpr uint32_t kB3 = kB2 + 1024;                 // fp32 b3 [16]
     static constexpr uint32_t kImage = kB3 + 64;                // bytes staged
     static constexpr uint32_t kXBytes = 128u * K1 * 2;          // one observation tile
-    static constexpr uint32_t kPBytes = 2u * 128 * A * 4;       // one slot's partials [2][128][A]
+    static constexpr int kTeamWarps = TW;                       // epilogue warps per slot
+    static constexpr int kSplit = TW / 4;                       // column parts of a lane quarter
+    static constexpr uint32_t kPBytes = kSplit * 128u * A * 4;  // one slot's partials [kSplit][128][A]
     static constexpr uint32_t kLboX = 16 * 128;                 // K-chunk stride, 128 rows
     static constexpr uint32_t kLboW = 32 * 128;                 // K-chunk stride, 256 rows
     static constexpr int kNX = NX;
     static constexpr uint32_t kTmemCols = 512;
-    static constexpr int kEpiWarps = 16;                        // two teams of 8
-    static constexpr int kTeamThreads = 256;
-    static constexpr int kIssuerWarp = kEpiWarps;               // warps 16 and 17
+    static constexpr int kEpiWarps = 2 * TW;                    // two teams
+    static constexpr int kTeamThreads = 32 * TW;
+    static constexpr int kIssuerWarp = kEpiWarps;               // this warp and the next
     static constexpr int kOps = 3;                              // MMA groups per tile
 
     // Shared-memory state of the engine (the kernel places one instance in
@@ -102,7 +105,7 @@ struct Eng2 {
             for (int s = 0; s < 2; ++s) {
                 mbar_init(&acc_full[s], 1);
                 mbar_init(&ep_done[s], kTeamThreads);
-                mbar_init(&p_full[s], 8);
+                mbar_init(&p_full[s], TW);
                 mbar_init(&p_free[s], 1);
             }
             for (int b = 0; b < NX; ++b) {
@@ -245,33 +248,39 @@ struct Eng2 {
     };
 
     // --------------------------------------------------------------- epilogue
-    // One warp of slot S's epilogue team (S = warp / 8).
+    // One warp of slot S's epilogue team (S = warp / TW). Warp w of a team
+    // handles lane quarter w % 4 and the accumulator columns of its part
+    // (w / 4): 64 columns when TW = 8, all 128 (two passes of 64) when TW = 4.
     template <int S>
     struct Epilogue {
+        static constexpr int kPasses = 2 / kSplit;            // 64-column passes per group
         uint32_t t = 0;               // first tile of the next run
         Slot sl;
         uint32_t pt = 0;              // partial tiles written (all runs)
         float d[2][4];                // partial logits: [row block][m16n8 accumulator]
-        uint32_t w3[2][4][2];         // layer-3 B fragments: [L2 half][16-neuron block][b0, b1]
+        uint32_t w3[2][4][2];         // TW = 8: layer-3 B fragments [L2 half][block][b0, b1]
         uint32_t p_base_off = 0;      // byte offset of the partial buffers in shared memory
 
         __device__ static int quarter() { return (int)(threadIdx.x >> 5) & 3; }
-        __device__ static int part() { return (int)(threadIdx.x >> 7) & 1; }
+        __device__ static int part() { return kSplit == 2 ? (int)(threadIdx.x >> 7) & 1 : 0; }
 
-        // Loads this warp's W3 fragments (action g = lane / 4 of its neurons);
-        // after the policy is staged.
-        __device__ void init(const uint8_t* smem) {
+        // Layer-3 B fragment (action g = lane / 4) for the 16 neurons k0 .. k0 + 15.
+        __device__ static void w3_frag(const uint8_t* smem, int k0, uint32_t& b0, uint32_t& b1) {
             const int lane = threadIdx.x & 31, g = lane >> 2, tq = lane & 3;
+            b0 = *reinterpret_cast<const uint32_t*>(smem + kW3 + tc::cm_offset(g, k0 + 2 * tq, 16, 2));
+            b1 = *reinterpret_cast<const uint32_t*>(smem + kW3 + tc::cm_offset(g, k0 + 8 + 2 * tq, 16, 2));
+        }
+
+        // TW = 8: loads this warp's W3 fragments into registers (after the
+        // policy is staged; again after a restage).
+        __device__ void init(const uint8_t* smem) {
+            if constexpr (kSplit == 2) {
 #pragma unroll
-            for (int half = 0; half < 2; ++half)
+                for (int half = 0; half < 2; ++half)
 #pragma unroll
-                for (int kb = 0; kb < 4; ++kb)
-#pragma unroll
-                    for (int r = 0; r < 2; ++r) {
-                        const int k = 128 * half + 64 * part() + 16 * kb + 8 * r + 2 * tq;
-                        w3[half][kb][r] = *reinterpret_cast<const uint32_t*>(
-                            smem + kW3 + tc::cm_offset(g, k, 16, 2));
-                    }
+                    for (int kb = 0; kb < 4; ++kb)
+                        w3_frag(smem, 128 * half + 64 * part() + 16 * kb, w3[half][kb][0], w3[half][kb][1]);
+            }
         }
 
         // bf16(relu(v + bias)) of 32 columns (lane = row), packed in pairs.
@@ -286,43 +295,45 @@ struct Eng2 {
             }
         }
 
-        // Group 0's epilogue: h1 of this warp's 64 columns of H (neurons 128 +
-        // 64p ..) and of ACC (neurons 64p ..), packed into the columns of H it
-        // read (32-neuron block B: h1[128 + 32B ..] at H[32B, +16), h1[32B ..]
-        // at H[32B + 16, +16)).
+        // Group 0's epilogue: h1 of this warp's columns of H (neurons 128 + c ..)
+        // and of ACC (neurons c ..), packed into the columns of H it read
+        // (32-neuron block B: h1[128 + 32B ..] at H[32B, +16), h1[32B ..] at
+        // H[32B + 16, +16)).
         __device__ void serve_l1(uint8_t* smem, uint32_t tbase, Bars& b) {
             const uint32_t h = tbase + 256u * S, acc = h + 128u;
             const uint32_t lane_q = (uint32_t)(32 * quarter()) << 16;
-            const uint32_t c0 = 64u * part();
             const float* b1 = reinterpret_cast<const float*>(smem + kB1);
             tc::fence_after_sync();
             uint32_t v[32], pk[16];
 #pragma unroll
-            for (int c = 0; c < 2; ++c) {
-                tc::tmem_ld32x1(h + lane_q + c0 + 32u * c, v);
-                convert(v, b1 + 128 + c0 + 32 * c, pk);
-                tc::tmem_st16(h + lane_q + c0 + 32u * c, pk);
-            }
+            for (int ps = 0; ps < kPasses; ++ps) {
+                const uint32_t c0 = 64u * (part() * kPasses + ps);
 #pragma unroll
-            for (int c = 0; c < 2; ++c) {
-                tc::tmem_ld32x1(acc + lane_q + c0 + 32u * c, v);
-                convert(v, b1 + c0 + 32 * c, pk);
-                tc::tmem_st16(h + lane_q + c0 + 32u * c + 16u, pk);
+                for (int c = 0; c < 2; ++c) {
+                    tc::tmem_ld32x1(h + lane_q + c0 + 32u * c, v);
+                    convert(v, b1 + 128 + c0 + 32 * c, pk);
+                    tc::tmem_st16(h + lane_q + c0 + 32u * c, pk);
+                }
+#pragma unroll
+                for (int c = 0; c < 2; ++c) {
+                    tc::tmem_ld32x1(acc + lane_q + c0 + 32u * c, v);
+                    convert(v, b1 + c0 + 32 * c, pk);
+                    tc::tmem_st16(h + lane_q + c0 + 32u * c + 16u, pk);
+                }
             }
             tc::tmem_wait_st();
             tc::fence_before_sync();
             mbar_arrive_release(&b.ep_done[S]);
         }
 
-        // Group 1 + HALF's epilogue: layer 2's neurons 128 HALF + 64p .. + 64 of
-        // the 32 rows of this warp's lane quarter (two 16-row blocks), then
-        // their share of layer 3 into the partial logits d.
+        // Group 1 + HALF's epilogue: layer 2's neurons 128 HALF + c .. of the 32
+        // rows of this warp's lane quarter (two 16-row blocks), then their share
+        // of layer 3 into the partial logits d.
         template <int HALF>
         __device__ void serve_l2(uint8_t* smem, uint32_t tbase, Bars& b, int* err) {
             const int lane = threadIdx.x & 31, g = lane >> 2, tq = lane & 3;
             const uint32_t acc = tbase + 256u * S + 128u;
             const uint32_t lane_q = (uint32_t)(32 * quarter()) << 16;
-            const uint32_t c0 = 64u * part();
             tc::fence_after_sync();
             if (HALF == 0) {
 #pragma unroll
@@ -330,33 +341,44 @@ struct Eng2 {
 #pragma unroll
                     for (int i = 0; i < 4; ++i) d[rb][i] = 0.f;
             }
-            const float* b2 = reinterpret_cast<const float*>(smem + kB2) + 128 * HALF + c0;
 #pragma unroll
-            for (int rb = 0; rb < 2; ++rb)
+            for (int ps = 0; ps < kPasses; ++ps) {
+                const uint32_t c0 = 64u * (part() * kPasses + ps);
+                const float* b2 = reinterpret_cast<const float*>(smem + kB2) + 128 * HALF + c0;
 #pragma unroll
-                for (int cc = 0; cc < 2; ++cc) {
-                    uint32_t x[16];
-                    tc::tmem_ld16x256b_x4(acc + lane_q + ((uint32_t)(16 * rb) << 16) + c0 + 32u * cc, x);
-                    if (rb == 1 && cc == 1) {
-                        tc::fence_before_sync();
-                        mbar_arrive_release(&b.ep_done[S]);    // the accumulator is read
+                for (int rb = 0; rb < 2; ++rb)
+#pragma unroll
+                    for (int cc = 0; cc < 2; ++cc) {
+                        uint32_t x[16];
+                        tc::tmem_ld16x256b_x4(acc + lane_q + ((uint32_t)(16 * rb) << 16) + c0 + 32u * cc, x);
+                        if (ps == kPasses - 1 && rb == 1 && cc == 1) {
+                            tc::fence_before_sync();
+                            mbar_arrive_release(&b.ep_done[S]);    // the accumulator is read
+                        }
+#pragma unroll
+                        for (int kh = 0; kh < 2; ++kh) {
+                            // 16-neuron block kb of these 64: this thread's columns
+                            // 16 kb + 2 tq (+1) and 16 kb + 8 + 2 tq (+1)
+                            const int kb = 2 * cc + kh;
+                            const float2 bl = *reinterpret_cast<const float2*>(b2 + 16 * kb + 2 * tq);
+                            const float2 bh = *reinterpret_cast<const float2*>(b2 + 16 * kb + 8 + 2 * tq);
+                            const uint32_t* xx = x + 8 * kh;
+                            uint32_t a[4];
+                            a[0] = tc::bias_relu_bf16x2(__uint_as_float(xx[0]), __uint_as_float(xx[1]), bl.x, bl.y);
+                            a[1] = tc::bias_relu_bf16x2(__uint_as_float(xx[2]), __uint_as_float(xx[3]), bl.x, bl.y);
+                            a[2] = tc::bias_relu_bf16x2(__uint_as_float(xx[4]), __uint_as_float(xx[5]), bh.x, bh.y);
+                            a[3] = tc::bias_relu_bf16x2(__uint_as_float(xx[6]), __uint_as_float(xx[7]), bh.x, bh.y);
+                            uint32_t b0, b1;
+                            if constexpr (kSplit == 2) {
+                                b0 = w3[HALF][kb][0];
+                                b1 = w3[HALF][kb][1];
+                            } else {
+                                w3_frag(smem, 128 * HALF + (int)c0 + 16 * kb, b0, b1);
+                            }
+                            mma_m16n8k16(d[rb], a, b0, b1);
+                        }
                     }
-#pragma unroll
-                    for (int kh = 0; kh < 2; ++kh) {
-                        // 16-neuron block kb of the warp's 64: this thread's columns
-                        // 16 kb + 2 tq (+1) and 16 kb + 8 + 2 tq (+1)
-                        const int kb = 2 * cc + kh;
-                        const float2 bl = *reinterpret_cast<const float2*>(b2 + 16 * kb + 2 * tq);
-                        const float2 bh = *reinterpret_cast<const float2*>(b2 + 16 * kb + 8 + 2 * tq);
-                        const uint32_t* xx = x + 8 * kh;
-                        uint32_t a[4];
-                        a[0] = tc::bias_relu_bf16x2(__uint_as_float(xx[0]), __uint_as_float(xx[1]), bl.x, bl.y);
-                        a[1] = tc::bias_relu_bf16x2(__uint_as_float(xx[2]), __uint_as_float(xx[3]), bl.x, bl.y);
-                        a[2] = tc::bias_relu_bf16x2(__uint_as_float(xx[4]), __uint_as_float(xx[5]), bh.x, bh.y);
-                        a[3] = tc::bias_relu_bf16x2(__uint_as_float(xx[6]), __uint_as_float(xx[7]), bh.x, bh.y);
-                        mma_m16n8k16(d[rb], a, w3[HALF][kb][0], w3[HALF][kb][1]);
-                    }
-                }
+            }
             if (HALF == 1) {
                 // partials of this warp's neurons: rows 32 q + 16 rb + g (+ 8),
                 // actions 2 tq, 2 tq + 1

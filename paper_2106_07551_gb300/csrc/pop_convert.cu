@@ -8,11 +8,9 @@
 //   kind 2, bf16 tensor-core image: W1 [256][K1], W2 [256][256], W3 [16][256] as
 //                   bf16 in the core-matrix K-major layout (8 rows x 16 bytes per
 //                   core matrix, row groups 128 B apart, K chunks rows x 16 B
-//                   apart), then fp32 b1 [256], b2 [256], b3 [16], then W3 again
-//                   as fp32 [16][256] holding the bf16-rounded weights (rows
-//                   past the output width zero: the CUDA-core layer 3 of the
-//                   pipelined engine reads these); with the fold flag, input 15
-//                   (constant 1) is dropped and its bf16 weight added to b1.
+//                   apart), then fp32 b1 [256], b2 [256], b3 [16]; with the fold
+//                   flag, input 15 (constant 1) is dropped and its bf16 weight
+//                   added to b1.
 // Every destination word is computed by one thread from its source values, so
 // the image is the same whatever the launch shape. bf16 rounding is to
 // nearest even on the bit pattern; infinities and NaNs keep their high half.
@@ -87,11 +85,7 @@ __device__ uint32_t tc_word(const float* p, const int* d, bool fold, int64_t i) 
         float v;
         if (j < 256) v = fold ? __fadd_rn(b1[j], bf16_value(W1[j * in + kLeducConstFeature])) : b1[j];
         else if (j < 512) v = b2[j - 256];
-        else if (j < 528) v = j - 512 < a ? b3[j - 512] : 0.f;
-        else {
-            const int64_t w = j - 528, row = w / 256, k = w % 256;
-            v = row < a ? bf16_value(W3[row * 256 + k]) : 0.f;
-        }
+        else v = j - 512 < a ? b3[j - 512] : 0.f;
         return __float_as_uint(v);
     }
     // byte offset o inside the region -> (row, k) of its low half

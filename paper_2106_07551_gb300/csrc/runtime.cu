@@ -61,6 +61,8 @@ struct malib_ctx {
     int64_t out_cap = 0;
     uint8_t* scratch = nullptr;        // solver work space (LP tableaus that do not fit on chip)
     int64_t scratch_cap = 0;
+    uint8_t* lwork = nullptr;          // tensor-core Leduc evaluation: hand states and queues
+    int64_t lwork_cap = 0;
 
     int64_t launches = 0;
     bool timing = false;
@@ -374,6 +376,7 @@ void malib_destroy(malib_ctx* c) {
     cudaFree(c->d_pairs);
     cudaFree(c->d_out);
     cudaFree(c->scratch);
+    cudaFree(c->lwork);
     cudaFree(c->d_stage);
     cudaFree(c->d_jobs);
     delete c;
@@ -622,7 +625,18 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
         if (kind == MALIB_ENV_KUHN) {
             CK(launch_kuhn_eval(a, c->n_sm, c->stream), "Kuhn eval kernel");
         } else if (leduc_tc) {
-            CK(launch_leduc_eval_tc(a, c->n_sm, c->stream), "Leduc tensor-core eval kernel");
+            int64_t n_seg = 0;
+            const int64_t units = leduc_tc_units(n_pairs, n_episodes, c->n_sm, &n_seg);
+            const int64_t grid = std::min<int64_t>(units, c->n_sm);
+            const int64_t per = (n_episodes + n_seg - 1) / n_seg;
+            LeducWork lw{};
+            lw.max_hands = (int32_t)std::min<int64_t>(per, kLeducTcMaxHands);
+            // per CTA: 8 bytes of state and 4 two-byte queue entries per hand
+            if ((r = ensure(c, c->lwork, c->lwork_cap, grid * lw.max_hands * 16, "Leduc work space")) != MALIB_OK)
+                return r;
+            lw.hands = reinterpret_cast<uint2*>(c->lwork);
+            lw.queues = reinterpret_cast<uint16_t*>(c->lwork + grid * lw.max_hands * 8);
+            CK(launch_leduc_eval_tc(a, lw, c->n_sm, c->stream), "Leduc tensor-core eval kernel");
         } else {
             CK(launch_leduc_eval_f32(a, c->dims[1], c->n_sm, c->stream), "Leduc eval kernel");
         }

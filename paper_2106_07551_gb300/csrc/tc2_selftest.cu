@@ -5,9 +5,10 @@
 //
 // One persistent CTA per SM, tiles of 128 rows dealt round robin; `reps`
 // repeats the row set (the same logits are written again), so a small input
-// gives a long, compute-only run. Warps 0-17 are the engine; warps 18-21
-// convert rows to a bf16 observation tile (one row per thread) and, two tiles
-// behind, add each row's two partial logits and b3 and store them.
+// gives a long, compute-only run. The engine's warps come first (two
+// epilogue teams of kTW warps, two MMA warps); the last four warps convert
+// rows to a bf16 observation tile (one row per thread) and, two tiles behind,
+// add each row's partial logits and b3 and store them.
 #include "device_common.cuh"
 #include "internal.h"
 #include "malib.h"
@@ -17,13 +18,14 @@ namespace malib {
 
 namespace {
 
-constexpr int kThreads = 22 * 32;
-constexpr int kIoWarp = 18;
+constexpr int kTW = 8;                       // epilogue warps per slot
+constexpr int kIoWarp = 4 * kTW / 2 + 2;     // after both teams and the two MMA warps
+constexpr int kThreads = (kIoWarp + 4) * 32;
 constexpr uint32_t kLag = 2;                 // results of tile i are taken after producing tile i + 2
 
 template <int K1, int A>
 struct ProbeLayout {
-    using E = Eng2<K1, A>;
+    using E = Eng2<K1, A, 3, kTW>;
     static constexpr uint32_t kX = (E::kImage + 1023u) / 1024u * 1024u;
     static constexpr uint32_t kP = kX + E::kNX * E::kXBytes;
     static constexpr uint32_t kSmem = kP + 2 * E::kPBytes;
@@ -35,7 +37,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mlp_tc2_probe_kernel(const float* __restrict__ arena, const int64_t* __restrict__ pol_offset,
                          int32_t pid, const float* __restrict__ x,
                          int in, int64_t n_rows, int32_t reps, float* __restrict__ out, int* err) {
-    using E = Eng2<K1, A>;
+    using E = Eng2<K1, A, 3, kTW>;
     using L = ProbeLayout<K1, A>;
     extern __shared__ __align__(1024) uint8_t smem[];
     __shared__ typename E::Bars bars;
@@ -58,7 +60,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int64_t tiles = row_tiles * reps;
     const uint32_t n = (uint32_t)((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);
 
-    if (warp < 8) {
+    if (warp < kTW) {
         typename E::template Epilogue<0> ep;
         ep.p_base_off = L::kP;
         E::wait(bars, &bars.stage, 0u, err);
@@ -124,8 +126,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float* p = reinterpret_cast<const float*>(smem + L::kP + sl * E::kPBytes);
                 if (row < n_rows) {
 #pragma unroll
-                    for (int a = 0; a < A; ++a)
-                        out[row * A + a] = __fadd_rn(__fadd_rn(p[r * A + a], p[(128 + r) * A + a]), b3[a]);
+                    for (int a = 0; a < A; ++a) {
+                        float v = p[r * A + a];
+                        if (E::kSplit == 2) v = __fadd_rn(v, p[(128 + r) * A + a]);
+                        out[row * A + a] = __fadd_rn(v, b3[a]);
+                    }
                 }
                 asm volatile("bar.sync 2, 128;" ::: "memory");
                 if (r == 0) mbar_arrive_release(&bars.p_free[sl]);
