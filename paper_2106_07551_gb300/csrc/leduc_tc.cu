@@ -17,12 +17,12 @@
 // other queue of s, which becomes current when the phase ends (queues never
 // change while they are read). The phase of a unit's first decisions deals the
 // hands from their Philox keys.
-// Warps (7 warpgroups; setmaxnreg moves registers between them):
-//  * 0-15: the engine's epilogue teams (mlp_tc2.cuh), 16-17: its MMA threads,
-//    18-19 idle;
-//  * 20-23 producers: one row per thread, the hand's observation into a bf16
-//    tile (feature 15, constant 1, is folded into b1);
-//  * 24-27 consumers: one row per thread, the logits (two partials + b3), the
+// Warps, in warpgroups (setmaxnreg moves registers between them):
+//  * the engine's two epilogue teams (mlp_tc2.cuh), then a warpgroup whose
+//    first two warps hold its MMA threads (two idle);
+//  * producers (4 warps): one row per thread, the hand's observation into a
+//    bf16 tile (feature 15, constant 1, is folded into b1);
+//  * consumers (4 warps): one row per thread, the logits (partials + b3), the
 //    masked softmax draw keyed by (episode, decision, seat), the transition,
 //    the payoff sums of finished hands, the queue of the next acting seat.
 // Every wait is bounded.
@@ -37,10 +37,17 @@ namespace malib {
 namespace {
 
 constexpr int kK1 = 16;                    // observation inputs after folding feature 15
-using E = Eng2<kK1, 3, 3, 8>;
-constexpr int kWarps = 28;
+constexpr int kTW = 8;                     // epilogue warps per engine slot
+using E = Eng2<kK1, 3, 3, kTW>;
+constexpr int kEpiWG = kTW / 2;            // warpgroups of the two epilogue teams
+constexpr int kMmaWG = kEpiWG, kProdWG = kEpiWG + 1, kConsWG = kEpiWG + 2;
+constexpr int kWarps = 4 * (kEpiWG + 3);
 constexpr int kThreads = 32 * kWarps;
-constexpr int kProdWarp = 20, kConsWarp = 24;
+constexpr int kProdWarp = 4 * kProdWG, kConsWarp = 4 * kConsWG;
+// registers per thread after setmaxnreg: epilogue, MMA, producer, consumer
+// warpgroups (their sum over the CTA stays within the launch's allocation)
+constexpr int kRegEpi = kTW == 8 ? 80 : 112, kRegMma = 56, kRegProd = kTW == 8 ? 48 : 64,
+              kRegCons = kTW == 8 ? 80 : 128;
 constexpr int kMaxDec = 8;
 constexpr uint32_t kX = (E::kImage + 1023u) / 1024u * 1024u;     // X tiles
 constexpr uint32_t kP = kX + E::kNX * E::kXBytes;                  // partial logits
@@ -218,10 +225,10 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
     long long sums[3] = {0, 0, 0};
     auto nothing = [] {};
 
-    if (wg < 4) {
-        // ---- epilogue teams (warps 0-7 slot 0, 8-15 slot 1)
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 80;" ::: "memory");
-        if (warp < 8) {
+    if (wg < kEpiWG) {
+        // ---- epilogue teams (warps 0 .. kTW - 1 slot 0, then slot 1)
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegEpi) : "memory");
+        if (warp < kTW) {
             E::Epilogue<0> ep;
             ep.p_base_off = kP;
             drive(a, w, bars, ctl, smem, [&](const Phase& ph) { ep.run(smem, tbase, bars, ph.nt, a.err); },
@@ -233,16 +240,16 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                   [&] { ep.init(smem); }, sums);
         }
         end_cta(tbase);
-    } else if (wg == 4) {
-        // ---- the MMA threads (warps 16, 17); warps 18-19 idle
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 56;" ::: "memory");
-        if (warp == 16) {
+    } else if (wg == kMmaWG) {
+        // ---- the MMA threads (the warpgroup's first two warps; two idle)
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegMma) : "memory");
+        if (warp == 4 * kMmaWG) {
             E::Issuer<0> is;
             drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
                 if (lane == 0) is.run(smem, smem_u32(smem + kX), tbase, bars, ph.nt, a.err);
             }, nothing, sums);
             if (lane == 0) is.finish(bars, a.err);
-        } else if (warp == 17) {
+        } else if (warp == 4 * kMmaWG + 1) {
             E::Issuer<1> is;
             drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
                 if (lane == 0) is.run(smem, smem_u32(smem + kX), tbase, bars, ph.nt, a.err);
@@ -252,28 +259,40 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
             drive(a, w, bars, ctl, smem, [](const Phase&) {}, nothing, sums);
         }
         end_cta(tbase);
-    } else if (wg == 5) {
+    } else if (wg == kProdWG) {
         // ---- producers: observation rows, one per thread
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 48;" ::: "memory");
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegProd) : "memory");
         const int r = tid - kProdWarp * 32;
         const uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
         drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
+            // the next tile's hand (queue entry, state) is loaded before this
+            // tile's wait, so that its global-memory latency overlaps
+            int nslot = r;
+            uint2 nst = make_uint2(0, 0);
+            if (!ph.first && r < ph.n) {
+                nslot = (int)ph.qin[r];
+                nst = hands[nslot];
+            }
             for (uint32_t i = 0; i < ph.nt; ++i) {
                 const uint32_t T = ph.tile + i;
                 const int buf = (int)(T % E::kNX);
-                if (T >= (uint32_t)E::kNX) E::wait(bars, &bars.x_free[buf], ((T / E::kNX) - 1) & 1u, a.err);
-                uint8_t* xt = smem + kX + buf * E::kXBytes;
                 const int idx = (int)i * 128 + r;
+                const int slot = nslot;
+                const uint2 st = nst;
+                const int nidx = idx + 128;
+                if (nidx < ph.n) {
+                    nslot = ph.first ? nidx : (int)ph.qin[nidx];
+                    if (!ph.first) nst = hands[nslot];
+                }
                 uint32_t wv[8] = {0, 0, 0, 0, 0, 0, 0, 0};
                 if (idx < ph.n) {
-                    const int slot = ph.first ? idx : (int)ph.qin[idx];
                     LeducHand h;
                     int t;
                     if (ph.first) {
                         leduc_deal(h, (uint64_t)ph.pair * (uint64_t)a.n_episodes + (uint64_t)(ph.e_lo + slot), a.seed);
                         t = 0;
                     } else {
-                        unpack(hands[slot], h, t);
+                        unpack(st, h, t);
                     }
                     float ob[17];
                     leduc_obs(h, ob);
@@ -281,6 +300,8 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                     for (int q = 0; q < 7; ++q) wv[q] = tc::pack_bf16(ob[2 * q], ob[2 * q + 1]);
                     wv[7] = tc::pack_bf16(ob[14], ob[16]);   // feature 15 is folded into b1
                 }
+                if (T >= (uint32_t)E::kNX) E::wait(bars, &bars.x_free[buf], ((T / E::kNX) - 1) & 1u, a.err);
+                uint8_t* xt = smem + kX + buf * E::kXBytes;
                 *reinterpret_cast<uint4*>(xt + E::x_offset(r, 0)) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
                 *reinterpret_cast<uint4*>(xt + E::x_offset(r, 8)) = make_uint4(wv[4], wv[5], wv[6], wv[7]);
                 fence_proxy_async_smem();
@@ -291,16 +312,32 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else {
         // ---- consumers: draw, transition, sums, next queue; one row per thread
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 80;" ::: "memory");
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegCons) : "memory");
         const int r = tid - kConsWarp * 32;
         uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
         uint16_t* q_base = w.queues + (size_t)blockIdx.x * 4 * w.max_hands;
         drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
             const float* b3 = reinterpret_cast<const float*>(smem + E::kB3);
             const int s = ph.s;
+            // the next tile's hand is loaded before this tile's wait
+            int nslot = r;
+            uint2 nst = make_uint2(0, 0);
+            if (!ph.first && r < ph.n) {
+                nslot = (int)ph.qin[r];
+                nst = hands[nslot];
+            }
             for (uint32_t i = 0; i < ph.nt; ++i) {
                 const uint32_t T = ph.tile + i;
                 const int sl = (int)(T & 1u);
+                const int cslot = nslot;
+                const uint2 cst = nst;
+                {
+                    const int nidx = (int)i * 128 + 128 + r;
+                    if (nidx < ph.n) {
+                        nslot = ph.first ? nidx : (int)ph.qin[nidx];
+                        if (!ph.first) nst = hands[nslot];
+                    }
+                }
                 E::wait(bars, &bars.p_full[sl], (T >> 1) & 1u, a.err);
                 const float* pp = reinterpret_cast<const float*>(smem + kP + sl * E::kPBytes);
                 const int idx = (int)i * 128 + r;
@@ -308,13 +345,15 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                 if (idx < ph.n) {
 #pragma unroll
                     for (int q = 0; q < 3; ++q)
-                        lg[q] = __fadd_rn(__fadd_rn(pp[r * 3 + q], pp[(128 + r) * 3 + q]), b3[q]);
+                        lg[q] = __fadd_rn(E::kSplit == 2 ? __fadd_rn(pp[r * 3 + q], pp[(128 + r) * 3 + q])
+                                                          : pp[r * 3 + q],
+                                          b3[q]);
                 }
                 asm volatile("bar.sync 3, 128;" ::: "memory");
                 if (r == 0) mbar_arrive_release(&bars.p_free[sl]);
                 int next = -1, slot = 0;
                 if (idx < ph.n) {
-                    slot = ph.first ? idx : (int)ph.qin[idx];
+                    slot = cslot;
                     LeducHand h;
                     int t;
                     const int64_t e = ph.e_lo + slot;
@@ -323,7 +362,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                         leduc_deal(h, gid, a.seed);
                         t = 0;
                     } else {
-                        unpack(hands[slot], h, t);
+                        unpack(cst, h, t);
                     }
                     const float u = u24(draw(gid, (uint32_t)t, (uint32_t)s, a.seed).x);
                     const unsigned legal = leduc_legal(h);
