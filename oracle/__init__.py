@@ -52,6 +52,8 @@ def _L():
             sig = {
                 "orc_philox": (None, [P, u64, P, i64]),
                 "orc_det_expf": (None, [P, P, i64]),
+                "orc_det_log1pf": (None, [P, P, i64]),
+                "orc_contact_force": (None, [f32, f32, f32, f32, f32, P]),
                 "orc_sample": (None, [P, P, P, C.c_int, P, i64]),
                 "orc_bf16_round": (f32, [f32]),
                 "orc_mlp_forward": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, i64, P]),
@@ -63,12 +65,12 @@ def _L():
                 "orc_leduc_exact": (C.c_double, [P, P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int]),
                 "orc_leduc_eval": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P, i32, i64,
                                           i64, u64, P, i64, P, P, P, P, P, P, P, P, C.c_int]),
-                "orc_spread_step": (None, [C.c_int, C.c_int, P, P, P, C.c_float]),
+                "orc_spread_step": (None, [C.c_int, C.c_int, P, P, P, C.c_float, C.c_int]),
                 "orc_spread_obs": (None, [C.c_int, C.c_int, P, C.c_int, P]),
                 "orc_spread_reset": (None, [C.c_int, C.c_int, u64, u64, P]),
                 "orc_spread_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                               C.c_int, C.c_int, C.c_int, i64, i64, i64, P, i32, i64,
-                                              u64, P, P, P, P, P, C.c_int, C.c_float]),
+                                              u64, P, P, P, P, P, C.c_int, C.c_float, C.c_int]),
                 "orc_sl_reset": (None, [u64, u64, P]),
                 "orc_sl_step": (None, [P, P, P]),
                 "orc_sl_obs": (None, [P, P]),
@@ -79,6 +81,16 @@ def _L():
                 "orc_adversary_obs": (None, [P, P]),
                 "orc_adversary_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
                                                  P, i32, i64, u64, P, P, P, P, P, C.c_int]),
+                "orc_push_reset": (None, [u64, u64, P]),
+                "orc_push_step": (None, [P, P, P]),
+                "orc_push_obs": (None, [P, P]),
+                "orc_push_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
+                                            P, i32, i64, u64, P, P, P, P, P, C.c_int]),
+                "orc_tag_reset": (None, [u64, u64, P]),
+                "orc_tag_step": (None, [P, P, P]),
+                "orc_tag_obs": (None, [P, P]),
+                "orc_tag_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
+                                           P, i32, i64, u64, P, P, P, P, P, C.c_int]),
             }
             for name, (res, args) in sig.items():
                 fn = getattr(lib, name)
@@ -110,6 +122,22 @@ def det_expf(x: np.ndarray) -> np.ndarray:
     y = np.empty_like(x)
     _L().orc_det_expf(_p(x), _p(y), x.size)
     return y
+
+
+def det_log1pf(x: np.ndarray) -> np.ndarray:
+    """log(1 + x) for x in [0, 1] by the fp32 atanh series (contact model)."""
+    x = _c(x, np.float32)
+    y = np.empty_like(x)
+    _L().orc_det_log1pf(_p(x), _p(y), x.size)
+    return y
+
+
+def contact_force(a, b, dmin: float):
+    """Soft contact force on the disk at a from the disk at b (radii summing to
+    dmin): (force [2] fp32, whether one acts)."""
+    out = np.zeros(3, np.float32)
+    _L().orc_contact_force(float(a[0]), float(a[1]), float(b[0]), float(b[1]), float(dmin), _p(out))
+    return out[:2].copy(), bool(out[2])
 
 
 def sample(logits: np.ndarray, legal: np.ndarray, u: np.ndarray) -> np.ndarray:
@@ -228,14 +256,15 @@ def leduc_eval(params_list, dims, pairs, n_episodes, seed, bf16=False, n_rec=0,
 
 # ---------------------------------------------------------------- spread
 def spread_step(state: np.ndarray, N: int, L: int, actions,
-                local_ratio=None) -> tuple[np.ndarray, np.ndarray]:
+                local_ratio=None, contact: bool = False) -> tuple[np.ndarray, np.ndarray]:
     """One transition; local_ratio (None: the unweighted reward) weights the
-    shared cover term by 1 - local_ratio and the agent's collisions by it."""
+    shared cover term by 1 - local_ratio and the agent's collisions by it;
+    contact adds the soft contact forces between the agents."""
     st = _c(state, np.float32).copy()
     act = _c(actions, np.int32)
     rew = np.zeros(N, np.float32)
     _L().orc_spread_step(N, L, _p(st), _p(act), _p(rew),
-                         -1.0 if local_ratio is None else float(local_ratio))
+                         -1.0 if local_ratio is None else float(local_ratio), int(bool(contact)))
     return st, rew
 
 
@@ -253,7 +282,8 @@ def spread_reset(N: int, L: int, g: int, seed: int) -> np.ndarray:
 
 
 def spread_rollout(params_list, dims, N, L, T, n_envs, pairs, n_episodes, seed, bf16=False,
-                   env_lo=0, env_hi=None, ext_logits=None, n_threads=0, local_ratio=None):
+                   env_lo=0, env_hi=None, ext_logits=None, n_threads=0, local_ratio=None,
+                   contact=False):
     """Rollout over envs [env_lo, env_hi). Returns dict of obs [E][T][W][N][in],
     action int8 [E][T][W][N], reward [E][T][W][N], logits [E][T][W][N][A]."""
     env_hi = n_envs if env_hi is None else env_hi
@@ -270,7 +300,7 @@ def spread_rollout(params_list, dims, N, L, T, n_envs, pairs, n_episodes, seed, 
                             env_lo, env_hi, _p(pairs), pairs.shape[0], n_episodes,
                             C.c_uint64(seed), _p(ext), _p(out["obs"]), _p(out["action"]),
                             _p(out["reward"]), _p(out["logits"]), n_threads,
-                            -1.0 if local_ratio is None else float(local_ratio))
+                            -1.0 if local_ratio is None else float(local_ratio), int(bool(contact)))
     del arrs
     return out
 
@@ -374,3 +404,61 @@ def adversary_rollout(params_list, dims, T, n_envs, pairs, n_episodes, seed, bf1
                                _p(out["logits"]), n_threads)
     del arrs
     return out
+
+
+# ---- simple push and simple tag (App. B.1) ----
+# push state: px,py,vx,vy of agents 0 (adversary), 1 (good); lx,ly of the
+# landmark (10 floats). tag state: px,py,vx,vy of agents 0..2 (adversaries), 3
+# (good); ox,oy of the two obstacles (20 floats).
+PUSH_N, PUSH_L, PUSH_OBS, PUSH_STATE = 2, 1, 8, 10
+TAG_N, TAG_L, TAG_OBS, TAG_STATE = 4, 2, 16, 20
+
+
+def _scen(name, N, OBS, STATE):
+    def reset(g: int, seed: int) -> np.ndarray:
+        st = np.zeros(STATE, np.float32)
+        getattr(_L(), f"orc_{name}_reset")(C.c_uint64(g), C.c_uint64(seed), _p(st))
+        return st
+
+    def step(state: np.ndarray, actions) -> tuple[np.ndarray, np.ndarray]:
+        st = _c(state, np.float32).copy()
+        act = _c(actions, np.int32)
+        rew = np.zeros(N, np.float32)
+        getattr(_L(), f"orc_{name}_step")(_p(st), _p(act), _p(rew))
+        return st, rew
+
+    def obs(state: np.ndarray) -> np.ndarray:
+        st = _c(state, np.float32)
+        out = np.zeros((N, OBS), np.float32)
+        getattr(_L(), f"orc_{name}_obs")(_p(st), _p(out))
+        return out
+
+    def rollout(params_list, dims, T, n_envs, pairs, n_episodes, seed, bf16=False,
+                env_lo=0, env_hi=None, ext_logits=None, n_threads=0):
+        env_hi = n_envs if env_hi is None else env_hi
+        W = env_hi - env_lo
+        i, h1, h2, A = dims
+        assert i == OBS and A == 5
+        arrs, tbl = _param_table(params_list)
+        prs = _c(pairs, np.int32).reshape(-1, N)
+        out = dict(obs=np.zeros((n_episodes, T, W, N, i), np.float32),
+                   action=np.zeros((n_episodes, T, W, N), np.int8),
+                   reward=np.zeros((n_episodes, T, W, N), np.float32),
+                   logits=np.zeros((n_episodes, T, W, N, A), np.float32))
+        ext = None if ext_logits is None else _c(ext_logits, np.float32).reshape(n_episodes, T, W, N, A)
+        getattr(_L(), f"orc_{name}_rollout")(
+            C.cast(tbl, C.c_void_p), h1, h2, int(bf16), T, n_envs, env_lo, env_hi, _p(prs),
+            prs.shape[0], n_episodes, C.c_uint64(seed), _p(ext), _p(out["obs"]),
+            _p(out["action"]), _p(out["reward"]), _p(out["logits"]), n_threads)
+        del arrs
+        return out
+
+    return reset, step, obs, rollout
+
+
+push_reset, push_step, push_obs, push_rollout = _scen("push", PUSH_N, PUSH_OBS, PUSH_STATE)
+push_rollout.__doc__ = """Rollout over envs [env_lo, env_hi) of the simple push (2 agents, obs 8,
+5 actions). Returns the arrays of spread_rollout."""
+tag_reset, tag_step, tag_obs, tag_rollout = _scen("tag", TAG_N, TAG_OBS, TAG_STATE)
+tag_rollout.__doc__ = """Rollout over envs [env_lo, env_hi) of the simple tag (4 agents, obs 16,
+5 actions). Returns the arrays of spread_rollout."""

@@ -22,6 +22,15 @@
 //    landmarks of which one is the target; good agents are rewarded for being
 //    close to the target and for the adversary being far from it, the adversary
 //    (which is not told the target) for being close to it.
+//  * App. B.1 "Simple Push": one good agent, one adversary, one landmark; the
+//    good agent is rewarded by its distance to the landmark, the adversary by
+//    the difference of the two distances, so it learns to push.
+//  * App. B.1 "Simple Tag": one faster good agent, three slower adversaries,
+//    two obstacles that block the way; -10 to the good agent and +10 to the
+//    adversaries for each hit.
+//  * Collisions of App. B.1 as forces (push, tag, and spread as an option): a
+//    soft contact model between disks, a stated reading (the paper gives no
+//    force law).
 // Kuhn and Leduc rules are not given in the paper; the textbook rules are used,
 // each reading stated at the function that takes it below.
 //
@@ -35,8 +44,13 @@
 // invariants), the simple adversary (hand-worked geometry, the reward
 // identity against fp64, the spread dynamics and reset, symmetries) and the
 // simple speaker listener (hand-worked geometry, the one-step message delay,
-// the immobile speaker, the spread dynamics and reset, the target draw) are
-// pinned by the CPU tests, and whole spread episodes under forced actions (at
+// the immobile speaker, the spread dynamics and reset, the target draw), the
+// contact model (log1p against the library, the force against its formula in
+// fp64, zero beyond the margin, equal and opposite pairs, total velocity
+// against the closed form), simple push (hand-worked geometry, contact on both
+// agents) and simple tag (speed limits against the capped recursion, the hit
+// rule, immovable obstacles, the observation layout) are pinned by the CPU
+// tests, and whole spread episodes under forced actions (at
 // rest; a constant force from rest) match closed forms; episode returns of the
 // particle scenarios under sampled policies beyond those are "parity unpinned"
 // (no closed form exists).
@@ -559,24 +573,118 @@ float dist2d(float ax, float ay, float bx, float by) {
     return std::sqrt(sq);
 }
 
+// ---------------------------------------------------------------------------
+// det_log1pf: log(1 + y) for y in [0, 1] in fp32, every step one correctly
+// rounded IEEE operation. Method: log(1 + y) = 2 atanh(z) with z = y / (2 + y)
+// in [0, 1/3], and atanh(z) = z (1 + z^2/3 + z^4/5 + ... + z^16/17) (the odd
+// power series, truncated after z^17: the next term is below 2^-32 relative),
+// in Horner form in w = z^2 with fused multiply-adds.
+// ---------------------------------------------------------------------------
+float det_log1pf(float y) {
+    if (!(y > 0.0f)) return 0.0f;
+    const float z = y / (2.0f + y);
+    const float w = z * z;
+    float p = 0x1.e1e1e2p-5f;         // 1/17
+    p = fmaf(p, w, 0x1.111112p-4f);   // 1/15
+    p = fmaf(p, w, 0x1.3b13b2p-4f);   // 1/13
+    p = fmaf(p, w, 0x1.745d18p-4f);   // 1/11
+    p = fmaf(p, w, 0x1.c71c72p-4f);   // 1/9
+    p = fmaf(p, w, 0x1.24924ap-3f);   // 1/7
+    p = fmaf(p, w, 0x1.99999ap-3f);   // 1/5
+    p = fmaf(p, w, 0x1.555556p-2f);   // 1/3
+    p = fmaf(p, w, 1.0f);
+    return (2.0f * z) * p;
+}
+
+// ---------------------------------------------------------------------------
+// Contact between two colliding disks (App. B.1 names collisions and
+// "obstacles block the way" but gives no force law; this is the soft contact
+// model of the particle environments the paper runs, restated as a reading):
+// centres a and b, radii summing to dmin, delta = a - b, d = |delta|. The
+// penetration is a softplus of the overlap with margin k = 0.001,
+//   pen = k * log(1 + exp((dmin - d) / k)),
+// and the force on a is F_c * pen * delta / d with F_c = 100 (b gets its
+// negative). Evaluated in fp32 in this order: dx, dy, q = dx*dx + dy*dy,
+// d = sqrt(q), x = (dmin - d) / k, softplus(x) = max(x, 0) +
+// log1p(exp(-|x|)) (det_expf, det_log1pf), pen = k * softplus, c = (F_c * pen)
+// / d, force (c*dx, c*dy). No force when d == 0 or pen == 0 (which holds once
+// d - dmin >= 87 k, where det_expf gives 0). Returns whether a force acts.
+// ---------------------------------------------------------------------------
+const float CONTACT_MARGIN = 0.001f;
+const float CONTACT_FORCE = 100.0f;
+
+bool contact_force(float ax, float ay, float bx, float by, float dmin, float* fx, float* fy) {
+    const float dx = ax - bx, dy = ay - by;
+    const float q = dx * dx + dy * dy;
+    const float d = std::sqrt(q);
+    if (d == 0.0f) return false;
+    const float x = (dmin - d) / CONTACT_MARGIN;
+    const float ax_ = std::fabs(x);
+    const float sp = (x > 0.0f ? x : 0.0f) + det_log1pf(det_expf(-ax_));
+    const float pen = CONTACT_MARGIN * sp;
+    if (pen == 0.0f) return false;
+    const float c = (CONTACT_FORCE * pen) / d;
+    *fx = c * dx;
+    *fy = c * dy;
+    return true;
+}
+
+// Adds the contact forces between every pair of the n movable disks (ascending
+// pairs a < b; disk i at (px[i], py[i]) with radius rad[i]) to F: a gets +f, b
+// gets -f. Then, for every movable disk a (ascending) and every immovable disk
+// o (ascending; at (ox[o], oy[o]), radius orad[o]), the force on a. A force is
+// added only where one acts, so with no contact F keeps its bits.
+void add_contacts(int n, const float* px, const float* py, const float* rad, int m, const float* ox,
+                  const float* oy, const float* orad, float* Fx, float* Fy) {
+    for (int a = 0; a < n; ++a)
+        for (int b = a + 1; b < n; ++b) {
+            float fx, fy;
+            if (contact_force(px[a], py[a], px[b], py[b], rad[a] + rad[b], &fx, &fy)) {
+                Fx[a] = Fx[a] + fx; Fy[a] = Fy[a] + fy;
+                Fx[b] = Fx[b] - fx; Fy[b] = Fy[b] - fy;
+            }
+        }
+    for (int a = 0; a < n; ++a)
+        for (int o = 0; o < m; ++o) {
+            float fx, fy;
+            if (contact_force(px[a], py[a], ox[o], oy[o], rad[a] + orad[o], &fx, &fy)) {
+                Fx[a] = Fx[a] + fx; Fy[a] = Fy[a] + fy;
+            }
+        }
+}
+
+// Unit action force of the five discrete actions (0 noop, 1 +x, 2 -x, 3 +y, 4 -y).
+void action_force(int act, float* fx, float* fy) {
+    *fx = 0.0f; *fy = 0.0f;
+    switch (act) {
+        case 1: *fx = 1.0f; break;
+        case 2: *fx = -1.0f; break;
+        case 3: *fy = 1.0f; break;
+        case 4: *fy = -1.0f; break;
+        default: break;
+    }
+}
+
 // local_ratio < 0: r_i = -(cover + collisions_i) (the workloads' reward);
 // otherwise the App. B.1 weighting of the shared and the local term:
 // r_i = -((1 - local_ratio) * cover + local_ratio * collisions_i), evaluated
 // as written (one rounding per operation, no contraction).
-void spread_step(Spread& s, const int* action, float* reward, float local_ratio) {
+// contact: the agents (radius 0.15) also push each other apart with the soft
+// contact forces of add_contacts, computed from the positions before the move
+// and added to the action forces (landmarks do not collide).
+void spread_step(Spread& s, const int* action, float* reward, float local_ratio, bool contact = false) {
+    float Fx[16], Fy[16];
+    for (int i = 0; i < s.N; ++i) action_force(action[i], &Fx[i], &Fy[i]);
+    if (contact) {
+        float rad[16];
+        for (int i = 0; i < s.N; ++i) rad[i] = 0.15f;
+        add_contacts(s.N, s.px, s.py, rad, 0, nullptr, nullptr, nullptr, Fx, Fy);
+    }
     for (int i = 0; i < s.N; ++i) {
-        float fx = 0.0f, fy = 0.0f;
-        switch (action[i]) {
-            case 1: fx = 1.0f; break;
-            case 2: fx = -1.0f; break;
-            case 3: fy = 1.0f; break;
-            case 4: fy = -1.0f; break;
-            default: break;
-        }
         s.vx[i] = s.vx[i] * 0.75f;
         s.vy[i] = s.vy[i] * 0.75f;
-        s.vx[i] = s.vx[i] + fx * 0.1f;
-        s.vy[i] = s.vy[i] + fy * 0.1f;
+        s.vx[i] = s.vx[i] + Fx[i] * 0.1f;
+        s.vy[i] = s.vy[i] + Fy[i] * 0.1f;
         s.px[i] = s.px[i] + s.vx[i] * 0.1f;
         s.py[i] = s.py[i] + s.vy[i] * 0.1f;
     }
@@ -735,6 +843,179 @@ void sl_step(SpeakerListener& a, const int* action, float* reward) {
     reward[1] = -d;
 }
 
+// ---------------------------------------------------------------------------
+// Simple push (App. B.1; readings of its description, constants of the spread
+// scenario): agent 0 is the adversary, agent 1 the good agent, one landmark.
+// Reset as spread (same chance counters, N = 2, L = 1). Both agents are disks
+// of radius 0.15 that push each other with the soft contact forces (the
+// landmark does not collide); unit action forces, mass 1, dt 0.1, damping
+// 0.25. Rewards after the move, with d_i = |p_i - landmark|:
+//   good agent r_1 = -d_1;   adversary r_0 = d_1 - d_0
+// (close to the landmark itself, and the good agent far from it: the
+// difference of the distances). Observation of agent i (8 floats): velocity,
+// position, landmark - p_i, the other agent - p_i.
+// ---------------------------------------------------------------------------
+struct Push {
+    Spread s;
+};
+
+void push_reset(Push& a, uint64_t g, uint64_t seed) { spread_reset(a.s, 2, 1, g, seed); }
+
+void push_obs(const Push& a, int i, float* o) {
+    const Spread& s = a.s;
+    const int j = 1 - i;
+    o[0] = s.vx[i]; o[1] = s.vy[i];
+    o[2] = s.px[i]; o[3] = s.py[i];
+    o[4] = s.lx[0] - s.px[i]; o[5] = s.ly[0] - s.py[i];
+    o[6] = s.px[j] - s.px[i]; o[7] = s.py[j] - s.py[i];
+}
+
+void push_step(Push& a, const int* action, float* reward) {
+    Spread& s = a.s;
+    float Fx[2], Fy[2];
+    for (int i = 0; i < 2; ++i) action_force(action[i], &Fx[i], &Fy[i]);
+    const float rad[2] = {0.15f, 0.15f};
+    add_contacts(2, s.px, s.py, rad, 0, nullptr, nullptr, nullptr, Fx, Fy);
+    for (int i = 0; i < 2; ++i) {
+        s.vx[i] = s.vx[i] * 0.75f;
+        s.vy[i] = s.vy[i] * 0.75f;
+        s.vx[i] = s.vx[i] + Fx[i] * 0.1f;
+        s.vy[i] = s.vy[i] + Fy[i] * 0.1f;
+        s.px[i] = s.px[i] + s.vx[i] * 0.1f;
+        s.py[i] = s.py[i] + s.vy[i] * 0.1f;
+    }
+    const float d0 = dist2d(s.px[0], s.py[0], s.lx[0], s.ly[0]);
+    const float d1 = dist2d(s.px[1], s.py[1], s.lx[0], s.ly[0]);
+    reward[0] = d1 - d0;
+    reward[1] = -d1;
+}
+
+// ---------------------------------------------------------------------------
+// Simple tag (App. B.1; readings of its description: "the good agent is
+// faster", "-10 for each collision" / "+10 for each collision", "obstacles
+// block the way"; sizes, accelerations and speed limits as stated readings):
+// agents 0..2 are the adversaries (radius 0.075, action force 3, speed limit
+// 1.0), agent 3 the good agent (radius 0.05, action force 4, speed limit 1.3),
+// two obstacles (radius 0.2, immovable). Reset as spread (same chance
+// counters, N = 4, the obstacles in the landmark slots L = 2). Every pair of
+// agents and every (agent, obstacle) pair collides with the soft contact
+// forces, from the positions before the move. Per agent (ascending): v <- v *
+// 0.75; v <- v + F * 0.1 (mass 1); if |v| > limit, v <- (v / |v|) * limit per
+// component; p <- p + v * 0.1. After the move adversary i hits the good agent
+// when |p_i - p_3| < 0.075 + 0.05; with h the number of hits, r_3 = -10 h and
+// every adversary gets r_i = 10 h. Observation of agent i (16 floats):
+// velocity, position, obstacles - p_i, the other agents - p_i (ascending),
+// then the good agent's velocity for an adversary (zeros for the good agent).
+// ---------------------------------------------------------------------------
+struct Tag {
+    Spread s;
+};
+
+const float TAG_RAD[4] = {0.075f, 0.075f, 0.075f, 0.05f};
+const float TAG_ACCEL[4] = {3.0f, 3.0f, 3.0f, 4.0f};
+const float TAG_VMAX[4] = {1.0f, 1.0f, 1.0f, 1.3f};
+const float TAG_OBST_RAD[2] = {0.2f, 0.2f};
+
+void tag_reset(Tag& a, uint64_t g, uint64_t seed) { spread_reset(a.s, 4, 2, g, seed); }
+
+void tag_obs(const Tag& a, int i, float* o) {
+    const Spread& s = a.s;
+    int k = 0;
+    o[k++] = s.vx[i]; o[k++] = s.vy[i];
+    o[k++] = s.px[i]; o[k++] = s.py[i];
+    for (int l = 0; l < 2; ++l) { o[k++] = s.lx[l] - s.px[i]; o[k++] = s.ly[l] - s.py[i]; }
+    for (int j = 0; j < 4; ++j) {
+        if (j == i) continue;
+        o[k++] = s.px[j] - s.px[i]; o[k++] = s.py[j] - s.py[i];
+    }
+    if (i < 3) { o[k++] = s.vx[3]; o[k++] = s.vy[3]; }
+    else { o[k++] = 0.0f; o[k++] = 0.0f; }
+}
+
+void tag_step(Tag& a, const int* action, float* reward) {
+    Spread& s = a.s;
+    float Fx[4], Fy[4];
+    for (int i = 0; i < 4; ++i) {
+        float ux, uy;
+        action_force(action[i], &ux, &uy);
+        Fx[i] = TAG_ACCEL[i] * ux;
+        Fy[i] = TAG_ACCEL[i] * uy;
+    }
+    add_contacts(4, s.px, s.py, TAG_RAD, 2, s.lx, s.ly, TAG_OBST_RAD, Fx, Fy);
+    for (int i = 0; i < 4; ++i) {
+        s.vx[i] = s.vx[i] * 0.75f;
+        s.vy[i] = s.vy[i] * 0.75f;
+        s.vx[i] = s.vx[i] + Fx[i] * 0.1f;
+        s.vy[i] = s.vy[i] + Fy[i] * 0.1f;
+        const float speed = std::sqrt(s.vx[i] * s.vx[i] + s.vy[i] * s.vy[i]);
+        if (speed > TAG_VMAX[i]) {
+            s.vx[i] = (s.vx[i] / speed) * TAG_VMAX[i];
+            s.vy[i] = (s.vy[i] / speed) * TAG_VMAX[i];
+        }
+        s.px[i] = s.px[i] + s.vx[i] * 0.1f;
+        s.py[i] = s.py[i] + s.vy[i] * 0.1f;
+    }
+    int hits = 0;
+    for (int i = 0; i < 3; ++i)
+        if (dist2d(s.px[i], s.py[i], s.px[3], s.py[3]) < TAG_RAD[i] + TAG_RAD[3]) ++hits;
+    for (int i = 0; i < 3; ++i) reward[i] = 10.0f * (float)hits;
+    reward[3] = -10.0f * (float)hits;
+}
+
+// One rollout driver for the fixed-size scenarios (push, tag): Env supplies N,
+// IN, reset, obs and step; all actions legal.
+struct PushEnvDef {
+    using S = Push;
+    static const int N = 2, IN = 8;
+    static void reset(S& a, uint64_t g, uint64_t seed) { push_reset(a, g, seed); }
+    static void obs(const S& a, int i, float* o) { push_obs(a, i, o); }
+    static void step(S& a, const int* act, float* r) { push_step(a, act, r); }
+};
+struct TagEnvDef {
+    using S = Tag;
+    static const int N = 4, IN = 16;
+    static void reset(S& a, uint64_t g, uint64_t seed) { tag_reset(a, g, seed); }
+    static void obs(const S& a, int i, float* o) { tag_obs(a, i, o); }
+    static void step(S& a, const int* act, float* r) { tag_step(a, act, r); }
+};
+
+template <class Env>
+void scenario_rollout(const float* const* params, int h1, int h2, int bf16, int T, int64_t n_envs,
+                      int64_t env_lo, int64_t env_hi, const int32_t* pairs, int32_t n_pairs,
+                      int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
+                      int8_t* action, float* reward, float* logits, int n_threads) {
+    const int N = Env::N, in = Env::IN, A = 5;
+    int64_t per = n_envs / n_pairs;
+    int64_t W = env_hi - env_lo;
+    parallel_for(W * n_episodes, n_threads, [&](int64_t job) {
+        int64_t ep = job / W, e = env_lo + job % W;
+        int64_t row = e / per;
+        typename Env::S st;
+        uint64_t g = (uint64_t)ep * (uint64_t)n_envs + (uint64_t)e;
+        Env::reset(st, g, seed);
+        for (int t = 0; t < T; ++t) {
+            int act[Env::N];
+            for (int i = 0; i < N; ++i) {
+                int64_t idx = ((ep * T + t) * W + (e - env_lo)) * N + i;
+                float o[Env::IN], lg[8];
+                Env::obs(st, i, o);
+                Mlp m{params[pairs[row * N + i]], in, h1, h2, A, bf16};
+                mlp_logits(m, o, lg);
+                uint8_t legal[8] = {1, 1, 1, 1, 1, 1, 1, 1};
+                float u = uniform24(draw(g, (uint32_t)t, (uint32_t)i, seed).x[0]);
+                act[i] = sample_masked(ext_logits ? ext_logits + idx * A : lg, legal, A, u);
+                if (obs) std::memcpy(obs + idx * in, o, sizeof(float) * in);
+                if (logits) std::memcpy(logits + idx * A, lg, sizeof(float) * A);
+                if (action) action[idx] = (int8_t)act[i];
+            }
+            float r[Env::N];
+            Env::step(st, act, r);
+            if (reward)
+                for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
+        }
+    });
+}
+
 }  // namespace
 
 // ===========================================================================
@@ -751,6 +1032,18 @@ void orc_philox(const uint32_t* ctr, uint64_t seed, uint32_t* out, int64_t n) {
 
 void orc_det_expf(const float* x, float* y, int64_t n) {
     for (int64_t i = 0; i < n; ++i) y[i] = det_expf(x[i]);
+}
+
+void orc_det_log1pf(const float* x, float* y, int64_t n) {
+    for (int64_t i = 0; i < n; ++i) y[i] = det_log1pf(x[i]);
+}
+
+// Contact force on disk a from disk b (radii summing to dmin): out[0..1] the
+// force, out[2] = 1 when one acts (else 0 and a zero force).
+void orc_contact_force(float ax, float ay, float bx, float by, float dmin, float* out) {
+    float fx = 0.0f, fy = 0.0f;
+    const bool on = contact_force(ax, ay, bx, by, dmin, &fx, &fy);
+    out[0] = fx; out[1] = fy; out[2] = on ? 1.0f : 0.0f;
 }
 
 void orc_sample(const float* logits, const uint8_t* legal, const float* u, int A, int32_t* out, int64_t n) {
@@ -892,7 +1185,7 @@ void orc_leduc_eval(const float* const* params, int in, int h1, int h2, int out,
 // One transition from a given state (for hand-worked checks). state: px,py,vx,vy
 // for N agents then lx,ly for L landmarks (packed [4N + 2L]); updated in place.
 void orc_spread_step(int N, int L, float* state, const int32_t* action, float* reward,
-                     float local_ratio) {
+                     float local_ratio, int contact) {
     Spread s;
     s.N = N; s.L = L;
     for (int i = 0; i < N; ++i) {
@@ -900,7 +1193,7 @@ void orc_spread_step(int N, int L, float* state, const int32_t* action, float* r
         s.vx[i] = state[4 * i + 2]; s.vy[i] = state[4 * i + 3];
     }
     for (int l = 0; l < L; ++l) { s.lx[l] = state[4 * N + 2 * l]; s.ly[l] = state[4 * N + 2 * l + 1]; }
-    spread_step(s, action, reward, local_ratio);
+    spread_step(s, action, reward, local_ratio, contact != 0);
     for (int i = 0; i < N; ++i) {
         state[4 * i] = s.px[i]; state[4 * i + 1] = s.py[i];
         state[4 * i + 2] = s.vx[i]; state[4 * i + 3] = s.vy[i];
@@ -938,7 +1231,7 @@ void orc_spread_rollout(const float* const* params, int in, int h1, int h2, int 
                         int N, int L, int T, int64_t n_envs, int64_t env_lo, int64_t env_hi,
                         const int32_t* pairs, int32_t n_pairs, int64_t n_episodes, uint64_t seed,
                         const float* ext_logits, float* obs, int8_t* action, float* reward,
-                        float* logits, int n_threads, float local_ratio) {
+                        float* logits, int n_threads, float local_ratio, int contact) {
     int64_t per = n_envs / n_pairs;
     int64_t W = env_hi - env_lo;
     parallel_for(W * n_episodes, n_threads, [&](int64_t job) {
@@ -963,7 +1256,7 @@ void orc_spread_rollout(const float* const* params, int in, int h1, int h2, int 
                 if (action) action[idx] = (int8_t)act[i];
             }
             float r[16];
-            spread_step(s, act, r, local_ratio);
+            spread_step(s, act, r, local_ratio, contact != 0);
             if (reward)
                 for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
         }
@@ -1127,6 +1420,73 @@ void orc_sl_rollout(const float* const* params, int h1, int h2, int bf16, int T,
                 for (int i = 0; i < N; ++i) reward[((ep * T + t) * W + (e - env_lo)) * N + i] = r[i];
         }
     });
+}
+
+// ---- Simple push and simple tag ----
+// state: px,py,vx,vy of the agents, then lx,ly of the landmarks / obstacles
+// (push [4*2 + 2] = 10 floats, tag [4*4 + 2*2] = 20 floats).
+static void sc_load(const float* state, int N, int L, Spread& s) {
+    s.N = N; s.L = L;
+    for (int i = 0; i < N; ++i) {
+        s.px[i] = state[4 * i]; s.py[i] = state[4 * i + 1];
+        s.vx[i] = state[4 * i + 2]; s.vy[i] = state[4 * i + 3];
+    }
+    for (int l = 0; l < L; ++l) { s.lx[l] = state[4 * N + 2 * l]; s.ly[l] = state[4 * N + 2 * l + 1]; }
+}
+static void sc_store(const Spread& s, float* state) {
+    for (int i = 0; i < s.N; ++i) {
+        state[4 * i] = s.px[i]; state[4 * i + 1] = s.py[i];
+        state[4 * i + 2] = s.vx[i]; state[4 * i + 3] = s.vy[i];
+    }
+    for (int l = 0; l < s.L; ++l) { state[4 * s.N + 2 * l] = s.lx[l]; state[4 * s.N + 2 * l + 1] = s.ly[l]; }
+}
+
+void orc_push_reset(uint64_t g, uint64_t seed, float* state) {
+    Push a;
+    push_reset(a, g, seed);
+    sc_store(a.s, state);
+}
+void orc_push_step(float* state, const int32_t* action, float* reward) {
+    Push a;
+    sc_load(state, 2, 1, a.s);
+    push_step(a, action, reward);
+    sc_store(a.s, state);
+}
+void orc_push_obs(const float* state, float* obs /*[2][8]*/) {
+    Push a;
+    sc_load(state, 2, 1, a.s);
+    for (int i = 0; i < 2; ++i) push_obs(a, i, obs + i * 8);
+}
+void orc_push_rollout(const float* const* params, int h1, int h2, int bf16, int T, int64_t n_envs,
+                      int64_t env_lo, int64_t env_hi, const int32_t* pairs, int32_t n_pairs,
+                      int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
+                      int8_t* action, float* reward, float* logits, int n_threads) {
+    scenario_rollout<PushEnvDef>(params, h1, h2, bf16, T, n_envs, env_lo, env_hi, pairs, n_pairs,
+                                 n_episodes, seed, ext_logits, obs, action, reward, logits, n_threads);
+}
+
+void orc_tag_reset(uint64_t g, uint64_t seed, float* state) {
+    Tag a;
+    tag_reset(a, g, seed);
+    sc_store(a.s, state);
+}
+void orc_tag_step(float* state, const int32_t* action, float* reward) {
+    Tag a;
+    sc_load(state, 4, 2, a.s);
+    tag_step(a, action, reward);
+    sc_store(a.s, state);
+}
+void orc_tag_obs(const float* state, float* obs /*[4][16]*/) {
+    Tag a;
+    sc_load(state, 4, 2, a.s);
+    for (int i = 0; i < 4; ++i) tag_obs(a, i, obs + i * 16);
+}
+void orc_tag_rollout(const float* const* params, int h1, int h2, int bf16, int T, int64_t n_envs,
+                     int64_t env_lo, int64_t env_hi, const int32_t* pairs, int32_t n_pairs,
+                     int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
+                     int8_t* action, float* reward, float* logits, int n_threads) {
+    scenario_rollout<TagEnvDef>(params, h1, h2, bf16, T, n_envs, env_lo, env_hi, pairs, n_pairs,
+                                n_episodes, seed, ext_logits, obs, action, reward, logits, n_threads);
 }
 
 }  // extern "C"
