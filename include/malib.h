@@ -51,7 +51,9 @@ typedef enum malib_env_kind {
     MALIB_ENV_LEDUC = 2,      /* Leduc hold'em: 6 cards, 2 rounds, raises 2 then 4 */
     MALIB_ENV_SPREAD = 3,     /* cooperative particle spread (App. B.1) */
     MALIB_ENV_ADVERSARY = 4,  /* simple adversary (App. B.1): 1 adversary, 2 good agents */
-    MALIB_ENV_SPEAKER_LISTENER = 5  /* simple speaker listener (App. B.1): speaker, listener */
+    MALIB_ENV_SPEAKER_LISTENER = 5, /* simple speaker listener (App. B.1): speaker, listener */
+    MALIB_ENV_PUSH = 6,       /* simple push (App. B.1): 1 adversary, 1 good agent, 1 landmark */
+    MALIB_ENV_TAG = 7         /* simple tag (App. B.1): 3 adversaries, 1 good agent, 2 obstacles */
 } malib_env_kind;
 
 typedef enum malib_policy_kind {
@@ -68,6 +70,7 @@ typedef enum malib_dtype {
 #define MALIB_DUMP_LOGITS 1u          /* record logits (and obs, actions) in a malib_traj */
 #define MALIB_EXACT_EXPECTATION 2u    /* Kuhn: exact enumeration instead of Monte Carlo */
 #define MALIB_SPREAD_LOCAL_RATIO 4u   /* SPREAD: weight the reward terms by local_ratio */
+#define MALIB_SPREAD_CONTACT 8u       /* SPREAD: agents push each other apart (contact forces) */
 
 typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
 
@@ -82,8 +85,13 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  *           n_landmarks 2, obs_dim 14, n_actions 5, episode_len >= 1
  *   SPEAKER_LISTENER: n_agents 2 (agent 0 the speaker, 1 the listener),
  *           n_landmarks 3, obs_dim 11, n_actions 5, episode_len >= 1
- * n_envs is the number of parallel environments of a rollout (SPREAD,
- * ADVERSARY, SPEAKER_LISTENER).
+ *   PUSH:   n_agents 2 (agent 0 the adversary, 1 the good agent),
+ *           n_landmarks 1, obs_dim 8, n_actions 5, episode_len >= 1
+ *   TAG:    n_agents 4 (agents 0..2 the adversaries, 3 the good agent),
+ *           n_landmarks 2 (the obstacles), obs_dim 16, n_actions 5,
+ *           episode_len >= 1
+ * n_envs is the number of parallel environments of a rollout (the particle
+ * scenarios SPREAD, ADVERSARY, SPEAKER_LISTENER, PUSH, TAG).
  * SPREAD reward of agent i after a step (App. B.1), with cover = sum over
  * landmarks of the distance to the nearest agent and coll_i = the number of
  * agents closer than 0.3 to agent i:
@@ -104,6 +112,25 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  * step. Both agents get r = -d(p_1, target) after the step. Observations (11
  * floats): speaker - one-hot of the target, zeros; listener - velocity, the
  * three landmarks - p_1, one-hot of the last message (zeros before the first).
+ * Contact forces (App. B.1 names collisions and obstacles that block the way
+ * but no force law; this is the soft contact model of the particle
+ * environments): disks whose radii sum to dmin at distance d push each other
+ * along the line of centres with force 100 * pen, pen = 0.001 * log(1 +
+ * exp((dmin - d) / 0.001)), computed from the positions before the move and
+ * added to the action forces. SPREAD with MALIB_SPREAD_CONTACT: the agents
+ * (radius 0.15) push each other.
+ * PUSH (App. B.1 simple push): agents of radius 0.15 that push each other, the
+ * spread dynamics otherwise. With d_i = |p_i - landmark| after the step: good
+ * agent r_1 = -d_1, adversary r_0 = d_1 - d_0. Observation of agent i (8
+ * floats): velocity, position, landmark - p_i, the other agent - p_i.
+ * TAG (App. B.1 simple tag): adversaries of radius 0.075 with action force 3
+ * and speed limit 1.0, the good agent of radius 0.05 with action force 4 and
+ * speed limit 1.3, immovable obstacles of radius 0.2; every agent pair and
+ * every agent-obstacle pair collides. After the step an adversary hits the
+ * good agent when closer than 0.125; with h hits, r_3 = -10 h and each
+ * adversary gets 10 h. Observation of agent i (16 floats): velocity, position,
+ * obstacles - p_i, the other agents - p_i (ascending), the good agent's
+ * velocity for an adversary (zeros for the good agent).
  */
 typedef struct malib_env_spec {
     int32_t env_kind;
@@ -205,7 +232,10 @@ int malib_pop_reset(malib_ctx* ctx);
 /*
  * malib_rollout - batched multi-agent rollout (Sec. 3.1, X(theta) ~ P(s, a, s'
  * | a ~ Comb_t); the Actor with k environments of the architecture figure).
- * SPREAD, ADVERSARY and SPEAKER_LISTENER (App. B.1 particle scenarios).
+ * SPREAD, ADVERSARY, SPEAKER_LISTENER, PUSH and TAG (App. B.1 particle
+ * scenarios). Kernels: SPREAD N = 8 (obs 34, bf16 34-256-256-5 policies) on
+ * the tensor cores; SPREAD N = 3 (obs 18) and the other scenarios with fp32
+ * MLPs of hidden width 64, at most 128 environments per combination.
  * pair_ids (host or device) int32 [n_pairs][n_agents] holds one
  * policy id per agent for each combination; the n_envs environments are split
  * evenly and contiguously over the combinations (n_envs % n_pairs == 0).

@@ -79,7 +79,7 @@ struct EvalArgs {
 };
 
 struct RolloutArgs {
-    int32_t env_kind;            // MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY or MALIB_ENV_SPEAKER_LISTENER
+    int32_t env_kind;            // MALIB_ENV_SPREAD or another particle scenario
     const float* arena;
     const int64_t* pol_offset;
     int32_t n_pol;
@@ -99,6 +99,7 @@ struct RolloutArgs {
     uint8_t* done;
     float* logits;               // may be null
     float local_ratio;           // < 0: r_i = -(cover + coll_i); else the weighted reward
+    int32_t contact;             // SPREAD: agents push each other apart (soft contact forces)
 };
 
 // Launchers (return cudaGetLastError() of the launch). `grid_hint` = SM count.

@@ -164,11 +164,23 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
                             "speaker-listener spec needs n_agents 2, n_landmarks 3, obs_dim 11, n_actions 5");
             if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
             break;
+        case MALIB_ENV_PUSH:
+            if (s->n_agents != 2 || s->n_landmarks != 1 || s->obs_dim != 8 || s->n_actions != 5)
+                return fail(c, MALIB_EINVAL, "push spec needs n_agents 2, n_landmarks 1, obs_dim 8, n_actions 5");
+            if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
+            break;
+        case MALIB_ENV_TAG:
+            if (s->n_agents != 4 || s->n_landmarks != 2 || s->obs_dim != 16 || s->n_actions != 5)
+                return fail(c, MALIB_EINVAL, "tag spec needs n_agents 4, n_landmarks 2, obs_dim 16, n_actions 5");
+            if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
+            break;
         default:
             return fail(c, MALIB_EINVAL, "unknown env_kind %d", s->env_kind);
     }
-    if (s->flags & ~(MALIB_DUMP_LOGITS | MALIB_EXACT_EXPECTATION | MALIB_SPREAD_LOCAL_RATIO))
+    if (s->flags & ~(MALIB_DUMP_LOGITS | MALIB_EXACT_EXPECTATION | MALIB_SPREAD_LOCAL_RATIO | MALIB_SPREAD_CONTACT))
         return fail(c, MALIB_EINVAL, "unknown flags 0x%x", s->flags);
+    if ((s->flags & MALIB_SPREAD_CONTACT) && s->env_kind != MALIB_ENV_SPREAD)
+        return fail(c, MALIB_EINVAL, "MALIB_SPREAD_CONTACT applies to SPREAD only");
     if (s->flags & MALIB_SPREAD_LOCAL_RATIO) {
         if (s->env_kind != MALIB_ENV_SPREAD)
             return fail(c, MALIB_EINVAL, "MALIB_SPREAD_LOCAL_RATIO applies to SPREAD only");
@@ -668,7 +680,8 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
         return fail(c, MALIB_ESTATE, "rollout spec differs from the population's environment");
     // scenarios of the fp32 rollout kernel other than spread (one policy width, hidden 64)
     const bool other = spec->env_kind == MALIB_ENV_ADVERSARY ||
-                       spec->env_kind == MALIB_ENV_SPEAKER_LISTENER;
+                       spec->env_kind == MALIB_ENV_SPEAKER_LISTENER || spec->env_kind == MALIB_ENV_PUSH ||
+                       spec->env_kind == MALIB_ENV_TAG;
     if (spec->env_kind != MALIB_ENV_SPREAD && !other)
         return fail(c, MALIB_EUNSUPPORTED, "rollout is built for the particle environments");
     if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");
@@ -715,6 +728,7 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     a.obs_pad = (spec->obs_dim + 3) / 4 * 4;
     a.episode_len = spec->episode_len;
     a.local_ratio = (spec->flags & MALIB_SPREAD_LOCAL_RATIO) ? spec->local_ratio : -1.0f;
+    a.contact = (spec->flags & MALIB_SPREAD_CONTACT) ? 1 : 0;
     a.n_envs = spec->n_envs;
     a.n_episodes = n_episodes;
     a.seed = seed;

@@ -4,6 +4,7 @@
 // operation so that any two implementations of these steps agree bit for bit.
 #pragma once
 
+#include "contact.cuh"
 #include "device_common.cuh"
 
 namespace malib {
@@ -102,15 +103,25 @@ constexpr float kCollideSq = 0x1.70a3d8p-4f;
 // square root is monotone, so the minimum over agents of the rounded distances
 // to a landmark equals the rounded root of the minimum squared distance: one
 // root per landmark gives the same bits as one per (landmark, agent).
-template <int N>
+// kContact: the agents (disks of radius 0.15) also push each other apart with
+// the soft contact forces (contact.cuh), taken from the positions before the
+// move and added to the action forces; landmarks do not collide.
+template <int N, bool kContact = false>
 __device__ __forceinline__ void spread_step(SpreadEnv<N>& s, const int (&act)[N], float (&r)[N],
                                             float local_ratio) {
+    float Fx[N], Fy[N];
+#pragma unroll
+    for (int i = 0; i < N; ++i) unit_force(act[i], Fx[i], Fy[i]);
+    if constexpr (kContact) {
+        float rad[N];
+#pragma unroll
+        for (int i = 0; i < N; ++i) rad[i] = 0.15f;
+        add_contacts<N, 0>(s.px, s.py, rad, nullptr, nullptr, nullptr, Fx, Fy);
+    }
 #pragma unroll
     for (int i = 0; i < N; ++i) {
-        const float fx = act[i] == 1 ? 1.f : (act[i] == 2 ? -1.f : 0.f);
-        const float fy = act[i] == 3 ? 1.f : (act[i] == 4 ? -1.f : 0.f);
-        s.vx[i] = __fadd_rn(__fmul_rn(s.vx[i], 0.75f), __fmul_rn(fx, 0.1f));
-        s.vy[i] = __fadd_rn(__fmul_rn(s.vy[i], 0.75f), __fmul_rn(fy, 0.1f));
+        s.vx[i] = __fadd_rn(__fmul_rn(s.vx[i], 0.75f), __fmul_rn(Fx[i], 0.1f));
+        s.vy[i] = __fadd_rn(__fmul_rn(s.vy[i], 0.75f), __fmul_rn(Fy[i], 0.1f));
         s.px[i] = __fadd_rn(s.px[i], __fmul_rn(s.vx[i], 0.1f));
         s.py[i] = __fadd_rn(s.py[i], __fmul_rn(s.vy[i], 0.1f));
     }

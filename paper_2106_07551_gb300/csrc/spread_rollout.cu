@@ -13,10 +13,13 @@
 // engine. The observation tile is laid out [row][agent][obs_pad], the order of
 // the trajectory, so each episode's observations of a step leave shared memory
 // as one bulk copy; actions, rewards and done flags are stored per thread.
-// The same kernel, templated on the scenario, runs the simple adversary and the
-// simple speaker listener (App. B.1) with their own environment code.
+// The same kernel, templated on the scenario, runs the simple adversary, the
+// simple speaker listener, the simple push and the simple tag (App. B.1) with
+// their own environment code, and spread with contact forces between agents.
 #include "adversary_env.cuh"
+#include "push_env.cuh"
 #include "sl_env.cuh"
+#include "tag_env.cuh"
 #include "device_common.cuh"
 #include "internal.h"
 #include "mlp_f32.cuh"
@@ -26,17 +29,26 @@ namespace malib {
 
 namespace {
 
+// Shared memory: the N policies, the observation tile X, layer 1's output H1
+// and the logits LG. When the tiles of all N agents do not fit (the simple tag),
+// the kernel runs per agent (kPerAgent): X and LG hold one agent's rows, each
+// agent's observations are built just before its pass and stored to the
+// trajectory from registers, and its action is drawn right after it.
 template <int N, int IN, int H>
 struct SpreadF32Smem {
     static_assert(H == 64, "the 256-row engine has 64 hidden units");
     using M = MlpF32R8<IN, 5>;
     using L = F32Layout<IN, H, 5>;
     static constexpr int R = M::kRows;            // 2 episode slots x 128 envs
+    static constexpr size_t kAllBytes =
+        (size_t)(N * L::kSize + N * R * M::XS + R * M::HS + N * R * M::LS) * 4;
+    static constexpr bool kPerAgent = kAllBytes > 232448;
+    static constexpr int kNX = kPerAgent ? 1 : N;   // agents' tiles held at once
     static constexpr int kW = 0;
     static constexpr int kX = kW + N * L::kSize;
-    static constexpr int kH1 = kX + N * R * M::XS;
+    static constexpr int kH1 = kX + kNX * R * M::XS;
     static constexpr int kLG = kH1 + R * M::HS;
-    static constexpr int kFloats = kLG + N * R * M::LS;
+    static constexpr int kFloats = kLG + kNX * R * M::LS;
     static constexpr size_t kBytes = (size_t)kFloats * 4;
     static_assert(kBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
 };
@@ -44,8 +56,10 @@ struct SpreadF32Smem {
 // kScen: kSpread - cooperative spread (N agents, N landmarks); kAdversary - the
 // simple adversary (N = 3, two landmarks, obs 14); kSpeakerListener - the simple
 // speaker listener (N = 2, three landmarks, obs 11; the speaker may take
-// actions 0..2 only).
-constexpr int kSpread = 0, kAdversary = 1, kSpeakerListener = 2;
+// actions 0..2 only); kPush - the simple push (N = 2, one landmark, obs 8);
+// kTag - the simple tag (N = 4, two obstacles, obs 16); kSpreadContact -
+// spread whose agents also push each other apart.
+constexpr int kSpread = 0, kAdversary = 1, kSpeakerListener = 2, kPush = 3, kTag = 4, kSpreadContact = 5;
 
 template <int kScen, int N>
 struct ScenarioEnv {
@@ -59,12 +73,22 @@ template <int N>
 struct ScenarioEnv<kSpeakerListener, N> {
     using type = SlEnv;
 };
+template <int N>
+struct ScenarioEnv<kPush, N> {
+    using type = PushEnv;
+};
+template <int N>
+struct ScenarioEnv<kTag, N> {
+    using type = TagEnv;
+};
 
 template <int N, int IN, int H, int kScen = kSpread>
 __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs a) {
     static_assert(kScen != kAdversary || (N == 3 && IN == kAdvObs), "the simple adversary has 3 agents, obs 14");
     static_assert(kScen != kSpeakerListener || (N == 2 && IN == kSlObs),
                   "the simple speaker listener has 2 agents, obs 11");
+    static_assert(kScen != kPush || (N == 2 && IN == kPushObs), "the simple push has 2 agents, obs 8");
+    static_assert(kScen != kTag || (N == 4 && IN == kTagObs), "the simple tag has 4 agents, obs 16");
     using SM = SpreadF32Smem<N, IN, H>;
     using M = typename SM::M;
     using L = typename SM::L;
@@ -79,7 +103,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 
     const int tid = threadIdx.x;
     const int slot = tid >> 7, v = tid & 127;        // episode slot, env of the combination
-    for (int i = tid; i < R * N * XS; i += blockDim.x) X[i] = 0.f;
+    for (int i = tid; i < R * SM::kNX * XS; i += blockDim.x) X[i] = 0.f;
     if (tid == 0) mbar_init(&bar, 1);
     __syncthreads();
     uint32_t parity = 0;
@@ -134,16 +158,76 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
         if (mine) {
             if constexpr (kScen == kAdversary) adv_reset(s, g, a.seed);
             else if constexpr (kScen == kSpeakerListener) sl_reset(s, g, a.seed);
+            else if constexpr (kScen == kPush) push_reset(s, g, a.seed);
+            else if constexpr (kScen == kTag) tag_reset(s, g, a.seed);
             else spread_reset<N>(s, g, a.seed);
         }
 
         for (int t = 0; t < T; ++t) {
+            if constexpr (SM::kPerAgent) {
+                // one agent at a time: its observations (to X and the
+                // trajectory), its pass, its draw
+                int act[N];
+                const int64_t ix = ((ep * T + t) * a.n_envs + env) * N;
+#pragma unroll
+                for (int i = 0; i < N; ++i) {
+                    if (mine) {
+                        float o[XS];
+                        if constexpr (kScen == kTag) tag_obs<XS>(s, i, o);
+                        else if constexpr (kScen == kPush) push_obs<XS>(s, i, o);
+                        else if constexpr (kScen == kAdversary) adv_obs<XS>(s, i, o);
+                        else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, i, o);
+                        else spread_obs<N, XS>(s, i, o);
+                        float4* xr = reinterpret_cast<float4*>(X + tid * XS);
+                        float4* gr = reinterpret_cast<float4*>(a.obs + (ix + i) * XS);
+#pragma unroll
+                        for (int q = 0; q < XS / 4; ++q) {
+                            const float4 f = make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                            xr[q] = f;
+                            gr[q] = f;
+                        }
+                    }
+                    __syncthreads();
+                    const float* w = Ws + i * L::kSize;
+                    M::template layer1<XS>(X, H1, w + L::kW1T, w + L::kB1);
+                    M::layer23(H1, LG, w + L::kW2T, w + L::kB2, w + L::kW3, w + L::kB3);
+                    if (mine) {
+                        // LG is rewritten only after the next pass's layer-1 barrier
+                        float lg[5];
+#pragma unroll
+                        for (int k = 0; k < 5; ++k) lg[k] = LG[tid * M::LS + k];
+                        const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
+                        const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : 0x1Fu;
+                        act[i] = sample_masked<5>(lg, legal, uu);
+                        if (a.logits)
+#pragma unroll
+                            for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
+                    }
+                }
+                if (mine) {
+                    float r[N];
+                    if constexpr (kScen == kAdversary) adv_step(s, act, r);
+                    else if constexpr (kScen == kSpeakerListener) sl_step(s, act, r);
+                    else if constexpr (kScen == kPush) push_step(s, act, r);
+                    else if constexpr (kScen == kTag) tag_step(s, act, r);
+                    else spread_step<N, kScen == kSpreadContact>(s, act, r, a.local_ratio);
+#pragma unroll
+                    for (int i = 0; i < N; ++i) {
+                        a.action[ix + i] = (uint8_t)act[i];
+                        a.reward[ix + i] = r[i];
+                    }
+                    a.done[(ep * T + t) * a.n_envs + env] = (t == T - 1) ? 1 : 0;
+                }
+                continue;
+            }
             if (mine) {
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
                     float o[XS];
                     if constexpr (kScen == kAdversary) adv_obs<XS>(s, i, o);
                     else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, i, o);
+                    else if constexpr (kScen == kPush) push_obs<XS>(s, i, o);
+                    else if constexpr (kScen == kTag) tag_obs<XS>(s, i, o);
                     else spread_obs<N, XS>(s, i, o);
                     float4* xr = reinterpret_cast<float4*>(X + (tid * N + i) * XS);
 #pragma unroll
@@ -188,7 +272,9 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                 }
                 if constexpr (kScen == kAdversary) adv_step(s, act, r);
                 else if constexpr (kScen == kSpeakerListener) sl_step(s, act, r);
-                else spread_step<N>(s, act, r, a.local_ratio);
+                else if constexpr (kScen == kPush) push_step(s, act, r);
+                else if constexpr (kScen == kTag) tag_step(s, act, r);
+                else spread_step<N, kScen == kSpreadContact>(s, act, r, a.local_ratio);
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
                     a.action[ix + i] = (uint8_t)act[i];
@@ -235,7 +321,17 @@ cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm
         if (hidden == 64) return launch_spread_nih<2, kSlObs, 64, kSpeakerListener>(a, n_sm, s);
         return cudaErrorInvalidValue;
     }
-    if (a.n_agents == 3 && a.obs_dim == 18 && hidden == 64) return launch_spread_nih<3, 18, 64>(a, n_sm, s);
+    if (a.env_kind == MALIB_ENV_PUSH) {
+        if (hidden == 64) return launch_spread_nih<2, kPushObs, 64, kPush>(a, n_sm, s);
+        return cudaErrorInvalidValue;
+    }
+    if (a.env_kind == MALIB_ENV_TAG) {
+        if (hidden == 64) return launch_spread_nih<4, kTagObs, 64, kTag>(a, n_sm, s);
+        return cudaErrorInvalidValue;
+    }
+    if (a.n_agents == 3 && a.obs_dim == 18 && hidden == 64)
+        return a.contact ? launch_spread_nih<3, 18, 64, kSpreadContact>(a, n_sm, s)
+                         : launch_spread_nih<3, 18, 64>(a, n_sm, s);
     return cudaErrorInvalidValue;
 }
 

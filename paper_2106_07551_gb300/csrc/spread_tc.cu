@@ -82,6 +82,8 @@ __device__ __forceinline__ bool pair_valid(const RolloutArgs& a, int pair) {
     return ok;
 }
 
+// kContact: the agents also push each other apart (soft contact forces).
+template <bool kContact>
 __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t stage_bar;             // W1 and the biases staged
@@ -285,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
 #pragma unroll
                     for (int i = 0; i < kN; ++i) act[i] = ag[i * 128 + e];
                     float r[kN];
-                    spread_step<kN>(s, act, r, a.local_ratio);
+                    spread_step<kN, kContact>(s, act, r, a.local_ratio);
 #pragma unroll
                     for (int i = 0; i < kN; ++i) a.reward[ix + i] = r[i];
                     a.done[(ep * T + t) * a.n_envs + env] = (t == T - 1) ? 1 : 0;
@@ -305,15 +307,20 @@ bool spread_tc_supported(int n_agents, int obs_dim, int n_actions, int64_t envs_
            envs_per_pair <= 128;
 }
 
-cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s) {
-    if (a.n_pairs == 0 || a.n_episodes == 0) return cudaSuccess;
-    cudaError_t err = cudaFuncSetAttribute(spread_rollout_tc_kernel,
+template <bool kContact>
+cudaError_t launch_tc(const RolloutArgs& a, int n_sm, cudaStream_t s) {
+    cudaError_t err = cudaFuncSetAttribute(spread_rollout_tc_kernel<kContact>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (err != cudaSuccess) return err;
     const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
     const int64_t ctas = items < n_sm ? items : n_sm;
-    spread_rollout_tc_kernel<<<(unsigned)ctas, kThreads, kSmem, s>>>(a);
+    spread_rollout_tc_kernel<kContact><<<(unsigned)ctas, kThreads, kSmem, s>>>(a);
     return cudaGetLastError();
+}
+
+cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s) {
+    if (a.n_pairs == 0 || a.n_episodes == 0) return cudaSuccess;
+    return a.contact ? launch_tc<true>(a, n_sm, s) : launch_tc<false>(a, n_sm, s);
 }
 
 }  // namespace malib

@@ -26,7 +26,7 @@ import numpy as np
 SEED_BASE = 2106075510
 
 ENV_KUHN, ENV_LEDUC, ENV_SPREAD, ENV_ADVERSARY = 1, 2, 3, 4
-ENV_SPEAKER_LISTENER = 5
+ENV_SPEAKER_LISTENER, ENV_PUSH, ENV_TAG = 5, 6, 7
 POL_TABULAR, POL_MLP = 1, 2
 F32, BF16 = 0, 1
 
@@ -174,6 +174,42 @@ def speaker_listener(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_epis
         w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
     n_pairs = max(1, n_envs // envs_per_pair)
     w.pair_ids = rng.integers(0, pop, size=(n_pairs, 2)).astype(np.int32)
+    return w
+
+
+def push(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_episodes: int = 1,
+         episode_len: int = 25, envs_per_pair: int = 128, seed: int = SEED_BASE + 8,
+         with_bias: bool = False, name: str | None = None) -> Workload:
+    """Simple push (App. B.1): agent 0 the adversary, agent 1 the good agent,
+    one landmark, contact forces between the agents; MLP 8-hidden-hidden-5
+    fp32 policies from one shared pool, assigned by the seed per (block of
+    envs_per_pair envs, agent slot)."""
+    rng = np.random.default_rng(seed)
+    dims = (8, hidden, hidden, 5)
+    w = Workload(name or f"push_{n_envs}env_mlp{hidden}_f32", ENV_PUSH, 2, 1, 8, 5,
+                 episode_len, n_envs, n_episodes=n_episodes, seed=seed)
+    for _ in range(pop):
+        w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
+    n_pairs = max(1, n_envs // envs_per_pair)
+    w.pair_ids = rng.integers(0, pop, size=(n_pairs, 2)).astype(np.int32)
+    return w
+
+
+def tag(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_episodes: int = 1,
+        episode_len: int = 25, envs_per_pair: int = 128, seed: int = SEED_BASE + 9,
+        with_bias: bool = False, name: str | None = None) -> Workload:
+    """Simple tag (App. B.1): agents 0..2 the adversaries, agent 3 the good
+    agent, two obstacles, contact forces among all of them; MLP
+    16-hidden-hidden-5 fp32 policies from one shared pool, assigned by the seed
+    per (block of envs_per_pair envs, agent slot)."""
+    rng = np.random.default_rng(seed)
+    dims = (16, hidden, hidden, 5)
+    w = Workload(name or f"tag_{n_envs}env_mlp{hidden}_f32", ENV_TAG, 4, 2, 16, 5,
+                 episode_len, n_envs, n_episodes=n_episodes, seed=seed)
+    for _ in range(pop):
+        w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
+    n_pairs = max(1, n_envs // envs_per_pair)
+    w.pair_ids = rng.integers(0, pop, size=(n_pairs, 4)).astype(np.int32)
     return w
 
 
