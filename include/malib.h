@@ -375,6 +375,57 @@ int malib_meta_aggregate(malib_ctx* ctx, const double* payoff, int32_t n_games, 
 int malib_exploitability(malib_ctx* ctx, const int32_t* ids0, const double* x, int32_t n0,
                          const int32_t* ids1, const double* y, int32_t n1, double* out);
 
+/* ---- learner side: the next stage of the loop, consuming traj_out ---- */
+
+/*
+ * malib_learn_pg - one independent learner's policy-gradient step (Sec. 3.3
+ * "Independent Learning": one learner per policy, trained on its own agents'
+ * experience; App. C.2: the training workflow samples rollout episodes into a
+ * batch for the learner's optimize()). For policy `policy_id` its samples S
+ * are every (episode, step, environment, agent) of the rollout in traj whose
+ * combination (pair_ids [n_pairs][n_agents], host or device, the table the
+ * rollout used) gives that agent policy_id; M = |S|. With G the discounted
+ * return-to-go of a sample within its episode (G_t = r_t + gamma G_{t+1}),
+ * b the mean of G over S and H the entropy of the policy's softmax over the
+ * 5 actions, the loss is
+ *   L = -(1/M) sum_S [ (G - b) log pi(a | o) + entropy_coef H(pi(. | o)) ]
+ * and grad_out (host or device, float [P]) receives dL/dparams in the
+ * malib_policy_desc parameter layout (W1, b1, W2, b2, W3, b3; P parameters).
+ * stats_out (optional, host or device, double [4]) receives M, b, L and the
+ * mean entropy. traj: obs, action and reward of malib_rollout (device memory
+ * of the context's device, the rollout's spec, n_episodes and episode_len).
+ * Built for particle-scenario populations of fp32 MLPs in-64-64-5 with in
+ * <= 32 (EUNSUPPORTED otherwise); gamma in [0, 1], entropy_coef >= 0.
+ * Deterministic (fixed-order sums, no atomics). A host output makes the call
+ * wait for the stream. Errors: EINVAL, ESTATE, EUNSUPPORTED.
+ */
+int malib_learn_pg(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                   int64_t n_episodes, const malib_traj* traj, int32_t policy_id, float gamma,
+                   float entropy_coef, float* grad_out, double* stats_out);
+
+/*
+ * malib_adam_step - one Adam step (the optimizer of App. C.2's training
+ * config; Kingma and Ba, with bias correction) on n parameters, in place:
+ *   m <- beta1 m + (1 - beta1) g;  v <- beta2 v + (1 - beta2) g^2;
+ *   params <- params - lr (m / (1 - beta1^step)) / (sqrt(v / (1 - beta2^step)) + eps).
+ * params, grad, m, v: float [n] device buffers of the context's device (the
+ * caller owns them; m and v start at zero). step >= 1 counts the calls.
+ * Asynchronous on the context's stream. Errors: EINVAL.
+ */
+int malib_adam_step(malib_ctx* ctx, float* params, const float* grad, float* m, float* v, int64_t n,
+                    int64_t step, float lr, float beta1, float beta2, float eps);
+
+/*
+ * malib_pop_update - replaces the parameters of loaded policy `policy_id`
+ * (Sec. 3.1: the learner's new policy goes back into the population that the
+ * next rollouts and evaluations use). params: host or device, the
+ * malib_policy_desc layout of the policy's shape, nbytes its size. The
+ * policy's kernel image is rebuilt in place; work already queued on the
+ * context's stream sees the old parameters. Returns once the caller's buffer
+ * may be reused. Errors: EINVAL, ESTATE.
+ */
+int malib_pop_update(malib_ctx* ctx, int32_t policy_id, const float* params, int64_t nbytes);
+
 /* ---- measurement and self-test entry points (used by tests and the benchmark) ---- */
 
 /* Total decisions (env-steps: one decision by the acting seat) played by the

@@ -268,6 +268,29 @@ class Context:
                                              _ptr(y), _ptr(row_out), _ptr(col_out),
                                              _ptr(value_out)))
 
+    def learn_pg(self, spec, pair_ids, n_episodes, traj, policy_id, gamma, entropy_coef, grad_out,
+                 stats_out=None):
+        """Policy-gradient step of one policy on a rollout's samples: the
+        gradient (policy-parameter layout) into grad_out and (M, baseline,
+        loss, mean entropy) into stats_out (fp64 [4]); host or device buffers."""
+        t = Traj(_ptr(traj["obs"]), _ptr(traj["action"]), _ptr(traj["reward"]), None, None)
+        _check(self.lib, self.handle,
+               self.lib.malib_learn_pg(self.handle, C.byref(spec), _ptr(pair_ids), int(pair_ids.shape[0]),
+                                       n_episodes, C.byref(t), policy_id, gamma, entropy_coef,
+                                       _ptr(grad_out), _ptr(stats_out) if stats_out is not None else None))
+
+    def adam_step(self, params, grad, m, v, step, lr, beta1=0.9, beta2=0.999, eps=1e-8):
+        """One Adam step on device buffers (parameters, gradient, moments) in place."""
+        n = int(params.numel()) if hasattr(params, "numel") else int(params.size)
+        _check(self.lib, self.handle,
+               self.lib.malib_adam_step(self.handle, _ptr(params), _ptr(grad), _ptr(m), _ptr(v), n, step,
+                                        lr, beta1, beta2, eps))
+
+    def pop_update(self, policy_id, params):
+        """Replaces a loaded policy's parameters (same shape), host or device."""
+        nbytes = int(params.numel()) * 4 if hasattr(params, "numel") else int(params.size) * 4
+        _check(self.lib, self.handle, self.lib.malib_pop_update(self.handle, policy_id, _ptr(params), nbytes))
+
     def exploitability(self, ids0, x, ids1, y):
         """(b0, b1, exploitability) of the seat mixtures (ids with fp64 weights)."""
         ids0 = np.ascontiguousarray(ids0, np.int32)

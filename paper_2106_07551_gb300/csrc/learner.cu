@@ -1,0 +1,497 @@
+// Learner-side update on the device: one independent learner's policy-gradient
+// step on the samples a rollout wrote (Sec. 3.3 "Independent Learning": one
+// learner per policy, trained on its own agents' experience; App. C.2: the
+// training workflow's optimize() with Adam and an entropy coefficient).
+//
+// For policy p with samples S_p (each (episode, step, environment, agent) whose
+// combination gives that agent policy p; M = |S_p|):
+//   L = -(1/M) sum_i [ (G_i - b) log pi(a_i | o_i) + beta H(pi(. | o_i)) ],
+// G the discounted return-to-go within the episode, b the mean of G over S_p,
+// H the entropy of the softmax over the 5 actions. The gradient by the chain
+// rule: dL/dz_j = (1/M) [ (G - b)(pi_j - [j = a]) + beta pi_j (log pi_j + H) ],
+// back through W3, the ReLUs (pre-activation > 0) and W2, W1.
+//
+// Kernels, in stream order:
+//  1. learn_slots_kernel: the (combination, agent) slots acting with p, in
+//     ascending order (one block).
+//  2. learn_returns_kernel: G of every sample by the backward recursion
+//     G_t = r_t + gamma G_{t+1}, one thread per (slot, episode, env), and
+//     per-block fp64 sums of G.
+//  3. learn_baseline_kernel: M and b = sum G / M in a fixed order (one block).
+//  4. learn_grad_kernel: persistent CTAs over tiles of 128 samples: forward
+//     (fp32 FMA, hidden 64), logits, softmax, dL/dz, the backward pass, and
+//     the weight gradients accumulated in registers over the CTA's tiles;
+//     each CTA writes its partial gradient.
+//  5. learn_reduce_kernel: the partials summed over CTAs in a fixed order into
+//     the gradient (the malib_policy_desc layout) and the loss statistics.
+// Deterministic: no atomics, every sum in a fixed order.
+// Adam (Kingma and Ba): learn_adam_kernel, elementwise with bias correction.
+#include <cmath>
+
+#include "device_common.cuh"
+#include "internal.h"
+
+namespace malib {
+
+namespace {
+
+constexpr int kH = 64, kA = 5, kTile = 128, kThreads = 256;
+constexpr int kHS = kH + 1;          // row stride of the per-sample hidden tiles
+constexpr int kXS = kLearnMaxIn + 1;   // row stride of the observation tile
+
+// Shared-memory layout of learn_grad_kernel (floats).
+constexpr int kSW1T = 0;                          // [in][64]: W1T[k][j] = W1[j][k]
+constexpr int kSB1 = kSW1T + kLearnMaxIn * kH;
+constexpr int kSW2T = kSB1 + kH;                  // [64][64]: W2T[k][j] = W2[j][k]
+constexpr int kSW2 = kSW2T + kH * kH;             // [64][64]: W2[j][k]
+constexpr int kSB2 = kSW2 + kH * kH;
+constexpr int kSW3 = kSB2 + kH;                   // [5][64]
+constexpr int kSB3 = kSW3 + kA * kH;              // [8]
+constexpr int kSX = kSB3 + 8;                     // [128][kXS]
+constexpr int kSH1 = kSX + kTile * kXS;           // [128][65] post-ReLU layer 1
+constexpr int kSH2 = kSH1 + kTile * kHS;          // [128][65] post-ReLU layer 2
+constexpr int kSD2 = kSH2 + kTile * kHS;          // [128][65] dL/d(pre-activation 2)
+constexpr int kSD1 = kSD2 + kTile * kHS;          // [128][65] dL/d(pre-activation 1)
+constexpr int kSDZ = kSD1 + kTile * kHS;          // [128][8] dL/dz
+constexpr int kSFloats = kSDZ + kTile * 8;
+constexpr size_t kSBytes = (size_t)kSFloats * 4;
+static_assert(kSBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
+
+__global__ void __launch_bounds__(1024) learn_slots_kernel(LearnArgs a) {
+    __shared__ int warp_n[32];
+    __shared__ int base;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int total = a.n_pairs * a.n_agents;
+    if (tid == 0) base = 0;
+    __syncthreads();
+    for (int c0 = 0; c0 < total; c0 += blockDim.x) {
+        const int i = c0 + tid;
+        const int pid = i < total ? a.pairs[i] : -1;
+        if (i < total && (pid < 0 || pid >= a.n_pol)) atomicOr(a.err, ERRBIT_BAD_PAIR);
+        const bool mine = i < total && pid == a.policy;
+        const unsigned m = __ballot_sync(0xffffffffu, mine);
+        if (lane == 0) warp_n[warp] = __popc(m);
+        __syncthreads();
+        int before = base;
+        for (int w = 0; w < warp; ++w) before += warp_n[w];
+        if (mine) a.slots[before + __popc(m & ((1u << lane) - 1u))] = i;   // c * n_agents + k
+        __syncthreads();
+        if (tid == 0) {
+            int n = 0;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) n += warp_n[w];
+            base += n;
+        }
+        __syncthreads();
+    }
+    if (tid == 0) *a.n_slots = base;
+}
+
+__global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
+    __shared__ double red[256];
+    const int epp = (int)(a.n_envs / a.n_pairs);
+    const int64_t n_seq = (int64_t)(*a.n_slots) * a.n_episodes * epp;
+    double sum = 0.0;
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < n_seq;
+         q += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t slot = q / (a.n_episodes * epp);
+        const int64_t rem = q - slot * a.n_episodes * epp;
+        const int64_t e = rem / epp;
+        const int r = (int)(rem - e * epp);
+        const int ck = a.slots[slot];
+        const int c = ck / a.n_agents, k = ck - c * a.n_agents;
+        const int64_t env = (int64_t)c * epp + r;
+        float G = 0.f;
+        for (int t = a.T - 1; t >= 0; --t) {
+            G = __fadd_rn(a.reward[((e * a.T + t) * a.n_envs + env) * a.n_agents + k], __fmul_rn(a.gamma, G));
+            a.G[((slot * a.n_episodes + e) * a.T + t) * epp + r] = G;
+            sum += (double)G;
+        }
+    }
+    red[threadIdx.x] = sum;
+    __syncthreads();
+    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+        if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) a.gsum[blockIdx.x] = red[0];
+}
+
+__global__ void learn_baseline_kernel(LearnArgs a, int n_blocks) {
+    if (threadIdx.x != 0) return;
+    double s = 0.0;
+    for (int b = 0; b < n_blocks; ++b) s += a.gsum[b];
+    const int epp = (int)(a.n_envs / a.n_pairs);
+    const double M = (double)(*a.n_slots) * (double)a.n_episodes * (double)a.T * (double)epp;
+    a.stats[0] = M;
+    a.stats[1] = M > 0 ? s / M : 0.0;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
+    extern __shared__ __align__(16) float sm[];
+    const int tid = threadIdx.x;
+    const int in = a.in;
+    const float* pol = a.arena + a.pol_off;
+    // the policy (F32Layout: W1T [in][64], b1, W2T [64][64], b2, W3 [5][64], b3)
+    for (int i = tid; i < in * kH; i += kThreads) sm[kSW1T + i] = pol[i];
+    for (int i = tid; i < kH; i += kThreads) sm[kSB1 + i] = pol[in * kH + i];
+    for (int i = tid; i < kH * kH; i += kThreads) {
+        const float w = pol[in * kH + kH + i];               // W2T[k][j], i = k * 64 + j
+        sm[kSW2T + i] = w;
+        sm[kSW2 + (i & (kH - 1)) * kH + (i >> 6)] = w;        // W2[j][k]
+    }
+    for (int i = tid; i < kH; i += kThreads) sm[kSB2 + i] = pol[in * kH + kH + kH * kH + i];
+    for (int i = tid; i < kA * kH; i += kThreads) sm[kSW3 + i] = pol[in * kH + 2 * kH + kH * kH + i];
+    if (tid < kA) sm[kSB3 + tid] = pol[in * kH + 2 * kH + kH * kH + kA * kH + tid];
+    __syncthreads();
+
+    const int epp = (int)(a.n_envs / a.n_pairs);
+    const int64_t M = (int64_t)(*a.n_slots) * a.n_episodes * a.T * epp;
+    const float invM = M > 0 ? (float)(1.0 / (double)M) : 0.f;
+    const float base = (float)a.stats[1];
+    const int64_t n_tiles = (M + kTile - 1) / kTile;
+
+    // this thread's gradient entries, accumulated over the CTA's tiles
+    const int jb = tid >> 4, kb = tid & 15;                  // dW2: rows 4 jb.., cols 4 kb..
+    float gW2[4][4] = {};
+    const int nW1 = kH * in;                                 // dW1 entries t + 256 q
+    float gW1[(kH * kLearnMaxIn + kThreads - 1) / kThreads] = {};
+    float gW3[2] = {};                                       // entries t, t + 256 of [5][64]
+    float gB = 0.f;                                          // b1 (t < 64), b2 (64..127), b3 (128..132)
+    float lsum = 0.f, hsum = 0.f;                            // loss and entropy of this thread's samples
+    const int sg = tid >> 4, ng = tid & 15;                  // layers: samples 8 sg.., neurons 4 ng..
+
+    float* X = sm + kSX;
+    float* H1 = sm + kSH1;
+    float* H2 = sm + kSH2;
+    float* D2 = sm + kSD2;
+    float* D1 = sm + kSD1;
+    float* DZ = sm + kSDZ;
+    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+        const int64_t s0 = tile * kTile;
+        // the tile's observations (zero rows past M)
+        for (int i = tid; i < kTile * in; i += kThreads) {
+            const int row = i / in, k = i - row * in;
+            const int64_t s = s0 + row;
+            float v = 0.f;
+            if (s < M) {
+                const int r = (int)(s % epp);
+                const int64_t q = s / epp;                    // (slot, e, t)
+                const int t = (int)(q % a.T);
+                const int64_t q2 = q / a.T;
+                const int64_t e = q2 % a.n_episodes, slot = q2 / a.n_episodes;
+                const int ck = a.slots[slot];
+                const int c = ck / a.n_agents, ka = ck - c * a.n_agents;
+                const int64_t env = (int64_t)c * epp + r;
+                v = a.obs[(((e * a.T + t) * a.n_envs + env) * a.n_agents + ka) * a.xs + k];
+            }
+            X[row * kXS + k] = v;
+        }
+        __syncthreads();
+        // layer 1: H1 = relu(W1 x + b1)
+        {
+            float acc[8][4];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) acc[i][q] = sm[kSB1 + 4 * ng + q];
+            for (int k = 0; k < in; ++k) {
+                const float4 w = *reinterpret_cast<const float4*>(sm + kSW1T + k * kH + 4 * ng);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float x = X[(8 * sg + i) * kXS + k];
+                    acc[i][0] = fmaf(w.x, x, acc[i][0]);
+                    acc[i][1] = fmaf(w.y, x, acc[i][1]);
+                    acc[i][2] = fmaf(w.z, x, acc[i][2]);
+                    acc[i][3] = fmaf(w.w, x, acc[i][3]);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) H1[(8 * sg + i) * kHS + 4 * ng + q] = fmaxf(acc[i][q], 0.f);
+        }
+        __syncthreads();
+        // layer 2: H2 = relu(W2 h1 + b2)
+        {
+            float acc[8][4];
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) acc[i][q] = sm[kSB2 + 4 * ng + q];
+#pragma unroll 4
+            for (int k = 0; k < kH; ++k) {
+                const float4 w = *reinterpret_cast<const float4*>(sm + kSW2T + k * kH + 4 * ng);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float x = H1[(8 * sg + i) * kHS + k];
+                    acc[i][0] = fmaf(w.x, x, acc[i][0]);
+                    acc[i][1] = fmaf(w.y, x, acc[i][1]);
+                    acc[i][2] = fmaf(w.z, x, acc[i][2]);
+                    acc[i][3] = fmaf(w.w, x, acc[i][3]);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) H2[(8 * sg + i) * kHS + 4 * ng + q] = fmaxf(acc[i][q], 0.f);
+        }
+        __syncthreads();
+        // logits, softmax and dL/dz, one sample per thread
+        if (tid < kTile) {
+            const int64_t s = s0 + tid;
+            float dz[kA] = {0.f, 0.f, 0.f, 0.f, 0.f};
+            if (s < M) {
+                const int r = (int)(s % epp);
+                const int64_t q = s / epp;
+                const int t = (int)(q % a.T);
+                const int64_t q2 = q / a.T;
+                const int64_t e = q2 % a.n_episodes, slot = q2 / a.n_episodes;
+                const int ck = a.slots[slot];
+                const int c = ck / a.n_agents, ka = ck - c * a.n_agents;
+                const int64_t env = (int64_t)c * epp + r;
+                const int act = a.action[((e * a.T + t) * a.n_envs + env) * a.n_agents + ka];
+                const float adv = a.G[s] - base;
+                float z[kA];
+#pragma unroll
+                for (int j = 0; j < kA; ++j) z[j] = sm[kSB3 + j];
+                for (int h = 0; h < kH; ++h) {
+                    const float x = H2[tid * kHS + h];
+#pragma unroll
+                    for (int j = 0; j < kA; ++j) z[j] = fmaf(sm[kSW3 + j * kH + h], x, z[j]);
+                }
+                float m = z[0];
+#pragma unroll
+                for (int j = 1; j < kA; ++j) m = fmaxf(m, z[j]);
+                float S = 0.f;
+#pragma unroll
+                for (int j = 0; j < kA; ++j) S += expf(z[j] - m);
+                const float lS = logf(S);
+                float logp[kA], pi[kA], H = 0.f;
+#pragma unroll
+                for (int j = 0; j < kA; ++j) {
+                    logp[j] = z[j] - m - lS;
+                    pi[j] = expf(logp[j]);
+                    H -= pi[j] * logp[j];
+                }
+                float lp_a = logp[0];
+#pragma unroll
+                for (int j = 1; j < kA; ++j)
+                    if (j == act) lp_a = logp[j];
+#pragma unroll
+                for (int j = 0; j < kA; ++j)
+                    dz[j] = (adv * (pi[j] - (j == act ? 1.f : 0.f)) + a.beta * pi[j] * (logp[j] + H)) * invM;
+                lsum -= adv * lp_a + a.beta * H;
+                hsum += H;
+            }
+#pragma unroll
+            for (int j = 0; j < kA; ++j) DZ[tid * 8 + j] = dz[j];
+        }
+        __syncthreads();
+        // D2 = (dz W3) * [h2 > 0]
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int s = 8 * sg + i;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int j = 4 * ng + q;
+                float v = 0.f;
+#pragma unroll
+                for (int c = 0; c < kA; ++c) v = fmaf(DZ[s * 8 + c], sm[kSW3 + c * kH + j], v);
+                D2[s * kHS + j] = H2[s * kHS + j] > 0.f ? v : 0.f;
+            }
+        }
+        __syncthreads();
+        // D1 = (D2 W2) * [h1 > 0]
+        {
+            float acc[8][4] = {};
+#pragma unroll 4
+            for (int j = 0; j < kH; ++j) {
+                const float4 w = *reinterpret_cast<const float4*>(sm + kSW2 + j * kH + 4 * ng);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float d = D2[(8 * sg + i) * kHS + j];
+                    acc[i][0] = fmaf(w.x, d, acc[i][0]);
+                    acc[i][1] = fmaf(w.y, d, acc[i][1]);
+                    acc[i][2] = fmaf(w.z, d, acc[i][2]);
+                    acc[i][3] = fmaf(w.w, d, acc[i][3]);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int s = 8 * sg + i, k = 4 * ng + q;
+                    D1[s * kHS + k] = H1[s * kHS + k] > 0.f ? acc[i][q] : 0.f;
+                }
+        }
+        __syncthreads();
+        // weight gradients of the tile
+        for (int s = 0; s < kTile; ++s) {
+            float d[4], h[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                d[q] = D2[s * kHS + 4 * jb + q];
+                h[q] = H1[s * kHS + 4 * kb + q];
+            }
+#pragma unroll
+            for (int p = 0; p < 4; ++p)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) gW2[p][q] = fmaf(d[p], h[q], gW2[p][q]);
+        }
+#pragma unroll
+        for (int q = 0; q < (int)(sizeof(gW1) / sizeof(float)); ++q) {
+            const int e = tid + kThreads * q;
+            if (e < nW1) {
+                const int j = e / in, k = e - j * in;
+                float g = gW1[q];
+                for (int s = 0; s < kTile; ++s) g = fmaf(D1[s * kHS + j], X[s * kXS + k], g);
+                gW1[q] = g;
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int e = tid + kThreads * q;
+            if (e < kA * kH) {
+                const int c = e / kH, j = e - c * kH;
+                float g = gW3[q];
+                for (int s = 0; s < kTile; ++s) g = fmaf(DZ[s * 8 + c], H2[s * kHS + j], g);
+                gW3[q] = g;
+            }
+        }
+        if (tid < 2 * kH + kA) {
+            float g = gB;
+            if (tid < kH)
+                for (int s = 0; s < kTile; ++s) g += D1[s * kHS + tid];
+            else if (tid < 2 * kH)
+                for (int s = 0; s < kTile; ++s) g += D2[s * kHS + tid - kH];
+            else
+                for (int s = 0; s < kTile; ++s) g += DZ[s * 8 + tid - 2 * kH];
+            gB = g;
+        }
+        __syncthreads();                        // the tile's buffers are rewritten next
+    }
+
+    // this CTA's partial gradient, in the malib_policy_desc layout:
+    // W1 [64][in], b1, W2 [64][64], b2, W3 [5][64], b3, then loss and entropy sums
+    const int P = kH * in + kH + kH * kH + kH + kA * kH + kA;
+    float* out = a.gpart + (int64_t)blockIdx.x * (P + 2);
+#pragma unroll
+    for (int q = 0; q < (int)(sizeof(gW1) / sizeof(float)); ++q) {
+        const int e = tid + kThreads * q;
+        if (e < nW1) out[e] = gW1[q];                             // j * in + k
+    }
+    const int oW2 = kH * in + kH;
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) out[oW2 + (4 * jb + p) * kH + 4 * kb + q] = gW2[p][q];
+    const int oW3 = oW2 + kH * kH + kH;
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+        const int e = tid + kThreads * q;
+        if (e < kA * kH) out[oW3 + e] = gW3[q];
+    }
+    if (tid < kH) out[kH * in + tid] = gB;                          // b1
+    else if (tid < 2 * kH) out[oW2 + kH * kH + tid - kH] = gB;      // b2
+    else if (tid < 2 * kH + kA) out[oW3 + kA * kH + tid - 2 * kH] = gB;   // b3
+    // loss and entropy sums of the CTA (fixed-order tree in shared memory)
+    __syncthreads();
+    float* red = sm + kSX;
+    red[tid] = lsum;
+    red[kThreads + tid] = hsum;
+    __syncthreads();
+    for (int w = kThreads / 2; w > 0; w >>= 1) {
+        if (tid < w) {
+            red[tid] += red[tid + w];
+            red[kThreads + tid] += red[kThreads + tid + w];
+        }
+        __syncthreads();
+    }
+    if (tid == 0) {
+        out[P] = red[0];
+        out[P + 1] = red[kThreads];
+    }
+}
+
+__global__ void learn_reduce_kernel(LearnArgs a, int P) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= P + 2) return;
+    double s = 0.0;
+    for (int b = 0; b < a.grid; ++b) s += (double)a.gpart[(int64_t)b * (P + 2) + j];
+    if (j < P) a.grad[j] = (float)s;
+    else if (j == P) a.stats[2] = a.stats[0] > 0 ? s / a.stats[0] : 0.0;   // loss: (1/M) sum of -(A log pi + beta H)
+    else a.stats[3] = a.stats[0] > 0 ? s / a.stats[0] : 0.0;              // mean entropy
+}
+
+__global__ void learn_adam_kernel(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1,
+                                  float b2, float eps, float c1, float c2) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const float gi = g[i];
+        const float mi = b1 * m[i] + (1.f - b1) * gi;
+        const float vi = b2 * v[i] + (1.f - b2) * gi * gi;
+        m[i] = mi;
+        v[i] = vi;
+        p[i] -= lr * (mi / c1) / (sqrtf(vi / c2) + eps);
+    }
+}
+
+}  // namespace
+
+int64_t learn_param_count(int in) { return (int64_t)kH * in + kH + kH * kH + kH + kA * kH + kA; }
+
+bool learn_supported(int in, int h1, int h2, int n_actions) {
+    return in >= 1 && in <= kLearnMaxIn && h1 == kH && h2 == kH && n_actions == kA;
+}
+
+// Upper bounds of the work space (bytes, each region on a 256-byte boundary).
+int64_t learn_work_bytes(int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes, int32_t T,
+                         int in, int grid, int ret_blocks) {
+    auto up = [](int64_t b) { return (b + 255) / 256 * 256; };
+    const int64_t slots = (int64_t)n_pairs * n_agents;
+    const int64_t samples = slots * n_episodes * T * (n_envs / n_pairs);
+    return up(slots * 4) + up(4) + up(samples * 4) + up((int64_t)ret_blocks * 8) + up(4 * 8) +
+           up((int64_t)grid * (learn_param_count(in) + 2) * 4);
+}
+
+void learn_work_layout(uint8_t* base, int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes,
+                       int32_t T, int in, int grid, int ret_blocks, LearnArgs* a) {
+    int64_t off = 0;
+    auto take = [&](int64_t bytes) {
+        uint8_t* p = base + off;
+        off += (bytes + 255) / 256 * 256;
+        return p;
+    };
+    const int64_t slots = (int64_t)n_pairs * n_agents;
+    const int64_t samples = slots * n_episodes * T * (n_envs / n_pairs);
+    a->slots = reinterpret_cast<int32_t*>(take(slots * 4));
+    a->n_slots = reinterpret_cast<int32_t*>(take(4));
+    a->G = reinterpret_cast<float*>(take(samples * 4));
+    a->gsum = reinterpret_cast<double*>(take((int64_t)ret_blocks * 8));
+    a->stats = reinterpret_cast<double*>(take(4 * 8));
+    a->gpart = reinterpret_cast<float*>(take((int64_t)grid * (learn_param_count(in) + 2) * 4));
+    a->grid = grid;
+}
+
+cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s) {
+    learn_slots_kernel<<<1, 1024, 0, s>>>(a);
+    learn_returns_kernel<<<ret_blocks, 256, 0, s>>>(a);
+    learn_baseline_kernel<<<1, 32, 0, s>>>(a, ret_blocks);
+    cudaError_t err = cudaFuncSetAttribute(learn_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)kSBytes);
+    if (err != cudaSuccess) return err;
+    learn_grad_kernel<<<a.grid, kThreads, kSBytes, s>>>(a);
+    const int P = (int)learn_param_count(a.in);
+    learn_reduce_kernel<<<(P + 2 + 255) / 256, 256, 0, s>>>(a, P);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_learn_adam(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1,
+                              float b2, float eps, float c1, float c2, int n_sm, cudaStream_t s) {
+    if (n == 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 4 * (int64_t)n_sm) blocks = 4 * (int64_t)n_sm;
+    learn_adam_kernel<<<(unsigned)blocks, 256, 0, s>>>(p, g, m, v, n, lr, b1, b2, eps, c1, c2);
+    return cudaGetLastError();
+}
+
+}  // namespace malib

@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -63,6 +64,10 @@ struct malib_ctx {
     int64_t scratch_cap = 0;
     uint8_t* lwork = nullptr;          // tensor-core Leduc evaluation: hand states and queues
     int64_t lwork_cap = 0;
+    uint8_t* learn_work = nullptr;     // policy-gradient step: slots, returns, partial gradients
+    int64_t learn_work_cap = 0;
+    float* learn_grad = nullptr;       // the gradient when the caller's buffer is host memory
+    int64_t learn_grad_cap = 0;
 
     int64_t launches = 0;
     bool timing = false;
@@ -211,6 +216,27 @@ int upload_tables(malib_ctx* c) {
     CK(cudaStreamSynchronize(c->stream), "upload");
     c->tables_dirty = false;
     return MALIB_OK;
+}
+
+// The conversion of a policy's parameters into its kernel image: kind, flags
+// and image size (words).
+void conv_job(int env_kind, int kind, int dtype, const int* dims, ConvJob* jb) {
+    std::memcpy(jb->dims, dims, sizeof jb->dims);
+    jb->flags = 0;
+    if (kind == MALIB_POL_TABULAR) {
+        jb->kind = kConvTable;
+        jb->size = 8;
+    } else if (dtype == MALIB_BF16 && tc_image_shape(dims)) {
+        const bool fold = leduc_tc_fold(env_kind, dims[0]);
+        jb->kind = kConvTc;
+        jb->flags = fold ? kConvFold : 0;
+        jb->size = tc_image_bytes(fold ? dims[0] - 1 : dims[0]) / 4;
+    } else {
+        jb->kind = kConvF32;
+        jb->flags = dtype == MALIB_BF16 ? kConvRound : 0;   // bf16 weights, fp32 biases
+        jb->size = ((int64_t)dims[0] * dims[1] + dims[1] + (int64_t)dims[1] * dims[2] + dims[2] +
+                    (int64_t)dims[3] * dims[2] + dims[3] + 3) / 4 * 4;
+    }
 }
 
 int stage_pairs(malib_ctx* c, const int32_t* pair_ids, int64_t n_ints, int width, bool poker,
@@ -389,6 +415,8 @@ void malib_destroy(malib_ctx* c) {
     cudaFree(c->d_out);
     cudaFree(c->scratch);
     cudaFree(c->lwork);
+    cudaFree(c->learn_work);
+    cudaFree(c->learn_grad);
     cudaFree(c->d_stage);
     cudaFree(c->d_jobs);
     delete c;
@@ -471,22 +499,7 @@ int malib_pop_load(malib_ctx* c, const malib_env_spec* spec, const malib_policy_
         if (d.kind != ref_kind || d.dtype != ref_dtype || std::memcmp(d.dims, ref_dims, 16) != 0)
             return fail(c, MALIB_EINVAL, "policy %d: every policy of a population shares kind, dtype and dims", i);
         ConvJob& jb = jobs[i];
-        std::memcpy(jb.dims, d.dims, sizeof jb.dims);
-        jb.flags = 0;
-        if (d.kind == MALIB_POL_TABULAR) {
-            jb.kind = kConvTable;
-            jb.size = 8;
-        } else if (d.dtype == MALIB_BF16 && tc_image_shape(d.dims)) {
-            const bool fold = leduc_tc_fold(spec->env_kind, d.dims[0]);
-            jb.kind = kConvTc;
-            jb.flags = fold ? kConvFold : 0;
-            jb.size = tc_image_bytes(fold ? d.dims[0] - 1 : d.dims[0]) / 4;
-        } else {
-            jb.kind = kConvF32;
-            jb.flags = d.dtype == MALIB_BF16 ? kConvRound : 0;   // bf16 weights, fp32 biases
-            jb.size = ((int64_t)d.dims[0] * d.dims[1] + d.dims[1] + (int64_t)d.dims[1] * d.dims[2] +
-                       d.dims[2] + (int64_t)d.dims[3] * d.dims[2] + d.dims[3] + 3) / 4 * 4;
-        }
+        conv_job(spec->env_kind, d.kind, d.dtype, d.dims, &jb);
         jb.src = stage_floats;
         jb.dst = c->arena_used + image_floats;
         rec.offset = jb.dst;
@@ -747,6 +760,146 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     }
     time_end(c, e0, e1);
     c->launches += 1;
+    return MALIB_OK;
+}
+
+int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                   int64_t n_episodes, const malib_traj* traj, int32_t policy_id, float gamma,
+                   float entropy_coef, float* grad_out, double* stats_out) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    int r;
+    if ((r = check_spec(c, spec)) != MALIB_OK) return r;
+    if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
+    if (!same_env(c->spec, *spec))
+        return fail(c, MALIB_ESTATE, "spec differs from the population's environment");
+    if (spec->env_kind == MALIB_ENV_KUHN || spec->env_kind == MALIB_ENV_LEDUC)
+        return fail(c, MALIB_EUNSUPPORTED, "the learner step is built for the particle rollouts");
+    if (c->pol_kind != MALIB_POL_MLP || c->pol_dtype != MALIB_F32 ||
+        !learn_supported(c->dims[0], c->dims[1], c->dims[2], c->dims[3]))
+        return fail(c, MALIB_EUNSUPPORTED, "the learner step is built for fp32 MLPs in-64-64-5 (in <= %d)",
+                    kLearnMaxIn);
+    if (policy_id < 0 || policy_id >= (int32_t)c->pols.size())
+        return fail(c, MALIB_EINVAL, "policy_id %d is not in the population", policy_id);
+    if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");
+    if (spec->n_envs < 1 || spec->n_envs % n_pairs != 0)
+        return fail(c, MALIB_EINVAL, "n_envs (%lld) must be a positive multiple of n_pairs (%d)",
+                    (long long)spec->n_envs, n_pairs);
+    if (n_episodes < 0) return fail(c, MALIB_EINVAL, "n_episodes < 0");
+    if (!(gamma >= 0.0f && gamma <= 1.0f)) return fail(c, MALIB_EINVAL, "gamma must lie in [0, 1]");
+    if (!(entropy_coef >= 0.0f && entropy_coef < 1e30f)) return fail(c, MALIB_EINVAL, "entropy_coef must be >= 0");
+    if (!pair_ids || !traj || !grad_out) return fail(c, MALIB_EINVAL, "pair_ids, traj or grad_out is NULL");
+    if (!traj->obs || !traj->action || !traj->reward) return fail(c, MALIB_EINVAL, "trajectory buffer missing");
+    const void* tp[3] = {traj->obs, traj->action, traj->reward};
+    for (const void* p : tp)
+        if (!is_device_ptr(c, p))
+            return fail(c, MALIB_EINVAL, "trajectory buffers must be device memory of the context's device");
+    const int gw = ptr_where(grad_out, c->device);
+    const int sw = stats_out ? ptr_where(stats_out, c->device) : kPtrHost;
+    if (gw == kPtrOther || sw == kPtrOther)
+        return fail(c, MALIB_EINVAL, "grad_out or stats_out lives on another device than the context's");
+    if ((r = upload_tables(c)) != MALIB_OK) return r;
+    const int32_t* dpairs = nullptr;
+    if ((r = stage_pairs(c, pair_ids, (int64_t)n_pairs * spec->n_agents, spec->n_agents, false, &dpairs)) !=
+        MALIB_OK)
+        return r;
+    const int in = c->dims[0];
+    const int64_t P = learn_param_count(in);
+    const int grid = c->n_sm;
+    const int ret_blocks = 2 * c->n_sm;
+    const int64_t bytes = learn_work_bytes(n_pairs, spec->n_agents, spec->n_envs, n_episodes,
+                                           spec->episode_len, in, grid, ret_blocks);
+    if ((r = ensure(c, c->learn_work, c->learn_work_cap, bytes, "learner work space")) != MALIB_OK) return r;
+    LearnArgs a{};
+    learn_work_layout(c->learn_work, n_pairs, spec->n_agents, spec->n_envs, n_episodes, spec->episode_len, in,
+                      grid, ret_blocks, &a);
+    if (gw == kPtrHere) {
+        a.grad = grad_out;
+    } else {
+        if ((r = ensure(c, c->learn_grad, c->learn_grad_cap, P, "gradient staging")) != MALIB_OK) return r;
+        a.grad = c->learn_grad;
+    }
+    a.arena = c->arena;
+    a.pol_off = c->pols[policy_id].offset;
+    a.in = in;
+    a.xs = (spec->obs_dim + 3) / 4 * 4;
+    a.pairs = dpairs;
+    a.n_pairs = n_pairs;
+    a.n_agents = spec->n_agents;
+    a.n_pol = (int32_t)c->pols.size();
+    a.policy = policy_id;
+    a.T = spec->episode_len;
+    a.n_envs = spec->n_envs;
+    a.n_episodes = n_episodes;
+    a.obs = traj->obs;
+    a.action = traj->action;
+    a.reward = traj->reward;
+    a.gamma = gamma;
+    a.beta = entropy_coef;
+    a.err = c->d_err;
+    CK(launch_learn_pg(a, ret_blocks, c->stream), "policy-gradient kernels");
+    c->launches += 5;
+    if (gw != kPtrHere)
+        CK(cudaMemcpyAsync(grad_out, a.grad, P * 4, cudaMemcpyDeviceToHost, c->stream), "gradient copy");
+    if (stats_out)
+        CK(cudaMemcpyAsync(stats_out, a.stats, 4 * 8, sw == kPtrHere ? cudaMemcpyDeviceToDevice
+                                                                     : cudaMemcpyDeviceToHost, c->stream),
+           "statistics copy");
+    if (gw != kPtrHere || (stats_out && sw != kPtrHere)) {
+        CK(cudaStreamSynchronize(c->stream), "learner step");
+        if ((r = read_device_errors(c)) != MALIB_OK) return r;
+    }
+    return MALIB_OK;
+}
+
+int malib_adam_step(malib_ctx* c, float* params, const float* grad, float* m, float* v, int64_t n, int64_t step,
+                    float lr, float beta1, float beta2, float eps) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (n < 0) return fail(c, MALIB_EINVAL, "n < 0");
+    if (n == 0) return MALIB_OK;
+    if (!params || !grad || !m || !v) return fail(c, MALIB_EINVAL, "a buffer is NULL");
+    const void* ptrs[4] = {params, grad, m, v};
+    for (const void* p : ptrs)
+        if (!is_device_ptr(c, p)) return fail(c, MALIB_EINVAL, "Adam buffers must be device memory of the context's device");
+    if (step < 1) return fail(c, MALIB_EINVAL, "step must be >= 1");
+    if (!(lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) || !(beta2 >= 0.0f && beta2 < 1.0f) || !(eps > 0.0f))
+        return fail(c, MALIB_EINVAL, "need lr >= 0, 0 <= beta1, beta2 < 1, eps > 0");
+    const float c1 = (float)(1.0 - std::pow((double)beta1, (double)step));
+    const float c2 = (float)(1.0 - std::pow((double)beta2, (double)step));
+    CK(launch_learn_adam(params, grad, m, v, n, lr, beta1, beta2, eps, c1 > 0.f ? c1 : 1.f, c2 > 0.f ? c2 : 1.f,
+                         c->n_sm, c->stream),
+       "Adam kernel");
+    c->launches += 1;
+    return MALIB_OK;
+}
+
+int malib_pop_update(malib_ctx* c, int32_t policy_id, const float* params, int64_t nbytes) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
+    if (policy_id < 0 || policy_id >= (int32_t)c->pols.size())
+        return fail(c, MALIB_EINVAL, "policy_id %d is not in the population", policy_id);
+    const PolicyRec& rec = c->pols[policy_id];
+    const int64_t count = rec.kind == MALIB_POL_TABULAR ? 6 : mlp_param_floats(rec.dims);
+    if (!params || nbytes != count * 4)
+        return fail(c, MALIB_EINVAL, "params NULL or nbytes %lld != %lld", (long long)nbytes,
+                    (long long)(count * 4));
+    if (ptr_where(params, c->device) == kPtrOther)
+        return fail(c, MALIB_EINVAL, "params live on another device than the context's");
+    ConvJob jb{};
+    conv_job(c->spec.env_kind, rec.kind, rec.dtype, rec.dims, &jb);
+    jb.src = 0;
+    jb.dst = rec.offset;
+    int r;
+    if ((r = ensure(c, c->d_stage, c->stage_cap, (count + 3) / 4 * 4, "parameter staging")) != MALIB_OK) return r;
+    if ((r = ensure(c, c->d_jobs, c->jobs_cap, (int64_t)1, "conversion jobs")) != MALIB_OK) return r;
+    CK(cudaMemcpyAsync(c->d_stage, params, nbytes, cudaMemcpyDefault, c->stream), "parameter upload");
+    CK(cudaMemcpyAsync(c->d_jobs, &jb, sizeof jb, cudaMemcpyHostToDevice, c->stream), "conversion job");
+    CK(launch_pop_convert(c->d_jobs, 1, jb.size, c->d_stage, c->arena, c->stream), "population conversion kernel");
+    c->launches += 1;
+    // the caller may free or reuse its buffer once this returns
+    CK(cudaStreamSynchronize(c->stream), "population update");
     return MALIB_OK;
 }
 

@@ -1,0 +1,188 @@
+"""GPU parity for the learner-side update (Sec. 3.3 independent learning; App.
+C.2 training workflow): the policy-gradient step of one policy on a GPU
+rollout's samples, Adam, and the population update that closes the loop.
+
+The oracle (oracle/learner.py, fp64) gathers the same samples from the
+trajectory the GPU wrote and computes the gradient; the GPU's fp32 gradient
+must match per parameter block within 1e-4 of the block's largest magnitude
+(fp32 forward and fp32 per-CTA sums of a few thousand terms, summed across
+CTAs in fp64: relative errors of order 1e-6), M exactly, the baseline and
+mean entropy within 1e-5 relative, the loss (a mean of cancelling terms)
+within 1e-5 of the terms' scale. Adam matches the fp64 recursion within
+1e-6 relative. After pop_update, the next rollout replays bit for bit against
+the oracle's rollout of the updated parameters."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from oracle import learner
+from gpu_util import context, load_population, logits_close, need_gpu, spec_of
+
+pytestmark = pytest.mark.gpu
+
+from paper_2106_07551_gb300 import MALIB_DUMP_LOGITS, MalibError, alloc_traj
+
+
+def rollout(ctx, w, n_eps, seed, flags=0):
+    spec = spec_of(w, flags)
+    traj = alloc_traj(spec, n_eps, logits=bool(flags & MALIB_DUMP_LOGITS))
+    ctx.rollout(spec, w.pair_ids, n_eps, seed, traj)
+    ctx.sync()
+    return spec, traj
+
+
+def blocks(dims):
+    i, h1, h2, a = dims
+    sizes = [h1 * i, h1, h2 * h1, h2, a * h2, a]
+    return np.cumsum([0] + sizes)
+
+
+def check_grad(g, o, dims):
+    cut = blocks(dims)
+    for lo, hi in zip(cut[:-1], cut[1:]):
+        scale = np.abs(o[lo:hi]).max()
+        np.testing.assert_allclose(g[lo:hi], o[lo:hi], rtol=0, atol=1e-4 * scale + 1e-12)
+
+
+def learn(ctx, w, spec, traj, n_eps, pid, gamma, beta, device_out=False):
+    torch = need_gpu()
+    P = int(blocks(w.policies[0].dims)[-1])
+    if device_out:
+        g = torch.zeros(P, dtype=torch.float32, device="cuda")
+        st = torch.zeros(4, dtype=torch.float64, device="cuda")
+        ctx.learn_pg(spec, w.pair_ids, n_eps, traj, pid, gamma, beta, g, st)
+        ctx.sync()
+        return g.cpu().numpy(), st.cpu().numpy()
+    g = np.zeros(P, np.float32)
+    st = np.zeros(4, np.float64)
+    ctx.learn_pg(spec, w.pair_ids, n_eps, traj, pid, gamma, beta, g, st)
+    return g, st
+
+
+def host(traj):
+    return {k: v.cpu().numpy() for k, v in traj.items()}
+
+
+def oracle_grad(w, tr, pid, gamma, beta):
+    obs, act, ret = learner.gather(tr, w.pair_ids, w.n_envs, w.n_agents, w.obs_dim, pid, gamma)
+    return learner.pg_grad(w.policies[pid].params, w.policies[pid].dims, obs, act, ret, beta)
+
+
+@pytest.mark.parametrize("make,kw", [(workloads.spread, dict(n_agents=3, n_envs=1024, pop=6)),
+                                     (workloads.tag, dict(n_envs=512, pop=5)),
+                                     (workloads.push, dict(n_envs=384, pop=4, envs_per_pair=64))])
+def test_policy_gradient_parity(make, kw):
+    need_gpu()
+    w = make(with_bias=True, seed=77, **kw)
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 2, 99)
+    tr = host(traj)
+    for pid, gamma, beta, dev in ((0, 0.95, 0.001, False), (1, 0.0, 0.0, True), (2, 1.0, 0.1, False)):
+        g, st = learn(ctx, w, spec, traj, 2, pid, gamma, beta, dev)
+        o, (M, b, loss, ent) = oracle_grad(w, tr, pid, gamma, beta)
+        assert st[0] == M and M > 0
+        np.testing.assert_allclose([st[1], st[3]], [b, ent], rtol=1e-5, atol=1e-7)
+        # the loss is a mean of terms of order |G - b| |log pi| that cancel: an
+        # absolute bound relative to those terms, not to the (small) mean
+        assert abs(st[2] - loss) <= 1e-5 * (1.0 + np.abs(tr["reward"]).max() * w.episode_len)
+        check_grad(g, o, w.policies[pid].dims)
+        # deterministic
+        g2, st2 = learn(ctx, w, spec, traj, 2, pid, gamma, beta, dev)
+        assert np.array_equal(g, g2) and np.array_equal(st, st2)
+    ctx.close()
+
+
+def test_policy_without_samples():
+    need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=256, pop=6, seed=5)
+    w.pair_ids[:] = np.array([0, 1, 2], np.int32)              # policies 3..5 never act
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 1, 3)
+    g, st = learn(ctx, w, spec, traj, 1, 4, 0.9, 0.01)
+    assert np.all(g == 0) and np.all(st == 0)
+    ctx.close()
+
+
+def test_adam_parity():
+    torch = need_gpu()
+    rng = np.random.default_rng(8)
+    n = 10_000
+    p0 = rng.normal(size=n).astype(np.float32)
+    ctx = context()
+    p = torch.from_numpy(p0.copy()).cuda()
+    m = torch.zeros(n, device="cuda")
+    v = torch.zeros(n, device="cuda")
+    rp, rm, rv = p0.astype(np.float64), np.zeros(n), np.zeros(n)
+    for step in range(1, 6):
+        gr = rng.normal(size=n).astype(np.float32)
+        ctx.adam_step(p, torch.from_numpy(gr).cuda(), m, v, step, 1e-3)
+        rp, rm, rv = learner.adam(rp, gr, rm, rv, step, 1e-3)
+        ctx.sync()
+        np.testing.assert_allclose(p.cpu().numpy(), rp, rtol=1e-6, atol=1e-7)
+        # m is a running sum of terms of order 0.1 |g| that can cancel: absolute
+        np.testing.assert_allclose(m.cpu().numpy(), rm, rtol=1e-5, atol=1e-7)
+    ctx.close()
+
+
+def test_training_loop_closes():
+    """rollout -> policy gradient -> Adam -> pop_update -> rollout: the second
+    rollout replays bit for bit against the oracle with the updated policy."""
+    torch = need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=512, pop=4, with_bias=True, seed=21)
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 1, 11)
+    pid = int(w.pair_ids[0, 0])
+    P = int(blocks(w.policies[pid].dims)[-1])
+    g = torch.zeros(P, device="cuda")
+    ctx.learn_pg(spec, w.pair_ids, 1, traj, pid, 0.95, 0.001, g)
+    params = torch.from_numpy(w.policies[pid].params.astype(np.float32)).cuda()
+    m = torch.zeros(P, device="cuda")
+    v = torch.zeros(P, device="cuda")
+    ctx.adam_step(params, g, m, v, 1, 1e-2)
+    ctx.pop_update(pid, params)
+    new = params.cpu().numpy()
+    assert not np.array_equal(new, w.policies[pid].params)
+    w.policies[pid].params = new
+    spec, traj2 = rollout(ctx, w, 1, 12, MALIB_DUMP_LOGITS)
+    tr = host(traj2)
+    ref = oracle.spread_rollout([p.params for p in w.policies], w.policies[0].dims, 3, 3, w.episode_len,
+                                w.n_envs, w.pair_ids, 1, 12, ext_logits=tr["logits"])
+    np.testing.assert_array_equal(tr["obs"][..., :w.obs_dim], ref["obs"])
+    np.testing.assert_array_equal(tr["action"].astype(np.int8), ref["action"])
+    n_bad, worst = logits_close(tr["logits"], ref["logits"], 1e-5)
+    assert n_bad == 0, (n_bad, worst)
+    # a host buffer works as well, and restores the old parameters
+    old = np.asarray(workloads.spread(n_agents=3, n_envs=512, pop=4, with_bias=True, seed=21)
+                     .policies[pid].params, np.float32)
+    ctx.pop_update(pid, old)
+    ctx.close()
+
+
+def test_learner_refusals():
+    torch = need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=256, pop=3, seed=2)
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 1, 1)
+    g = np.zeros(int(blocks(w.policies[0].dims)[-1]), np.float32)
+    for pid, gamma, beta in ((3, 0.9, 0.0), (-1, 0.9, 0.0), (0, 1.5, 0.0), (0, 0.9, -1.0)):
+        with pytest.raises(MalibError, match="EINVAL"):
+            ctx.learn_pg(spec, w.pair_ids, 1, traj, pid, gamma, beta, g)
+    with pytest.raises(MalibError, match="EINVAL"):
+        ctx.pop_update(0, np.zeros(5, np.float32))
+    with pytest.raises(MalibError, match="EINVAL"):
+        ctx.adam_step(torch.zeros(4, device="cuda"), np.zeros(4, np.float32), torch.zeros(4, device="cuda"),
+                      torch.zeros(4, device="cuda"), 1, 1e-3)
+    ctx.close()
+    # a bf16 (tensor-core) population has no learner kernel
+    wb = workloads.spread(n_agents=8, n_envs=128, pop=2, hidden=256, dtype=workloads.BF16, seed=3)
+    ctx = context()
+    load_population(ctx, wb)
+    spec, traj = rollout(ctx, wb, 1, 1)
+    with pytest.raises(MalibError, match="EUNSUPPORTED"):
+        ctx.learn_pg(spec, wb.pair_ids, 1, traj, 0, 0.9, 0.0, np.zeros(100, np.float32))
+    ctx.close()
