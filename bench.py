@@ -61,7 +61,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "speaker_listener",
-                                           "leduc_bf16", "spread8", "meta"],
+                                           "leduc_bf16", "spread8", "meta", "learner"],
                     default="leduc_bf16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -813,12 +813,162 @@ def run_meta(args):
     return 0
 
 
+LEARN_EPISODES = 10
+
+
+def learn_flop(dims):
+    """Algorithmic flops of one sample's policy-gradient step: the forward (as
+    mlp_flop) and the backward (dL/dh2 and dL/dh1 through W3 and W2, the
+    weight gradients of W3, W2, W1; bias sums excluded)."""
+    i, h1, h2, a = dims
+    return mlp_flop(dims) + 2 * (a * h2 + h2 * h1) + 2 * (a * h2 + h2 * h1 + h1 * i)
+
+
+def run_learner(args):
+    """The learner-side update (Sec. 3.3 independent learning, App. C.2): one
+    training iteration of every policy of the spread population (N = 3, 4,096
+    envs, population 16, MLP 18-64-64-5 fp32) on LEARN_EPISODES episodes of
+    its rollout: per policy, malib_learn_pg on its samples and malib_adam_step.
+    A step covers every sample once (each belongs to one policy)."""
+    import numpy as np
+    import torch
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import workloads
+    from paper_2106_07551_gb300 import Context, alloc_traj, make_spec, policy_desc
+
+    w = workloads.config(3, n_episodes=LEARN_EPISODES)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+    ctx = Context(local, stream)
+    spec = make_spec(w.env_kind, w.n_agents, w.obs_dim, w.n_actions, w.n_landmarks, w.episode_len, w.n_envs)
+    ctx.pop_load(spec, [policy_desc(p.kind, p.dtype, p.seat, p.dims, p.params) for p in w.policies])
+    d_pairs = torch.from_numpy(w.pair_ids).to(dev)
+    traj = alloc_traj(spec, w.n_episodes)
+    ctx.rollout(spec, d_pairs, w.n_episodes, w.seed + rank, traj)
+    dims = w.policies[0].dims
+    n_pol = len(w.policies)
+    P = int(dims[1] * dims[0] + dims[1] + dims[2] * dims[1] + dims[2] + dims[3] * dims[2] + dims[3])
+    grads = torch.zeros((n_pol, P), dtype=torch.float32, device=dev)
+    params = torch.from_numpy(np.stack([p.params for p in w.policies]).astype(np.float32)).to(dev)
+    m = torch.zeros_like(params)
+    v = torch.zeros_like(params)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    samples = w.n_envs * w.episode_len * w.n_episodes * w.n_agents
+    state = {"t": 0}
+
+    def step():
+        state["t"] += 1
+        for pid in range(n_pol):
+            ctx.learn_pg(spec, d_pairs, w.n_episodes, traj, pid, 0.95, 0.001, grads[pid])
+            ctx.adam_step(params[pid], grads[pid], m[pid], v[pid], state["t"], 1e-4)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    ctx.sync()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    launches0 = ctx.launch_count()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clocks:
+        for k in range(args.steps):
+            flush.zero_()
+            ev[k][0].record(stream)
+            step()
+            ev[k][1].record(stream)
+        torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    launches = ctx.launch_count() - launches0
+    ctx.sync()
+    total_ms = sum(a.elapsed_time(c) for a, c in ev)
+    total_ms_max = max_over_ranks(total_ms, world, dev)
+    value = sum_over_ranks(float(samples * args.steps), world, dev) / (total_ms_max / 1e3)
+    peaks = load_peaks()
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
+    peak = n_sm * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
+    achieved = samples * learn_flop(dims) / (total_ms / args.steps / 1e3) / 1e12
+    e2e = None
+    cpu = None
+    if rank == 0:
+        # e2e: the trajectory from pinned host memory, every policy's gradient back
+        h_obs = traj["obs"].cpu().pin_memory()
+        h_act = traj["action"].cpu().pin_memory()
+        h_rew = traj["reward"].cpu().pin_memory()
+        h_g = torch.empty_like(grads, device="cpu").pin_memory()
+        reps = max(1, args.e2e_steps // 5)
+        t_e2e = 0.0
+        for k in range(reps + 1):
+            torch.cuda.synchronize(dev)
+            s0 = time.perf_counter()
+            traj["obs"].copy_(h_obs, non_blocking=True)
+            traj["action"].copy_(h_act, non_blocking=True)
+            traj["reward"].copy_(h_rew, non_blocking=True)
+            step()
+            h_g.copy_(grads, non_blocking=True)
+            torch.cuda.synchronize(dev)
+            if k > 0:
+                t_e2e += time.perf_counter() - s0
+        e2e = {"value": samples * reps / t_e2e, "unit": "samples/s",
+               "h2d_bytes_per_step": int(h_obs.numel() * 4 + h_act.numel() + h_rew.numel() * 4),
+               "d2h_bytes_per_step": int(h_g.numel() * 4), "steps": reps}
+        if world == 1 and not args.no_cpu_baseline:
+            from oracle import learner as ol
+            tr = {"obs": h_obs.numpy(), "action": h_act.numpy(), "reward": h_rew.numpy()}
+            n_done, t_cpu, n_s = 0, 0.0, 0
+            while t_cpu < 10.0 and n_done < n_pol:
+                s0 = time.perf_counter()
+                o, a_, r_ = ol.gather(tr, w.pair_ids, w.n_envs, w.n_agents, w.obs_dim, n_done, 0.95)
+                ol.pg_grad(w.policies[n_done].params, dims, o, a_, r_, 0.001)
+                t_cpu += time.perf_counter() - s0
+                n_s += o.shape[0]
+                n_done += 1
+            cpu = {"value": n_s / t_cpu, "unit": "samples/s", "cores": cpu_count(), "kind": "oracle",
+                   "sample": f"{n_done} of the {n_pol} policies' gradients ({n_s} samples, {t_cpu:.1f} s, "
+                             "numpy fp64)"}
+    clk = clocks.summary()
+    ctx.close()
+    if rank == 0:
+        line = {"metric": "learner samples/sec (policy-gradient step and Adam of every policy)",
+                "value": value, "unit": "samples/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                "data": "synthetic",
+                "config": {"workload": f"learner_spread_n3_4096env_mlp18-64-64-5_f32_{w.n_episodes}episodes_"
+                                       f"pop{n_pol}", "samples_per_step": samples, "policies": n_pol,
+                           "l2": "flushed (256 MiB write) before every timed step"},
+                "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                             "frac": achieved / peak, "traffic": None, "kernel": "learn_grad_kernel",
+                             "peak_basis": f"fp32 FMA: {n_sm} SMs (queried) x {FP32_LANES_PER_SM} lanes x 2 "
+                                           f"flop x {sm_max:.0f} MHz",
+                             "algorithmic": f"{learn_flop(dims)} flop per sample (forward and backward, "
+                                            "bias sums excluded); whole step timed"},
+                "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "gpu_launches": launches}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "meta":
         return run_meta(args)
+    if args.workload == "learner":
+        return run_learner(args)
     return run_ours(args)
 
 
