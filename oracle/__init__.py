@@ -86,6 +86,11 @@ def _L():
                 "orc_push_obs": (None, [P, P]),
                 "orc_push_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
                                             P, i32, i64, u64, P, P, P, P, P, C.c_int]),
+                "orc_ref_reset": (None, [u64, u64, P]),
+                "orc_ref_step": (None, [P, P, P, f32]),
+                "orc_ref_obs": (None, [P, P]),
+                "orc_ref_rollout": (None, [P, C.c_int, C.c_int, C.c_int, C.c_int, i64, i64, i64,
+                                           P, i32, i64, u64, P, P, P, P, P, C.c_int, f32]),
                 "orc_tag_reset": (None, [u64, u64, P]),
                 "orc_tag_step": (None, [P, P, P]),
                 "orc_tag_obs": (None, [P, P]),
@@ -462,3 +467,54 @@ push_rollout.__doc__ = """Rollout over envs [env_lo, env_hi) of the simple push 
 tag_reset, tag_step, tag_obs, tag_rollout = _scen("tag", TAG_N, TAG_OBS, TAG_STATE)
 tag_rollout.__doc__ = """Rollout over envs [env_lo, env_hi) of the simple tag (4 agents, obs 16,
 5 actions). Returns the arrays of spread_rollout."""
+
+
+# ---- simple reference (App. B.1) ----
+# state: px,py,vx,vy of agents 0, 1; lx,ly of the three landmarks; the two goals;
+# the two last messages (-1: none) (18 floats). Action a = 5 * message + move.
+REF_N, REF_L, REF_OBS, REF_A, REF_STATE = 2, 3, 14, 15, 18
+
+
+def ref_reset(g: int, seed: int) -> np.ndarray:
+    st = np.zeros(REF_STATE, np.float32)
+    _L().orc_ref_reset(C.c_uint64(g), C.c_uint64(seed), _p(st))
+    return st
+
+
+def ref_step(state: np.ndarray, actions, local_ratio: float = 0.5) -> tuple[np.ndarray, np.ndarray]:
+    st = _c(state, np.float32).copy()
+    act = _c(actions, np.int32)
+    rew = np.zeros(REF_N, np.float32)
+    _L().orc_ref_step(_p(st), _p(act), _p(rew), float(local_ratio))
+    return st, rew
+
+
+def ref_obs(state: np.ndarray) -> np.ndarray:
+    st = _c(state, np.float32)
+    out = np.zeros((REF_N, REF_OBS), np.float32)
+    _L().orc_ref_obs(_p(st), _p(out))
+    return out
+
+
+def ref_rollout(params_list, dims, T, n_envs, pairs, n_episodes, seed, bf16=False,
+                env_lo=0, env_hi=None, ext_logits=None, n_threads=0, local_ratio=None):
+    """Rollout over envs [env_lo, env_hi) of the simple reference (2 agents,
+    obs 14, 15 actions); local_ratio None: 0.5. Returns the arrays of
+    spread_rollout."""
+    env_hi = n_envs if env_hi is None else env_hi
+    W = env_hi - env_lo
+    i, h1, h2, A = dims
+    assert i == REF_OBS and A == REF_A
+    arrs, tbl = _param_table(params_list)
+    prs = _c(pairs, np.int32).reshape(-1, REF_N)
+    out = dict(obs=np.zeros((n_episodes, T, W, REF_N, i), np.float32),
+               action=np.zeros((n_episodes, T, W, REF_N), np.int8),
+               reward=np.zeros((n_episodes, T, W, REF_N), np.float32),
+               logits=np.zeros((n_episodes, T, W, REF_N, A), np.float32))
+    ext = None if ext_logits is None else _c(ext_logits, np.float32).reshape(n_episodes, T, W, REF_N, A)
+    _L().orc_ref_rollout(C.cast(tbl, C.c_void_p), h1, h2, int(bf16), T, n_envs, env_lo, env_hi, _p(prs),
+                         prs.shape[0], n_episodes, C.c_uint64(seed), _p(ext), _p(out["obs"]),
+                         _p(out["action"]), _p(out["reward"]), _p(out["logits"]), n_threads,
+                         0.5 if local_ratio is None else float(local_ratio))
+    del arrs
+    return out

@@ -28,6 +28,9 @@
 //  * App. B.1 "Simple Tag": one faster good agent, three slower adversaries,
 //    two obstacles that block the way; -10 to the good agent and +10 to the
 //    adversaries for each hit.
+//  * App. B.1 "Simple Reference": two agents that each know only the other's
+//    goal landmark, both speaking and moving, rewarded by their own distance
+//    and the average distance, weighted by local_ratio.
 //  * Collisions of App. B.1 as forces (push, tag, and spread as an option): a
 //    soft contact model between disks, a stated reading (the paper gives no
 //    force law).
@@ -49,8 +52,9 @@
 // fp64, zero beyond the margin, equal and opposite pairs, total velocity
 // against the closed form), simple push (hand-worked geometry, contact on both
 // agents) and simple tag (speed limits against the capped recursion, the hit
-// rule, immovable obstacles, the observation layout) are pinned by the CPU
-// tests, and whole spread episodes under forced actions (at
+// rule, immovable obstacles, the observation layout) and simple reference
+// (hand-worked rewards, the message delay, the moves against spread, the goal
+// draws) are pinned by the CPU tests, and whole spread episodes under forced actions (at
 // rest; a constant force from rest) match closed forms; episode returns of the
 // particle scenarios under sampled policies beyond those are "parity unpinned"
 // (no closed form exists).
@@ -154,7 +158,7 @@ int sample_masked(const float* logits, const uint8_t* legal, int A, float u) {
     if (first < 0) return -1;
     float m = logits[first];
     for (int a = first + 1; a < A; ++a) if (legal[a] && logits[a] > m) m = logits[a];
-    float e[8];
+    float e[16];
     float S = 0.0f;
     for (int a = 0; a < A; ++a) {
         e[a] = legal[a] ? det_expf(logits[a] - m) : 0.0f;
@@ -962,29 +966,104 @@ void tag_step(Tag& a, const int* action, float* reward) {
     reward[3] = -10.0f * (float)hits;
 }
 
-// One rollout driver for the fixed-size scenarios (push, tag): Env supplies N,
-// IN, reset, obs and step; all actions legal.
+// ---------------------------------------------------------------------------
+// Simple reference (App. B.1; readings of its description and of the speaker
+// listener it is said to resemble): two agents, three landmarks; each agent has
+// a goal landmark that only the other agent is told; both are speakers and
+// listeners. An action is a move and a message at once: a = 5 * message +
+// move (move 0..4 as in spread, message 0..2 naming a landmark), 15 actions.
+// Reset as spread (N = 2, L = 3, same chance counters); agent i's goal =
+// pick(x of the chance draw with step field 0xC0000000 + i, 3); no message yet.
+// Step: the spread dynamics for both agents (no contact), then each agent's
+// message is stored, seen by the other agent from the next step on. Rewards
+// after the move, d_i = |p_i - goal landmark of i|, rho = local_ratio (0.5
+// unless given): r_i = -((1 - rho) * ((d_0 + d_1) * 0.5) + rho * d_i) ("locally
+// ... their distance to their target landmark; globally ... the average
+// distance"), each operation rounded in fp32 in this order. Observation of
+// agent i (14 floats): velocity, the three landmarks - p_i, the other agent's
+// goal as a one-hot, the other agent's last message as a one-hot (zeros before
+// the first).
+// ---------------------------------------------------------------------------
+struct Reference {
+    Spread s;
+    int goal[2];
+    int msg[2];          // -1: none yet
+    float rho;
+};
+
+void ref_reset(Reference& a, uint64_t g, uint64_t seed) {
+    spread_reset(a.s, 2, 3, g, seed);
+    for (int i = 0; i < 2; ++i) {
+        a.goal[i] = (int)pick(draw(g, 0xC0000000u + (uint32_t)i, CHANCE, seed).x[0], 3);
+        a.msg[i] = -1;
+    }
+}
+
+void ref_obs(const Reference& a, int i, float* o) {
+    const Spread& s = a.s;
+    const int j = 1 - i;
+    for (int k = 0; k < 14; ++k) o[k] = 0.0f;
+    o[0] = s.vx[i]; o[1] = s.vy[i];
+    for (int l = 0; l < 3; ++l) { o[2 + 2 * l] = s.lx[l] - s.px[i]; o[3 + 2 * l] = s.ly[l] - s.py[i]; }
+    o[8 + a.goal[j]] = 1.0f;
+    if (a.msg[j] >= 0) o[11 + a.msg[j]] = 1.0f;
+}
+
+void ref_step(Reference& a, const int* action, float* reward) {
+    Spread& s = a.s;
+    for (int i = 0; i < 2; ++i) {
+        float fx, fy;
+        action_force(action[i] % 5, &fx, &fy);
+        s.vx[i] = s.vx[i] * 0.75f;
+        s.vy[i] = s.vy[i] * 0.75f;
+        s.vx[i] = s.vx[i] + fx * 0.1f;
+        s.vy[i] = s.vy[i] + fy * 0.1f;
+        s.px[i] = s.px[i] + s.vx[i] * 0.1f;
+        s.py[i] = s.py[i] + s.vy[i] * 0.1f;
+    }
+    for (int i = 0; i < 2; ++i) a.msg[i] = action[i] / 5;
+    float d[2];
+    for (int i = 0; i < 2; ++i) d[i] = dist2d(s.px[i], s.py[i], s.lx[a.goal[i]], s.ly[a.goal[i]]);
+    const float mean = (d[0] + d[1]) * 0.5f;
+    for (int i = 0; i < 2; ++i) {
+        const float shared = (1.0f - a.rho) * mean;
+        const float local = a.rho * d[i];
+        reward[i] = -(shared + local);
+    }
+}
+
+// One rollout driver for the fixed-size scenarios (push, tag, reference): Env
+// supplies N, IN, A, reset, obs and step; all actions legal.
 struct PushEnvDef {
     using S = Push;
-    static const int N = 2, IN = 8;
+    static const int N = 2, IN = 8, A = 5;
     static void reset(S& a, uint64_t g, uint64_t seed) { push_reset(a, g, seed); }
     static void obs(const S& a, int i, float* o) { push_obs(a, i, o); }
     static void step(S& a, const int* act, float* r) { push_step(a, act, r); }
 };
 struct TagEnvDef {
     using S = Tag;
-    static const int N = 4, IN = 16;
+    static const int N = 4, IN = 16, A = 5;
     static void reset(S& a, uint64_t g, uint64_t seed) { tag_reset(a, g, seed); }
     static void obs(const S& a, int i, float* o) { tag_obs(a, i, o); }
     static void step(S& a, const int* act, float* r) { tag_step(a, act, r); }
 };
+struct RefEnvDef {
+    using S = Reference;
+    static const int N = 2, IN = 14, A = 15;
+    static float rho;
+    static void reset(S& a, uint64_t g, uint64_t seed) { ref_reset(a, g, seed); a.rho = rho; }
+    static void obs(const S& a, int i, float* o) { ref_obs(a, i, o); }
+    static void step(S& a, const int* act, float* r) { ref_step(a, act, r); }
+};
+float RefEnvDef::rho = 0.5f;
 
 template <class Env>
 void scenario_rollout(const float* const* params, int h1, int h2, int bf16, int T, int64_t n_envs,
                       int64_t env_lo, int64_t env_hi, const int32_t* pairs, int32_t n_pairs,
                       int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
                       int8_t* action, float* reward, float* logits, int n_threads) {
-    const int N = Env::N, in = Env::IN, A = 5;
+    const int N = Env::N, in = Env::IN, A = Env::A;
     int64_t per = n_envs / n_pairs;
     int64_t W = env_hi - env_lo;
     parallel_for(W * n_episodes, n_threads, [&](int64_t job) {
@@ -997,11 +1076,12 @@ void scenario_rollout(const float* const* params, int h1, int h2, int bf16, int 
             int act[Env::N];
             for (int i = 0; i < N; ++i) {
                 int64_t idx = ((ep * T + t) * W + (e - env_lo)) * N + i;
-                float o[Env::IN], lg[8];
+                float o[Env::IN], lg[16];
                 Env::obs(st, i, o);
                 Mlp m{params[pairs[row * N + i]], in, h1, h2, A, bf16};
                 mlp_logits(m, o, lg);
-                uint8_t legal[8] = {1, 1, 1, 1, 1, 1, 1, 1};
+                uint8_t legal[16];
+                for (int q = 0; q < 16; ++q) legal[q] = 1;
                 float u = uniform24(draw(g, (uint32_t)t, (uint32_t)i, seed).x[0]);
                 act[i] = sample_masked(ext_logits ? ext_logits + idx * A : lg, legal, A, u);
                 if (obs) std::memcpy(obs + idx * in, o, sizeof(float) * in);
@@ -1486,6 +1566,45 @@ void orc_tag_rollout(const float* const* params, int h1, int h2, int bf16, int T
                      int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
                      int8_t* action, float* reward, float* logits, int n_threads) {
     scenario_rollout<TagEnvDef>(params, h1, h2, bf16, T, n_envs, env_lo, env_hi, pairs, n_pairs,
+                                n_episodes, seed, ext_logits, obs, action, reward, logits, n_threads);
+}
+
+// ---- Simple reference ----
+// state: px,py,vx,vy of the 2 agents, lx,ly of the 3 landmarks, the two goals
+// and the two last messages (-1: none) as floats ([4*2 + 2*3 + 4] = 18).
+static void ref_load(const float* st, Reference& a, float rho) {
+    sc_load(st, 2, 3, a.s);
+    a.goal[0] = (int)st[14]; a.goal[1] = (int)st[15];
+    a.msg[0] = (int)st[16]; a.msg[1] = (int)st[17];
+    a.rho = rho;
+}
+static void ref_store(const Reference& a, float* st) {
+    sc_store(a.s, st);
+    st[14] = (float)a.goal[0]; st[15] = (float)a.goal[1];
+    st[16] = (float)a.msg[0]; st[17] = (float)a.msg[1];
+}
+void orc_ref_reset(uint64_t g, uint64_t seed, float* state) {
+    Reference a;
+    ref_reset(a, g, seed);
+    ref_store(a, state);
+}
+void orc_ref_step(float* state, const int32_t* action, float* reward, float rho) {
+    Reference a;
+    ref_load(state, a, rho);
+    ref_step(a, action, reward);
+    ref_store(a, state);
+}
+void orc_ref_obs(const float* state, float* obs /*[2][14]*/) {
+    Reference a;
+    ref_load(state, a, 0.5f);
+    for (int i = 0; i < 2; ++i) ref_obs(a, i, obs + i * 14);
+}
+void orc_ref_rollout(const float* const* params, int h1, int h2, int bf16, int T, int64_t n_envs,
+                     int64_t env_lo, int64_t env_hi, const int32_t* pairs, int32_t n_pairs,
+                     int64_t n_episodes, uint64_t seed, const float* ext_logits, float* obs,
+                     int8_t* action, float* reward, float* logits, int n_threads, float rho) {
+    RefEnvDef::rho = rho;
+    scenario_rollout<RefEnvDef>(params, h1, h2, bf16, T, n_envs, env_lo, env_hi, pairs, n_pairs,
                                 n_episodes, seed, ext_logits, obs, action, reward, logits, n_threads);
 }
 
