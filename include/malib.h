@@ -53,7 +53,8 @@ typedef enum malib_env_kind {
     MALIB_ENV_ADVERSARY = 4,  /* simple adversary (App. B.1): 1 adversary, 2 good agents */
     MALIB_ENV_SPEAKER_LISTENER = 5, /* simple speaker listener (App. B.1): speaker, listener */
     MALIB_ENV_PUSH = 6,       /* simple push (App. B.1): 1 adversary, 1 good agent, 1 landmark */
-    MALIB_ENV_TAG = 7         /* simple tag (App. B.1): 3 adversaries, 1 good agent, 2 obstacles */
+    MALIB_ENV_TAG = 7,        /* simple tag (App. B.1): 3 adversaries, 1 good agent, 2 obstacles */
+    MALIB_ENV_REFERENCE = 8   /* simple reference (App. B.1): 2 agents that speak and move */
 } malib_env_kind;
 
 typedef enum malib_policy_kind {
@@ -69,7 +70,7 @@ typedef enum malib_dtype {
 /* Flags of malib_env_spec.flags and malib_eval_payoff_ex(). */
 #define MALIB_DUMP_LOGITS 1u          /* record logits (and obs, actions) in a malib_traj */
 #define MALIB_EXACT_EXPECTATION 2u    /* Kuhn: exact enumeration instead of Monte Carlo */
-#define MALIB_SPREAD_LOCAL_RATIO 4u   /* SPREAD: weight the reward terms by local_ratio */
+#define MALIB_SPREAD_LOCAL_RATIO 4u   /* SPREAD, REFERENCE: weight the reward terms by local_ratio */
 #define MALIB_SPREAD_CONTACT 8u       /* SPREAD: agents push each other apart (contact forces) */
 
 typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
@@ -90,8 +91,10 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  *   TAG:    n_agents 4 (agents 0..2 the adversaries, 3 the good agent),
  *           n_landmarks 2 (the obstacles), obs_dim 16, n_actions 5,
  *           episode_len >= 1
+ *   REFERENCE: n_agents 2, n_landmarks 3, obs_dim 14, n_actions 15 (a = 5 *
+ *           message + move), episode_len >= 1
  * n_envs is the number of parallel environments of a rollout (the particle
- * scenarios SPREAD, ADVERSARY, SPEAKER_LISTENER, PUSH, TAG).
+ * scenarios SPREAD, ADVERSARY, SPEAKER_LISTENER, PUSH, TAG, REFERENCE).
  * SPREAD reward of agent i after a step (App. B.1), with cover = sum over
  * landmarks of the distance to the nearest agent and coll_i = the number of
  * agents closer than 0.3 to agent i:
@@ -131,6 +134,15 @@ typedef struct malib_ctx malib_ctx;   /* opaque, library-owned */
  * adversary gets 10 h. Observation of agent i (16 floats): velocity, position,
  * obstacles - p_i, the other agents - p_i (ascending), the good agent's
  * velocity for an adversary (zeros for the good agent).
+ * REFERENCE (App. B.1 simple reference): at reset agent i's goal is one of the
+ * three landmarks (chance draw with step field 0xC0000000 + i), told only to
+ * the other agent. Action a moves by a % 5 (the spread dynamics, no contact)
+ * and sends message a / 5 (0..2), which the other agent observes from the next
+ * step on. With d_i = |p_i - goal_i| after the step and rho = local_ratio
+ * (MALIB_SPREAD_LOCAL_RATIO; 0.5 without it): r_i = -((1 - rho) ((d_0 + d_1)
+ * 0.5) + rho d_i). Observation of agent i (14 floats): velocity, the three
+ * landmarks - p_i, the other agent's goal as a one-hot, the other agent's last
+ * message as a one-hot (zeros before the first).
  */
 typedef struct malib_env_spec {
     int32_t env_kind;
@@ -232,8 +244,8 @@ int malib_pop_reset(malib_ctx* ctx);
 /*
  * malib_rollout - batched multi-agent rollout (Sec. 3.1, X(theta) ~ P(s, a, s'
  * | a ~ Comb_t); the Actor with k environments of the architecture figure).
- * SPREAD, ADVERSARY, SPEAKER_LISTENER, PUSH and TAG (App. B.1 particle
- * scenarios). Kernels: SPREAD N = 8 (obs 34, bf16 34-256-256-5 policies) on
+ * SPREAD, ADVERSARY, SPEAKER_LISTENER, PUSH, TAG and REFERENCE (App. B.1
+ * particle scenarios). Kernels: SPREAD N = 8 (obs 34, bf16 34-256-256-5 policies) on
  * the tensor cores; SPREAD N = 3 (obs 18) and the other scenarios with fp32
  * MLPs of hidden width 64, at most 128 environments per combination.
  * pair_ids (host or device) int32 [n_pairs][n_agents] holds one

@@ -16,14 +16,14 @@ import numpy as np
 from . import _abi
 from ._abi import (MALIB_BF16, MALIB_DUMP_LOGITS, MALIB_ENOTCONVERGED, MALIB_ENV_KUHN,
                    MALIB_ENV_LEDUC, MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY, MALIB_ENV_SPEAKER_LISTENER,
-                   MALIB_ENV_PUSH, MALIB_ENV_TAG, MALIB_EXACT_EXPECTATION, MALIB_F32, MALIB_POL_MLP,
+                   MALIB_ENV_PUSH, MALIB_ENV_TAG, MALIB_ENV_REFERENCE, MALIB_EXACT_EXPECTATION, MALIB_F32, MALIB_POL_MLP,
                    MALIB_POL_TABULAR, MALIB_SPREAD_CONTACT, EnvSpec, PolicyDesc, Traj)
 
 __all__ = ["MalibError", "Context", "EnvSpec", "make_spec", "policy_desc", "alloc_traj",
            "alloc_eval_dump", "malib_create", "malib_pop_load", "malib_rollout",
            "malib_eval_payoff", "malib_eval_payoff_ex", "malib_eval_payoff_noalloc", "MALIB_ENV_KUHN", "MALIB_ENV_LEDUC",
            "MALIB_ENV_SPREAD", "MALIB_ENV_ADVERSARY", "MALIB_ENV_SPEAKER_LISTENER", "MALIB_ENV_PUSH",
-           "MALIB_ENV_TAG", "MALIB_POL_TABULAR", "MALIB_POL_MLP", "MALIB_F32", "MALIB_BF16",
+           "MALIB_ENV_TAG", "MALIB_ENV_REFERENCE", "MALIB_POL_TABULAR", "MALIB_POL_MLP", "MALIB_F32", "MALIB_BF16",
            "MALIB_DUMP_LOGITS", "MALIB_EXACT_EXPECTATION", "MALIB_SPREAD_CONTACT", "MALIB_ENOTCONVERGED"]
 
 

@@ -18,7 +18,7 @@ STATUS_NAMES = {0: "OK", -1: "EINVAL", -2: "ENOMEM", -3: "ECUDA", -4: "ESTATE", 
                 -6: "EUNSUPPORTED", -7: "ENOTCONVERGED"}
 
 MALIB_ENV_KUHN, MALIB_ENV_LEDUC, MALIB_ENV_SPREAD, MALIB_ENV_ADVERSARY = 1, 2, 3, 4
-MALIB_ENV_SPEAKER_LISTENER, MALIB_ENV_PUSH, MALIB_ENV_TAG = 5, 6, 7
+MALIB_ENV_SPEAKER_LISTENER, MALIB_ENV_PUSH, MALIB_ENV_TAG, MALIB_ENV_REFERENCE = 5, 6, 7, 8
 MALIB_POL_TABULAR, MALIB_POL_MLP = 1, 2
 MALIB_F32, MALIB_BF16 = 0, 1
 MALIB_DUMP_LOGITS, MALIB_EXACT_EXPECTATION, MALIB_SPREAD_LOCAL_RATIO = 1, 2, 4

@@ -174,6 +174,11 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
                 return fail(c, MALIB_EINVAL, "push spec needs n_agents 2, n_landmarks 1, obs_dim 8, n_actions 5");
             if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
             break;
+        case MALIB_ENV_REFERENCE:
+            if (s->n_agents != 2 || s->n_landmarks != 3 || s->obs_dim != 14 || s->n_actions != 15)
+                return fail(c, MALIB_EINVAL, "reference spec needs n_agents 2, n_landmarks 3, obs_dim 14, n_actions 15");
+            if (s->episode_len < 1) return fail(c, MALIB_EINVAL, "episode_len must be >= 1");
+            break;
         case MALIB_ENV_TAG:
             if (s->n_agents != 4 || s->n_landmarks != 2 || s->obs_dim != 16 || s->n_actions != 5)
                 return fail(c, MALIB_EINVAL, "tag spec needs n_agents 4, n_landmarks 2, obs_dim 16, n_actions 5");
@@ -187,8 +192,8 @@ int check_spec(malib_ctx* c, const malib_env_spec* s) {
     if ((s->flags & MALIB_SPREAD_CONTACT) && s->env_kind != MALIB_ENV_SPREAD)
         return fail(c, MALIB_EINVAL, "MALIB_SPREAD_CONTACT applies to SPREAD only");
     if (s->flags & MALIB_SPREAD_LOCAL_RATIO) {
-        if (s->env_kind != MALIB_ENV_SPREAD)
-            return fail(c, MALIB_EINVAL, "MALIB_SPREAD_LOCAL_RATIO applies to SPREAD only");
+        if (s->env_kind != MALIB_ENV_SPREAD && s->env_kind != MALIB_ENV_REFERENCE)
+            return fail(c, MALIB_EINVAL, "MALIB_SPREAD_LOCAL_RATIO applies to SPREAD and REFERENCE only");
         if (!(s->local_ratio >= 0.0f && s->local_ratio <= 1.0f))
             return fail(c, MALIB_EINVAL, "local_ratio must lie in [0, 1]");
     }
@@ -694,7 +699,7 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     // scenarios of the fp32 rollout kernel other than spread (one policy width, hidden 64)
     const bool other = spec->env_kind == MALIB_ENV_ADVERSARY ||
                        spec->env_kind == MALIB_ENV_SPEAKER_LISTENER || spec->env_kind == MALIB_ENV_PUSH ||
-                       spec->env_kind == MALIB_ENV_TAG;
+                       spec->env_kind == MALIB_ENV_TAG || spec->env_kind == MALIB_ENV_REFERENCE;
     if (spec->env_kind != MALIB_ENV_SPREAD && !other)
         return fail(c, MALIB_EUNSUPPORTED, "rollout is built for the particle environments");
     if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");

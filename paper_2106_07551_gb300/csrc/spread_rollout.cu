@@ -14,10 +14,12 @@
 // the trajectory, so each episode's observations of a step leave shared memory
 // as one bulk copy; actions, rewards and done flags are stored per thread.
 // The same kernel, templated on the scenario, runs the simple adversary, the
-// simple speaker listener, the simple push and the simple tag (App. B.1) with
-// their own environment code, and spread with contact forces between agents.
+// simple speaker listener, the simple push, the simple tag and the simple
+// reference (App. B.1) with their own environment code, and spread with contact
+// forces between agents.
 #include "adversary_env.cuh"
 #include "push_env.cuh"
+#include "ref_env.cuh"
 #include "sl_env.cuh"
 #include "tag_env.cuh"
 #include "device_common.cuh"
@@ -34,11 +36,11 @@ namespace {
 // the kernel runs per agent (kPerAgent): X and LG hold one agent's rows, each
 // agent's observations are built just before its pass and stored to the
 // trajectory from registers, and its action is drawn right after it.
-template <int N, int IN, int H>
+template <int N, int IN, int H, int A = 5>
 struct SpreadF32Smem {
     static_assert(H == 64, "the 256-row engine has 64 hidden units");
-    using M = MlpF32R8<IN, 5>;
-    using L = F32Layout<IN, H, 5>;
+    using M = MlpF32R8<IN, A>;
+    using L = F32Layout<IN, H, A>;
     static constexpr int R = M::kRows;            // 2 episode slots x 128 envs
     static constexpr size_t kAllBytes =
         (size_t)(N * L::kSize + N * R * M::XS + R * M::HS + N * R * M::LS) * 4;
@@ -58,8 +60,11 @@ struct SpreadF32Smem {
 // speaker listener (N = 2, three landmarks, obs 11; the speaker may take
 // actions 0..2 only); kPush - the simple push (N = 2, one landmark, obs 8);
 // kTag - the simple tag (N = 4, two obstacles, obs 16); kSpreadContact -
-// spread whose agents also push each other apart.
-constexpr int kSpread = 0, kAdversary = 1, kSpeakerListener = 2, kPush = 3, kTag = 4, kSpreadContact = 5;
+// spread whose agents also push each other apart; kReference - the simple
+// reference (N = 2, three landmarks, obs 14, 15 actions: move and message).
+constexpr int kSpread = 0, kAdversary = 1, kSpeakerListener = 2, kPush = 3, kTag = 4, kSpreadContact = 5,
+              kReference = 6;
+__host__ __device__ constexpr int actions_of(int scen) { return scen == kReference ? kRefActions : 5; }
 
 template <int kScen, int N>
 struct ScenarioEnv {
@@ -81,6 +86,10 @@ template <int N>
 struct ScenarioEnv<kTag, N> {
     using type = TagEnv;
 };
+template <int N>
+struct ScenarioEnv<kReference, N> {
+    using type = RefEnv;
+};
 
 template <int N, int IN, int H, int kScen = kSpread>
 __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs a) {
@@ -89,7 +98,9 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                   "the simple speaker listener has 2 agents, obs 11");
     static_assert(kScen != kPush || (N == 2 && IN == kPushObs), "the simple push has 2 agents, obs 8");
     static_assert(kScen != kTag || (N == 4 && IN == kTagObs), "the simple tag has 4 agents, obs 16");
-    using SM = SpreadF32Smem<N, IN, H>;
+    static_assert(kScen != kReference || (N == 2 && IN == kRefObs), "the simple reference has 2 agents, obs 14");
+    constexpr int A = actions_of(kScen);
+    using SM = SpreadF32Smem<N, IN, H, A>;
     using M = typename SM::M;
     using L = typename SM::L;
     constexpr int R = SM::R;
@@ -160,6 +171,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
             else if constexpr (kScen == kSpeakerListener) sl_reset(s, g, a.seed);
             else if constexpr (kScen == kPush) push_reset(s, g, a.seed);
             else if constexpr (kScen == kTag) tag_reset(s, g, a.seed);
+            else if constexpr (kScen == kReference) ref_reset(s, g, a.seed);
             else spread_reset<N>(s, g, a.seed);
         }
 
@@ -174,6 +186,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                     if (mine) {
                         float o[XS];
                         if constexpr (kScen == kTag) tag_obs<XS>(s, i, o);
+                        else if constexpr (kScen == kReference) ref_obs<XS>(s, i, o);
                         else if constexpr (kScen == kPush) push_obs<XS>(s, i, o);
                         else if constexpr (kScen == kAdversary) adv_obs<XS>(s, i, o);
                         else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, i, o);
@@ -193,15 +206,15 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                     M::layer23(H1, LG, w + L::kW2T, w + L::kB2, w + L::kW3, w + L::kB3);
                     if (mine) {
                         // LG is rewritten only after the next pass's layer-1 barrier
-                        float lg[5];
+                        float lg[A];
 #pragma unroll
-                        for (int k = 0; k < 5; ++k) lg[k] = LG[tid * M::LS + k];
+                        for (int k = 0; k < A; ++k) lg[k] = LG[tid * M::LS + k];
                         const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
-                        const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : 0x1Fu;
-                        act[i] = sample_masked<5>(lg, legal, uu);
+                        const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : (1u << A) - 1u;
+                        act[i] = sample_masked<A>(lg, legal, uu);
                         if (a.logits)
 #pragma unroll
-                            for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
+                            for (int k = 0; k < A; ++k) a.logits[(ix + i) * A + k] = lg[k];
                     }
                 }
                 if (mine) {
@@ -210,6 +223,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                     else if constexpr (kScen == kSpeakerListener) sl_step(s, act, r);
                     else if constexpr (kScen == kPush) push_step(s, act, r);
                     else if constexpr (kScen == kTag) tag_step(s, act, r);
+                    else if constexpr (kScen == kReference) ref_step(s, act, r, a.local_ratio < 0.f ? 0.5f : a.local_ratio);
                     else spread_step<N, kScen == kSpreadContact>(s, act, r, a.local_ratio);
 #pragma unroll
                     for (int i = 0; i < N; ++i) {
@@ -228,6 +242,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                     else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, i, o);
                     else if constexpr (kScen == kPush) push_obs<XS>(s, i, o);
                     else if constexpr (kScen == kTag) tag_obs<XS>(s, i, o);
+                    else if constexpr (kScen == kReference) ref_obs<XS>(s, i, o);
                     else spread_obs<N, XS>(s, i, o);
                     float4* xr = reinterpret_cast<float4*>(X + (tid * N + i) * XS);
 #pragma unroll
@@ -260,20 +275,21 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                 const int64_t ix = ((ep * T + t) * a.n_envs + env) * N;
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
-                    float lg[5];
+                    float lg[A];
 #pragma unroll
-                    for (int k = 0; k < 5; ++k) lg[k] = LG[(i * R + tid) * M::LS + k];
+                    for (int k = 0; k < A; ++k) lg[k] = LG[(i * R + tid) * M::LS + k];
                     const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
-                    const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : 0x1Fu;
-                    act[i] = sample_masked<5>(lg, legal, uu);
+                    const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : (1u << A) - 1u;
+                    act[i] = sample_masked<A>(lg, legal, uu);
                     if (a.logits)
 #pragma unroll
-                        for (int k = 0; k < 5; ++k) a.logits[(ix + i) * 5 + k] = lg[k];
+                        for (int k = 0; k < A; ++k) a.logits[(ix + i) * A + k] = lg[k];
                 }
                 if constexpr (kScen == kAdversary) adv_step(s, act, r);
                 else if constexpr (kScen == kSpeakerListener) sl_step(s, act, r);
                 else if constexpr (kScen == kPush) push_step(s, act, r);
                 else if constexpr (kScen == kTag) tag_step(s, act, r);
+                else if constexpr (kScen == kReference) ref_step(s, act, r, a.local_ratio < 0.f ? 0.5f : a.local_ratio);
                 else spread_step<N, kScen == kSpreadContact>(s, act, r, a.local_ratio);
 #pragma unroll
                 for (int i = 0; i < N; ++i) {
@@ -291,7 +307,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 
 template <int N, int IN, int H, int kScen = kSpread>
 cudaError_t launch_spread_nih(const RolloutArgs& a, int n_sm, cudaStream_t s) {
-    using SM = SpreadF32Smem<N, IN, H>;
+    using SM = SpreadF32Smem<N, IN, H, actions_of(kScen)>;
     cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H, kScen>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SM::kBytes);
@@ -323,6 +339,10 @@ cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm
     }
     if (a.env_kind == MALIB_ENV_PUSH) {
         if (hidden == 64) return launch_spread_nih<2, kPushObs, 64, kPush>(a, n_sm, s);
+        return cudaErrorInvalidValue;
+    }
+    if (a.env_kind == MALIB_ENV_REFERENCE) {
+        if (hidden == 64) return launch_spread_nih<2, kRefObs, 64, kReference>(a, n_sm, s);
         return cudaErrorInvalidValue;
     }
     if (a.env_kind == MALIB_ENV_TAG) {

@@ -154,3 +154,26 @@ def test_contact_flag_refused_outside_spread():
     with pytest.raises(MalibError, match="EINVAL"):
         ctx.rollout(spec, w.pair_ids, 1, 0, alloc_traj(spec, 1))
     ctx.close()
+
+
+@pytest.mark.parametrize("n_envs,epp,n_eps,ratio", [(512, 64, 3, None), (256, 128, 2, 0.2), (48, 16, 5, 1.0)])
+def test_reference_replay_parity(n_envs, epp, n_eps, ratio):
+    """Simple reference (15 actions: a move and a message), with and without
+    local_ratio."""
+    need_gpu()
+    w = workloads.reference(n_envs=n_envs, pop=5, envs_per_pair=epp, with_bias=True, seed=1200 + epp)
+    ctx = context()
+    load_population(ctx, w)
+    spec = spec_of(w, MALIB_DUMP_LOGITS, local_ratio=ratio)
+    traj = alloc_traj(spec, n_eps, logits=True)
+    ctx.rollout(spec, w.pair_ids, n_eps, 777, traj)
+    ctx.sync()
+    g = {k: v.cpu().numpy() for k, v in traj.items()}
+
+    def replay(params, dims, T, n_envs, pairs, n_eps, seed, env_lo=0, env_hi=None, ext_logits=None):
+        return oracle.ref_rollout(params, dims, T, n_envs, pairs, n_eps, seed, env_lo=env_lo,
+                                  env_hi=env_hi, ext_logits=ext_logits, local_ratio=ratio)
+
+    check(replay, w, g, n_eps, 777, 0, n_envs)
+    assert g["action"].max() >= 5                   # messages other than 0 are sent
+    ctx.close()

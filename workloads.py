@@ -26,7 +26,7 @@ import numpy as np
 SEED_BASE = 2106075510
 
 ENV_KUHN, ENV_LEDUC, ENV_SPREAD, ENV_ADVERSARY = 1, 2, 3, 4
-ENV_SPEAKER_LISTENER, ENV_PUSH, ENV_TAG = 5, 6, 7
+ENV_SPEAKER_LISTENER, ENV_PUSH, ENV_TAG, ENV_REFERENCE = 5, 6, 7, 8
 POL_TABULAR, POL_MLP = 1, 2
 F32, BF16 = 0, 1
 
@@ -210,6 +210,24 @@ def tag(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_episodes: int = 1
         w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
     n_pairs = max(1, n_envs // envs_per_pair)
     w.pair_ids = rng.integers(0, pop, size=(n_pairs, 4)).astype(np.int32)
+    return w
+
+
+def reference(n_envs: int = 4096, pop: int = 16, hidden: int = 64, n_episodes: int = 1,
+              episode_len: int = 25, envs_per_pair: int = 128, seed: int = SEED_BASE + 10,
+              with_bias: bool = False, name: str | None = None) -> Workload:
+    """Simple reference (App. B.1): 2 agents that speak and move, three
+    landmarks; MLP 14-hidden-hidden-15 fp32 policies (15 = 5 moves x 3
+    messages) from one shared pool, assigned by the seed per (block of
+    envs_per_pair envs, agent slot)."""
+    rng = np.random.default_rng(seed)
+    dims = (14, hidden, hidden, 15)
+    w = Workload(name or f"reference_{n_envs}env_mlp{hidden}_f32", ENV_REFERENCE, 2, 3, 14, 15,
+                 episode_len, n_envs, n_episodes=n_episodes, seed=seed)
+    for _ in range(pop):
+        w.policies.append(Policy(POL_MLP, F32, -1, dims, random_mlp(rng, dims, with_bias)))
+    n_pairs = max(1, n_envs // envs_per_pair)
+    w.pair_ids = rng.integers(0, pop, size=(n_pairs, 2)).astype(np.int32)
     return w
 
 
