@@ -61,7 +61,7 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "speaker_listener",
-                                           "leduc_bf16", "spread8", "meta", "learner", "push", "tag"],
+                                           "leduc_bf16", "spread8", "meta", "learner", "push", "tag", "reference"],
                     default="leduc_bf16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -181,6 +181,8 @@ def workload(name: str, rank: int, hands=None):
         w = workloads.push(n_envs=4096, pop=16, n_episodes=100 if hands is None else hands)
     elif name == "tag":
         w = workloads.tag(n_envs=4096, pop=16, n_episodes=100 if hands is None else hands)
+    elif name == "reference":
+        w = workloads.reference(n_envs=4096, pop=16, n_episodes=100 if hands is None else hands)
     else:
         w = workloads.config(3, **({"n_episodes": 100} if hands is None else over))
     return w
@@ -209,10 +211,10 @@ def config_of(w, name):
         return {"workload": f"simple_speaker_listener_4096env_mlp11-64-64-5_f32_{w.n_episodes}episodes",
                 "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
                 "episode_len": 25, "l2": "trajectory output exceeds L2; flushed as well"}
-    if name in ("push", "tag"):
-        return {"workload": f"simple_{name}_4096env_mlp{w.obs_dim}-64-64-5_f32_{w.n_episodes}episodes",
+    if name in ("push", "tag", "reference"):
+        return {"workload": f"simple_{name}_4096env_mlp{w.obs_dim}-64-64-{w.n_actions}_f32_{w.n_episodes}episodes",
                 "envs": w.n_envs, "combinations": w.n_pairs, "episodes_per_env": w.n_episodes,
-                "episode_len": 25, "contact_forces": True,
+                "episode_len": 25, "contact_forces": name != "reference",
                 "l2": "trajectory output exceeds L2; flushed as well"}
     if name == "kuhn":
         return {"workload": "kuhn_4x4_tabular_10000hands", "pairs": w.n_pairs,
@@ -268,8 +270,8 @@ def oracle_rollout_sample(w, name, target_s: float, threads: int):
         elif name == "speaker_listener":
             oracle.sl_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, eps, w.seed,
                               env_lo=0, env_hi=n, n_threads=threads)
-        elif name in ("push", "tag"):
-            roll = oracle.push_rollout if name == "push" else oracle.tag_rollout
+        elif name in ("push", "tag", "reference"):
+            roll = {"push": oracle.push_rollout, "tag": oracle.tag_rollout, "reference": oracle.ref_rollout}[name]
             roll(params, dims, w.episode_len, w.n_envs, w.pair_ids, eps, w.seed, env_lo=0, env_hi=n,
                  n_threads=threads)
         else:
@@ -381,8 +383,8 @@ def oracle_step_fn(w, name, threads, per_step):
         elif name == "speaker_listener":
             oracle.sl_rollout(params, dims, w.episode_len, w.n_envs, w.pair_ids, 1, seed,
                               env_lo=0, env_hi=n, n_threads=threads)
-        elif name in ("push", "tag"):
-            roll = oracle.push_rollout if name == "push" else oracle.tag_rollout
+        elif name in ("push", "tag", "reference"):
+            roll = {"push": oracle.push_rollout, "tag": oracle.tag_rollout, "reference": oracle.ref_rollout}[name]
             roll(params, dims, w.episode_len, w.n_envs, w.pair_ids, 1, seed, env_lo=0, env_hi=n,
                  n_threads=threads)
         else:
@@ -455,7 +457,7 @@ def run_ours(args):
     d_pairs = torch.from_numpy(w.pair_ids).to(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     seed0 = w.seed + 1_000_003 * rank
-    rollout = args.workload in ("spread3", "spread8", "adversary3", "speaker_listener", "push", "tag")
+    rollout = args.workload in ("spread3", "spread8", "adversary3", "speaker_listener", "push", "tag", "reference")
     if rollout:
         traj = alloc_traj(spec, w.n_episodes)
         steps_per_call = w.n_envs * w.episode_len * w.n_episodes
@@ -521,6 +523,7 @@ def run_ours(args):
              "speaker_listener": "spread_rollout_f32_kernel<2,11,64,2>",
              "push": "spread_rollout_f32_kernel<2,8,64,3>",
              "tag": "spread_rollout_f32_kernel<4,16,64,4>",
+             "reference": "spread_rollout_f32_kernel<2,14,64,6>",
              "leduc_bf16": "leduc_eval_tc_kernel",
              "spread8": "spread_rollout_tc_kernel"}[args.workload]
     basis = (f"fp32 FMA: {n_sm} SMs (queried) x {FP32_LANES_PER_SM} lanes x 2 flop"
