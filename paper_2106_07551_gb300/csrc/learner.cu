@@ -20,8 +20,10 @@
 //  3. learn_baseline_kernel: M and b = sum G / M in a fixed order (one block).
 //  4. learn_grad_kernel: persistent CTAs over tiles of 128 samples: forward
 //     (fp32 FMA, hidden 64), logits, softmax, dL/dz, the backward pass, and
-//     the weight gradients accumulated in registers over the CTA's tiles;
-//     each CTA writes its partial gradient.
+//     the weight gradients accumulated in registers over the CTA's tiles (each
+//     thread a 4 x 4 block of dW2 and a few entries of the rest); the tile's
+//     activations are stored feature-major in shared memory so that every
+//     product reads 16-byte vectors; each CTA writes its partial gradient.
 //  5. learn_reduce_kernel: the partials summed over CTAs in a fixed order into
 //     the gradient (the malib_policy_desc layout) and the loss statistics.
 // Deterministic: no atomics, every sum in a fixed order.
@@ -36,8 +38,12 @@ namespace malib {
 namespace {
 
 constexpr int kH = 64, kA = 5, kTile = 128, kThreads = 256;
-constexpr int kHS = kH + 1;          // row stride of the per-sample hidden tiles
-constexpr int kXS = kLearnMaxIn + 1;   // row stride of the observation tile
+// The per-tile activations are stored feature-major ([feature][sample], rows of
+// kTS floats, 16-byte aligned), so that a thread's 8 samples or 4 consecutive
+// samples are one or two 16-byte loads; kTS = 132 spreads rows 16 apart over
+// the banks.
+constexpr int kTS = kTile + 4;
+constexpr int kXR = kLearnMaxIn;     // observation feature rows
 
 // Shared-memory layout of learn_grad_kernel (floats).
 constexpr int kSW1T = 0;                          // [in][64]: W1T[k][j] = W1[j][k]
@@ -47,15 +53,16 @@ constexpr int kSW2 = kSW2T + kH * kH;             // [64][64]: W2[j][k]
 constexpr int kSB2 = kSW2 + kH * kH;
 constexpr int kSW3 = kSB2 + kH;                   // [5][64]
 constexpr int kSB3 = kSW3 + kA * kH;              // [8]
-constexpr int kSX = kSB3 + 8;                     // [128][kXS]
-constexpr int kSH1 = kSX + kTile * kXS;           // [128][65] post-ReLU layer 1
-constexpr int kSH2 = kSH1 + kTile * kHS;          // [128][65] post-ReLU layer 2
-constexpr int kSD2 = kSH2 + kTile * kHS;          // [128][65] dL/d(pre-activation 2)
-constexpr int kSD1 = kSD2 + kTile * kHS;          // [128][65] dL/d(pre-activation 1)
-constexpr int kSDZ = kSD1 + kTile * kHS;          // [128][8] dL/dz
-constexpr int kSFloats = kSDZ + kTile * 8;
+constexpr int kSX = kSB3 + 8;                     // XT [in][kTS] observations
+constexpr int kSH1 = kSX + kXR * kTS;             // H1T [64][kTS] post-ReLU layer 1
+constexpr int kSH2 = kSH1 + kH * kTS;             // H2T [64][kTS] post-ReLU layer 2
+constexpr int kSD2 = kSH2 + kH * kTS;             // D2T [64][kTS] dL/d(pre-activation 2)
+constexpr int kSD1 = kSD2 + kH * kTS;             // D1T [64][kTS] dL/d(pre-activation 1)
+constexpr int kSDZ = kSD1 + kH * kTS;             // DZT [8][kTS] dL/dz
+constexpr int kSFloats = kSDZ + 8 * kTS;
 constexpr size_t kSBytes = (size_t)kSFloats * 4;
 static_assert(kSBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
+static_assert(kSX % 4 == 0 && kTS % 4 == 0, "16-byte aligned rows");
 
 __global__ void __launch_bounds__(1024) learn_slots_kernel(LearnArgs a) {
     __shared__ int warp_n[32];
@@ -126,6 +133,53 @@ __global__ void learn_baseline_kernel(LearnArgs a, int n_blocks) {
     a.stats[1] = M > 0 ? s / M : 0.0;
 }
 
+// Sample s of the policy's sample order: (slot, episode, step, env) -> the
+// trajectory index of its (episode, step, env, agent).
+__device__ __forceinline__ int64_t sample_index(const LearnArgs& a, int64_t s, int epp) {
+    const int r = (int)(s % epp);
+    const int64_t q = s / epp;                        // (slot, e, t)
+    const int t = (int)(q % a.T);
+    const int64_t q2 = q / a.T;
+    const int64_t e = q2 % a.n_episodes, slot = q2 / a.n_episodes;
+    const int ck = a.slots[slot];
+    const int c = ck / a.n_agents, ka = ck - c * a.n_agents;
+    const int64_t env = (int64_t)c * epp + r;
+    return ((e * a.T + t) * a.n_envs + env) * a.n_agents + ka;
+}
+
+// H_out[j][s] = relu(b[j] + sum_k W[k][j] H_in[k][s]) for this thread's 8
+// samples (8 sg ..) and 4 outputs (ng + 16 q): two 16-byte loads of H_in and
+// four weights per k.
+__device__ __forceinline__ void dense_relu(const float* __restrict__ Win, const float* __restrict__ b,
+                                           const float* __restrict__ Hin, int K, float* __restrict__ Hout,
+                                           int sg, int ng) {
+    float acc[4][8];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[q][i] = b[ng + 16 * q];
+#pragma unroll 4
+    for (int k = 0; k < K; ++k) {
+        const float4 x0 = *reinterpret_cast<const float4*>(Hin + k * kTS + 8 * sg);
+        const float4 x1 = *reinterpret_cast<const float4*>(Hin + k * kTS + 8 * sg + 4);
+        const float x[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float w = Win[k * kH + ng + 16 * q];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[q][i] = fmaf(w, x[i], acc[q][i]);
+        }
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        float* o = Hout + (ng + 16 * q) * kTS + 8 * sg;
+        *reinterpret_cast<float4*>(o) = make_float4(fmaxf(acc[q][0], 0.f), fmaxf(acc[q][1], 0.f),
+                                                    fmaxf(acc[q][2], 0.f), fmaxf(acc[q][3], 0.f));
+        *reinterpret_cast<float4*>(o + 4) = make_float4(fmaxf(acc[q][4], 0.f), fmaxf(acc[q][5], 0.f),
+                                                        fmaxf(acc[q][6], 0.f), fmaxf(acc[q][7], 0.f));
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int tid = threadIdx.x;
@@ -150,112 +204,58 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
     const float base = (float)a.stats[1];
     const int64_t n_tiles = (M + kTile - 1) / kTile;
 
+    float* XT = sm + kSX;
+    float* H1T = sm + kSH1;
+    float* H2T = sm + kSH2;
+    float* D2T = sm + kSD2;
+    float* D1T = sm + kSD1;
+    float* DZT = sm + kSDZ;
+    const int sg = tid >> 4, ng = tid & 15;           // layers: samples 8 sg .., outputs ng + 16 q
     // this thread's gradient entries, accumulated over the CTA's tiles
-    const int jb = tid >> 4, kb = tid & 15;                  // dW2: rows 4 jb.., cols 4 kb..
-    float gW2[4][4] = {};
-    const int nW1 = kH * in;                                 // dW1 entries t + 256 q
-    float gW1[(kH * kLearnMaxIn + kThreads - 1) / kThreads] = {};
-    float gW3[2] = {};                                       // entries t, t + 256 of [5][64]
-    float gB = 0.f;                                          // b1 (t < 64), b2 (64..127), b3 (128..132)
-    float lsum = 0.f, hsum = 0.f;                            // loss and entropy of this thread's samples
-    const int sg = tid >> 4, ng = tid & 15;                  // layers: samples 8 sg.., neurons 4 ng..
-
-    float* X = sm + kSX;
-    float* H1 = sm + kSH1;
-    float* H2 = sm + kSH2;
-    float* D2 = sm + kSD2;
-    float* D1 = sm + kSD1;
-    float* DZ = sm + kSDZ;
+    float gW2[4][4] = {};                              // dW2[ng' + 16 p][kb + 16 q], ng' = sg
+    const int w1j = tid & 63, w1k = tid >> 6;          // dW1[w1j][w1k + 4 q]
+    float gW1[kLearnMaxIn / 4] = {};
+    float gW3[2] = {};                                 // dW3 entries tid, tid + 256 of [5][64]
+    float gB = 0.f;                                    // b1 (tid < 64), b2 (64..127), b3 (128..132)
+    float lsum = 0.f, hsum = 0.f;                      // loss and entropy of this thread's samples
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
         const int64_t s0 = tile * kTile;
-        // the tile's observations (zero rows past M)
-        for (int i = tid; i < kTile * in; i += kThreads) {
-            const int row = i / in, k = i - row * in;
-            const int64_t s = s0 + row;
-            float v = 0.f;
+        // the tile's observations (feature-major; zero columns past M), and for
+        // the logits phase each sample's action and return
+        int act = 0;
+        float ret = 0.f;
+        {
+            const int r = tid & (kTile - 1), half = tid >> 7;
+            const int64_t s = s0 + r;
             if (s < M) {
-                const int r = (int)(s % epp);
-                const int64_t q = s / epp;                    // (slot, e, t)
-                const int t = (int)(q % a.T);
-                const int64_t q2 = q / a.T;
-                const int64_t e = q2 % a.n_episodes, slot = q2 / a.n_episodes;
-                const int ck = a.slots[slot];
-                const int c = ck / a.n_agents, ka = ck - c * a.n_agents;
-                const int64_t env = (int64_t)c * epp + r;
-                v = a.obs[(((e * a.T + t) * a.n_envs + env) * a.n_agents + ka) * a.xs + k];
-            }
-            X[row * kXS + k] = v;
-        }
-        __syncthreads();
-        // layer 1: H1 = relu(W1 x + b1)
-        {
-            float acc[8][4];
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-#pragma unroll
-                for (int q = 0; q < 4; ++q) acc[i][q] = sm[kSB1 + 4 * ng + q];
-            for (int k = 0; k < in; ++k) {
-                const float4 w = *reinterpret_cast<const float4*>(sm + kSW1T + k * kH + 4 * ng);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const float x = X[(8 * sg + i) * kXS + k];
-                    acc[i][0] = fmaf(w.x, x, acc[i][0]);
-                    acc[i][1] = fmaf(w.y, x, acc[i][1]);
-                    acc[i][2] = fmaf(w.z, x, acc[i][2]);
-                    acc[i][3] = fmaf(w.w, x, acc[i][3]);
+                const int64_t ix = sample_index(a, s, epp);
+                const float* orow = a.obs + ix * a.xs;
+                for (int k = half; k < in; k += 2) XT[k * kTS + r] = orow[k];
+                if (half == 0) {
+                    act = a.action[ix];
+                    ret = a.G[s];
                 }
+            } else {
+                for (int k = half; k < in; k += 2) XT[k * kTS + r] = 0.f;
             }
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-#pragma unroll
-                for (int q = 0; q < 4; ++q) H1[(8 * sg + i) * kHS + 4 * ng + q] = fmaxf(acc[i][q], 0.f);
         }
         __syncthreads();
-        // layer 2: H2 = relu(W2 h1 + b2)
-        {
-            float acc[8][4];
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-#pragma unroll
-                for (int q = 0; q < 4; ++q) acc[i][q] = sm[kSB2 + 4 * ng + q];
-#pragma unroll 4
-            for (int k = 0; k < kH; ++k) {
-                const float4 w = *reinterpret_cast<const float4*>(sm + kSW2T + k * kH + 4 * ng);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const float x = H1[(8 * sg + i) * kHS + k];
-                    acc[i][0] = fmaf(w.x, x, acc[i][0]);
-                    acc[i][1] = fmaf(w.y, x, acc[i][1]);
-                    acc[i][2] = fmaf(w.z, x, acc[i][2]);
-                    acc[i][3] = fmaf(w.w, x, acc[i][3]);
-                }
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-#pragma unroll
-                for (int q = 0; q < 4; ++q) H2[(8 * sg + i) * kHS + 4 * ng + q] = fmaxf(acc[i][q], 0.f);
-        }
+        dense_relu(sm + kSW1T, sm + kSB1, XT, in, H1T, sg, ng);
         __syncthreads();
-        // logits, softmax and dL/dz, one sample per thread
+        dense_relu(sm + kSW2T, sm + kSB2, H1T, kH, H2T, sg, ng);
+        __syncthreads();
+        // logits, softmax and dL/dz, one sample per thread (threads 0 .. 127)
         if (tid < kTile) {
             const int64_t s = s0 + tid;
             float dz[kA] = {0.f, 0.f, 0.f, 0.f, 0.f};
             if (s < M) {
-                const int r = (int)(s % epp);
-                const int64_t q = s / epp;
-                const int t = (int)(q % a.T);
-                const int64_t q2 = q / a.T;
-                const int64_t e = q2 % a.n_episodes, slot = q2 / a.n_episodes;
-                const int ck = a.slots[slot];
-                const int c = ck / a.n_agents, ka = ck - c * a.n_agents;
-                const int64_t env = (int64_t)c * epp + r;
-                const int act = a.action[((e * a.T + t) * a.n_envs + env) * a.n_agents + ka];
-                const float adv = a.G[s] - base;
+                const float adv = ret - base;
                 float z[kA];
 #pragma unroll
                 for (int j = 0; j < kA; ++j) z[j] = sm[kSB3 + j];
+#pragma unroll 8
                 for (int h = 0; h < kH; ++h) {
-                    const float x = H2[tid * kHS + h];
+                    const float x = H2T[h * kTS + tid];
 #pragma unroll
                     for (int j = 0; j < kA; ++j) z[j] = fmaf(sm[kSW3 + j * kH + h], x, z[j]);
                 }
@@ -284,68 +284,104 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
                 hsum += H;
             }
 #pragma unroll
-            for (int j = 0; j < kA; ++j) DZ[tid * 8 + j] = dz[j];
+            for (int j = 0; j < kA; ++j) DZT[j * kTS + tid] = dz[j];
         }
         __syncthreads();
-        // D2 = (dz W3) * [h2 > 0]
+        // D2 = (dz W3) * [h2 > 0]: samples 8 sg .., units ng + 16 q
+        {
+            float dzv[kA][8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int s = 8 * sg + i;
+            for (int c = 0; c < kA; ++c) {
+                const float4 d0 = *reinterpret_cast<const float4*>(DZT + c * kTS + 8 * sg);
+                const float4 d1 = *reinterpret_cast<const float4*>(DZT + c * kTS + 8 * sg + 4);
+                dzv[c][0] = d0.x; dzv[c][1] = d0.y; dzv[c][2] = d0.z; dzv[c][3] = d0.w;
+                dzv[c][4] = d1.x; dzv[c][5] = d1.y; dzv[c][6] = d1.z; dzv[c][7] = d1.w;
+            }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                const int j = 4 * ng + q;
-                float v = 0.f;
+                const int j = ng + 16 * q;
+                float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-                for (int c = 0; c < kA; ++c) v = fmaf(DZ[s * 8 + c], sm[kSW3 + c * kH + j], v);
-                D2[s * kHS + j] = H2[s * kHS + j] > 0.f ? v : 0.f;
+                for (int c = 0; c < kA; ++c) {
+                    const float w = sm[kSW3 + c * kH + j];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) v[i] = fmaf(dzv[c][i], w, v[i]);
+                }
+                const float4 h0 = *reinterpret_cast<const float4*>(H2T + j * kTS + 8 * sg);
+                const float4 h1 = *reinterpret_cast<const float4*>(H2T + j * kTS + 8 * sg + 4);
+                float* o = D2T + j * kTS + 8 * sg;
+                *reinterpret_cast<float4*>(o) = make_float4(h0.x > 0.f ? v[0] : 0.f, h0.y > 0.f ? v[1] : 0.f,
+                                                            h0.z > 0.f ? v[2] : 0.f, h0.w > 0.f ? v[3] : 0.f);
+                *reinterpret_cast<float4*>(o + 4) = make_float4(h1.x > 0.f ? v[4] : 0.f, h1.y > 0.f ? v[5] : 0.f,
+                                                                h1.z > 0.f ? v[6] : 0.f, h1.w > 0.f ? v[7] : 0.f);
             }
         }
         __syncthreads();
-        // D1 = (D2 W2) * [h1 > 0]
+        // D1 = (D2 W2) * [h1 > 0]: samples 8 sg .., units ng + 16 q
         {
-            float acc[8][4] = {};
+            float acc[4][8] = {};
 #pragma unroll 4
             for (int j = 0; j < kH; ++j) {
-                const float4 w = *reinterpret_cast<const float4*>(sm + kSW2 + j * kH + 4 * ng);
+                const float4 d0 = *reinterpret_cast<const float4*>(D2T + j * kTS + 8 * sg);
+                const float4 d1 = *reinterpret_cast<const float4*>(D2T + j * kTS + 8 * sg + 4);
+                const float d[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const float d = D2[(8 * sg + i) * kHS + j];
-                    acc[i][0] = fmaf(w.x, d, acc[i][0]);
-                    acc[i][1] = fmaf(w.y, d, acc[i][1]);
-                    acc[i][2] = fmaf(w.z, d, acc[i][2]);
-                    acc[i][3] = fmaf(w.w, d, acc[i][3]);
+                for (int q = 0; q < 4; ++q) {
+                    const float w = sm[kSW2 + j * kH + ng + 16 * q];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) acc[q][i] = fmaf(w, d[i], acc[q][i]);
                 }
             }
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int s = 8 * sg + i, k = 4 * ng + q;
-                    D1[s * kHS + k] = H1[s * kHS + k] > 0.f ? acc[i][q] : 0.f;
-                }
+            for (int q = 0; q < 4; ++q) {
+                const int k = ng + 16 * q;
+                const float4 h0 = *reinterpret_cast<const float4*>(H1T + k * kTS + 8 * sg);
+                const float4 h1 = *reinterpret_cast<const float4*>(H1T + k * kTS + 8 * sg + 4);
+                float* o = D1T + k * kTS + 8 * sg;
+                *reinterpret_cast<float4*>(o) =
+                    make_float4(h0.x > 0.f ? acc[q][0] : 0.f, h0.y > 0.f ? acc[q][1] : 0.f,
+                                h0.z > 0.f ? acc[q][2] : 0.f, h0.w > 0.f ? acc[q][3] : 0.f);
+                *reinterpret_cast<float4*>(o + 4) =
+                    make_float4(h1.x > 0.f ? acc[q][4] : 0.f, h1.y > 0.f ? acc[q][5] : 0.f,
+                                h1.z > 0.f ? acc[q][6] : 0.f, h1.w > 0.f ? acc[q][7] : 0.f);
+            }
         }
         __syncthreads();
-        // weight gradients of the tile
-        for (int s = 0; s < kTile; ++s) {
-            float d[4], h[4];
+        // the tile's weight gradients, 4 samples per 16-byte load
+#pragma unroll 2
+        for (int s = 0; s < kTile; s += 4) {
+            float4 d[4], h[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                d[q] = D2[s * kHS + 4 * jb + q];
-                h[q] = H1[s * kHS + 4 * kb + q];
+            for (int p = 0; p < 4; ++p) {
+                d[p] = *reinterpret_cast<const float4*>(D2T + (sg + 16 * p) * kTS + s);
+                h[p] = *reinterpret_cast<const float4*>(H1T + (ng + 16 * p) * kTS + s);
             }
 #pragma unroll
             for (int p = 0; p < 4; ++p)
 #pragma unroll
-                for (int q = 0; q < 4; ++q) gW2[p][q] = fmaf(d[p], h[q], gW2[p][q]);
+                for (int q = 0; q < 4; ++q) {
+                    float g = gW2[p][q];
+                    g = fmaf(d[p].x, h[q].x, g);
+                    g = fmaf(d[p].y, h[q].y, g);
+                    g = fmaf(d[p].z, h[q].z, g);
+                    g = fmaf(d[p].w, h[q].w, g);
+                    gW2[p][q] = g;
+                }
         }
+        for (int s = 0; s < kTile; s += 4) {
+            const float4 d = *reinterpret_cast<const float4*>(D1T + w1j * kTS + s);
 #pragma unroll
-        for (int q = 0; q < (int)(sizeof(gW1) / sizeof(float)); ++q) {
-            const int e = tid + kThreads * q;
-            if (e < nW1) {
-                const int j = e / in, k = e - j * in;
-                float g = gW1[q];
-                for (int s = 0; s < kTile; ++s) g = fmaf(D1[s * kHS + j], X[s * kXS + k], g);
-                gW1[q] = g;
+            for (int q = 0; q < kLearnMaxIn / 4; ++q) {
+                const int k = w1k + 4 * q;
+                if (k < in) {
+                    const float4 x = *reinterpret_cast<const float4*>(XT + k * kTS + s);
+                    float g = gW1[q];
+                    g = fmaf(d.x, x.x, g);
+                    g = fmaf(d.y, x.y, g);
+                    g = fmaf(d.z, x.z, g);
+                    g = fmaf(d.w, x.w, g);
+                    gW1[q] = g;
+                }
             }
         }
 #pragma unroll
@@ -354,18 +390,28 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
             if (e < kA * kH) {
                 const int c = e / kH, j = e - c * kH;
                 float g = gW3[q];
-                for (int s = 0; s < kTile; ++s) g = fmaf(DZ[s * 8 + c], H2[s * kHS + j], g);
+                for (int s = 0; s < kTile; s += 4) {
+                    const float4 d = *reinterpret_cast<const float4*>(DZT + c * kTS + s);
+                    const float4 x = *reinterpret_cast<const float4*>(H2T + j * kTS + s);
+                    g = fmaf(d.x, x.x, g);
+                    g = fmaf(d.y, x.y, g);
+                    g = fmaf(d.z, x.z, g);
+                    g = fmaf(d.w, x.w, g);
+                }
                 gW3[q] = g;
             }
         }
         if (tid < 2 * kH + kA) {
+            const float* row = tid < kH ? D1T + tid * kTS : tid < 2 * kH ? D2T + (tid - kH) * kTS
+                                                                         : DZT + (tid - 2 * kH) * kTS;
             float g = gB;
-            if (tid < kH)
-                for (int s = 0; s < kTile; ++s) g += D1[s * kHS + tid];
-            else if (tid < 2 * kH)
-                for (int s = 0; s < kTile; ++s) g += D2[s * kHS + tid - kH];
-            else
-                for (int s = 0; s < kTile; ++s) g += DZ[s * 8 + tid - 2 * kH];
+            for (int s = 0; s < kTile; s += 4) {
+                const float4 d = *reinterpret_cast<const float4*>(row + s);
+                g += d.x;
+                g += d.y;
+                g += d.z;
+                g += d.w;
+            }
             gB = g;
         }
         __syncthreads();                        // the tile's buffers are rewritten next
@@ -376,15 +422,15 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
     const int P = kH * in + kH + kH * kH + kH + kA * kH + kA;
     float* out = a.gpart + (int64_t)blockIdx.x * (P + 2);
 #pragma unroll
-    for (int q = 0; q < (int)(sizeof(gW1) / sizeof(float)); ++q) {
-        const int e = tid + kThreads * q;
-        if (e < nW1) out[e] = gW1[q];                             // j * in + k
+    for (int q = 0; q < kLearnMaxIn / 4; ++q) {
+        const int k = w1k + 4 * q;
+        if (k < in) out[w1j * in + k] = gW1[q];
     }
     const int oW2 = kH * in + kH;
 #pragma unroll
     for (int p = 0; p < 4; ++p)
 #pragma unroll
-        for (int q = 0; q < 4; ++q) out[oW2 + (4 * jb + p) * kH + 4 * kb + q] = gW2[p][q];
+        for (int q = 0; q < 4; ++q) out[oW2 + (sg + 16 * p) * kH + ng + 16 * q] = gW2[p][q];
     const int oW3 = oW2 + kH * kH + kH;
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
