@@ -123,10 +123,14 @@ __global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
     if (threadIdx.x == 0) a.gsum[blockIdx.x] = red[0];
 }
 
+// One warp: lane l sums blocks l, l + 32, ... in order, then a fixed xor tree.
 __global__ void learn_baseline_kernel(LearnArgs a, int n_blocks) {
-    if (threadIdx.x != 0) return;
+    const int lane = threadIdx.x & 31;
     double s = 0.0;
-    for (int b = 0; b < n_blocks; ++b) s += a.gsum[b];
+    for (int b = lane; b < n_blocks; b += 32) s += a.gsum[b];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (threadIdx.x != 0) return;
     const int epp = (int)(a.n_envs / a.n_pairs);
     const double M = (double)(*a.n_slots) * (double)a.n_episodes * (double)a.T * (double)epp;
     a.stats[0] = M;
@@ -462,8 +466,14 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
 __global__ void learn_reduce_kernel(LearnArgs a, int P) {
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
     if (j >= P + 2) return;
-    double s = 0.0;
-    for (int b = 0; b < a.grid; ++b) s += (double)a.gpart[(int64_t)b * (P + 2) + j];
+    // eight interleaved partial sums (independent loads), combined in a fixed order
+    double p8[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
+    int b = 0;
+    for (; b + 8 <= a.grid; b += 8)
+#pragma unroll
+        for (int u = 0; u < 8; ++u) p8[u] += (double)a.gpart[(int64_t)(b + u) * (P + 2) + j];
+    for (; b < a.grid; ++b) p8[0] += (double)a.gpart[(int64_t)b * (P + 2) + j];
+    const double s = ((p8[0] + p8[1]) + (p8[2] + p8[3])) + ((p8[4] + p8[5]) + (p8[6] + p8[7]));
     if (j < P) a.grad[j] = (float)s;
     else if (j == P) a.stats[2] = a.stats[0] > 0 ? s / a.stats[0] : 0.0;   // loss: (1/M) sum of -(A log pi + beta H)
     else a.stats[3] = a.stats[0] > 0 ? s / a.stats[0] : 0.0;              // mean entropy

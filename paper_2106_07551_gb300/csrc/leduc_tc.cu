@@ -104,13 +104,14 @@ struct Phase {
 
 // The unit and phase loop, run by every role in its own copy (each copy
 // compiled within its warpgroup's register budget); all copies pass the same
-// CTA barriers in the same order. on_phase(ph) does the role's share of a
+// CTA barriers in the same order; wait_stage: the role waits for a new policy
+// image to land before its phase. on_phase(ph) does the role's share of a
 // phase, on_stage() its work after a new policy has landed, on_unit(sums)
 // adds the unit's payoff sums (consumers hold them; the others add zeros).
 template <class OnPhase, class OnStage>
 __device__ __forceinline__ void drive(const EvalArgs& a, const LeducWork& w, E::Bars& bars, Ctl& ctl,
                                       uint8_t* smem, OnPhase&& on_phase, OnStage&& on_stage,
-                                      long long* sums) {
+                                      long long* sums, bool wait_stage = true) {
     const int tid = threadIdx.x;
     const int64_t n_seg = w.n_seg;
     const int64_t n_units = (int64_t)a.n_pairs * n_seg;
@@ -155,7 +156,11 @@ __device__ __forceinline__ void drive(const EvalArgs& a, const LeducWork& w, E::
                 // previous phase ended with a CTA barrier); ctl is written again
                 // only after the next CTA barrier
                 if (tid == 0) E::stage(smem, reinterpret_cast<const uint8_t*>(a.arena + a.pol_offset[pol]), bars);
-                E::wait(bars, &bars.stage, ctl.stagings & 1u, a.err);
+                // the producers and consumers do not wait: the producers' tiles do
+                // not depend on the policy (they build the phase's first tiles while
+                // it lands), and the consumers read the image (b3) only after a
+                // p_full, which the engine announces after it has waited for it
+                if (wait_stage) E::wait(bars, &bars.stage, ctl.stagings & 1u, a.err);
                 on_stage();
             }
             if (n > 0) {
@@ -308,7 +313,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                 asm volatile("bar.sync 2, 128;" ::: "memory");
                 if (r == 0) mbar_arrive_release(&bars.x_full[buf]);
             }
-        }, nothing, sums);
+        }, nothing, sums, /*wait_stage=*/false);
         end_cta(tbase);
     } else {
         // ---- consumers: draw, transition, sums, next queue; one row per thread
@@ -426,7 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                             (uint16_t)slot;
                 }
             }
-        }, nothing, sums);
+        }, nothing, sums, /*wait_stage=*/false);
         end_cta(tbase);
     }
 }
