@@ -56,3 +56,37 @@ def test_quick_start_payoff_table_and_rollout():
     done = traj["done"].cpu().numpy()
     assert np.all(done[:, -1] == 1) and np.all(done[:, :-1] == 0)
     assert np.all(traj["reward"].cpu().numpy() <= 0)
+
+
+def test_quick_start_learner_loop():
+    """rollout -> policy gradient -> Adam -> population update, as a user would
+    write it; the loss statistics are finite and the next rollout runs."""
+    torch = need_gpu()
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2106_07551_gb300 import (MALIB_ENV_SPREAD, MALIB_F32, MALIB_POL_MLP, Context, alloc_traj,
+                                        make_spec, policy_desc)
+    rng = np.random.default_rng(0)
+    dims = (18, 64, 64, 5)
+    params = [_mlp(rng, dims) for _ in range(16)]
+    spec = make_spec(MALIB_ENV_SPREAD, 3, 18, 5, n_landmarks=3, episode_len=25, n_envs=4096)
+    with Context(0) as ctx:
+        ids = ctx.pop_load(spec, [policy_desc(MALIB_POL_MLP, MALIB_F32, -1, dims, p) for p in params])
+        combos = rng.integers(0, 16, (32, 3)).astype(np.int32)
+        combos[0, 0] = 0                                  # policy 0 acts somewhere
+        traj = alloc_traj(spec, 2)
+        ctx.rollout(spec, combos, 2, 7, traj)
+        P = params[0].size
+        grad = torch.zeros(P, device="cuda")
+        stats = torch.zeros(4, dtype=torch.float64, device="cuda")
+        ctx.learn_pg(spec, combos, 2, traj, 0, 0.95, 0.001, grad, stats)
+        w = torch.from_numpy(params[0]).cuda()
+        m, v = torch.zeros_like(w), torch.zeros_like(w)
+        ctx.adam_step(w, grad, m, v, 1, 1e-4)
+        ctx.pop_update(int(ids[0]), w)
+        ctx.rollout(spec, combos, 2, 8, traj)
+        ctx.sync()
+        st = stats.cpu().numpy()
+        assert st[0] == (combos == 0).sum() * 128 * 2 * 25 and np.all(np.isfinite(st))
+        assert torch.isfinite(grad).all() and grad.abs().max() > 0
+        assert np.all(traj["done"][:, -1].cpu().numpy() == 1)
