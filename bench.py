@@ -850,8 +850,9 @@ def run_learner(args):
     """The learner-side update (Sec. 3.3 independent learning, App. C.2): one
     training iteration of every policy of the spread population (N = 3, 4,096
     envs, population 16, MLP 18-64-64-5 fp32) on LEARN_EPISODES episodes of
-    its rollout: per policy, malib_learn_pg on its samples and malib_adam_step.
-    A step covers every sample once (each belongs to one policy)."""
+    its rollout: malib_learn_pg_batch over the whole population (each policy its
+    own independent learner) and one malib_adam_step over all parameters. A step
+    covers every sample once (each belongs to one policy)."""
     import numpy as np
     import torch
 
@@ -886,11 +887,12 @@ def run_learner(args):
     samples = w.n_envs * w.episode_len * w.n_episodes * w.n_agents
     state = {"t": 0}
 
+    ids = np.arange(n_pol, dtype=np.int32)
+
     def step():
         state["t"] += 1
-        for pid in range(n_pol):
-            ctx.learn_pg(spec, d_pairs, w.n_episodes, traj, pid, 0.95, 0.001, grads[pid])
-            ctx.adam_step(params[pid], grads[pid], m[pid], v[pid], state["t"], 1e-4)
+        ctx.learn_pg_batch(spec, d_pairs, w.n_episodes, traj, ids, 0.95, 0.001, grads)
+        ctx.adam_step(params, grads, m, v, state["t"], 1e-4)
 
     for _ in range(args.warmup):
         step()

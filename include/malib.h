@@ -408,12 +408,27 @@ int malib_exploitability(malib_ctx* ctx, const int32_t* ids0, const double* x, i
  * of the context's device, the rollout's spec, n_episodes and episode_len).
  * Built for particle-scenario populations of fp32 MLPs in-64-64-5 with in
  * <= 32 (EUNSUPPORTED otherwise); gamma in [0, 1], entropy_coef >= 0.
- * Deterministic (fixed-order sums, no atomics). A host output makes the call
- * wait for the stream. Errors: EINVAL, ESTATE, EUNSUPPORTED.
+ * Deterministic (fixed-order sums, no atomics). Waits for the stream before
+ * returning. Errors: EINVAL, ESTATE, EUNSUPPORTED.
  */
 int malib_learn_pg(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
                    int64_t n_episodes, const malib_traj* traj, int32_t policy_id, float gamma,
                    float entropy_coef, float* grad_out, double* stats_out);
+
+/*
+ * malib_learn_pg_batch - malib_learn_pg for n_policies distinct policies at
+ * once, each its own independent learner (Sec. 3.3), in one launch sequence:
+ * policy_ids (host) int32 [n_policies], grad_out (host or device) float
+ * [n_policies][P], stats_out (optional, host or device) double
+ * [n_policies][4], each row malib_learn_pg's for that policy up to the
+ * rounding of its sums (a batch shares the policies' tiles among the CTAs
+ * differently; a given batch is deterministic). A repeated id gives EINVAL. Waits for the stream before returning. Errors: EINVAL,
+ * ESTATE, EUNSUPPORTED.
+ */
+int malib_learn_pg_batch(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                         int64_t n_episodes, const malib_traj* traj, const int32_t* policy_ids,
+                         int32_t n_policies, float gamma, float entropy_coef, float* grad_out,
+                         double* stats_out);
 
 /*
  * malib_adam_step - one Adam step (the optimizer of App. C.2's training

@@ -279,6 +279,17 @@ class Context:
                                        n_episodes, C.byref(t), policy_id, gamma, entropy_coef,
                                        _ptr(grad_out), _ptr(stats_out) if stats_out is not None else None))
 
+    def learn_pg_batch(self, spec, pair_ids, n_episodes, traj, policy_ids, gamma, entropy_coef, grad_out,
+                       stats_out=None):
+        """learn_pg for several distinct policies in one call: grad_out
+        [n][P] and stats_out [n][4], host or device."""
+        ids = np.ascontiguousarray(policy_ids, np.int32)
+        t = Traj(_ptr(traj["obs"]), _ptr(traj["action"]), _ptr(traj["reward"]), None, None)
+        _check(self.lib, self.handle,
+               self.lib.malib_learn_pg_batch(self.handle, C.byref(spec), _ptr(pair_ids), int(pair_ids.shape[0]),
+                                             n_episodes, C.byref(t), _ptr(ids), len(ids), gamma, entropy_coef,
+                                             _ptr(grad_out), _ptr(stats_out) if stats_out is not None else None))
+
     def adam_step(self, params, grad, m, v, step, lr, beta1=0.9, beta2=0.999, eps=1e-8):
         """One Adam step on device buffers (parameters, gradient, moments) in place."""
         n = int(params.numel()) if hasattr(params, "numel") else int(params.size)

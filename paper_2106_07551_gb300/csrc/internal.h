@@ -121,16 +121,19 @@ cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s);
 bool spread_tc_supported(int n_agents, int obs_dim, int n_actions, int64_t envs_per_pair);
-// Learner-side policy-gradient step (learner.cu) on a rollout's samples of one
-// policy: fp32 MLPs in-64-64-5 with in <= kLearnMaxIn.
+// Learner-side policy-gradient step (learner.cu) on a rollout's samples of a
+// batch of policies (each its own independent learner): fp32 MLPs in-64-64-5
+// with in <= kLearnMaxIn.
 constexpr int kLearnMaxIn = 32;
 struct LearnArgs {
     const float* arena;          // population arena (F32Layout images)
-    int64_t pol_off;             // float offset of the policy's image
+    const int32_t* pols;         // device [nb] policy ids of the batch (distinct)
+    const int64_t* pol_offs;     // device [nb] float offsets of their images
+    int32_t nb;                  // policies in the batch
     int32_t in;                  // observation width (policy input)
     int32_t xs;                  // observation row stride of the trajectory (in rounded up to 4)
     const int32_t* pairs;        // device [n_pairs][n_agents]
-    int32_t n_pairs, n_agents, n_pol, policy, T;
+    int32_t n_pairs, n_agents, n_pol, T;
     int64_t n_envs, n_episodes;
     const float* obs;            // [E][T][n_envs][n_agents][xs]
     const uint8_t* action;       // [E][T][n_envs][n_agents]
@@ -138,21 +141,23 @@ struct LearnArgs {
     float gamma, beta;
     int* err;
     // work space (learn_work_layout)
-    int32_t* slots;              // [n_pairs * n_agents] (c * n_agents + k) acting with the policy
-    int32_t* n_slots;
-    float* G;                    // [samples] returns-to-go in sample order
-    double* gsum;                // [return blocks] partial sums of G
-    double* stats;               // [4] M, baseline, loss, mean entropy
-    float* gpart;                // [grid][P + 2] per-CTA partial gradients, loss and entropy sums
-    float* grad;                 // [P] the gradient (malib_policy_desc layout)
+    int32_t* slots;              // [nb][n_pairs * n_agents] (c * n_agents + k) acting with each policy
+    int32_t* n_slots;            // [nb]
+    int64_t* samp_off;           // [nb + 1] first sample of each policy in G
+    int64_t* tile_off;           // [nb + 1] first 128-sample tile of each policy
+    float* G;                    // [samples] returns-to-go, policy by policy in sample order
+    double* gsum;                // [nb][return blocks] partial sums of G
+    double* stats;               // [nb][4] M, baseline, loss, mean entropy
+    float* gpart;                // [nb][grid][P + 2] per-CTA partial gradients, loss and entropy sums
+    float* grad;                 // [nb][P] the gradients (malib_policy_desc layout)
     int32_t grid;
 };
 int64_t learn_param_count(int in);
 bool learn_supported(int in, int h1, int h2, int n_actions);
-int64_t learn_work_bytes(int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes, int32_t T,
-                         int in, int grid, int ret_blocks);
-void learn_work_layout(uint8_t* base, int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes,
-                       int32_t T, int in, int grid, int ret_blocks, LearnArgs* a);
+int64_t learn_work_bytes(int32_t nb, int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes,
+                         int32_t T, int in, int grid, int ret_blocks);
+void learn_work_layout(uint8_t* base, int32_t nb, int32_t n_pairs, int32_t n_agents, int64_t n_envs,
+                       int64_t n_episodes, int32_t T, int in, int grid, int ret_blocks, LearnArgs* a);
 cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s);
 cudaError_t launch_learn_adam(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1,
                               float b2, float eps, float c1, float c2, int n_sm, cudaStream_t s);

@@ -64,24 +64,28 @@ constexpr size_t kSBytes = (size_t)kSFloats * 4;
 static_assert(kSBytes <= 232448, "fits the 227 KB of shared memory of a CTA");
 static_assert(kSX % 4 == 0 && kTS % 4 == 0, "16-byte aligned rows");
 
+// One block per policy b of the batch: the slots acting with it, ascending.
 __global__ void __launch_bounds__(1024) learn_slots_kernel(LearnArgs a) {
     __shared__ int warp_n[32];
     __shared__ int base;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int b = blockIdx.x;
     const int total = a.n_pairs * a.n_agents;
+    const int policy = a.pols[b];
+    int32_t* slots = a.slots + (int64_t)b * total;
     if (tid == 0) base = 0;
     __syncthreads();
     for (int c0 = 0; c0 < total; c0 += blockDim.x) {
         const int i = c0 + tid;
         const int pid = i < total ? a.pairs[i] : -1;
-        if (i < total && (pid < 0 || pid >= a.n_pol)) atomicOr(a.err, ERRBIT_BAD_PAIR);
-        const bool mine = i < total && pid == a.policy;
+        if (b == 0 && i < total && (pid < 0 || pid >= a.n_pol)) atomicOr(a.err, ERRBIT_BAD_PAIR);
+        const bool mine = i < total && pid == policy;
         const unsigned m = __ballot_sync(0xffffffffu, mine);
         if (lane == 0) warp_n[warp] = __popc(m);
         __syncthreads();
         int before = base;
         for (int w = 0; w < warp; ++w) before += warp_n[w];
-        if (mine) a.slots[before + __popc(m & ((1u << lane) - 1u))] = i;   // c * n_agents + k
+        if (mine) slots[before + __popc(m & ((1u << lane) - 1u))] = i;   // c * n_agents + k
         __syncthreads();
         if (tid == 0) {
             int n = 0;
@@ -90,13 +94,35 @@ __global__ void __launch_bounds__(1024) learn_slots_kernel(LearnArgs a) {
         }
         __syncthreads();
     }
-    if (tid == 0) *a.n_slots = base;
+    if (tid == 0) a.n_slots[b] = base;
 }
 
+// The batch's sample and tile offsets (prefix sums over the policies; one thread).
+__global__ void learn_plan_kernel(LearnArgs a) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    const int64_t per_slot = a.n_episodes * a.T * (a.n_envs / a.n_pairs);
+    int64_t s = 0, t = 0;
+    for (int b = 0; b < a.nb; ++b) {
+        a.samp_off[b] = s;
+        a.tile_off[b] = t;
+        const int64_t M = (int64_t)a.n_slots[b] * per_slot;
+        s += M;
+        t += (M + 127) / 128;
+    }
+    a.samp_off[a.nb] = s;
+    a.tile_off[a.nb] = t;
+}
+
+// Grid (blocks, nb): G of every sample of policy b by the backward recursion
+// G_t = r_t + gamma G_{t+1}, one thread per (slot, episode, env), and per-block
+// fp64 sums of G.
 __global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
     __shared__ double red[256];
+    const int b = blockIdx.y;
     const int epp = (int)(a.n_envs / a.n_pairs);
-    const int64_t n_seq = (int64_t)(*a.n_slots) * a.n_episodes * epp;
+    const int64_t n_seq = (int64_t)a.n_slots[b] * a.n_episodes * epp;
+    const int32_t* slots = a.slots + (int64_t)b * a.n_pairs * a.n_agents;
+    float* G = a.G + a.samp_off[b];
     double sum = 0.0;
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < n_seq;
          q += (int64_t)gridDim.x * blockDim.x) {
@@ -104,14 +130,14 @@ __global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
         const int64_t rem = q - slot * a.n_episodes * epp;
         const int64_t e = rem / epp;
         const int r = (int)(rem - e * epp);
-        const int ck = a.slots[slot];
+        const int ck = slots[slot];
         const int c = ck / a.n_agents, k = ck - c * a.n_agents;
         const int64_t env = (int64_t)c * epp + r;
-        float G = 0.f;
+        float g = 0.f;
         for (int t = a.T - 1; t >= 0; --t) {
-            G = __fadd_rn(a.reward[((e * a.T + t) * a.n_envs + env) * a.n_agents + k], __fmul_rn(a.gamma, G));
-            a.G[((slot * a.n_episodes + e) * a.T + t) * epp + r] = G;
-            sum += (double)G;
+            g = __fadd_rn(a.reward[((e * a.T + t) * a.n_envs + env) * a.n_agents + k], __fmul_rn(a.gamma, g));
+            G[((slot * a.n_episodes + e) * a.T + t) * epp + r] = g;
+            sum += (double)g;
         }
     }
     red[threadIdx.x] = sum;
@@ -120,32 +146,33 @@ __global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
         if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
         __syncthreads();
     }
-    if (threadIdx.x == 0) a.gsum[blockIdx.x] = red[0];
+    if (threadIdx.x == 0) a.gsum[(int64_t)b * gridDim.x + blockIdx.x] = red[0];
 }
 
-// One warp: lane l sums blocks l, l + 32, ... in order, then a fixed xor tree.
+// One warp per policy b: lane l sums blocks l, l + 32, ... in order, then a
+// fixed xor tree; M and the baseline b = sum G / M.
 __global__ void learn_baseline_kernel(LearnArgs a, int n_blocks) {
     const int lane = threadIdx.x & 31;
+    const int b = blockIdx.x;
     double s = 0.0;
-    for (int b = lane; b < n_blocks; b += 32) s += a.gsum[b];
+    for (int k = lane; k < n_blocks; k += 32) s += a.gsum[(int64_t)b * n_blocks + k];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
     if (threadIdx.x != 0) return;
-    const int epp = (int)(a.n_envs / a.n_pairs);
-    const double M = (double)(*a.n_slots) * (double)a.n_episodes * (double)a.T * (double)epp;
-    a.stats[0] = M;
-    a.stats[1] = M > 0 ? s / M : 0.0;
+    const double M = (double)(a.samp_off[b + 1] - a.samp_off[b]);
+    a.stats[4 * b] = M;
+    a.stats[4 * b + 1] = M > 0 ? s / M : 0.0;
 }
 
 // Sample s of the policy's sample order: (slot, episode, step, env) -> the
 // trajectory index of its (episode, step, env, agent).
-__device__ __forceinline__ int64_t sample_index(const LearnArgs& a, int64_t s, int epp) {
+__device__ __forceinline__ int64_t sample_index(const LearnArgs& a, const int32_t* slots, int64_t s, int epp) {
     const int r = (int)(s % epp);
     const int64_t q = s / epp;                        // (slot, e, t)
     const int t = (int)(q % a.T);
     const int64_t q2 = q / a.T;
     const int64_t e = q2 % a.n_episodes, slot = q2 / a.n_episodes;
-    const int ck = a.slots[slot];
+    const int ck = slots[slot];
     const int c = ck / a.n_agents, ka = ck - c * a.n_agents;
     const int64_t env = (int64_t)c * epp + r;
     return ((e * a.T + t) * a.n_envs + env) * a.n_agents + ka;
@@ -184,29 +211,19 @@ __device__ __forceinline__ void dense_relu(const float* __restrict__ Win, const 
     }
 }
 
+// A CTA's contiguous share [lo, hi) of the batch's tiles (all policies' tiles
+// in policy order).
+__device__ __forceinline__ int64_t share_lo(const LearnArgs& a, int64_t c) {
+    return a.tile_off[a.nb] * c / a.grid;
+}
+
 __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
     extern __shared__ __align__(16) float sm[];
     const int tid = threadIdx.x;
     const int in = a.in;
-    const float* pol = a.arena + a.pol_off;
-    // the policy (F32Layout: W1T [in][64], b1, W2T [64][64], b2, W3 [5][64], b3)
-    for (int i = tid; i < in * kH; i += kThreads) sm[kSW1T + i] = pol[i];
-    for (int i = tid; i < kH; i += kThreads) sm[kSB1 + i] = pol[in * kH + i];
-    for (int i = tid; i < kH * kH; i += kThreads) {
-        const float w = pol[in * kH + kH + i];               // W2T[k][j], i = k * 64 + j
-        sm[kSW2T + i] = w;
-        sm[kSW2 + (i & (kH - 1)) * kH + (i >> 6)] = w;        // W2[j][k]
-    }
-    for (int i = tid; i < kH; i += kThreads) sm[kSB2 + i] = pol[in * kH + kH + kH * kH + i];
-    for (int i = tid; i < kA * kH; i += kThreads) sm[kSW3 + i] = pol[in * kH + 2 * kH + kH * kH + i];
-    if (tid < kA) sm[kSB3 + tid] = pol[in * kH + 2 * kH + kH * kH + kA * kH + tid];
-    __syncthreads();
-
     const int epp = (int)(a.n_envs / a.n_pairs);
-    const int64_t M = (int64_t)(*a.n_slots) * a.n_episodes * a.T * epp;
-    const float invM = M > 0 ? (float)(1.0 / (double)M) : 0.f;
-    const float base = (float)a.stats[1];
-    const int64_t n_tiles = (M + kTile - 1) / kTile;
+    const int P = kH * in + kH + kH * kH + kH + kA * kH + kA;
+    const int64_t lo = share_lo(a, blockIdx.x), hi = share_lo(a, blockIdx.x + 1);
 
     float* XT = sm + kSX;
     float* H1T = sm + kSH1;
@@ -222,8 +239,90 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
     float gW3[2] = {};                                 // dW3 entries tid, tid + 256 of [5][64]
     float gB = 0.f;                                    // b1 (tid < 64), b2 (64..127), b3 (128..132)
     float lsum = 0.f, hsum = 0.f;                      // loss and entropy of this thread's samples
-    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-        const int64_t s0 = tile * kTile;
+    int b = -1;                                        // the batch's policy of the current tiles
+    int64_t M = 0, t0 = 0;
+    float invM = 0.f, base = 0.f;
+    const int32_t* slots = nullptr;
+    const float* Gb = nullptr;
+    // this CTA's partial gradient of policy b, in the malib_policy_desc layout:
+    // W1 [64][in], b1, W2 [64][64], b2, W3 [5][64], b3, then loss and entropy sums
+    auto flush = [&]() {
+        float* out = a.gpart + ((int64_t)b * a.grid + blockIdx.x) * (P + 2);
+#pragma unroll
+        for (int q = 0; q < kLearnMaxIn / 4; ++q) {
+            const int k = w1k + 4 * q;
+            if (k < in) out[w1j * in + k] = gW1[q];
+        }
+        const int oW2 = kH * in + kH;
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) out[oW2 + (sg + 16 * p) * kH + ng + 16 * q] = gW2[p][q];
+        const int oW3 = oW2 + kH * kH + kH;
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int e = tid + kThreads * q;
+            if (e < kA * kH) out[oW3 + e] = gW3[q];
+        }
+        if (tid < kH) out[kH * in + tid] = gB;                          // b1
+        else if (tid < 2 * kH) out[oW2 + kH * kH + tid - kH] = gB;      // b2
+        else if (tid < 2 * kH + kA) out[oW3 + kA * kH + tid - 2 * kH] = gB;   // b3
+        // loss and entropy sums (fixed-order tree in shared memory; the tiles'
+        // buffers are free between tiles)
+        float* red = sm + kSX;
+        red[tid] = lsum;
+        red[kThreads + tid] = hsum;
+        __syncthreads();
+        for (int w = kThreads / 2; w > 0; w >>= 1) {
+            if (tid < w) {
+                red[tid] += red[tid + w];
+                red[kThreads + tid] += red[kThreads + tid + w];
+            }
+            __syncthreads();
+        }
+        if (tid == 0) {
+            out[P] = red[0];
+            out[P + 1] = red[kThreads];
+        }
+        __syncthreads();
+    };
+    for (int64_t tile = lo; tile < hi; ++tile) {
+        if (b < 0 || tile >= a.tile_off[b + 1]) {
+            // the next policy of the batch with tiles: flush the previous one's
+            // partials, stage this one (F32Layout: W1T [in][64], b1, W2T [64][64],
+            // b2, W3 [5][64], b3), restart the sums
+            if (b >= 0) flush();
+            if (b < 0) b = 0;
+            while (tile >= a.tile_off[b + 1]) ++b;
+            const float* pol = a.arena + a.pol_offs[b];
+            for (int i = tid; i < in * kH; i += kThreads) sm[kSW1T + i] = pol[i];
+            for (int i = tid; i < kH; i += kThreads) sm[kSB1 + i] = pol[in * kH + i];
+            for (int i = tid; i < kH * kH; i += kThreads) {
+                const float w = pol[in * kH + kH + i];               // W2T[k][j], i = k * 64 + j
+                sm[kSW2T + i] = w;
+                sm[kSW2 + (i & (kH - 1)) * kH + (i >> 6)] = w;        // W2[j][k]
+            }
+            for (int i = tid; i < kH; i += kThreads) sm[kSB2 + i] = pol[in * kH + kH + kH * kH + i];
+            for (int i = tid; i < kA * kH; i += kThreads) sm[kSW3 + i] = pol[in * kH + 2 * kH + kH * kH + i];
+            if (tid < kA) sm[kSB3 + tid] = pol[in * kH + 2 * kH + kH * kH + kA * kH + tid];
+            M = a.samp_off[b + 1] - a.samp_off[b];
+            invM = M > 0 ? (float)(1.0 / (double)M) : 0.f;
+            base = (float)a.stats[4 * b + 1];
+            slots = a.slots + (int64_t)b * a.n_pairs * a.n_agents;
+            Gb = a.G + a.samp_off[b];
+            t0 = a.tile_off[b];
+#pragma unroll
+            for (int p = 0; p < 4; ++p)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) gW2[p][q] = 0.f;
+#pragma unroll
+            for (int q = 0; q < kLearnMaxIn / 4; ++q) gW1[q] = 0.f;
+            gW3[0] = gW3[1] = 0.f;
+            gB = 0.f;
+            lsum = hsum = 0.f;
+            __syncthreads();
+        }
+        const int64_t s0 = (tile - t0) * kTile;
         // the tile's observations (feature-major; zero columns past M), and for
         // the logits phase each sample's action and return
         int act = 0;
@@ -232,12 +331,12 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
             const int r = tid & (kTile - 1), half = tid >> 7;
             const int64_t s = s0 + r;
             if (s < M) {
-                const int64_t ix = sample_index(a, s, epp);
+                const int64_t ix = sample_index(a, slots, s, epp);
                 const float* orow = a.obs + ix * a.xs;
                 for (int k = half; k < in; k += 2) XT[k * kTS + r] = orow[k];
                 if (half == 0) {
                     act = a.action[ix];
-                    ret = a.G[s];
+                    ret = Gb[s];
                 }
             } else {
                 for (int k = half; k < in; k += 2) XT[k * kTS + r] = 0.f;
@@ -421,62 +520,37 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
         __syncthreads();                        // the tile's buffers are rewritten next
     }
 
-    // this CTA's partial gradient, in the malib_policy_desc layout:
-    // W1 [64][in], b1, W2 [64][64], b2, W3 [5][64], b3, then loss and entropy sums
-    const int P = kH * in + kH + kH * kH + kH + kA * kH + kA;
-    float* out = a.gpart + (int64_t)blockIdx.x * (P + 2);
-#pragma unroll
-    for (int q = 0; q < kLearnMaxIn / 4; ++q) {
-        const int k = w1k + 4 * q;
-        if (k < in) out[w1j * in + k] = gW1[q];
-    }
-    const int oW2 = kH * in + kH;
-#pragma unroll
-    for (int p = 0; p < 4; ++p)
-#pragma unroll
-        for (int q = 0; q < 4; ++q) out[oW2 + (sg + 16 * p) * kH + ng + 16 * q] = gW2[p][q];
-    const int oW3 = oW2 + kH * kH + kH;
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-        const int e = tid + kThreads * q;
-        if (e < kA * kH) out[oW3 + e] = gW3[q];
-    }
-    if (tid < kH) out[kH * in + tid] = gB;                          // b1
-    else if (tid < 2 * kH) out[oW2 + kH * kH + tid - kH] = gB;      // b2
-    else if (tid < 2 * kH + kA) out[oW3 + kA * kH + tid - 2 * kH] = gB;   // b3
-    // loss and entropy sums of the CTA (fixed-order tree in shared memory)
-    __syncthreads();
-    float* red = sm + kSX;
-    red[tid] = lsum;
-    red[kThreads + tid] = hsum;
-    __syncthreads();
-    for (int w = kThreads / 2; w > 0; w >>= 1) {
-        if (tid < w) {
-            red[tid] += red[tid + w];
-            red[kThreads + tid] += red[kThreads + tid + w];
-        }
-        __syncthreads();
-    }
-    if (tid == 0) {
-        out[P] = red[0];
-        out[P + 1] = red[kThreads];
-    }
+    if (b >= 0) flush();
 }
 
+// Grid (blocks, nb): policy b's gradient as the sum, in CTA order, of the
+// partials of the CTAs whose tile share meets b's tiles (eight interleaved
+// partial sums, combined in a fixed order); its loss and mean entropy.
 __global__ void learn_reduce_kernel(LearnArgs a, int P) {
     const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    const int b = blockIdx.y;
     if (j >= P + 2) return;
-    // eight interleaved partial sums (independent loads), combined in a fixed order
+    const int64_t t_lo = a.tile_off[b], t_hi = a.tile_off[b + 1];
+    int c_lo = 0, c_hi = 0;                  // CTAs [c_lo, c_hi) hold partials of b
+    if (t_hi > t_lo) {
+        while (share_lo(a, c_lo + 1) <= t_lo) ++c_lo;
+        c_hi = c_lo + 1;
+        while (c_hi < a.grid && share_lo(a, c_hi) < t_hi) ++c_hi;
+    }
+    // (a CTA with an empty share wrote no partial: it is skipped)
+    const float* part = a.gpart + (int64_t)b * a.grid * (P + 2) + j;
     double p8[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
-    int b = 0;
-    for (; b + 8 <= a.grid; b += 8)
-#pragma unroll
-        for (int u = 0; u < 8; ++u) p8[u] += (double)a.gpart[(int64_t)(b + u) * (P + 2) + j];
-    for (; b < a.grid; ++b) p8[0] += (double)a.gpart[(int64_t)b * (P + 2) + j];
+    int u = 0;
+    for (int c = c_lo; c < c_hi; ++c)
+        if (share_lo(a, c + 1) > share_lo(a, c)) {
+            p8[u] += (double)part[(int64_t)c * (P + 2)];
+            u = (u + 1) & 7;
+        }
     const double s = ((p8[0] + p8[1]) + (p8[2] + p8[3])) + ((p8[4] + p8[5]) + (p8[6] + p8[7]));
-    if (j < P) a.grad[j] = (float)s;
-    else if (j == P) a.stats[2] = a.stats[0] > 0 ? s / a.stats[0] : 0.0;   // loss: (1/M) sum of -(A log pi + beta H)
-    else a.stats[3] = a.stats[0] > 0 ? s / a.stats[0] : 0.0;              // mean entropy
+    double* st = a.stats + 4 * b;
+    if (j < P) a.grad[(int64_t)b * P + j] = (float)s;
+    else if (j == P) st[2] = st[0] > 0 ? s / st[0] : 0.0;   // loss: (1/M) sum of -(A log pi + beta H)
+    else st[3] = st[0] > 0 ? s / st[0] : 0.0;              // mean entropy
 }
 
 __global__ void learn_adam_kernel(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1,
@@ -499,18 +573,21 @@ bool learn_supported(int in, int h1, int h2, int n_actions) {
     return in >= 1 && in <= kLearnMaxIn && h1 == kH && h2 == kH && n_actions == kA;
 }
 
-// Upper bounds of the work space (bytes, each region on a 256-byte boundary).
-int64_t learn_work_bytes(int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes, int32_t T,
-                         int in, int grid, int ret_blocks) {
+// Upper bounds of the work space (bytes, each region on a 256-byte boundary):
+// the distinct policies of a batch own disjoint slots, so their samples together
+// are at most every (episode, step, env, agent).
+int64_t learn_work_bytes(int32_t nb, int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes,
+                         int32_t T, int in, int grid, int ret_blocks) {
     auto up = [](int64_t b) { return (b + 255) / 256 * 256; };
     const int64_t slots = (int64_t)n_pairs * n_agents;
     const int64_t samples = slots * n_episodes * T * (n_envs / n_pairs);
-    return up(slots * 4) + up(4) + up(samples * 4) + up((int64_t)ret_blocks * 8) + up(4 * 8) +
-           up((int64_t)grid * (learn_param_count(in) + 2) * 4);
+    return up((int64_t)nb * 4) + up((int64_t)nb * 8) + up((int64_t)nb * slots * 4) + up((int64_t)nb * 4) +
+           2 * up((int64_t)(nb + 1) * 8) + up(samples * 4) + up((int64_t)nb * ret_blocks * 8) +
+           up((int64_t)nb * 4 * 8) + up((int64_t)nb * grid * (learn_param_count(in) + 2) * 4);
 }
 
-void learn_work_layout(uint8_t* base, int32_t n_pairs, int32_t n_agents, int64_t n_envs, int64_t n_episodes,
-                       int32_t T, int in, int grid, int ret_blocks, LearnArgs* a) {
+void learn_work_layout(uint8_t* base, int32_t nb, int32_t n_pairs, int32_t n_agents, int64_t n_envs,
+                       int64_t n_episodes, int32_t T, int in, int grid, int ret_blocks, LearnArgs* a) {
     int64_t off = 0;
     auto take = [&](int64_t bytes) {
         uint8_t* p = base + off;
@@ -519,25 +596,32 @@ void learn_work_layout(uint8_t* base, int32_t n_pairs, int32_t n_agents, int64_t
     };
     const int64_t slots = (int64_t)n_pairs * n_agents;
     const int64_t samples = slots * n_episodes * T * (n_envs / n_pairs);
-    a->slots = reinterpret_cast<int32_t*>(take(slots * 4));
-    a->n_slots = reinterpret_cast<int32_t*>(take(4));
+    a->pols = reinterpret_cast<int32_t*>(take((int64_t)nb * 4));
+    a->pol_offs = reinterpret_cast<int64_t*>(take((int64_t)nb * 8));
+    a->slots = reinterpret_cast<int32_t*>(take((int64_t)nb * slots * 4));
+    a->n_slots = reinterpret_cast<int32_t*>(take((int64_t)nb * 4));
+    a->samp_off = reinterpret_cast<int64_t*>(take((int64_t)(nb + 1) * 8));
+    a->tile_off = reinterpret_cast<int64_t*>(take((int64_t)(nb + 1) * 8));
     a->G = reinterpret_cast<float*>(take(samples * 4));
-    a->gsum = reinterpret_cast<double*>(take((int64_t)ret_blocks * 8));
-    a->stats = reinterpret_cast<double*>(take(4 * 8));
-    a->gpart = reinterpret_cast<float*>(take((int64_t)grid * (learn_param_count(in) + 2) * 4));
+    a->gsum = reinterpret_cast<double*>(take((int64_t)nb * ret_blocks * 8));
+    a->stats = reinterpret_cast<double*>(take((int64_t)nb * 4 * 8));
+    a->gpart = reinterpret_cast<float*>(take((int64_t)nb * grid * (learn_param_count(in) + 2) * 4));
+    a->nb = nb;
     a->grid = grid;
 }
 
 cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s) {
-    learn_slots_kernel<<<1, 1024, 0, s>>>(a);
-    learn_returns_kernel<<<ret_blocks, 256, 0, s>>>(a);
-    learn_baseline_kernel<<<1, 32, 0, s>>>(a, ret_blocks);
+    if (a.nb <= 0) return cudaSuccess;
+    learn_slots_kernel<<<a.nb, 1024, 0, s>>>(a);
+    learn_plan_kernel<<<1, 32, 0, s>>>(a);
+    learn_returns_kernel<<<dim3(ret_blocks, a.nb), 256, 0, s>>>(a);
+    learn_baseline_kernel<<<a.nb, 32, 0, s>>>(a, ret_blocks);
     cudaError_t err = cudaFuncSetAttribute(learn_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)kSBytes);
     if (err != cudaSuccess) return err;
     learn_grad_kernel<<<a.grid, kThreads, kSBytes, s>>>(a);
     const int P = (int)learn_param_count(a.in);
-    learn_reduce_kernel<<<(P + 2 + 255) / 256, 256, 0, s>>>(a, P);
+    learn_reduce_kernel<<<dim3((P + 2 + 255) / 256, a.nb), 256, 0, s>>>(a, P);
     return cudaGetLastError();
 }
 

@@ -768,11 +768,12 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
     return MALIB_OK;
 }
 
-int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
-                   int64_t n_episodes, const malib_traj* traj, int32_t policy_id, float gamma,
-                   float entropy_coef, float* grad_out, double* stats_out) {
-    if (!c) return MALIB_EINVAL;
-    DeviceGuard g(c->device);
+namespace {
+
+// The policy-gradient step of nb distinct policies (host ids) in one batch.
+int learn_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                int64_t n_episodes, const malib_traj* traj, const int32_t* ids, int32_t nb, float gamma,
+                float entropy_coef, float* grad_out, double* stats_out) {
     int r;
     if ((r = check_spec(c, spec)) != MALIB_OK) return r;
     if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
@@ -784,8 +785,16 @@ int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair
         !learn_supported(c->dims[0], c->dims[1], c->dims[2], c->dims[3]))
         return fail(c, MALIB_EUNSUPPORTED, "the learner step is built for fp32 MLPs in-64-64-5 (in <= %d)",
                     kLearnMaxIn);
-    if (policy_id < 0 || policy_id >= (int32_t)c->pols.size())
-        return fail(c, MALIB_EINVAL, "policy_id %d is not in the population", policy_id);
+    if (nb < 1 || !ids) return fail(c, MALIB_EINVAL, "the batch needs at least one policy id");
+    std::vector<int32_t> hid(ids, ids + nb);
+    std::vector<int64_t> hoff(nb);
+    for (int32_t b = 0; b < nb; ++b) {
+        if (hid[b] < 0 || hid[b] >= (int32_t)c->pols.size())
+            return fail(c, MALIB_EINVAL, "policy id %d is not in the population", hid[b]);
+        for (int32_t q = 0; q < b; ++q)
+            if (hid[q] == hid[b]) return fail(c, MALIB_EINVAL, "policy id %d appears twice in the batch", hid[b]);
+        hoff[b] = c->pols[hid[b]].offset;
+    }
     if (n_pairs < 1) return fail(c, MALIB_EINVAL, "n_pairs must be >= 1");
     if (spec->n_envs < 1 || spec->n_envs % n_pairs != 0)
         return fail(c, MALIB_EINVAL, "n_envs (%lld) must be a positive multiple of n_pairs (%d)",
@@ -812,27 +821,30 @@ int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair
     const int64_t P = learn_param_count(in);
     const int grid = c->n_sm;
     const int ret_blocks = 2 * c->n_sm;
-    const int64_t bytes = learn_work_bytes(n_pairs, spec->n_agents, spec->n_envs, n_episodes,
+    const int64_t bytes = learn_work_bytes(nb, n_pairs, spec->n_agents, spec->n_envs, n_episodes,
                                            spec->episode_len, in, grid, ret_blocks);
     if ((r = ensure(c, c->learn_work, c->learn_work_cap, bytes, "learner work space")) != MALIB_OK) return r;
     LearnArgs a{};
-    learn_work_layout(c->learn_work, n_pairs, spec->n_agents, spec->n_envs, n_episodes, spec->episode_len, in,
+    learn_work_layout(c->learn_work, nb, n_pairs, spec->n_agents, spec->n_envs, n_episodes, spec->episode_len, in,
                       grid, ret_blocks, &a);
     if (gw == kPtrHere) {
         a.grad = grad_out;
     } else {
-        if ((r = ensure(c, c->learn_grad, c->learn_grad_cap, P, "gradient staging")) != MALIB_OK) return r;
+        if ((r = ensure(c, c->learn_grad, c->learn_grad_cap, (int64_t)nb * P, "gradient staging")) != MALIB_OK)
+            return r;
         a.grad = c->learn_grad;
     }
+    CK(cudaMemcpyAsync(const_cast<int32_t*>(a.pols), hid.data(), (size_t)nb * 4, cudaMemcpyHostToDevice,
+                       c->stream), "policy ids");
+    CK(cudaMemcpyAsync(const_cast<int64_t*>(a.pol_offs), hoff.data(), (size_t)nb * 8, cudaMemcpyHostToDevice,
+                       c->stream), "policy offsets");
     a.arena = c->arena;
-    a.pol_off = c->pols[policy_id].offset;
     a.in = in;
     a.xs = (spec->obs_dim + 3) / 4 * 4;
     a.pairs = dpairs;
     a.n_pairs = n_pairs;
     a.n_agents = spec->n_agents;
     a.n_pol = (int32_t)c->pols.size();
-    a.policy = policy_id;
     a.T = spec->episode_len;
     a.n_envs = spec->n_envs;
     a.n_episodes = n_episodes;
@@ -843,18 +855,37 @@ int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair
     a.beta = entropy_coef;
     a.err = c->d_err;
     CK(launch_learn_pg(a, ret_blocks, c->stream), "policy-gradient kernels");
-    c->launches += 5;
+    c->launches += 6;
     if (gw != kPtrHere)
-        CK(cudaMemcpyAsync(grad_out, a.grad, P * 4, cudaMemcpyDeviceToHost, c->stream), "gradient copy");
+        CK(cudaMemcpyAsync(grad_out, a.grad, (size_t)nb * P * 4, cudaMemcpyDeviceToHost, c->stream),
+           "gradient copy");
     if (stats_out)
-        CK(cudaMemcpyAsync(stats_out, a.stats, 4 * 8, sw == kPtrHere ? cudaMemcpyDeviceToDevice
-                                                                     : cudaMemcpyDeviceToHost, c->stream),
+        CK(cudaMemcpyAsync(stats_out, a.stats, (size_t)nb * 4 * 8,
+                           sw == kPtrHere ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, c->stream),
            "statistics copy");
-    if (gw != kPtrHere || (stats_out && sw != kPtrHere)) {
-        CK(cudaStreamSynchronize(c->stream), "learner step");
-        if ((r = read_device_errors(c)) != MALIB_OK) return r;
-    }
-    return MALIB_OK;
+    // the host vectors of ids and offsets are copied before they go out of scope
+    CK(cudaStreamSynchronize(c->stream), "learner step");
+    return read_device_errors(c);
+}
+
+}  // namespace
+
+int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                   int64_t n_episodes, const malib_traj* traj, int32_t policy_id, float gamma,
+                   float entropy_coef, float* grad_out, double* stats_out) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    return learn_batch(c, spec, pair_ids, n_pairs, n_episodes, traj, &policy_id, 1, gamma, entropy_coef, grad_out,
+                       stats_out);
+}
+
+int malib_learn_pg_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                         int64_t n_episodes, const malib_traj* traj, const int32_t* policy_ids,
+                         int32_t n_policies, float gamma, float entropy_coef, float* grad_out, double* stats_out) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    return learn_batch(c, spec, pair_ids, n_pairs, n_episodes, traj, policy_ids, n_policies, gamma, entropy_coef,
+                       grad_out, stats_out);
 }
 
 int malib_adam_step(malib_ctx* c, float* params, const float* grad, float* m, float* v, int64_t n, int64_t step,

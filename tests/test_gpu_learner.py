@@ -94,6 +94,39 @@ def test_policy_gradient_parity(make, kw):
     ctx.close()
 
 
+def test_policy_gradient_batch():
+    """Every policy of a population in one call (including policies without
+    samples) against the oracle, and against the single-policy entry point."""
+    torch = need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=1024, pop=9, with_bias=True, seed=88)
+    w.pair_ids[w.pair_ids == 8] = 7                      # policy 8 never acts
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 2, 5)
+    tr = host(traj)
+    P = int(blocks(w.policies[0].dims)[-1])
+    ids = np.array([3, 8, 0, 1, 2, 4, 5, 6, 7], np.int32)
+    g = torch.zeros((len(ids), P), device="cuda")
+    st = torch.zeros((len(ids), 4), dtype=torch.float64, device="cuda")
+    ctx.learn_pg_batch(spec, w.pair_ids, 2, traj, ids, 0.9, 0.01, g, st)
+    ctx.sync()
+    g, st = g.cpu().numpy(), st.cpu().numpy()
+    for row, pid in enumerate(ids):
+        o, (M, b, loss, ent) = oracle_grad(w, tr, int(pid), 0.9, 0.01)
+        assert st[row, 0] == M
+        if M == 0:
+            assert np.all(g[row] == 0) and np.all(st[row] == 0)
+            continue
+        np.testing.assert_allclose([st[row, 1], st[row, 3]], [b, ent], rtol=1e-5, atol=1e-7)
+        check_grad(g[row], o, w.policies[pid].dims)
+        g1, st1 = learn(ctx, w, spec, traj, 2, int(pid), 0.9, 0.01)
+        check_grad(g[row], g1.astype(np.float64), w.policies[pid].dims)
+    with pytest.raises(MalibError, match="EINVAL"):
+        ctx.learn_pg_batch(spec, w.pair_ids, 2, traj, np.array([1, 2, 1], np.int32), 0.9, 0.0,
+                           np.zeros((3, P), np.float32))
+    ctx.close()
+
+
 def test_policy_without_samples():
     need_gpu()
     w = workloads.spread(n_agents=3, n_envs=256, pop=6, seed=5)
