@@ -901,6 +901,8 @@ def run_learner(args):
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
     launches0 = ctx.launch_count()
+    ctx.set_timing(True)                 # learn_grad_kernel's own CUDA-event time
+    ctx.main_kernel_ms(reset=True)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize(dev)
@@ -915,6 +917,8 @@ def run_learner(args):
         torch.distributed.barrier()
     launches = ctx.launch_count() - launches0
     ctx.sync()
+    grad_ms, grad_n = ctx.main_kernel_ms(reset=True)
+    ctx.set_timing(False)
     total_ms = sum(a.elapsed_time(c) for a, c in ev)
     total_ms_max = max_over_ranks(total_ms, world, dev)
     value = sum_over_ranks(float(samples * args.steps), world, dev) / (total_ms_max / 1e3)
@@ -922,7 +926,8 @@ def run_learner(args):
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
     peak = n_sm * FP32_LANES_PER_SM * 2 * sm_max * 1e6 / 1e12
-    achieved = samples * learn_flop(dims) / (total_ms / args.steps / 1e3) / 1e12
+    grad_avg_ms = grad_ms / max(grad_n, 1)
+    achieved = samples * learn_flop(dims) / (grad_avg_ms / 1e3) / 1e12
     e2e = None
     cpu = None
     if rank == 0:
@@ -977,7 +982,8 @@ def run_learner(args):
                              "peak_basis": f"fp32 FMA: {n_sm} SMs (queried) x {FP32_LANES_PER_SM} lanes x 2 "
                                            f"flop x {sm_max:.0f} MHz",
                              "algorithmic": f"{learn_flop(dims)} flop per sample (forward and backward, "
-                                            "bias sums excluded); whole step timed"},
+                                            f"bias sums excluded) x {samples} samples per launch",
+                             "kernel_ms": grad_avg_ms, "step_share": grad_avg_ms / (total_ms / args.steps)},
                 "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "gpu_launches": launches}
         print(json.dumps(line), flush=True)
     if world > 1:

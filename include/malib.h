@@ -464,7 +464,8 @@ int malib_eval_stats(malib_ctx* ctx, int64_t* n_decisions);
 int64_t malib_launch_count(const malib_ctx* ctx);
 
 /* Enables (1) or disables (0) CUDA-event timing of each call's main kernel on
- * the context's stream; malib_main_kernel_ms() returns the summed milliseconds
+ * the context's stream (for malib_learn_pg[_batch], the gradient kernel);
+ * malib_main_kernel_ms() returns the summed milliseconds
  * of the timed launches since the last reset (waits for the stream) and the
  * number of launches timed in *n_launches (may be NULL); reset clears both. */
 int malib_set_timing(malib_ctx* ctx, int enable);

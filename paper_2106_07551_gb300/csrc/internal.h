@@ -158,7 +158,9 @@ int64_t learn_work_bytes(int32_t nb, int32_t n_pairs, int32_t n_agents, int64_t 
                          int32_t T, int in, int grid, int ret_blocks);
 void learn_work_layout(uint8_t* base, int32_t nb, int32_t n_pairs, int32_t n_agents, int64_t n_envs,
                        int64_t n_episodes, int32_t T, int in, int grid, int ret_blocks, LearnArgs* a);
-cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s);
+// g0 / g1 (optional): events recorded just before and after learn_grad_kernel.
+cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s, cudaEvent_t g0 = nullptr,
+                            cudaEvent_t g1 = nullptr);
 cudaError_t launch_learn_adam(float* p, const float* g, float* m, float* v, int64_t n, float lr, float b1,
                               float b2, float eps, float c1, float c2, int n_sm, cudaStream_t s);
 cudaError_t launch_zero_u64(unsigned long long* p, int64_t n, cudaStream_t s);

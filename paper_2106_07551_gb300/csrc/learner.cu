@@ -610,7 +610,7 @@ void learn_work_layout(uint8_t* base, int32_t nb, int32_t n_pairs, int32_t n_age
     a->grid = grid;
 }
 
-cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s) {
+cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s, cudaEvent_t g0, cudaEvent_t g1) {
     if (a.nb <= 0) return cudaSuccess;
     learn_slots_kernel<<<a.nb, 1024, 0, s>>>(a);
     learn_plan_kernel<<<1, 32, 0, s>>>(a);
@@ -619,7 +619,9 @@ cudaError_t launch_learn_pg(const LearnArgs& a, int ret_blocks, cudaStream_t s) 
     cudaError_t err = cudaFuncSetAttribute(learn_grad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)kSBytes);
     if (err != cudaSuccess) return err;
+    if (g0) cudaEventRecord(g0, s);
     learn_grad_kernel<<<a.grid, kThreads, kSBytes, s>>>(a);
+    if (g1) cudaEventRecord(g1, s);
     const int P = (int)learn_param_count(a.in);
     learn_reduce_kernel<<<dim3((P + 2 + 255) / 256, a.nb), 256, 0, s>>>(a, P);
     return cudaGetLastError();

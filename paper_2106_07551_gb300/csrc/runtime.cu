@@ -854,7 +854,15 @@ int learn_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_id
     a.gamma = gamma;
     a.beta = entropy_coef;
     a.err = c->d_err;
-    CK(launch_learn_pg(a, ret_blocks, c->stream), "policy-gradient kernels");
+    // with timing on, the gradient kernel (the step's dominant one) is the timed launch
+    cudaEvent_t g0 = nullptr, g1 = nullptr;
+    if (c->timing && (cudaEventCreate(&g0) != cudaSuccess || cudaEventCreate(&g1) != cudaSuccess)) {
+        cudaGetLastError();
+        if (g0) cudaEventDestroy(g0);
+        g0 = g1 = nullptr;
+    }
+    CK(launch_learn_pg(a, ret_blocks, c->stream, g0, g1), "policy-gradient kernels");
+    if (g0) c->events.emplace_back(g0, g1);
     c->launches += 6;
     if (gw != kPtrHere)
         CK(cudaMemcpyAsync(grad_out, a.grad, (size_t)nb * P * 4, cudaMemcpyDeviceToHost, c->stream),

@@ -84,8 +84,13 @@ def test_quick_start_learner_loop():
         m, v = torch.zeros_like(w), torch.zeros_like(w)
         ctx.adam_step(w, grad, m, v, 1, 1e-4)
         ctx.pop_update(int(ids[0]), w)
+        grads = torch.zeros((len(params), P), device="cuda")
+        ctx.learn_pg_batch(spec, combos, 2, traj, list(range(len(params))), 0.95, 0.001, grads)
         ctx.rollout(spec, combos, 2, 8, traj)
         ctx.sync()
+        # the batched call's row 0 is the single call's gradient up to the order of
+        # its partial sums (the CTAs' shares of the tiles differ)
+        assert (grads[0] - grad).abs().max() <= 1e-4 * grad.abs().max()
         st = stats.cpu().numpy()
         assert st[0] == (combos == 0).sum() * 128 * 2 * 25 and np.all(np.isfinite(st))
         assert torch.isfinite(grad).all() and grad.abs().max() > 0
