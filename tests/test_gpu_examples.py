@@ -80,12 +80,13 @@ def test_quick_start_learner_loop():
         grad = torch.zeros(P, device="cuda")
         stats = torch.zeros(4, dtype=torch.float64, device="cuda")
         ctx.learn_pg(spec, combos, 2, traj, 0, 0.95, 0.001, grad, stats)
+        # every policy at once, on the same weights and trajectory
+        grads = torch.zeros((len(params), P), device="cuda")
+        ctx.learn_pg_batch(spec, combos, 2, traj, list(range(len(params))), 0.95, 0.001, grads)
         w = torch.from_numpy(params[0]).cuda()
         m, v = torch.zeros_like(w), torch.zeros_like(w)
         ctx.adam_step(w, grad, m, v, 1, 1e-4)
         ctx.pop_update(int(ids[0]), w)
-        grads = torch.zeros((len(params), P), device="cuda")
-        ctx.learn_pg_batch(spec, combos, 2, traj, list(range(len(params))), 0.95, 0.001, grads)
         ctx.rollout(spec, combos, 2, 8, traj)
         ctx.sync()
         # the batched call's row 0 is the single call's gradient up to the order of
