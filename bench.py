@@ -37,15 +37,20 @@ FP32_LANES_PER_SM = 128
 # figure is a one-episode capture x 2 (65,536 environments: one episode's output
 # is 15x the L2, so the traffic grows in proportion);
 # the evaluation kernels' traffic is the staging of the population, which does
-# not grow with the hands per pair.
+# not grow with the hands per pair; the learner's gradient kernel was captured
+# on the learner step's own workload.
 NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1441536 + 512,
     "kuhn_eval_kernel": 13312,
     "spread_rollout_f32_kernel<3,18,64,0>": 1373184 + 2559883520,
-    "leduc_eval_tc_kernel": 19404800 + 493824,
+    "leduc_eval_tc_kernel": 19406080 + 503040,
     "spread_rollout_f32_kernel<3,14,64,1>": 1683968 + 2068428800,
     "spread_rollout_f32_kernel<2,11,64,2>": 1547520 + 1034004736,
     "spread_rollout_tc_kernel": (20857088 + 1914217984) * 2,
+    "learn_grad_kernel": 511446016 + 3254016,
+    "spread_rollout_f32_kernel<2,8,64,3>": 1031936 + 706821376,
+    "spread_rollout_f32_kernel<4,16,64,4>": 8131072 + 2782468352,
+    "spread_rollout_f32_kernel<2,14,64,6>": 2387712 + 1377357056,
 }
 
 
@@ -978,7 +983,8 @@ def run_learner(args):
                                        f"pop{n_pol}", "samples_per_step": samples, "policies": n_pol,
                            "l2": "flushed (256 MiB write) before every timed step"},
                 "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                             "frac": achieved / peak, "traffic": None, "kernel": "learn_grad_kernel",
+                             "frac": achieved / peak, "traffic": NCU_TRAFFIC_PER_LAUNCH.get("learn_grad_kernel"),
+                             "kernel": "learn_grad_kernel",
                              "peak_basis": f"fp32 FMA: {n_sm} SMs (queried) x {FP32_LANES_PER_SM} lanes x 2 "
                                            f"flop x {sm_max:.0f} MHz",
                              "algorithmic": f"{learn_flop(dims)} flop per sample (forward and backward, "
