@@ -20,9 +20,19 @@ What it follows:
    over S_p (a baseline), H the entropy of the softmax over all actions.
    Adam as in Kingma and Ba (2015), with bias correction.
 
-Parity status: the gradient is pinned by central finite differences of the
-loss and by torch.autograd in fp64 (tests/test_oracle_learner.py); Adam by its
-first-step closed form and a hand-iterated scalar sequence.
+The PPO variant (the paper's learners are PPO/A2C-style; it prints no loss):
+Schulman et al. (2017)'s clipped surrogate with the same advantage A = G - b,
+       L = -(1/M) sum_i [ min(rho_i A_i, clip(rho_i, 1 - eps, 1 + eps) A_i)
+                          + beta H(pi(. | o_i)) ],
+rho_i = pi(a_i | o_i) / mu(a_i | o_i), mu the behavior policy that acted in the
+rollout, known from the logits the rollout recorded. At rho = 1 (the first
+epoch on fresh samples) its gradient is the policy gradient's.
+
+Parity status: the gradients are pinned by central finite differences of the
+losses and by torch.autograd in fp64 (tests/test_oracle_learner.py); the PPO
+gradient also by its two limits, the policy gradient at mu = pi and the
+entropy term alone when every sample is clipped; Adam by its first-step closed
+form and a hand-iterated scalar sequence.
 """
 from __future__ import annotations
 
@@ -79,6 +89,25 @@ def gather(traj: dict, pairs, n_envs: int, n_agents: int, obs_dim: int, policy_i
     return np.concatenate(obs), np.concatenate(act), np.concatenate(ret)
 
 
+def gather_logits(traj: dict, pairs, n_envs: int, n_agents: int, policy_id: int):
+    """The behavior logits [M][A] that the rollout recorded for policy_id's
+    samples (traj["logits"] [E][T][n_envs][N][A]), in gather()'s order."""
+    slots = samples(pairs, n_envs, n_agents, policy_id)
+    n_pairs = np.asarray(pairs).reshape(-1, n_agents).shape[0]
+    epp = n_envs // n_pairs
+    lg = np.asarray(traj["logits"], np.float64)
+    if not slots:
+        return np.zeros((0, lg.shape[-1]))
+    return np.concatenate([lg[:, :, c * epp:(c + 1) * epp, k, :].reshape(-1, lg.shape[-1]) for c, k in slots])
+
+
+def log_softmax(z: np.ndarray) -> np.ndarray:
+    """Row-wise log pi of logits z [M][A] (fp64, max-shifted)."""
+    z = np.asarray(z, np.float64)
+    zmax = z.max(axis=1, keepdims=True)
+    return z - zmax - np.log(np.exp(z - zmax).sum(axis=1, keepdims=True))
+
+
 def pg_loss(params, dims, obs, act, ret, beta: float):
     """The loss L above and (mean entropy, baseline)."""
     W1, b1, W2, b2, W3, b3 = unpack(params, dims)
@@ -133,6 +162,78 @@ def pg_grad(params, dims, obs, act, ret, beta: float):
     grad[:] = np.concatenate([dW1.ravel(), db1, dW2.ravel(), db2, dW3.ravel(), db3])
     loss = -(A * logp[np.arange(M), act] + beta * H).sum() / M
     return grad, (M, b, loss, H.mean())
+
+
+def ppo_loss(params, dims, obs, act, ret, blogits, beta: float, eps: float):
+    """The clipped-surrogate loss L of the PPO variant above (fp64)."""
+    W1, b1, W2, b2, W3, b3 = unpack(params, dims)
+    M = obs.shape[0]
+    if M == 0:
+        return 0.0
+    h1 = np.maximum(obs @ W1.T + b1, 0.0)
+    h2 = np.maximum(h1 @ W2.T + b2, 0.0)
+    logp = log_softmax(h2 @ W3.T + b3)
+    H = -(np.exp(logp) * logp).sum(axis=1)
+    A = ret - ret.mean()
+    idx = np.arange(M)
+    rho = np.exp(logp[idx, act] - log_softmax(blogits)[idx, act])
+    surr = np.minimum(rho * A, np.clip(rho, 1.0 - eps, 1.0 + eps) * A)
+    return -(surr + beta * H).sum() / M
+
+
+def ppo_grad(params, dims, obs, act, ret, blogits, beta: float, eps: float):
+    """dL/dparams of the clipped surrogate (fp64), with the chain rule written
+    out. The unclipped term is the minimum, and carries the gradient, when
+    rho A <= clip(rho) A (ties go to it); the clipped one is constant in the
+    parameters. So
+      dL/dz_j = (1/M) [ active A rho (pi_j - [j = a]) + beta pi_j (log pi_j + H) ],
+    then back through the layers as in pg_grad. Also returns (M, baseline,
+    loss, mean entropy)."""
+    W1, b1, W2, b2, W3, b3 = unpack(params, dims)
+    M = obs.shape[0]
+    grad = np.zeros(np.asarray(params).size)
+    if M == 0:
+        return grad, (0, 0.0, 0.0, 0.0)
+    pre1 = obs @ W1.T + b1
+    h1 = np.maximum(pre1, 0.0)
+    pre2 = h1 @ W2.T + b2
+    h2 = np.maximum(pre2, 0.0)
+    logp = log_softmax(h2 @ W3.T + b3)
+    pi = np.exp(logp)
+    H = -(pi * logp).sum(axis=1)
+    b = ret.mean()
+    A = ret - b
+    idx = np.arange(M)
+    rho = np.exp(logp[idx, act] - log_softmax(blogits)[idx, act])
+    clipped = np.clip(rho, 1.0 - eps, 1.0 + eps) * A
+    active = rho * A <= clipped
+    onehot = np.zeros_like(pi)
+    onehot[idx, act] = 1.0
+    dz = (np.where(active, A * rho, 0.0)[:, None] * (pi - onehot) + beta * pi * (logp + H[:, None])) / M
+    dW3 = dz.T @ h2
+    db3 = dz.sum(0)
+    d2 = (dz @ W3) * (pre2 > 0)
+    dW2 = d2.T @ h1
+    db2 = d2.sum(0)
+    d1 = (d2 @ W2) * (pre1 > 0)
+    dW1 = d1.T @ obs
+    db1 = d1.sum(0)
+    grad[:] = np.concatenate([dW1.ravel(), db1, dW2.ravel(), db2, dW3.ravel(), db3])
+    loss = -(np.minimum(rho * A, clipped) + beta * H).sum() / M
+    return grad, (M, b, loss, H.mean())
+
+
+def ppo_margin(params, dims, obs, act, blogits, eps: float) -> float:
+    """The smallest distance of any sample's ratio to a clip edge 1 -/+ eps:
+    where it is tiny, fp32 and fp64 may take that sample's branch differently."""
+    W1, b1, W2, b2, W3, b3 = unpack(params, dims)
+    if obs.shape[0] == 0:
+        return np.inf
+    h1 = np.maximum(obs @ W1.T + b1, 0.0)
+    h2 = np.maximum(h1 @ W2.T + b2, 0.0)
+    idx = np.arange(obs.shape[0])
+    rho = np.exp(log_softmax(h2 @ W3.T + b3)[idx, act] - log_softmax(blogits)[idx, act])
+    return float(np.minimum(np.abs(rho - (1.0 - eps)), np.abs(rho - (1.0 + eps))).min())
 
 
 def adam(params, grad, m, v, step: int, lr: float, beta1: float = 0.9, beta2: float = 0.999,
