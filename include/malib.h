@@ -431,6 +431,30 @@ int malib_learn_pg_batch(malib_ctx* ctx, const malib_env_spec* spec, const int32
                          double* stats_out);
 
 /*
+ * malib_learn_ppo_batch - malib_learn_pg_batch with PPO's clipped surrogate
+ * (Schulman et al. 2017; the paper's learners are PPO/A2C-style, Sec. 3.3 and
+ * App. C.2) in place of (G - b) log pi(a | o): with A = G - b as above and
+ * rho = pi(a | o) / mu(a | o), mu the behavior policy that acted in the rollout,
+ *   L = -(1/M) sum_S [ min(rho A, clip(rho, 1 - clip_eps, 1 + clip_eps) A)
+ *                      + entropy_coef H(pi(. | o)) ].
+ * mu is read from traj->logits, the logits [n_episodes][T][n_envs][N][5] that
+ * malib_rollout recorded under MALIB_DUMP_LOGITS (device memory of the
+ * context's device; EINVAL when NULL); pi is the loaded policy, so after
+ * malib_pop_update the same samples give the next epoch's gradient. Where the
+ * unclipped term is the minimum (ties included) it carries the gradient
+ * A rho (pi - onehot(a)) / M at the logits; elsewhere the surrogate is constant.
+ * With the loaded policy equal to the behavior policy (rho = 1) the gradient
+ * is malib_learn_pg_batch's up to rounding. clip_eps in (0, 1). Rows of
+ * grad_out and stats_out as in malib_learn_pg_batch (stats: M, b, L, mean
+ * entropy). Waits for the stream before returning. Errors: EINVAL, ESTATE,
+ * EUNSUPPORTED.
+ */
+int malib_learn_ppo_batch(malib_ctx* ctx, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                          int64_t n_episodes, const malib_traj* traj, const int32_t* policy_ids,
+                          int32_t n_policies, float gamma, float entropy_coef, float clip_eps, float* grad_out,
+                          double* stats_out);
+
+/*
  * malib_adam_step - one Adam step (the optimizer of App. C.2's training
  * config; Kingma and Ba, with bias correction) on n parameters, in place:
  *   m <- beta1 m + (1 - beta1) g;  v <- beta2 v + (1 - beta2) g^2;

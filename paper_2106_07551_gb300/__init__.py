@@ -290,6 +290,20 @@ class Context:
                                              n_episodes, C.byref(t), _ptr(ids), len(ids), gamma, entropy_coef,
                                              _ptr(grad_out), _ptr(stats_out) if stats_out is not None else None))
 
+    def learn_ppo_batch(self, spec, pair_ids, n_episodes, traj, policy_ids, gamma, entropy_coef, clip_eps,
+                        grad_out, stats_out=None):
+        """learn_pg_batch with PPO's clipped surrogate against the behavior
+        logits traj["logits"] that the rollout recorded (MALIB_DUMP_LOGITS)."""
+        ids = np.ascontiguousarray(policy_ids, np.int32)
+        lg = traj.get("logits")
+        t = Traj(_ptr(traj["obs"]), _ptr(traj["action"]), _ptr(traj["reward"]), None,
+                 _ptr(lg) if lg is not None else None)
+        _check(self.lib, self.handle,
+               self.lib.malib_learn_ppo_batch(self.handle, C.byref(spec), _ptr(pair_ids), int(pair_ids.shape[0]),
+                                              n_episodes, C.byref(t), _ptr(ids), len(ids), gamma, entropy_coef,
+                                              clip_eps, _ptr(grad_out),
+                                              _ptr(stats_out) if stats_out is not None else None))
+
     def adam_step(self, params, grad, m, v, step, lr, beta1=0.9, beta2=0.999, eps=1e-8):
         """One Adam step on device buffers (parameters, gradient, moments) in place."""
         n = int(params.numel()) if hasattr(params, "numel") else int(params.size)

@@ -34,7 +34,8 @@ EXPORTS = (
     "malib_selftest_sample",
     "malib_selftest_mma", "malib_selftest_mlp_tc", "malib_meta_fictitious_play", "malib_meta_lp_nash",
     "malib_meta_lp_nash_ex",
-    "malib_meta_aggregate", "malib_exploitability", "malib_learn_pg", "malib_learn_pg_batch", "malib_adam_step",
+    "malib_meta_aggregate", "malib_exploitability", "malib_learn_pg", "malib_learn_pg_batch",
+    "malib_learn_ppo_batch", "malib_adam_step",
     "malib_pop_update",
 )
 
@@ -109,6 +110,8 @@ def load(path: str | None = None):
                                          C.c_float, P, P]),
             "malib_learn_pg_batch": (C.c_int, [P, C.POINTER(EnvSpec), P, i32, i64, C.POINTER(Traj), P, i32,
                                                C.c_float, C.c_float, P, P]),
+            "malib_learn_ppo_batch": (C.c_int, [P, C.POINTER(EnvSpec), P, i32, i64, C.POINTER(Traj), P, i32,
+                                                C.c_float, C.c_float, C.c_float, P, P]),
             "malib_adam_step": (C.c_int, [P, P, P, P, P, i64, i64, C.c_float, C.c_float, C.c_float, C.c_float]),
             "malib_pop_update": (C.c_int, [P, i32, P, i64]),
         }

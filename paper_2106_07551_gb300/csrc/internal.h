@@ -139,6 +139,10 @@ struct LearnArgs {
     const uint8_t* action;       // [E][T][n_envs][n_agents]
     const float* reward;         // [E][T][n_envs][n_agents]
     float gamma, beta;
+    // PPO (clip > 0): the behavior policy's logits [E][T][n_envs][n_agents][5]
+    // that the rollout recorded, and the clip range; clip == 0: the policy gradient
+    const float* blogits;
+    float clip;
     int* err;
     // work space (learn_work_layout)
     int32_t* slots;              // [nb][n_pairs * n_agents] (c * n_agents + k) acting with each policy

@@ -10,6 +10,12 @@
 // H the entropy of the softmax over the 5 actions. The gradient by the chain
 // rule: dL/dz_j = (1/M) [ (G - b)(pi_j - [j = a]) + beta pi_j (log pi_j + H) ],
 // back through W3, the ReLUs (pre-activation > 0) and W2, W1.
+// The PPO variant (clip > 0; Schulman et al. 2017's clipped surrogate, the
+// same advantage A = G - b) replaces (G - b) log pi(a | o) by
+// min(rho A, clip(rho, 1 - eps, 1 + eps) A), rho = pi(a | o) / mu(a | o) with mu
+// the behavior policy whose logits the rollout recorded; the unclipped term
+// carries the gradient A rho (pi_j - [j = a]) where it is the minimum (ties
+// to it), the clipped one none.
 //
 // Kernels, in stream order:
 //  1. learn_slots_kernel: the (combination, agent) slots acting with p, in
@@ -326,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
         // the tile's observations (feature-major; zero columns past M), and for
         // the logits phase each sample's action and return
         int act = 0;
-        float ret = 0.f;
+        float ret = 0.f, lmu = 0.f;
         {
             const int r = tid & (kTile - 1), half = tid >> 7;
             const int64_t s = s0 + r;
@@ -337,6 +343,24 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
                 if (half == 0) {
                     act = a.action[ix];
                     ret = Gb[s];
+                    if (a.clip > 0.f) {
+                        // log mu(a | o): the behavior policy's log-softmax at the action taken
+                        const float* bl = a.blogits + ix * kA;
+                        float l[kA];
+#pragma unroll
+                        for (int j = 0; j < kA; ++j) l[j] = bl[j];
+                        float m = l[0];
+#pragma unroll
+                        for (int j = 1; j < kA; ++j) m = fmaxf(m, l[j]);
+                        float S = 0.f;
+#pragma unroll
+                        for (int j = 0; j < kA; ++j) S += expf(l[j] - m);
+                        float la = l[0];
+#pragma unroll
+                        for (int j = 1; j < kA; ++j)
+                            if (j == act) la = l[j];
+                        lmu = la - m - logf(S);
+                    }
                 }
             } else {
                 for (int k = half; k < in; k += 2) XT[k * kTS + r] = 0.f;
@@ -380,10 +404,23 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
 #pragma unroll
                 for (int j = 1; j < kA; ++j)
                     if (j == act) lp_a = logp[j];
+                if (a.clip > 0.f) {
+                    // PPO: min(rho A, clip(rho) A); the unclipped term carries the
+                    // gradient A rho (pi - [j = a]) when it is the minimum (ties to it)
+                    const float rho = expf(lp_a - lmu);
+                    const float unc = rho * adv;
+                    const float clp = fminf(fmaxf(rho, 1.f - a.clip), 1.f + a.clip) * adv;
+                    const float w = unc <= clp ? unc : 0.f;
 #pragma unroll
-                for (int j = 0; j < kA; ++j)
-                    dz[j] = (adv * (pi[j] - (j == act ? 1.f : 0.f)) + a.beta * pi[j] * (logp[j] + H)) * invM;
-                lsum -= adv * lp_a + a.beta * H;
+                    for (int j = 0; j < kA; ++j)
+                        dz[j] = (w * (pi[j] - (j == act ? 1.f : 0.f)) + a.beta * pi[j] * (logp[j] + H)) * invM;
+                    lsum -= fminf(unc, clp) + a.beta * H;
+                } else {
+#pragma unroll
+                    for (int j = 0; j < kA; ++j)
+                        dz[j] = (adv * (pi[j] - (j == act ? 1.f : 0.f)) + a.beta * pi[j] * (logp[j] + H)) * invM;
+                    lsum -= adv * lp_a + a.beta * H;
+                }
                 hsum += H;
             }
 #pragma unroll

@@ -771,9 +771,10 @@ int malib_rollout(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_
 namespace {
 
 // The policy-gradient step of nb distinct policies (host ids) in one batch.
+// clip > 0: the PPO surrogate against the behavior logits traj->logits; 0: the policy gradient.
 int learn_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
                 int64_t n_episodes, const malib_traj* traj, const int32_t* ids, int32_t nb, float gamma,
-                float entropy_coef, float* grad_out, double* stats_out) {
+                float entropy_coef, float clip, float* grad_out, double* stats_out) {
     int r;
     if ((r = check_spec(c, spec)) != MALIB_OK) return r;
     if (!c->has_pop) return fail(c, MALIB_ESTATE, "no population loaded");
@@ -808,6 +809,11 @@ int learn_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_id
     for (const void* p : tp)
         if (!is_device_ptr(c, p))
             return fail(c, MALIB_EINVAL, "trajectory buffers must be device memory of the context's device");
+    if (clip != 0.0f) {
+        if (!(clip > 0.0f && clip < 1.0f)) return fail(c, MALIB_EINVAL, "clip_eps must lie in (0, 1)");
+        if (!traj->logits || !is_device_ptr(c, traj->logits))
+            return fail(c, MALIB_EINVAL, "the PPO step needs the behavior logits (traj->logits, device memory)");
+    }
     const int gw = ptr_where(grad_out, c->device);
     const int sw = stats_out ? ptr_where(stats_out, c->device) : kPtrHost;
     if (gw == kPtrOther || sw == kPtrOther)
@@ -853,6 +859,8 @@ int learn_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_id
     a.reward = traj->reward;
     a.gamma = gamma;
     a.beta = entropy_coef;
+    a.clip = clip;
+    a.blogits = clip > 0.0f ? traj->logits : nullptr;
     a.err = c->d_err;
     // with timing on, the gradient kernel (the step's dominant one) is the timed launch
     cudaEvent_t g0 = nullptr, g1 = nullptr;
@@ -883,8 +891,8 @@ int malib_learn_pg(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair
                    float entropy_coef, float* grad_out, double* stats_out) {
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);
-    return learn_batch(c, spec, pair_ids, n_pairs, n_episodes, traj, &policy_id, 1, gamma, entropy_coef, grad_out,
-                       stats_out);
+    return learn_batch(c, spec, pair_ids, n_pairs, n_episodes, traj, &policy_id, 1, gamma, entropy_coef, 0.0f,
+                       grad_out, stats_out);
 }
 
 int malib_learn_pg_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
@@ -893,7 +901,18 @@ int malib_learn_pg_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t
     if (!c) return MALIB_EINVAL;
     DeviceGuard g(c->device);
     return learn_batch(c, spec, pair_ids, n_pairs, n_episodes, traj, policy_ids, n_policies, gamma, entropy_coef,
-                       grad_out, stats_out);
+                       0.0f, grad_out, stats_out);
+}
+
+int malib_learn_ppo_batch(malib_ctx* c, const malib_env_spec* spec, const int32_t* pair_ids, int32_t n_pairs,
+                          int64_t n_episodes, const malib_traj* traj, const int32_t* policy_ids,
+                          int32_t n_policies, float gamma, float entropy_coef, float clip_eps, float* grad_out,
+                          double* stats_out) {
+    if (!c) return MALIB_EINVAL;
+    DeviceGuard g(c->device);
+    if (!(clip_eps > 0.0f && clip_eps < 1.0f)) return fail(c, MALIB_EINVAL, "clip_eps must lie in (0, 1)");
+    return learn_batch(c, spec, pair_ids, n_pairs, n_episodes, traj, policy_ids, n_policies, gamma, entropy_coef,
+                       clip_eps, grad_out, stats_out);
 }
 
 int malib_adam_step(malib_ctx* c, float* params, const float* grad, float* m, float* v, int64_t n, int64_t step,

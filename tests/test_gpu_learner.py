@@ -219,3 +219,115 @@ def test_learner_refusals():
     with pytest.raises(MalibError, match="EUNSUPPORTED"):
         ctx.learn_pg(spec, wb.pair_ids, 1, traj, 0, 0.9, 0.0, np.zeros(100, np.float32))
     ctx.close()
+
+
+# ---- PPO: the clipped surrogate against the behavior logits the rollout recorded
+
+def perturbed(w, pids, scale, seed):
+    """New parameters for the policies pids (the behavior policies stay in w)."""
+    rng = np.random.default_rng(seed)
+    return {pid: (w.policies[pid].params + rng.normal(0, scale, w.policies[pid].params.shape)).astype(np.float32)
+            for pid in pids}
+
+
+def ppo_oracle(w, tr, pid, params, gamma, beta, eps):
+    obs, act, ret = learner.gather(tr, w.pair_ids, w.n_envs, w.n_agents, w.obs_dim, pid, gamma)
+    blog = learner.gather_logits(tr, w.pair_ids, w.n_envs, w.n_agents, pid)
+    dims = w.policies[pid].dims
+    return (learner.ppo_grad(params, dims, obs, act, ret, blog, beta, eps),
+            learner.ppo_margin(params, dims, obs, act, blog, eps), (obs, act, ret, blog))
+
+
+@pytest.mark.parametrize("make,kw", [(workloads.spread, dict(n_agents=3, n_envs=256, pop=6)),
+                                     (workloads.tag, dict(n_envs=256, pop=5))])
+def test_ppo_parity(make, kw):
+    """Policies moved away from the ones that acted: the GPU's clipped-surrogate
+    gradient against the oracle's. A sample whose ratio lies within the fp32
+    error (a few 1e-6) of a clip edge may take the other branch on the GPU, so
+    the clip range is chosen among nearby values as one that leaves every
+    ratio at least 2e-5 from both edges; samples are clipped on both sides."""
+    torch = need_gpu()
+    w = make(with_bias=True, seed=71, **kw)
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 2, 41, MALIB_DUMP_LOGITS)
+    tr = host(traj)
+    ids, counts = np.unique(w.pair_ids, return_counts=True)
+    pids = [int(p) for p in ids[np.argsort(-counts, kind="stable")][:2]]   # the two busiest policies
+    new = perturbed(w, pids, 0.05, 5)
+    gamma, beta = 0.95, 0.01
+    for eps in np.linspace(0.15, 0.25, 21):
+        eps = float(eps)
+        res = {pid: ppo_oracle(w, tr, pid, new[pid], gamma, beta, eps) for pid in pids}
+        if min(r[1] for r in res.values()) > 2e-5:
+            break
+    else:
+        pytest.fail("no clip range with a clear margin")
+    # both branches are exercised
+    obs, act, ret, blog = res[pids[0]][2]
+    dims = w.policies[0].dims
+    W1, b1, W2, b2, W3, b3 = learner.unpack(new[pids[0]], dims)
+    z = np.maximum(np.maximum(obs @ W1.T + b1, 0) @ W2.T + b2, 0) @ W3.T + b3
+    idx = np.arange(obs.shape[0])
+    rho = np.exp(learner.log_softmax(z)[idx, act] - learner.log_softmax(blog)[idx, act])
+    assert (rho > 1 + eps).any() and (rho < 1 - eps).any() and (np.abs(rho - 1) < eps).any()
+    for pid in pids:
+        ctx.pop_update(pid, new[pid])
+    P = int(blocks(dims)[-1])
+    g = torch.zeros((len(pids), P), device="cuda")
+    st = torch.zeros((len(pids), 4), dtype=torch.float64, device="cuda")
+    ctx.learn_ppo_batch(spec, w.pair_ids, 2, traj, pids, gamma, beta, eps, g, st)
+    ctx.sync()
+    g, st = g.cpu().numpy(), st.cpu().numpy()
+    for row, pid in enumerate(pids):
+        o, (M, b, loss, ent) = res[pid][0]
+        assert st[row, 0] == M and M > 0
+        np.testing.assert_allclose([st[row, 1], st[row, 3]], [b, ent], rtol=1e-5, atol=1e-7)
+        assert abs(st[row, 2] - loss) <= 1e-5 * (1.0 + np.abs(tr["reward"]).max() * w.episode_len)
+        check_grad(g[row], o, dims)
+    # deterministic
+    g2 = torch.zeros((len(pids), P), device="cuda")
+    ctx.learn_ppo_batch(spec, w.pair_ids, 2, traj, pids, gamma, beta, eps, g2)
+    ctx.sync()
+    assert np.array_equal(g, g2.cpu().numpy())
+    ctx.close()
+
+
+def test_ppo_on_policy_is_the_policy_gradient():
+    """The policies that acted, unchanged: every ratio is 1 up to rounding, and
+    the PPO gradient is the policy gradient's."""
+    torch = need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=1024, pop=6, with_bias=True, seed=72)
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 2, 43, MALIB_DUMP_LOGITS)
+    P = int(blocks(w.policies[0].dims)[-1])
+    ids = [0, 3, 5]
+    g_ppo = torch.zeros((3, P), device="cuda")
+    g_pg = torch.zeros((3, P), device="cuda")
+    ctx.learn_ppo_batch(spec, w.pair_ids, 2, traj, ids, 0.9, 0.001, 0.2, g_ppo)
+    ctx.learn_pg_batch(spec, w.pair_ids, 2, traj, ids, 0.9, 0.001, g_pg)
+    ctx.sync()
+    for row, pid in enumerate(ids):
+        check_grad(g_ppo[row].cpu().numpy(), g_pg[row].cpu().numpy().astype(np.float64), w.policies[pid].dims)
+    ctx.close()
+
+
+def test_ppo_refusals():
+    torch = need_gpu()
+    w = workloads.spread(n_agents=3, n_envs=256, pop=3, seed=73)
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 1, 3)                       # no logits recorded
+    P = int(blocks(w.policies[0].dims)[-1])
+    g = torch.zeros((1, P), device="cuda")
+    with pytest.raises(MalibError, match="EINVAL"):
+        ctx.learn_ppo_batch(spec, w.pair_ids, 1, traj, [0], 0.9, 0.0, 0.2, g)
+    spec, traj = rollout(ctx, w, 1, 3, MALIB_DUMP_LOGITS)
+    for eps in (0.0, -0.1, 1.0, float("nan")):
+        with pytest.raises(MalibError, match="EINVAL"):
+            ctx.learn_ppo_batch(spec, w.pair_ids, 1, traj, [0], 0.9, 0.0, eps, g)
+    ctx.learn_ppo_batch(spec, w.pair_ids, 1, traj, [0], 0.9, 0.0, 0.2, g)
+    ctx.sync()
+    assert torch.isfinite(g).all()
+    ctx.close()
