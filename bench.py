@@ -66,7 +66,8 @@ def parse():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["leduc", "kuhn", "spread3", "adversary3", "speaker_listener",
-                                           "leduc_bf16", "spread8", "meta", "learner", "push", "tag", "reference"],
+                                           "leduc_bf16", "spread8", "meta", "learner", "learner_ppo", "push", "tag",
+                                           "reference"],
                     default="leduc_bf16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
@@ -876,10 +877,13 @@ def run_learner(args):
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
     ctx = Context(local, stream)
-    spec = make_spec(w.env_kind, w.n_agents, w.obs_dim, w.n_actions, w.n_landmarks, w.episode_len, w.n_envs)
+    ppo = args.workload == "learner_ppo"
+    from paper_2106_07551_gb300 import MALIB_DUMP_LOGITS
+    spec = make_spec(w.env_kind, w.n_agents, w.obs_dim, w.n_actions, w.n_landmarks, w.episode_len, w.n_envs,
+                     MALIB_DUMP_LOGITS if ppo else 0)
     ctx.pop_load(spec, [policy_desc(p.kind, p.dtype, p.seat, p.dims, p.params) for p in w.policies])
     d_pairs = torch.from_numpy(w.pair_ids).to(dev)
-    traj = alloc_traj(spec, w.n_episodes)
+    traj = alloc_traj(spec, w.n_episodes, logits=ppo)
     ctx.rollout(spec, d_pairs, w.n_episodes, w.seed + rank, traj)
     dims = w.policies[0].dims
     n_pol = len(w.policies)
@@ -896,7 +900,10 @@ def run_learner(args):
 
     def step():
         state["t"] += 1
-        ctx.learn_pg_batch(spec, d_pairs, w.n_episodes, traj, ids, 0.95, 0.001, grads)
+        if ppo:
+            ctx.learn_ppo_batch(spec, d_pairs, w.n_episodes, traj, ids, 0.95, 0.001, 0.2, grads)
+        else:
+            ctx.learn_pg_batch(spec, d_pairs, w.n_episodes, traj, ids, 0.95, 0.001, grads)
         ctx.adam_step(params, grads, m, v, state["t"], 1e-4)
 
     for _ in range(args.warmup):
@@ -940,6 +947,7 @@ def run_learner(args):
         h_obs = traj["obs"].cpu().pin_memory()
         h_act = traj["action"].cpu().pin_memory()
         h_rew = traj["reward"].cpu().pin_memory()
+        h_lg = traj["logits"].cpu().pin_memory() if ppo else None
         h_g = torch.empty_like(grads, device="cpu").pin_memory()
         reps = max(1, args.e2e_steps // 5)
         t_e2e = 0.0
@@ -949,22 +957,31 @@ def run_learner(args):
             traj["obs"].copy_(h_obs, non_blocking=True)
             traj["action"].copy_(h_act, non_blocking=True)
             traj["reward"].copy_(h_rew, non_blocking=True)
+            if ppo:
+                traj["logits"].copy_(h_lg, non_blocking=True)
             step()
             h_g.copy_(grads, non_blocking=True)
             torch.cuda.synchronize(dev)
             if k > 0:
                 t_e2e += time.perf_counter() - s0
         e2e = {"value": samples * reps / t_e2e, "unit": "samples/s",
-               "h2d_bytes_per_step": int(h_obs.numel() * 4 + h_act.numel() + h_rew.numel() * 4),
+               "h2d_bytes_per_step": int(h_obs.numel() * 4 + h_act.numel() + h_rew.numel() * 4 +
+                                         (h_lg.numel() * 4 if ppo else 0)),
                "d2h_bytes_per_step": int(h_g.numel() * 4), "steps": reps}
         if world == 1 and not args.no_cpu_baseline:
             from oracle import learner as ol
             tr = {"obs": h_obs.numpy(), "action": h_act.numpy(), "reward": h_rew.numpy()}
+            if ppo:
+                tr["logits"] = h_lg.numpy()
             n_done, t_cpu, n_s = 0, 0.0, 0
             while t_cpu < 10.0 and n_done < n_pol:
                 s0 = time.perf_counter()
                 o, a_, r_ = ol.gather(tr, w.pair_ids, w.n_envs, w.n_agents, w.obs_dim, n_done, 0.95)
-                ol.pg_grad(w.policies[n_done].params, dims, o, a_, r_, 0.001)
+                if ppo:
+                    bl = ol.gather_logits(tr, w.pair_ids, w.n_envs, w.n_agents, n_done)
+                    ol.ppo_grad(w.policies[n_done].params, dims, o, a_, r_, bl, 0.001, 0.2)
+                else:
+                    ol.pg_grad(w.policies[n_done].params, dims, o, a_, r_, 0.001)
                 t_cpu += time.perf_counter() - s0
                 n_s += o.shape[0]
                 n_done += 1
@@ -974,16 +991,19 @@ def run_learner(args):
     clk = clocks.summary()
     ctx.close()
     if rank == 0:
-        line = {"metric": "learner samples/sec (policy-gradient step and Adam of every policy)",
+        line = {"metric": ("learner samples/sec (PPO clipped-surrogate step and Adam of every policy)" if ppo
+                           else "learner samples/sec (policy-gradient step and Adam of every policy)"),
                 "value": value, "unit": "samples/s", "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
                 "data": "synthetic",
-                "config": {"workload": f"learner_spread_n3_4096env_mlp18-64-64-5_f32_{w.n_episodes}episodes_"
-                                       f"pop{n_pol}", "samples_per_step": samples, "policies": n_pol,
+                "config": {"workload": f"learner{'_ppo' if ppo else ''}_spread_n3_4096env_mlp18-64-64-5_f32_"
+                                       f"{w.n_episodes}episodes_pop{n_pol}", "samples_per_step": samples,
+                           "policies": n_pol,
                            "l2": "flushed (256 MiB write) before every timed step"},
                 "roofline": {"bound": "alu", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                             "frac": achieved / peak, "traffic": NCU_TRAFFIC_PER_LAUNCH.get("learn_grad_kernel"),
+                             "frac": achieved / peak,
+                             "traffic": None if ppo else NCU_TRAFFIC_PER_LAUNCH.get("learn_grad_kernel"),
                              "kernel": "learn_grad_kernel",
                              "peak_basis": f"fp32 FMA: {n_sm} SMs (queried) x {FP32_LANES_PER_SM} lanes x 2 "
                                            f"flop x {sm_max:.0f} MHz",
@@ -1003,7 +1023,7 @@ def main():
         return run_reference(args)
     if args.workload == "meta":
         return run_meta(args)
-    if args.workload == "learner":
+    if args.workload in ("learner", "learner_ppo"):
         return run_learner(args)
     return run_ours(args)
 
