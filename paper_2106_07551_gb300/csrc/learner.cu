@@ -38,6 +38,7 @@
 
 #include "device_common.cuh"
 #include "internal.h"
+#include "mlp_f32.cuh"      // packed fp32 pair helpers (f2_fma: two IEEE fmaf per instruction)
 
 namespace malib {
 
@@ -185,36 +186,51 @@ __device__ __forceinline__ int64_t sample_index(const LearnArgs& a, const int32_
 }
 
 // H_out[j][s] = relu(b[j] + sum_k W[k][j] H_in[k][s]) for this thread's 8
-// samples (8 sg ..) and 4 outputs (ng + 16 q): two 16-byte loads of H_in and
-// four weights per k.
+// samples (8 sg ..) and 4 outputs (ng + 16 q): per k two 16-byte loads of H_in
+// (four sample pairs) and four weights, each duplicated into a pair, for 16
+// packed FMAs (each lane an fmaf in the same order as a scalar loop).
 __device__ __forceinline__ void dense_relu(const float* __restrict__ Win, const float* __restrict__ b,
                                            const float* __restrict__ Hin, int K, float* __restrict__ Hout,
                                            int sg, int ng) {
-    float acc[4][8];
+    using u64 = unsigned long long;
+    u64 acc[4][4];
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
+    for (int q = 0; q < 4; ++q) {
+        const u64 b2 = f2_dup(b[ng + 16 * q]);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) acc[q][i] = b[ng + 16 * q];
+        for (int i = 0; i < 4; ++i) acc[q][i] = b2;
+    }
 #pragma unroll 4
     for (int k = 0; k < K; ++k) {
-        const float4 x0 = *reinterpret_cast<const float4*>(Hin + k * kTS + 8 * sg);
-        const float4 x1 = *reinterpret_cast<const float4*>(Hin + k * kTS + 8 * sg + 4);
-        const float x[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+        const ulonglong2 x0 = *reinterpret_cast<const ulonglong2*>(Hin + k * kTS + 8 * sg);
+        const ulonglong2 x1 = *reinterpret_cast<const ulonglong2*>(Hin + k * kTS + 8 * sg + 4);
+        const u64 x[4] = {x0.x, x0.y, x1.x, x1.y};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-            const float w = Win[k * kH + ng + 16 * q];
+            const u64 w = f2_dup(Win[k * kH + ng + 16 * q]);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) acc[q][i] = fmaf(w, x[i], acc[q][i]);
+            for (int i = 0; i < 4; ++i) f2_fma(acc[q][i], x[i], w);
         }
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        float* o = Hout + (ng + 16 * q) * kTS + 8 * sg;
-        *reinterpret_cast<float4*>(o) = make_float4(fmaxf(acc[q][0], 0.f), fmaxf(acc[q][1], 0.f),
-                                                    fmaxf(acc[q][2], 0.f), fmaxf(acc[q][3], 0.f));
-        *reinterpret_cast<float4*>(o + 4) = make_float4(fmaxf(acc[q][4], 0.f), fmaxf(acc[q][5], 0.f),
-                                                        fmaxf(acc[q][6], 0.f), fmaxf(acc[q][7], 0.f));
+        ulonglong2* o = reinterpret_cast<ulonglong2*>(Hout + (ng + 16 * q) * kTS + 8 * sg);
+        o[0] = make_ulonglong2(f2_relu(acc[q][0]), f2_relu(acc[q][1]));
+        o[1] = make_ulonglong2(f2_relu(acc[q][2]), f2_relu(acc[q][3]));
     }
+}
+
+// The 8 values of a sample-pair row (four pairs) where the activations h are
+// positive, else 0 (the ReLU's derivative), stored at o.
+__device__ __forceinline__ void store_masked(float* __restrict__ o, const unsigned long long (&v)[4],
+                                             const float* __restrict__ h) {
+    const float4 h0 = *reinterpret_cast<const float4*>(h);
+    const float4 h1 = *reinterpret_cast<const float4*>(h + 4);
+    const float2 v0 = f2_split(v[0]), v1 = f2_split(v[1]), v2 = f2_split(v[2]), v3 = f2_split(v[3]);
+    *reinterpret_cast<float4*>(o) = make_float4(h0.x > 0.f ? v0.x : 0.f, h0.y > 0.f ? v0.y : 0.f,
+                                                h0.z > 0.f ? v1.x : 0.f, h0.w > 0.f ? v1.y : 0.f);
+    *reinterpret_cast<float4*>(o + 4) = make_float4(h1.x > 0.f ? v2.x : 0.f, h1.y > 0.f ? v2.y : 0.f,
+                                                    h1.z > 0.f ? v3.x : 0.f, h1.w > 0.f ? v3.y : 0.f);
 }
 
 // A CTA's contiguous share [lo, hi) of the batch's tiles (all policies' tiles
@@ -427,63 +443,50 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
             for (int j = 0; j < kA; ++j) DZT[j * kTS + tid] = dz[j];
         }
         __syncthreads();
-        // D2 = (dz W3) * [h2 > 0]: samples 8 sg .., units ng + 16 q
+        // D2 = (dz W3) * [h2 > 0]: samples 8 sg .. (four pairs), units ng + 16 q
         {
-            float dzv[kA][8];
+            using u64 = unsigned long long;
+            u64 dzv[kA][4];
 #pragma unroll
             for (int c = 0; c < kA; ++c) {
-                const float4 d0 = *reinterpret_cast<const float4*>(DZT + c * kTS + 8 * sg);
-                const float4 d1 = *reinterpret_cast<const float4*>(DZT + c * kTS + 8 * sg + 4);
-                dzv[c][0] = d0.x; dzv[c][1] = d0.y; dzv[c][2] = d0.z; dzv[c][3] = d0.w;
-                dzv[c][4] = d1.x; dzv[c][5] = d1.y; dzv[c][6] = d1.z; dzv[c][7] = d1.w;
+                const ulonglong2 d0 = *reinterpret_cast<const ulonglong2*>(DZT + c * kTS + 8 * sg);
+                const ulonglong2 d1 = *reinterpret_cast<const ulonglong2*>(DZT + c * kTS + 8 * sg + 4);
+                dzv[c][0] = d0.x; dzv[c][1] = d0.y; dzv[c][2] = d1.x; dzv[c][3] = d1.y;
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int j = ng + 16 * q;
-                float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                u64 v[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
                 for (int c = 0; c < kA; ++c) {
-                    const float w = sm[kSW3 + c * kH + j];
+                    const u64 w = f2_dup(sm[kSW3 + c * kH + j]);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) v[i] = fmaf(dzv[c][i], w, v[i]);
+                    for (int i = 0; i < 4; ++i) f2_fma(v[i], dzv[c][i], w);
                 }
-                const float4 h0 = *reinterpret_cast<const float4*>(H2T + j * kTS + 8 * sg);
-                const float4 h1 = *reinterpret_cast<const float4*>(H2T + j * kTS + 8 * sg + 4);
-                float* o = D2T + j * kTS + 8 * sg;
-                *reinterpret_cast<float4*>(o) = make_float4(h0.x > 0.f ? v[0] : 0.f, h0.y > 0.f ? v[1] : 0.f,
-                                                            h0.z > 0.f ? v[2] : 0.f, h0.w > 0.f ? v[3] : 0.f);
-                *reinterpret_cast<float4*>(o + 4) = make_float4(h1.x > 0.f ? v[4] : 0.f, h1.y > 0.f ? v[5] : 0.f,
-                                                                h1.z > 0.f ? v[6] : 0.f, h1.w > 0.f ? v[7] : 0.f);
+                store_masked(D2T + j * kTS + 8 * sg, v, H2T + j * kTS + 8 * sg);
             }
         }
         __syncthreads();
-        // D1 = (D2 W2) * [h1 > 0]: samples 8 sg .., units ng + 16 q
+        // D1 = (D2 W2) * [h1 > 0]: samples 8 sg .. (four pairs), units ng + 16 q
         {
-            float acc[4][8] = {};
+            using u64 = unsigned long long;
+            u64 acc[4][4] = {};
 #pragma unroll 4
             for (int j = 0; j < kH; ++j) {
-                const float4 d0 = *reinterpret_cast<const float4*>(D2T + j * kTS + 8 * sg);
-                const float4 d1 = *reinterpret_cast<const float4*>(D2T + j * kTS + 8 * sg + 4);
-                const float d[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+                const ulonglong2 d0 = *reinterpret_cast<const ulonglong2*>(D2T + j * kTS + 8 * sg);
+                const ulonglong2 d1 = *reinterpret_cast<const ulonglong2*>(D2T + j * kTS + 8 * sg + 4);
+                const u64 d[4] = {d0.x, d0.y, d1.x, d1.y};
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    const float w = sm[kSW2 + j * kH + ng + 16 * q];
+                    const u64 w = f2_dup(sm[kSW2 + j * kH + ng + 16 * q]);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i) acc[q][i] = fmaf(w, d[i], acc[q][i]);
+                    for (int i = 0; i < 4; ++i) f2_fma(acc[q][i], d[i], w);
                 }
             }
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 const int k = ng + 16 * q;
-                const float4 h0 = *reinterpret_cast<const float4*>(H1T + k * kTS + 8 * sg);
-                const float4 h1 = *reinterpret_cast<const float4*>(H1T + k * kTS + 8 * sg + 4);
-                float* o = D1T + k * kTS + 8 * sg;
-                *reinterpret_cast<float4*>(o) =
-                    make_float4(h0.x > 0.f ? acc[q][0] : 0.f, h0.y > 0.f ? acc[q][1] : 0.f,
-                                h0.z > 0.f ? acc[q][2] : 0.f, h0.w > 0.f ? acc[q][3] : 0.f);
-                *reinterpret_cast<float4*>(o + 4) =
-                    make_float4(h1.x > 0.f ? acc[q][4] : 0.f, h1.y > 0.f ? acc[q][5] : 0.f,
-                                h1.z > 0.f ? acc[q][6] : 0.f, h1.w > 0.f ? acc[q][7] : 0.f);
+                store_masked(D1T + k * kTS + 8 * sg, acc[q], H1T + k * kTS + 8 * sg);
             }
         }
         __syncthreads();
