@@ -331,3 +331,42 @@ def test_ppo_refusals():
     ctx.sync()
     assert torch.isfinite(g).all()
     ctx.close()
+
+
+def test_ppo_batch_with_an_idle_policy_and_push():
+    """PPO over every policy of a push population, one of which never acts (its
+    row and statistics stay zero), after one Adam-free perturbation of the
+    others; each row against the oracle."""
+    torch = need_gpu()
+    w = workloads.push(n_envs=384, pop=4, envs_per_pair=64, with_bias=True, seed=74)
+    w.pair_ids[w.pair_ids == 3] = 2                      # policy 3 never acts
+    ctx = context()
+    load_population(ctx, w)
+    spec, traj = rollout(ctx, w, 2, 47, MALIB_DUMP_LOGITS)
+    tr = host(traj)
+    pids = [0, 1, 2]
+    new = perturbed(w, pids, 0.03, 9)
+    for eps in np.linspace(0.15, 0.25, 21):
+        eps = float(eps)
+        res = {pid: ppo_oracle(w, tr, pid, new[pid], 0.9, 0.005, eps) for pid in pids}
+        if min(r[1] for r in res.values()) > 2e-5:
+            break
+    else:
+        pytest.fail("no clip range with a clear margin")
+    for pid in pids:
+        ctx.pop_update(pid, new[pid])
+    dims = w.policies[0].dims
+    P = int(blocks(dims)[-1])
+    ids = [3, 0, 1, 2]
+    g = torch.zeros((4, P), device="cuda")
+    st = torch.zeros((4, 4), dtype=torch.float64, device="cuda")
+    ctx.learn_ppo_batch(spec, w.pair_ids, 2, traj, ids, 0.9, 0.005, eps, g, st)
+    ctx.sync()
+    g, st = g.cpu().numpy(), st.cpu().numpy()
+    assert np.all(g[0] == 0) and np.all(st[0] == 0)
+    for row, pid in enumerate(ids[1:], start=1):
+        o, (M, b, loss, ent) = res[pid][0]
+        assert st[row, 0] == M and M > 0
+        np.testing.assert_allclose([st[row, 1], st[row, 3]], [b, ent], rtol=1e-5, atol=1e-7)
+        check_grad(g[row], o, dims)
+    ctx.close()
