@@ -68,6 +68,10 @@ def test_fp_bit_exact_off_chip_and_max(ctx):
     check_fp_exact(t1, 300, *run_fp(ctx, t1, 300))
     t2 = rng.normal(size=(1, 1024, 1024))           # the largest supported table
     check_fp_exact(t2, 50, *run_fp(ctx, t2, 50))
+    t3 = rng.normal(size=(3, 256, 200))             # 256 rows, one per thread, read from L2
+    check_fp_exact(t3, 120, *run_fp(ctx, t3, 120))
+    t4 = rng.normal(size=(2, 257, 100))             # 257 rows: two per thread for some
+    check_fp_exact(t4, 120, *run_fp(ctx, t4, 120))
 
 
 def test_fp_many_games(ctx):
