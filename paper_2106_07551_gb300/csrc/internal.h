@@ -114,9 +114,14 @@ struct LeducWork {
     uint16_t* queues;            // [grid][2 seats][2 queues][max_hands]
     int32_t max_hands;
     int64_t n_seg;               // segments per pair (set by the launcher)
+    int32_t split_from;          // pairs from this one on are played in 2 n_seg segments
+    int64_t n_units;             // units of the call
 };
-// Units (pair, segment) of a call and the segments per pair.
-int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n_seg_out);
+// Units (pair, segment) of a call: n_seg segments per pair, and twice as many
+// for the pairs from *split_from on (the last ones claimed, so that the CTAs
+// finish closer together).
+int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n_seg_out,
+                       int32_t* split_from_out);
 cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_f32(const RolloutArgs& a, int hidden, int n_sm, cudaStream_t s);
 cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s);

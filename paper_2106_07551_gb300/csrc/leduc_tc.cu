@@ -114,7 +114,8 @@ __device__ __forceinline__ void drive(const EvalArgs& a, const LeducWork& w, E::
                                       long long* sums, bool wait_stage = true) {
     const int tid = threadIdx.x;
     const int64_t n_seg = w.n_seg;
-    const int64_t n_units = (int64_t)a.n_pairs * n_seg;
+    const int64_t n_units = w.n_units;
+    const int64_t n_whole = (int64_t)w.split_from * n_seg;   // units before the split pairs
     uint16_t* q_base = w.queues + (size_t)blockIdx.x * 4 * w.max_hands;   // [seat][queue][max_hands]
     uint32_t tile = 0;
     while (true) {
@@ -123,9 +124,13 @@ __device__ __forceinline__ void drive(const EvalArgs& a, const LeducWork& w, E::
             const int64_t u = (int64_t)atomicAdd(a.work, 1ull);
             ctl.unit = u < n_units ? u : -1;
             if (u < n_units) {
-                const int pair = (int)(u / n_seg);
-                const int64_t seg = u % n_seg;
-                const int64_t per = (a.n_episodes + n_seg - 1) / n_seg;
+                // pairs before split_from in n_seg segments, the others in 2 n_seg
+                const bool split = u >= n_whole;
+                const int64_t ns = split ? 2 * n_seg : n_seg;
+                const int64_t v = split ? u - n_whole : u;
+                const int pair = (int)(split ? w.split_from + v / ns : v / ns);
+                const int64_t seg = v % ns;
+                const int64_t per = (a.n_episodes + ns - 1) / ns;
                 ctl.pair = pair;
                 ctl.e_lo = seg * per;
                 const int64_t hi = min(a.n_episodes, ctl.e_lo + per);
@@ -438,12 +443,19 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
 
 }  // namespace
 
-int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n_seg_out) {
+int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n_seg_out,
+                       int32_t* split_from_out) {
     int64_t n_seg = (n_episodes + kLeducTcMaxHands - 1) / kLeducTcMaxHands;
     // enough units for every SM when pairs are few
     while ((int64_t)n_pairs * n_seg < n_sm && (n_episodes + n_seg - 1) / n_seg > 256) ++n_seg;
+    // when there are more pairs than SMs, the last n_sm pairs (the last units
+    // claimed) are played in halves: a unit's time varies with its policies,
+    // and shorter last units leave the CTAs closer together at the end
+    int32_t split_from = n_pairs;
+    if ((int64_t)n_pairs > n_sm && (n_episodes + 2 * n_seg - 1) / (2 * n_seg) >= 256) split_from = n_pairs - n_sm;
     *n_seg_out = n_seg;
-    return (int64_t)n_pairs * n_seg;
+    *split_from_out = split_from;
+    return (int64_t)split_from * n_seg + (int64_t)(n_pairs - split_from) * 2 * n_seg;
 }
 
 cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm, cudaStream_t s) {
@@ -452,10 +464,13 @@ cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (err != cudaSuccess) return err;
     int64_t n_seg = 0;
-    const int64_t units = leduc_tc_units(a.n_pairs, a.n_episodes, n_sm, &n_seg);
+    int32_t split_from = 0;
+    const int64_t units = leduc_tc_units(a.n_pairs, a.n_episodes, n_sm, &n_seg, &split_from);
     const int64_t grid = units < n_sm ? units : n_sm;
     LeducWork ww = w;
     ww.n_seg = n_seg;
+    ww.split_from = split_from;
+    ww.n_units = units;
     leduc_eval_tc_kernel<<<(unsigned)grid, kThreads, kSmem, s>>>(a, ww);
     return cudaGetLastError();
 }

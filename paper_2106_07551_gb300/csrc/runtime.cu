@@ -656,7 +656,8 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
             CK(launch_kuhn_eval(a, c->n_sm, c->stream), "Kuhn eval kernel");
         } else if (leduc_tc) {
             int64_t n_seg = 0;
-            const int64_t units = leduc_tc_units(n_pairs, n_episodes, c->n_sm, &n_seg);
+            int32_t split_from = 0;
+            const int64_t units = leduc_tc_units(n_pairs, n_episodes, c->n_sm, &n_seg, &split_from);
             const int64_t grid = std::min<int64_t>(units, c->n_sm);
             const int64_t per = (n_episodes + n_seg - 1) / n_seg;
             LeducWork lw{};
