@@ -65,6 +65,21 @@ def test_full_replay_parity(orc, n_eps):
     ctx.close()
 
 
+def test_split_tail_units_replay(orc):
+    """More pairs than SMs: the last pairs claimed are played in two halves of
+    their hands. 13 x 13 pairs x 600 hands, every hand of every pair replayed
+    and the integer sums compared exactly."""
+    torch = need_gpu()
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    w = workloads.leduc(pop=13, hidden=256, dtype=workloads.BF16, with_bias=True, seed=613)
+    assert w.n_pairs > n_sm                      # the split applies
+    ctx = context()
+    load_population(ctx, w)
+    res, d = run(ctx, w, 600, 29, 600)
+    replay(orc, w, res, d, 600, 29, 600, full=True)
+    ctx.close()
+
+
 def test_full_workload_every_cell(orc):
     """64x64 pairs x 16,384 hands: 16 hands of every pair replayed; all 4,096
     entries against the exact tree expectation."""
