@@ -211,6 +211,9 @@ __device__ __forceinline__ void end_cta(uint32_t tbase) {
     if ((threadIdx.x >> 5) == 0) tc::tmem_dealloc(tbase, E::kTmemCols);
 }
 
+// kDump: the call records its first n_dump hands of every pair (the consumers'
+// recording code is compiled out of the other instance).
+template <bool kDump>
 __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, LeducWork w) {
     extern __shared__ __align__(1024) uint8_t smem[];
     __shared__ E::Bars bars;
@@ -377,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
                     const float u = u24(draw(gid, (uint32_t)t, (uint32_t)s, a.seed).x);
                     const unsigned legal = leduc_legal(h);
                     const int act = sample_masked<3>(lg, legal, u);
-                    const bool rec = e < a.n_dump;
+                    const bool rec = kDump && e < a.n_dump;
                     const int64_t rb = ((int64_t)ph.pair * a.n_dump + e) * kMaxDec;
                     if (rec) {
                         if (a.d_obs) {
@@ -460,8 +463,8 @@ int64_t leduc_tc_units(int32_t n_pairs, int64_t n_episodes, int n_sm, int64_t* n
 
 cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0) return cudaSuccess;
-    cudaError_t err = cudaFuncSetAttribute(leduc_eval_tc_kernel,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+    auto kern = a.n_dump > 0 ? leduc_eval_tc_kernel<true> : leduc_eval_tc_kernel<false>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (err != cudaSuccess) return err;
     int64_t n_seg = 0;
     int32_t split_from = 0;
@@ -471,7 +474,7 @@ cudaError_t launch_leduc_eval_tc(const EvalArgs& a, const LeducWork& w, int n_sm
     ww.n_seg = n_seg;
     ww.split_from = split_from;
     ww.n_units = units;
-    leduc_eval_tc_kernel<<<(unsigned)grid, kThreads, kSmem, s>>>(a, ww);
+    kern<<<(unsigned)grid, kThreads, kSmem, s>>>(a, ww);
     return cudaGetLastError();
 }
 

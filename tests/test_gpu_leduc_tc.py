@@ -62,6 +62,8 @@ def test_full_replay_parity(orc, n_eps):
     res2, d2 = run(ctx, w, n_eps, 77, n_eps)          # deterministic
     np.testing.assert_array_equal(res2, res)
     np.testing.assert_array_equal(d2["logits"], d["logits"])
+    # the kernel instance without the recording code plays the same hands
+    np.testing.assert_array_equal(ctx.eval_payoff(w.pair_ids, n_eps, 77), res)
     ctx.close()
 
 
@@ -77,6 +79,7 @@ def test_split_tail_units_replay(orc):
     load_population(ctx, w)
     res, d = run(ctx, w, 600, 29, 600)
     replay(orc, w, res, d, 600, 29, 600, full=True)
+    np.testing.assert_array_equal(ctx.eval_payoff(w.pair_ids, 600, 29), res)   # no recording
     ctx.close()
 
 
