@@ -418,6 +418,9 @@ __device__ __forceinline__ void layer23_n(int nb, const float* H1, float* LG, co
 
 }  // namespace t8
 
+// kDump: the call records its first n_dump hands of every pair (the recording
+// code is compiled out of the other instance).
+template <bool kDump>
 __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
     using namespace t8;
     extern __shared__ __align__(128) float smem[];
@@ -546,7 +549,7 @@ __global__ void __launch_bounds__(256, 1) leduc_eval_f32_t8_kernel(EvalArgs a) {
                 const unsigned legal = leduc_legal(h);
                 const float u = u24(draw(g, (uint32_t)t, (uint32_t)seat, a.seed).x);
                 const int act = sample_masked<3>(lg, legal, u);
-                const bool rec = e < a.n_dump;
+                const bool rec = kDump && e < a.n_dump;
                 const int64_t rb = ((int64_t)pair * a.n_dump + e) * kLeducMaxDec;
                 if (rec) {
                     if (a.d_obs) {
@@ -637,15 +640,15 @@ cudaError_t launch_leduc_eval_f32(const EvalArgs& a, int hidden, int n_sm, cudaS
     if (a.n_pairs == 0) return cudaSuccess;
     if (hidden == 128) {
         if (!a.work) return cudaErrorInvalidValue;       // the kernel claims hands from a.work
-        cudaError_t err = cudaFuncSetAttribute(leduc_eval_f32_t8_kernel,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize,
+        auto kern = a.n_dump > 0 ? leduc_eval_f32_t8_kernel<true> : leduc_eval_f32_t8_kernel<false>;
+        cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)t8::kBytes);
         if (err != cudaSuccess) return err;
         const int64_t total = (int64_t)a.n_pairs * a.n_episodes;
         int64_t grid = (total + t8::kSlots - 1) / t8::kSlots;
         if (grid > n_sm) grid = n_sm;
         if (grid < 1) grid = 1;
-        leduc_eval_f32_t8_kernel<<<(unsigned)grid, 256, t8::kBytes, s>>>(a);
+        kern<<<(unsigned)grid, 256, t8::kBytes, s>>>(a);
         return cudaGetLastError();
     }
     if (hidden == 64) return launch_leduc_h<64>(a, n_sm, s);

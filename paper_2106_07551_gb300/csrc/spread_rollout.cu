@@ -91,7 +91,9 @@ struct ScenarioEnv<kReference, N> {
     using type = RefEnv;
 };
 
-template <int N, int IN, int H, int kScen = kSpread>
+// kLogits: the call records the logits (the recording code is compiled out of
+// the other instance).
+template <int N, int IN, int H, int kScen = kSpread, bool kLogits = false>
 __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs a) {
     static_assert(kScen != kAdversary || (N == 3 && IN == kAdvObs), "the simple adversary has 3 agents, obs 14");
     static_assert(kScen != kSpeakerListener || (N == 2 && IN == kSlObs),
@@ -212,7 +214,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                         const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
                         const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : (1u << A) - 1u;
                         act[i] = sample_masked<A>(lg, legal, uu);
-                        if (a.logits)
+                        if (kLogits)
 #pragma unroll
                             for (int k = 0; k < A; ++k) a.logits[(ix + i) * A + k] = lg[k];
                     }
@@ -281,7 +283,7 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                     const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
                     const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : (1u << A) - 1u;
                     act[i] = sample_masked<A>(lg, legal, uu);
-                    if (a.logits)
+                    if (kLogits)
 #pragma unroll
                         for (int k = 0; k < A; ++k) a.logits[(ix + i) * A + k] = lg[k];
                 }
@@ -308,14 +310,14 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
 template <int N, int IN, int H, int kScen = kSpread>
 cudaError_t launch_spread_nih(const RolloutArgs& a, int n_sm, cudaStream_t s) {
     using SM = SpreadF32Smem<N, IN, H, actions_of(kScen)>;
-    cudaError_t err = cudaFuncSetAttribute(spread_rollout_f32_kernel<N, IN, H, kScen>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)SM::kBytes);
+    auto kern = a.logits ? spread_rollout_f32_kernel<N, IN, H, kScen, true>
+                         : spread_rollout_f32_kernel<N, IN, H, kScen, false>;
+    cudaError_t err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SM::kBytes);
     if (err != cudaSuccess) return err;
     const int64_t units = (int64_t)a.n_pairs * ((a.n_episodes + 1) / 2);
     int64_t grid = units < n_sm ? units : n_sm;
     if (grid < 1) grid = 1;
-    spread_rollout_f32_kernel<N, IN, H, kScen><<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
+    kern<<<(unsigned)grid, 256, SM::kBytes, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -83,7 +83,9 @@ __device__ __forceinline__ bool pair_valid(const RolloutArgs& a, int pair) {
 }
 
 // kContact: the agents also push each other apart (soft contact forces).
-template <bool kContact>
+// kLogits: the call records the logits (the recording code is compiled out of
+// the other instances).
+template <bool kContact, bool kLogits>
 __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t stage_bar;             // W1 and the biases staged
@@ -246,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
                         for (int q = 0; q < kA; ++q) l5[q] = lp[q];
                         const float u = u24(draw(gid, (uint32_t)t, (uint32_t)kj, a.seed).x);
                         const int act = sample_masked<kA>(l5, 0x1Fu, u);
-                        if (a.logits)
+                        if (kLogits)
 #pragma unroll
                             for (int q = 0; q < kA; ++q) a.logits[(ix + kj) * kA + q] = l5[q];
                         a.action[ix + kj] = (uint8_t)act;
@@ -307,20 +309,22 @@ bool spread_tc_supported(int n_agents, int obs_dim, int n_actions, int64_t envs_
            envs_per_pair <= 128;
 }
 
-template <bool kContact>
+template <bool kContact, bool kLogits>
 cudaError_t launch_tc(const RolloutArgs& a, int n_sm, cudaStream_t s) {
-    cudaError_t err = cudaFuncSetAttribute(spread_rollout_tc_kernel<kContact>,
+    cudaError_t err = cudaFuncSetAttribute(spread_rollout_tc_kernel<kContact, kLogits>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
     if (err != cudaSuccess) return err;
     const int64_t items = (int64_t)a.n_pairs * a.n_episodes;
     const int64_t ctas = items < n_sm ? items : n_sm;
-    spread_rollout_tc_kernel<kContact><<<(unsigned)ctas, kThreads, kSmem, s>>>(a);
+    spread_rollout_tc_kernel<kContact, kLogits><<<(unsigned)ctas, kThreads, kSmem, s>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_spread_rollout_tc(const RolloutArgs& a, int n_sm, cudaStream_t s) {
     if (a.n_pairs == 0 || a.n_episodes == 0) return cudaSuccess;
-    return a.contact ? launch_tc<true>(a, n_sm, s) : launch_tc<false>(a, n_sm, s);
+    if (a.logits)
+        return a.contact ? launch_tc<true, true>(a, n_sm, s) : launch_tc<false, true>(a, n_sm, s);
+    return a.contact ? launch_tc<true, false>(a, n_sm, s) : launch_tc<false, false>(a, n_sm, s);
 }
 
 }  // namespace malib
