@@ -40,6 +40,17 @@ constexpr int kObs = 34, kObsPad = 36, kK1 = 48, kA = 5;
 using Eng = MlpTc<kK1, 256, 16, true, /*kBarId=*/1>;    // biases staged with the weights
 constexpr int kThreads = 512;
 constexpr int kEngineThreads = 256;
+// registers per thread after setmaxnreg: the engine's two warpgroups and the two
+// environment groups' (whose 8-agent steps and observations need more), summing
+// to the launch's 128 per thread
+constexpr int kRegLaunch = 128, kRegEngine = 120, kRegEnv = 136;
+static_assert(kRegEngine + kRegEnv == 2 * kRegLaunch, "register split within the launch's allocation");
+
+template <int R>
+__device__ __forceinline__ void set_max_regs() {
+    if constexpr (R > kRegLaunch) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R) : "memory");
+    else if constexpr (R < kRegLaunch) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R) : "memory");
+}
 constexpr int kGroups = 2;
 constexpr int kLgStride = kA;                                     // logits row stride (floats)
 constexpr uint32_t kX = Eng::kSmemBytes;                          // X tiles [group][buffer]
@@ -133,6 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
 
     if (warp < 8) {
         // ------------------------------------------------------------ engine
+        set_max_regs<kRegEngine>();
         uint32_t stage_par = 0, mma_par = 0, x_bits = 0;   // x_full[g][b] phase: bit 2 g + b
         int staged = -1;                                   // policy id in shared memory
         for (int64_t it = lo; it < hi;) {
@@ -193,6 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
             }
         }
     } else {
+        set_max_regs<kRegEnv>();
         // ------------------------------------------------------------ environment groups
         const int g = (warp - 8) >> 2;
         const int e = tid - kEngineThreads - g * 128;     // environment within the block
