@@ -43,10 +43,10 @@ NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1441536 + 512,
     "kuhn_eval_kernel": 13312,
     "spread_rollout_f32_kernel<3,18,64,0>": 1373184 + 2559883520,
-    "leduc_eval_tc_kernel": 19399168 + 465920,
+    "leduc_eval_tc_kernel": 19416064 + 490240,
     "spread_rollout_f32_kernel<3,14,64,1>": 1683968 + 2068428800,
     "spread_rollout_f32_kernel<2,11,64,2>": 1547520 + 1034004736,
-    "spread_rollout_tc_kernel": (20857088 + 1914217984) * 2,
+    "spread_rollout_tc_kernel": (18220032 + 1910865664) * 2,
     "learn_grad_kernel": 511446016 + 3254016,
     "spread_rollout_f32_kernel<2,8,64,3>": 1031936 + 706821376,
     "spread_rollout_f32_kernel<4,16,64,4>": 8131072 + 2782468352,

@@ -46,8 +46,19 @@ constexpr int kThreads = 32 * kWarps;
 constexpr int kProdWarp = 4 * kProdWG, kConsWarp = 4 * kConsWG;
 // registers per thread after setmaxnreg: epilogue, MMA, producer, consumer
 // warpgroups (their sum over the CTA stays within the launch's allocation)
-constexpr int kRegEpi = kTW == 8 ? 80 : 112, kRegMma = 56, kRegProd = kTW == 8 ? 48 : 64,
-              kRegCons = kTW == 8 ? 80 : 128;
+constexpr int kRegEpi = kTW == 8 ? 80 : 112, kRegMma = kTW == 8 ? 48 : 56, kRegProd = kTW == 8 ? 48 : 64,
+              kRegCons = kTW == 8 ? 88 : 128;
+constexpr int kRegLaunch = 65536 / kThreads / 8 * 8;   // the launch's registers per thread
+static_assert((kEpiWG * kRegEpi + kRegMma + kRegProd + kRegCons) <= (kEpiWG + 3) * kRegLaunch,
+              "register split within the launch's allocation");
+
+// setmaxnreg to R registers per thread: inc above the launch's count, dec below.
+template <int R>
+__device__ __forceinline__ void set_max_regs() {
+    static_assert(R % 8 == 0 && R >= 24 && R <= 256, "setmaxnreg's range");
+    if constexpr (R > kRegLaunch) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R) : "memory");
+    else if constexpr (R < kRegLaunch) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R) : "memory");
+}
 constexpr int kMaxDec = 8;
 constexpr uint32_t kX = (E::kImage + 1023u) / 1024u * 1024u;     // X tiles
 constexpr uint32_t kP = kX + E::kNX * E::kXBytes;                  // partial logits
@@ -240,7 +251,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
 
     if (wg < kEpiWG) {
         // ---- epilogue teams (warps 0 .. kTW - 1 slot 0, then slot 1)
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegEpi) : "memory");
+        set_max_regs<kRegEpi>();
         if (warp < kTW) {
             E::Epilogue<0> ep;
             ep.p_base_off = kP;
@@ -255,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else if (wg == kMmaWG) {
         // ---- the MMA threads (the warpgroup's first two warps; two idle)
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegMma) : "memory");
+        set_max_regs<kRegMma>();
         if (warp == 4 * kMmaWG) {
             E::Issuer<0> is;
             drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
@@ -274,7 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else if (wg == kProdWG) {
         // ---- producers: observation rows, one per thread
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegProd) : "memory");
+        set_max_regs<kRegProd>();
         const int r = tid - kProdWarp * 32;
         const uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
         drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
@@ -325,7 +336,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else {
         // ---- consumers: draw, transition, sums, next queue; one row per thread
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegCons) : "memory");
+        set_max_regs<kRegCons>();
         const int r = tid - kConsWarp * 32;
         uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
         uint16_t* q_base = w.queues + (size_t)blockIdx.x * 4 * w.max_hands;
