@@ -180,19 +180,28 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
         for (int t = 0; t < T; ++t) {
             if constexpr (SM::kPerAgent) {
                 // one agent at a time: its observations (to X and the
-                // trajectory), its pass, its draw
-                int act[N];
+                // trajectory), its pass, its draw. The loop stays rolled, so the
+                // MLP's code appears once (instruction fetch limited the unrolled
+                // form); the observation is built by a copy per constant agent
+                // index (no dynamic indexing of the state in registers), and the
+                // actions are packed one byte per agent.
+                static_assert(N <= 4, "one byte per agent's action in a 32-bit word");
+                uint32_t act_pk = 0;
                 const int64_t ix = ((ep * T + t) * a.n_envs + env) * N;
-#pragma unroll
+#pragma unroll 1
                 for (int i = 0; i < N; ++i) {
                     if (mine) {
                         float o[XS];
-                        if constexpr (kScen == kTag) tag_obs<XS>(s, i, o);
-                        else if constexpr (kScen == kReference) ref_obs<XS>(s, i, o);
-                        else if constexpr (kScen == kPush) push_obs<XS>(s, i, o);
-                        else if constexpr (kScen == kAdversary) adv_obs<XS>(s, i, o);
-                        else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, i, o);
-                        else spread_obs<N, XS>(s, i, o);
+#pragma unroll
+                        for (int j = 0; j < N; ++j) {
+                            if (j != i) continue;
+                            if constexpr (kScen == kTag) tag_obs<XS>(s, j, o);
+                            else if constexpr (kScen == kReference) ref_obs<XS>(s, j, o);
+                            else if constexpr (kScen == kPush) push_obs<XS>(s, j, o);
+                            else if constexpr (kScen == kAdversary) adv_obs<XS>(s, j, o);
+                            else if constexpr (kScen == kSpeakerListener) sl_obs<XS>(s, j, o);
+                            else spread_obs<N, XS>(s, j, o);
+                        }
                         float4* xr = reinterpret_cast<float4*>(X + tid * XS);
                         float4* gr = reinterpret_cast<float4*>(a.obs + (ix + i) * XS);
 #pragma unroll
@@ -213,13 +222,16 @@ __global__ void __launch_bounds__(256, 1) spread_rollout_f32_kernel(RolloutArgs 
                         for (int k = 0; k < A; ++k) lg[k] = LG[tid * M::LS + k];
                         const float uu = u24(draw(g, (uint32_t)t, (uint32_t)i, a.seed).x);
                         const unsigned legal = (kScen == kSpeakerListener && i == 0) ? kSlSpeakerLegal : (1u << A) - 1u;
-                        act[i] = sample_masked<A>(lg, legal, uu);
+                        act_pk |= (uint32_t)sample_masked<A>(lg, legal, uu) << (8 * i);
                         if (kLogits)
 #pragma unroll
                             for (int k = 0; k < A; ++k) a.logits[(ix + i) * A + k] = lg[k];
                     }
                 }
                 if (mine) {
+                    int act[N];
+#pragma unroll
+                    for (int i = 0; i < N; ++i) act[i] = (int)((act_pk >> (8 * i)) & 0xffu);
                     float r[N];
                     if constexpr (kScen == kAdversary) adv_step(s, act, r);
                     else if constexpr (kScen == kSpeakerListener) sl_step(s, act, r);
