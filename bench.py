@@ -49,7 +49,7 @@ NCU_TRAFFIC_PER_LAUNCH = {
     "spread_rollout_tc_kernel": (18220032 + 1910865664) * 2,
     "learn_grad_kernel": 511446016 + 3254016,
     "spread_rollout_f32_kernel<2,8,64,3>": 1031936 + 706821376,
-    "spread_rollout_f32_kernel<4,16,64,4>": 8131072 + 2782468352,
+    "spread_rollout_f32_kernel<4,16,64,4>": 3663872 + 2780089856,
     "spread_rollout_f32_kernel<2,14,64,6>": 2387712 + 1377357056,
 }
 
