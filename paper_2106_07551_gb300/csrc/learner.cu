@@ -490,41 +490,55 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
             }
         }
         __syncthreads();
-        // the tile's weight gradients, 4 samples per 16-byte load
+        // the tile's weight gradients, 4 samples per 16-byte load; packed pairs
+        // of consecutive samples (the even and odd samples' sums, added at the
+        // tile's end)
+        {
+            using u64 = unsigned long long;
+            u64 t2[4][4] = {};
 #pragma unroll 2
-        for (int s = 0; s < kTile; s += 4) {
-            float4 d[4], h[4];
+            for (int s = 0; s < kTile; s += 4) {
+                ulonglong2 d[4], h[4];
 #pragma unroll
-            for (int p = 0; p < 4; ++p) {
-                d[p] = *reinterpret_cast<const float4*>(D2T + (sg + 16 * p) * kTS + s);
-                h[p] = *reinterpret_cast<const float4*>(H1T + (ng + 16 * p) * kTS + s);
+                for (int p = 0; p < 4; ++p) {
+                    d[p] = *reinterpret_cast<const ulonglong2*>(D2T + (sg + 16 * p) * kTS + s);
+                    h[p] = *reinterpret_cast<const ulonglong2*>(H1T + (ng + 16 * p) * kTS + s);
+                }
+#pragma unroll
+                for (int p = 0; p < 4; ++p)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        f2_fma(t2[p][q], d[p].x, h[q].x);
+                        f2_fma(t2[p][q], d[p].y, h[q].y);
+                    }
             }
 #pragma unroll
             for (int p = 0; p < 4; ++p)
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    float g = gW2[p][q];
-                    g = fmaf(d[p].x, h[q].x, g);
-                    g = fmaf(d[p].y, h[q].y, g);
-                    g = fmaf(d[p].z, h[q].z, g);
-                    g = fmaf(d[p].w, h[q].w, g);
-                    gW2[p][q] = g;
+                    const float2 v = f2_split(t2[p][q]);
+                    gW2[p][q] += v.x + v.y;
                 }
         }
-        for (int s = 0; s < kTile; s += 4) {
-            const float4 d = *reinterpret_cast<const float4*>(D1T + w1j * kTS + s);
+        {
+            using u64 = unsigned long long;
+            u64 t1[kLearnMaxIn / 4] = {};
+            for (int s = 0; s < kTile; s += 4) {
+                const ulonglong2 d = *reinterpret_cast<const ulonglong2*>(D1T + w1j * kTS + s);
+#pragma unroll
+                for (int q = 0; q < kLearnMaxIn / 4; ++q) {
+                    const int k = w1k + 4 * q;
+                    if (k < in) {
+                        const ulonglong2 x = *reinterpret_cast<const ulonglong2*>(XT + k * kTS + s);
+                        f2_fma(t1[q], d.x, x.x);
+                        f2_fma(t1[q], d.y, x.y);
+                    }
+                }
+            }
 #pragma unroll
             for (int q = 0; q < kLearnMaxIn / 4; ++q) {
-                const int k = w1k + 4 * q;
-                if (k < in) {
-                    const float4 x = *reinterpret_cast<const float4*>(XT + k * kTS + s);
-                    float g = gW1[q];
-                    g = fmaf(d.x, x.x, g);
-                    g = fmaf(d.y, x.y, g);
-                    g = fmaf(d.z, x.z, g);
-                    g = fmaf(d.w, x.w, g);
-                    gW1[q] = g;
-                }
+                const float2 v = f2_split(t1[q]);
+                gW1[q] += v.x + v.y;
             }
         }
 #pragma unroll
@@ -532,16 +546,15 @@ __global__ void __launch_bounds__(kThreads, 1) learn_grad_kernel(LearnArgs a) {
             const int e = tid + kThreads * q;
             if (e < kA * kH) {
                 const int c = e / kH, j = e - c * kH;
-                float g = gW3[q];
+                unsigned long long t3 = 0ull;
                 for (int s = 0; s < kTile; s += 4) {
-                    const float4 d = *reinterpret_cast<const float4*>(DZT + c * kTS + s);
-                    const float4 x = *reinterpret_cast<const float4*>(H2T + j * kTS + s);
-                    g = fmaf(d.x, x.x, g);
-                    g = fmaf(d.y, x.y, g);
-                    g = fmaf(d.z, x.z, g);
-                    g = fmaf(d.w, x.w, g);
+                    const ulonglong2 d = *reinterpret_cast<const ulonglong2*>(DZT + c * kTS + s);
+                    const ulonglong2 x = *reinterpret_cast<const ulonglong2*>(H2T + j * kTS + s);
+                    f2_fma(t3, d.x, x.x);
+                    f2_fma(t3, d.y, x.y);
                 }
-                gW3[q] = g;
+                const float2 v = f2_split(t3);
+                gW3[q] += v.x + v.y;
             }
         }
         if (tid < 2 * kH + kA) {
