@@ -47,7 +47,7 @@ NCU_TRAFFIC_PER_LAUNCH = {
     "spread_rollout_f32_kernel<3,14,64,1>": 1683968 + 2068428800,
     "spread_rollout_f32_kernel<2,11,64,2>": 1547520 + 1034004736,
     "spread_rollout_tc_kernel": (18220032 + 1910865664) * 2,
-    "learn_grad_kernel": 511446016 + 3254016,
+    "learn_grad_kernel": 510880512 + 3277568,
     "spread_rollout_f32_kernel<2,8,64,3>": 1031936 + 706821376,
     "spread_rollout_f32_kernel<4,16,64,4>": 3663872 + 2780089856,
     "spread_rollout_f32_kernel<2,14,64,6>": 2387712 + 1377357056,
