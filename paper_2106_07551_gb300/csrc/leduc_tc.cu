@@ -52,13 +52,6 @@ constexpr int kRegLaunch = 65536 / kThreads / 8 * 8;   // the launch's registers
 static_assert((kEpiWG * kRegEpi + kRegMma + kRegProd + kRegCons) <= (kEpiWG + 3) * kRegLaunch,
               "register split within the launch's allocation");
 
-// setmaxnreg to R registers per thread: inc above the launch's count, dec below.
-template <int R>
-__device__ __forceinline__ void set_max_regs() {
-    static_assert(R % 8 == 0 && R >= 24 && R <= 256, "setmaxnreg's range");
-    if constexpr (R > kRegLaunch) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R) : "memory");
-    else if constexpr (R < kRegLaunch) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R) : "memory");
-}
 constexpr int kMaxDec = 8;
 constexpr uint32_t kX = (E::kImage + 1023u) / 1024u * 1024u;     // X tiles
 constexpr uint32_t kP = kX + E::kNX * E::kXBytes;                  // partial logits
@@ -251,7 +244,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
 
     if (wg < kEpiWG) {
         // ---- epilogue teams (warps 0 .. kTW - 1 slot 0, then slot 1)
-        set_max_regs<kRegEpi>();
+        tc::set_max_regs<kRegEpi, kRegLaunch>();
         if (warp < kTW) {
             E::Epilogue<0> ep;
             ep.p_base_off = kP;
@@ -266,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else if (wg == kMmaWG) {
         // ---- the MMA threads (the warpgroup's first two warps; two idle)
-        set_max_regs<kRegMma>();
+        tc::set_max_regs<kRegMma, kRegLaunch>();
         if (warp == 4 * kMmaWG) {
             E::Issuer<0> is;
             drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
@@ -285,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else if (wg == kProdWG) {
         // ---- producers: observation rows, one per thread
-        set_max_regs<kRegProd>();
+        tc::set_max_regs<kRegProd, kRegLaunch>();
         const int r = tid - kProdWarp * 32;
         const uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
         drive(a, w, bars, ctl, smem, [&](const Phase& ph) {
@@ -336,7 +329,7 @@ __global__ void __launch_bounds__(kThreads, 1) leduc_eval_tc_kernel(EvalArgs a, 
         end_cta(tbase);
     } else {
         // ---- consumers: draw, transition, sums, next queue; one row per thread
-        set_max_regs<kRegCons>();
+        tc::set_max_regs<kRegCons, kRegLaunch>();
         const int r = tid - kConsWarp * 32;
         uint2* hands = w.hands + (size_t)blockIdx.x * w.max_hands;
         uint16_t* q_base = w.queues + (size_t)blockIdx.x * 4 * w.max_hands;

@@ -46,11 +46,6 @@ constexpr int kEngineThreads = 256;
 constexpr int kRegLaunch = 128, kRegEngine = 120, kRegEnv = 136;
 static_assert(kRegEngine + kRegEnv == 2 * kRegLaunch, "register split within the launch's allocation");
 
-template <int R>
-__device__ __forceinline__ void set_max_regs() {
-    if constexpr (R > kRegLaunch) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R) : "memory");
-    else if constexpr (R < kRegLaunch) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R) : "memory");
-}
 constexpr int kGroups = 2;
 constexpr int kLgStride = kA;                                     // logits row stride (floats)
 constexpr uint32_t kX = Eng::kSmemBytes;                          // X tiles [group][buffer]
@@ -144,7 +139,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
 
     if (warp < 8) {
         // ------------------------------------------------------------ engine
-        set_max_regs<kRegEngine>();
+        tc::set_max_regs<kRegEngine, kRegLaunch>();
         uint32_t stage_par = 0, mma_par = 0, x_bits = 0;   // x_full[g][b] phase: bit 2 g + b
         int staged = -1;                                   // policy id in shared memory
         for (int64_t it = lo; it < hi;) {
@@ -205,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1) spread_rollout_tc_kernel(RolloutA
             }
         }
     } else {
-        set_max_regs<kRegEnv>();
+        tc::set_max_regs<kRegEnv, kRegLaunch>();
         // ------------------------------------------------------------ environment groups
         const int g = (warp - 8) >> 2;
         const int e = tid - kEngineThreads - g * 128;     // environment within the block

@@ -252,5 +252,16 @@ __device__ __forceinline__ uint32_t bias_relu_bf16x2(float x0, float x1, float b
     return r;
 }
 
+// setmaxnreg to R registers per thread in a kernel launched with kLaunch per
+// thread: inc above the launch's count, dec below it, nothing at it (an inc to
+// fewer registers, or a dec to more, is an illegal instruction). All threads
+// of the warpgroup call it.
+template <int R, int kLaunch>
+__device__ __forceinline__ void set_max_regs() {
+    static_assert(R % 8 == 0 && R >= 24 && R <= 256, "setmaxnreg's range");
+    if constexpr (R > kLaunch) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R) : "memory");
+    else if constexpr (R < kLaunch) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R) : "memory");
+}
+
 }  // namespace tc
 }  // namespace malib
