@@ -140,11 +140,26 @@ __global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
         const int ck = slots[slot];
         const int c = ck / a.n_agents, k = ck - c * a.n_agents;
         const int64_t env = (int64_t)c * epp + r;
+        // backward over the episode, 8 steps at a time: the 8 rewards are loaded
+        // together (the stores to G would otherwise hold each load behind the
+        // previous step's store), then the same recurrence in the same order
         float g = 0.f;
-        for (int t = a.T - 1; t >= 0; --t) {
-            g = __fadd_rn(a.reward[((e * a.T + t) * a.n_envs + env) * a.n_agents + k], __fmul_rn(a.gamma, g));
-            G[((slot * a.n_episodes + e) * a.T + t) * epp + r] = g;
-            sum += (double)g;
+        for (int t_hi = a.T; t_hi > 0; t_hi -= 8) {
+            float rv[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int t = t_hi - 1 - u;
+                rv[u] = t >= 0 ? a.reward[((e * a.T + t) * a.n_envs + env) * a.n_agents + k] : 0.f;
+            }
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                const int t = t_hi - 1 - u;
+                if (t >= 0) {
+                    g = __fadd_rn(rv[u], __fmul_rn(a.gamma, g));
+                    G[((slot * a.n_episodes + e) * a.T + t) * epp + r] = g;
+                    sum += (double)g;
+                }
+            }
         }
     }
     red[threadIdx.x] = sum;
@@ -586,19 +601,30 @@ __global__ void learn_reduce_kernel(LearnArgs a, int P) {
     const int64_t t_lo = a.tile_off[b], t_hi = a.tile_off[b + 1];
     int c_lo = 0, c_hi = 0;                  // CTAs [c_lo, c_hi) hold partials of b
     if (t_hi > t_lo) {
+        // c_lo: the first CTA whose share ends past t_lo; c_hi: the first CTA
+        // after it whose share starts at or past t_hi (or the grid's end). Both
+        // start from the shares' proportional position and step to the exact one.
+        const int64_t n_t = a.tile_off[a.nb];
+        c_lo = (int)min((int64_t)a.grid - 1, t_lo * a.grid / n_t);
+        while (c_lo > 0 && share_lo(a, c_lo) > t_lo) --c_lo;
         while (share_lo(a, c_lo + 1) <= t_lo) ++c_lo;
-        c_hi = c_lo + 1;
+        c_hi = (int)max((int64_t)c_lo + 1, min((int64_t)a.grid, (t_hi * a.grid + n_t - 1) / n_t));
+        while (c_hi > c_lo + 1 && share_lo(a, c_hi - 1) >= t_hi) --c_hi;
         while (c_hi < a.grid && share_lo(a, c_hi) < t_hi) ++c_hi;
     }
     // (a CTA with an empty share wrote no partial: it is skipped)
     const float* part = a.gpart + (int64_t)b * a.grid * (P + 2) + j;
     double p8[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
     int u = 0;
-    for (int c = c_lo; c < c_hi; ++c)
-        if (share_lo(a, c + 1) > share_lo(a, c)) {
+    int64_t s_c = share_lo(a, c_lo);
+    for (int c = c_lo; c < c_hi; ++c) {
+        const int64_t s_n = share_lo(a, c + 1);
+        if (s_n > s_c) {
             p8[u] += (double)part[(int64_t)c * (P + 2)];
             u = (u + 1) & 7;
         }
+        s_c = s_n;
+    }
     const double s = ((p8[0] + p8[1]) + (p8[2] + p8[3])) + ((p8[4] + p8[5]) + (p8[6] + p8[7]));
     double* st = a.stats + 4 * b;
     if (j < P) a.grad[(int64_t)b * P + j] = (float)s;
