@@ -21,20 +21,7 @@ __global__ void finalize_kernel(const unsigned long long* acc, int32_t n_pairs, 
                                 double* out) {
     const int p = blockIdx.x * blockDim.x + threadIdx.x;
     if (p >= n_pairs) return;
-    const long long s1 = (long long)acc[2 * p], s2 = (long long)acc[2 * p + 1];
-    const double dn = (double)n, d1 = (double)s1, d2 = (double)s2;
-    const double mean = __ddiv_rn(d1, dn);
-    double se = 0.0;
-    if (n >= 2) {
-        const double q = __ddiv_rn(__dmul_rn(d1, d1), dn);
-        double var = __ddiv_rn(__dsub_rn(d2, q), (double)(n - 1));
-        if (var < 0.0) var = 0.0;
-        se = __dsqrt_rn(__ddiv_rn(var, dn));
-    }
-    out[4 * p + 0] = mean;
-    out[4 * p + 1] = se;
-    out[4 * p + 2] = d1;
-    out[4 * p + 3] = d2;
+    finalize_pair((long long)acc[2 * p], (long long)acc[2 * p + 1], n, out + 4 * p);
 }
 
 __global__ void philox_kernel(const uint32_t* ctr, uint64_t seed, uint32_t* out, int64_t n) {

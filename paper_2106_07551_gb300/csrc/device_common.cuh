@@ -223,4 +223,24 @@ __device__ __forceinline__ long long warp_sum_ll(long long v) {
     return v;
 }
 
+// One payoff-table row from a pair's integer sums over n hands (Sec. 3.2, the
+// Monte-Carlo mean per combination): mean, standard error of the mean (sample
+// variance with n - 1, clamped at 0), and the two sums as doubles. Correctly
+// rounded double operations, so every caller writes the same bits.
+__device__ __forceinline__ void finalize_pair(long long s1, long long s2, int64_t n, double* row) {
+    const double dn = (double)n, d1 = (double)s1, d2 = (double)s2;
+    const double mean = __ddiv_rn(d1, dn);
+    double se = 0.0;
+    if (n >= 2) {
+        const double q = __ddiv_rn(__dmul_rn(d1, d1), dn);
+        double var = __ddiv_rn(__dsub_rn(d2, q), (double)(n - 1));
+        if (var < 0.0) var = 0.0;
+        se = __dsqrt_rn(__ddiv_rn(var, dn));
+    }
+    row[0] = mean;
+    row[1] = se;
+    row[2] = d1;
+    row[3] = d2;
+}
+
 }  // namespace malib

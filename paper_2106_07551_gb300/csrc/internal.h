@@ -68,6 +68,9 @@ struct EvalArgs {
     unsigned long long* acc;     // [n_pairs][2]
     unsigned long long* n_dec;   // total decisions (env-steps) of the call
     unsigned long long* work;    // [n_pairs] hands claimed so far (zeroed per call)
+    double* fin_out;             // Kuhn: [n_pairs][4] table written by each pair's last
+                                 // block (work[] counts its finished blocks); null: a
+                                 // separate finalize launch writes it
     int* err;
     // optional dump of the first n_dump episodes of each pair
     int64_t n_dump;

@@ -64,19 +64,18 @@ __device__ __forceinline__ KuhnHand kuhn_play(const float (&t0)[6], const float 
 __global__ void __launch_bounds__(256) kuhn_eval_kernel(EvalArgs a) {
     const int pair = blockIdx.y;
     const int p0 = a.pairs[2 * pair], p1 = a.pairs[2 * pair + 1];
-    if (!pair_ok(a, p0, p1)) {
-        if (threadIdx.x == 0 && blockIdx.x == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
-        return;
-    }
+    const bool ok = pair_ok(a, p0, p1);
+    if (!ok && threadIdx.x == 0 && blockIdx.x == 0) atomicOr(a.err, ERRBIT_BAD_PAIR);
     float t0[6], t1[6];
 #pragma unroll
     for (int i = 0; i < 6; ++i) {
-        t0[i] = a.arena[a.pol_offset[p0] + i];
-        t1[i] = a.arena[a.pol_offset[p1] + i];
+        t0[i] = ok ? a.arena[a.pol_offset[p0] + i] : 0.f;
+        t1[i] = ok ? a.arena[a.pol_offset[p1] + i] : 0.f;
     }
     long long s1 = 0, s2 = 0, nd = 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < a.n_episodes; e += stride) {
+    const int64_t n_play = ok ? a.n_episodes : 0;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n_play; e += stride) {
         const uint64_t g = (uint64_t)pair * (uint64_t)a.n_episodes + (uint64_t)e;
         const KuhnHand h = kuhn_play(t0, t1, g, a.seed);
         s1 += h.payoff;
@@ -97,6 +96,17 @@ __global__ void __launch_bounds__(256) kuhn_eval_kernel(EvalArgs a) {
         }
     }
     block_add_sums(s1, s2, nd, a.acc + 2 * pair, a.n_dec);
+    // the pair's last block to finish writes its table row (its sums are final:
+    // every block fenced its additions before counting itself)
+    if (a.fin_out && threadIdx.x == 0) {
+        __threadfence();
+        if (atomicAdd(a.work + pair, 1ull) == (unsigned long long)gridDim.x - 1ull) {
+            __threadfence();
+            const long long f1 = (long long)__ldcg(a.acc + 2 * pair);
+            const long long f2 = (long long)__ldcg(a.acc + 2 * pair + 1);
+            finalize_pair(f1, f2, a.n_episodes, a.fin_out + 4 * (int64_t)pair);
+        }
+    }
 }
 
 // Exact expected seat-0 payoff: the 6 deals, each 1/6, times the betting tree.

@@ -653,6 +653,7 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
         CK(launch_zero_u64(c->acc, (int64_t)n_pairs * 3 + 1, c->stream), "zero kernel");
         time_begin(c, &e0, &e1);
         if (kind == MALIB_ENV_KUHN) {
+            a.fin_out = dout;                 // each pair's last block writes its row
             CK(launch_kuhn_eval(a, c->n_sm, c->stream), "Kuhn eval kernel");
         } else if (leduc_tc) {
             int64_t n_seg = 0;
@@ -672,8 +673,8 @@ int malib_eval_payoff_ex(malib_ctx* c, const int32_t* pair_ids, int32_t n_pairs,
             CK(launch_leduc_eval_f32(a, c->dims[1], c->n_sm, c->stream), "Leduc eval kernel");
         }
         time_end(c, e0, e1);
-        CK(launch_finalize(c->acc, n_pairs, n_episodes, dout, c->stream), "finalize kernel");
-        c->launches += 3;
+        if (!a.fin_out) CK(launch_finalize(c->acc, n_pairs, n_episodes, dout, c->stream), "finalize kernel");
+        c->launches += a.fin_out ? 2 : 3;
     }
     if (host_out) {
         CK(cudaMemcpyAsync(payoff_out, dout, (size_t)n_pairs * 32, cudaMemcpyDeviceToHost,
