@@ -41,7 +41,7 @@ FP32_LANES_PER_SM = 128
 # on the learner step's own workload.
 NCU_TRAFFIC_PER_LAUNCH = {
     "leduc_eval_f32_t8_kernel": 1441536 + 512,
-    "kuhn_eval_kernel": 13312,
+    "kuhn_eval_kernel": 26880,
     "spread_rollout_f32_kernel<3,18,64,0>": 1373184 + 2559883520,
     "leduc_eval_tc_kernel": 19416064 + 490240,
     "spread_rollout_f32_kernel<3,14,64,1>": 1683968 + 2068428800,
