@@ -130,6 +130,12 @@ __global__ void __launch_bounds__(256) learn_returns_kernel(LearnArgs a) {
     const int64_t n_seq = (int64_t)a.n_slots[b] * a.n_episodes * epp;
     const int32_t* slots = a.slots + (int64_t)b * a.n_pairs * a.n_agents;
     float* G = a.G + a.samp_off[b];
+    if ((int64_t)blockIdx.x * blockDim.x >= n_seq) {
+        // no sequence of policy b reaches this block: its partial is 0, as the
+        // reduction below would give, without the barriers
+        if (threadIdx.x == 0) a.gsum[(int64_t)b * gridDim.x + blockIdx.x] = 0.0;
+        return;
+    }
     double sum = 0.0;
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < n_seq;
          q += (int64_t)gridDim.x * blockDim.x) {
